@@ -1,0 +1,839 @@
+// C ABI of the ESP solver (include/esp.h): context, table upload and validation, solve driver.
+#include <cmath>
+#include <cstdint>
+#include <cstring>
+#include <new>
+#include <vector>
+
+#include <cuda_runtime.h>
+
+#include "esp.h"
+#include "esp_debug.h"
+#include "esp_kernels.h"
+#include "esp_plan.h"
+
+using namespace esp;
+
+namespace {
+
+struct GraphKey {
+    double eta0 = 0, tol = 0;
+    int32_t step = -1, mode = -1, T = -1;
+    uint32_t flags = 0;
+    const void *lt = nullptr, *dt = nullptr, *ht = nullptr, *gt = nullptr;
+    bool has_l0 = false;
+    bool operator==(const GraphKey &o) const
+    {
+        return eta0 == o.eta0 && tol == o.tol && step == o.step && mode == o.mode && T == o.T && flags == o.flags &&
+               lt == o.lt && dt == o.dt && ht == o.ht && gt == o.gt && has_l0 == o.has_l0;
+    }
+};
+
+template <typename T>
+struct DevArr {
+    T *p = nullptr;
+    size_t n = 0;
+};
+
+}  // namespace
+
+struct esp_ctx {
+    int device = 0;
+    cudaStream_t stream = nullptr;
+    int sm_count = 0;
+    bool poisoned = false;
+    bool loaded = false;
+    bool solved = false;
+
+    int32_t S = 0, J = 0, R = 0, P = 0, rg = 0, n_groups = 0;
+    int64_t n_opt = 0;
+    std::vector<void *> table_bufs;  // everything freed on reload
+    int32_t *units = nullptr;
+    double *values = nullptr;
+    int64_t *off = nullptr;
+    uint16_t *group = nullptr;
+    int64_t *cap = nullptr;
+    double *vmax = nullptr;
+    int32_t *umax = nullptr;
+
+    TileDesc *tiles = nullptr;
+    int32_t *warp_begin = nullptr;
+    int32_t n_warps = 0, tile_opt = 0, grid = 0;
+
+    double *lam = nullptr, *p64 = nullptr, *job_val = nullptr, *job_min = nullptr;
+    double *best_dual = nullptr, *primal = nullptr, *dual = nullptr, *lambda0 = nullptr;
+    float *p32 = nullptr, *ebound = nullptr;
+    unsigned long long *U = nullptr, *U_final = nullptr, *hash = nullptr;
+    int32_t *sel = nullptr, *rounds_run = nullptr, *converged = nullptr, *status = nullptr, *frozen = nullptr,
+            *feasible = nullptr;
+    unsigned int *err = nullptr;
+    unsigned int *valflags = nullptr;
+
+    // trace buffers (grown on demand, freed on destroy)
+    DevArr<double> lt;
+    DevArr<long long> dt;
+    DevArr<unsigned long long> ht;
+    DevArr<double> gt;
+
+    cudaGraphExec_t gexec = nullptr;
+    GraphKey gkey;
+    int64_t last_launches = 0;
+    int32_t last_T = 0;
+};
+
+namespace {
+
+esp_status cuda_fail(esp_ctx *c, cudaError_t e)
+{
+    (void)e;
+    if (c)
+        c->poisoned = true;
+    return ESP_ERR_CUDA;
+}
+
+#define ESP_CUDA(call)                                  \
+    do {                                                \
+        cudaError_t e_ = (call);                        \
+        if (e_ != cudaSuccess) {                        \
+            cudaGetLastError();                         \
+            return cuda_fail(ctx, e_);                  \
+        }                                               \
+    } while (0)
+
+template <typename T>
+esp_status dev_alloc(esp_ctx *ctx, T **p, size_t count, size_t pad_bytes = 64)
+{
+    void *q = nullptr;
+    const size_t bytes = count * sizeof(T) + pad_bytes;
+    cudaError_t e = cudaMalloc(&q, bytes);
+    if (e == cudaErrorMemoryAllocation) {
+        cudaGetLastError();
+        return ESP_ERR_OOM;
+    }
+    if (e != cudaSuccess)
+        return cuda_fail(ctx, e);
+    e = cudaMemsetAsync(q, 0, bytes, ctx->stream);
+    if (e != cudaSuccess)
+        return cuda_fail(ctx, e);
+    ctx->table_bufs.push_back(q);
+    *p = static_cast<T *>(q);
+    return ESP_OK;
+}
+
+void release_table(esp_ctx *ctx)
+{
+    if (ctx->gexec) {
+        cudaGraphExecDestroy(ctx->gexec);
+        ctx->gexec = nullptr;
+        ctx->gkey = GraphKey();
+    }
+    for (void *p : ctx->table_bufs)
+        cudaFree(p);
+    ctx->table_bufs.clear();
+    ctx->loaded = false;
+    ctx->solved = false;
+}
+
+template <typename T>
+esp_status grow(esp_ctx *ctx, DevArr<T> &a, size_t n)
+{
+    if (a.n >= n && a.p)
+        return ESP_OK;
+    if (a.p)
+        cudaFree(a.p);
+    a.p = nullptr;
+    a.n = 0;
+    void *q = nullptr;
+    cudaError_t e = cudaMalloc(&q, n * sizeof(T) + 64);
+    if (e == cudaErrorMemoryAllocation) {
+        cudaGetLastError();
+        return ESP_ERR_OOM;
+    }
+    if (e != cudaSuccess)
+        return cuda_fail(ctx, e);
+    a.p = static_cast<T *>(q);
+    a.n = n;
+    return ESP_OK;
+}
+
+DevTable dev_table(const esp_ctx *c)
+{
+    DevTable t;
+    t.units = c->units;
+    t.values = c->values;
+    t.job_off = c->off;
+    t.group = c->group;
+    t.cap = c->cap;
+    t.n_opt = c->n_opt;
+    t.S = c->S;
+    t.J = c->J;
+    t.R = c->R;
+    t.P = c->P;
+    t.r_global = c->rg;
+    t.n_groups = c->n_groups;
+    return t;
+}
+
+DevState dev_state(const esp_ctx *c)
+{
+    DevState s;
+    s.lam = c->lam;
+    s.p64 = c->p64;
+    s.p32 = c->p32;
+    s.ebound = c->ebound;
+    s.U = c->U;
+    s.U_final = c->U_final;
+    s.hash = c->hash;
+    s.sel = c->sel;
+    s.job_val = c->job_val;
+    s.job_min = c->job_min;
+    s.rounds_run = c->rounds_run;
+    s.converged = c->converged;
+    s.status = c->status;
+    s.frozen = c->frozen;
+    s.best_dual = c->best_dual;
+    s.primal = c->primal;
+    s.dual = c->dual;
+    s.feasible = c->feasible;
+    s.vmax = c->vmax;
+    s.umax = c->umax;
+    s.err = c->err;
+    s.lam_trace = nullptr;
+    s.dem_trace = nullptr;
+    s.hash_trace = nullptr;
+    s.dual_trace = nullptr;
+    return s;
+}
+
+esp_status check_ctx(esp_ctx *ctx)
+{
+    if (!ctx)
+        return ESP_ERR_INVALID_ARG;
+    if (ctx->poisoned)
+        return ESP_ERR_STATE;
+    return ESP_OK;
+}
+
+esp_status check_shape(int32_t S, int32_t J, int32_t R, int32_t P, int32_t rg, bool grouped, int32_t *n_groups)
+{
+    if (S < 1 || J < 0 || R < 1 || R > kMaxR || P < 1)
+        return ESP_ERR_INVALID_ARG;
+    if (!grouped) {
+        if (P != R || rg != R)
+            return ESP_ERR_INVALID_ARG;
+        *n_groups = 0;
+        return ESP_OK;
+    }
+    if (rg < 0 || rg >= R)
+        return ESP_ERR_INVALID_ARG;
+    const int32_t per = R - rg;
+    if (P <= rg || (P - rg) % per != 0)
+        return ESP_ERR_INVALID_ARG;
+    const int32_t ng = (P - rg) / per;
+    if (ng < 1 || ng > 65536)
+        return ESP_ERR_INVALID_ARG;
+    *n_groups = ng;
+    return ESP_OK;
+}
+
+// Upload (host or device source), validate on the device, plan, allocate the solve state.
+esp_status load_common(esp_ctx *ctx, int32_t S, int32_t J, int32_t R, int32_t P, int32_t rg, const int64_t *job_off,
+                       const int32_t *units, const double *values, const uint16_t *group, const int64_t *capacity,
+                       bool device_src)
+{
+    esp_status st = check_ctx(ctx);
+    if (st != ESP_OK)
+        return st;
+    if (!job_off || !capacity || (J > 0 && (!units || !values)))
+        return ESP_ERR_INVALID_ARG;
+    int32_t n_groups = 0;
+    const bool grouped = group != nullptr;
+    if ((st = check_shape(S, J, R, P, rg, grouped, &n_groups)) != ESP_OK)
+        return st;
+    if (!grouped)
+        rg = R;
+    ESP_CUDA(cudaSetDevice(ctx->device));
+    release_table(ctx);
+
+    const int64_t n_jobs = (int64_t)S * J;
+    std::vector<int64_t> h_off;
+    const int64_t *off_host = job_off;
+    if (device_src) {
+        h_off.resize(n_jobs + 1);
+        ESP_CUDA(cudaMemcpyAsync(h_off.data(), job_off, (n_jobs + 1) * sizeof(int64_t), cudaMemcpyDeviceToHost,
+                                 ctx->stream));
+        ESP_CUDA(cudaStreamSynchronize(ctx->stream));
+        off_host = h_off.data();
+    }
+    const int64_t n_opt = off_host[n_jobs];
+    if (off_host[0] != 0 || n_opt < n_jobs || n_opt > ((int64_t)1 << 40))
+        return ESP_ERR_INVALID_ARG;
+
+    ctx->S = S;
+    ctx->J = J;
+    ctx->R = R;
+    ctx->P = P;
+    ctx->rg = rg;
+    ctx->n_groups = n_groups;
+    ctx->n_opt = n_opt;
+
+#define ALLOC(ptr, count)                                 \
+    do {                                                  \
+        esp_status a_ = dev_alloc(ctx, &(ptr), (count));  \
+        if (a_ != ESP_OK) {                               \
+            release_table(ctx);                           \
+            return a_;                                    \
+        }                                                 \
+    } while (0)
+
+    ALLOC(ctx->units, (size_t)n_opt * R);
+    ALLOC(ctx->values, (size_t)n_opt);
+    ALLOC(ctx->off, (size_t)n_jobs + 1);
+    ctx->group = nullptr;
+    if (grouped)
+        ALLOC(ctx->group, (size_t)n_opt);
+    ALLOC(ctx->cap, (size_t)S * P);
+    ALLOC(ctx->vmax, (size_t)S);
+    ALLOC(ctx->umax, (size_t)S * R);
+    ALLOC(ctx->valflags, 4);
+
+    const cudaMemcpyKind kind = device_src ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice;
+    ESP_CUDA(cudaMemcpyAsync(ctx->units, units, (size_t)n_opt * R * sizeof(int32_t), kind, ctx->stream));
+    ESP_CUDA(cudaMemcpyAsync(ctx->values, values, (size_t)n_opt * sizeof(double), kind, ctx->stream));
+    ESP_CUDA(cudaMemcpyAsync(ctx->off, job_off, (size_t)(n_jobs + 1) * sizeof(int64_t), kind, ctx->stream));
+    if (grouped)
+        ESP_CUDA(cudaMemcpyAsync(ctx->group, group, (size_t)n_opt * sizeof(uint16_t), kind, ctx->stream));
+    ESP_CUDA(cudaMemcpyAsync(ctx->cap, capacity, (size_t)S * P * sizeof(int64_t), kind, ctx->stream));
+
+    const DevTable t = dev_table(ctx);
+    ESP_CUDA(launch_validate(t, ctx->vmax, ctx->umax, ctx->valflags, ctx->stream));
+    unsigned int vflags = 0;
+    ESP_CUDA(cudaMemcpyAsync(&vflags, ctx->valflags, sizeof(unsigned int), cudaMemcpyDeviceToHost, ctx->stream));
+    ESP_CUDA(cudaStreamSynchronize(ctx->stream));
+    if (vflags != 0) {
+        release_table(ctx);
+        return ESP_ERR_INVALID_ARG;
+    }
+
+    // plan the evaluation pass
+    const int tile_opt = tile_options(R, grouped);
+    const int per_sm = pass_ctas_per_sm(R, grouped, P);
+    if (per_sm < 1) {
+        release_table(ctx);
+        return ESP_ERR_UNSUPPORTED;
+    }
+    const int max_warps = ctx->sm_count * per_sm * kWarpsPerCta;
+    Plan plan;
+    if (!plan_tiles(off_host, S, J, tile_opt, max_warps, plan) || !check_plan(off_host, S, J, plan)) {
+        release_table(ctx);
+        return ESP_ERR_INVALID_ARG;
+    }
+    ctx->n_warps = plan.n_warps;
+    ctx->tile_opt = plan.tile_opt;
+    ctx->grid = (plan.n_warps + kWarpsPerCta - 1) / kWarpsPerCta;
+    ALLOC(ctx->tiles, plan.tiles.size() + 1);
+    ALLOC(ctx->warp_begin, plan.warp_begin.size());
+    if (!plan.tiles.empty())
+        ESP_CUDA(cudaMemcpyAsync(ctx->tiles, plan.tiles.data(), plan.tiles.size() * sizeof(TileDesc),
+                                 cudaMemcpyHostToDevice, ctx->stream));
+    ESP_CUDA(cudaMemcpyAsync(ctx->warp_begin, plan.warp_begin.data(), plan.warp_begin.size() * sizeof(int32_t),
+                             cudaMemcpyHostToDevice, ctx->stream));
+
+    // solve state
+    const size_t SP = (size_t)S * P, SJ = (size_t)n_jobs;
+    ALLOC(ctx->lam, SP);
+    ALLOC(ctx->p64, SP);
+    ALLOC(ctx->p32, SP);
+    ALLOC(ctx->ebound, (size_t)S);
+    ALLOC(ctx->U, SP);
+    ALLOC(ctx->U_final, SP);
+    ALLOC(ctx->hash, (size_t)S);
+    ALLOC(ctx->sel, SJ);
+    ALLOC(ctx->job_val, SJ);
+    ALLOC(ctx->job_min, SJ);
+    ALLOC(ctx->rounds_run, (size_t)S);
+    ALLOC(ctx->converged, (size_t)S);
+    ALLOC(ctx->status, (size_t)S);
+    ALLOC(ctx->frozen, (size_t)S);
+    ALLOC(ctx->feasible, (size_t)S);
+    ALLOC(ctx->best_dual, (size_t)S);
+    ALLOC(ctx->primal, (size_t)S);
+    ALLOC(ctx->dual, (size_t)S);
+    ALLOC(ctx->lambda0, SP);
+    ALLOC(ctx->err, 4);
+#undef ALLOC
+    ESP_CUDA(cudaStreamSynchronize(ctx->stream));
+    ctx->loaded = true;
+    ctx->solved = false;
+    return ESP_OK;
+}
+
+esp_status check_params(const esp_ctx *ctx, const esp_params *p)
+{
+    if (!p)
+        return ESP_ERR_INVALID_ARG;
+    if (!(p->eta0 > 0.0) || !std::isfinite(p->eta0))
+        return ESP_ERR_INVALID_ARG;
+    if (p->step != ESP_STEP_FIXED && p->step != ESP_STEP_INV_SQRT)
+        return ESP_ERR_INVALID_ARG;
+    if (p->mode != ESP_PRICE_RAW && p->mode != ESP_PRICE_NORMALIZED)
+        return ESP_ERR_INVALID_ARG;
+    if (p->max_rounds < 0 || p->max_rounds > 100000000)
+        return ESP_ERR_INVALID_ARG;
+    if (!(p->tol >= 0.0) || !std::isfinite(p->tol))
+        return ESP_ERR_INVALID_ARG;
+    if (p->flags & ~(uint32_t)(ESP_FLAG_EXACT_ONLY | ESP_FLAG_PER_ROUND_LAUNCH))
+        return ESP_ERR_INVALID_ARG;
+    if (p->lambda0) {
+        const size_t n = (size_t)ctx->S * ctx->P;
+        for (size_t i = 0; i < n; ++i)
+            if (!(p->lambda0[i] >= 0.0) || !std::isfinite(p->lambda0[i]))
+                return ESP_ERR_INVALID_ARG;
+    }
+    return ESP_OK;
+}
+
+// Queues one whole solve on the stream (captured into a graph when the stream allows it).
+esp_status enqueue_solve(esp_ctx *ctx, const esp_params *p, const DevState &st, bool has_l0)
+{
+    const DevTable t = dev_table(ctx);
+    DevPlan pl;
+    pl.tiles = ctx->tiles;
+    pl.warp_begin = ctx->warp_begin;
+    pl.n_warps = ctx->n_warps;
+    pl.tile_opt = ctx->tile_opt;
+    SolveArgs a;
+    a.eta0 = p->eta0;
+    a.step = p->step;
+    a.mode = p->mode;
+    a.T = p->max_rounds;
+    a.tol = p->tol;
+    a.flags = p->flags;
+    a.exact_only = (p->flags & ESP_FLAG_EXACT_ONLY) ? 1 : 0;
+    const int T = p->max_rounds;
+
+    auto issue = [&]() -> cudaError_t {
+        cudaError_t e = launch_init(t, st, a, has_l0 ? ctx->lambda0 : nullptr, ctx->stream);
+        for (int r = 0; r < T && e == cudaSuccess; ++r) {
+            if (ctx->grid > 0)
+                e = launch_pass(t, st, pl, a, r, PASS_ROUND, ctx->grid, ctx->stream);
+            if (e == cudaSuccess)
+                e = launch_update(t, st, a, r, ctx->stream);
+        }
+        if (e == cudaSuccess && ctx->grid > 0)
+            e = launch_pass(t, st, pl, a, T, PASS_FINAL, ctx->grid, ctx->stream);
+        if (e == cudaSuccess)
+            e = launch_objectives(t, st, a, ctx->stream);
+        return e;
+    };
+    ctx->last_launches = 3 + 2LL * T - (ctx->grid > 0 ? 0 : (T + 1));
+    ctx->last_T = T;
+
+    GraphKey key;
+    key.eta0 = p->eta0;
+    key.tol = p->tol;
+    key.step = p->step;
+    key.mode = p->mode;
+    key.T = T;
+    key.flags = p->flags;
+    key.lt = st.lam_trace;
+    key.dt = st.dem_trace;
+    key.ht = st.hash_trace;
+    key.gt = st.dual_trace;
+    key.has_l0 = has_l0;
+
+    if (ctx->stream == nullptr) {   // the legacy default stream cannot be captured
+        ESP_CUDA(issue());
+        return ESP_OK;
+    }
+    if (!(ctx->gexec && ctx->gkey == key)) {
+        if (ctx->gexec) {
+            cudaGraphExecDestroy(ctx->gexec);
+            ctx->gexec = nullptr;
+        }
+        cudaGraph_t g = nullptr;
+        ESP_CUDA(cudaStreamBeginCapture(ctx->stream, cudaStreamCaptureModeThreadLocal));
+        cudaError_t e = issue();
+        cudaError_t e2 = cudaStreamEndCapture(ctx->stream, &g);
+        if (e != cudaSuccess || e2 != cudaSuccess) {
+            if (g)
+                cudaGraphDestroy(g);
+            return cuda_fail(ctx, e != cudaSuccess ? e : e2);
+        }
+        e = cudaGraphInstantiate(&ctx->gexec, g, 0);
+        cudaGraphDestroy(g);
+        if (e != cudaSuccess) {
+            ctx->gexec = nullptr;
+            return cuda_fail(ctx, e);
+        }
+        ctx->gkey = key;
+    }
+    ESP_CUDA(cudaGraphLaunch(ctx->gexec, ctx->stream));
+    return ESP_OK;
+}
+
+esp_status read_results(esp_ctx *ctx, esp_result *out)
+{
+    const int S = ctx->S;
+    std::vector<int32_t> rr(S), cv(S), ss(S), fe(S);
+    std::vector<double> pr(S), du(S), bd(S);
+    ESP_CUDA(cudaMemcpyAsync(rr.data(), ctx->rounds_run, S * 4, cudaMemcpyDeviceToHost, ctx->stream));
+    ESP_CUDA(cudaMemcpyAsync(cv.data(), ctx->converged, S * 4, cudaMemcpyDeviceToHost, ctx->stream));
+    ESP_CUDA(cudaMemcpyAsync(ss.data(), ctx->status, S * 4, cudaMemcpyDeviceToHost, ctx->stream));
+    ESP_CUDA(cudaMemcpyAsync(fe.data(), ctx->feasible, S * 4, cudaMemcpyDeviceToHost, ctx->stream));
+    ESP_CUDA(cudaMemcpyAsync(pr.data(), ctx->primal, S * 8, cudaMemcpyDeviceToHost, ctx->stream));
+    ESP_CUDA(cudaMemcpyAsync(du.data(), ctx->dual, S * 8, cudaMemcpyDeviceToHost, ctx->stream));
+    ESP_CUDA(cudaMemcpyAsync(bd.data(), ctx->best_dual, S * 8, cudaMemcpyDeviceToHost, ctx->stream));
+    ESP_CUDA(cudaStreamSynchronize(ctx->stream));
+    bool overflow = false;
+    for (int s = 0; s < S; ++s) {
+        out[s].rounds_run = rr[s];
+        out[s].converged = cv[s];
+        out[s].feasible = fe[s];
+        out[s].status = ss[s] ? ESP_ERR_OVERFLOW : ESP_OK;
+        out[s].primal = pr[s];
+        out[s].dual = du[s];
+        out[s].best_dual = bd[s];
+        overflow |= ss[s] != 0;
+    }
+    return overflow ? ESP_ERR_OVERFLOW : ESP_OK;
+}
+
+esp_status check_device_error(esp_ctx *ctx)
+{
+    unsigned int e = 0;
+    ESP_CUDA(cudaMemcpyAsync(&e, ctx->err, sizeof(e), cudaMemcpyDeviceToHost, ctx->stream));
+    ESP_CUDA(cudaStreamSynchronize(ctx->stream));
+    if (e & DEV_ERR_TIMEOUT) {
+        ctx->poisoned = true;
+        return ESP_ERR_TIMEOUT;
+    }
+    return ESP_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char *esp_status_string(esp_status s)
+{
+    switch (s) {
+    case ESP_OK: return "ok";
+    case ESP_ERR_INVALID_ARG: return "invalid argument";
+    case ESP_ERR_OVERFLOW: return "overflow (a price became non-finite)";
+    case ESP_ERR_OOM: return "out of memory";
+    case ESP_ERR_CUDA: return "CUDA error";
+    case ESP_ERR_NOT_LOADED: return "no table loaded / nothing solved";
+    case ESP_ERR_TIMEOUT: return "device wait timed out";
+    case ESP_ERR_STATE: return "context unusable after an earlier CUDA error or timeout";
+    case ESP_ERR_UNSUPPORTED: return "unsupported device";
+    }
+    return "unknown status";
+}
+
+esp_status esp_create(esp_ctx **out, int device, void *cuda_stream)
+{
+    if (!out)
+        return ESP_ERR_INVALID_ARG;
+    *out = nullptr;
+    int n = 0;
+    if (cudaGetDeviceCount(&n) != cudaSuccess || n == 0) {
+        cudaGetLastError();
+        return ESP_ERR_UNSUPPORTED;
+    }
+    if (device < 0) {
+        if (cudaGetDevice(&device) != cudaSuccess)
+            return ESP_ERR_CUDA;
+    }
+    if (device >= n)
+        return ESP_ERR_INVALID_ARG;
+    cudaDeviceProp prop;
+    if (cudaGetDeviceProperties(&prop, device) != cudaSuccess)
+        return ESP_ERR_CUDA;
+    if (prop.major != 10 || prop.minor != 3)
+        return ESP_ERR_UNSUPPORTED;
+    esp_ctx *ctx = new (std::nothrow) esp_ctx();
+    if (!ctx)
+        return ESP_ERR_OOM;
+    ctx->device = device;
+    ctx->stream = static_cast<cudaStream_t>(cuda_stream);
+    ctx->sm_count = prop.multiProcessorCount;
+    if (cudaSetDevice(device) != cudaSuccess) {
+        delete ctx;
+        return ESP_ERR_CUDA;
+    }
+    *out = ctx;
+    return ESP_OK;
+}
+
+esp_status esp_set_stream(esp_ctx *ctx, void *cuda_stream)
+{
+    esp_status st = check_ctx(ctx);
+    if (st != ESP_OK)
+        return st;
+    if (ctx->stream != static_cast<cudaStream_t>(cuda_stream) && ctx->gexec) {
+        cudaGraphExecDestroy(ctx->gexec);
+        ctx->gexec = nullptr;
+        ctx->gkey = GraphKey();
+    }
+    ctx->stream = static_cast<cudaStream_t>(cuda_stream);
+    return ESP_OK;
+}
+
+esp_status esp_load_options(esp_ctx *ctx, int32_t S, int32_t J, int32_t R, int32_t P, int32_t r_global,
+                            const int64_t *job_offsets, const int32_t *units, const double *values,
+                            const uint16_t *group, const int64_t *capacity)
+{
+    return load_common(ctx, S, J, R, P, r_global, job_offsets, units, values, group, capacity, false);
+}
+
+esp_status esp_load_options_device(esp_ctx *ctx, int32_t S, int32_t J, int32_t R, int32_t P, int32_t r_global,
+                                   const int64_t *job_offsets, const int32_t *units, const double *values,
+                                   const uint16_t *group, const int64_t *capacity)
+{
+    return load_common(ctx, S, J, R, P, r_global, job_offsets, units, values, group, capacity, true);
+}
+
+esp_status esp_solve_async(esp_ctx *ctx, const esp_params *params)
+{
+    esp_status st = check_ctx(ctx);
+    if (st != ESP_OK)
+        return st;
+    if (!ctx->loaded)
+        return ESP_ERR_NOT_LOADED;
+    if ((st = check_params(ctx, params)) != ESP_OK)
+        return st;
+    if (params->lambda_trace || params->demand_trace || params->selhash_trace || params->dual_trace)
+        return ESP_ERR_INVALID_ARG;
+    ESP_CUDA(cudaSetDevice(ctx->device));
+    const size_t SP = (size_t)ctx->S * ctx->P;
+    if (params->lambda0)
+        ESP_CUDA(cudaMemcpyAsync(ctx->lambda0, params->lambda0, SP * sizeof(double), cudaMemcpyHostToDevice,
+                                 ctx->stream));
+    const DevState ds = dev_state(ctx);
+    if ((st = enqueue_solve(ctx, params, ds, params->lambda0 != nullptr)) != ESP_OK)
+        return st;
+    ctx->solved = true;
+    return ESP_OK;
+}
+
+esp_status esp_solve(esp_ctx *ctx, const esp_params *params, esp_result *out)
+{
+    esp_status st = check_ctx(ctx);
+    if (st != ESP_OK)
+        return st;
+    if (!ctx->loaded)
+        return ESP_ERR_NOT_LOADED;
+    if ((st = check_params(ctx, params)) != ESP_OK)
+        return st;
+    ESP_CUDA(cudaSetDevice(ctx->device));
+    const size_t S = ctx->S, P = ctx->P, T = params->max_rounds;
+    if (params->lambda0)
+        ESP_CUDA(cudaMemcpyAsync(ctx->lambda0, params->lambda0, S * P * sizeof(double), cudaMemcpyHostToDevice,
+                                 ctx->stream));
+    DevState ds = dev_state(ctx);
+    // traces: device copies start from the caller's contents, so rows never written stay as they were
+    if (params->lambda_trace) {
+        if ((st = grow(ctx, ctx->lt, S * (T + 1) * P)) != ESP_OK)
+            return st;
+        ESP_CUDA(cudaMemcpyAsync(ctx->lt.p, params->lambda_trace, S * (T + 1) * P * 8, cudaMemcpyHostToDevice,
+                                 ctx->stream));
+        ds.lam_trace = ctx->lt.p;
+    }
+    if (params->demand_trace && T > 0) {
+        if ((st = grow(ctx, ctx->dt, S * T * P)) != ESP_OK)
+            return st;
+        ESP_CUDA(cudaMemcpyAsync(ctx->dt.p, params->demand_trace, S * T * P * 8, cudaMemcpyHostToDevice,
+                                 ctx->stream));
+        ds.dem_trace = ctx->dt.p;
+    }
+    if (params->selhash_trace && T > 0) {
+        if ((st = grow(ctx, ctx->ht, S * T)) != ESP_OK)
+            return st;
+        ESP_CUDA(cudaMemcpyAsync(ctx->ht.p, params->selhash_trace, S * T * 8, cudaMemcpyHostToDevice, ctx->stream));
+        ds.hash_trace = ctx->ht.p;
+    }
+    if (params->dual_trace) {
+        if ((st = grow(ctx, ctx->gt, S * (T + 1))) != ESP_OK)
+            return st;
+        ESP_CUDA(cudaMemcpyAsync(ctx->gt.p, params->dual_trace, S * (T + 1) * 8, cudaMemcpyHostToDevice, ctx->stream));
+        ds.dual_trace = ctx->gt.p;
+    }
+    if ((st = enqueue_solve(ctx, params, ds, params->lambda0 != nullptr)) != ESP_OK)
+        return st;
+    ctx->solved = true;
+    if ((st = check_device_error(ctx)) != ESP_OK)
+        return st;
+    if (params->lambda_trace)
+        ESP_CUDA(cudaMemcpyAsync(params->lambda_trace, ctx->lt.p, S * (T + 1) * P * 8, cudaMemcpyDeviceToHost,
+                                 ctx->stream));
+    if (ds.dem_trace)
+        ESP_CUDA(cudaMemcpyAsync(params->demand_trace, ctx->dt.p, S * T * P * 8, cudaMemcpyDeviceToHost, ctx->stream));
+    if (ds.hash_trace)
+        ESP_CUDA(cudaMemcpyAsync(params->selhash_trace, ctx->ht.p, S * T * 8, cudaMemcpyDeviceToHost, ctx->stream));
+    if (params->dual_trace)
+        ESP_CUDA(cudaMemcpyAsync(params->dual_trace, ctx->gt.p, S * (T + 1) * 8, cudaMemcpyDeviceToHost, ctx->stream));
+    if (out)
+        return read_results(ctx, out);
+    ESP_CUDA(cudaStreamSynchronize(ctx->stream));
+    return ESP_OK;
+}
+
+esp_status esp_get_result(esp_ctx *ctx, esp_result *out)
+{
+    esp_status st = check_ctx(ctx);
+    if (st != ESP_OK)
+        return st;
+    if (!out)
+        return ESP_ERR_INVALID_ARG;
+    if (!ctx->solved)
+        return ESP_ERR_NOT_LOADED;
+    if ((st = check_device_error(ctx)) != ESP_OK)
+        return st;
+    return read_results(ctx, out);
+}
+
+static esp_status get_array(esp_ctx *ctx, void *out, const void *src, size_t bytes)
+{
+    esp_status st = check_ctx(ctx);
+    if (st != ESP_OK)
+        return st;
+    if (!out)
+        return ESP_ERR_INVALID_ARG;
+    if (!ctx->solved)
+        return ESP_ERR_NOT_LOADED;
+    if ((st = check_device_error(ctx)) != ESP_OK)
+        return st;
+    ESP_CUDA(cudaMemcpyAsync(out, src, bytes, cudaMemcpyDeviceToHost, ctx->stream));
+    ESP_CUDA(cudaStreamSynchronize(ctx->stream));
+    return ESP_OK;
+}
+
+esp_status esp_get_prices(esp_ctx *ctx, double *out)
+{
+    if (!ctx)
+        return ESP_ERR_INVALID_ARG;
+    return get_array(ctx, out, ctx->lam, (size_t)ctx->S * ctx->P * sizeof(double));
+}
+
+esp_status esp_get_selection(esp_ctx *ctx, int32_t *out)
+{
+    if (!ctx)
+        return ESP_ERR_INVALID_ARG;
+    return get_array(ctx, out, ctx->sel, (size_t)ctx->S * ctx->J * sizeof(int32_t));
+}
+
+esp_status esp_get_demand(esp_ctx *ctx, int64_t *out)
+{
+    if (!ctx)
+        return ESP_ERR_INVALID_ARG;
+    return get_array(ctx, out, ctx->U_final, (size_t)ctx->S * ctx->P * sizeof(int64_t));
+}
+
+esp_status esp_evaluate(esp_ctx *ctx, const double *lambda, int32_t mode, uint32_t flags, int32_t *sel,
+                        int64_t *demand, double *min_score)
+{
+    esp_status st = check_ctx(ctx);
+    if (st != ESP_OK)
+        return st;
+    if (!ctx->loaded)
+        return ESP_ERR_NOT_LOADED;
+    if (!lambda || (mode != ESP_PRICE_RAW && mode != ESP_PRICE_NORMALIZED) || (flags & ~ESP_FLAG_EXACT_ONLY))
+        return ESP_ERR_INVALID_ARG;
+    const size_t SP = (size_t)ctx->S * ctx->P, SJ = (size_t)ctx->S * ctx->J;
+    for (size_t i = 0; i < SP; ++i)
+        if (!(lambda[i] >= 0.0) || !std::isfinite(lambda[i]))
+            return ESP_ERR_INVALID_ARG;
+    ESP_CUDA(cudaSetDevice(ctx->device));
+    ESP_CUDA(cudaMemcpyAsync(ctx->lambda0, lambda, SP * sizeof(double), cudaMemcpyHostToDevice, ctx->stream));
+    const DevTable t = dev_table(ctx);
+    DevState ds = dev_state(ctx);
+    DevPlan pl;
+    pl.tiles = ctx->tiles;
+    pl.warp_begin = ctx->warp_begin;
+    pl.n_warps = ctx->n_warps;
+    pl.tile_opt = ctx->tile_opt;
+    SolveArgs a;
+    a.eta0 = 1.0;
+    a.step = 0;
+    a.mode = mode;
+    a.T = 0;
+    a.tol = 0.0;
+    a.flags = flags;
+    a.exact_only = (flags & ESP_FLAG_EXACT_ONLY) ? 1 : 0;
+    ESP_CUDA(launch_init(t, ds, a, ctx->lambda0, ctx->stream));
+    if (ctx->grid > 0)
+        ESP_CUDA(launch_pass(t, ds, pl, a, 0, PASS_FINAL, ctx->grid, ctx->stream));
+    ESP_CUDA(launch_objectives(t, ds, a, ctx->stream));
+    ctx->solved = true;
+    if ((st = check_device_error(ctx)) != ESP_OK)
+        return st;
+    if (sel)
+        ESP_CUDA(cudaMemcpyAsync(sel, ctx->sel, SJ * 4, cudaMemcpyDeviceToHost, ctx->stream));
+    if (demand)
+        ESP_CUDA(cudaMemcpyAsync(demand, ctx->U_final, SP * 8, cudaMemcpyDeviceToHost, ctx->stream));
+    if (min_score)
+        ESP_CUDA(cudaMemcpyAsync(min_score, ctx->job_min, SJ * 8, cudaMemcpyDeviceToHost, ctx->stream));
+    ESP_CUDA(cudaStreamSynchronize(ctx->stream));
+    return ESP_OK;
+}
+
+esp_status esp_last_launch_count(esp_ctx *ctx, int64_t *out)
+{
+    if (!ctx || !out)
+        return ESP_ERR_INVALID_ARG;
+    *out = ctx->last_launches;
+    return ESP_OK;
+}
+
+void esp_destroy(esp_ctx *ctx)
+{
+    if (!ctx)
+        return;
+    cudaSetDevice(ctx->device);
+    if (!ctx->poisoned)
+        cudaStreamSynchronize(ctx->stream);
+    release_table(ctx);
+    if (ctx->lt.p) cudaFree(ctx->lt.p);
+    if (ctx->dt.p) cudaFree(ctx->dt.p);
+    if (ctx->ht.p) cudaFree(ctx->ht.p);
+    if (ctx->gt.p) cudaFree(ctx->gt.p);
+    delete ctx;
+}
+
+int32_t esp_debug_tile_options(int32_t R, int32_t grouped)
+{
+    return tile_options(R, grouped != 0);
+}
+
+esp_status esp_debug_plan(const int64_t *job_offsets, int32_t S, int32_t J, int32_t tile_opt, int32_t max_warps,
+                          int32_t *tiles, int32_t tiles_cap, int32_t *warp_begin, int32_t warps_cap,
+                          int32_t *n_tiles, int32_t *n_warps)
+{
+    if (!job_offsets || S < 1 || J < 0 || !n_tiles || !n_warps)
+        return ESP_ERR_INVALID_ARG;
+    Plan p;
+    if (!plan_tiles(job_offsets, S, J, tile_opt, max_warps, p) || !check_plan(job_offsets, S, J, p))
+        return ESP_ERR_INVALID_ARG;
+    *n_tiles = (int32_t)p.tiles.size();
+    *n_warps = p.n_warps;
+    if ((int32_t)p.tiles.size() > tiles_cap || p.n_warps + 1 > warps_cap + 1 || !tiles || !warp_begin)
+        return ESP_ERR_OOM;
+    for (size_t i = 0; i < p.tiles.size(); ++i) {
+        const TileDesc &d = p.tiles[i];
+        int32_t *w = tiles + 8 * i;
+        w[0] = (int32_t)(uint32_t)(d.opt_begin & 0xffffffff);
+        w[1] = (int32_t)(d.opt_begin >> 32);
+        w[2] = (int32_t)(uint32_t)(d.job_begin & 0xffffffff);
+        w[3] = (int32_t)(d.job_begin >> 32);
+        w[4] = d.n_opt;
+        w[5] = d.n_job;
+        w[6] = d.scenario;
+        w[7] = (int32_t)d.flags;
+    }
+    for (int32_t w = 0; w <= p.n_warps; ++w)
+        warp_begin[w] = p.warp_begin[w];
+    return ESP_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,98 @@
+// Shared host/device definitions of the ESP solver library (not part of the public ABI).
+#pragma once
+
+#include <cstdint>
+
+#if defined(__CUDACC__)
+#define ESP_HD __host__ __device__ __forceinline__
+#else
+#define ESP_HD inline
+#endif
+
+namespace esp {
+
+constexpr int kMaxR = 16;            // stored resource columns per option
+constexpr int kWarpsPerCta = 4;      // warps of a CTA; each warp owns its own stage ring
+constexpr int kStages = 2;           // TMA stages per warp
+constexpr int kStageDataBytes = 8192;// option bytes (units + values [+ group]) one stage aims at
+
+// Tile flags. A tile is a run of whole jobs of one scenario whose options are contiguous, or one
+// chunk of a job with more options than a tile holds ("big" job).
+enum : uint32_t {
+    TILE_BIG = 1u,        // chunk of a big job
+    TILE_BIG_FIRST = 2u,  // first chunk of its job
+    TILE_BIG_LAST = 4u,   // last chunk of its job
+};
+
+struct TileDesc {
+    int64_t opt_begin;    // first global option of the tile
+    int64_t job_begin;    // global job index (s*J + j) of the first job starting in the tile, or of the big job
+    int32_t n_opt;        // options in the tile (1 .. tile_opt)
+    int32_t n_job;        // jobs starting in the tile (big chunks: 1 on the first chunk, else 0)
+    int32_t scenario;
+    uint32_t flags;
+};
+static_assert(sizeof(TileDesc) == 32, "TileDesc is 32 bytes");
+
+// Options per tile for R stored columns: about kStageDataBytes of option data, a multiple of 32.
+ESP_HD int tile_options(int R, bool grouped)
+{
+    int per = 4 * R + 8 + (grouped ? 2 : 0);
+    int t = (kStageDataBytes / per) & ~31;
+    return t < 32 ? 32 : t;
+}
+
+ESP_HD int round16(int x) { return (x + 15) & ~15; }
+
+// Byte layout of one stage. Every region starts 16-byte aligned and has room for the up-to-15
+// bytes the bulk copy reads before and after its data to keep source and size 16-byte aligned.
+struct StageLayout {
+    int off, units, vals, grp, bytes;
+};
+
+ESP_HD StageLayout stage_layout(int tile_opt, int R, bool grouped)
+{
+    StageLayout L;
+    L.off = 0;
+    L.units = round16((tile_opt + 1) * 8 + 32);
+    L.vals = L.units + round16(tile_opt * R * 4 + 32);
+    L.grp = L.vals + round16(tile_opt * 8 + 32);
+    L.bytes = L.grp + (grouped ? round16(tile_opt * 2 + 32) : 0);
+    return L;
+}
+
+// Per-warp shared memory: kStages stages, the fp32 screen values of the current tile, the fp32
+// prices of the current scenario (grouped tables) and the stage barriers.
+struct WarpSmem {
+    int stage_bytes, qbuf, p32, bars, bytes;
+};
+
+ESP_HD WarpSmem warp_smem(int tile_opt, int R, bool grouped, int P)
+{
+    WarpSmem W;
+    StageLayout L = stage_layout(tile_opt, R, grouped);
+    W.stage_bytes = L.bytes;
+    W.qbuf = kStages * L.bytes;
+    W.p32 = W.qbuf + round16(tile_opt * 4);
+    W.bars = W.p32 + (grouped ? round16(P * 4) : 0);
+    W.bytes = W.bars + 16 * kStages;
+    return W;
+}
+
+// Device status words (bit flags in ctx error word).
+enum : uint32_t {
+    DEV_ERR_TIMEOUT = 1u,
+    DEV_ERR_BAD_TABLE = 2u,
+    DEV_ERR_PLAN = 4u,
+};
+
+// Load-time validation flags.
+enum : uint32_t {
+    VAL_UNITS_NEG = 1u,
+    VAL_VALUE_NONFINITE = 2u,
+    VAL_OFFSETS = 4u,
+    VAL_GROUP_RANGE = 8u,
+    VAL_CAPACITY = 16u,
+};
+
+}  // namespace esp

@@ -1,0 +1,1066 @@
+// Device kernels of the ESP tatonnement (Sec. 3.2 of the paper) for sm_103a.
+//
+// One evaluation pass (a best response of every job, Sec. 3.2.2; Eq. esp_score without Gamma) runs
+// as warps that each own a static list of tiles. A tile is a run of whole jobs of one scenario (or
+// one chunk of a job larger than a tile); its option bytes are contiguous in HBM and arrive in the
+// warp's shared-memory stage by 1-D bulk copies (cp.async.bulk + mbarrier), one tile ahead of the
+// tile being evaluated.
+//
+// Exactness. The returned choice is the lexicographic minimum of (s, local index) with
+//   s = fma(p_{R-1}, u_{R-1}, ... fma(p_0, u_0, -v))         (fp64, r = 0 .. R-1)
+// exactly as the oracle computes it. GB300 runs fp64 at a small fraction of its fp32 rate, so each
+// option is first scored in fp32, q = the same chain in fp32, with |q - s| <= E for every option of
+// the scenario (E from the bound below). A job whose smallest q beats every other q by more than 2E
+// has that option as its exact argmin; otherwise every option with q <= m1 + 2E (rounded up) is
+// rescored in fp64 and the exact lexicographic minimum is taken. Proof: s_i <= s_w implies
+// q_i - E <= s_i <= s_w <= q_w + E = m1 + E. The bound (fp32 unit roundoff u = 2^-24, all
+// magnitudes M = |v| + sum_r p_r u_r, inputs rounded to fp32 once, R fused steps, fp64 error
+// R 2^-53 M, subnormal absolute error below 2^-100 in total) is
+//   |q - s| <= (R + 3) u M (1 + small) + 2^-100 ;   E = (4R + 16) u M_s + 2^-100,
+// with M_s = max|v| + sum_r max p_r * max u_r over the scenario, a factor of about 4 to spare.
+// A scenario whose prices or values leave [2^-100, 2^100] in magnitude is evaluated in fp64 only.
+//
+// Aggregation. Demands of the chosen options are summed in int64 registers per lane, reduced
+// across the warp and added with one 64-bit atomic per priced resource per warp and scenario:
+// integer addition is associative, so U is identical on every run.
+
+#include <cmath>
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "esp_kernels.h"
+
+namespace esp {
+
+namespace {
+
+constexpr unsigned FULL = 0xffffffffu;
+constexpr int kIdxNone = 0x7fffffff;
+
+// ---------------------------------------------------------------------------------------------
+// PTX helpers: mbarrier + 1-D bulk copy (TMA engine), sm_90+ forms that sm_103a accepts.
+
+__device__ __forceinline__ uint32_t smem_u32(const void *p)
+{
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count)
+{
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void fence_barrier_init()
+{
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes)
+{
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity)
+{
+    uint32_t done;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(done)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return done != 0;
+}
+
+__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void *src, uint32_t bytes, uint32_t bar)
+{
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+        "l"(src), "r"(bytes), "r"(bar)
+        : "memory");
+}
+
+__device__ __forceinline__ void fence_proxy_async()
+{
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+// Bounded wait on a stage barrier: gives up after ~2^26 polls (seconds), flags a timeout and
+// returns false so the kernel can finish instead of hanging.
+__device__ __forceinline__ bool wait_stage(uint32_t bar, uint32_t parity, unsigned int *err)
+{
+    for (uint32_t it = 0; it < (1u << 26); ++it) {
+        if (mbar_try_wait(bar, parity))
+            return true;
+        if (it > 64)
+            __nanosleep(32);
+    }
+    atomicOr(err, DEV_ERR_TIMEOUT);
+    return false;
+}
+
+__device__ __forceinline__ uint64_t splitmix64_mix(uint64_t z)
+{
+    z = (z ^ (z >> 30)) * 0xbf58476d1ce4e5b9ULL;
+    z = (z ^ (z >> 27)) * 0x94d049bb133111ebULL;
+    return z ^ (z >> 31);
+}
+
+// ---------------------------------------------------------------------------------------------
+// Per-job running state of the fp32 screen: the smallest q with its index, and the smallest q of
+// every other option. Commutative and associative (ties keep the lower index).
+
+struct Best {
+    float m1;
+    int idx;
+    float m2;
+};
+
+__device__ __forceinline__ Best best_none() { return Best{INFINITY, kIdxNone, INFINITY}; }
+
+__device__ __forceinline__ Best combine(const Best &a, const Best &b)
+{
+    const bool take_b = (b.m1 < a.m1) || (b.m1 == a.m1 && b.idx < a.idx);
+    const Best &lo = take_b ? b : a;
+    const Best &hi = take_b ? a : b;
+    return Best{lo.m1, lo.idx, fminf(fminf(lo.m2, hi.m2), hi.m1)};
+}
+
+__device__ __forceinline__ Best shfl_up_best(const Best &x, int d)
+{
+    return Best{__shfl_up_sync(FULL, x.m1, d), __shfl_up_sync(FULL, x.idx, d), __shfl_up_sync(FULL, x.m2, d)};
+}
+
+__device__ __forceinline__ Best shfl_best(const Best &x, int src)
+{
+    return Best{__shfl_sync(FULL, x.m1, src), __shfl_sync(FULL, x.idx, src), __shfl_sync(FULL, x.m2, src)};
+}
+
+__device__ __forceinline__ Best allreduce_best(Best x)
+{
+#pragma unroll
+    for (int d = 16; d >= 1; d >>= 1)
+        x = combine(x, Best{__shfl_xor_sync(FULL, x.m1, d), __shfl_xor_sync(FULL, x.idx, d),
+                            __shfl_xor_sync(FULL, x.m2, d)});
+    return x;
+}
+
+// Exact (s, idx) lexicographic minimum across the warp.
+__device__ __forceinline__ void allreduce_exact(double &s, int &idx)
+{
+#pragma unroll
+    for (int d = 16; d >= 1; d >>= 1) {
+        const double os = __shfl_xor_sync(FULL, s, d);
+        const int oi = __shfl_xor_sync(FULL, idx, d);
+        if (os < s || (os == s && oi < idx)) {
+            s = os;
+            idx = oi;
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------------------------
+// Scoring. Both chains run r = 0 .. R-1 with one correctly rounded fused multiply-add per column.
+
+template <int RT>
+struct Cols {
+    static constexpr int N = RT ? RT : kMaxR;
+};
+
+struct ScenarioPrices {
+    float pf[kMaxR];       // fp32 per-unit price of each globally priced stored column
+    double pd[kMaxR];      // fp64 per-unit price of each globally priced stored column
+    const float *p32s;     // fp32 prices of the scenario in shared memory (grouped tables)
+    const double *p64g;    // fp64 prices of the scenario in global memory
+    float e2;              // 2E, +inf: exact evaluation
+    bool exact;
+    bool skip;             // scenario already stopped
+};
+
+template <int RT>
+__device__ __forceinline__ float screen_score(const int32_t *u, double v, int g, const ScenarioPrices &sp, int R,
+                                              int rg, bool grouped)
+{
+    float q = -__double2float_rn(v);
+#pragma unroll
+    for (int r = 0; r < Cols<RT>::N; ++r) {
+        if (RT == 0 && r >= R)
+            break;
+        float price;
+        if (grouped && r >= rg)
+            price = sp.p32s[rg + (R - rg) * g + (r - rg)];
+        else
+            price = sp.pf[r];
+        q = __fmaf_rn(price, __int2float_rn(u[r]), q);
+    }
+    return q;
+}
+
+template <int RT>
+__device__ __forceinline__ double exact_score(const int32_t *u, double v, int g, const ScenarioPrices &sp, int R,
+                                              int rg, bool grouped)
+{
+    double s = -v;
+#pragma unroll
+    for (int r = 0; r < Cols<RT>::N; ++r) {
+        if (RT == 0 && r >= R)
+            break;
+        double price;
+        if (grouped && r >= rg)
+            price = __ldg(sp.p64g + rg + (R - rg) * g + (r - rg));
+        else
+            price = sp.pd[r];
+        s = __fma_rn(price, __int2double_rn(u[r]), s);
+    }
+    return s;
+}
+
+template <int RT>
+__device__ __forceinline__ void load_units_smem(const int32_t *p, int32_t *u, int R)
+{
+    if (RT == 4) {
+        const int4 a = *reinterpret_cast<const int4 *>(p);
+        u[0] = a.x; u[1] = a.y; u[2] = a.z; u[3] = a.w;
+    } else if (RT == 6) {
+        const int2 a = reinterpret_cast<const int2 *>(p)[0];
+        const int2 b = reinterpret_cast<const int2 *>(p)[1];
+        const int2 c = reinterpret_cast<const int2 *>(p)[2];
+        u[0] = a.x; u[1] = a.y; u[2] = b.x; u[3] = b.y; u[4] = c.x; u[5] = c.y;
+    } else if (RT == 8) {
+        const int4 a = reinterpret_cast<const int4 *>(p)[0];
+        const int4 b = reinterpret_cast<const int4 *>(p)[1];
+        u[0] = a.x; u[1] = a.y; u[2] = a.z; u[3] = a.w; u[4] = b.x; u[5] = b.y; u[6] = b.z; u[7] = b.w;
+    } else {
+#pragma unroll
+        for (int r = 0; r < Cols<RT>::N; ++r)
+            u[r] = (r < R) ? p[r] : 0;
+    }
+}
+
+template <int RT>
+__device__ __forceinline__ void load_units_global(const int32_t *p, int32_t *u, int R)
+{
+#pragma unroll
+    for (int r = 0; r < Cols<RT>::N; ++r)
+        u[r] = (RT != 0 || r < R) ? __ldg(p + r) : 0;
+}
+
+// ---------------------------------------------------------------------------------------------
+// The warp's evaluation context.
+
+template <int RT>
+struct WarpCtx {
+    // table and outputs
+    DevTable t;
+    DevState st;
+    int R, rg;
+    bool grouped;
+    int kind;                 // PassKind
+    bool want_min;            // job_min needed (final pass or dual trace)
+    bool want_hash;           // selection fingerprint needed
+    // scenario
+    int s;
+    ScenarioPrices sp;
+    // accumulators (per lane)
+    long long acc[Cols<RT>::N];
+    unsigned long long hacc;
+};
+
+template <int RT>
+__device__ void flush(WarpCtx<RT> &c, int lane)
+{
+    if (c.s < 0)
+        return;
+    const int ncol = c.grouped ? c.rg : c.R;
+    unsigned long long *dst = (c.kind == PASS_ROUND ? c.st.U : c.st.U_final) + (size_t)c.s * c.t.P;
+#pragma unroll
+    for (int r = 0; r < Cols<RT>::N; ++r) {
+        if (r >= ncol)
+            break;
+        long long v = c.acc[r];
+#pragma unroll
+        for (int d = 16; d >= 1; d >>= 1)
+            v += __shfl_xor_sync(FULL, v, d);
+        if (lane == 0 && v != 0)
+            atomicAdd(dst + r, (unsigned long long)v);
+        c.acc[r] = 0;
+    }
+    if (c.want_hash) {
+        unsigned long long h = c.hacc;
+#pragma unroll
+        for (int d = 16; d >= 1; d >>= 1)
+            h += __shfl_xor_sync(FULL, h, d);
+        if (lane == 0)
+            atomicAdd(c.st.hash + c.s, h);
+        c.hacc = 0;
+    }
+}
+
+template <int RT>
+__device__ void enter_scenario(WarpCtx<RT> &c, int s, float *p32s_smem, int lane)
+{
+    flush(c, lane);
+    c.s = s;
+    const int P = c.t.P;
+    c.sp.skip = (c.kind == PASS_ROUND) && (__ldcg(c.st.frozen + s) != 0);
+    const float e = __ldcg(c.st.ebound + s);
+    c.sp.exact = !(e < INFINITY);
+    c.sp.e2 = c.sp.exact ? INFINITY : 2.0f * e;
+    c.sp.p64g = c.st.p64 + (size_t)s * P;
+    const int ncol = c.grouped ? c.rg : c.R;
+#pragma unroll
+    for (int r = 0; r < Cols<RT>::N; ++r) {
+        const bool have = r < ncol;
+        c.sp.pf[r] = have ? __ldcg(c.st.p32 + (size_t)s * P + r) : 0.0f;
+        c.sp.pd[r] = have ? __ldcg(c.st.p64 + (size_t)s * P + r) : 0.0;
+    }
+    if (c.grouped) {
+        __syncwarp();
+        for (int k = lane; k < P; k += 32)
+            p32s_smem[k] = __ldcg(c.st.p32 + (size_t)s * P + k);
+        __syncwarp();
+        c.sp.p32s = p32s_smem;
+    } else {
+        c.sp.p32s = nullptr;
+    }
+}
+
+// Records the winner of a job: demand, fingerprint, and the per-job outputs of the final pass.
+// u/v are the winner's units and value; s64 its exact reduced cost when already known.
+template <int RT>
+__device__ __forceinline__ void take_winner(WarpCtx<RT> &c, int64_t job, int local, const int32_t *u, double v,
+                                            int g, bool have_s64, double s64)
+{
+    const int R = c.R;
+    const int P = c.t.P;
+#pragma unroll
+    for (int r = 0; r < Cols<RT>::N; ++r) {
+        if (RT == 0 && r >= R)
+            break;
+        if (c.grouped && r >= c.rg) {
+            unsigned long long *dst = (c.kind == PASS_ROUND ? c.st.U : c.st.U_final) + (size_t)c.s * P;
+            atomicAdd(dst + c.rg + (R - c.rg) * g + (r - c.rg), (unsigned long long)(long long)u[r]);
+        } else {
+            c.acc[r] += u[r];
+        }
+    }
+    if (c.want_hash)
+        c.hacc += splitmix64_mix(((uint64_t)(uint32_t)(job - (int64_t)c.s * c.t.J) << 32) | (uint32_t)local);
+    if (c.kind == PASS_FINAL) {
+        c.st.sel[job] = local;
+        c.st.job_val[job] = v;
+    }
+    if (c.want_min) {
+        if (!have_s64)
+            s64 = exact_score<RT>(u, v, g, c.sp, R, c.rg, c.grouped);
+        c.st.job_min[job] = s64;
+    }
+}
+
+// Exact resolution of one job whose screen was ambiguous: every option with q <= thr (all options
+// in exact mode) is rescored in fp64; returns the lexicographic minimum of (s, job-local index).
+// In-tile jobs read the stage; chunked (big) jobs read global memory and recompute q identically.
+template <int RT>
+__device__ void resolve_job(WarpCtx<RT> &c, int lane, bool in_smem, const int32_t *units_s, const double *vals_s,
+                            const uint16_t *grp_s, const float *qbuf, int jstart, int jend, int64_t gfirst,
+                            float thr, double &s_out, int &local_out)
+{
+    const int R = c.R;
+    double best_s = INFINITY;
+    int best_i = kIdxNone;
+    int32_t u[Cols<RT>::N];
+    for (int o = jstart + lane; o < jend; o += 32) {
+        double v;
+        int g = 0;
+        float q;
+        if (in_smem) {
+            load_units_smem<RT>(units_s + (size_t)o * R, u, R);
+            v = vals_s[o];
+            if (c.grouped)
+                g = grp_s[o];
+            q = qbuf[o];
+        } else {
+            const int64_t og = gfirst + o;
+            load_units_global<RT>(c.t.units + og * R, u, R);
+            v = __ldg(c.t.values + og);
+            if (c.grouped)
+                g = __ldg(c.t.group + og);
+            q = screen_score<RT>(u, v, g, c.sp, R, c.rg, c.grouped);
+        }
+        if (c.sp.exact || q <= thr) {
+            const double s = exact_score<RT>(u, v, g, c.sp, R, c.rg, c.grouped);
+            const int li = o - jstart;
+            if (s < best_s || (s == best_s && li < best_i)) {
+                best_s = s;
+                best_i = li;
+            }
+        }
+    }
+    allreduce_exact(best_s, best_i);
+    s_out = best_s;
+    local_out = best_i;
+}
+
+// Evaluates one staged tile.
+template <int RT>
+__device__ void process_tile(WarpCtx<RT> &c, const TileDesc &d, const unsigned char *stage, const StageLayout &SL,
+                             float *qbuf, int64_t &big_first, Best &big_carry, int lane)
+{
+    const int R = c.R;
+    const int n = d.n_opt;
+    const bool big = (d.flags & TILE_BIG) != 0;
+
+    // data offsets inside the stage (the bulk copies start at the 16-byte boundary below the data)
+    const int du = (int)((d.opt_begin * R * 4) & 15);
+    const int dv = (int)((d.opt_begin * 8) & 15);
+    const int dg = (int)((d.opt_begin * 2) & 15);
+    const int doff = (int)((d.job_begin * 8) & 15);
+    const int32_t *units_s = reinterpret_cast<const int32_t *>(stage + SL.units + du);
+    const double *vals_s = reinterpret_cast<const double *>(stage + SL.vals + dv);
+    const uint16_t *grp_s = reinterpret_cast<const uint16_t *>(stage + SL.grp + dg);
+    const long long *off_s = reinterpret_cast<const long long *>(stage + SL.off + doff);
+
+    int chunk_base = 0;
+    Best carry = best_none();
+    if (big) {
+        if (d.flags & TILE_BIG_FIRST) {
+            big_first = d.opt_begin;
+            big_carry = best_none();
+        }
+        chunk_base = (int)(d.opt_begin - big_first);
+        carry = big_carry;
+    }
+    Best priv = best_none();
+    bool priv_dirty = false;
+    int open_start = 0;      // tile-local start of the job open at the start of the row
+    int wp = 0;              // first job of the tile not yet closed
+    const int n_job = d.n_job;
+
+    for (int b = 0; b < n; b += 32) {
+        const int i = b + lane;
+        const bool valid = i < n;
+        int32_t u[Cols<RT>::N];
+        float q = INFINITY;
+        if (valid) {
+            load_units_smem<RT>(units_s + (size_t)i * R, u, R);
+            const double v = vals_s[i];
+            const int g = c.grouped ? (int)grp_s[i] : 0;
+            q = screen_score<RT>(u, v, g, c.sp, R, c.rg, c.grouped);
+            if (!big)
+                qbuf[i] = q;
+        }
+
+        // heads (first option of a job) and ends (last option of a job) in this row
+        uint32_t H, E;
+        int sa = 0x7fffffff;
+        if (!big) {
+            const int k0 = wp + lane;
+            sa = (k0 < n_job) ? (int)(off_s[k0] - d.opt_begin) : 0x7fffffff;
+            const int sb = (k0 + 1 < n_job) ? (int)(off_s[k0 + 1] - d.opt_begin) : (k0 + 1 == n_job ? n : 0x7fffffff);
+            const int hb = sa - b, eb = sb - 1 - b;
+            H = __reduce_or_sync(FULL, (hb >= 0 && hb < 32) ? (1u << hb) : 0u);
+            E = __reduce_or_sync(FULL, (eb >= 0 && eb < 32) ? (1u << eb) : 0u);
+        } else {
+            H = ((d.flags & TILE_BIG_FIRST) && b == 0) ? 1u : 0u;
+            const int eb = n - 1 - b;
+            E = ((d.flags & TILE_BIG_LAST) && eb >= 0 && eb < 32) ? (1u << eb) : 0u;
+        }
+
+        Best x = valid ? Best{q, i + chunk_base, INFINITY} : best_none();
+        if (H == 0u && E == 0u) {    // the whole row lies inside the open job: fold per lane
+            priv = combine(priv, x);
+            priv_dirty = true;
+            continue;
+        }
+        if (priv_dirty) {
+            carry = combine(carry, allreduce_best(priv));
+            priv = best_none();
+            priv_dirty = false;
+        }
+        // segmented inclusive scan; lanes before the first head continue the open job (carry)
+        const uint32_t le = (lane == 31) ? FULL : ((2u << lane) - 1u);
+        const int seg_lo = 31 - __clz(H & le);
+        if (H != FULL) {
+#pragma unroll
+            for (int dd = 1; dd < 32; dd <<= 1) {
+                const Best o = shfl_up_best(x, dd);
+                if (lane >= dd && lane - dd >= seg_lo)
+                    x = combine(o, x);
+            }
+        }
+        if (seg_lo < 0)
+            x = combine(carry, x);
+
+        const bool closing = (E >> lane) & 1u;
+        const uint32_t lt = (1u << lane) - 1u;
+        // tile-local start of each lane's job
+        int jstart;
+        if (big)
+            jstart = 0;
+        else
+            jstart = (seg_lo >= 0) ? (b + seg_lo) : open_start;
+        const int64_t job = big ? d.job_begin : (d.job_begin + wp + __popc(E & lt));
+
+        // next row's open job
+        const Best last = shfl_best(x, 31);
+        const int last_start = __shfl_sync(FULL, jstart, 31);
+        if ((E >> 31) & 1u) {
+            carry = best_none();
+        } else {
+            carry = last;
+            open_start = last_start;
+        }
+
+        // unambiguous closings finish here; ambiguous ones are resolved exactly by the warp
+        const float thr = __fadd_ru(x.m1, c.sp.e2);
+        const bool amb = closing && (c.sp.exact || !(x.m2 > thr));
+        if (closing && !amb) {
+            const int li = big ? x.idx : (x.idx - jstart);
+            int32_t uw[Cols<RT>::N];
+            double vw;
+            int gw = 0;
+            if (big) {
+                const int64_t og = big_first + x.idx;
+                load_units_global<RT>(c.t.units + og * R, uw, R);
+                vw = __ldg(c.t.values + og);
+                if (c.grouped)
+                    gw = __ldg(c.t.group + og);
+            } else {
+                load_units_smem<RT>(units_s + (size_t)x.idx * R, uw, R);
+                vw = vals_s[x.idx];
+                if (c.grouped)
+                    gw = grp_s[x.idx];
+            }
+            take_winner<RT>(c, job, li, uw, vw, gw, false, 0.0);
+        }
+        uint32_t amask = __ballot_sync(FULL, amb);
+        if (amask)
+            __syncwarp();   // this row's qbuf writes are visible to every lane before resolution
+        while (amask) {
+            const int cl = __ffs(amask) - 1;
+            amask &= amask - 1;
+            const int js = __shfl_sync(FULL, jstart, cl);
+            const float th = __shfl_sync(FULL, thr, cl);
+            const long long jb = __shfl_sync(FULL, (long long)job, cl);
+            double s_w;
+            int li_w;
+            if (big) {
+                resolve_job<RT>(c, lane, false, units_s, vals_s, grp_s, qbuf, 0, chunk_base + b + cl + 1, big_first,
+                                th, s_w, li_w);
+            } else {
+                resolve_job<RT>(c, lane, true, units_s, vals_s, grp_s, qbuf, js, b + cl + 1, 0, th, s_w, li_w);
+            }
+            if (lane == 0) {
+                int32_t uw[Cols<RT>::N];
+                double vw;
+                int gw = 0;
+                if (big) {
+                    const int64_t og = big_first + li_w;
+                    load_units_global<RT>(c.t.units + og * R, uw, R);
+                    vw = __ldg(c.t.values + og);
+                    if (c.grouped)
+                        gw = __ldg(c.t.group + og);
+                } else {
+                    const int o = js + li_w;
+                    load_units_smem<RT>(units_s + (size_t)o * R, uw, R);
+                    vw = vals_s[o];
+                    if (c.grouped)
+                        gw = grp_s[o];
+                }
+                take_winner<RT>(c, jb, li_w, uw, vw, gw, true, s_w);
+            }
+        }
+        if (!big)
+            wp += __popc(E);
+    }
+    if (big) {
+        if (priv_dirty)
+            carry = combine(carry, allreduce_best(priv));
+        big_carry = carry;
+    }
+}
+
+// Issues the bulk copies of tile d into a stage; lane 0 only.
+__device__ __forceinline__ void issue_tile(const DevTable &t, const TileDesc &d, unsigned char *stage,
+                                           const StageLayout &SL, uint32_t bar)
+{
+    const int R = t.R;
+    const int64_t ub = d.opt_begin * R * 4, ue = (d.opt_begin + d.n_opt) * R * 4;
+    const int64_t ulo = ub & ~int64_t(15), uhi = (ue + 15) & ~int64_t(15);
+    const int64_t vb = d.opt_begin * 8, ve = (d.opt_begin + d.n_opt) * 8;
+    const int64_t vlo = vb & ~int64_t(15), vhi = (ve + 15) & ~int64_t(15);
+    uint32_t total = (uint32_t)(uhi - ulo) + (uint32_t)(vhi - vlo);
+    int64_t olo = 0, ohi = 0, glo = 0, ghi = 0;
+    const bool offs = !(d.flags & TILE_BIG);
+    if (offs) {
+        const int64_t ob = d.job_begin * 8, oe = (d.job_begin + d.n_job + 1) * 8;
+        olo = ob & ~int64_t(15);
+        ohi = (oe + 15) & ~int64_t(15);
+        total += (uint32_t)(ohi - olo);
+    }
+    if (t.group) {
+        const int64_t gb = d.opt_begin * 2, ge = (d.opt_begin + d.n_opt) * 2;
+        glo = gb & ~int64_t(15);
+        ghi = (ge + 15) & ~int64_t(15);
+        total += (uint32_t)(ghi - glo);
+    }
+    fence_proxy_async();
+    mbar_arrive_expect_tx(bar, total);
+    const unsigned char *ubase = reinterpret_cast<const unsigned char *>(t.units);
+    const unsigned char *vbase = reinterpret_cast<const unsigned char *>(t.values);
+    bulk_g2s(smem_u32(stage + SL.units), ubase + ulo, (uint32_t)(uhi - ulo), bar);
+    bulk_g2s(smem_u32(stage + SL.vals), vbase + vlo, (uint32_t)(vhi - vlo), bar);
+    if (offs)
+        bulk_g2s(smem_u32(stage + SL.off), reinterpret_cast<const unsigned char *>(t.job_off) + olo,
+                 (uint32_t)(ohi - olo), bar);
+    if (t.group)
+        bulk_g2s(smem_u32(stage + SL.grp), reinterpret_cast<const unsigned char *>(t.group) + glo,
+                 (uint32_t)(ghi - glo), bar);
+}
+
+// One evaluation pass over every tile: a best response of every job of every (non-stopped) scenario.
+template <int RT>
+__global__ void __launch_bounds__(kWarpsPerCta * 32) k_pass(DevTable t, DevState st, DevPlan pl, SolveArgs a,
+                                                              int round, int kind)
+{
+    extern __shared__ __align__(128) unsigned char smem[];
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+    const int w = blockIdx.x * kWarpsPerCta + wid;
+    if (w >= pl.n_warps)
+        return;
+    const int k_begin = pl.warp_begin[w], k_end = pl.warp_begin[w + 1];
+    if (k_begin >= k_end)
+        return;
+
+    const bool grouped = t.group != nullptr;
+    const WarpSmem WS = warp_smem(pl.tile_opt, t.R, grouped, t.P);
+    const StageLayout SL = stage_layout(pl.tile_opt, t.R, grouped);
+    unsigned char *wsm = smem + (size_t)wid * WS.bytes;
+    float *qbuf = reinterpret_cast<float *>(wsm + WS.qbuf);
+    float *p32s = reinterpret_cast<float *>(wsm + WS.p32);
+    const uint32_t bar0 = smem_u32(wsm + WS.bars);
+
+    WarpCtx<RT> c;
+    c.t = t;
+    c.st = st;
+    c.R = RT ? RT : t.R;
+    c.rg = t.r_global;
+    c.grouped = grouped;
+    c.kind = kind;
+    c.want_min = (kind == PASS_FINAL) || (st.dual_trace != nullptr);
+    c.want_hash = (kind == PASS_ROUND) && (st.hash_trace != nullptr);
+    c.s = -1;
+#pragma unroll
+    for (int r = 0; r < Cols<RT>::N; ++r)
+        c.acc[r] = 0;
+    c.hacc = 0;
+    (void)a;
+    (void)round;
+
+    if (lane == 0) {
+        for (int s = 0; s < kStages; ++s)
+            mbar_init(bar0 + 8 * s, 1);
+        fence_barrier_init();
+    }
+    __syncwarp();
+
+    // prologue: the first kStages-1 tiles in flight
+    int issued = k_begin;
+    while (issued < k_end && issued < k_begin + kStages - 1) {
+        if (lane == 0) {
+            const int sidx = (issued - k_begin) % kStages;
+            issue_tile(t, pl.tiles[issued], wsm + sidx * SL.bytes, SL, bar0 + 8 * sidx);
+        }
+        ++issued;
+    }
+    int64_t big_first = 0;
+    Best big_carry = best_none();
+    int failed_at = -1;
+    for (int k = k_begin; k < k_end; ++k) {
+        if (issued < k_end) {   // refill the stage the previous tile used
+            __syncwarp();
+            if (lane == 0) {
+                const int sidx = (issued - k_begin) % kStages;
+                issue_tile(t, pl.tiles[issued], wsm + sidx * SL.bytes, SL, bar0 + 8 * sidx);
+            }
+            ++issued;
+        }
+        const TileDesc d = pl.tiles[k];
+        const int sidx = (k - k_begin) % kStages;
+        const uint32_t parity = (uint32_t)(((k - k_begin) / kStages) & 1);
+        if (!wait_stage(bar0 + 8 * sidx, parity, st.err)) {
+            failed_at = k;
+            break;
+        }
+        if (d.scenario != c.s)
+            enter_scenario<RT>(c, d.scenario, p32s, lane);
+        if (!c.sp.skip)
+            process_tile<RT>(c, d, wsm + sidx * SL.bytes, SL, qbuf, big_first, big_carry, lane);
+        __syncwarp();
+    }
+    if (failed_at < 0) {
+        flush<RT>(c, lane);
+    } else {
+        // a copy never completed: wait (bounded) for every copy still in flight, then leave
+        for (int k = failed_at; k < issued; ++k) {
+            const int sidx = (k - k_begin) % kStages;
+            wait_stage(bar0 + 8 * sidx, (uint32_t)(((k - k_begin) / kStages) & 1), st.err);
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------------------------
+// Price update (Eq. price_update), one warp per scenario, and the screen bound of the new prices.
+
+__device__ __forceinline__ double warp_sum_fixed(double x)
+{
+#pragma unroll
+    for (int d = 16; d >= 1; d >>= 1)
+        x += __shfl_xor_sync(FULL, x, d);
+    return x;
+}
+
+__device__ __forceinline__ double warp_max(double x)
+{
+#pragma unroll
+    for (int d = 16; d >= 1; d >>= 1)
+        x = fmax(x, __shfl_xor_sync(FULL, x, d));
+    return x;
+}
+
+// Effective prices p = lambda (RAW) or lambda / C (NORMALIZED), their fp32 copy, and the bound E.
+__device__ void set_prices(const DevTable &t, const DevState &st, const SolveArgs &a, int s, int lane)
+{
+    const int P = t.P, R = t.R;
+    bool huge = false;
+    for (int k = lane; k < P; k += 32) {
+        const double lam = st.lam[(size_t)s * P + k];
+        const double p = (a.mode == 1) ? lam / (double)t.cap[(size_t)s * P + k] : lam;
+        st.p64[(size_t)s * P + k] = p;
+        st.p32[(size_t)s * P + k] = __double2float_rn(p);
+        huge |= !(p <= 0x1p100);
+    }
+    __syncwarp();
+    // M_s = max|v| + sum_r (max price of column r over groups) * (max unit of column r)
+    double term = 0.0;
+    if (lane < R) {
+        double pmax = 0.0;
+        if (t.group == nullptr || lane < t.r_global) {
+            pmax = st.p64[(size_t)s * P + lane];
+        } else {
+            for (int gi = 0; gi < t.n_groups; ++gi)
+                pmax = fmax(pmax, st.p64[(size_t)s * P + t.r_global + (R - t.r_global) * gi + (lane - t.r_global)]);
+        }
+        term = pmax * (double)st.umax[(size_t)s * R + lane];
+    }
+    const double M = st.vmax[s] + warp_sum_fixed(term);
+    huge = __any_sync(FULL, huge);
+    if (lane == 0) {
+        float e;
+        if (a.exact_only || huge || !(M <= 0x1p100)) {
+            e = INFINITY;
+        } else {
+            const double eb = (4.0 * R + 16.0) * 0x1p-24 * M * (1.0 + 0x1p-20) + 0x1p-100;
+            e = __double2float_ru(eb);
+        }
+        st.ebound[s] = e;
+    }
+}
+
+__global__ void k_init(DevTable t, DevState st, SolveArgs a, const double *lambda0)
+{
+    const int lane = threadIdx.x & 31;
+    const int s = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+    if (s >= t.S)
+        return;
+    const int P = t.P;
+    for (int k = lane; k < P; k += 32) {
+        const double l0 = lambda0 ? lambda0[(size_t)s * P + k] : 0.0;
+        st.lam[(size_t)s * P + k] = l0;
+        st.U[(size_t)s * P + k] = 0ull;
+        st.U_final[(size_t)s * P + k] = 0ull;
+        if (st.lam_trace)
+            st.lam_trace[((size_t)s * (a.T + 1)) * P + k] = l0;
+    }
+    if (lane == 0) {
+        st.hash[s] = 0ull;
+        st.rounds_run[s] = 0;
+        st.converged[s] = 0;
+        st.status[s] = 0;
+        st.frozen[s] = 0;
+        st.best_dual[s] = INFINITY;
+    }
+    __syncwarp();
+    set_prices(t, st, a, s, lane);
+}
+
+__global__ void k_update(DevTable t, DevState st, SolveArgs a, int round)
+{
+    const int lane = threadIdx.x & 31;
+    const int s = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+    if (s >= t.S)
+        return;
+    if (st.frozen[s])
+        return;
+    const int P = t.P, J = t.J, T = a.T;
+    const size_t sp = (size_t)s * P;
+
+    if (st.dual_trace) {   // g(lambda^t) from the minimal reduced costs of round t
+        double part = 0.0;
+        for (int j = lane; j < J; j += 32)
+            part += -st.job_min[(size_t)s * J + j];
+        double lc = 0.0;
+        for (int k = lane; k < P; k += 32)
+            lc += (a.mode == 1) ? st.lam[sp + k] : st.lam[sp + k] * (double)t.cap[sp + k];
+        const double g = warp_sum_fixed(part) + warp_sum_fixed(lc);
+        if (lane == 0) {
+            st.dual_trace[(size_t)s * (T + 1) + round] = g;
+            if (g < st.best_dual[s])
+                st.best_dual[s] = g;
+        }
+    }
+    if (st.hash_trace && lane == 0) {
+        st.hash_trace[(size_t)s * T + round] = st.hash[s];
+        st.hash[s] = 0ull;
+    }
+
+    double eta = a.eta0;
+    if (a.step == 1)
+        eta = a.eta0 / sqrt((double)(round + 1));
+    bool bad = false;
+    double dmax = 0.0, amax = 0.0;
+    for (int k = lane; k < P; k += 32) {
+        const long long U = (long long)st.U[sp + k];
+        const long long C = t.cap[sp + k];
+        if (st.dem_trace)
+            st.dem_trace[((size_t)s * T + round) * P + k] = U;
+        double excess = (double)(U - C);
+        if (a.mode == 1)
+            excess = excess / (double)C;
+        const double lam = st.lam[sp + k];
+        const double moved = __fma_rn(eta, excess, lam);
+        const double nl = moved > 0.0 ? moved : 0.0;
+        bad |= !isfinite(nl);
+        dmax = fmax(dmax, fabs(nl - lam));
+        amax = fmax(amax, fabs(lam));
+    }
+    bad = __any_sync(FULL, bad);
+    dmax = warp_max(dmax);
+    amax = warp_max(amax);
+    if (bad) {
+        for (int k = lane; k < P; k += 32)
+            st.U[sp + k] = 0ull;
+        if (lane == 0) {
+            st.status[s] = 2;
+            st.frozen[s] = 1;
+        }
+        return;
+    }
+    for (int k = lane; k < P; k += 32) {
+        const long long U = (long long)st.U[sp + k];
+        const long long C = t.cap[sp + k];
+        double excess = (double)(U - C);
+        if (a.mode == 1)
+            excess = excess / (double)C;
+        const double moved = __fma_rn(eta, excess, st.lam[sp + k]);
+        const double nl = moved > 0.0 ? moved : 0.0;
+        st.lam[sp + k] = nl;
+        st.U[sp + k] = 0ull;
+        if (st.lam_trace)
+            st.lam_trace[((size_t)s * (T + 1) + round + 1) * P + k] = nl;
+    }
+    const bool conv = (a.tol > 0.0) && (dmax <= a.tol * fmax(1.0, amax));
+    if (lane == 0) {
+        st.rounds_run[s] = round + 1;
+        if (conv) {
+            st.converged[s] = 1;
+            st.frozen[s] = 1;
+        }
+    }
+    __syncwarp();
+    set_prices(t, st, a, s, lane);
+}
+
+// Final objectives: primal = sum of chosen values, dual g(lambda) at the final prices, feasibility.
+__global__ void k_objectives(DevTable t, DevState st, SolveArgs a)
+{
+    const int lane = threadIdx.x & 31;
+    const int s = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+    if (s >= t.S)
+        return;
+    const int P = t.P, J = t.J;
+    const size_t sp = (size_t)s * P;
+    double pv = 0.0, pm = 0.0, lc = 0.0;
+    for (int j = lane; j < J; j += 32) {
+        pv += st.job_val[(size_t)s * J + j];
+        pm += -st.job_min[(size_t)s * J + j];
+    }
+    bool feas = true;
+    for (int k = lane; k < P; k += 32) {
+        lc += (a.mode == 1) ? st.lam[sp + k] : st.lam[sp + k] * (double)t.cap[sp + k];
+        feas &= (long long)st.U_final[sp + k] <= t.cap[sp + k];
+    }
+    const double primal = warp_sum_fixed(pv);
+    const double g = warp_sum_fixed(pm) + warp_sum_fixed(lc);
+    feas = __all_sync(FULL, feas);
+    if (lane == 0) {
+        st.primal[s] = primal;
+        st.dual[s] = g;
+        st.feasible[s] = feas ? 1 : 0;
+        const double bd = st.best_dual[s];
+        st.best_dual[s] = (st.dual_trace && bd < g) ? bd : g;
+        if (st.dual_trace)
+            st.dual_trace[(size_t)s * (a.T + 1) + st.rounds_run[s]] = g;
+        if (st.lam_trace) {
+            // the final prices also close the trace at row rounds_run (already written by the update)
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------------------------
+// Load-time validation and per-scenario maxima (max |v|, max unit per column).
+
+__global__ void k_validate_options(DevTable t, double *vmax, int32_t *umax, unsigned int *flags)
+{
+  for (int s = blockIdx.y; s < t.S; s += gridDim.y) {
+    const int64_t a = t.job_off[(int64_t)s * t.J];
+    const int64_t b = t.job_off[(int64_t)(s + 1) * t.J];
+    const int R = t.R;
+    double vm = 0.0;
+    int32_t um[kMaxR];
+    for (int r = 0; r < kMaxR; ++r)
+        um[r] = 0;
+    unsigned int bad = 0;
+    for (int64_t o = a + (int64_t)blockIdx.x * blockDim.x + threadIdx.x; o < b; o += (int64_t)gridDim.x * blockDim.x) {
+        const double v = t.values[o];
+        if (!isfinite(v))
+            bad |= VAL_VALUE_NONFINITE;
+        else
+            vm = fmax(vm, fabs(v));
+        for (int r = 0; r < R; ++r) {
+            const int32_t u = t.units[o * R + r];
+            if (u < 0)
+                bad |= VAL_UNITS_NEG;
+            um[r] = max(um[r], u);
+        }
+        if (t.group && (int)t.group[o] >= t.n_groups)
+            bad |= VAL_GROUP_RANGE;
+    }
+    if (bad)
+        atomicOr(flags, bad);
+    // non-negative doubles order like their bit patterns
+    atomicMax(reinterpret_cast<unsigned long long *>(vmax + s), (unsigned long long)__double_as_longlong(vm));
+    for (int r = 0; r < R; ++r)
+        atomicMax(umax + (size_t)s * R + r, um[r]);
+  }
+}
+
+__global__ void k_validate_offsets(DevTable t, unsigned int *flags)
+{
+    const int64_t n = (int64_t)t.S * t.J;
+    unsigned int bad = 0;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t k = t.job_off[i + 1] - t.job_off[i];
+        if (k < 1 || k > 0x7fffffffLL)
+            bad |= VAL_OFFSETS;
+    }
+    if (blockIdx.x == 0 && threadIdx.x == 0) {
+        if (t.job_off[0] != 0 || t.job_off[n] != t.n_opt)
+            bad |= VAL_OFFSETS;
+    }
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < (int64_t)t.S * t.P;
+         i += (int64_t)gridDim.x * blockDim.x)
+        if (t.cap[i] <= 0)
+            bad |= VAL_CAPACITY;
+    if (bad)
+        atomicOr(flags, bad);
+}
+
+template <int RT>
+void *pass_kernel_ptr()
+{
+    return reinterpret_cast<void *>(&k_pass<RT>);
+}
+
+}  // namespace
+
+int pass_smem_bytes(int R, bool grouped, int P)
+{
+    const int topt = tile_options(R, grouped);
+    return kWarpsPerCta * warp_smem(topt, R, grouped, P).bytes;
+}
+
+static const void *pass_kernel_for(int R)
+{
+    switch (R) {
+    case 4: return pass_kernel_ptr<4>();
+    case 6: return pass_kernel_ptr<6>();
+    case 8: return pass_kernel_ptr<8>();
+    default: return pass_kernel_ptr<0>();
+    }
+}
+
+int pass_ctas_per_sm(int R, bool grouped, int P)
+{
+    const void *fn = pass_kernel_for(R);
+    const int smem = pass_smem_bytes(R, grouped, P);
+    if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess)
+        return 0;
+    int n = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, fn, kWarpsPerCta * 32, smem) != cudaSuccess)
+        return 0;
+    return n;
+}
+
+cudaError_t launch_validate(const DevTable &t, double *vmax, int32_t *umax, unsigned int *flags, cudaStream_t stream)
+{
+    if (t.S > 0) {
+        const int64_t per = t.n_opt / (t.S > 0 ? t.S : 1) + 1;
+        int gx = (int)((per + 255) / 256);
+        gx = gx < 1 ? 1 : (gx > 256 ? 256 : gx);
+        dim3 grid(gx, t.S < 65535 ? t.S : 65535);
+        k_validate_options<<<grid, 256, 0, stream>>>(t, vmax, umax, flags);
+    }
+    k_validate_offsets<<<256, 256, 0, stream>>>(t, flags);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_init(const DevTable &t, const DevState &st, const SolveArgs &a, const double *lambda0,
+                        cudaStream_t stream)
+{
+    const int wpb = 4;
+    k_init<<<(t.S + wpb - 1) / wpb, 32 * wpb, 0, stream>>>(t, st, a, lambda0);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_pass(const DevTable &t, const DevState &st, const DevPlan &pl, const SolveArgs &a, int round,
+                        PassKind kind, int grid, cudaStream_t stream)
+{
+    const bool grouped = t.group != nullptr;
+    const int smem = pass_smem_bytes(t.R, grouped, t.P);
+    switch (t.R) {
+    case 4: k_pass<4><<<grid, kWarpsPerCta * 32, smem, stream>>>(t, st, pl, a, round, kind); break;
+    case 6: k_pass<6><<<grid, kWarpsPerCta * 32, smem, stream>>>(t, st, pl, a, round, kind); break;
+    case 8: k_pass<8><<<grid, kWarpsPerCta * 32, smem, stream>>>(t, st, pl, a, round, kind); break;
+    default: k_pass<0><<<grid, kWarpsPerCta * 32, smem, stream>>>(t, st, pl, a, round, kind); break;
+    }
+    return cudaGetLastError();
+}
+
+cudaError_t launch_update(const DevTable &t, const DevState &st, const SolveArgs &a, int round, cudaStream_t stream)
+{
+    const int wpb = 4;
+    k_update<<<(t.S + wpb - 1) / wpb, 32 * wpb, 0, stream>>>(t, st, a, round);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_objectives(const DevTable &t, const DevState &st, const SolveArgs &a, cudaStream_t stream)
+{
+    const int wpb = 4;
+    k_objectives<<<(t.S + wpb - 1) / wpb, 32 * wpb, 0, stream>>>(t, st, a);
+    return cudaGetLastError();
+}
+
+}  // namespace esp

@@ -1,0 +1,82 @@
+// Kernel interfaces of the ESP solver library (internal; the public ABI is include/esp.h).
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "esp_common.h"
+
+namespace esp {
+
+struct DevTable {
+    const int32_t *units;     // n_opt * R
+    const double *values;     // n_opt
+    const int64_t *job_off;   // S*J + 1
+    const uint16_t *group;    // n_opt or nullptr
+    const int64_t *cap;       // S * P
+    int64_t n_opt;
+    int32_t S, J, R, P, r_global, n_groups;
+};
+
+struct DevState {
+    double *lam;              // S*P prices lambda
+    double *p64;              // S*P per-unit prices (lambda, or lambda / C in NORMALIZED mode)
+    float *p32;               // S*P the same rounded to fp32 (the screen's prices)
+    float *ebound;            // S   screen error bound E of the current prices; +inf: exact evaluation
+    unsigned long long *U;    // S*P demand of the round being evaluated (int64 two's complement)
+    unsigned long long *U_final; // S*P demand of the final selection
+    unsigned long long *hash; // S   selection fingerprint of the round being evaluated
+    int32_t *sel;             // S*J final selection (local index)
+    double *job_val;          // S*J value of the final choice
+    double *job_min;          // S*J minimal reduced cost (final pass; every round when tracing the dual)
+    int32_t *rounds_run;      // S
+    int32_t *converged;       // S
+    int32_t *status;          // S   0 or 2 (a price became non-finite)
+    int32_t *frozen;          // S   1 once a scenario stopped (converged or non-finite)
+    double *best_dual;        // S
+    double *primal;           // S
+    double *dual;             // S
+    int32_t *feasible;        // S
+    const double *vmax;       // S   max |v| of the scenario (load time)
+    const int32_t *umax;      // S*R max unit of each stored column in the scenario (load time)
+    unsigned int *err;        // device error word (DEV_ERR_*)
+    double *lam_trace;        // S*(T+1)*P or nullptr
+    long long *dem_trace;     // S*T*P or nullptr
+    unsigned long long *hash_trace; // S*T or nullptr
+    double *dual_trace;       // S*(T+1) or nullptr
+};
+
+struct DevPlan {
+    const TileDesc *tiles;
+    const int32_t *warp_begin;  // n_warps + 1
+    int32_t n_warps;
+    int32_t tile_opt;
+};
+
+struct SolveArgs {
+    double eta0;
+    int32_t step, mode, T;
+    double tol;
+    uint32_t flags;
+    int32_t exact_only;
+};
+
+enum PassKind : int32_t { PASS_ROUND = 0, PASS_FINAL = 1 };
+
+// Dynamic shared memory per CTA of the evaluation kernel.
+int pass_smem_bytes(int R, bool grouped, int P);
+
+// Maximum resident CTAs per SM of the evaluation kernel for this table shape (0 if it cannot run).
+int pass_ctas_per_sm(int R, bool grouped, int P);
+
+cudaError_t launch_validate(const DevTable &t, double *vmax, int32_t *umax, unsigned int *flags,
+                            cudaStream_t stream);
+cudaError_t launch_init(const DevTable &t, const DevState &st, const SolveArgs &a, const double *lambda0,
+                        cudaStream_t stream);
+cudaError_t launch_pass(const DevTable &t, const DevState &st, const DevPlan &pl, const SolveArgs &a,
+                        int round, PassKind kind, int grid, cudaStream_t stream);
+cudaError_t launch_update(const DevTable &t, const DevState &st, const SolveArgs &a, int round,
+                          cudaStream_t stream);
+cudaError_t launch_objectives(const DevTable &t, const DevState &st, const SolveArgs &a, cudaStream_t stream);
+
+}  // namespace esp

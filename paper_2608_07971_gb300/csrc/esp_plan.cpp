@@ -1,0 +1,137 @@
+// Host tile planner: static work split of one evaluation pass over warps and tiles.
+#include "esp_plan.h"
+
+#include <algorithm>
+
+namespace esp {
+
+bool plan_tiles(const int64_t *off, int32_t S, int32_t J, int32_t tile_opt, int32_t max_warps, Plan &out)
+{
+    out.tiles.clear();
+    out.warp_begin.clear();
+    out.tile_opt = tile_opt;
+    const int64_t n_jobs = (int64_t)S * J;
+    if (tile_opt < 32 || (tile_opt & 31) || max_warps < 1)
+        return false;
+    if (n_jobs == 0) {
+        out.n_warps = 0;
+        out.warp_begin.push_back(0);
+        return true;
+    }
+    const int64_t total = off[n_jobs];
+    if (off[0] != 0 || total < n_jobs)
+        return false;
+    for (int64_t j = 0; j < n_jobs; ++j)   // every job needs at least one option
+        if (off[j + 1] <= off[j])
+            return false;
+    int64_t want = (total + tile_opt - 1) / tile_opt;  // at least a full tile of work per warp
+    int32_t W = (int32_t)std::min<int64_t>(max_warps, std::max<int64_t>(1, want));
+    W = (int32_t)std::min<int64_t>(W, n_jobs);
+
+    std::vector<int64_t> jb(W + 1);
+    jb[0] = 0;
+    jb[W] = n_jobs;
+    for (int32_t w = 1; w < W; ++w) {
+        const int64_t target = (int64_t)((__int128)total * w / W);
+        jb[w] = std::lower_bound(off, off + n_jobs, target) - off;
+        if (jb[w] < jb[w - 1])
+            jb[w] = jb[w - 1];
+    }
+    out.warp_begin.resize(W + 1);
+    for (int32_t w = 0; w < W; ++w) {
+        out.warp_begin[w] = (int32_t)out.tiles.size();
+        int64_t j = jb[w];
+        const int64_t jend = jb[w + 1];
+        while (j < jend) {
+            const int32_t s = (int32_t)(j / J);
+            const int64_t K = off[j + 1] - off[j];
+            if (K < 1)
+                return false;
+            if (K > tile_opt) {
+                const int64_t nch = (K + tile_opt - 1) / tile_opt;
+                for (int64_t c = 0; c < nch; ++c) {
+                    TileDesc d;
+                    d.opt_begin = off[j] + c * tile_opt;
+                    d.job_begin = j;
+                    d.n_opt = (int32_t)std::min<int64_t>(tile_opt, K - c * tile_opt);
+                    d.n_job = (c == 0) ? 1 : 0;
+                    d.scenario = s;
+                    d.flags = TILE_BIG | (c == 0 ? TILE_BIG_FIRST : 0u) | (c == nch - 1 ? TILE_BIG_LAST : 0u);
+                    out.tiles.push_back(d);
+                }
+                ++j;
+                continue;
+            }
+            const int64_t opt0 = off[j];
+            const int64_t s_end = (int64_t)(s + 1) * J;
+            int64_t jj = j;
+            while (jj < jend && jj < s_end && off[jj + 1] - opt0 <= tile_opt)
+                ++jj;
+            TileDesc d;
+            d.opt_begin = opt0;
+            d.job_begin = j;
+            d.n_opt = (int32_t)(off[jj] - opt0);
+            d.n_job = (int32_t)(jj - j);
+            d.scenario = s;
+            d.flags = 0;
+            out.tiles.push_back(d);
+            j = jj;
+        }
+    }
+    out.warp_begin[W] = (int32_t)out.tiles.size();
+    out.n_warps = W;
+    return true;
+}
+
+bool check_plan(const int64_t *off, int32_t S, int32_t J, const Plan &p)
+{
+    const int64_t n_jobs = (int64_t)S * J;
+    if ((int32_t)p.warp_begin.size() != p.n_warps + 1)
+        return false;
+    if (p.warp_begin.front() != 0 || p.warp_begin.back() != (int32_t)p.tiles.size())
+        return false;
+    for (int32_t w = 0; w < p.n_warps; ++w)
+        if (p.warp_begin[w] > p.warp_begin[w + 1])
+            return false;
+    int64_t next_job = 0;
+    int64_t big_next_opt = -1;  // expected opt_begin of the next chunk of an open big job
+    for (const TileDesc &d : p.tiles) {
+        if (d.n_opt < 1 || d.n_opt > p.tile_opt)
+            return false;
+        if (d.scenario < 0 || d.scenario >= S)
+            return false;
+        if (d.flags & TILE_BIG) {
+            const int64_t j = d.job_begin;
+            if (d.flags & TILE_BIG_FIRST) {
+                if (big_next_opt >= 0 || j != next_job || d.opt_begin != off[j] || d.n_job != 1)
+                    return false;
+            } else if (d.opt_begin != big_next_opt || d.n_job != 0 || j != next_job) {
+                return false;
+            }
+            if (j / J != d.scenario || d.opt_begin + d.n_opt > off[j + 1])
+                return false;
+            if (d.flags & TILE_BIG_LAST) {
+                if (d.opt_begin + d.n_opt != off[j + 1])
+                    return false;
+                big_next_opt = -1;
+                next_job = j + 1;
+            } else {
+                if (d.n_opt != p.tile_opt)
+                    return false;
+                big_next_opt = d.opt_begin + d.n_opt;
+            }
+        } else {
+            if (big_next_opt >= 0 || d.job_begin != next_job || d.n_job < 1)
+                return false;
+            const int64_t j1 = d.job_begin + d.n_job;
+            if (j1 > n_jobs || d.opt_begin != off[d.job_begin] || d.opt_begin + d.n_opt != off[j1])
+                return false;
+            if (d.job_begin / J != d.scenario || (j1 - 1) / J != d.scenario)
+                return false;
+            next_job = j1;
+        }
+    }
+    return big_next_opt < 0 && next_job == n_jobs;
+}
+
+}  // namespace esp

@@ -1,0 +1,28 @@
+// Host tile planner of the ESP solver (internal).
+#pragma once
+
+#include <cstdint>
+#include <vector>
+
+#include "esp_common.h"
+
+namespace esp {
+
+struct Plan {
+    std::vector<TileDesc> tiles;
+    std::vector<int32_t> warp_begin;  // n_warps + 1
+    int32_t n_warps = 0;
+    int32_t tile_opt = 0;
+};
+
+// Splits the jobs of a CSR table (offsets job_off[0 .. S*J]) into at most max_warps contiguous
+// warp ranges of about equal option counts (cut at job boundaries), and each range into tiles of
+// whole jobs of one scenario with at most tile_opt options; a job with more than tile_opt options
+// becomes consecutive chunks of one warp. Returns false on inconsistent offsets.
+bool plan_tiles(const int64_t *job_off, int32_t S, int32_t J, int32_t tile_opt, int32_t max_warps, Plan &out);
+
+// Checks a plan against the table: every job covered exactly once and in order, chunks complete,
+// every tile inside the table. Returns false on the first violation.
+bool check_plan(const int64_t *job_off, int32_t S, int32_t J, const Plan &p);
+
+}  // namespace esp

@@ -1,0 +1,290 @@
+"""Thin ctypes binding of libesp.so (include/esp.h). Argument marshalling only: every step of the
+solve runs in the library's CUDA kernels. The binding fails loudly when the library is missing.
+
+Functions keep the C names (esp_create, esp_load_options, esp_solve, ...). ``Solver`` bundles them
+for numpy / torch callers.
+"""
+
+from __future__ import annotations
+
+import ctypes
+import dataclasses
+import os
+from typing import Optional
+
+import numpy as np
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libesp.so")
+
+ESP_OK, ESP_ERR_INVALID_ARG, ESP_ERR_OVERFLOW, ESP_ERR_OOM, ESP_ERR_CUDA = 0, 1, 2, 3, 4
+ESP_ERR_NOT_LOADED, ESP_ERR_TIMEOUT, ESP_ERR_STATE, ESP_ERR_UNSUPPORTED = 5, 6, 7, 8
+ESP_PRICE_RAW, ESP_PRICE_NORMALIZED = 0, 1
+ESP_STEP_FIXED, ESP_STEP_INV_SQRT = 0, 1
+ESP_FLAG_EXACT_ONLY, ESP_FLAG_PER_ROUND_LAUNCH = 0x1, 0x2
+
+EXPORTED = [
+    "esp_create", "esp_set_stream", "esp_load_options", "esp_load_options_device", "esp_solve",
+    "esp_solve_async", "esp_get_result", "esp_get_prices", "esp_get_selection", "esp_get_demand",
+    "esp_evaluate", "esp_last_launch_count", "esp_status_string", "esp_destroy",
+    "esp_debug_tile_options", "esp_debug_plan",
+]
+
+
+class EspError(RuntimeError):
+    def __init__(self, status: int, what: str):
+        self.status = status
+        super().__init__(f"{what}: {esp_status_string(status)} ({status})")
+
+
+class esp_params(ctypes.Structure):
+    _fields_ = [("eta0", ctypes.c_double), ("step", ctypes.c_int32), ("mode", ctypes.c_int32),
+                ("max_rounds", ctypes.c_int32), ("flags", ctypes.c_uint32), ("tol", ctypes.c_double),
+                ("lambda0", ctypes.c_void_p), ("lambda_trace", ctypes.c_void_p),
+                ("demand_trace", ctypes.c_void_p), ("selhash_trace", ctypes.c_void_p),
+                ("dual_trace", ctypes.c_void_p)]
+
+
+class esp_result(ctypes.Structure):
+    _fields_ = [("rounds_run", ctypes.c_int32), ("converged", ctypes.c_int32),
+                ("feasible", ctypes.c_int32), ("status", ctypes.c_int32),
+                ("primal", ctypes.c_double), ("dual", ctypes.c_double), ("best_dual", ctypes.c_double)]
+
+
+_lib = None
+
+
+def load_library(path: Optional[str] = None):
+    """Loads libesp.so (build it with paper_2608_07971_gb300.build.build()). Raises if missing."""
+    global _lib
+    if _lib is not None and path is None:
+        return _lib
+    path = path or LIB_PATH
+    if not os.path.exists(path):
+        raise RuntimeError(f"libesp.so not found at {path}; run paper_2608_07971_gb300.build.build() "
+                           "(there is no CPU fallback)")
+    lib = ctypes.CDLL(path)
+    vp, i32, u32, i64 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_uint32, ctypes.c_int64
+    st = ctypes.c_int
+    sig = {
+        "esp_create": ([ctypes.POINTER(vp), ctypes.c_int, vp], st),
+        "esp_set_stream": ([vp, vp], st),
+        "esp_load_options": ([vp, i32, i32, i32, i32, i32, vp, vp, vp, vp, vp], st),
+        "esp_load_options_device": ([vp, i32, i32, i32, i32, i32, vp, vp, vp, vp, vp], st),
+        "esp_solve": ([vp, ctypes.POINTER(esp_params), vp], st),
+        "esp_solve_async": ([vp, ctypes.POINTER(esp_params)], st),
+        "esp_get_result": ([vp, vp], st),
+        "esp_get_prices": ([vp, vp], st),
+        "esp_get_selection": ([vp, vp], st),
+        "esp_get_demand": ([vp, vp], st),
+        "esp_evaluate": ([vp, vp, i32, u32, vp, vp, vp], st),
+        "esp_last_launch_count": ([vp, ctypes.POINTER(i64)], st),
+        "esp_status_string": ([st], ctypes.c_char_p),
+        "esp_destroy": ([vp], None),
+        "esp_debug_tile_options": ([i32, i32], i32),
+        "esp_debug_plan": ([vp, i32, i32, i32, i32, vp, i32, vp, i32, ctypes.POINTER(i32), ctypes.POINTER(i32)], st),
+    }
+    for name, (args, res) in sig.items():
+        fn = getattr(lib, name)
+        fn.argtypes = args
+        fn.restype = res
+    if path == LIB_PATH or _lib is None:
+        _lib = lib
+    return lib
+
+
+def esp_status_string(status: int) -> str:
+    return load_library().esp_status_string(status).decode()
+
+
+def _check(status: int, what: str, ok=(ESP_OK,)):
+    if status not in ok:
+        raise EspError(status, what)
+    return status
+
+
+def _p(a) -> Optional[int]:
+    """Address of a numpy array or torch tensor (None for None)."""
+    if a is None:
+        return None
+    if isinstance(a, np.ndarray):
+        return a.ctypes.data
+    return int(a.data_ptr())
+
+
+# --- the C calls, same names -------------------------------------------------------------------
+
+def esp_create(device: int = -1, stream: Optional[int] = None) -> int:
+    h = ctypes.c_void_p()
+    _check(load_library().esp_create(ctypes.byref(h), device, stream), "esp_create")
+    return h.value
+
+
+def esp_set_stream(ctx: int, stream: Optional[int]) -> None:
+    _check(load_library().esp_set_stream(ctx, stream), "esp_set_stream")
+
+
+def esp_load_options(ctx, S, J, R, P, r_global, job_offsets, units, values, group, capacity) -> None:
+    _check(load_library().esp_load_options(ctx, S, J, R, P, r_global, _p(job_offsets), _p(units), _p(values),
+                                           _p(group), _p(capacity)), "esp_load_options")
+
+
+def esp_load_options_device(ctx, S, J, R, P, r_global, job_offsets, units, values, group, capacity) -> None:
+    _check(load_library().esp_load_options_device(ctx, S, J, R, P, r_global, _p(job_offsets), _p(units),
+                                                  _p(values), _p(group), _p(capacity)),
+           "esp_load_options_device")
+
+
+def esp_solve(ctx: int, params: esp_params, results) -> int:
+    return _check(load_library().esp_solve(ctx, ctypes.byref(params), _p(results)), "esp_solve",
+                  ok=(ESP_OK, ESP_ERR_OVERFLOW))
+
+
+def esp_solve_async(ctx: int, params: esp_params) -> None:
+    _check(load_library().esp_solve_async(ctx, ctypes.byref(params)), "esp_solve_async")
+
+
+def esp_get_result(ctx: int, results) -> int:
+    return _check(load_library().esp_get_result(ctx, _p(results)), "esp_get_result", ok=(ESP_OK, ESP_ERR_OVERFLOW))
+
+
+def esp_get_prices(ctx: int, out) -> None:
+    _check(load_library().esp_get_prices(ctx, _p(out)), "esp_get_prices")
+
+
+def esp_get_selection(ctx: int, out) -> None:
+    _check(load_library().esp_get_selection(ctx, _p(out)), "esp_get_selection")
+
+
+def esp_get_demand(ctx: int, out) -> None:
+    _check(load_library().esp_get_demand(ctx, _p(out)), "esp_get_demand")
+
+
+def esp_evaluate(ctx: int, lam, mode: int, flags: int, sel, demand, min_score) -> None:
+    _check(load_library().esp_evaluate(ctx, _p(lam), mode, flags, _p(sel), _p(demand), _p(min_score)),
+           "esp_evaluate")
+
+
+def esp_last_launch_count(ctx: int) -> int:
+    n = ctypes.c_int64()
+    _check(load_library().esp_last_launch_count(ctx, ctypes.byref(n)), "esp_last_launch_count")
+    return n.value
+
+
+def esp_destroy(ctx: int) -> None:
+    load_library().esp_destroy(ctx)
+
+
+# --- convenience ---------------------------------------------------------------------------------
+
+RESULT_DTYPE = np.dtype([("rounds_run", np.int32), ("converged", np.int32), ("feasible", np.int32),
+                         ("status", np.int32), ("primal", np.float64), ("dual", np.float64),
+                         ("best_dual", np.float64)])
+assert RESULT_DTYPE.itemsize == ctypes.sizeof(esp_result)
+
+
+@dataclasses.dataclass
+class Solution:
+    lam: np.ndarray          # S x P
+    sel: np.ndarray          # S x J
+    demand: np.ndarray       # S x P
+    result: np.ndarray       # S records of RESULT_DTYPE
+    status: int
+    lambda_trace: Optional[np.ndarray] = None   # S x (T+1) x P
+    demand_trace: Optional[np.ndarray] = None   # S x T x P
+    selhash_trace: Optional[np.ndarray] = None  # S x T
+    dual_trace: Optional[np.ndarray] = None     # S x (T+1)
+
+
+class Solver:
+    """A context holding one option table (workloads.OptionTable-like) on the GPU."""
+
+    def __init__(self, table=None, device: int = -1, stream: Optional[int] = None):
+        self.ctx = esp_create(device, stream)
+        self.shape = None
+        if table is not None:
+            self.load(table)
+
+    def close(self):
+        if self.ctx:
+            esp_destroy(self.ctx)
+            self.ctx = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def load(self, t):
+        arrs = dict(job_off=np.ascontiguousarray(t.job_off, np.int64),
+                    units=np.ascontiguousarray(t.units, np.int32),
+                    values=np.ascontiguousarray(t.values, np.float64),
+                    group=None if t.group is None else np.ascontiguousarray(t.group, np.uint16),
+                    cap=np.ascontiguousarray(t.capacity, np.int64))
+        esp_load_options(self.ctx, t.S, t.J, t.R, t.P, t.r_global, arrs["job_off"], arrs["units"],
+                         arrs["values"], arrs["group"], arrs["cap"])
+        self.shape = (t.S, t.J, t.R, t.P)
+
+    def load_device(self, S, J, R, P, r_global, job_off, units, values, group, cap):
+        """Table given as device tensors (torch); copied device-to-device."""
+        esp_load_options_device(self.ctx, S, J, R, P, r_global, job_off, units, values, group, cap)
+        self.shape = (S, J, R, P)
+
+    def params(self, eta0, rounds, mode=ESP_PRICE_NORMALIZED, step=ESP_STEP_FIXED, tol=0.0, flags=0,
+               lambda0=None) -> esp_params:
+        prm = esp_params()
+        prm.eta0, prm.step, prm.mode, prm.max_rounds, prm.flags, prm.tol = eta0, step, mode, rounds, flags, tol
+        prm.lambda0 = _p(lambda0)
+        return prm
+
+    def solve(self, eta0, rounds, mode=ESP_PRICE_NORMALIZED, step=ESP_STEP_FIXED, tol=0.0, flags=0,
+              lambda0=None, traces=False) -> Solution:
+        S, J, R, P = self.shape
+        T = rounds
+        l0 = None if lambda0 is None else np.ascontiguousarray(lambda0, np.float64).reshape(S, P)
+        prm = self.params(eta0, rounds, mode, step, tol, flags, l0)
+        lt = dt = ht = gt = None
+        if traces:
+            lt = np.full((S, T + 1, P), np.nan)
+            dt = np.zeros((S, T, P), np.int64)
+            ht = np.zeros((S, T), np.uint64)
+            gt = np.full((S, T + 1), np.nan)
+            prm.lambda_trace, prm.demand_trace, prm.selhash_trace, prm.dual_trace = _p(lt), _p(dt), _p(ht), _p(gt)
+        res = np.zeros(S, RESULT_DTYPE)
+        status = esp_solve(self.ctx, prm, res)
+        lam = np.zeros((S, P))
+        sel = np.zeros((S, J), np.int32)
+        dem = np.zeros((S, P), np.int64)
+        esp_get_prices(self.ctx, lam)
+        esp_get_selection(self.ctx, sel)
+        esp_get_demand(self.ctx, dem)
+        return Solution(lam, sel, dem, res, status, lt, dt, ht, gt)
+
+    def evaluate(self, lam, mode=ESP_PRICE_NORMALIZED, flags=0):
+        S, J, R, P = self.shape
+        lam = np.ascontiguousarray(lam, np.float64).reshape(S, P)
+        sel = np.zeros((S, J), np.int32)
+        dem = np.zeros((S, P), np.int64)
+        ms = np.zeros((S, J))
+        esp_evaluate(self.ctx, lam, mode, flags, sel, dem, ms)
+        return sel, dem, ms
+
+    def launches(self) -> int:
+        return esp_last_launch_count(self.ctx)
+
+
+def plan(job_off: np.ndarray, S: int, J: int, tile_opt: int, max_warps: int):
+    """Host tile planner (no GPU): returns (tiles as an n x 8 int32 array, warp_begin)."""
+    lib = load_library()
+    job_off = np.ascontiguousarray(job_off, np.int64)
+    nt, nw = ctypes.c_int32(), ctypes.c_int32()
+    st = lib.esp_debug_plan(_p(job_off), S, J, tile_opt, max_warps, None, 0, None, 0, ctypes.byref(nt),
+                            ctypes.byref(nw))
+    if st not in (ESP_OK, ESP_ERR_OOM):
+        raise EspError(st, "esp_debug_plan")
+    tiles = np.zeros((max(nt.value, 1), 8), np.int32)
+    wb = np.zeros(nw.value + 1, np.int32)
+    _check(lib.esp_debug_plan(_p(job_off), S, J, tile_opt, max_warps, _p(tiles), nt.value, _p(wb), nw.value,
+                              ctypes.byref(nt), ctypes.byref(nw)), "esp_debug_plan")
+    return tiles[:nt.value], wb

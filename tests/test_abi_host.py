@@ -1,0 +1,122 @@
+"""Host-side checks of the C-ABI library that need no GPU: it loads, exports every function that
+include/*.h declares, reports no GPU cleanly, and its tile planner covers every job exactly once."""
+
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+from paper_2608_07971_gb300 import esp, workloads as W
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2608_07971_gb300 import build
+    build.build()
+    return esp.load_library()
+
+
+def declared_functions():
+    names = []
+    for h in ("esp.h", "esp_debug.h"):
+        src = open(os.path.join(ROOT, "include", h)).read()
+        src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+        names += re.findall(r"^\s*(?:const\s+)?\w+\s*\*?\s*(esp_\w+)\s*\(", src, flags=re.M)
+    return sorted(set(names))
+
+
+def test_exports_every_declared_function(lib):
+    names = declared_functions()
+    assert len(names) >= 15
+    for n in names:
+        assert hasattr(lib, n), n
+    assert set(names) == set(esp.EXPORTED)
+
+
+def test_status_strings(lib):
+    for s in range(9):
+        assert esp.esp_status_string(s)
+    assert esp.esp_status_string(99) == "unknown status"
+
+
+def test_create_without_gpu_is_unsupported(lib):
+    import torch
+    if torch.cuda.is_available():
+        pytest.skip("a GPU is present")
+    h = ctypes.c_void_p()
+    assert lib.esp_create(ctypes.byref(h), -1, None) == esp.ESP_ERR_UNSUPPORTED
+    assert lib.esp_create(None, -1, None) == esp.ESP_ERR_INVALID_ARG
+
+
+def test_null_context_rejected(lib):
+    assert lib.esp_solve(None, None, None) == esp.ESP_ERR_INVALID_ARG
+    assert lib.esp_get_prices(None, None) == esp.ESP_ERR_INVALID_ARG
+    lib.esp_destroy(None)
+
+
+def tiles_cover(job_off, S, J, tiles, wb, tile_opt):
+    """Independent re-check of a plan: each job once, in order, chunks contiguous and complete."""
+    opt_begin = tiles[:, 0].astype(np.int64) & 0xFFFFFFFF | (tiles[:, 1].astype(np.int64) << 32)
+    job_begin = tiles[:, 2].astype(np.int64) & 0xFFFFFFFF | (tiles[:, 3].astype(np.int64) << 32)
+    n_opt, n_job, scen, flags = tiles[:, 4], tiles[:, 5], tiles[:, 6], tiles[:, 7]
+    covered = np.zeros(S * J, np.int64)  # options covered per job
+    for k in range(len(tiles)):
+        assert 1 <= n_opt[k] <= tile_opt
+        if flags[k] & 1:  # big chunk
+            j = job_begin[k]
+            covered[j] += n_opt[k]
+            assert job_off[j] <= opt_begin[k] and opt_begin[k] + n_opt[k] <= job_off[j + 1]
+        else:
+            j0, j1 = job_begin[k], job_begin[k] + n_job[k]
+            assert opt_begin[k] == job_off[j0] and opt_begin[k] + n_opt[k] == job_off[j1]
+            covered[j0:j1] += np.diff(job_off[j0:j1 + 1])
+            assert np.all(np.arange(j0, j1) // J == scen[k])
+    assert np.array_equal(covered, np.diff(job_off))
+    assert wb[0] == 0 and wb[-1] == len(tiles) and np.all(np.diff(wb) >= 0)
+
+
+@pytest.mark.parametrize("case", ["uniform16", "zipf", "big", "mixed", "ones"])
+def test_planner_covers_every_job(lib, case):
+    rng = np.random.default_rng(5)
+    S, J = 3, 500
+    if case == "uniform16":
+        K = np.full(S * J, 16)
+    elif case == "zipf":
+        K = np.minimum(256, rng.zipf(1.3, S * J))
+    elif case == "big":
+        K = rng.choice([1, 700, 768, 1500], S * J)
+    elif case == "mixed":
+        K = rng.integers(1, 300, S * J)
+    else:
+        K = np.ones(S * J, np.int64)
+    off = np.zeros(S * J + 1, np.int64)
+    off[1:] = np.cumsum(K)
+    for tile_opt in (32, 256):
+        for warps in (1, 7, 64, 5000):
+            tiles, wb = esp.plan(off, S, J, tile_opt, warps)
+            assert len(wb) - 1 <= warps
+            tiles_cover(off, S, J, tiles, wb, tile_opt)
+
+
+def test_planner_balances_options(lib):
+    t = W.whatif_batch(scenarios=range(16), J=2048).table
+    tiles, wb = esp.plan(t.job_off, t.S, t.J, 256, 600)
+    per_warp = np.array([tiles[wb[w]:wb[w + 1], 4].sum() for w in range(len(wb) - 1)])
+    assert per_warp.sum() == t.n_opt
+    assert per_warp.max() - per_warp.min() <= 32
+
+
+def test_planner_rejects_bad_offsets(lib):
+    off = np.array([0, 3, 3, 5], np.int64)   # an empty job
+    with pytest.raises(esp.EspError):
+        esp.plan(off, 1, 3, 32, 4)
+
+
+def test_tile_options(lib):
+    assert lib.esp_debug_tile_options(6, 0) == 256
+    assert lib.esp_debug_tile_options(4, 0) % 32 == 0
+    assert lib.esp_debug_tile_options(8, 1) % 32 == 0

@@ -1,0 +1,233 @@
+"""Parity of the CUDA path (through the C ABI) with the oracle, element by element.
+
+The bar: selections, integer demands and selection fingerprints bit-exact; the price trajectory
+within 1e-12 relative per step (bit-exact is expected: both sides perform the same IEEE operations);
+primal and dual objectives within 1e-9 relative (the GPU sums in a fixed tree, the oracle in job
+order).
+"""
+
+import numpy as np
+import pytest
+
+import oracle
+from paper_2608_07971_gb300 import esp, workloads as W
+
+pytestmark = pytest.mark.gpu
+
+MODES = {esp.ESP_PRICE_RAW: oracle.RAW, esp.ESP_PRICE_NORMALIZED: oracle.NORMALIZED}
+STEPS = {esp.ESP_STEP_FIXED: oracle.STEP_FIXED, esp.ESP_STEP_INV_SQRT: oracle.STEP_INV_SQRT}
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    import torch
+    if not torch.cuda.is_available():
+        pytest.skip("needs a GPU")
+    from paper_2608_07971_gb300 import build
+    build.build()
+    esp.load_library()
+
+
+def rel_err(a, b):
+    a, b = np.asarray(a, np.float64), np.asarray(b, np.float64)
+    den = np.maximum(np.abs(b), 1e-300)
+    d = np.abs(a - b)
+    return float(np.max(np.where(d == 0, 0.0, d / den))) if a.size else 0.0
+
+
+def check_solution(t, sol, scen_ids, eta, T, mode, step, tol=0.0, lambda0=None, traces=True):
+    """Compares GPU scenarios (rows of sol) with the oracle run of the same scenarios of t."""
+    ot = oracle.OracleTable(t)
+    for row, s in enumerate(scen_ids):
+        l0 = None if lambda0 is None else lambda0[row]
+        ref = oracle.solve_scenario(ot, s, eta, T, mode=MODES[mode], step=STEPS[step], tol=tol, lambda0=l0,
+                                    traces=traces)
+        r = sol.result[row]
+        assert r["rounds_run"] == ref.rounds_run, (s, r["rounds_run"], ref.rounds_run)
+        assert r["converged"] == ref.converged
+        assert (r["status"] != 0) == (ref.status != 0)
+        assert np.array_equal(sol.sel[row], ref.sel), f"selection differs in scenario {s}"
+        assert np.array_equal(sol.demand[row], ref.demand), f"demand differs in scenario {s}"
+        assert rel_err(sol.lam[row], ref.lam) <= 1e-12
+        assert r["feasible"] == ref.feasible
+        assert abs(r["primal"] - ref.primal) <= 1e-9 * max(1.0, abs(ref.primal))
+        assert abs(r["dual"] - ref.dual) <= 1e-9 * max(1.0, abs(ref.dual))
+        if traces:
+            n = ref.rounds_run
+            assert rel_err(sol.lambda_trace[row, :n + 1], ref.lambda_trace[:n + 1]) <= 1e-12
+            assert np.array_equal(sol.demand_trace[row, :n], ref.demand_trace[:n]), f"U^t differs in {s}"
+            assert np.array_equal(sol.selhash_trace[row, :n], ref.selhash_trace[:n]), f"hash differs in {s}"
+            assert rel_err(sol.dual_trace[row, :n + 1], ref.dual_trace[:n + 1]) <= 1e-9
+            assert abs(r["best_dual"] - ref.best_dual) <= 1e-9 * max(1.0, abs(ref.best_dual))
+    return True
+
+
+# ---------------------------------------------------------------------------------------------
+# The benchmark workloads (sizes the oracle finishes in seconds)
+
+@pytest.mark.parametrize("mode", [esp.ESP_PRICE_NORMALIZED, esp.ESP_PRICE_RAW])
+@pytest.mark.parametrize("step", [esp.ESP_STEP_FIXED, esp.ESP_STEP_INV_SQRT])
+def test_tiny_cluster_full(mode, step):
+    w = W.tiny_cluster()
+    eta = w.eta0 if mode == esp.ESP_PRICE_NORMALIZED else 1e-7
+    s = esp.Solver(w.table)
+    sol = s.solve(eta, w.rounds, mode=mode, step=step, traces=True)
+    check_solution(w.table, sol, [0], eta, w.rounds, mode, step)
+
+
+def test_cluster_512_full():
+    w = W.cluster_512()
+    s = esp.Solver(w.table)
+    sol = s.solve(w.eta0, w.rounds, traces=True)
+    check_solution(w.table, sol, [0], w.eta0, w.rounds, esp.ESP_PRICE_NORMALIZED, esp.ESP_STEP_FIXED)
+
+
+def test_whatif_batch_scenarios():
+    ids = [0, 1, 2, 77, 512, 1023]
+    w = W.whatif_batch(scenarios=ids)
+    s = esp.Solver(w.table)
+    sol = s.solve(w.eta0, w.rounds, traces=True)
+    check_solution(w.table, sol, list(range(len(ids))), w.eta0, w.rounds, esp.ESP_PRICE_NORMALIZED,
+                   esp.ESP_STEP_FIXED)
+
+
+def test_placement_expanded_short():
+    w = W.placement_expanded(J=512)
+    s = esp.Solver(w.table)
+    T = 60
+    sol = s.solve(w.eta0, T, traces=True)
+    check_solution(w.table, sol, [0], w.eta0, T, esp.ESP_PRICE_NORMALIZED, esp.ESP_STEP_FIXED)
+
+
+def test_heavy_tail_short():
+    w = W.heavy_tail(scenarios=[0, 9], J=8192)
+    s = esp.Solver(w.table)
+    T = 80
+    sol = s.solve(w.eta0, T, traces=True)
+    check_solution(w.table, sol, [0, 1], w.eta0, T, esp.ESP_PRICE_NORMALIZED, esp.ESP_STEP_FIXED)
+
+
+# ---------------------------------------------------------------------------------------------
+# Identical prices: esp_evaluate against the oracle's best response (bit-exact selections/demands)
+
+@pytest.mark.parametrize("name", ["tiny_cluster", "cluster_512", "heavy_tail"])
+def test_evaluate_at_oracle_prices(name):
+    if name == "heavy_tail":
+        w = W.heavy_tail(scenarios=[3], J=4096)
+    else:
+        w = W.make(name)
+    t = w.table
+    ref = oracle.solve_scenario(t, 0, w.eta0, 40, traces=True)
+    s = esp.Solver(t)
+    for ti in (0, 5, 17, 39):
+        lam = ref.lambda_trace[ti][None, :]
+        sel, dem, ms = s.evaluate(lam)
+        rsel, rdem, rms = oracle.best_response(t, 0, lam[0], oracle.NORMALIZED)
+        assert np.array_equal(sel[0], rsel)
+        assert np.array_equal(dem[0], rdem)
+        assert np.array_equal(ms[0], rms)     # the minimal reduced cost is the same fp64 chain
+
+
+# ---------------------------------------------------------------------------------------------
+# Ragged, degenerate and extreme tables
+
+@pytest.mark.parametrize("case", ["k1", "ragged", "big_jobs", "tile_edges", "r16", "grouped_many",
+                                  "ties", "single_job"])
+def test_edge_tables(case):
+    rng = np.random.default_rng(hash(case) % 2**32)
+    if case == "k1":
+        t = W.random_table(rng, S=3, J=1000, R=6, kmin=1, kmax=1)
+    elif case == "ragged":
+        t = W.random_table(rng, S=4, J=700, R=6, kmin=1, kmax=300)
+    elif case == "big_jobs":
+        t = W.random_table(rng, S=2, J=9, R=6, kmin=600, kmax=2500)
+    elif case == "tile_edges":
+        t = W.random_table(rng, S=2, J=300, R=6, kmin=31, kmax=33)
+    elif case == "r16":
+        t = W.random_table(rng, S=2, J=200, R=16, kmin=1, kmax=70)
+    elif case == "grouped_many":
+        t = W.random_table(rng, S=2, J=300, R=5, kmin=1, kmax=400, groups=200, r_global=3)
+    elif case == "ties":
+        t = W.random_table(rng, S=2, J=400, R=4, kmin=2, kmax=20, umax=8, dyadic=True)
+        # many exact duplicates
+        for j in range(t.S * t.J):
+            a, b = t.job_off[j], t.job_off[j + 1]
+            t.units[a + 1:b] = t.units[a]
+            t.values[a + 1:b:2] = t.values[a]
+    else:
+        t = W.random_table(rng, S=1, J=1, R=3, kmin=5000, kmax=5000)
+    for mode, eta in ((esp.ESP_PRICE_NORMALIZED, 0.3), (esp.ESP_PRICE_RAW, 1e-4)):
+        s = esp.Solver(t)
+        T = 30
+        sol = s.solve(eta, T, mode=mode, traces=True)
+        check_solution(t, sol, list(range(t.S)), eta, T, mode, esp.ESP_STEP_FIXED)
+        exact = s.solve(eta, T, mode=mode, flags=esp.ESP_FLAG_EXACT_ONLY, traces=True)
+        assert np.array_equal(exact.sel, sol.sel)
+        assert np.array_equal(exact.lambda_trace, sol.lambda_trace)
+        assert np.array_equal(exact.demand_trace, sol.demand_trace)
+
+
+def test_zero_rounds_and_empty_jobs():
+    rng = np.random.default_rng(3)
+    t = W.random_table(rng, S=2, J=50, R=4, kmin=1, kmax=9)
+    s = esp.Solver(t)
+    sol = s.solve(0.1, 0, traces=True)
+    check_solution(t, sol, [0, 1], 0.1, 0, esp.ESP_PRICE_NORMALIZED, esp.ESP_STEP_FIXED)
+    e = W.OptionTable(2, 0, 3, 3, 3, np.zeros(1, np.int64), np.zeros((0, 3), np.int32), np.zeros(0),
+                      None, np.full((2, 3), 10, np.int64))
+    s2 = esp.Solver(e)
+    lam0 = np.full((2, 3), 5.0)
+    sol = s2.solve(0.5, 20, mode=esp.ESP_PRICE_RAW, lambda0=lam0, traces=True)
+    check_solution(e, sol, [0, 1], 0.5, 20, esp.ESP_PRICE_RAW, esp.ESP_STEP_FIXED, lambda0=lam0)
+
+
+def test_warm_start_and_tolerance():
+    w = W.tiny_cluster()
+    t = w.table
+    s = esp.Solver(t)
+    lam0 = np.abs(np.random.default_rng(1).normal(size=(1, t.P)))
+    sol = s.solve(w.eta0, 150, step=esp.ESP_STEP_INV_SQRT, tol=2e-3, lambda0=lam0, traces=True)
+    check_solution(t, sol, [0], w.eta0, 150, esp.ESP_PRICE_NORMALIZED, esp.ESP_STEP_INV_SQRT, tol=2e-3,
+                   lambda0=lam0)
+
+
+def test_extreme_magnitudes_take_the_exact_path():
+    rng = np.random.default_rng(9)
+    t = W.random_table(rng, S=3, J=100, R=4, kmin=1, kmax=12)
+    t.values[: t.n_opt // 3] *= 2.0**120          # beyond the fp32 screen's range
+    t.values[t.n_opt // 3: 2 * t.n_opt // 3] *= 2.0**-140   # fp32 subnormal / zero
+    s = esp.Solver(t)
+    for mode, eta in ((esp.ESP_PRICE_RAW, 1e25), (esp.ESP_PRICE_RAW, 1e-30), (esp.ESP_PRICE_NORMALIZED, 0.2)):
+        sol = s.solve(eta, 12, mode=mode, traces=True)
+        check_solution(t, sol, [0, 1, 2], eta, 12, mode, esp.ESP_STEP_FIXED)
+
+
+def test_nonfinite_prices_reported():
+    t = W.random_table(np.random.default_rng(2), S=2, J=20, R=2, kmin=1, kmax=3, umax=2**30)
+    t.capacity[:] = 1
+    s = esp.Solver(t)
+    sol = s.solve(1e300, 5, mode=esp.ESP_PRICE_RAW, traces=True)
+    assert sol.status == esp.ESP_ERR_OVERFLOW
+    check_solution(t, sol, [0, 1], 1e300, 5, esp.ESP_PRICE_RAW, esp.ESP_STEP_FIXED)
+
+
+def test_invalid_tables_rejected():
+    rng = np.random.default_rng(4)
+    t = W.random_table(rng, S=1, J=10, R=3, kmin=1, kmax=4)
+    s = esp.Solver()
+    bad = W.OptionTable(**{**t.__dict__, "units": t.units.copy()})
+    bad.units[3, 1] = -1
+    with pytest.raises(esp.EspError) as e:
+        s.load(bad)
+    assert e.value.status == esp.ESP_ERR_INVALID_ARG
+    bad = W.OptionTable(**{**t.__dict__, "values": t.values.copy()})
+    bad.values[2] = np.inf
+    with pytest.raises(esp.EspError):
+        s.load(bad)
+    bad = W.OptionTable(**{**t.__dict__, "capacity": t.capacity.copy()})
+    bad.capacity[0, 0] = 0
+    with pytest.raises(esp.EspError):
+        s.load(bad)
+    s.load(t)   # a good table still loads afterwards
+    sol = s.solve(0.1, 5)
+    assert sol.status == esp.ESP_OK
