@@ -1,0 +1,417 @@
+#!/usr/bin/env python3
+"""Throughput of the ESP tatonnement (Sec. 3.2) on GB300: option-evaluations per second.
+
+One step = one full solve of the workload through the C ABI: T price rounds (each a best response
+of every job over every option, the int64 demand sum and the price update of Eq. price_update) and
+the final best response, for every scenario of the batch. `value` is measured with the table already
+resident in HBM; `e2e` repeats the step through the public API with host inputs (pinned), i.e. the
+upload, validation and planning of the table, the solve, and the read-back of selections and prices.
+
+Default workload: whatif_batch (1024 independent 512-GPU scenarios, J=2048, K=16, R=6, T=300).
+Multi-GPU (torchrun): every rank solves its own 1024 scenarios (weak scaling, no data-path collective).
+--impl reference times the oracle (the plain single-threaded C restatement of the method) instead.
+"""
+
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+from paper_2608_07971_gb300 import workloads as W  # noqa: E402
+
+MODE_NAMES = {0: "raw", 1: "normalized"}
+STEP_NAMES = {0: "fixed", 1: "inv_sqrt"}
+L2_BYTES = 129 * 2**20
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="whatif_batch", choices=sorted(W.WORKLOADS))
+    ap.add_argument("--rounds", type=int, default=None, help="override T (changes the workload)")
+    ap.add_argument("--scenarios", type=int, default=None, help="override S (profiling of a smaller case)")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0, help="oracle time budget of the CPU baseline")
+    ap.add_argument("--graph", action="store_true",
+                    help="time the CUDA-graph launch path (no per-pass events, roofline from a second pass-timed run)")
+    return ap.parse_args()
+
+
+def rank_info():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", str(rank)))
+    return rank, world, local
+
+
+def scenario_ids(name: str, rank: int, per=None):
+    """Weak scaling: rank r solves its own block of scenarios (same per-rank work)."""
+    per = per or {"whatif_batch": 1024, "heavy_tail": 16}.get(name, 1)
+    return list(range(rank * per, (rank + 1) * per))
+
+
+def make_workload(name: str, rank: int, per=None) -> W.Workload:
+    return W.make(name, scenarios=scenario_ids(name, rank, per))
+
+
+def config_of(w: W.Workload, T: int) -> dict:
+    t = w.table
+    K = t.option_counts()
+    return {
+        "workload": w.name, "S": t.S, "J": t.J, "R": t.R, "P": t.P,
+        "K_mean": round(float(K.mean()), 3), "K_max": int(K.max()),
+        "rounds": T, "eta0": w.eta0, "price_mode": MODE_NAMES[w.mode], "step": STEP_NAMES[w.step],
+        "n_opt": t.n_opt, "table_bytes": t.table_bytes(),
+        "l2": "inputs larger than L2 (table %.2f GB vs 129 MB L2)" % (t.table_bytes() / 1e9)
+        if t.table_bytes() > L2_BYTES else "table fits in L2 (latency-bound workload)",
+        "evals_per_step": t.n_opt * (T + 1),
+    }
+
+
+def measured_peak():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            pk = json.load(f)
+        return float(pk["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+def kernel_traffic(n_opt_launch: int):
+    """DRAM bytes per evaluation pass from the committed ncu summary, scaled to this workload's
+    option count, or None when the kernel source changed since the counters were taken."""
+    path = os.path.join(ROOT, "profiles", "k_pass_traffic.json")
+    src = os.path.join(ROOT, "paper_2608_07971_gb300", "csrc", "esp_kernels.cu")
+    try:
+        with open(path) as f:
+            rec = json.load(f)
+        sha = hashlib.sha256(open(src, "rb").read()).hexdigest()
+        if rec.get("kernel_source_sha256") != sha:
+            return None
+        return float(rec["dram_bytes_per_launch"]) / float(rec["options_per_launch"]) * n_opt_launch
+    except Exception:
+        return None
+
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons during the timed region."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, uuid=None):
+        self.uuid = uuid
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        fd, self.path = tempfile.mkstemp(prefix="clocks_", suffix=".csv")
+        os.close(fd)
+        cmd = ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-lms", "200"]
+        if self.uuid:
+            cmd.insert(1, f"--id={self.uuid}")
+        try:
+            self.out = open(self.path, "w")
+            self.proc = subprocess.Popen(cmd, stdout=self.out, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            time.sleep(0.25)
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+            self.out.close()
+
+    def summary(self):
+        rows = []
+        try:
+            for line in open(self.path):
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) >= 8:
+                    rows.append(parts)
+        except Exception:
+            pass
+        finally:
+            try:
+                os.unlink(self.path)
+            except Exception:
+                pass
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+        sm = [float(r[0]) for r in rows if r[0].replace(".", "").isdigit()]
+        mx = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[4 + i].lower().startswith("active")})
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(rows)}
+
+
+def cpu_baseline(w: W.Workload, T: int, budget_s: float) -> dict:
+    """The oracle as it stands, single-threaded, on whole scenarios of the same workload until the
+    time budget is spent (at least one scenario; the first `rounds` of it if one scenario alone would
+    far exceed the budget)."""
+    import oracle
+    t = w.table
+    ot = oracle.OracleTable(t)
+    lib = oracle.load()
+    per_round = t.n_opt / t.S
+    # rough rate to bound a single scenario: 3 ns per option-evaluation
+    rounds = T
+    if per_round * (T + 1) * 3e-9 > 4 * budget_s:
+        rounds = max(1, int(budget_s / (per_round * 3e-9)) - 1)
+    evals, n, t0 = 0, 0, time.perf_counter()
+    while n < t.S:
+        oracle.solve_scenario(ot, n, w.eta0, rounds, mode=w.mode, step=w.step, lib=lib)
+        evals += int(t.job_off[(n + 1) * t.J] - t.job_off[n * t.J]) * (rounds + 1)
+        n += 1
+        if time.perf_counter() - t0 >= budget_s:
+            break
+    dt = time.perf_counter() - t0
+    what = f"{n} of {t.S} scenarios of {w.name}, " + (f"all {T} rounds + final pass" if rounds == T
+                                                       else f"first {rounds} rounds + final pass")
+    return {"value": evals / dt, "unit": "option-evals/s", "cores": 1, "kind": "oracle",
+            "sample": what + f", {dt:.1f} s on 1 of {os.cpu_count()} host cores"}
+
+
+def run_reference(args):
+    rank, world, _ = rank_info()
+    if rank != 0:
+        return 0
+    w = make_workload(args.workload, 0, args.scenarios)
+    T = args.rounds if args.rounds is not None else w.rounds
+    w.rounds = T
+    import oracle
+    t = w.table
+    ot = oracle.OracleTable(t)
+    lib = oracle.load()
+    # one step = the oracle's full solve of a fixed number of scenarios, about 1-2 s of CPU work
+    per_scen = t.n_opt / t.S * (T + 1)
+    t0 = time.perf_counter()
+    oracle.solve_scenario(ot, 0, w.eta0, T, mode=w.mode, step=w.step, lib=lib)
+    one = time.perf_counter() - t0
+    m = int(max(1, min(t.S, round(1.5 / max(one, 1e-6)))))
+    rounds = T
+    if one > 6.0:       # scenario too large for a step: a prefix of its rounds
+        rounds = max(1, int(T * 1.5 / one))
+        m = 1
+
+    def step(i):
+        for k in range(m):
+            s = (i * m + k) % t.S
+            oracle.solve_scenario(ot, s, w.eta0, rounds, mode=w.mode, step=w.step, lib=lib)
+
+    for i in range(args.warmup):
+        step(i)
+    t0 = time.perf_counter()
+    for i in range(args.steps):
+        step(args.warmup + i)
+    dt = (time.perf_counter() - t0) / args.steps
+    evals = m * (t.n_opt / t.S) * (rounds + 1)
+    value = evals / dt
+    sample = f"{m} scenario(s) of {w.name} per step, " + (f"all {T} rounds + final pass" if rounds == T
+                                                         else f"first {rounds} rounds + final pass")
+    line = {
+        "impl": "reference", "metric": "option-evaluations/sec", "value": value, "unit": "option-evals/s",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic (seeded generator)", "config": config_of(w, T),
+        "cpu_baseline": {"value": value, "unit": "option-evals/s", "cores": 1, "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": value, "unit": "option-evals/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def run_ours(args):
+    import torch
+    rank, world, local = rank_info()
+    if not torch.cuda.is_available():
+        raise SystemExit("bench.py needs a CUDA GPU (no CPU fallback)")
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+
+    from paper_2608_07971_gb300 import build, esp
+    if not os.path.exists(esp.LIB_PATH):
+        build.build()
+    esp.load_library()
+
+    w = make_workload(args.workload, rank, args.scenarios)
+    T = args.rounds if args.rounds is not None else w.rounds
+    t = w.table
+    stream = torch.cuda.Stream()
+    solver = esp.Solver(t, device=local, stream=stream.cuda_stream)
+
+    flags_timed = 0 if args.graph else esp.ESP_FLAG_PASS_EVENTS
+    prm = solver.params(w.eta0, T, mode=w.mode, step=w.step, flags=flags_timed)
+    ctx = solver.ctx
+
+    def barrier():
+        if dist is not None:
+            dist.barrier()
+
+    # warm-up (also builds the CUDA graph when --graph)
+    for _ in range(args.warmup):
+        esp.esp_solve_async(ctx, prm)
+    stream.synchronize()
+    esp.esp_pass_times(ctx, reset=True)
+    launches_per_step = esp.esp_last_launch_count(ctx)
+
+    uuid = None
+    try:
+        uuid = str(torch.cuda.get_device_properties(local).uuid)
+        if uuid and not uuid.startswith("GPU-"):
+            uuid = "GPU-" + uuid
+    except Exception:
+        uuid = None
+
+    barrier()
+    torch.cuda.synchronize()
+    ev0 = torch.cuda.Event(enable_timing=True)
+    ev1 = torch.cuda.Event(enable_timing=True)
+    with ClockSampler(uuid) as clk:
+        ev0.record(stream)
+        for _ in range(args.steps):
+            esp.esp_solve_async(ctx, prm)
+        ev1.record(stream)
+        stream.synchronize()
+    torch.cuda.synchronize()
+    barrier()
+    ms = ev0.elapsed_time(ev1) / args.steps
+    res = np.zeros(t.S, esp.RESULT_DTYPE)
+    st = esp.esp_get_result(ctx, res)
+    assert np.all(res["rounds_run"] == T) or st != 0, "unexpected early stop"
+
+    pass_ms, n_pass = esp.esp_pass_times(ctx, reset=True)
+    if args.graph:   # roofline from a second, pass-timed run of the same steps
+        prm_ev = solver.params(w.eta0, T, mode=w.mode, step=w.step, flags=esp.ESP_FLAG_PASS_EVENTS)
+        for _ in range(args.steps):
+            esp.esp_solve_async(ctx, prm_ev)
+        pass_ms, n_pass = esp.esp_pass_times(ctx, reset=True)
+
+    evals_step = t.n_opt * (T + 1)
+    ms_max = ms
+    if dist is not None:
+        x = torch.tensor([ms], device="cuda", dtype=torch.float64)
+        dist.all_reduce(x, op=dist.ReduceOp.MAX)
+        ms_max = float(x.item())
+        y = torch.tensor([float(evals_step)], device="cuda", dtype=torch.float64)
+        dist.all_reduce(y)
+        evals_total = float(y.item())
+    else:
+        evals_total = float(evals_step)
+    value = evals_total / (ms_max / 1e3)
+
+    # roofline of the dominant kernel (the evaluation pass): algorithmic bytes = the option table
+    peak, peak_kind = measured_peak()
+    pass_avg_ms = pass_ms / max(n_pass, 1)
+    bytes_pass = t.table_bytes()
+    achieved = bytes_pass / (pass_avg_ms / 1e3) / 1e9 if n_pass else None
+    traffic = kernel_traffic(t.n_opt)
+    roofline = {"bound": "hbm", "kernel": "k_pass (best response + demand aggregation)",
+                "achieved": achieved, "peak": peak, "unit": "GB/s",
+                "frac": (achieved / peak) if achieved else None, "traffic": traffic,
+                "peak_kind": f"{peak_kind} hbm_gbs (copy)",
+                "bytes_per_launch": bytes_pass, "avg_launch_ms": pass_avg_ms, "launches_timed": n_pass,
+                "share_of_step": (pass_ms / args.steps) / ms if ms else None}
+
+    # end to end through the public API with host inputs
+    e2e = None
+    if not args.no_e2e:
+        pin = lambda a: torch.from_numpy(np.ascontiguousarray(a)).pin_memory()  # noqa: E731
+        h_off, h_units, h_vals = pin(t.job_off), pin(t.units), pin(t.values)
+        h_grp = None if t.group is None else pin(t.group.view(np.int16))
+        h_cap = pin(t.capacity)
+        h_sel = torch.empty((t.S, t.J), dtype=torch.int32).pin_memory()
+        h_lam = torch.empty((t.S, t.P), dtype=torch.float64).pin_memory()
+        prm_e2e = solver.params(w.eta0, T, mode=w.mode, step=w.step, flags=0)
+        res_e = np.zeros(t.S, esp.RESULT_DTYPE)
+
+        def e2e_step():
+            esp.esp_load_options(ctx, t.S, t.J, t.R, t.P, t.r_global, h_off, h_units, h_vals, h_grp, h_cap)
+            esp.esp_solve(ctx, prm_e2e, res_e)
+            esp.esp_get_selection(ctx, h_sel)
+            esp.esp_get_prices(ctx, h_lam)
+
+        for _ in range(max(1, args.warmup)):
+            e2e_step()
+        barrier()
+        t0 = time.perf_counter()
+        for _ in range(args.steps):
+            e2e_step()
+        e2e_s = (time.perf_counter() - t0) / args.steps
+        barrier()
+        if dist is not None:
+            x = torch.tensor([e2e_s], device="cuda", dtype=torch.float64)
+            dist.all_reduce(x, op=dist.ReduceOp.MAX)
+            e2e_s = float(x.item())
+        h2d = t.job_off.nbytes + t.units.nbytes + t.values.nbytes + t.capacity.nbytes + \
+            (0 if t.group is None else t.group.nbytes)
+        d2h = h_sel.numel() * 4 + h_lam.numel() * 8 + t.S * esp.RESULT_DTYPE.itemsize
+        e2e = {"value": evals_total / e2e_s, "unit": "option-evals/s", "h2d_bytes_per_step": int(h2d),
+               "d2h_bytes_per_step": int(d2h), "ms_per_step": e2e_s * 1e3}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(w, T, args.cpu_seconds)
+
+    clocks = clk.summary()
+    line = {
+        "metric": "option-evaluations/sec", "value": value, "unit": "option-evals/s",
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_max,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic (seeded generator, shapes of the named workload)",
+        "config": {**config_of(w, T), "parallelism": f"scenarios sharded over {world} GPU(s), no collective",
+                   "launch": "CUDA graph, one launch per pass" if args.graph else
+                   "one launch per pass (events around each evaluation pass)"},
+        "rounds_per_sec": T / (ms_max / 1e3),
+        "roofline": roofline,
+        "cpu_baseline": cpu,
+        "e2e": e2e,
+        "clocks": {k: clocks.get(k) for k in ("sm_mhz", "sm_max_mhz", "reasons")},
+        "gpu_launches": int(launches_per_step * args.steps),
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    solver.close()
+    if dist is not None:
+        dist.destroy_process_group()
+    return 0
+
+
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -60,6 +60,8 @@ typedef enum { ESP_STEP_FIXED = 0, ESP_STEP_INV_SQRT = 1 } esp_step_rule;
 /* esp_params.flags */
 #define ESP_FLAG_EXACT_ONLY 0x1u       /* evaluate every option in fp64 (no fp32 screen); same results, slower */
 #define ESP_FLAG_PER_ROUND_LAUNCH 0x2u /* one kernel launch per round (CUDA graph) instead of the persistent loop */
+#define ESP_FLAG_PASS_EVENTS 0x4u      /* record a CUDA event pair around every evaluation-pass launch
+                                          (direct launches, no graph); read with esp_pass_times */
 
 typedef struct {
     double eta0;            /* > 0, finite */
@@ -154,6 +156,11 @@ esp_status esp_evaluate(esp_ctx *ctx, const double *lambda, int32_t mode, uint32
 
 /* Number of kernel launches the last esp_solve / esp_solve_async issued. */
 esp_status esp_last_launch_count(esp_ctx *ctx, int64_t *out);
+
+/* Device time of the evaluation passes recorded with ESP_FLAG_PASS_EVENTS since the last reset:
+ * *total_ms receives the summed CUDA-event durations (measured on the context's stream) and *count
+ * the number of passes. Waits for the stream. reset != 0 clears the record afterwards. */
+esp_status esp_pass_times(esp_ctx *ctx, double *total_ms, int64_t *count, int32_t reset);
 
 /* Static description of a string for a status. Never NULL. */
 const char *esp_status_string(esp_status status);

@@ -79,6 +79,10 @@ struct esp_ctx {
     GraphKey gkey;
     int64_t last_launches = 0;
     int32_t last_T = 0;
+
+    // ESP_FLAG_PASS_EVENTS: event pairs around evaluation passes; pool reused after a reset
+    std::vector<cudaEvent_t> ev_pool;
+    size_t ev_used = 0;
 };
 
 namespace {
@@ -382,7 +386,7 @@ esp_status check_params(const esp_ctx *ctx, const esp_params *p)
         return ESP_ERR_INVALID_ARG;
     if (!(p->tol >= 0.0) || !std::isfinite(p->tol))
         return ESP_ERR_INVALID_ARG;
-    if (p->flags & ~(uint32_t)(ESP_FLAG_EXACT_ONLY | ESP_FLAG_PER_ROUND_LAUNCH))
+    if (p->flags & ~(uint32_t)(ESP_FLAG_EXACT_ONLY | ESP_FLAG_PER_ROUND_LAUNCH | ESP_FLAG_PASS_EVENTS))
         return ESP_ERR_INVALID_ARG;
     if (p->lambda0) {
         const size_t n = (size_t)ctx->S * ctx->P;
@@ -412,16 +416,36 @@ esp_status enqueue_solve(esp_ctx *ctx, const esp_params *p, const DevState &st, 
     a.exact_only = (p->flags & ESP_FLAG_EXACT_ONLY) ? 1 : 0;
     const int T = p->max_rounds;
 
+    const bool timed = (p->flags & ESP_FLAG_PASS_EVENTS) != 0;
+    auto pass = [&](int r, PassKind kind) -> cudaError_t {
+        if (!timed)
+            return launch_pass(t, st, pl, a, r, kind, ctx->grid, ctx->stream);
+        while (ctx->ev_pool.size() < ctx->ev_used + 2) {
+            cudaEvent_t ev;
+            cudaError_t e = cudaEventCreate(&ev);
+            if (e != cudaSuccess)
+                return e;
+            ctx->ev_pool.push_back(ev);
+        }
+        cudaEvent_t e0 = ctx->ev_pool[ctx->ev_used], e1 = ctx->ev_pool[ctx->ev_used + 1];
+        ctx->ev_used += 2;
+        cudaError_t e = cudaEventRecord(e0, ctx->stream);
+        if (e == cudaSuccess)
+            e = launch_pass(t, st, pl, a, r, kind, ctx->grid, ctx->stream);
+        if (e == cudaSuccess)
+            e = cudaEventRecord(e1, ctx->stream);
+        return e;
+    };
     auto issue = [&]() -> cudaError_t {
         cudaError_t e = launch_init(t, st, a, has_l0 ? ctx->lambda0 : nullptr, ctx->stream);
         for (int r = 0; r < T && e == cudaSuccess; ++r) {
             if (ctx->grid > 0)
-                e = launch_pass(t, st, pl, a, r, PASS_ROUND, ctx->grid, ctx->stream);
+                e = pass(r, PASS_ROUND);
             if (e == cudaSuccess)
                 e = launch_update(t, st, a, r, ctx->stream);
         }
         if (e == cudaSuccess && ctx->grid > 0)
-            e = launch_pass(t, st, pl, a, T, PASS_FINAL, ctx->grid, ctx->stream);
+            e = pass(T, PASS_FINAL);
         if (e == cudaSuccess)
             e = launch_objectives(t, st, a, ctx->stream);
         return e;
@@ -442,7 +466,7 @@ esp_status enqueue_solve(esp_ctx *ctx, const esp_params *p, const DevState &st, 
     key.gt = st.dual_trace;
     key.has_l0 = has_l0;
 
-    if (ctx->stream == nullptr) {   // the legacy default stream cannot be captured
+    if (ctx->stream == nullptr || timed) {   // the legacy default stream cannot be captured
         ESP_CUDA(issue());
         return ESP_OK;
     }
@@ -786,6 +810,27 @@ esp_status esp_last_launch_count(esp_ctx *ctx, int64_t *out)
     return ESP_OK;
 }
 
+esp_status esp_pass_times(esp_ctx *ctx, double *total_ms, int64_t *count, int32_t reset)
+{
+    esp_status st = check_ctx(ctx);
+    if (st != ESP_OK)
+        return st;
+    if (!total_ms || !count)
+        return ESP_ERR_INVALID_ARG;
+    ESP_CUDA(cudaStreamSynchronize(ctx->stream));
+    double sum = 0.0;
+    for (size_t i = 0; i + 1 < ctx->ev_used; i += 2) {
+        float ms = 0.0f;
+        ESP_CUDA(cudaEventElapsedTime(&ms, ctx->ev_pool[i], ctx->ev_pool[i + 1]));
+        sum += ms;
+    }
+    *total_ms = sum;
+    *count = (int64_t)(ctx->ev_used / 2);
+    if (reset)
+        ctx->ev_used = 0;
+    return ESP_OK;
+}
+
 void esp_destroy(esp_ctx *ctx)
 {
     if (!ctx)
@@ -798,6 +843,8 @@ void esp_destroy(esp_ctx *ctx)
     if (ctx->dt.p) cudaFree(ctx->dt.p);
     if (ctx->ht.p) cudaFree(ctx->ht.p);
     if (ctx->gt.p) cudaFree(ctx->gt.p);
+    for (cudaEvent_t e : ctx->ev_pool)
+        cudaEventDestroy(e);
     delete ctx;
 }
 

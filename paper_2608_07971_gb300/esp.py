@@ -21,12 +21,12 @@ ESP_OK, ESP_ERR_INVALID_ARG, ESP_ERR_OVERFLOW, ESP_ERR_OOM, ESP_ERR_CUDA = 0, 1,
 ESP_ERR_NOT_LOADED, ESP_ERR_TIMEOUT, ESP_ERR_STATE, ESP_ERR_UNSUPPORTED = 5, 6, 7, 8
 ESP_PRICE_RAW, ESP_PRICE_NORMALIZED = 0, 1
 ESP_STEP_FIXED, ESP_STEP_INV_SQRT = 0, 1
-ESP_FLAG_EXACT_ONLY, ESP_FLAG_PER_ROUND_LAUNCH = 0x1, 0x2
+ESP_FLAG_EXACT_ONLY, ESP_FLAG_PER_ROUND_LAUNCH, ESP_FLAG_PASS_EVENTS = 0x1, 0x2, 0x4
 
 EXPORTED = [
     "esp_create", "esp_set_stream", "esp_load_options", "esp_load_options_device", "esp_solve",
     "esp_solve_async", "esp_get_result", "esp_get_prices", "esp_get_selection", "esp_get_demand",
-    "esp_evaluate", "esp_last_launch_count", "esp_status_string", "esp_destroy",
+    "esp_evaluate", "esp_last_launch_count", "esp_pass_times", "esp_status_string", "esp_destroy",
     "esp_debug_tile_options", "esp_debug_plan",
 ]
 
@@ -79,6 +79,7 @@ def load_library(path: Optional[str] = None):
         "esp_get_demand": ([vp, vp], st),
         "esp_evaluate": ([vp, vp, i32, u32, vp, vp, vp], st),
         "esp_last_launch_count": ([vp, ctypes.POINTER(i64)], st),
+        "esp_pass_times": ([vp, ctypes.POINTER(ctypes.c_double), ctypes.POINTER(i64), i32], st),
         "esp_status_string": ([st], ctypes.c_char_p),
         "esp_destroy": ([vp], None),
         "esp_debug_tile_options": ([i32, i32], i32),
@@ -169,6 +170,14 @@ def esp_last_launch_count(ctx: int) -> int:
     n = ctypes.c_int64()
     _check(load_library().esp_last_launch_count(ctx, ctypes.byref(n)), "esp_last_launch_count")
     return n.value
+
+
+def esp_pass_times(ctx: int, reset: bool = True):
+    """(summed milliseconds, number) of the evaluation passes timed with ESP_FLAG_PASS_EVENTS."""
+    ms, n = ctypes.c_double(), ctypes.c_int64()
+    _check(load_library().esp_pass_times(ctx, ctypes.byref(ms), ctypes.byref(n), 1 if reset else 0),
+           "esp_pass_times")
+    return ms.value, n.value
 
 
 def esp_destroy(ctx: int) -> None:
