@@ -1,6 +1,7 @@
 // C ABI of the ESP solver (include/esp.h): context, table upload and validation, solve driver.
 #include <cmath>
 #include <cstdint>
+#include <algorithm>
 #include <cstring>
 #include <new>
 #include <vector>
@@ -47,6 +48,7 @@ struct esp_ctx {
 
     int32_t S = 0, J = 0, R = 0, P = 0, rg = 0, n_groups = 0;
     int64_t n_opt = 0;
+    int32_t small_units = 0;
     std::vector<void *> table_bufs;  // everything freed on reload
     int32_t *units = nullptr;
     double *values = nullptr;
@@ -58,7 +60,7 @@ struct esp_ctx {
 
     TileDesc *tiles = nullptr;
     int32_t *warp_begin = nullptr;
-    int32_t n_warps = 0, tile_opt = 0, grid = 0;
+    int32_t n_warps = 0, tile_opt = 0, grid = 0, uniform_k = 0;
 
     double *lam = nullptr, *p64 = nullptr, *job_val = nullptr, *job_min = nullptr;
     double *best_dual = nullptr, *primal = nullptr, *dual = nullptr, *lambda0 = nullptr;
@@ -175,6 +177,7 @@ DevTable dev_table(const esp_ctx *c)
     t.P = c->P;
     t.r_global = c->rg;
     t.n_groups = c->n_groups;
+    t.small_units = c->small_units;
     return t;
 }
 
@@ -312,16 +315,30 @@ esp_status load_common(esp_ctx *ctx, int32_t S, int32_t J, int32_t R, int32_t P,
     const DevTable t = dev_table(ctx);
     ESP_CUDA(launch_validate(t, ctx->vmax, ctx->umax, ctx->valflags, ctx->stream));
     unsigned int vflags = 0;
+    std::vector<int32_t> h_umax((size_t)S * R);
     ESP_CUDA(cudaMemcpyAsync(&vflags, ctx->valflags, sizeof(unsigned int), cudaMemcpyDeviceToHost, ctx->stream));
+    ESP_CUDA(cudaMemcpyAsync(h_umax.data(), ctx->umax, h_umax.size() * sizeof(int32_t), cudaMemcpyDeviceToHost,
+                             ctx->stream));
     ESP_CUDA(cudaStreamSynchronize(ctx->stream));
     if (vflags != 0) {
         release_table(ctx);
         return ESP_ERR_INVALID_ARG;
     }
+    ctx->small_units = 1;
+    for (int32_t x : h_umax)
+        if (x >= (1 << 23))
+            ctx->small_units = 0;
 
     // plan the evaluation pass
-    const int tile_opt = tile_options(R, grouped);
-    const int per_sm = pass_ctas_per_sm(R, grouped, P);
+    int64_t max_k = 1, min_k = n_jobs ? INT64_MAX : 1;
+    for (int64_t j = 0; j < n_jobs; ++j) {
+        const int64_t k = off_host[j + 1] - off_host[j];
+        max_k = std::max<int64_t>(max_k, k);
+        min_k = std::min<int64_t>(min_k, k);
+    }
+    ctx->uniform_k = (min_k == max_k && max_k <= 32 && (max_k & (max_k - 1)) == 0) ? (int32_t)max_k : 0;
+    const int tile_opt = tile_options_for(R, grouped, max_k);
+    const int per_sm = pass_ctas_per_sm(R, grouped, P, tile_opt);
     if (per_sm < 1) {
         release_table(ctx);
         return ESP_ERR_UNSUPPORTED;
@@ -406,6 +423,7 @@ esp_status enqueue_solve(esp_ctx *ctx, const esp_params *p, const DevState &st, 
     pl.warp_begin = ctx->warp_begin;
     pl.n_warps = ctx->n_warps;
     pl.tile_opt = ctx->tile_opt;
+    pl.uniform_k = ctx->uniform_k;
     SolveArgs a;
     a.eta0 = p->eta0;
     a.step = p->step;
@@ -777,6 +795,7 @@ esp_status esp_evaluate(esp_ctx *ctx, const double *lambda, int32_t mode, uint32
     pl.warp_begin = ctx->warp_begin;
     pl.n_warps = ctx->n_warps;
     pl.tile_opt = ctx->tile_opt;
+    pl.uniform_k = ctx->uniform_k;
     SolveArgs a;
     a.eta0 = 1.0;
     a.step = 0;

@@ -42,6 +42,18 @@ ESP_HD int tile_options(int R, bool grouped)
     return t < 32 ? 32 : t;
 }
 
+// Tile size for a table whose largest job has max_k options: large enough that every job of up to
+// the maximum tile size stays whole (its exact resolution then reads the stage), at least 128
+// options, and otherwise small so that more warps fit per SM.
+ESP_HD int tile_options_for(int R, bool grouped, long long max_k)
+{
+    const int cap = tile_options(R, grouped);
+    long long t = (max_k + 31) & ~31LL;
+    if (t < 128)
+        t = 128;
+    return t > cap ? cap : (int)t;
+}
+
 ESP_HD int round16(int x) { return (x + 15) & ~15; }
 
 // Byte layout of one stage. Every region starts 16-byte aligned and has room for the up-to-15

@@ -14,9 +14,10 @@
 // has that option as its exact argmin; otherwise every option with q <= m1 + 2E (rounded up) is
 // rescored in fp64 and the exact lexicographic minimum is taken. Proof: s_i <= s_w implies
 // q_i - E <= s_i <= s_w <= q_w + E = m1 + E. The bound (fp32 unit roundoff u = 2^-24, all
-// magnitudes M = |v| + sum_r p_r u_r, inputs rounded to fp32 once, R fused steps, fp64 error
+// magnitudes M = |v| + sum_r p_r u_r, prices rounded to fp32 once, v truncated to fp32 (error
+// below 2u|v|, or below 2^-100 when |v| < 2^-100), units exact, R fused steps, fp64 error
 // R 2^-53 M, subnormal absolute error below 2^-100 in total) is
-//   |q - s| <= (R + 3) u M (1 + small) + 2^-100 ;   E = (4R + 16) u M_s + 2^-100,
+//   |q - s| <= (R + 4) u M (1 + small) + 2^-99 ;   E = (4R + 16) u M_s + 2^-99,
 // with M_s = max|v| + sum_r max p_r * max u_r over the scenario, a factor of about 4 to spare.
 // A scenario whose prices or values leave [2^-100, 2^100] in magnitude is evaluated in fp64 only.
 //
@@ -147,20 +148,6 @@ __device__ __forceinline__ Best allreduce_best(Best x)
     return x;
 }
 
-// Exact (s, idx) lexicographic minimum across the warp.
-__device__ __forceinline__ void allreduce_exact(double &s, int &idx)
-{
-#pragma unroll
-    for (int d = 16; d >= 1; d >>= 1) {
-        const double os = __shfl_xor_sync(FULL, s, d);
-        const int oi = __shfl_xor_sync(FULL, idx, d);
-        if (os < s || (os == s && oi < idx)) {
-            s = os;
-            idx = oi;
-        }
-    }
-}
-
 // ---------------------------------------------------------------------------------------------
 // Scoring. Both chains run r = 0 .. R-1 with one correctly rounded fused multiply-add per column.
 
@@ -177,13 +164,33 @@ struct ScenarioPrices {
     float e2;              // 2E, +inf: exact evaluation
     bool exact;
     bool skip;             // scenario already stopped
+    bool small_units;      // every unit of the table is below 2^23
 };
+
+// fp32 value of v truncated toward zero (relative error < 2^-23) for 2^-100 <= |v| <= 2^100, and 0
+// (absolute error < 2^-100) below; integer ops only (a double-to-float conversion would run on the
+// fp64 pipe). Scenarios with larger values are evaluated exactly and never use the result.
+__device__ __forceinline__ float f32_of_f64(double v)
+{
+    const uint32_t hi = (uint32_t)__double2hiint(v);
+    const uint32_t lo = (uint32_t)__double2loint(v);
+    const uint32_t ex = (hi >> 20) & 0x7ffu;
+    const uint32_t bits = (hi & 0x80000000u) | ((ex - 896u) << 23) | ((hi & 0xfffffu) << 3) | (lo >> 29);
+    return (ex >= 923u) ? __uint_as_float(bits) : 0.0f;
+}
+
+// Exact fp32 value of a unit count: 2^23 + u is exact in fp32 for 0 <= u < 2^23, so one OR and one
+// subtraction replace the int-to-float conversion; larger tables use the conversion instruction.
+__device__ __forceinline__ float f32_of_units(int32_t u, bool small)
+{
+    return small ? (__uint_as_float(0x4b000000u | (uint32_t)u) - 8388608.0f) : __int2float_rn(u);
+}
 
 template <int RT>
 __device__ __forceinline__ float screen_score(const int32_t *u, double v, int g, const ScenarioPrices &sp, int R,
                                               int rg, bool grouped)
 {
-    float q = -__double2float_rn(v);
+    float q = -f32_of_f64(v);
 #pragma unroll
     for (int r = 0; r < Cols<RT>::N; ++r) {
         if (RT == 0 && r >= R)
@@ -193,7 +200,7 @@ __device__ __forceinline__ float screen_score(const int32_t *u, double v, int g,
             price = sp.p32s[rg + (R - rg) * g + (r - rg)];
         else
             price = sp.pf[r];
-        q = __fmaf_rn(price, __int2float_rn(u[r]), q);
+        q = __fmaf_rn(price, f32_of_units(u[r], sp.small_units), q);
     }
     return q;
 }
@@ -260,6 +267,8 @@ struct WarpCtx {
     int kind;                 // PassKind
     bool want_min;            // job_min needed (final pass or dual trace)
     bool want_hash;           // selection fingerprint needed
+    int uniform_k;            // > 0: every job has this many options (a power of two <= 32)
+    int log2_k;
     // scenario
     int s;
     ScenarioPrices sp;
@@ -309,6 +318,7 @@ __device__ void enter_scenario(WarpCtx<RT> &c, int s, float *p32s_smem, int lane
     c.sp.exact = !(e < INFINITY);
     c.sp.e2 = c.sp.exact ? INFINITY : 2.0f * e;
     c.sp.p64g = c.st.p64 + (size_t)s * P;
+    c.sp.small_units = c.t.small_units != 0;
     const int ncol = c.grouped ? c.rg : c.R;
 #pragma unroll
     for (int r = 0; r < Cols<RT>::N; ++r) {
@@ -359,48 +369,130 @@ __device__ __forceinline__ void take_winner(WarpCtx<RT> &c, int64_t job, int loc
     }
 }
 
-// Exact resolution of one job whose screen was ambiguous: every option with q <= thr (all options
-// in exact mode) is rescored in fp64; returns the lexicographic minimum of (s, job-local index).
-// In-tile jobs read the stage; chunked (big) jobs read global memory and recompute q identically.
+// Signed-integer key with the order of the doubles (no NaN occurs); -0.0 and +0.0 share key 0.
+__device__ __forceinline__ long long order_key(double x)
+{
+    long long b = __double_as_longlong(x);
+    if ((b << 1) == 0)
+        b = 0;
+    return b ^ ((b >> 63) & 0x7fffffffffffffffLL);
+}
+
+__device__ __forceinline__ double key_value(long long k)
+{
+    return __longlong_as_double(k ^ ((k >> 63) & 0x7fffffffffffffffLL));
+}
+
+template <int RT>
+__device__ __forceinline__ void load_option(const WarpCtx<RT> &c, bool in_smem, const int32_t *units_s,
+                                            const double *vals_s, const uint16_t *grp_s, int o, int64_t gfirst,
+                                            int32_t *u, double &v, int &g)
+{
+    const int R = c.R;
+    g = 0;
+    if (in_smem) {
+        load_units_smem<RT>(units_s + (size_t)o * R, u, R);
+        v = vals_s[o];
+        if (c.grouped)
+            g = grp_s[o];
+    } else {
+        const int64_t og = gfirst + o;
+        load_units_global<RT>(c.t.units + og * R, u, R);
+        v = __ldg(c.t.values + og);
+        if (c.grouped)
+            g = __ldg(c.t.group + og);
+    }
+}
+
+// Exact resolution of one job whose screen was ambiguous. Survivors are the options with
+// q <= thr (every option in exact mode); the answer is their lexicographic minimum of (s, index).
+// A survivor whose units, value and group equal those of the lowest-index survivor c0 has the same
+// s and a higher index, so it cannot win: only survivors that differ from c0 are rescored in fp64,
+// and exact duplicates (common: configurations that differ only in knobs that leave the profile
+// unchanged) cost no fp64 work at all. In-tile jobs read the stage; chunked (big) jobs read global
+// memory and recompute q with the same instructions. Returns the job-local index; s_out is set when
+// has_s is true (always when need_s).
 template <int RT>
 __device__ void resolve_job(WarpCtx<RT> &c, int lane, bool in_smem, const int32_t *units_s, const double *vals_s,
                             const uint16_t *grp_s, const float *qbuf, int jstart, int jend, int64_t gfirst,
-                            float thr, double &s_out, int &local_out)
+                            float thr, bool need_s, double &s_out, bool &has_s, int &local_out)
 {
     const int R = c.R;
-    double best_s = INFINITY;
-    int best_i = kIdxNone;
     int32_t u[Cols<RT>::N];
+    double v;
+    int g;
+    // lowest-index survivor
+    int first = kIdxNone;
     for (int o = jstart + lane; o < jend; o += 32) {
-        double v;
-        int g = 0;
         float q;
         if (in_smem) {
-            load_units_smem<RT>(units_s + (size_t)o * R, u, R);
-            v = vals_s[o];
-            if (c.grouped)
-                g = grp_s[o];
             q = qbuf[o];
         } else {
-            const int64_t og = gfirst + o;
-            load_units_global<RT>(c.t.units + og * R, u, R);
-            v = __ldg(c.t.values + og);
-            if (c.grouped)
-                g = __ldg(c.t.group + og);
+            load_option<RT>(c, false, units_s, vals_s, grp_s, o, gfirst, u, v, g);
             q = screen_score<RT>(u, v, g, c.sp, R, c.rg, c.grouped);
         }
         if (c.sp.exact || q <= thr) {
-            const double s = exact_score<RT>(u, v, g, c.sp, R, c.rg, c.grouped);
-            const int li = o - jstart;
-            if (s < best_s || (s == best_s && li < best_i)) {
-                best_s = s;
-                best_i = li;
-            }
+            first = o;
+            break;
         }
     }
-    allreduce_exact(best_s, best_i);
-    s_out = best_s;
-    local_out = best_i;
+    first = __reduce_min_sync(FULL, first);
+    int32_t u0[Cols<RT>::N];
+    double v0;
+    int g0;
+    load_option<RT>(c, in_smem, units_s, vals_s, grp_s, first, gfirst, u0, v0, g0);
+
+    long long best_key = 0x7fffffffffffffffLL;
+    int best_i = kIdxNone;
+    bool distinct = false;
+    for (int o = jstart + lane; o < jend; o += 32) {
+        if (o <= first)
+            continue;
+        load_option<RT>(c, in_smem, units_s, vals_s, grp_s, o, gfirst, u, v, g);
+        const float q = in_smem ? qbuf[o] : screen_score<RT>(u, v, g, c.sp, R, c.rg, c.grouped);
+        if (!(c.sp.exact || q <= thr))
+            continue;
+        bool same = (__double_as_longlong(v) == __double_as_longlong(v0)) && (g == g0);
+#pragma unroll
+        for (int r = 0; r < Cols<RT>::N; ++r)
+            if (RT != 0 || r < R)
+                same &= (u[r] == u0[r]);
+        if (same)
+            continue;
+        distinct = true;
+        const long long k = order_key(exact_score<RT>(u, v, g, c.sp, R, c.rg, c.grouped));
+        if (k < best_key || (k == best_key && o < best_i)) {
+            best_key = k;
+            best_i = o;
+        }
+    }
+    const bool any = __any_sync(FULL, distinct);
+    if (!any) {
+        local_out = first - jstart;
+        has_s = need_s;
+        if (need_s)
+            s_out = exact_score<RT>(u0, v0, g0, c.sp, R, c.rg, c.grouped);
+        return;
+    }
+    if (lane == 0) {
+        const long long k0 = order_key(exact_score<RT>(u0, v0, g0, c.sp, R, c.rg, c.grouped));
+        if (k0 < best_key || (k0 == best_key && first < best_i)) {
+            best_key = k0;
+            best_i = first;
+        }
+    }
+#pragma unroll
+    for (int d = 16; d >= 1; d >>= 1) {
+        const long long ok = __shfl_xor_sync(FULL, best_key, d);
+        const int oi = __shfl_xor_sync(FULL, best_i, d);
+        if (ok < best_key || (ok == best_key && oi < best_i)) {
+            best_key = ok;
+            best_i = oi;
+        }
+    }
+    local_out = best_i - jstart;
+    s_out = key_value(best_key);
+    has_s = true;
 }
 
 // Evaluates one staged tile.
@@ -452,65 +544,83 @@ __device__ void process_tile(WarpCtx<RT> &c, const TileDesc &d, const unsigned c
                 qbuf[i] = q;
         }
 
-        // heads (first option of a job) and ends (last option of a job) in this row
-        uint32_t H, E;
-        int sa = 0x7fffffff;
-        if (!big) {
-            const int k0 = wp + lane;
-            sa = (k0 < n_job) ? (int)(off_s[k0] - d.opt_begin) : 0x7fffffff;
-            const int sb = (k0 + 1 < n_job) ? (int)(off_s[k0 + 1] - d.opt_begin) : (k0 + 1 == n_job ? n : 0x7fffffff);
-            const int hb = sa - b, eb = sb - 1 - b;
-            H = __reduce_or_sync(FULL, (hb >= 0 && hb < 32) ? (1u << hb) : 0u);
-            E = __reduce_or_sync(FULL, (eb >= 0 && eb < 32) ? (1u << eb) : 0u);
-        } else {
-            H = ((d.flags & TILE_BIG_FIRST) && b == 0) ? 1u : 0u;
-            const int eb = n - 1 - b;
-            E = ((d.flags & TILE_BIG_LAST) && eb >= 0 && eb < 32) ? (1u << eb) : 0u;
-        }
-
-        Best x = valid ? Best{q, i + chunk_base, INFINITY} : best_none();
-        if (H == 0u && E == 0u) {    // the whole row lies inside the open job: fold per lane
-            priv = combine(priv, x);
-            priv_dirty = true;
-            continue;
-        }
-        if (priv_dirty) {
-            carry = combine(carry, allreduce_best(priv));
-            priv = best_none();
-            priv_dirty = false;
-        }
-        // segmented inclusive scan; lanes before the first head continue the open job (carry)
-        const uint32_t le = (lane == 31) ? FULL : ((2u << lane) - 1u);
-        const int seg_lo = 31 - __clz(H & le);
-        if (H != FULL) {
-#pragma unroll
-            for (int dd = 1; dd < 32; dd <<= 1) {
-                const Best o = shfl_up_best(x, dd);
-                if (lane >= dd && lane - dd >= seg_lo)
-                    x = combine(o, x);
-            }
-        }
-        if (seg_lo < 0)
-            x = combine(carry, x);
-
-        const bool closing = (E >> lane) & 1u;
-        const uint32_t lt = (1u << lane) - 1u;
-        // tile-local start of each lane's job
+        Best x;
+        bool closing;
         int jstart;
-        if (big)
-            jstart = 0;
-        else
-            jstart = (seg_lo >= 0) ? (b + seg_lo) : open_start;
-        const int64_t job = big ? d.job_begin : (d.job_begin + wp + __popc(E & lt));
-
-        // next row's open job
-        const Best last = shfl_best(x, 31);
-        const int last_start = __shfl_sync(FULL, jstart, 31);
-        if ((E >> 31) & 1u) {
-            carry = best_none();
+        int64_t job;
+        if (c.uniform_k > 0) {
+            // every job has uniform_k options (a power of two <= 32) and tiles start at job
+            // boundaries, so each aligned group of uniform_k lanes is one job: an xor butterfly
+            const int K = c.uniform_k;
+            x = valid ? Best{q, i, INFINITY} : best_none();
+            for (int dd = 1; dd < K; dd <<= 1)
+                x = combine(x, Best{__shfl_xor_sync(FULL, x.m1, dd), __shfl_xor_sync(FULL, x.idx, dd),
+                                    __shfl_xor_sync(FULL, x.m2, dd)});
+            closing = valid && ((i & (K - 1)) == K - 1);
+            jstart = i & ~(K - 1);
+            job = d.job_begin + (i >> c.log2_k);
         } else {
-            carry = last;
-            open_start = last_start;
+            // heads (first option of a job) and ends (last option of a job) in this row
+            uint32_t H, E;
+            int sa = 0x7fffffff;
+            if (!big) {
+                const int k0 = wp + lane;
+                sa = (k0 < n_job) ? (int)(off_s[k0] - d.opt_begin) : 0x7fffffff;
+                const int sb = (k0 + 1 < n_job) ? (int)(off_s[k0 + 1] - d.opt_begin) : (k0 + 1 == n_job ? n : 0x7fffffff);
+                const int hb = sa - b, eb = sb - 1 - b;
+                H = __reduce_or_sync(FULL, (hb >= 0 && hb < 32) ? (1u << hb) : 0u);
+                E = __reduce_or_sync(FULL, (eb >= 0 && eb < 32) ? (1u << eb) : 0u);
+            } else {
+                H = ((d.flags & TILE_BIG_FIRST) && b == 0) ? 1u : 0u;
+                const int eb = n - 1 - b;
+                E = ((d.flags & TILE_BIG_LAST) && eb >= 0 && eb < 32) ? (1u << eb) : 0u;
+            }
+
+            x = valid ? Best{q, i + chunk_base, INFINITY} : best_none();
+            if (H == 0u && E == 0u) {    // the whole row lies inside the open job: fold per lane
+                priv = combine(priv, x);
+                priv_dirty = true;
+                continue;
+            }
+            if (priv_dirty) {
+                carry = combine(carry, allreduce_best(priv));
+                priv = best_none();
+                priv_dirty = false;
+            }
+            // segmented inclusive scan; lanes before the first head continue the open job (carry)
+            const uint32_t le = (lane == 31) ? FULL : ((2u << lane) - 1u);
+            const int seg_lo = 31 - __clz(H & le);
+            if (H != FULL) {
+    #pragma unroll
+                for (int dd = 1; dd < 32; dd <<= 1) {
+                    const Best o = shfl_up_best(x, dd);
+                    if (lane >= dd && lane - dd >= seg_lo)
+                        x = combine(o, x);
+                }
+            }
+            if (seg_lo < 0)
+                x = combine(carry, x);
+
+            closing = (E >> lane) & 1u;
+            const uint32_t lt = (1u << lane) - 1u;
+            // tile-local start of each lane's job
+            if (big)
+                jstart = 0;
+            else
+                jstart = (seg_lo >= 0) ? (b + seg_lo) : open_start;
+            job = big ? d.job_begin : (d.job_begin + wp + __popc(E & lt));
+
+            // next row's open job
+            const Best last = shfl_best(x, 31);
+            const int last_start = __shfl_sync(FULL, jstart, 31);
+            if ((E >> 31) & 1u) {
+                carry = best_none();
+            } else {
+                carry = last;
+                open_start = last_start;
+            }
+            if (!big)
+                wp += __popc(E);
         }
 
         // unambiguous closings finish here; ambiguous ones are resolved exactly by the warp
@@ -544,13 +654,15 @@ __device__ void process_tile(WarpCtx<RT> &c, const TileDesc &d, const unsigned c
             const int js = __shfl_sync(FULL, jstart, cl);
             const float th = __shfl_sync(FULL, thr, cl);
             const long long jb = __shfl_sync(FULL, (long long)job, cl);
-            double s_w;
+            double s_w = 0.0;
+            bool has_s = false;
             int li_w;
             if (big) {
                 resolve_job<RT>(c, lane, false, units_s, vals_s, grp_s, qbuf, 0, chunk_base + b + cl + 1, big_first,
-                                th, s_w, li_w);
+                                th, c.want_min, s_w, has_s, li_w);
             } else {
-                resolve_job<RT>(c, lane, true, units_s, vals_s, grp_s, qbuf, js, b + cl + 1, 0, th, s_w, li_w);
+                resolve_job<RT>(c, lane, true, units_s, vals_s, grp_s, qbuf, js, b + cl + 1, 0, th, c.want_min, s_w,
+                                has_s, li_w);
             }
             if (lane == 0) {
                 int32_t uw[Cols<RT>::N];
@@ -569,11 +681,9 @@ __device__ void process_tile(WarpCtx<RT> &c, const TileDesc &d, const unsigned c
                     if (c.grouped)
                         gw = grp_s[o];
                 }
-                take_winner<RT>(c, jb, li_w, uw, vw, gw, true, s_w);
+                take_winner<RT>(c, jb, li_w, uw, vw, gw, has_s, s_w);
             }
         }
-        if (!big)
-            wp += __popc(E);
     }
     if (big) {
         if (priv_dirty)
@@ -651,6 +761,8 @@ __global__ void __launch_bounds__(kWarpsPerCta * 32) k_pass(DevTable t, DevState
     c.kind = kind;
     c.want_min = (kind == PASS_FINAL) || (st.dual_trace != nullptr);
     c.want_hash = (kind == PASS_ROUND) && (st.hash_trace != nullptr);
+    c.uniform_k = pl.uniform_k;
+    c.log2_k = pl.uniform_k > 0 ? __ffs(pl.uniform_k) - 1 : 0;
     c.s = -1;
 #pragma unroll
     for (int r = 0; r < Cols<RT>::N; ++r)
@@ -762,7 +874,7 @@ __device__ void set_prices(const DevTable &t, const DevState &st, const SolveArg
         if (a.exact_only || huge || !(M <= 0x1p100)) {
             e = INFINITY;
         } else {
-            const double eb = (4.0 * R + 16.0) * 0x1p-24 * M * (1.0 + 0x1p-20) + 0x1p-100;
+            const double eb = (4.0 * R + 16.0) * 0x1p-24 * M * (1.0 + 0x1p-20) + 0x1p-99;
             e = __double2float_ru(eb);
         }
         st.ebound[s] = e;
@@ -986,10 +1098,9 @@ void *pass_kernel_ptr()
 
 }  // namespace
 
-int pass_smem_bytes(int R, bool grouped, int P)
+int pass_smem_bytes(int R, bool grouped, int P, int tile_opt)
 {
-    const int topt = tile_options(R, grouped);
-    return kWarpsPerCta * warp_smem(topt, R, grouped, P).bytes;
+    return kWarpsPerCta * warp_smem(tile_opt, R, grouped, P).bytes;
 }
 
 static const void *pass_kernel_for(int R)
@@ -1002,10 +1113,10 @@ static const void *pass_kernel_for(int R)
     }
 }
 
-int pass_ctas_per_sm(int R, bool grouped, int P)
+int pass_ctas_per_sm(int R, bool grouped, int P, int tile_opt)
 {
     const void *fn = pass_kernel_for(R);
-    const int smem = pass_smem_bytes(R, grouped, P);
+    const int smem = pass_smem_bytes(R, grouped, P, tile_opt);
     if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess)
         return 0;
     int n = 0;
@@ -1039,7 +1150,7 @@ cudaError_t launch_pass(const DevTable &t, const DevState &st, const DevPlan &pl
                         PassKind kind, int grid, cudaStream_t stream)
 {
     const bool grouped = t.group != nullptr;
-    const int smem = pass_smem_bytes(t.R, grouped, t.P);
+    const int smem = pass_smem_bytes(t.R, grouped, t.P, pl.tile_opt);
     switch (t.R) {
     case 4: k_pass<4><<<grid, kWarpsPerCta * 32, smem, stream>>>(t, st, pl, a, round, kind); break;
     case 6: k_pass<6><<<grid, kWarpsPerCta * 32, smem, stream>>>(t, st, pl, a, round, kind); break;

@@ -16,6 +16,7 @@ struct DevTable {
     const int64_t *cap;       // S * P
     int64_t n_opt;
     int32_t S, J, R, P, r_global, n_groups;
+    int32_t small_units;      // 1 if every unit is below 2^23
 };
 
 struct DevState {
@@ -51,6 +52,7 @@ struct DevPlan {
     const int32_t *warp_begin;  // n_warps + 1
     int32_t n_warps;
     int32_t tile_opt;
+    int32_t uniform_k;          // > 0: every job has exactly this many options, a power of two <= 32
 };
 
 struct SolveArgs {
@@ -64,10 +66,10 @@ struct SolveArgs {
 enum PassKind : int32_t { PASS_ROUND = 0, PASS_FINAL = 1 };
 
 // Dynamic shared memory per CTA of the evaluation kernel.
-int pass_smem_bytes(int R, bool grouped, int P);
+int pass_smem_bytes(int R, bool grouped, int P, int tile_opt);
 
 // Maximum resident CTAs per SM of the evaluation kernel for this table shape (0 if it cannot run).
-int pass_ctas_per_sm(int R, bool grouped, int P);
+int pass_ctas_per_sm(int R, bool grouped, int P, int tile_opt);
 
 cudaError_t launch_validate(const DevTable &t, double *vmax, int32_t *umax, unsigned int *flags,
                             cudaStream_t stream);

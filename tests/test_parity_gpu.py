@@ -132,7 +132,7 @@ def test_evaluate_at_oracle_prices(name):
 # Ragged, degenerate and extreme tables
 
 @pytest.mark.parametrize("case", ["k1", "ragged", "big_jobs", "tile_edges", "r16", "grouped_many",
-                                  "ties", "single_job"])
+                                  "ties", "single_job", "u2", "u32", "u16dups", "u8grouped"])
 def test_edge_tables(case):
     rng = np.random.default_rng(hash(case) % 2**32)
     if case == "k1":
@@ -154,6 +154,18 @@ def test_edge_tables(case):
             a, b = t.job_off[j], t.job_off[j + 1]
             t.units[a + 1:b] = t.units[a]
             t.values[a + 1:b:2] = t.values[a]
+    elif case == "u2":
+        t = W.random_table(rng, S=3, J=333, R=6, kmin=2, kmax=2)
+    elif case == "u32":
+        t = W.random_table(rng, S=2, J=257, R=4, kmin=32, kmax=32)
+    elif case == "u16dups":
+        t = W.random_table(rng, S=3, J=500, R=6, kmin=16, kmax=16, umax=6, dyadic=True)
+        for j in range(t.S * t.J):
+            a = t.job_off[j]
+            t.units[a + 8:a + 16] = t.units[a:a + 8]
+            t.values[a + 8:a + 16] = t.values[a:a + 8]
+    elif case == "u8grouped":
+        t = W.random_table(rng, S=2, J=300, R=8, kmin=8, kmax=8, groups=16, r_global=6)
     else:
         t = W.random_table(rng, S=1, J=1, R=3, kmin=5000, kmax=5000)
     for mode, eta in ((esp.ESP_PRICE_NORMALIZED, 0.3), (esp.ESP_PRICE_RAW, 1e-4)):
