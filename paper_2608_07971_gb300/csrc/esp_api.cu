@@ -328,6 +328,8 @@ esp_status load_common(esp_ctx *ctx, int32_t S, int32_t J, int32_t R, int32_t P,
     for (int32_t x : h_umax)
         if (x >= (1 << 23))
             ctx->small_units = 0;
+    // duplicates are marked in the device copy only (validation has already read the units)
+    ESP_CUDA(launch_mark_duplicates(dev_table(ctx), ctx->units, ctx->stream));
 
     // plan the evaluation pass
     int64_t max_k = 1, min_k = n_jobs ? INT64_MAX : 1;
@@ -336,9 +338,9 @@ esp_status load_common(esp_ctx *ctx, int32_t S, int32_t J, int32_t R, int32_t P,
         max_k = std::max<int64_t>(max_k, k);
         min_k = std::min<int64_t>(min_k, k);
     }
-    ctx->uniform_k = (min_k == max_k && max_k <= 32 && (max_k & (max_k - 1)) == 0) ? (int32_t)max_k : 0;
+    ctx->uniform_k = (!grouped && min_k == max_k && max_k <= 32 && (max_k & (max_k - 1)) == 0) ? (int32_t)max_k : 0;
     const int tile_opt = tile_options_for(R, grouped, max_k);
-    const int per_sm = pass_ctas_per_sm(R, grouped, P, tile_opt);
+    const int per_sm = pass_ctas_per_sm(R, grouped, ctx->uniform_k > 0, P, tile_opt);
     if (per_sm < 1) {
         release_table(ctx);
         return ESP_ERR_UNSUPPORTED;

@@ -14,6 +14,8 @@ namespace esp {
 constexpr int kMaxR = 16;            // stored resource columns per option
 constexpr int kWarpsPerCta = 4;      // warps of a CTA; each warp owns its own stage ring
 constexpr int kStages = 2;           // TMA stages per warp
+constexpr int kMinCtasPerSm = 5;     // register budget of the uniform-K evaluation kernel: 5 CTAs (20 warps) per SM
+constexpr int kMinCtasPerSmGeneral = 4;  // the general kernel: 4 CTAs (16 warps) per SM
 constexpr int kStageDataBytes = 8192;// option bytes (units + values [+ group]) one stage aims at
 
 // Tile flags. A tile is a run of whole jobs of one scenario whose options are contiguous, or one

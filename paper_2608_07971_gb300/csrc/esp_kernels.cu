@@ -110,45 +110,6 @@ __device__ __forceinline__ uint64_t splitmix64_mix(uint64_t z)
 }
 
 // ---------------------------------------------------------------------------------------------
-// Per-job running state of the fp32 screen: the smallest q with its index, and the smallest q of
-// every other option. Commutative and associative (ties keep the lower index).
-
-struct Best {
-    float m1;
-    int idx;
-    float m2;
-};
-
-__device__ __forceinline__ Best best_none() { return Best{INFINITY, kIdxNone, INFINITY}; }
-
-__device__ __forceinline__ Best combine(const Best &a, const Best &b)
-{
-    const bool take_b = (b.m1 < a.m1) || (b.m1 == a.m1 && b.idx < a.idx);
-    const Best &lo = take_b ? b : a;
-    const Best &hi = take_b ? a : b;
-    return Best{lo.m1, lo.idx, fminf(fminf(lo.m2, hi.m2), hi.m1)};
-}
-
-__device__ __forceinline__ Best shfl_up_best(const Best &x, int d)
-{
-    return Best{__shfl_up_sync(FULL, x.m1, d), __shfl_up_sync(FULL, x.idx, d), __shfl_up_sync(FULL, x.m2, d)};
-}
-
-__device__ __forceinline__ Best shfl_best(const Best &x, int src)
-{
-    return Best{__shfl_sync(FULL, x.m1, src), __shfl_sync(FULL, x.idx, src), __shfl_sync(FULL, x.m2, src)};
-}
-
-__device__ __forceinline__ Best allreduce_best(Best x)
-{
-#pragma unroll
-    for (int d = 16; d >= 1; d >>= 1)
-        x = combine(x, Best{__shfl_xor_sync(FULL, x.m1, d), __shfl_xor_sync(FULL, x.idx, d),
-                            __shfl_xor_sync(FULL, x.m2, d)});
-    return x;
-}
-
-// ---------------------------------------------------------------------------------------------
 // Scoring. Both chains run r = 0 .. R-1 with one correctly rounded fused multiply-add per column.
 
 template <int RT>
@@ -158,7 +119,6 @@ struct Cols {
 
 struct ScenarioPrices {
     float pf[kMaxR];       // fp32 per-unit price of each globally priced stored column
-    double pd[kMaxR];      // fp64 per-unit price of each globally priced stored column
     const float *p32s;     // fp32 prices of the scenario in shared memory (grouped tables)
     const double *p64g;    // fp64 prices of the scenario in global memory
     float e2;              // 2E, +inf: exact evaluation
@@ -186,46 +146,40 @@ __device__ __forceinline__ float f32_of_units(int32_t u, bool small)
     return small ? (__uint_as_float(0x4b000000u | (uint32_t)u) - 8388608.0f) : __int2float_rn(u);
 }
 
-template <int RT>
+template <int RT, bool G>
 __device__ __forceinline__ float screen_score(const int32_t *u, double v, int g, const ScenarioPrices &sp, int R,
-                                              int rg, bool grouped)
+                                              int rg)
 {
     float q = -f32_of_f64(v);
 #pragma unroll
     for (int r = 0; r < Cols<RT>::N; ++r) {
         if (RT == 0 && r >= R)
             break;
-        float price;
-        if (grouped && r >= rg)
-            price = sp.p32s[rg + (R - rg) * g + (r - rg)];
-        else
-            price = sp.pf[r];
+        const float price = (G && r >= rg) ? sp.p32s[rg + (R - rg) * g + (r - rg)] : sp.pf[r];
         q = __fmaf_rn(price, f32_of_units(u[r], sp.small_units), q);
     }
     return q;
 }
 
-template <int RT>
+template <int RT, bool G>
 __device__ __forceinline__ double exact_score(const int32_t *u, double v, int g, const ScenarioPrices &sp, int R,
-                                              int rg, bool grouped)
+                                              int rg)
 {
     double s = -v;
 #pragma unroll
     for (int r = 0; r < Cols<RT>::N; ++r) {
         if (RT == 0 && r >= R)
             break;
-        double price;
-        if (grouped && r >= rg)
-            price = __ldg(sp.p64g + rg + (R - rg) * g + (r - rg));
-        else
-            price = sp.pd[r];
+        const double price = __ldg(sp.p64g + ((G && r >= rg) ? rg + (R - rg) * g + (r - rg) : r));
         s = __fma_rn(price, __int2double_rn(u[r]), s);
     }
     return s;
 }
 
+// Units of one option. The sign bit of column 0 marks an exact duplicate of an earlier option of
+// the same job (set at load time; units themselves are >= 0): it is removed here and returned.
 template <int RT>
-__device__ __forceinline__ void load_units_smem(const int32_t *p, int32_t *u, int R)
+__device__ __forceinline__ bool load_units_smem(const int32_t *p, int32_t *u, int R)
 {
     if (RT == 4) {
         const int4 a = *reinterpret_cast<const int4 *>(p);
@@ -244,45 +198,47 @@ __device__ __forceinline__ void load_units_smem(const int32_t *p, int32_t *u, in
         for (int r = 0; r < Cols<RT>::N; ++r)
             u[r] = (r < R) ? p[r] : 0;
     }
+    const bool dup = u[0] < 0;
+    u[0] &= 0x7fffffff;
+    return dup;
 }
 
 template <int RT>
-__device__ __forceinline__ void load_units_global(const int32_t *p, int32_t *u, int R)
+__device__ __forceinline__ bool load_units_global(const int32_t *p, int32_t *u, int R)
 {
 #pragma unroll
     for (int r = 0; r < Cols<RT>::N; ++r)
         u[r] = (RT != 0 || r < R) ? __ldg(p + r) : 0;
+    const bool dup = u[0] < 0;
+    u[0] &= 0x7fffffff;
+    return dup;
 }
 
 // ---------------------------------------------------------------------------------------------
 // The warp's evaluation context.
 
-template <int RT>
+template <int RT, bool G>
 struct WarpCtx {
-    // table and outputs
     DevTable t;
     DevState st;
     int R, rg;
-    bool grouped;
     int kind;                 // PassKind
     bool want_min;            // job_min needed (final pass or dual trace)
     bool want_hash;           // selection fingerprint needed
     int uniform_k;            // > 0: every job has this many options (a power of two <= 32)
     int log2_k;
-    // scenario
-    int s;
+    int s;                    // current scenario
     ScenarioPrices sp;
-    // accumulators (per lane)
-    long long acc[Cols<RT>::N];
+    long long acc[Cols<RT>::N];   // per-lane demand of the globally priced columns
     unsigned long long hacc;
 };
 
-template <int RT>
-__device__ void flush(WarpCtx<RT> &c, int lane)
+template <int RT, bool G>
+__device__ void flush(WarpCtx<RT, G> &c, int lane)
 {
     if (c.s < 0)
         return;
-    const int ncol = c.grouped ? c.rg : c.R;
+    const int ncol = G ? c.rg : c.R;
     unsigned long long *dst = (c.kind == PASS_ROUND ? c.st.U : c.st.U_final) + (size_t)c.s * c.t.P;
 #pragma unroll
     for (int r = 0; r < Cols<RT>::N; ++r) {
@@ -307,8 +263,8 @@ __device__ void flush(WarpCtx<RT> &c, int lane)
     }
 }
 
-template <int RT>
-__device__ void enter_scenario(WarpCtx<RT> &c, int s, float *p32s_smem, int lane)
+template <int RT, bool G>
+__device__ void enter_scenario(WarpCtx<RT, G> &c, int s, float *p32s_smem, int lane)
 {
     flush(c, lane);
     c.s = s;
@@ -319,14 +275,13 @@ __device__ void enter_scenario(WarpCtx<RT> &c, int s, float *p32s_smem, int lane
     c.sp.e2 = c.sp.exact ? INFINITY : 2.0f * e;
     c.sp.p64g = c.st.p64 + (size_t)s * P;
     c.sp.small_units = c.t.small_units != 0;
-    const int ncol = c.grouped ? c.rg : c.R;
+    const int ncol = G ? c.rg : c.R;
 #pragma unroll
     for (int r = 0; r < Cols<RT>::N; ++r) {
         const bool have = r < ncol;
         c.sp.pf[r] = have ? __ldcg(c.st.p32 + (size_t)s * P + r) : 0.0f;
-        c.sp.pd[r] = have ? __ldcg(c.st.p64 + (size_t)s * P + r) : 0.0;
     }
-    if (c.grouped) {
+    if (G) {
         __syncwarp();
         for (int k = lane; k < P; k += 32)
             p32s_smem[k] = __ldcg(c.st.p32 + (size_t)s * P + k);
@@ -338,19 +293,18 @@ __device__ void enter_scenario(WarpCtx<RT> &c, int s, float *p32s_smem, int lane
 }
 
 // Records the winner of a job: demand, fingerprint, and the per-job outputs of the final pass.
-// u/v are the winner's units and value; s64 its exact reduced cost when already known.
-template <int RT>
-__device__ __forceinline__ void take_winner(WarpCtx<RT> &c, int64_t job, int local, const int32_t *u, double v,
+// u/v/g are the winner's data; s64 its exact reduced cost when already known.
+template <int RT, bool G>
+__device__ __forceinline__ void take_winner(WarpCtx<RT, G> &c, int64_t job, int local, const int32_t *u, double v,
                                             int g, bool have_s64, double s64)
 {
     const int R = c.R;
-    const int P = c.t.P;
 #pragma unroll
     for (int r = 0; r < Cols<RT>::N; ++r) {
         if (RT == 0 && r >= R)
             break;
-        if (c.grouped && r >= c.rg) {
-            unsigned long long *dst = (c.kind == PASS_ROUND ? c.st.U : c.st.U_final) + (size_t)c.s * P;
+        if (G && r >= c.rg) {
+            unsigned long long *dst = (c.kind == PASS_ROUND ? c.st.U : c.st.U_final) + (size_t)c.s * c.t.P;
             atomicAdd(dst + c.rg + (R - c.rg) * g + (r - c.rg), (unsigned long long)(long long)u[r]);
         } else {
             c.acc[r] += u[r];
@@ -364,7 +318,7 @@ __device__ __forceinline__ void take_winner(WarpCtx<RT> &c, int64_t job, int loc
     }
     if (c.want_min) {
         if (!have_s64)
-            s64 = exact_score<RT>(u, v, g, c.sp, R, c.rg, c.grouped);
+            s64 = exact_score<RT, G>(u, v, g, c.sp, R, c.rg);
         c.st.job_min[job] = s64;
     }
 }
@@ -383,55 +337,51 @@ __device__ __forceinline__ double key_value(long long k)
     return __longlong_as_double(k ^ ((k >> 63) & 0x7fffffffffffffffLL));
 }
 
-template <int RT>
-__device__ __forceinline__ void load_option(const WarpCtx<RT> &c, bool in_smem, const int32_t *units_s,
+// Data of tile-local option o (stage) or of job option o (global, gfirst = the job's first option).
+template <int RT, bool G>
+__device__ __forceinline__ bool load_option(const WarpCtx<RT, G> &c, bool in_smem, const int32_t *units_s,
                                             const double *vals_s, const uint16_t *grp_s, int o, int64_t gfirst,
                                             int32_t *u, double &v, int &g)
 {
     const int R = c.R;
+    bool dup;
     g = 0;
     if (in_smem) {
-        load_units_smem<RT>(units_s + (size_t)o * R, u, R);
+        dup = load_units_smem<RT>(units_s + (size_t)o * R, u, R);
         v = vals_s[o];
-        if (c.grouped)
+        if (G)
             g = grp_s[o];
     } else {
         const int64_t og = gfirst + o;
-        load_units_global<RT>(c.t.units + og * R, u, R);
+        dup = load_units_global<RT>(c.t.units + og * R, u, R);
         v = __ldg(c.t.values + og);
-        if (c.grouped)
+        if (G)
             g = __ldg(c.t.group + og);
     }
+    return dup;
 }
 
 // Exact resolution of one job whose screen was ambiguous. Survivors are the options with
-// q <= thr (every option in exact mode); the answer is their lexicographic minimum of (s, index).
-// A survivor whose units, value and group equal those of the lowest-index survivor c0 has the same
-// s and a higher index, so it cannot win: only survivors that differ from c0 are rescored in fp64,
-// and exact duplicates (common: configurations that differ only in knobs that leave the profile
-// unchanged) cost no fp64 work at all. In-tile jobs read the stage; chunked (big) jobs read global
-// memory and recompute q with the same instructions. Returns the job-local index; s_out is set when
-// has_s is true (always when need_s).
-template <int RT>
-__device__ void resolve_job(WarpCtx<RT> &c, int lane, bool in_smem, const int32_t *units_s, const double *vals_s,
-                            const uint16_t *grp_s, const float *qbuf, int jstart, int jend, int64_t gfirst,
-                            float thr, bool need_s, double &s_out, bool &has_s, int &local_out)
+// q <= thr (every option in exact mode), duplicates excluded (each has an earlier identical twin,
+// so it can never be the lexicographic minimum); the answer is the survivors' minimum of
+// (s, index). A survivor whose data equal those of the lowest-index survivor c0 (a duplicate the
+// load-time marking did not cover) is skipped for the same reason, so only survivors that differ
+// from c0 are rescored in fp64. q is recomputed with the same instructions as the screen.
+// Returns the job-local index; s_out is set when has_s is true (always when need_s).
+template <int RT, bool G>
+__device__ void resolve_job(WarpCtx<RT, G> &c, int lane, bool in_smem, const int32_t *units_s, const double *vals_s,
+                            const uint16_t *grp_s, int jstart, int jend, int64_t gfirst, float thr, bool need_s,
+                            double &s_out, bool &has_s, int &local_out)
 {
     const int R = c.R;
     int32_t u[Cols<RT>::N];
     double v;
     int g;
-    // lowest-index survivor
     int first = kIdxNone;
     for (int o = jstart + lane; o < jend; o += 32) {
-        float q;
-        if (in_smem) {
-            q = qbuf[o];
-        } else {
-            load_option<RT>(c, false, units_s, vals_s, grp_s, o, gfirst, u, v, g);
-            q = screen_score<RT>(u, v, g, c.sp, R, c.rg, c.grouped);
-        }
-        if (c.sp.exact || q <= thr) {
+        if (load_option<RT, G>(c, in_smem, units_s, vals_s, grp_s, o, gfirst, u, v, g))
+            continue;
+        if (c.sp.exact || screen_score<RT, G>(u, v, g, c.sp, R, c.rg) <= thr) {
             first = o;
             break;
         }
@@ -440,7 +390,7 @@ __device__ void resolve_job(WarpCtx<RT> &c, int lane, bool in_smem, const int32_
     int32_t u0[Cols<RT>::N];
     double v0;
     int g0;
-    load_option<RT>(c, in_smem, units_s, vals_s, grp_s, first, gfirst, u0, v0, g0);
+    load_option<RT, G>(c, in_smem, units_s, vals_s, grp_s, first, gfirst, u0, v0, g0);
 
     long long best_key = 0x7fffffffffffffffLL;
     int best_i = kIdxNone;
@@ -448,9 +398,9 @@ __device__ void resolve_job(WarpCtx<RT> &c, int lane, bool in_smem, const int32_
     for (int o = jstart + lane; o < jend; o += 32) {
         if (o <= first)
             continue;
-        load_option<RT>(c, in_smem, units_s, vals_s, grp_s, o, gfirst, u, v, g);
-        const float q = in_smem ? qbuf[o] : screen_score<RT>(u, v, g, c.sp, R, c.rg, c.grouped);
-        if (!(c.sp.exact || q <= thr))
+        if (load_option<RT, G>(c, in_smem, units_s, vals_s, grp_s, o, gfirst, u, v, g))
+            continue;
+        if (!(c.sp.exact || screen_score<RT, G>(u, v, g, c.sp, R, c.rg) <= thr))
             continue;
         bool same = (__double_as_longlong(v) == __double_as_longlong(v0)) && (g == g0);
 #pragma unroll
@@ -460,22 +410,21 @@ __device__ void resolve_job(WarpCtx<RT> &c, int lane, bool in_smem, const int32_
         if (same)
             continue;
         distinct = true;
-        const long long k = order_key(exact_score<RT>(u, v, g, c.sp, R, c.rg, c.grouped));
+        const long long k = order_key(exact_score<RT, G>(u, v, g, c.sp, R, c.rg));
         if (k < best_key || (k == best_key && o < best_i)) {
             best_key = k;
             best_i = o;
         }
     }
-    const bool any = __any_sync(FULL, distinct);
-    if (!any) {
+    if (!__any_sync(FULL, distinct)) {
         local_out = first - jstart;
         has_s = need_s;
         if (need_s)
-            s_out = exact_score<RT>(u0, v0, g0, c.sp, R, c.rg, c.grouped);
+            s_out = exact_score<RT, G>(u0, v0, g0, c.sp, R, c.rg);
         return;
     }
     if (lane == 0) {
-        const long long k0 = order_key(exact_score<RT>(u0, v0, g0, c.sp, R, c.rg, c.grouped));
+        const long long k0 = order_key(exact_score<RT, G>(u0, v0, g0, c.sp, R, c.rg));
         if (k0 < best_key || (k0 == best_key && first < best_i)) {
             best_key = k0;
             best_i = first;
@@ -495,25 +444,145 @@ __device__ void resolve_job(WarpCtx<RT> &c, int lane, bool in_smem, const int32_
     has_s = true;
 }
 
-// Evaluates one staged tile.
-template <int RT>
-__device__ void process_tile(WarpCtx<RT> &c, const TileDesc &d, const unsigned char *stage, const StageLayout &SL,
-                             float *qbuf, int64_t &big_first, Best &big_carry, int lane)
+// Resolves, one after the other, the ambiguous jobs whose closing lanes are set in amask, and records
+// each winner (lane 0). big: the job is chunked and read from global memory.
+template <int RT, bool G>
+__device__ __forceinline__ void resolve_row(WarpCtx<RT, G> &c, int lane, uint32_t amask, bool big,
+                                            const int32_t *units_s, const double *vals_s, const uint16_t *grp_s,
+                                            int jstart, int jend, float thr, int64_t job, int64_t big_first)
+{
+    while (amask) {
+        const int cl = __ffs(amask) - 1;
+        amask &= amask - 1;
+        const int js = __shfl_sync(FULL, jstart, cl);
+        const int je = __shfl_sync(FULL, jend, cl);
+        const float th = __shfl_sync(FULL, thr, cl);
+        const long long jb = __shfl_sync(FULL, (long long)job, cl);
+        double s_w = 0.0;
+        bool has_s = false;
+        int li;
+        resolve_job<RT, G>(c, lane, !big, units_s, vals_s, grp_s, js, je, big ? big_first : 0, th, c.want_min,
+                           s_w, has_s, li);
+        if (lane == 0) {
+            int32_t uw[Cols<RT>::N];
+            double vw;
+            int gw;
+            load_option<RT, G>(c, !big, units_s, vals_s, grp_s, js + li, big ? big_first : 0, uw, vw, gw);
+            take_winner<RT, G>(c, jb, li, uw, vw, gw, has_s, s_w);
+        }
+    }
+}
+
+// Stage pointers of one tile (the bulk copies start at the 16-byte boundary below the data).
+struct StagePtrs {
+    const int32_t *units;
+    const double *vals;
+    const uint16_t *grp;
+    const long long *off;
+};
+
+__device__ __forceinline__ StagePtrs stage_ptrs(const TileDesc &d, const unsigned char *stage, const StageLayout &SL,
+                                                int R)
+{
+    StagePtrs p;
+    p.units = reinterpret_cast<const int32_t *>(stage + SL.units + (int)((d.opt_begin * R * 4) & 15));
+    p.vals = reinterpret_cast<const double *>(stage + SL.vals + (int)((d.opt_begin * 8) & 15));
+    p.grp = reinterpret_cast<const uint16_t *>(stage + SL.grp + (int)((d.opt_begin * 2) & 15));
+    p.off = reinterpret_cast<const long long *>(stage + SL.off + (int)((d.job_begin * 8) & 15));
+    return p;
+}
+
+// Tile of a table whose jobs all have K = uniform_k options (a power of two <= 32). Tiles start at
+// job boundaries, so each aligned group of K lanes of a row is one job: a log2(K)-step xor
+// butterfly gives every lane of the group the smallest and second-smallest screen value; when the
+// job is unambiguous the unique lane holding the smallest value is the winner and records it from
+// its own registers.
+template <int RT, bool G>
+__device__ void process_tile_uniform(WarpCtx<RT, G> &c, const TileDesc &d, const StagePtrs &sp, int lane)
+{
+    const int R = c.R;
+    const int n = d.n_opt;
+    const int K = c.uniform_k;
+    for (int b = 0; b < n; b += 32) {
+        const int i = b + lane;
+        const bool valid = i < n;
+        int32_t u[Cols<RT>::N];
+        double v = 0.0;
+        int g = 0;
+        float q = INFINITY;
+        if (valid) {
+            const bool dup = load_units_smem<RT>(sp.units + (size_t)i * R, u, R);
+            v = sp.vals[i];
+            if (G)
+                g = sp.grp[i];
+            if (!dup)
+                q = screen_score<RT, G>(u, v, g, c.sp, R, c.rg);
+        }
+        float m1 = q, m2 = INFINITY;
+        for (int dd = 1; dd < K; dd <<= 1) {
+            const float o1 = __shfl_xor_sync(FULL, m1, dd);
+            const float o2 = __shfl_xor_sync(FULL, m2, dd);
+            m2 = fminf(fminf(m2, o2), fmaxf(m1, o1));
+            m1 = fminf(m1, o1);
+        }
+        const float thr = __fadd_ru(m1, c.sp.e2);
+        const bool amb = c.sp.exact || !(m2 > thr);
+        const int64_t job = d.job_begin + (i >> c.log2_k);
+        if (valid && !amb && q == m1)
+            take_winner<RT, G>(c, job, i & (K - 1), u, v, g, false, 0.0);
+        const uint32_t amask = __ballot_sync(FULL, valid && amb && (i & (K - 1)) == 0);
+        if (amask)
+            resolve_row<RT, G>(c, lane, amask, false, sp.units, sp.vals, sp.grp, i, i + K, thr, job, 0);
+    }
+}
+
+// Per-job running state of the general (CSR) path: smallest screen value with its index, and the
+// smallest value of every other option. Commutative and associative (ties keep the lower index).
+struct Best {
+    float m1;
+    int idx;
+    float m2;
+};
+
+__device__ __forceinline__ Best best_none() { return Best{INFINITY, kIdxNone, INFINITY}; }
+
+__device__ __forceinline__ Best combine(const Best &a, const Best &b)
+{
+    const bool take_b = (b.m1 < a.m1) || (b.m1 == a.m1 && b.idx < a.idx);
+    return Best{take_b ? b.m1 : a.m1, take_b ? b.idx : a.idx, fminf(fminf(a.m2, b.m2), fmaxf(a.m1, b.m1))};
+}
+
+__device__ __forceinline__ Best shfl_up_best(const Best &x, int d)
+{
+    return Best{__shfl_up_sync(FULL, x.m1, d), __shfl_up_sync(FULL, x.idx, d), __shfl_up_sync(FULL, x.m2, d)};
+}
+
+__device__ __forceinline__ Best shfl_best(const Best &x, int src)
+{
+    return Best{__shfl_sync(FULL, x.m1, src), __shfl_sync(FULL, x.idx, src), __shfl_sync(FULL, x.m2, src)};
+}
+
+__device__ __forceinline__ Best allreduce_best(Best x)
+{
+#pragma unroll
+    for (int d = 16; d >= 1; d >>= 1)
+        x = combine(x, Best{__shfl_xor_sync(FULL, x.m1, d), __shfl_xor_sync(FULL, x.idx, d),
+                            __shfl_xor_sync(FULL, x.m2, d)});
+    return x;
+}
+
+// Tile of a general table (any job sizes). Rows of 32 options are reduced by a segmented scan:
+// heads (first options) and ends (last options) of jobs in the row come from the staged job
+// offsets; a job continuing from the previous row enters as a carry; rows entirely inside one job
+// only fold per lane. A job larger than a tile arrives as consecutive chunk tiles of this warp
+// (big_first / big_carry carry its state across them) and is resolved from global memory.
+template <int RT, bool G>
+__device__ void process_tile_general(WarpCtx<RT, G> &c, const TileDesc &d, const StagePtrs &sp, int64_t &big_first,
+                                     Best &big_carry, int lane)
 {
     const int R = c.R;
     const int n = d.n_opt;
     const bool big = (d.flags & TILE_BIG) != 0;
-
-    // data offsets inside the stage (the bulk copies start at the 16-byte boundary below the data)
-    const int du = (int)((d.opt_begin * R * 4) & 15);
-    const int dv = (int)((d.opt_begin * 8) & 15);
-    const int dg = (int)((d.opt_begin * 2) & 15);
-    const int doff = (int)((d.job_begin * 8) & 15);
-    const int32_t *units_s = reinterpret_cast<const int32_t *>(stage + SL.units + du);
-    const double *vals_s = reinterpret_cast<const double *>(stage + SL.vals + dv);
-    const uint16_t *grp_s = reinterpret_cast<const uint16_t *>(stage + SL.grp + dg);
-    const long long *off_s = reinterpret_cast<const long long *>(stage + SL.off + doff);
-
     int chunk_base = 0;
     Best carry = best_none();
     if (big) {
@@ -536,92 +605,70 @@ __device__ void process_tile(WarpCtx<RT> &c, const TileDesc &d, const unsigned c
         int32_t u[Cols<RT>::N];
         float q = INFINITY;
         if (valid) {
-            load_units_smem<RT>(units_s + (size_t)i * R, u, R);
-            const double v = vals_s[i];
-            const int g = c.grouped ? (int)grp_s[i] : 0;
-            q = screen_score<RT>(u, v, g, c.sp, R, c.rg, c.grouped);
-            if (!big)
-                qbuf[i] = q;
+            const bool dup = load_units_smem<RT>(sp.units + (size_t)i * R, u, R);
+            const double v = sp.vals[i];
+            const int g = G ? (int)sp.grp[i] : 0;
+            if (!dup)
+                q = screen_score<RT, G>(u, v, g, c.sp, R, c.rg);
         }
 
-        Best x;
-        bool closing;
-        int jstart;
-        int64_t job;
-        if (c.uniform_k > 0) {
-            // every job has uniform_k options (a power of two <= 32) and tiles start at job
-            // boundaries, so each aligned group of uniform_k lanes is one job: an xor butterfly
-            const int K = c.uniform_k;
-            x = valid ? Best{q, i, INFINITY} : best_none();
-            for (int dd = 1; dd < K; dd <<= 1)
-                x = combine(x, Best{__shfl_xor_sync(FULL, x.m1, dd), __shfl_xor_sync(FULL, x.idx, dd),
-                                    __shfl_xor_sync(FULL, x.m2, dd)});
-            closing = valid && ((i & (K - 1)) == K - 1);
-            jstart = i & ~(K - 1);
-            job = d.job_begin + (i >> c.log2_k);
+        // heads (first option of a job) and ends (last option of a job) in this row
+        uint32_t H, E;
+        if (!big) {
+            const int k0 = wp + lane;
+            const int sa = (k0 < n_job) ? (int)(sp.off[k0] - d.opt_begin) : 0x7fffffff;
+            const int sb = (k0 + 1 < n_job) ? (int)(sp.off[k0 + 1] - d.opt_begin) : (k0 + 1 == n_job ? n : 0x7fffffff);
+            const int hb = sa - b, eb = sb - 1 - b;
+            H = __reduce_or_sync(FULL, (hb >= 0 && hb < 32) ? (1u << hb) : 0u);
+            E = __reduce_or_sync(FULL, (eb >= 0 && eb < 32) ? (1u << eb) : 0u);
         } else {
-            // heads (first option of a job) and ends (last option of a job) in this row
-            uint32_t H, E;
-            int sa = 0x7fffffff;
-            if (!big) {
-                const int k0 = wp + lane;
-                sa = (k0 < n_job) ? (int)(off_s[k0] - d.opt_begin) : 0x7fffffff;
-                const int sb = (k0 + 1 < n_job) ? (int)(off_s[k0 + 1] - d.opt_begin) : (k0 + 1 == n_job ? n : 0x7fffffff);
-                const int hb = sa - b, eb = sb - 1 - b;
-                H = __reduce_or_sync(FULL, (hb >= 0 && hb < 32) ? (1u << hb) : 0u);
-                E = __reduce_or_sync(FULL, (eb >= 0 && eb < 32) ? (1u << eb) : 0u);
-            } else {
-                H = ((d.flags & TILE_BIG_FIRST) && b == 0) ? 1u : 0u;
-                const int eb = n - 1 - b;
-                E = ((d.flags & TILE_BIG_LAST) && eb >= 0 && eb < 32) ? (1u << eb) : 0u;
-            }
-
-            x = valid ? Best{q, i + chunk_base, INFINITY} : best_none();
-            if (H == 0u && E == 0u) {    // the whole row lies inside the open job: fold per lane
-                priv = combine(priv, x);
-                priv_dirty = true;
-                continue;
-            }
-            if (priv_dirty) {
-                carry = combine(carry, allreduce_best(priv));
-                priv = best_none();
-                priv_dirty = false;
-            }
-            // segmented inclusive scan; lanes before the first head continue the open job (carry)
-            const uint32_t le = (lane == 31) ? FULL : ((2u << lane) - 1u);
-            const int seg_lo = 31 - __clz(H & le);
-            if (H != FULL) {
-    #pragma unroll
-                for (int dd = 1; dd < 32; dd <<= 1) {
-                    const Best o = shfl_up_best(x, dd);
-                    if (lane >= dd && lane - dd >= seg_lo)
-                        x = combine(o, x);
-                }
-            }
-            if (seg_lo < 0)
-                x = combine(carry, x);
-
-            closing = (E >> lane) & 1u;
-            const uint32_t lt = (1u << lane) - 1u;
-            // tile-local start of each lane's job
-            if (big)
-                jstart = 0;
-            else
-                jstart = (seg_lo >= 0) ? (b + seg_lo) : open_start;
-            job = big ? d.job_begin : (d.job_begin + wp + __popc(E & lt));
-
-            // next row's open job
-            const Best last = shfl_best(x, 31);
-            const int last_start = __shfl_sync(FULL, jstart, 31);
-            if ((E >> 31) & 1u) {
-                carry = best_none();
-            } else {
-                carry = last;
-                open_start = last_start;
-            }
-            if (!big)
-                wp += __popc(E);
+            H = ((d.flags & TILE_BIG_FIRST) && b == 0) ? 1u : 0u;
+            const int eb = n - 1 - b;
+            E = ((d.flags & TILE_BIG_LAST) && eb >= 0 && eb < 32) ? (1u << eb) : 0u;
         }
+
+        Best x = valid ? Best{q, i + chunk_base, INFINITY} : best_none();
+        if (H == 0u && E == 0u) {    // the whole row lies inside the open job: fold per lane
+            priv = combine(priv, x);
+            priv_dirty = true;
+            continue;
+        }
+        if (priv_dirty) {
+            carry = combine(carry, allreduce_best(priv));
+            priv = best_none();
+            priv_dirty = false;
+        }
+        // segmented inclusive scan; lanes before the first head continue the open job (carry)
+        const uint32_t le = (lane == 31) ? FULL : ((2u << lane) - 1u);
+        const int seg_lo = 31 - __clz(H & le);
+        if (H != FULL) {
+#pragma unroll
+            for (int dd = 1; dd < 32; dd <<= 1) {
+                const Best o = shfl_up_best(x, dd);
+                if (lane >= dd && lane - dd >= seg_lo)
+                    x = combine(o, x);
+            }
+        }
+        if (seg_lo < 0)
+            x = combine(carry, x);
+
+        const bool closing = (E >> lane) & 1u;
+        const uint32_t lt = (1u << lane) - 1u;
+        const int jstart = big ? 0 : ((seg_lo >= 0) ? (b + seg_lo) : open_start);
+        const int64_t job = big ? d.job_begin : (d.job_begin + wp + __popc(E & lt));
+        const int jend = big ? (chunk_base + i + 1) : (i + 1);
+
+        // next row's open job
+        const Best last = shfl_best(x, 31);
+        const int last_start = __shfl_sync(FULL, jstart, 31);
+        if ((E >> 31) & 1u) {
+            carry = best_none();
+        } else {
+            carry = last;
+            open_start = last_start;
+        }
+        if (!big)
+            wp += __popc(E);
 
         // unambiguous closings finish here; ambiguous ones are resolved exactly by the warp
         const float thr = __fadd_ru(x.m1, c.sp.e2);
@@ -630,60 +677,14 @@ __device__ void process_tile(WarpCtx<RT> &c, const TileDesc &d, const unsigned c
             const int li = big ? x.idx : (x.idx - jstart);
             int32_t uw[Cols<RT>::N];
             double vw;
-            int gw = 0;
-            if (big) {
-                const int64_t og = big_first + x.idx;
-                load_units_global<RT>(c.t.units + og * R, uw, R);
-                vw = __ldg(c.t.values + og);
-                if (c.grouped)
-                    gw = __ldg(c.t.group + og);
-            } else {
-                load_units_smem<RT>(units_s + (size_t)x.idx * R, uw, R);
-                vw = vals_s[x.idx];
-                if (c.grouped)
-                    gw = grp_s[x.idx];
-            }
-            take_winner<RT>(c, job, li, uw, vw, gw, false, 0.0);
+            int gw;
+            load_option<RT, G>(c, !big, sp.units, sp.vals, sp.grp, big ? x.idx : x.idx, big ? big_first : 0, uw, vw,
+                               gw);
+            take_winner<RT, G>(c, job, li, uw, vw, gw, false, 0.0);
         }
-        uint32_t amask = __ballot_sync(FULL, amb);
+        const uint32_t amask = __ballot_sync(FULL, amb);
         if (amask)
-            __syncwarp();   // this row's qbuf writes are visible to every lane before resolution
-        while (amask) {
-            const int cl = __ffs(amask) - 1;
-            amask &= amask - 1;
-            const int js = __shfl_sync(FULL, jstart, cl);
-            const float th = __shfl_sync(FULL, thr, cl);
-            const long long jb = __shfl_sync(FULL, (long long)job, cl);
-            double s_w = 0.0;
-            bool has_s = false;
-            int li_w;
-            if (big) {
-                resolve_job<RT>(c, lane, false, units_s, vals_s, grp_s, qbuf, 0, chunk_base + b + cl + 1, big_first,
-                                th, c.want_min, s_w, has_s, li_w);
-            } else {
-                resolve_job<RT>(c, lane, true, units_s, vals_s, grp_s, qbuf, js, b + cl + 1, 0, th, c.want_min, s_w,
-                                has_s, li_w);
-            }
-            if (lane == 0) {
-                int32_t uw[Cols<RT>::N];
-                double vw;
-                int gw = 0;
-                if (big) {
-                    const int64_t og = big_first + li_w;
-                    load_units_global<RT>(c.t.units + og * R, uw, R);
-                    vw = __ldg(c.t.values + og);
-                    if (c.grouped)
-                        gw = __ldg(c.t.group + og);
-                } else {
-                    const int o = js + li_w;
-                    load_units_smem<RT>(units_s + (size_t)o * R, uw, R);
-                    vw = vals_s[o];
-                    if (c.grouped)
-                        gw = grp_s[o];
-                }
-                take_winner<RT>(c, jb, li_w, uw, vw, gw, has_s, s_w);
-            }
-        }
+            resolve_row<RT, G>(c, lane, amask, big, sp.units, sp.vals, sp.grp, jstart, jend, thr, job, big_first);
     }
     if (big) {
         if (priv_dirty)
@@ -692,9 +693,9 @@ __device__ void process_tile(WarpCtx<RT> &c, const TileDesc &d, const unsigned c
     }
 }
 
-// Issues the bulk copies of tile d into a stage; lane 0 only.
+// Issues the bulk copies of tile d into a stage; lane 0 only. Uniform tables need no job offsets.
 __device__ __forceinline__ void issue_tile(const DevTable &t, const TileDesc &d, unsigned char *stage,
-                                           const StageLayout &SL, uint32_t bar)
+                                           const StageLayout &SL, uint32_t bar, bool need_offsets)
 {
     const int R = t.R;
     const int64_t ub = d.opt_begin * R * 4, ue = (d.opt_begin + d.n_opt) * R * 4;
@@ -703,7 +704,7 @@ __device__ __forceinline__ void issue_tile(const DevTable &t, const TileDesc &d,
     const int64_t vlo = vb & ~int64_t(15), vhi = (ve + 15) & ~int64_t(15);
     uint32_t total = (uint32_t)(uhi - ulo) + (uint32_t)(vhi - vlo);
     int64_t olo = 0, ohi = 0, glo = 0, ghi = 0;
-    const bool offs = !(d.flags & TILE_BIG);
+    const bool offs = need_offsets && !(d.flags & TILE_BIG);
     if (offs) {
         const int64_t ob = d.job_begin * 8, oe = (d.job_begin + d.n_job + 1) * 8;
         olo = ob & ~int64_t(15);
@@ -731,9 +732,11 @@ __device__ __forceinline__ void issue_tile(const DevTable &t, const TileDesc &d,
 }
 
 // One evaluation pass over every tile: a best response of every job of every (non-stopped) scenario.
-template <int RT>
-__global__ void __launch_bounds__(kWarpsPerCta * 32) k_pass(DevTable t, DevState st, DevPlan pl, SolveArgs a,
-                                                              int round, int kind)
+// UNI selects the uniform-K row reduction (tables whose jobs all have the same power-of-two size up
+// to 32, never grouped); otherwise the general segmented path runs.
+template <int RT, bool G, bool UNI>
+__global__ void __launch_bounds__(kWarpsPerCta * 32, UNI ? kMinCtasPerSm : kMinCtasPerSmGeneral) k_pass(DevTable t, DevState st, DevPlan pl,
+                                                                          SolveArgs a, int round, int kind)
 {
     extern __shared__ __align__(128) unsigned char smem[];
     const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
@@ -744,20 +747,18 @@ __global__ void __launch_bounds__(kWarpsPerCta * 32) k_pass(DevTable t, DevState
     if (k_begin >= k_end)
         return;
 
-    const bool grouped = t.group != nullptr;
-    const WarpSmem WS = warp_smem(pl.tile_opt, t.R, grouped, t.P);
-    const StageLayout SL = stage_layout(pl.tile_opt, t.R, grouped);
+    const WarpSmem WS = warp_smem(pl.tile_opt, t.R, G, t.P);
+    const StageLayout SL = stage_layout(pl.tile_opt, t.R, G);
     unsigned char *wsm = smem + (size_t)wid * WS.bytes;
-    float *qbuf = reinterpret_cast<float *>(wsm + WS.qbuf);
     float *p32s = reinterpret_cast<float *>(wsm + WS.p32);
     const uint32_t bar0 = smem_u32(wsm + WS.bars);
+    const bool need_offsets = !UNI;
 
-    WarpCtx<RT> c;
+    WarpCtx<RT, G> c;
     c.t = t;
     c.st = st;
     c.R = RT ? RT : t.R;
     c.rg = t.r_global;
-    c.grouped = grouped;
     c.kind = kind;
     c.want_min = (kind == PASS_FINAL) || (st.dual_trace != nullptr);
     c.want_hash = (kind == PASS_ROUND) && (st.hash_trace != nullptr);
@@ -783,7 +784,7 @@ __global__ void __launch_bounds__(kWarpsPerCta * 32) k_pass(DevTable t, DevState
     while (issued < k_end && issued < k_begin + kStages - 1) {
         if (lane == 0) {
             const int sidx = (issued - k_begin) % kStages;
-            issue_tile(t, pl.tiles[issued], wsm + sidx * SL.bytes, SL, bar0 + 8 * sidx);
+            issue_tile(t, pl.tiles[issued], wsm + sidx * SL.bytes, SL, bar0 + 8 * sidx, need_offsets);
         }
         ++issued;
     }
@@ -795,7 +796,7 @@ __global__ void __launch_bounds__(kWarpsPerCta * 32) k_pass(DevTable t, DevState
             __syncwarp();
             if (lane == 0) {
                 const int sidx = (issued - k_begin) % kStages;
-                issue_tile(t, pl.tiles[issued], wsm + sidx * SL.bytes, SL, bar0 + 8 * sidx);
+                issue_tile(t, pl.tiles[issued], wsm + sidx * SL.bytes, SL, bar0 + 8 * sidx, need_offsets);
             }
             ++issued;
         }
@@ -807,19 +808,82 @@ __global__ void __launch_bounds__(kWarpsPerCta * 32) k_pass(DevTable t, DevState
             break;
         }
         if (d.scenario != c.s)
-            enter_scenario<RT>(c, d.scenario, p32s, lane);
-        if (!c.sp.skip)
-            process_tile<RT>(c, d, wsm + sidx * SL.bytes, SL, qbuf, big_first, big_carry, lane);
+            enter_scenario<RT, G>(c, d.scenario, p32s, lane);
+        if (!c.sp.skip) {
+            const StagePtrs ptrs = stage_ptrs(d, wsm + sidx * SL.bytes, SL, c.R);
+            if (UNI)
+                process_tile_uniform<RT, G>(c, d, ptrs, lane);
+            else
+                process_tile_general<RT, G>(c, d, ptrs, big_first, big_carry, lane);
+        }
         __syncwarp();
     }
     if (failed_at < 0) {
-        flush<RT>(c, lane);
+        flush<RT, G>(c, lane);
     } else {
         // a copy never completed: wait (bounded) for every copy still in flight, then leave
         for (int k = failed_at; k < issued; ++k) {
             const int sidx = (k - k_begin) % kStages;
             wait_stage(bar0 + 8 * sidx, (uint32_t)(((k - k_begin) / kStages) & 1), st.err);
         }
+    }
+}
+
+// ---------------------------------------------------------------------------------------------
+// Load-time marking of exact duplicates: option o of a job is marked (sign bit of its column-0
+// unit) when an earlier option of the same job has the same units, value and group. Such an option
+// ties its twin in every round and loses the tie on index, so it never changes a best response;
+// the screen skips it. One warp per job, jobs of up to kDedupMaxK options (larger jobs stay
+// unmarked and are still exact: the resolution also compares survivors with the first one).
+
+constexpr int kDedupMaxK = 1024;
+constexpr int kDedupWarps = 4;
+
+__device__ __forceinline__ uint64_t option_hash(const DevTable &t, int64_t o)
+{
+    uint64_t h = splitmix64_mix((uint64_t)__double_as_longlong(t.values[o]));
+    for (int r = 0; r < t.R; ++r)
+        h = splitmix64_mix(h ^ (uint64_t)(uint32_t)(t.units[o * t.R + r] & 0x7fffffff) ^ ((uint64_t)r << 40));
+    if (t.group)
+        h = splitmix64_mix(h ^ ((uint64_t)t.group[o] << 48));
+    return h;
+}
+
+__device__ __forceinline__ bool same_option(const DevTable &t, int64_t a, int64_t b)
+{
+    if (__double_as_longlong(t.values[a]) != __double_as_longlong(t.values[b]))
+        return false;
+    if (t.group && t.group[a] != t.group[b])
+        return false;
+    for (int r = 0; r < t.R; ++r)
+        if ((t.units[a * t.R + r] & 0x7fffffff) != (t.units[b * t.R + r] & 0x7fffffff))
+            return false;
+    return true;
+}
+
+__global__ void __launch_bounds__(kDedupWarps * 32) k_mark_duplicates(DevTable t, int32_t *units)
+{
+    __shared__ uint64_t hs[kDedupWarps][kDedupMaxK];
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+    const int64_t n_jobs = (int64_t)t.S * t.J;
+    for (int64_t j = (int64_t)blockIdx.x * kDedupWarps + wid; j < n_jobs; j += (int64_t)gridDim.x * kDedupWarps) {
+        const int64_t a = t.job_off[j];
+        const int K = (int)(t.job_off[j + 1] - a);
+        if (K < 2 || K > kDedupMaxK)
+            continue;
+        for (int k = lane; k < K; k += 32)
+            hs[wid][k] = option_hash(t, a + k);
+        __syncwarp();
+        for (int k = lane; k < K; k += 32) {
+            const uint64_t h = hs[wid][k];
+            for (int k2 = 0; k2 < k; ++k2) {
+                if (hs[wid][k2] == h && same_option(t, a + k, a + k2)) {
+                    units[(a + k) * t.R] |= (int32_t)0x80000000;
+                    break;
+                }
+            }
+        }
+        __syncwarp();
     }
 }
 
@@ -1090,10 +1154,10 @@ __global__ void k_validate_offsets(DevTable t, unsigned int *flags)
         atomicOr(flags, bad);
 }
 
-template <int RT>
+template <int RT, bool G, bool UNI>
 void *pass_kernel_ptr()
 {
-    return reinterpret_cast<void *>(&k_pass<RT>);
+    return reinterpret_cast<void *>(&k_pass<RT, G, UNI>);
 }
 
 }  // namespace
@@ -1103,19 +1167,35 @@ int pass_smem_bytes(int R, bool grouped, int P, int tile_opt)
     return kWarpsPerCta * warp_smem(tile_opt, R, grouped, P).bytes;
 }
 
-static const void *pass_kernel_for(int R)
+static const void *pass_kernel_for(int R, bool grouped, bool uni)
 {
+    if (grouped) {
+        switch (R) {
+        case 4: return pass_kernel_ptr<4, true, false>();
+        case 6: return pass_kernel_ptr<6, true, false>();
+        case 8: return pass_kernel_ptr<8, true, false>();
+        default: return pass_kernel_ptr<0, true, false>();
+        }
+    }
+    if (uni) {
+        switch (R) {
+        case 4: return pass_kernel_ptr<4, false, true>();
+        case 6: return pass_kernel_ptr<6, false, true>();
+        case 8: return pass_kernel_ptr<8, false, true>();
+        default: return pass_kernel_ptr<0, false, true>();
+        }
+    }
     switch (R) {
-    case 4: return pass_kernel_ptr<4>();
-    case 6: return pass_kernel_ptr<6>();
-    case 8: return pass_kernel_ptr<8>();
-    default: return pass_kernel_ptr<0>();
+    case 4: return pass_kernel_ptr<4, false, false>();
+    case 6: return pass_kernel_ptr<6, false, false>();
+    case 8: return pass_kernel_ptr<8, false, false>();
+    default: return pass_kernel_ptr<0, false, false>();
     }
 }
 
-int pass_ctas_per_sm(int R, bool grouped, int P, int tile_opt)
+int pass_ctas_per_sm(int R, bool grouped, bool uniform, int P, int tile_opt)
 {
-    const void *fn = pass_kernel_for(R);
+    const void *fn = pass_kernel_for(R, grouped, uniform && !grouped);
     const int smem = pass_smem_bytes(R, grouped, P, tile_opt);
     if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess)
         return 0;
@@ -1151,12 +1231,43 @@ cudaError_t launch_pass(const DevTable &t, const DevState &st, const DevPlan &pl
 {
     const bool grouped = t.group != nullptr;
     const int smem = pass_smem_bytes(t.R, grouped, t.P, pl.tile_opt);
-    switch (t.R) {
-    case 4: k_pass<4><<<grid, kWarpsPerCta * 32, smem, stream>>>(t, st, pl, a, round, kind); break;
-    case 6: k_pass<6><<<grid, kWarpsPerCta * 32, smem, stream>>>(t, st, pl, a, round, kind); break;
-    case 8: k_pass<8><<<grid, kWarpsPerCta * 32, smem, stream>>>(t, st, pl, a, round, kind); break;
-    default: k_pass<0><<<grid, kWarpsPerCta * 32, smem, stream>>>(t, st, pl, a, round, kind); break;
+    const dim3 block(kWarpsPerCta * 32);
+#define ESP_LAUNCH_PASS(RT_, G_, U_) k_pass<RT_, G_, U_><<<grid, block, smem, stream>>>(t, st, pl, a, round, kind)
+    if (grouped) {
+        switch (t.R) {
+        case 4: ESP_LAUNCH_PASS(4, true, false); break;
+        case 6: ESP_LAUNCH_PASS(6, true, false); break;
+        case 8: ESP_LAUNCH_PASS(8, true, false); break;
+        default: ESP_LAUNCH_PASS(0, true, false); break;
+        }
+    } else if (pl.uniform_k > 0) {
+        switch (t.R) {
+        case 4: ESP_LAUNCH_PASS(4, false, true); break;
+        case 6: ESP_LAUNCH_PASS(6, false, true); break;
+        case 8: ESP_LAUNCH_PASS(8, false, true); break;
+        default: ESP_LAUNCH_PASS(0, false, true); break;
+        }
+    } else {
+        switch (t.R) {
+        case 4: ESP_LAUNCH_PASS(4, false, false); break;
+        case 6: ESP_LAUNCH_PASS(6, false, false); break;
+        case 8: ESP_LAUNCH_PASS(8, false, false); break;
+        default: ESP_LAUNCH_PASS(0, false, false); break;
+        }
     }
+#undef ESP_LAUNCH_PASS
+    return cudaGetLastError();
+}
+
+cudaError_t launch_mark_duplicates(const DevTable &t, int32_t *units, cudaStream_t stream)
+{
+    const int64_t n_jobs = (int64_t)t.S * t.J;
+    if (n_jobs == 0)
+        return cudaSuccess;
+    int64_t blocks = (n_jobs + kDedupWarps - 1) / kDedupWarps;
+    if (blocks > 65536)
+        blocks = 65536;
+    k_mark_duplicates<<<(int)blocks, kDedupWarps * 32, 0, stream>>>(t, units);
     return cudaGetLastError();
 }
 

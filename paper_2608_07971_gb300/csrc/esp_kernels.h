@@ -69,10 +69,14 @@ enum PassKind : int32_t { PASS_ROUND = 0, PASS_FINAL = 1 };
 int pass_smem_bytes(int R, bool grouped, int P, int tile_opt);
 
 // Maximum resident CTAs per SM of the evaluation kernel for this table shape (0 if it cannot run).
-int pass_ctas_per_sm(int R, bool grouped, int P, int tile_opt);
+int pass_ctas_per_sm(int R, bool grouped, bool uniform, int P, int tile_opt);
 
 cudaError_t launch_validate(const DevTable &t, double *vmax, int32_t *umax, unsigned int *flags,
                             cudaStream_t stream);
+// Marks every option that repeats an earlier option of its job (units, value and group equal) by
+// setting the sign bit of its column-0 unit in `units` (the device copy of t.units).
+cudaError_t launch_mark_duplicates(const DevTable &t, int32_t *units, cudaStream_t stream);
+
 cudaError_t launch_init(const DevTable &t, const DevState &st, const SolveArgs &a, const double *lambda0,
                         cudaStream_t stream);
 cudaError_t launch_pass(const DevTable &t, const DevState &st, const DevPlan &pl, const SolveArgs &a,

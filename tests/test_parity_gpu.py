@@ -6,6 +6,8 @@ primal and dual objectives within 1e-9 relative (the GPU sums in a fixed tree, t
 order).
 """
 
+import zlib
+
 import numpy as np
 import pytest
 
@@ -132,9 +134,9 @@ def test_evaluate_at_oracle_prices(name):
 # Ragged, degenerate and extreme tables
 
 @pytest.mark.parametrize("case", ["k1", "ragged", "big_jobs", "tile_edges", "r16", "grouped_many",
-                                  "ties", "single_job", "u2", "u32", "u16dups", "u8grouped"])
+                                  "ties", "single_job", "u2", "u32", "u16dups", "u8grouped", "big_dups"])
 def test_edge_tables(case):
-    rng = np.random.default_rng(hash(case) % 2**32)
+    rng = np.random.default_rng(zlib.crc32(case.encode()))
     if case == "k1":
         t = W.random_table(rng, S=3, J=1000, R=6, kmin=1, kmax=1)
     elif case == "ragged":
@@ -164,6 +166,16 @@ def test_edge_tables(case):
             a = t.job_off[j]
             t.units[a + 8:a + 16] = t.units[a:a + 8]
             t.values[a + 8:a + 16] = t.values[a:a + 8]
+    elif case == "big_dups":
+        # jobs of 1000 (duplicates marked at load) and 1500 options (too large to mark: resolved
+        # by the comparison with the first survivor), most options repeating a few profiles
+        t = W.random_table(rng, S=2, J=6, R=6, kmin=1000, kmax=1500, umax=3, dyadic=True)
+        for j in range(t.S * t.J):
+            a, b = t.job_off[j], t.job_off[j + 1]
+            base = np.arange(a, b)
+            src = a + (base - a) % 7
+            t.units[base] = t.units[src]
+            t.values[base] = t.values[src]
     elif case == "u8grouped":
         t = W.random_table(rng, S=2, J=300, R=8, kmin=8, kmax=8, groups=16, r_global=6)
     else:
