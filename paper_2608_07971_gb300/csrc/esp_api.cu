@@ -339,7 +339,7 @@ esp_status load_common(esp_ctx *ctx, int32_t S, int32_t J, int32_t R, int32_t P,
         min_k = std::min<int64_t>(min_k, k);
     }
     ctx->uniform_k = (!grouped && min_k == max_k && max_k <= 32 && (max_k & (max_k - 1)) == 0) ? (int32_t)max_k : 0;
-    const int tile_opt = tile_options_for(R, grouped, max_k);
+    const int tile_opt = tile_options_for(R, grouped, max_k, ctx->uniform_k >= 4);
     const int per_sm = pass_ctas_per_sm(R, grouped, ctx->uniform_k > 0, P, tile_opt);
     if (per_sm < 1) {
         release_table(ctx);

@@ -14,7 +14,7 @@ namespace esp {
 constexpr int kMaxR = 16;            // stored resource columns per option
 constexpr int kWarpsPerCta = 4;      // warps of a CTA; each warp owns its own stage ring
 constexpr int kStages = 2;           // TMA stages per warp
-constexpr int kMinCtasPerSm = 5;     // register budget of the uniform-K evaluation kernel: 5 CTAs (20 warps) per SM
+constexpr int kMinCtasPerSm = 4;     // register budget of the uniform-K evaluation kernel: 4 CTAs (16 warps) per SM
 constexpr int kMinCtasPerSmGeneral = 4;  // the general kernel: 4 CTAs (16 warps) per SM
 constexpr int kStageDataBytes = 8192;// option bytes (units + values [+ group]) one stage aims at
 
@@ -47,9 +47,11 @@ ESP_HD int tile_options(int R, bool grouped)
 // Tile size for a table whose largest job has max_k options: large enough that every job of up to
 // the maximum tile size stays whole (its exact resolution then reads the stage), at least 128
 // options, and otherwise small so that more warps fit per SM.
-ESP_HD int tile_options_for(int R, bool grouped, long long max_k)
+ESP_HD int tile_options_for(int R, bool grouped, long long max_k, bool uniform4)
 {
     const int cap = tile_options(R, grouped);
+    if (uniform4)   // uniform jobs of 4..32 options: the largest tile (amortises per-tile work)
+        return cap;
     long long t = (max_k + 31) & ~31LL;
     if (t < 128)
         t = 128;

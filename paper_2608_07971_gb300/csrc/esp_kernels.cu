@@ -536,6 +536,100 @@ __device__ void process_tile_uniform(WarpCtx<RT, G> &c, const TileDesc &d, const
     }
 }
 
+// Units of the 4 consecutive options starting at p (16-byte aligned): six, four or eight 16-byte
+// shared loads for R = 6, 4, 8. Duplicate marks are removed and returned in dup[].
+template <int RT>
+__device__ __forceinline__ void load_units4_smem(const int32_t *p, int32_t (*u)[Cols<RT>::N], bool *dup, int R)
+{
+    if constexpr (RT == 4 || RT == 6 || RT == 8) {
+        constexpr int W = RT;
+        int32_t raw[4 * W];
+        const int4 *q4 = reinterpret_cast<const int4 *>(p);
+#pragma unroll
+        for (int k = 0; k < W; ++k) {
+            const int4 x = q4[k];
+            raw[4 * k] = x.x; raw[4 * k + 1] = x.y; raw[4 * k + 2] = x.z; raw[4 * k + 3] = x.w;
+        }
+#pragma unroll
+        for (int o = 0; o < 4; ++o)
+#pragma unroll
+            for (int r = 0; r < W; ++r)
+                u[o][r] = raw[o * W + r];
+    } else {
+#pragma unroll
+        for (int o = 0; o < 4; ++o)
+#pragma unroll
+            for (int r = 0; r < Cols<RT>::N; ++r)
+                u[o][r] = (r < R) ? p[o * R + r] : 0;
+    }
+#pragma unroll
+    for (int o = 0; o < 4; ++o) {
+        dup[o] = u[o][0] < 0;
+        u[o][0] &= 0x7fffffff;
+    }
+}
+
+// Tile of a table whose jobs all have K options, K in {4, 8, 16, 32}. Each lane evaluates 4
+// consecutive options of one job (a tile row block is 128 options), keeps their smallest and
+// second-smallest screen values, and a log2(K / 4)-step xor butterfly over the job's K / 4 lanes
+// completes the job. An unambiguous job's winner is the unique option holding the smallest value.
+template <int RT, bool G>
+__device__ void process_tile_uniform4(WarpCtx<RT, G> &c, const TileDesc &d, const StagePtrs &sp, int lane)
+{
+    const int R = c.R;
+    const int n = d.n_opt;
+    const int K = c.uniform_k;
+    const int KL = K >> 2;                  // lanes per job
+    for (int b = 0; b < n; b += 128) {
+        const int base = b + 4 * lane;
+        const bool valid = base < n;        // n is a multiple of K, hence of 4
+        float q[4] = {INFINITY, INFINITY, INFINITY, INFINITY};
+        if (valid) {
+            int32_t u[4][Cols<RT>::N];
+            bool dup[4];
+            load_units4_smem<RT>(sp.units + (size_t)base * R, u, dup, R);
+            const double2 va = reinterpret_cast<const double2 *>(sp.vals + base)[0];
+            const double2 vb = reinterpret_cast<const double2 *>(sp.vals + base)[1];
+            const double v[4] = {va.x, va.y, vb.x, vb.y};
+#pragma unroll
+            for (int o = 0; o < 4; ++o)
+                if (!dup[o])
+                    q[o] = screen_score<RT, G>(u[o], v[o], 0, c.sp, R, c.rg);
+        }
+        // smallest and second smallest of the lane's four values
+        float a0 = fminf(q[0], q[1]), a1 = fmaxf(q[0], q[1]);
+        float b0 = fminf(q[2], q[3]), b1 = fmaxf(q[2], q[3]);
+        float m1 = fminf(a0, b0);
+        float m2 = fminf(fmaxf(a0, b0), fminf(a1, b1));
+        for (int dd = 1; dd < KL; dd <<= 1) {
+            const float o1 = __shfl_xor_sync(FULL, m1, dd);
+            const float o2 = __shfl_xor_sync(FULL, m2, dd);
+            m2 = fminf(fminf(m2, o2), fmaxf(m1, o1));
+            m1 = fminf(m1, o1);
+        }
+        const float thr = __fadd_ru(m1, c.sp.e2);
+        const bool amb = c.sp.exact || !(m2 > thr);
+        if (valid && !amb) {
+            int w = -1;
+#pragma unroll
+            for (int o = 3; o >= 0; --o)
+                if (q[o] == m1)
+                    w = o;
+            if (w >= 0) {
+                const int i = base + w;
+                int32_t uw[Cols<RT>::N];
+                load_units_smem<RT>(sp.units + (size_t)i * R, uw, R);
+                take_winner<RT, G>(c, d.job_begin + (i >> c.log2_k), i & (K - 1), uw, sp.vals[i], 0, false, 0.0);
+            }
+        }
+        const int jstart = base & ~(K - 1);
+        const int64_t job = d.job_begin + (base >> c.log2_k);
+        const uint32_t amask = __ballot_sync(FULL, valid && amb && base == jstart);
+        if (amask)
+            resolve_row<RT, G>(c, lane, amask, false, sp.units, sp.vals, sp.grp, jstart, jstart + K, thr, job, 0);
+    }
+}
+
 // Per-job running state of the general (CSR) path: smallest screen value with its index, and the
 // smallest value of every other option. Commutative and associative (ties keep the lower index).
 struct Best {
@@ -811,7 +905,9 @@ __global__ void __launch_bounds__(kWarpsPerCta * 32, UNI ? kMinCtasPerSm : kMinC
             enter_scenario<RT, G>(c, d.scenario, p32s, lane);
         if (!c.sp.skip) {
             const StagePtrs ptrs = stage_ptrs(d, wsm + sidx * SL.bytes, SL, c.R);
-            if (UNI)
+            if (UNI && c.uniform_k >= 4)
+                process_tile_uniform4<RT, G>(c, d, ptrs, lane);
+            else if (UNI)
                 process_tile_uniform<RT, G>(c, d, ptrs, lane);
             else
                 process_tile_general<RT, G>(c, d, ptrs, big_first, big_carry, lane);
