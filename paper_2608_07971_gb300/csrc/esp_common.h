@@ -11,12 +11,31 @@
 
 namespace esp {
 
+// Tuning knobs (compile-time; the defaults are the measured best on GB300).
+#ifndef ESP_STAGES
+#define ESP_STAGES 2
+#endif
+#ifndef ESP_PREFETCH_TILES
+#define ESP_PREFETCH_TILES 0
+#endif
+#ifndef ESP_UNIFORM4_TILE
+#define ESP_UNIFORM4_TILE 128
+#endif
+#ifndef ESP_STAGE_DATA_BYTES
+#define ESP_STAGE_DATA_BYTES 8192
+#endif
+#ifndef ESP_MIN_CTAS_UNIFORM
+#define ESP_MIN_CTAS_UNIFORM 4
+#endif
+
 constexpr int kMaxR = 16;            // stored resource columns per option
 constexpr int kWarpsPerCta = 4;      // warps of a CTA; each warp owns its own stage ring
-constexpr int kStages = 2;           // TMA stages per warp
-constexpr int kMinCtasPerSm = 4;     // register budget of the uniform-K evaluation kernel: 4 CTAs (16 warps) per SM
+constexpr int kStages = ESP_STAGES;  // TMA stages per warp
+constexpr int kPrefetchTiles = ESP_PREFETCH_TILES;  // L2 prefetch distance, in tiles of the warp
+constexpr int kUniform4Tile = ESP_UNIFORM4_TILE;    // tile of the 4-options-per-lane path (0: largest)
+constexpr int kMinCtasPerSm = ESP_MIN_CTAS_UNIFORM; // register budget of the uniform-K evaluation kernel
 constexpr int kMinCtasPerSmGeneral = 4;  // the general kernel: 4 CTAs (16 warps) per SM
-constexpr int kStageDataBytes = 8192;// option bytes (units + values [+ group]) one stage aims at
+constexpr int kStageDataBytes = ESP_STAGE_DATA_BYTES;  // option bytes (units + values [+ group]) of a full stage
 
 // Tile flags. A tile is a run of whole jobs of one scenario whose options are contiguous, or one
 // chunk of a job with more options than a tile holds ("big" job).
@@ -50,8 +69,8 @@ ESP_HD int tile_options(int R, bool grouped)
 ESP_HD int tile_options_for(int R, bool grouped, long long max_k, bool uniform4)
 {
     const int cap = tile_options(R, grouped);
-    if (uniform4)   // uniform jobs of 4..32 options: the largest tile (amortises per-tile work)
-        return cap;
+    if (uniform4)   // uniform jobs of 4..32 options: a fixed tile (the largest by default)
+        return (kUniform4Tile > 0 && kUniform4Tile < cap) ? kUniform4Tile : cap;
     long long t = (max_k + 31) & ~31LL;
     if (t < 128)
         t = 128;

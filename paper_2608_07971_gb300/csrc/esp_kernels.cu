@@ -83,6 +83,12 @@ __device__ __forceinline__ void bulk_g2s(uint32_t dst, const void *src, uint32_t
         : "memory");
 }
 
+// Hint: bring [src, src + bytes) into L2 (16-byte aligned address and size).
+__device__ __forceinline__ void prefetch_l2(const void *src, uint32_t bytes)
+{
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src), "r"(bytes) : "memory");
+}
+
 __device__ __forceinline__ void fence_proxy_async()
 {
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -787,6 +793,19 @@ __device__ void process_tile_general(WarpCtx<RT, G> &c, const TileDesc &d, const
     }
 }
 
+// Asks L2 for the option bytes of tile d (lane 0 only), a few tiles before the stage copy of the
+// same bytes is issued: the DRAM latency is then hidden by L2 rather than by shared memory.
+__device__ __forceinline__ void prefetch_tile(const DevTable &t, const TileDesc &d)
+{
+    const int R = t.R;
+    const int64_t ub = d.opt_begin * R * 4, ue = (d.opt_begin + d.n_opt) * R * 4;
+    const int64_t ulo = ub & ~int64_t(15), uhi = (ue + 15) & ~int64_t(15);
+    const int64_t vb = d.opt_begin * 8, ve = (d.opt_begin + d.n_opt) * 8;
+    const int64_t vlo = vb & ~int64_t(15), vhi = (ve + 15) & ~int64_t(15);
+    prefetch_l2(reinterpret_cast<const unsigned char *>(t.units) + ulo, (uint32_t)(uhi - ulo));
+    prefetch_l2(reinterpret_cast<const unsigned char *>(t.values) + vlo, (uint32_t)(vhi - vlo));
+}
+
 // Issues the bulk copies of tile d into a stage; lane 0 only. Uniform tables need no job offsets.
 __device__ __forceinline__ void issue_tile(const DevTable &t, const TileDesc &d, unsigned char *stage,
                                            const StageLayout &SL, uint32_t bar, bool need_offsets)
@@ -882,6 +901,9 @@ __global__ void __launch_bounds__(kWarpsPerCta * 32, UNI ? kMinCtasPerSm : kMinC
         }
         ++issued;
     }
+    if (lane == 0)
+        for (int k = issued; k < k_end && k < k_begin + kPrefetchTiles; ++k)
+            prefetch_tile(t, pl.tiles[k]);
     int64_t big_first = 0;
     Best big_carry = best_none();
     int failed_at = -1;
@@ -891,6 +913,8 @@ __global__ void __launch_bounds__(kWarpsPerCta * 32, UNI ? kMinCtasPerSm : kMinC
             if (lane == 0) {
                 const int sidx = (issued - k_begin) % kStages;
                 issue_tile(t, pl.tiles[issued], wsm + sidx * SL.bytes, SL, bar0 + 8 * sidx, need_offsets);
+                if (kPrefetchTiles > 0 && k + kPrefetchTiles < k_end)
+                    prefetch_tile(t, pl.tiles[k + kPrefetchTiles]);
             }
             ++issued;
         }
