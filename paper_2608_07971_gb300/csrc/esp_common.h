@@ -25,7 +25,7 @@ namespace esp {
 #define ESP_STAGE_DATA_BYTES 8192
 #endif
 #ifndef ESP_MIN_CTAS_UNIFORM
-#define ESP_MIN_CTAS_UNIFORM 4
+#define ESP_MIN_CTAS_UNIFORM 5
 #endif
 
 constexpr int kMaxR = 16;            // stored resource columns per option
@@ -96,10 +96,10 @@ ESP_HD StageLayout stage_layout(int tile_opt, int R, bool grouped)
     return L;
 }
 
-// Per-warp shared memory: kStages stages, the fp32 screen values of the current tile, the fp32
-// prices of the current scenario (grouped tables) and the stage barriers.
+// Per-warp shared memory: kStages stages with their tile descriptors, the fp32 prices of the
+// current scenario (grouped tables) and the stage barriers.
 struct WarpSmem {
-    int stage_bytes, qbuf, p32, bars, bytes;
+    int stage_bytes, descs, p32, bars, bytes;
 };
 
 ESP_HD WarpSmem warp_smem(int tile_opt, int R, bool grouped, int P)
@@ -107,8 +107,8 @@ ESP_HD WarpSmem warp_smem(int tile_opt, int R, bool grouped, int P)
     WarpSmem W;
     StageLayout L = stage_layout(tile_opt, R, grouped);
     W.stage_bytes = L.bytes;
-    W.qbuf = kStages * L.bytes;
-    W.p32 = W.qbuf + round16(tile_opt * 4);
+    W.descs = kStages * L.bytes;          // the descriptor of the tile in each stage
+    W.p32 = W.descs + 32 * kStages;
     W.bars = W.p32 + (grouped ? round16(P * 4) : 0);
     W.bytes = W.bars + 16 * kStages;
     return W;

@@ -140,9 +140,11 @@ __device__ __forceinline__ float f32_of_f64(double v)
 {
     const uint32_t hi = (uint32_t)__double2hiint(v);
     const uint32_t lo = (uint32_t)__double2loint(v);
-    const uint32_t ex = (hi >> 20) & 0x7ffu;
-    const uint32_t bits = (hi & 0x80000000u) | ((ex - 896u) << 23) | ((hi & 0xfffffu) << 3) | (lo >> 29);
-    return (ex >= 923u) ? __uint_as_float(bits) : 0.0f;
+    // rebase the exponent (1023 -> 127); the sign bit is untouched for |v| >= 2^-127
+    const uint32_t t = hi - (896u << 20);
+    // 8 exponent and 23 mantissa bits; bit 31 comes out 0 because the rebased exponent is < 256
+    const uint32_t bits = __funnelshift_l(lo, t, 3) | (hi & 0x80000000u);
+    return ((hi << 1) >= (923u << 21)) ? __uint_as_float(bits) : 0.0f;
 }
 
 // Exact fp32 value of a unit count: 2^23 + u is exact in fp32 for 0 <= u < 2^23, so one OR and one
@@ -892,15 +894,24 @@ __global__ void __launch_bounds__(kWarpsPerCta * 32, UNI ? kMinCtasPerSm : kMinC
     }
     __syncwarp();
 
-    // prologue: the first kStages-1 tiles in flight
+    // prologue: the first kStages-1 tiles in flight. Lane 0 owns the descriptor stream: it reads
+    // each descriptor one tile before issuing it and leaves a copy beside the stage for the warp.
+    TileDesc *descs = reinterpret_cast<TileDesc *>(wsm + WS.descs);
     int issued = k_begin;
+    TileDesc dnext;
+    if (lane == 0)
+        dnext = pl.tiles[issued];
     while (issued < k_end && issued < k_begin + kStages - 1) {
         if (lane == 0) {
             const int sidx = (issued - k_begin) % kStages;
-            issue_tile(t, pl.tiles[issued], wsm + sidx * SL.bytes, SL, bar0 + 8 * sidx, need_offsets);
+            descs[sidx] = dnext;
+            issue_tile(t, dnext, wsm + sidx * SL.bytes, SL, bar0 + 8 * sidx, need_offsets);
+            if (issued + 1 < k_end)
+                dnext = pl.tiles[issued + 1];
         }
         ++issued;
     }
+    __syncwarp();
     if (lane == 0)
         for (int k = issued; k < k_end && k < k_begin + kPrefetchTiles; ++k)
             prefetch_tile(t, pl.tiles[k]);
@@ -909,16 +920,18 @@ __global__ void __launch_bounds__(kWarpsPerCta * 32, UNI ? kMinCtasPerSm : kMinC
     int failed_at = -1;
     for (int k = k_begin; k < k_end; ++k) {
         if (issued < k_end) {   // refill the stage the previous tile used
-            __syncwarp();
             if (lane == 0) {
                 const int sidx = (issued - k_begin) % kStages;
-                issue_tile(t, pl.tiles[issued], wsm + sidx * SL.bytes, SL, bar0 + 8 * sidx, need_offsets);
+                descs[sidx] = dnext;
+                issue_tile(t, dnext, wsm + sidx * SL.bytes, SL, bar0 + 8 * sidx, need_offsets);
+                if (issued + 1 < k_end)
+                    dnext = pl.tiles[issued + 1];
                 if (kPrefetchTiles > 0 && k + kPrefetchTiles < k_end)
                     prefetch_tile(t, pl.tiles[k + kPrefetchTiles]);
             }
             ++issued;
         }
-        const TileDesc d = pl.tiles[k];
+        const TileDesc d = descs[(k - k_begin) % kStages];
         const int sidx = (k - k_begin) % kStages;
         const uint32_t parity = (uint32_t)(((k - k_begin) / kStages) & 1);
         if (!wait_stage(bar0 + 8 * sidx, parity, st.err)) {
