@@ -154,6 +154,27 @@ esp_status esp_get_demand(esp_ctx *ctx, int64_t *out);           /* S*P demand o
 esp_status esp_evaluate(esp_ctx *ctx, const double *lambda, int32_t mode, uint32_t flags, int32_t *sel,
                         int64_t *demand, double *min_score);
 
+/* Best response at caller prices that allocates nothing (no cudaMalloc, no cudaFree, no host or
+ * device allocation by the library). The paper has no counterpart: this exists for callers that
+ * cannot allocate device memory where they need the answer, e.g. code running while another
+ * framework's caching allocator owns the device, or a scheduler loop that must not stall on the
+ * device synchronisation that cudaMalloc / cudaFree imply and works from memory reserved up front.
+ * Every pointer is a device pointer owned by the caller: the table (job_offsets S*J+1 int64,
+ * units n_opt*R int32 >= 0, values n_opt fp64 finite; every job non-empty; R <= 16, no groups),
+ * capacity S*R int64 > 0, lambda S*R (>= 0, finite, in the units of `mode`), and the outputs sel
+ * S*J, demand S*R (overwritten; int64), min_score S*J (may be NULL). The inputs are not validated.
+ * The per-unit prices go to one fixed scratch array of 65536 fp64 in the library's device memory,
+ * so S*R must not exceed 65536 (ESP_ERR_INVALID_ARG otherwise). The array exists once per GPU, is
+ * shared by every call and keeps the last call's contents; calls that may overlap on the GPU (on
+ * different streams, or from different threads) race on it and must be serialised by the caller.
+ * The first call on a device looks up the array's device address (once per device, under a lock);
+ * make that first call before any stream capture. Work is queued on `cuda_stream` (NULL: the legacy
+ * default stream); the call returns without waiting. Results equal esp_evaluate's.
+ * Errors: ESP_ERR_INVALID_ARG, ESP_ERR_UNSUPPORTED (device index >= 64), ESP_ERR_CUDA. */
+esp_status esp_evaluate_noalloc(int32_t S, int32_t J, int32_t R, const int64_t *job_offsets, const int32_t *units,
+                                const double *values, const int64_t *capacity, const double *lambda, int32_t mode,
+                                int32_t *sel, int64_t *demand, double *min_score, void *cuda_stream);
+
 /* Number of kernel launches the last esp_solve / esp_solve_async issued. */
 esp_status esp_last_launch_count(esp_ctx *ctx, int64_t *out);
 

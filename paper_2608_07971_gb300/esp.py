@@ -27,7 +27,7 @@ EXPORTED = [
     "esp_create", "esp_set_stream", "esp_load_options", "esp_load_options_device", "esp_solve",
     "esp_solve_async", "esp_get_result", "esp_get_prices", "esp_get_selection", "esp_get_demand",
     "esp_evaluate", "esp_last_launch_count", "esp_pass_times", "esp_status_string", "esp_destroy",
-    "esp_debug_tile_options", "esp_debug_plan",
+    "esp_debug_tile_options", "esp_debug_plan", "esp_evaluate_noalloc",
 ]
 
 
@@ -84,6 +84,7 @@ def load_library(path: Optional[str] = None):
         "esp_destroy": ([vp], None),
         "esp_debug_tile_options": ([i32, i32], i32),
         "esp_debug_plan": ([vp, i32, i32, i32, i32, vp, i32, vp, i32, ctypes.POINTER(i32), ctypes.POINTER(i32)], st),
+        "esp_evaluate_noalloc": ([i32, i32, i32, vp, vp, vp, vp, vp, i32, vp, vp, vp, vp], st),
     }
     for name, (args, res) in sig.items():
         fn = getattr(lib, name)
@@ -178,6 +179,14 @@ def esp_pass_times(ctx: int, reset: bool = True):
     _check(load_library().esp_pass_times(ctx, ctypes.byref(ms), ctypes.byref(n), 1 if reset else 0),
            "esp_pass_times")
     return ms.value, n.value
+
+
+def esp_evaluate_noalloc(S, J, R, job_offsets, units, values, capacity, lam, mode, sel, demand, min_score,
+                         stream: Optional[int] = None) -> None:
+    """Best response that allocates nothing (device tensors in and out; see include/esp.h)."""
+    _check(load_library().esp_evaluate_noalloc(S, J, R, _p(job_offsets), _p(units), _p(values), _p(capacity),
+                                               _p(lam), mode, _p(sel), _p(demand), _p(min_score), stream),
+           "esp_evaluate_noalloc")
 
 
 def esp_destroy(ctx: int) -> None:
