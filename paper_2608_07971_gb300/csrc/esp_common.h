@@ -27,9 +27,12 @@ namespace esp {
 #ifndef ESP_MIN_CTAS_UNIFORM
 #define ESP_MIN_CTAS_UNIFORM 5
 #endif
+#ifndef ESP_WARPS_PER_CTA
+#define ESP_WARPS_PER_CTA 4
+#endif
 
 constexpr int kMaxR = 16;            // stored resource columns per option
-constexpr int kWarpsPerCta = 4;      // warps of a CTA; each warp owns its own stage ring
+constexpr int kWarpsPerCta = ESP_WARPS_PER_CTA;  // warps of a CTA; each warp owns its own stage ring
 constexpr int kStages = ESP_STAGES;  // TMA stages per warp
 constexpr int kPrefetchTiles = ESP_PREFETCH_TILES;  // L2 prefetch distance, in tiles of the warp
 constexpr int kUniform4Tile = ESP_UNIFORM4_TILE;    // tile of the 4-options-per-lane path (0: largest)

@@ -897,17 +897,23 @@ __global__ void __launch_bounds__(kWarpsPerCta * 32, UNI ? kMinCtasPerSm : kMinC
     // prologue: the first kStages-1 tiles in flight. Lane 0 owns the descriptor stream: it reads
     // each descriptor one tile before issuing it and leaves a copy beside the stage for the warp.
     TileDesc *descs = reinterpret_cast<TileDesc *>(wsm + WS.descs);
+    const int4 *tiles4 = reinterpret_cast<const int4 *>(pl.tiles);   // a descriptor is two int4
     int issued = k_begin;
-    TileDesc dnext;
-    if (lane == 0)
-        dnext = pl.tiles[issued];
+    int4 dn0 = make_int4(0, 0, 0, 0), dn1 = dn0;
+    if (lane == 0) {
+        dn0 = __ldg(tiles4 + 2 * issued);
+        dn1 = __ldg(tiles4 + 2 * issued + 1);
+    }
     while (issued < k_end && issued < k_begin + kStages - 1) {
         if (lane == 0) {
             const int sidx = (issued - k_begin) % kStages;
-            descs[sidx] = dnext;
-            issue_tile(t, dnext, wsm + sidx * SL.bytes, SL, bar0 + 8 * sidx, need_offsets);
-            if (issued + 1 < k_end)
-                dnext = pl.tiles[issued + 1];
+            reinterpret_cast<int4 *>(descs + sidx)[0] = dn0;
+            reinterpret_cast<int4 *>(descs + sidx)[1] = dn1;
+            issue_tile(t, descs[sidx], wsm + sidx * SL.bytes, SL, bar0 + 8 * sidx, need_offsets);
+            if (issued + 1 < k_end) {
+                dn0 = __ldg(tiles4 + 2 * (issued + 1));
+                dn1 = __ldg(tiles4 + 2 * (issued + 1) + 1);
+            }
         }
         ++issued;
     }
@@ -922,10 +928,13 @@ __global__ void __launch_bounds__(kWarpsPerCta * 32, UNI ? kMinCtasPerSm : kMinC
         if (issued < k_end) {   // refill the stage the previous tile used
             if (lane == 0) {
                 const int sidx = (issued - k_begin) % kStages;
-                descs[sidx] = dnext;
-                issue_tile(t, dnext, wsm + sidx * SL.bytes, SL, bar0 + 8 * sidx, need_offsets);
-                if (issued + 1 < k_end)
-                    dnext = pl.tiles[issued + 1];
+                reinterpret_cast<int4 *>(descs + sidx)[0] = dn0;
+                reinterpret_cast<int4 *>(descs + sidx)[1] = dn1;
+                issue_tile(t, descs[sidx], wsm + sidx * SL.bytes, SL, bar0 + 8 * sidx, need_offsets);
+                if (issued + 1 < k_end) {
+                    dn0 = __ldg(tiles4 + 2 * (issued + 1));
+                    dn1 = __ldg(tiles4 + 2 * (issued + 1) + 1);
+                }
                 if (kPrefetchTiles > 0 && k + kPrefetchTiles < k_end)
                     prefetch_tile(t, pl.tiles[k + kPrefetchTiles]);
             }
