@@ -943,7 +943,7 @@ __global__ void __launch_bounds__(kWarpsPerCta * 32, UNI ? kMinCtasPerSm : kMinC
         const TileDesc d = descs[(k - k_begin) % kStages];
         const int sidx = (k - k_begin) % kStages;
         const uint32_t parity = (uint32_t)(((k - k_begin) / kStages) & 1);
-        if (!wait_stage(bar0 + 8 * sidx, parity, st.err)) {
+        if (!__all_sync(FULL, wait_stage(bar0 + 8 * sidx, parity, st.err))) {   // uniform decision
             failed_at = k;
             break;
         }
