@@ -30,6 +30,12 @@ namespace esp {
 #ifndef ESP_WARPS_PER_CTA
 #define ESP_WARPS_PER_CTA 4
 #endif
+#ifndef ESP_V32_HW
+#define ESP_V32_HW 0          // 1: fp64 -> fp32 of values by the conversion instruction (round to nearest)
+#endif
+#ifndef ESP_I2F_COLS
+#define ESP_I2F_COLS 0        // unit columns r < ESP_I2F_COLS use the int-to-float instruction
+#endif
 
 constexpr int kMaxR = 16;            // stored resource columns per option
 constexpr int kWarpsPerCta = ESP_WARPS_PER_CTA;  // warps of a CTA; each warp owns its own stage ring

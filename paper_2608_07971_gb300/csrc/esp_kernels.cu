@@ -154,17 +154,29 @@ __device__ __forceinline__ float f32_of_units(int32_t u, bool small)
     return small ? (__uint_as_float(0x4b000000u | (uint32_t)u) - 8388608.0f) : __int2float_rn(u);
 }
 
+// The fp32 value used by the screen: truncated by integer ops, or (ESP_V32_HW) rounded by the
+// conversion instruction; both are within 2^-23 relative (or 2^-100 absolute) of v in range.
+__device__ __forceinline__ float screen_value(double v)
+{
+#if ESP_V32_HW
+    return __double2float_rn(v);
+#else
+    return f32_of_f64(v);
+#endif
+}
+
 template <int RT, bool G>
 __device__ __forceinline__ float screen_score(const int32_t *u, double v, int g, const ScenarioPrices &sp, int R,
                                               int rg)
 {
-    float q = -f32_of_f64(v);
+    float q = -screen_value(v);
 #pragma unroll
     for (int r = 0; r < Cols<RT>::N; ++r) {
         if (RT == 0 && r >= R)
             break;
         const float price = (G && r >= rg) ? sp.p32s[rg + (R - rg) * g + (r - rg)] : sp.pf[r];
-        q = __fmaf_rn(price, f32_of_units(u[r], sp.small_units), q);
+        const float uf = (r < ESP_I2F_COLS) ? __int2float_rn(u[r]) : f32_of_units(u[r], sp.small_units);
+        q = __fmaf_rn(price, uf, q);
     }
     return q;
 }
