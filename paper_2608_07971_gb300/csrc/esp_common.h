@@ -34,7 +34,7 @@ namespace esp {
 #define ESP_V32_HW 0          // 1: fp64 -> fp32 of values by the conversion instruction (round to nearest)
 #endif
 #ifndef ESP_I2F_COLS
-#define ESP_I2F_COLS 0        // unit columns r < ESP_I2F_COLS use the int-to-float instruction
+#define ESP_I2F_COLS 16       // unit columns r < ESP_I2F_COLS use the int-to-float instruction
 #endif
 
 constexpr int kMaxR = 16;            // stored resource columns per option

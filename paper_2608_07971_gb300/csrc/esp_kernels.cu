@@ -62,15 +62,17 @@ __device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t byt
     asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
 }
 
-__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity)
+// Waits on the phase of the given parity; the thread may sleep until the phase completes or about
+// suspend_ns elapse, whichever is first.
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity, uint32_t suspend_ns)
 {
     uint32_t done;
     asm volatile(
         "{\n\t.reg .pred p;\n\t"
-        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
         "selp.u32 %0, 1, 0, p;\n\t}"
         : "=r"(done)
-        : "r"(bar), "r"(parity)
+        : "r"(bar), "r"(parity), "r"(suspend_ns)
         : "memory");
     return done != 0;
 }
@@ -94,16 +96,14 @@ __device__ __forceinline__ void fence_proxy_async()
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
-// Bounded wait on a stage barrier: gives up after ~2^26 polls (seconds), flags a timeout and
-// returns false so the kernel can finish instead of hanging.
+// Bounded wait on a stage barrier: sleeps until the copy lands (each attempt sleeps at most ~1 ms)
+// and gives up after 4096 attempts (seconds), flags a timeout and returns false so the kernel can
+// finish instead of hanging.
 __device__ __forceinline__ bool wait_stage(uint32_t bar, uint32_t parity, unsigned int *err)
 {
-    for (uint32_t it = 0; it < (1u << 26); ++it) {
-        if (mbar_try_wait(bar, parity))
+    for (uint32_t it = 0; it < 4096u; ++it)
+        if (mbar_try_wait(bar, parity, 1000000u))
             return true;
-        if (it > 64)
-            __nanosleep(32);
-    }
     atomicOr(err, DEV_ERR_TIMEOUT);
     return false;
 }
@@ -861,7 +861,7 @@ __device__ __forceinline__ void issue_tile(const DevTable &t, const TileDesc &d,
 // One evaluation pass over every tile: a best response of every job of every (non-stopped) scenario.
 // UNI selects the uniform-K row reduction (tables whose jobs all have the same power-of-two size up
 // to 32, never grouped); otherwise the general segmented path runs.
-template <int RT, bool G, bool UNI>
+template <int RT, bool G, bool UNI, bool PLAIN>
 __global__ void __launch_bounds__(kWarpsPerCta * 32, UNI ? kMinCtasPerSm : kMinCtasPerSmGeneral) k_pass(DevTable t, DevState st, DevPlan pl,
                                                                           SolveArgs a, int round, int kind)
 {
@@ -886,9 +886,10 @@ __global__ void __launch_bounds__(kWarpsPerCta * 32, UNI ? kMinCtasPerSm : kMinC
     c.st = st;
     c.R = RT ? RT : t.R;
     c.rg = t.r_global;
-    c.kind = kind;
-    c.want_min = (kind == PASS_FINAL) || (st.dual_trace != nullptr);
-    c.want_hash = (kind == PASS_ROUND) && (st.hash_trace != nullptr);
+    // PLAIN: a round pass without traces (the hot case), with every per-pass choice a constant
+    c.kind = PLAIN ? (int)PASS_ROUND : kind;
+    c.want_min = PLAIN ? false : ((kind == PASS_FINAL) || (st.dual_trace != nullptr));
+    c.want_hash = PLAIN ? false : ((kind == PASS_ROUND) && (st.hash_trace != nullptr));
     c.uniform_k = pl.uniform_k;
     c.log2_k = pl.uniform_k > 0 ? __ffs(pl.uniform_k) - 1 : 0;
     c.s = -1;
@@ -1308,10 +1309,47 @@ __global__ void k_validate_offsets(DevTable t, unsigned int *flags)
         atomicOr(flags, bad);
 }
 
+// Both instantiations (plain round pass and the general one) of a table shape.
 template <int RT, bool G, bool UNI>
-void *pass_kernel_ptr()
+struct PassKernels {
+    static const void *plain() { return reinterpret_cast<const void *>(&k_pass<RT, G, UNI, true>); }
+    static const void *other() { return reinterpret_cast<const void *>(&k_pass<RT, G, UNI, false>); }
+    static void launch(bool plain, int grid, int smem, cudaStream_t stream, const DevTable &t, const DevState &st,
+                       const DevPlan &pl, const SolveArgs &a, int round, int kind)
+    {
+        if (plain)
+            k_pass<RT, G, UNI, true><<<grid, kWarpsPerCta * 32, smem, stream>>>(t, st, pl, a, round, kind);
+        else
+            k_pass<RT, G, UNI, false><<<grid, kWarpsPerCta * 32, smem, stream>>>(t, st, pl, a, round, kind);
+    }
+};
+
+// Calls f.template operator()<RT, G, UNI>() for the instantiation that serves this table shape.
+template <typename F>
+auto dispatch_shape(int R, bool grouped, bool uni, F &&f)
 {
-    return reinterpret_cast<void *>(&k_pass<RT, G, UNI>);
+    if (grouped) {
+        switch (R) {
+        case 4: return f(PassKernels<4, true, false>());
+        case 6: return f(PassKernels<6, true, false>());
+        case 8: return f(PassKernels<8, true, false>());
+        default: return f(PassKernels<0, true, false>());
+        }
+    }
+    if (uni) {
+        switch (R) {
+        case 4: return f(PassKernels<4, false, true>());
+        case 6: return f(PassKernels<6, false, true>());
+        case 8: return f(PassKernels<8, false, true>());
+        default: return f(PassKernels<0, false, true>());
+        }
+    }
+    switch (R) {
+    case 4: return f(PassKernels<4, false, false>());
+    case 6: return f(PassKernels<6, false, false>());
+    case 8: return f(PassKernels<8, false, false>());
+    default: return f(PassKernels<0, false, false>());
+    }
 }
 
 }  // namespace
@@ -1321,42 +1359,22 @@ int pass_smem_bytes(int R, bool grouped, int P, int tile_opt)
     return kWarpsPerCta * warp_smem(tile_opt, R, grouped, P).bytes;
 }
 
-static const void *pass_kernel_for(int R, bool grouped, bool uni)
-{
-    if (grouped) {
-        switch (R) {
-        case 4: return pass_kernel_ptr<4, true, false>();
-        case 6: return pass_kernel_ptr<6, true, false>();
-        case 8: return pass_kernel_ptr<8, true, false>();
-        default: return pass_kernel_ptr<0, true, false>();
-        }
-    }
-    if (uni) {
-        switch (R) {
-        case 4: return pass_kernel_ptr<4, false, true>();
-        case 6: return pass_kernel_ptr<6, false, true>();
-        case 8: return pass_kernel_ptr<8, false, true>();
-        default: return pass_kernel_ptr<0, false, true>();
-        }
-    }
-    switch (R) {
-    case 4: return pass_kernel_ptr<4, false, false>();
-    case 6: return pass_kernel_ptr<6, false, false>();
-    case 8: return pass_kernel_ptr<8, false, false>();
-    default: return pass_kernel_ptr<0, false, false>();
-    }
-}
-
 int pass_ctas_per_sm(int R, bool grouped, bool uniform, int P, int tile_opt)
 {
-    const void *fn = pass_kernel_for(R, grouped, uniform && !grouped);
     const int smem = pass_smem_bytes(R, grouped, P, tile_opt);
-    if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess)
-        return 0;
-    int n = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, fn, kWarpsPerCta * 32, smem) != cudaSuccess)
-        return 0;
-    return n;
+    return dispatch_shape(R, grouped, uniform && !grouped, [&](auto k) -> int {
+        using K = decltype(k);
+        if (cudaFuncSetAttribute(K::plain(), cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess ||
+            cudaFuncSetAttribute(K::other(), cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess)
+            return 0;
+        int n = 0;
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, K::plain(), kWarpsPerCta * 32, smem) != cudaSuccess)
+            return 0;
+        int m = 0;
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&m, K::other(), kWarpsPerCta * 32, smem) != cudaSuccess)
+            return 0;
+        return n < m ? n : m;
+    });
 }
 
 cudaError_t launch_validate(const DevTable &t, double *vmax, int32_t *umax, unsigned int *flags, cudaStream_t stream)
@@ -1385,31 +1403,11 @@ cudaError_t launch_pass(const DevTable &t, const DevState &st, const DevPlan &pl
 {
     const bool grouped = t.group != nullptr;
     const int smem = pass_smem_bytes(t.R, grouped, t.P, pl.tile_opt);
-    const dim3 block(kWarpsPerCta * 32);
-#define ESP_LAUNCH_PASS(RT_, G_, U_) k_pass<RT_, G_, U_><<<grid, block, smem, stream>>>(t, st, pl, a, round, kind)
-    if (grouped) {
-        switch (t.R) {
-        case 4: ESP_LAUNCH_PASS(4, true, false); break;
-        case 6: ESP_LAUNCH_PASS(6, true, false); break;
-        case 8: ESP_LAUNCH_PASS(8, true, false); break;
-        default: ESP_LAUNCH_PASS(0, true, false); break;
-        }
-    } else if (pl.uniform_k > 0) {
-        switch (t.R) {
-        case 4: ESP_LAUNCH_PASS(4, false, true); break;
-        case 6: ESP_LAUNCH_PASS(6, false, true); break;
-        case 8: ESP_LAUNCH_PASS(8, false, true); break;
-        default: ESP_LAUNCH_PASS(0, false, true); break;
-        }
-    } else {
-        switch (t.R) {
-        case 4: ESP_LAUNCH_PASS(4, false, false); break;
-        case 6: ESP_LAUNCH_PASS(6, false, false); break;
-        case 8: ESP_LAUNCH_PASS(8, false, false); break;
-        default: ESP_LAUNCH_PASS(0, false, false); break;
-        }
-    }
-#undef ESP_LAUNCH_PASS
+    const bool plain = kind == PASS_ROUND && st.hash_trace == nullptr && st.dual_trace == nullptr;
+    dispatch_shape(t.R, grouped, pl.uniform_k > 0, [&](auto k) -> int {
+        decltype(k)::launch(plain, grid, smem, stream, t, st, pl, a, round, kind);
+        return 0;
+    });
     return cudaGetLastError();
 }
 
