@@ -310,6 +310,7 @@ def run_ours(args):
     assert np.all(res["rounds_run"] == T) or st != 0, "unexpected early stop"
 
     pass_ms, n_pass = esp.esp_pass_times(ctx, reset=True)
+    n_res, n_marked = esp.esp_debug_stats(ctx, reset=True)
     if args.graph:   # roofline from a second, pass-timed run of the same steps
         prm_ev = solver.params(w.eta0, T, mode=w.mode, step=w.step, flags=esp.ESP_FLAG_PASS_EVENTS)
         for _ in range(args.steps):
@@ -340,7 +341,9 @@ def run_ours(args):
                 "frac": (achieved / peak) if achieved else None, "traffic": traffic,
                 "peak_kind": f"{peak_kind} hbm_gbs (copy)",
                 "bytes_per_launch": bytes_pass, "avg_launch_ms": pass_avg_ms, "launches_timed": n_pass,
-                "share_of_step": (pass_ms / args.steps) / ms if ms else None}
+                "share_of_step": (pass_ms / args.steps) / ms if ms else None,
+                "exact_resolutions_per_pass": n_res / max(1, (args.warmup + args.steps) * (T + 1)),
+                "duplicates_marked": n_marked}
 
     # end to end through the public API with host inputs
     e2e = None

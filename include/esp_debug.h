@@ -1,5 +1,6 @@
 /*
- * esp_debug.h - host-only helpers of the ESP solver library for tests. They run no GPU code.
+ * esp_debug.h - helpers of the ESP solver library for tests: the host tile planner (no GPU code)
+ * and counters of a context.
  */
 #ifndef ESP_DEBUG_H
 #define ESP_DEBUG_H
@@ -11,6 +12,12 @@
 #ifdef __cplusplus
 extern "C" {
 #endif
+
+/* Counters of a loaded context: *resolutions = jobs whose fp32 screen was ambiguous and that were
+ * resolved in fp64 since the last reset (all evaluation passes, including esp_evaluate), *marked =
+ * options marked at load as exact duplicates of an earlier option of their job. Waits for the
+ * context's stream; reset != 0 zeroes the resolution counter. */
+esp_status esp_debug_stats(esp_ctx *ctx, int64_t *resolutions, int64_t *marked, int32_t reset);
 
 /* Options per tile the evaluation pass uses for R stored columns (grouped != 0: a group column is
  * present). */

@@ -70,6 +70,7 @@ struct esp_ctx {
             *feasible = nullptr;
     unsigned int *err = nullptr;
     unsigned int *valflags = nullptr;
+    unsigned long long *stats = nullptr;  // [0] exact resolutions (since the last read), [1] marked duplicates
 
     // trace buffers (grown on demand, freed on destroy)
     DevArr<double> lt;
@@ -205,6 +206,7 @@ DevState dev_state(const esp_ctx *c)
     s.vmax = c->vmax;
     s.umax = c->umax;
     s.err = c->err;
+    s.stats = c->stats;
     s.lam_trace = nullptr;
     s.dem_trace = nullptr;
     s.hash_trace = nullptr;
@@ -303,6 +305,7 @@ esp_status load_common(esp_ctx *ctx, int32_t S, int32_t J, int32_t R, int32_t P,
     ALLOC(ctx->vmax, (size_t)S);
     ALLOC(ctx->umax, (size_t)S * R);
     ALLOC(ctx->valflags, 4);
+    ALLOC(ctx->stats, 2);
 
     const cudaMemcpyKind kind = device_src ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice;
     ESP_CUDA(cudaMemcpyAsync(ctx->units, units, (size_t)n_opt * R * sizeof(int32_t), kind, ctx->stream));
@@ -329,7 +332,7 @@ esp_status load_common(esp_ctx *ctx, int32_t S, int32_t J, int32_t R, int32_t P,
         if (x >= (1 << 23))
             ctx->small_units = 0;
     // duplicates are marked in the device copy only (validation has already read the units)
-    ESP_CUDA(launch_mark_duplicates(dev_table(ctx), ctx->units, ctx->stream));
+    ESP_CUDA(launch_mark_duplicates(dev_table(ctx), ctx->units, ctx->stats + 1, ctx->stream));
 
     // plan the evaluation pass
     int64_t max_k = 1, min_k = n_jobs ? INT64_MAX : 1;
@@ -867,6 +870,23 @@ void esp_destroy(esp_ctx *ctx)
     for (cudaEvent_t e : ctx->ev_pool)
         cudaEventDestroy(e);
     delete ctx;
+}
+
+esp_status esp_debug_stats(esp_ctx *ctx, int64_t *resolutions, int64_t *marked, int32_t reset)
+{
+    esp_status st = check_ctx(ctx);
+    if (st != ESP_OK)
+        return st;
+    if (!ctx->loaded || !resolutions || !marked)
+        return ESP_ERR_INVALID_ARG;
+    unsigned long long h[2] = {0, 0};
+    ESP_CUDA(cudaMemcpyAsync(h, ctx->stats, sizeof(h), cudaMemcpyDeviceToHost, ctx->stream));
+    ESP_CUDA(cudaStreamSynchronize(ctx->stream));
+    *resolutions = (int64_t)h[0];
+    *marked = (int64_t)h[1];
+    if (reset)
+        ESP_CUDA(cudaMemsetAsync(ctx->stats, 0, sizeof(unsigned long long), ctx->stream));
+    return ESP_OK;
 }
 
 int32_t esp_debug_tile_options(int32_t R, int32_t grouped)

@@ -484,6 +484,7 @@ __device__ __forceinline__ void resolve_row(WarpCtx<RT, G> &c, int lane, uint32_
         resolve_job<RT, G>(c, lane, !big, units_s, vals_s, grp_s, js, je, big ? big_first : 0, th, c.want_min,
                            s_w, has_s, li);
         if (lane == 0) {
+            atomicAdd(c.st.stats, 1ull);
             int32_t uw[Cols<RT>::N];
             double vw;
             int gw;
@@ -1016,7 +1017,8 @@ __device__ __forceinline__ bool same_option(const DevTable &t, int64_t a, int64_
     return true;
 }
 
-__global__ void __launch_bounds__(kDedupWarps * 32) k_mark_duplicates(DevTable t, int32_t *units)
+__global__ void __launch_bounds__(kDedupWarps * 32) k_mark_duplicates(DevTable t, int32_t *units,
+                                                                     unsigned long long *marked)
 {
     __shared__ uint64_t hs[kDedupWarps][kDedupMaxK];
     const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
@@ -1034,6 +1036,7 @@ __global__ void __launch_bounds__(kDedupWarps * 32) k_mark_duplicates(DevTable t
             for (int k2 = 0; k2 < k; ++k2) {
                 if (hs[wid][k2] == h && same_option(t, a + k, a + k2)) {
                     units[(a + k) * t.R] |= (int32_t)0x80000000;
+                    atomicAdd(marked, 1ull);
                     break;
                 }
             }
@@ -1411,7 +1414,7 @@ cudaError_t launch_pass(const DevTable &t, const DevState &st, const DevPlan &pl
     return cudaGetLastError();
 }
 
-cudaError_t launch_mark_duplicates(const DevTable &t, int32_t *units, cudaStream_t stream)
+cudaError_t launch_mark_duplicates(const DevTable &t, int32_t *units, unsigned long long *marked, cudaStream_t stream)
 {
     const int64_t n_jobs = (int64_t)t.S * t.J;
     if (n_jobs == 0)
@@ -1419,7 +1422,7 @@ cudaError_t launch_mark_duplicates(const DevTable &t, int32_t *units, cudaStream
     int64_t blocks = (n_jobs + kDedupWarps - 1) / kDedupWarps;
     if (blocks > 65536)
         blocks = 65536;
-    k_mark_duplicates<<<(int)blocks, kDedupWarps * 32, 0, stream>>>(t, units);
+    k_mark_duplicates<<<(int)blocks, kDedupWarps * 32, 0, stream>>>(t, units, marked);
     return cudaGetLastError();
 }
 

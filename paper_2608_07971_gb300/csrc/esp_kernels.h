@@ -41,6 +41,7 @@ struct DevState {
     const double *vmax;       // S   max |v| of the scenario (load time)
     const int32_t *umax;      // S*R max unit of each stored column in the scenario (load time)
     unsigned int *err;        // device error word (DEV_ERR_*)
+    unsigned long long *stats;  // [0] exact resolutions since the last reset, [1] duplicates marked at load
     double *lam_trace;        // S*(T+1)*P or nullptr
     long long *dem_trace;     // S*T*P or nullptr
     unsigned long long *hash_trace; // S*T or nullptr
@@ -75,7 +76,7 @@ cudaError_t launch_validate(const DevTable &t, double *vmax, int32_t *umax, unsi
                             cudaStream_t stream);
 // Marks every option that repeats an earlier option of its job (units, value and group equal) by
 // setting the sign bit of its column-0 unit in `units` (the device copy of t.units).
-cudaError_t launch_mark_duplicates(const DevTable &t, int32_t *units, cudaStream_t stream);
+cudaError_t launch_mark_duplicates(const DevTable &t, int32_t *units, unsigned long long *marked, cudaStream_t stream);
 
 cudaError_t launch_init(const DevTable &t, const DevState &st, const SolveArgs &a, const double *lambda0,
                         cudaStream_t stream);

@@ -27,7 +27,7 @@ EXPORTED = [
     "esp_create", "esp_set_stream", "esp_load_options", "esp_load_options_device", "esp_solve",
     "esp_solve_async", "esp_get_result", "esp_get_prices", "esp_get_selection", "esp_get_demand",
     "esp_evaluate", "esp_last_launch_count", "esp_pass_times", "esp_status_string", "esp_destroy",
-    "esp_debug_tile_options", "esp_debug_plan", "esp_evaluate_noalloc",
+    "esp_debug_tile_options", "esp_debug_plan", "esp_debug_stats", "esp_evaluate_noalloc",
 ]
 
 
@@ -83,6 +83,7 @@ def load_library(path: Optional[str] = None):
         "esp_status_string": ([st], ctypes.c_char_p),
         "esp_destroy": ([vp], None),
         "esp_debug_tile_options": ([i32, i32], i32),
+        "esp_debug_stats": ([vp, ctypes.POINTER(i64), ctypes.POINTER(i64), i32], st),
         "esp_debug_plan": ([vp, i32, i32, i32, i32, vp, i32, vp, i32, ctypes.POINTER(i32), ctypes.POINTER(i32)], st),
         "esp_evaluate_noalloc": ([i32, i32, i32, vp, vp, vp, vp, vp, i32, vp, vp, vp, vp], st),
     }
@@ -187,6 +188,14 @@ def esp_evaluate_noalloc(S, J, R, job_offsets, units, values, capacity, lam, mod
     _check(load_library().esp_evaluate_noalloc(S, J, R, _p(job_offsets), _p(units), _p(values), _p(capacity),
                                                _p(lam), mode, _p(sel), _p(demand), _p(min_score), stream),
            "esp_evaluate_noalloc")
+
+
+def esp_debug_stats(ctx: int, reset: bool = True):
+    """(exact resolutions since the last reset, duplicates marked at load)."""
+    r, m = ctypes.c_int64(), ctypes.c_int64()
+    _check(load_library().esp_debug_stats(ctx, ctypes.byref(r), ctypes.byref(m), 1 if reset else 0),
+           "esp_debug_stats")
+    return r.value, m.value
 
 
 def esp_destroy(ctx: int) -> None:

@@ -255,3 +255,22 @@ def test_invalid_tables_rejected():
     s.load(t)   # a good table still loads afterwards
     sol = s.solve(0.1, 5)
     assert sol.status == esp.ESP_OK
+
+
+def test_duplicate_marking_matches_numpy_count():
+    """Options equal (units and value bits) to an earlier option of their job are marked at load;
+    the count equals an independent per-job count of repeated rows."""
+    w = W.whatif_batch(scenarios=[0, 3], J=1024)
+    t = w.table
+    rows = np.concatenate([t.units.view(np.uint32).reshape(t.n_opt, t.R),
+                           t.values.view(np.uint32).reshape(t.n_opt, 2)], axis=1)
+    want = 0
+    for j in range(t.S * t.J):
+        a, b = t.job_off[j], t.job_off[j + 1]
+        want += (b - a) - len(np.unique(rows[a:b], axis=0))
+    s = esp.Solver(t)
+    res, marked = esp.esp_debug_stats(s.ctx)
+    assert marked == want and want > 0
+    s.solve(w.eta0, 5)
+    res, _ = esp.esp_debug_stats(s.ctx)
+    assert res <= 0.05 * t.S * t.J * 6          # few exact resolutions once duplicates are marked
