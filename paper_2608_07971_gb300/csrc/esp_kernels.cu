@@ -312,8 +312,27 @@ __device__ void enter_scenario(WarpCtx<RT, G> &c, int s, float *p32s_smem, int l
     }
 }
 
-// Records the winner of a job: demand, fingerprint, and the per-job outputs of the final pass.
-// u/v/g are the winner's data; s64 its exact reduced cost when already known.
+// The per-job outputs of a winner beyond its demand: fingerprint, final-pass selection and value,
+// and its exact reduced cost (computed here unless s64 is given).
+template <int RT, bool G>
+__device__ __forceinline__ void take_winner_extras(WarpCtx<RT, G> &c, int64_t job, int local, const int32_t *u,
+                                                   double v, int g, bool have_s64 = false, double s64 = 0.0)
+{
+    if (c.want_hash)
+        c.hacc += splitmix64_mix(((uint64_t)(uint32_t)(job - (int64_t)c.s * c.t.J) << 32) | (uint32_t)local);
+    if (c.kind == PASS_FINAL) {
+        c.st.sel[job] = local;
+        c.st.job_val[job] = v;
+    }
+    if (c.want_min) {
+        if (!have_s64)
+            s64 = exact_score<RT, G>(u, v, g, c.sp, c.R, c.rg);
+        c.st.job_min[job] = s64;
+    }
+}
+
+// Records the winner of a job: its demand (per-lane int64 sums; grouped columns straight to the
+// scenario's accumulator) and the outputs of take_winner_extras. u/v/g are the winner's data.
 template <int RT, bool G>
 __device__ __forceinline__ void take_winner(WarpCtx<RT, G> &c, int64_t job, int local, const int32_t *u, double v,
                                             int g, bool have_s64, double s64)
@@ -330,17 +349,7 @@ __device__ __forceinline__ void take_winner(WarpCtx<RT, G> &c, int64_t job, int 
             c.acc[r] += u[r];
         }
     }
-    if (c.want_hash)
-        c.hacc += splitmix64_mix(((uint64_t)(uint32_t)(job - (int64_t)c.s * c.t.J) << 32) | (uint32_t)local);
-    if (c.kind == PASS_FINAL) {
-        c.st.sel[job] = local;
-        c.st.job_val[job] = v;
-    }
-    if (c.want_min) {
-        if (!have_s64)
-            s64 = exact_score<RT, G>(u, v, g, c.sp, R, c.rg);
-        c.st.job_min[job] = s64;
-    }
+    take_winner_extras<RT, G>(c, job, local, u, v, g, have_s64, s64);
 }
 
 // Signed-integer key with the order of the doubles (no NaN occurs); -0.0 and +0.0 share key 0.
@@ -601,6 +610,10 @@ __device__ void process_tile_uniform4(WarpCtx<RT, G> &c, const TileDesc &d, cons
     const int n = d.n_opt;
     const int K = c.uniform_k;
     const int KL = K >> 2;                  // lanes per job
+    int32_t acc32[Cols<RT>::N];
+#pragma unroll
+    for (int r = 0; r < Cols<RT>::N; ++r)
+        acc32[r] = 0;
     for (int b = 0; b < n; b += 128) {
         const int base = b + 4 * lane;
         const bool valid = base < n;        // n is a multiple of K, hence of 4
@@ -630,18 +643,30 @@ __device__ void process_tile_uniform4(WarpCtx<RT, G> &c, const TileDesc &d, cons
         }
         const float thr = __fadd_ru(m1, c.sp.e2);
         const bool amb = c.sp.exact || !(m2 > thr);
-        if (valid && !amb) {
-            int w = -1;
+        // the winner of an unambiguous job is the unique option holding m1; every lane loads the units
+        // of its candidate and adds them under a mask (no divergent branch on the hot path)
+        int w = -1;
 #pragma unroll
-            for (int o = 3; o >= 0; --o)
-                if (q[o] == m1)
-                    w = o;
-            if (w >= 0) {
-                const int i = base + w;
-                int32_t uw[Cols<RT>::N];
-                load_units_smem<RT>(sp.units + (size_t)i * R, uw, R);
-                take_winner<RT, G>(c, d.job_begin + (i >> c.log2_k), i & (K - 1), uw, sp.vals[i], 0, false, 0.0);
+        for (int o = 3; o >= 0; --o)
+            if (q[o] == m1)
+                w = o;
+        const bool won = valid && !amb && w >= 0;
+        const int iw = base + (won ? w : 0);       // inside the stage even for lanes past the tile's end
+        {
+            int32_t uw[Cols<RT>::N];
+            load_units_smem<RT>(sp.units + (size_t)iw * R, uw, R);
+            const int32_t keep = won ? -1 : 0;
+#pragma unroll
+            for (int r = 0; r < Cols<RT>::N; ++r) {
+                if (RT == 0 && r >= R)
+                    break;
+                if (c.sp.small_units)
+                    acc32[r] += uw[r] & keep;      // below 2^23 each: exact in 32 bits for the tile
+                else
+                    c.acc[r] += (long long)(uw[r] & keep);
             }
+            if (won && (c.kind == PASS_FINAL || c.want_hash || c.want_min))
+                take_winner_extras<RT, G>(c, d.job_begin + (iw >> c.log2_k), iw & (K - 1), uw, sp.vals[iw], 0);
         }
         const int jstart = base & ~(K - 1);
         const int64_t job = d.job_begin + (base >> c.log2_k);
@@ -649,6 +674,9 @@ __device__ void process_tile_uniform4(WarpCtx<RT, G> &c, const TileDesc &d, cons
         if (amask)
             resolve_row<RT, G>(c, lane, amask, false, sp.units, sp.vals, sp.grp, jstart, jstart + K, thr, job, 0);
     }
+#pragma unroll
+    for (int r = 0; r < Cols<RT>::N; ++r)
+        c.acc[r] += acc32[r];
 }
 
 // Per-job running state of the general (CSR) path: smallest screen value with its index, and the
