@@ -30,9 +30,6 @@ namespace esp {
 #ifndef ESP_WARPS_PER_CTA
 #define ESP_WARPS_PER_CTA 4
 #endif
-#ifndef ESP_BLOCKS_PER_ITER
-#define ESP_BLOCKS_PER_ITER 1 // row blocks of 128 options screened together by the four-options-per-lane path
-#endif
 #ifndef ESP_V32_HW
 #define ESP_V32_HW 0          // 1: fp64 -> fp32 of values by the conversion instruction (round to nearest)
 #endif

@@ -599,147 +599,65 @@ __device__ __forceinline__ void load_units4_smem(const int32_t *p, int32_t (*u)[
     }
 }
 
-// Screen of the 4 consecutive options a lane owns in a row block: the lane's smallest value m1 (its
-// option index lw and its units ub are kept, so the winner never reloads them) and its
-// second-smallest value m2. Branch-free; lanes past the tile's end report m1 = m2 = +inf.
-template <int RT>
-struct Block4 {
-    float m1, m2;
-    int lw;
-    int32_t ub[Cols<RT>::N];
-};
-
-template <int RT, bool G>
-__device__ __forceinline__ void screen_block4(const WarpCtx<RT, G> &c, const StagePtrs &sp, int base, bool valid,
-                                              Block4<RT> &o)
-{
-    const int R = c.R;
-    float q[4] = {INFINITY, INFINITY, INFINITY, INFINITY};
-    int32_t u[4][Cols<RT>::N];
-    if (valid) {
-        bool dup[4];
-        load_units4_smem<RT>(sp.units + (size_t)base * R, u, dup, R);
-        const double2 va = reinterpret_cast<const double2 *>(sp.vals + base)[0];
-        const double2 vb = reinterpret_cast<const double2 *>(sp.vals + base)[1];
-        const double v[4] = {va.x, va.y, vb.x, vb.y};
-#pragma unroll
-        for (int k = 0; k < 4; ++k) {
-            const float qk = screen_score<RT, G>(u[k], v[k], 0, c.sp, R, c.rg);
-            q[k] = dup[k] ? INFINITY : qk;
-        }
-    }
-    // pairwise tournament: the first minimum of each pair, then of the two winners
-    const bool s01 = q[1] < q[0], s23 = q[3] < q[2];
-    const float qa = s01 ? q[1] : q[0], qa2 = s01 ? q[0] : q[1];
-    const float qb = s23 ? q[3] : q[2], qb2 = s23 ? q[2] : q[3];
-    const bool sab = qb < qa;
-    o.m1 = sab ? qb : qa;
-    o.m2 = fminf(fmaxf(qa, qb), fminf(qa2, qb2));
-    o.lw = sab ? (s23 ? 3 : 2) : (s01 ? 1 : 0);
-#pragma unroll
-    for (int r = 0; r < Cols<RT>::N; ++r) {
-        if (RT == 0 && r >= R)
-            break;
-        const int32_t ua = s01 ? u[1][r] : u[0][r];
-        const int32_t ubb = s23 ? u[3][r] : u[2][r];
-        o.ub[r] = sab ? ubb : ua;
-    }
-}
-
-// Completes the jobs of one row block after the butterfly: the demand of each unambiguous job is
-// added by the unique lane whose local minimum equals the job's minimum (masked, no branch); the
-// outputs of non-plain passes follow for those lanes.
-template <int RT, bool G>
-__device__ __forceinline__ void finish_block4(WarpCtx<RT, G> &c, const StagePtrs &sp, const TileDesc &d,
-                                              const Block4<RT> &o, float jm1, bool amb, bool valid, int base,
-                                              int K, int32_t *acc32)
-{
-    const bool won = valid && !amb && o.m1 == jm1;
-    const int32_t keep = won ? -1 : 0;
-#pragma unroll
-    for (int r = 0; r < Cols<RT>::N; ++r) {
-        if (RT == 0 && r >= c.R)
-            break;
-        if (c.sp.small_units)
-            acc32[r] += o.ub[r] & keep;       // each below 2^23: exact in 32 bits for a tile
-        else
-            c.acc[r] += (long long)(o.ub[r] & keep);
-    }
-    if (won && (c.kind == PASS_FINAL || c.want_hash || c.want_min)) {
-        const int iw = base + o.lw;
-        take_winner_extras<RT, G>(c, d.job_begin + (iw >> c.log2_k), iw & (K - 1), o.ub, sp.vals[iw], 0);
-    }
-}
-
 // Tile of a table whose jobs all have K options, K in {4, 8, 16, 32}. Each lane evaluates 4
-// consecutive options of one job (a row block is 128 options, two blocks are handled together when
-// the tile has them), and a log2(K / 4)-step xor butterfly over the job's K / 4 lanes completes the
-// job's smallest and second-smallest values. Exact resolutions of ambiguous jobs follow the blocks.
+// consecutive options of one job (a tile row block is 128 options), keeps their smallest and
+// second-smallest screen values, and a log2(K / 4)-step xor butterfly over the job's K / 4 lanes
+// completes the job. An unambiguous job's winner is the unique option holding the smallest value.
 template <int RT, bool G>
 __device__ void process_tile_uniform4(WarpCtx<RT, G> &c, const TileDesc &d, const StagePtrs &sp, int lane)
 {
+    const int R = c.R;
     const int n = d.n_opt;
     const int K = c.uniform_k;
     const int KL = K >> 2;                  // lanes per job
-    int32_t acc32[Cols<RT>::N];
-#pragma unroll
-    for (int r = 0; r < Cols<RT>::N; ++r)
-        acc32[r] = 0;
-#if ESP_BLOCKS_PER_ITER == 2
-    for (int b = 0; b < n; b += 256) {
-        const int base0 = b + 4 * lane, base1 = base0 + 128;
-        const bool v0 = base0 < n, v1 = base1 < n;    // n is a multiple of K, hence of 4
-        Block4<RT> o0, o1;
-        screen_block4<RT, G>(c, sp, base0, v0, o0);
-        screen_block4<RT, G>(c, sp, base1, v1, o1);
-        float m10 = o0.m1, m20 = o0.m2, m11 = o1.m1, m21 = o1.m2;
-        for (int dd = 1; dd < KL; dd <<= 1) {
-            const float a1 = __shfl_xor_sync(FULL, m10, dd), a2 = __shfl_xor_sync(FULL, m20, dd);
-            const float b1 = __shfl_xor_sync(FULL, m11, dd), b2 = __shfl_xor_sync(FULL, m21, dd);
-            m20 = fminf(fminf(m20, a2), fmaxf(m10, a1));
-            m10 = fminf(m10, a1);
-            m21 = fminf(fminf(m21, b2), fmaxf(m11, b1));
-            m11 = fminf(m11, b1);
-        }
-        const float thr0 = __fadd_ru(m10, c.sp.e2), thr1 = __fadd_ru(m11, c.sp.e2);
-        const bool amb0 = c.sp.exact || !(m20 > thr0), amb1 = c.sp.exact || !(m21 > thr1);
-        finish_block4<RT, G>(c, sp, d, o0, m10, amb0, v0, base0, K, acc32);
-        finish_block4<RT, G>(c, sp, d, o1, m11, amb1, v1, base1, K, acc32);
-        const int js0 = base0 & ~(K - 1), js1 = base1 & ~(K - 1);
-        const uint32_t am0 = __ballot_sync(FULL, v0 && amb0 && base0 == js0);
-        const uint32_t am1 = __ballot_sync(FULL, v1 && amb1 && base1 == js1);
-        if (am0)
-            resolve_row<RT, G>(c, lane, am0, false, sp.units, sp.vals, sp.grp, js0, js0 + K, thr0,
-                               d.job_begin + (base0 >> c.log2_k), 0);
-        if (am1)
-            resolve_row<RT, G>(c, lane, am1, false, sp.units, sp.vals, sp.grp, js1, js1 + K, thr1,
-                               d.job_begin + (base1 >> c.log2_k), 0);
-    }
-#else
     for (int b = 0; b < n; b += 128) {
-        const int base0 = b + 4 * lane;
-        const bool v0 = base0 < n;                     // n is a multiple of K, hence of 4
-        Block4<RT> o0;
-        screen_block4<RT, G>(c, sp, base0, v0, o0);
-        float m10 = o0.m1, m20 = o0.m2;
-        for (int dd = 1; dd < KL; dd <<= 1) {
-            const float a1 = __shfl_xor_sync(FULL, m10, dd), a2 = __shfl_xor_sync(FULL, m20, dd);
-            m20 = fminf(fminf(m20, a2), fmaxf(m10, a1));
-            m10 = fminf(m10, a1);
-        }
-        const float thr0 = __fadd_ru(m10, c.sp.e2);
-        const bool amb0 = c.sp.exact || !(m20 > thr0);
-        finish_block4<RT, G>(c, sp, d, o0, m10, amb0, v0, base0, K, acc32);
-        const int js0 = base0 & ~(K - 1);
-        const uint32_t am0 = __ballot_sync(FULL, v0 && amb0 && base0 == js0);
-        if (am0)
-            resolve_row<RT, G>(c, lane, am0, false, sp.units, sp.vals, sp.grp, js0, js0 + K, thr0,
-                               d.job_begin + (base0 >> c.log2_k), 0);
-    }
-#endif
+        const int base = b + 4 * lane;
+        const bool valid = base < n;        // n is a multiple of K, hence of 4
+        float q[4] = {INFINITY, INFINITY, INFINITY, INFINITY};
+        if (valid) {
+            int32_t u[4][Cols<RT>::N];
+            bool dup[4];
+            load_units4_smem<RT>(sp.units + (size_t)base * R, u, dup, R);
+            const double2 va = reinterpret_cast<const double2 *>(sp.vals + base)[0];
+            const double2 vb = reinterpret_cast<const double2 *>(sp.vals + base)[1];
+            const double v[4] = {va.x, va.y, vb.x, vb.y};
 #pragma unroll
-    for (int r = 0; r < Cols<RT>::N; ++r)
-        c.acc[r] += acc32[r];
+            for (int o = 0; o < 4; ++o)
+                if (!dup[o])
+                    q[o] = screen_score<RT, G>(u[o], v[o], 0, c.sp, R, c.rg);
+        }
+        // smallest and second smallest of the lane's four values
+        float a0 = fminf(q[0], q[1]), a1 = fmaxf(q[0], q[1]);
+        float b0 = fminf(q[2], q[3]), b1 = fmaxf(q[2], q[3]);
+        float m1 = fminf(a0, b0);
+        float m2 = fminf(fmaxf(a0, b0), fminf(a1, b1));
+        for (int dd = 1; dd < KL; dd <<= 1) {
+            const float o1 = __shfl_xor_sync(FULL, m1, dd);
+            const float o2 = __shfl_xor_sync(FULL, m2, dd);
+            m2 = fminf(fminf(m2, o2), fmaxf(m1, o1));
+            m1 = fminf(m1, o1);
+        }
+        const float thr = __fadd_ru(m1, c.sp.e2);
+        const bool amb = c.sp.exact || !(m2 > thr);
+        if (valid && !amb) {
+            int w = -1;
+#pragma unroll
+            for (int o = 3; o >= 0; --o)
+                if (q[o] == m1)
+                    w = o;
+            if (w >= 0) {
+                const int i = base + w;
+                int32_t uw[Cols<RT>::N];
+                load_units_smem<RT>(sp.units + (size_t)i * R, uw, R);
+                take_winner<RT, G>(c, d.job_begin + (i >> c.log2_k), i & (K - 1), uw, sp.vals[i], 0, false, 0.0);
+            }
+        }
+        const int jstart = base & ~(K - 1);
+        const int64_t job = d.job_begin + (base >> c.log2_k);
+        const uint32_t amask = __ballot_sync(FULL, valid && amb && base == jstart);
+        if (amask)
+            resolve_row<RT, G>(c, lane, amask, false, sp.units, sp.vals, sp.grp, jstart, jstart + K, thr, job, 0);
+    }
 }
 
 // Per-job running state of the general (CSR) path: smallest screen value with its index, and the
