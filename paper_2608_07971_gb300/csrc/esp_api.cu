@@ -60,6 +60,8 @@ struct esp_ctx {
 
     TileDesc *tiles = nullptr;
     int32_t *warp_begin = nullptr;
+    int32_t *scen_warps = nullptr;   // warps owning tiles of each scenario
+    unsigned int *arrive = nullptr;  // per-scenario arrivals of the round pass in flight
     int32_t n_warps = 0, tile_opt = 0, grid = 0, uniform_k = 0;
 
     double *lam = nullptr, *p64 = nullptr, *job_val = nullptr, *job_min = nullptr;
@@ -207,6 +209,7 @@ DevState dev_state(const esp_ctx *c)
     s.umax = c->umax;
     s.err = c->err;
     s.stats = c->stats;
+    s.arrive = c->arrive;
     s.lam_trace = nullptr;
     s.dem_trace = nullptr;
     s.hash_trace = nullptr;
@@ -359,6 +362,22 @@ esp_status load_common(esp_ctx *ctx, int32_t S, int32_t J, int32_t R, int32_t P,
     ctx->grid = (plan.n_warps + kWarpsPerCta - 1) / kWarpsPerCta;
     ALLOC(ctx->tiles, plan.tiles.size() + 1);
     ALLOC(ctx->warp_begin, plan.warp_begin.size());
+    ALLOC(ctx->scen_warps, (size_t)S);
+    ALLOC(ctx->arrive, (size_t)S);
+    {
+        std::vector<int32_t> sw((size_t)S, 0);
+        for (int32_t w = 0; w < plan.n_warps; ++w) {
+            int32_t last = -1;
+            for (int32_t k = plan.warp_begin[w]; k < plan.warp_begin[w + 1]; ++k)
+                if (plan.tiles[k].scenario != last) {
+                    last = plan.tiles[k].scenario;
+                    ++sw[last];
+                }
+        }
+        ESP_CUDA(cudaMemcpyAsync(ctx->scen_warps, sw.data(), sw.size() * sizeof(int32_t), cudaMemcpyHostToDevice,
+                                 ctx->stream));
+        ESP_CUDA(cudaStreamSynchronize(ctx->stream));
+    }
     if (!plan.tiles.empty())
         ESP_CUDA(cudaMemcpyAsync(ctx->tiles, plan.tiles.data(), plan.tiles.size() * sizeof(TileDesc),
                                  cudaMemcpyHostToDevice, ctx->stream));
@@ -429,6 +448,10 @@ esp_status enqueue_solve(esp_ctx *ctx, const esp_params *p, const DevState &st, 
     pl.n_warps = ctx->n_warps;
     pl.tile_opt = ctx->tile_opt;
     pl.uniform_k = ctx->uniform_k;
+    // the last warp to finish a scenario in a round pass updates its prices (one launch per round);
+    // ESP_FLAG_PER_ROUND_LAUNCH keeps a separate update launch (also used when no warp has tiles)
+    const bool fused = ctx->grid > 0 && !(p->flags & ESP_FLAG_PER_ROUND_LAUNCH);
+    pl.scen_warps = fused ? ctx->scen_warps : nullptr;
     SolveArgs a;
     a.eta0 = p->eta0;
     a.step = p->step;
@@ -464,7 +487,7 @@ esp_status enqueue_solve(esp_ctx *ctx, const esp_params *p, const DevState &st, 
         for (int r = 0; r < T && e == cudaSuccess; ++r) {
             if (ctx->grid > 0)
                 e = pass(r, PASS_ROUND);
-            if (e == cudaSuccess)
+            if (e == cudaSuccess && !fused)
                 e = launch_update(t, st, a, r, ctx->stream);
         }
         if (e == cudaSuccess && ctx->grid > 0)
@@ -473,7 +496,7 @@ esp_status enqueue_solve(esp_ctx *ctx, const esp_params *p, const DevState &st, 
             e = launch_objectives(t, st, a, ctx->stream);
         return e;
     };
-    ctx->last_launches = 3 + 2LL * T - (ctx->grid > 0 ? 0 : (T + 1));
+    ctx->last_launches = 3 + (fused ? 1LL : 2LL) * T - (ctx->grid > 0 ? 0 : (T + 1));
     ctx->last_T = T;
 
     GraphKey key;
@@ -801,6 +824,7 @@ esp_status esp_evaluate(esp_ctx *ctx, const double *lambda, int32_t mode, uint32
     pl.n_warps = ctx->n_warps;
     pl.tile_opt = ctx->tile_opt;
     pl.uniform_k = ctx->uniform_k;
+    pl.scen_warps = nullptr;
     SolveArgs a;
     a.eta0 = 1.0;
     a.step = 0;

@@ -235,12 +235,197 @@ __device__ __forceinline__ bool load_units_global(const int32_t *p, int32_t *u, 
 }
 
 // ---------------------------------------------------------------------------------------------
+// Price update (Eq. price_update), one warp per scenario, and the screen bound of the new prices.
+
+__device__ __forceinline__ double warp_sum_fixed(double x)
+{
+#pragma unroll
+    for (int d = 16; d >= 1; d >>= 1)
+        x += __shfl_xor_sync(FULL, x, d);
+    return x;
+}
+
+__device__ __forceinline__ double warp_max(double x)
+{
+#pragma unroll
+    for (int d = 16; d >= 1; d >>= 1)
+        x = fmax(x, __shfl_xor_sync(FULL, x, d));
+    return x;
+}
+
+// Effective prices p = lambda (RAW) or lambda / C (NORMALIZED), their fp32 copy, and the bound E.
+__device__ void set_prices(const DevTable &t, const DevState &st, const SolveArgs &a, int s, int lane)
+{
+    const int P = t.P, R = t.R;
+    bool huge = false;
+    for (int k = lane; k < P; k += 32) {
+        const double lam = st.lam[(size_t)s * P + k];
+        const double p = (a.mode == 1) ? lam / (double)t.cap[(size_t)s * P + k] : lam;
+        st.p64[(size_t)s * P + k] = p;
+        st.p32[(size_t)s * P + k] = __double2float_rn(p);
+        huge |= !(p <= 0x1p100);
+    }
+    __syncwarp();
+    // M_s = max|v| + sum_r (max price of column r over groups) * (max unit of column r)
+    double term = 0.0;
+    if (lane < R) {
+        double pmax = 0.0;
+        if (t.group == nullptr || lane < t.r_global) {
+            pmax = st.p64[(size_t)s * P + lane];
+        } else {
+            for (int gi = 0; gi < t.n_groups; ++gi)
+                pmax = fmax(pmax, st.p64[(size_t)s * P + t.r_global + (R - t.r_global) * gi + (lane - t.r_global)]);
+        }
+        term = pmax * (double)st.umax[(size_t)s * R + lane];
+    }
+    const double M = st.vmax[s] + warp_sum_fixed(term);
+    huge = __any_sync(FULL, huge);
+    if (lane == 0) {
+        float e;
+        if (a.exact_only || huge || !(M <= 0x1p100)) {
+            e = INFINITY;
+        } else {
+            const double eb = (4.0 * R + 16.0) * 0x1p-24 * M * (1.0 + 0x1p-20) + 0x1p-99;
+            e = __double2float_ru(eb);
+        }
+        st.ebound[s] = e;
+    }
+}
+
+__global__ void k_init(DevTable t, DevState st, SolveArgs a, const double *lambda0)
+{
+    const int lane = threadIdx.x & 31;
+    const int s = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+    if (s >= t.S)
+        return;
+    const int P = t.P;
+    for (int k = lane; k < P; k += 32) {
+        const double l0 = lambda0 ? lambda0[(size_t)s * P + k] : 0.0;
+        st.lam[(size_t)s * P + k] = l0;
+        st.U[(size_t)s * P + k] = 0ull;
+        st.U_final[(size_t)s * P + k] = 0ull;
+        if (st.lam_trace)
+            st.lam_trace[((size_t)s * (a.T + 1)) * P + k] = l0;
+    }
+    if (lane == 0) {
+        st.hash[s] = 0ull;
+        st.arrive[s] = 0u;
+        st.rounds_run[s] = 0;
+        st.converged[s] = 0;
+        st.status[s] = 0;
+        st.frozen[s] = 0;
+        st.best_dual[s] = INFINITY;
+    }
+    __syncwarp();
+    set_prices(t, st, a, s, lane);
+}
+
+// Eq. price_update for scenario s after round `round` (one warp): traces, the projected step, the
+// stopping rule, and the prices and screen bound of the next round. Reads what other warps of the
+// same launch wrote (demand, minimal reduced costs, fingerprint) through L2.
+__device__ void update_scenario(const DevTable &t, const DevState &st, const SolveArgs &a, int s, int round,
+                                int lane)
+{
+    const int P = t.P, J = t.J, T = a.T;
+    const size_t sp = (size_t)s * P;
+
+    if (st.dual_trace) {   // g(lambda^t) from the minimal reduced costs of round t
+        double part = 0.0;
+        for (int j = lane; j < J; j += 32)
+            part += -__ldcg(st.job_min + (size_t)s * J + j);
+        double lc = 0.0;
+        for (int k = lane; k < P; k += 32)
+            lc += (a.mode == 1) ? st.lam[sp + k] : st.lam[sp + k] * (double)t.cap[sp + k];
+        const double g = warp_sum_fixed(part) + warp_sum_fixed(lc);
+        if (lane == 0) {
+            st.dual_trace[(size_t)s * (T + 1) + round] = g;
+            if (g < st.best_dual[s])
+                st.best_dual[s] = g;
+        }
+    }
+    if (st.hash_trace && lane == 0) {
+        st.hash_trace[(size_t)s * T + round] = __ldcg(st.hash + s);
+        st.hash[s] = 0ull;
+    }
+
+    double eta = a.eta0;
+    if (a.step == 1)
+        eta = a.eta0 / sqrt((double)(round + 1));
+    bool bad = false;
+    double dmax = 0.0, amax = 0.0;
+    for (int k = lane; k < P; k += 32) {
+        const long long U = (long long)__ldcg(st.U + sp + k);
+        const long long C = t.cap[sp + k];
+        if (st.dem_trace)
+            st.dem_trace[((size_t)s * T + round) * P + k] = U;
+        double excess = (double)(U - C);
+        if (a.mode == 1)
+            excess = excess / (double)C;
+        const double lam = st.lam[sp + k];
+        const double moved = __fma_rn(eta, excess, lam);
+        const double nl = moved > 0.0 ? moved : 0.0;
+        bad |= !isfinite(nl);
+        dmax = fmax(dmax, fabs(nl - lam));
+        amax = fmax(amax, fabs(lam));
+    }
+    bad = __any_sync(FULL, bad);
+    dmax = warp_max(dmax);
+    amax = warp_max(amax);
+    if (bad) {
+        for (int k = lane; k < P; k += 32)
+            st.U[sp + k] = 0ull;
+        if (lane == 0) {
+            st.status[s] = 2;
+            st.frozen[s] = 1;
+        }
+        return;
+    }
+    for (int k = lane; k < P; k += 32) {
+        const long long U = (long long)__ldcg(st.U + sp + k);
+        const long long C = t.cap[sp + k];
+        double excess = (double)(U - C);
+        if (a.mode == 1)
+            excess = excess / (double)C;
+        const double moved = __fma_rn(eta, excess, st.lam[sp + k]);
+        const double nl = moved > 0.0 ? moved : 0.0;
+        st.lam[sp + k] = nl;
+        st.U[sp + k] = 0ull;
+        if (st.lam_trace)
+            st.lam_trace[((size_t)s * (T + 1) + round + 1) * P + k] = nl;
+    }
+    const bool conv = (a.tol > 0.0) && (dmax <= a.tol * fmax(1.0, amax));
+    if (lane == 0) {
+        st.rounds_run[s] = round + 1;
+        if (conv) {
+            st.converged[s] = 1;
+            st.frozen[s] = 1;
+        }
+    }
+    __syncwarp();
+    set_prices(t, st, a, s, lane);
+}
+
+// Separate price-update launch (used when no warp owns tiles, e.g. J = 0).
+__global__ void k_update(DevTable t, DevState st, SolveArgs a, int round)
+{
+    const int lane = threadIdx.x & 31;
+    const int s = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+    if (s >= t.S || st.frozen[s])
+        return;
+    update_scenario(t, st, a, s, round, lane);
+}
+
+
+// ---------------------------------------------------------------------------------------------
 // The warp's evaluation context.
 
 template <int RT, bool G>
 struct WarpCtx {
     DevTable t;
     DevState st;
+    const int32_t *scen_warps;  // non-null: the last warp to finish a scenario in a round pass updates its prices
+    SolveArgs a;
+    int round;
     int R, rg;
     int kind;                 // PassKind
     bool want_min;            // job_min needed (final pass or dual trace)
@@ -280,6 +465,20 @@ __device__ void flush(WarpCtx<RT, G> &c, int lane)
         if (lane == 0)
             atomicAdd(c.st.hash + c.s, h);
         c.hacc = 0;
+    }
+    if (c.kind == PASS_ROUND && c.scen_warps != nullptr && !c.sp.skip) {
+        // arrive; the warp that completes the scenario's count applies Eq. price_update to it
+        __threadfence();
+        unsigned int old = 0;
+        if (lane == 0)
+            old = atomicAdd(c.st.arrive + c.s, 1u);
+        old = __shfl_sync(FULL, old, 0);
+        if (old + 1 == (unsigned int)__ldg(c.scen_warps + c.s)) {
+            __threadfence();
+            update_scenario(c.t, c.st, c.a, c.s, c.round, lane);
+            if (lane == 0)
+                c.st.arrive[c.s] = 0u;     // every warp of this pass has arrived
+        }
     }
 }
 
@@ -894,6 +1093,9 @@ __global__ void __launch_bounds__(kWarpsPerCta * 32, UNI ? kMinCtasPerSm : kMinC
     WarpCtx<RT, G> c;
     c.t = t;
     c.st = st;
+    c.scen_warps = pl.scen_warps;
+    c.a = a;
+    c.round = round;
     c.R = RT ? RT : t.R;
     c.rg = t.r_global;
     // PLAIN: a round pass without traces (the hot case), with every per-pass choice a constant
@@ -907,8 +1109,6 @@ __global__ void __launch_bounds__(kWarpsPerCta * 32, UNI ? kMinCtasPerSm : kMinC
     for (int r = 0; r < Cols<RT>::N; ++r)
         c.acc[r] = 0;
     c.hacc = 0;
-    (void)a;
-    (void)round;
 
     if (lane == 0) {
         for (int s = 0; s < kStages; ++s)
@@ -1052,178 +1252,6 @@ __global__ void __launch_bounds__(kDedupWarps * 32) k_mark_duplicates(DevTable t
         }
         __syncwarp();
     }
-}
-
-// ---------------------------------------------------------------------------------------------
-// Price update (Eq. price_update), one warp per scenario, and the screen bound of the new prices.
-
-__device__ __forceinline__ double warp_sum_fixed(double x)
-{
-#pragma unroll
-    for (int d = 16; d >= 1; d >>= 1)
-        x += __shfl_xor_sync(FULL, x, d);
-    return x;
-}
-
-__device__ __forceinline__ double warp_max(double x)
-{
-#pragma unroll
-    for (int d = 16; d >= 1; d >>= 1)
-        x = fmax(x, __shfl_xor_sync(FULL, x, d));
-    return x;
-}
-
-// Effective prices p = lambda (RAW) or lambda / C (NORMALIZED), their fp32 copy, and the bound E.
-__device__ void set_prices(const DevTable &t, const DevState &st, const SolveArgs &a, int s, int lane)
-{
-    const int P = t.P, R = t.R;
-    bool huge = false;
-    for (int k = lane; k < P; k += 32) {
-        const double lam = st.lam[(size_t)s * P + k];
-        const double p = (a.mode == 1) ? lam / (double)t.cap[(size_t)s * P + k] : lam;
-        st.p64[(size_t)s * P + k] = p;
-        st.p32[(size_t)s * P + k] = __double2float_rn(p);
-        huge |= !(p <= 0x1p100);
-    }
-    __syncwarp();
-    // M_s = max|v| + sum_r (max price of column r over groups) * (max unit of column r)
-    double term = 0.0;
-    if (lane < R) {
-        double pmax = 0.0;
-        if (t.group == nullptr || lane < t.r_global) {
-            pmax = st.p64[(size_t)s * P + lane];
-        } else {
-            for (int gi = 0; gi < t.n_groups; ++gi)
-                pmax = fmax(pmax, st.p64[(size_t)s * P + t.r_global + (R - t.r_global) * gi + (lane - t.r_global)]);
-        }
-        term = pmax * (double)st.umax[(size_t)s * R + lane];
-    }
-    const double M = st.vmax[s] + warp_sum_fixed(term);
-    huge = __any_sync(FULL, huge);
-    if (lane == 0) {
-        float e;
-        if (a.exact_only || huge || !(M <= 0x1p100)) {
-            e = INFINITY;
-        } else {
-            const double eb = (4.0 * R + 16.0) * 0x1p-24 * M * (1.0 + 0x1p-20) + 0x1p-99;
-            e = __double2float_ru(eb);
-        }
-        st.ebound[s] = e;
-    }
-}
-
-__global__ void k_init(DevTable t, DevState st, SolveArgs a, const double *lambda0)
-{
-    const int lane = threadIdx.x & 31;
-    const int s = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
-    if (s >= t.S)
-        return;
-    const int P = t.P;
-    for (int k = lane; k < P; k += 32) {
-        const double l0 = lambda0 ? lambda0[(size_t)s * P + k] : 0.0;
-        st.lam[(size_t)s * P + k] = l0;
-        st.U[(size_t)s * P + k] = 0ull;
-        st.U_final[(size_t)s * P + k] = 0ull;
-        if (st.lam_trace)
-            st.lam_trace[((size_t)s * (a.T + 1)) * P + k] = l0;
-    }
-    if (lane == 0) {
-        st.hash[s] = 0ull;
-        st.rounds_run[s] = 0;
-        st.converged[s] = 0;
-        st.status[s] = 0;
-        st.frozen[s] = 0;
-        st.best_dual[s] = INFINITY;
-    }
-    __syncwarp();
-    set_prices(t, st, a, s, lane);
-}
-
-__global__ void k_update(DevTable t, DevState st, SolveArgs a, int round)
-{
-    const int lane = threadIdx.x & 31;
-    const int s = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
-    if (s >= t.S)
-        return;
-    if (st.frozen[s])
-        return;
-    const int P = t.P, J = t.J, T = a.T;
-    const size_t sp = (size_t)s * P;
-
-    if (st.dual_trace) {   // g(lambda^t) from the minimal reduced costs of round t
-        double part = 0.0;
-        for (int j = lane; j < J; j += 32)
-            part += -st.job_min[(size_t)s * J + j];
-        double lc = 0.0;
-        for (int k = lane; k < P; k += 32)
-            lc += (a.mode == 1) ? st.lam[sp + k] : st.lam[sp + k] * (double)t.cap[sp + k];
-        const double g = warp_sum_fixed(part) + warp_sum_fixed(lc);
-        if (lane == 0) {
-            st.dual_trace[(size_t)s * (T + 1) + round] = g;
-            if (g < st.best_dual[s])
-                st.best_dual[s] = g;
-        }
-    }
-    if (st.hash_trace && lane == 0) {
-        st.hash_trace[(size_t)s * T + round] = st.hash[s];
-        st.hash[s] = 0ull;
-    }
-
-    double eta = a.eta0;
-    if (a.step == 1)
-        eta = a.eta0 / sqrt((double)(round + 1));
-    bool bad = false;
-    double dmax = 0.0, amax = 0.0;
-    for (int k = lane; k < P; k += 32) {
-        const long long U = (long long)st.U[sp + k];
-        const long long C = t.cap[sp + k];
-        if (st.dem_trace)
-            st.dem_trace[((size_t)s * T + round) * P + k] = U;
-        double excess = (double)(U - C);
-        if (a.mode == 1)
-            excess = excess / (double)C;
-        const double lam = st.lam[sp + k];
-        const double moved = __fma_rn(eta, excess, lam);
-        const double nl = moved > 0.0 ? moved : 0.0;
-        bad |= !isfinite(nl);
-        dmax = fmax(dmax, fabs(nl - lam));
-        amax = fmax(amax, fabs(lam));
-    }
-    bad = __any_sync(FULL, bad);
-    dmax = warp_max(dmax);
-    amax = warp_max(amax);
-    if (bad) {
-        for (int k = lane; k < P; k += 32)
-            st.U[sp + k] = 0ull;
-        if (lane == 0) {
-            st.status[s] = 2;
-            st.frozen[s] = 1;
-        }
-        return;
-    }
-    for (int k = lane; k < P; k += 32) {
-        const long long U = (long long)st.U[sp + k];
-        const long long C = t.cap[sp + k];
-        double excess = (double)(U - C);
-        if (a.mode == 1)
-            excess = excess / (double)C;
-        const double moved = __fma_rn(eta, excess, st.lam[sp + k]);
-        const double nl = moved > 0.0 ? moved : 0.0;
-        st.lam[sp + k] = nl;
-        st.U[sp + k] = 0ull;
-        if (st.lam_trace)
-            st.lam_trace[((size_t)s * (T + 1) + round + 1) * P + k] = nl;
-    }
-    const bool conv = (a.tol > 0.0) && (dmax <= a.tol * fmax(1.0, amax));
-    if (lane == 0) {
-        st.rounds_run[s] = round + 1;
-        if (conv) {
-            st.converged[s] = 1;
-            st.frozen[s] = 1;
-        }
-    }
-    __syncwarp();
-    set_prices(t, st, a, s, lane);
 }
 
 // Final objectives: primal = sum of chosen values, dual g(lambda) at the final prices, feasibility.

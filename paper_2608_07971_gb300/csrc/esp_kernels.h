@@ -42,6 +42,7 @@ struct DevState {
     const int32_t *umax;      // S*R max unit of each stored column in the scenario (load time)
     unsigned int *err;        // device error word (DEV_ERR_*)
     unsigned long long *stats;  // [0] exact resolutions since the last reset, [1] duplicates marked at load
+    unsigned int *arrive;     // S   warps of the current round pass that finished the scenario
     double *lam_trace;        // S*(T+1)*P or nullptr
     long long *dem_trace;     // S*T*P or nullptr
     unsigned long long *hash_trace; // S*T or nullptr
@@ -54,6 +55,7 @@ struct DevPlan {
     int32_t n_warps;
     int32_t tile_opt;
     int32_t uniform_k;          // > 0: every job has exactly this many options, a power of two <= 32
+    const int32_t *scen_warps;  // S warps owning tiles of each scenario; non-null: round passes update prices
 };
 
 struct SolveArgs {

@@ -274,3 +274,23 @@ def test_duplicate_marking_matches_numpy_count():
     s.solve(w.eta0, 5)
     res, _ = esp.esp_debug_stats(s.ctx)
     assert res <= 0.05 * t.S * t.J * 6          # few exact resolutions once duplicates are marked
+
+
+@pytest.mark.parametrize("name", ["whatif", "heavy", "grouped"])
+def test_fused_update_equals_separate_update_launch(name):
+    """The price update done by the last warp of each scenario inside the evaluation pass gives the
+    same trajectory as the separate update launch (ESP_FLAG_PER_ROUND_LAUNCH)."""
+    if name == "whatif":
+        t = W.whatif_batch(scenarios=[2, 9, 40], J=700).table
+    elif name == "heavy":
+        t = W.heavy_tail(scenarios=[1], J=3000).table
+    else:
+        t = W.random_table(np.random.default_rng(8), S=3, J=200, R=6, kmin=1, kmax=900, groups=10, r_global=4)
+    s = esp.Solver(t)
+    a = s.solve(0.05, 40, traces=True)
+    b = s.solve(0.05, 40, flags=esp.ESP_FLAG_PER_ROUND_LAUNCH, traces=True)
+    for f in ("lam", "sel", "demand", "lambda_trace", "demand_trace", "selhash_trace", "dual_trace"):
+        assert np.array_equal(getattr(a, f), getattr(b, f), equal_nan=True), f
+    assert s.launches() == 2 * 40 + 3
+    s.solve(0.05, 40)
+    assert s.launches() == 40 + 3
