@@ -59,9 +59,10 @@ typedef enum { ESP_STEP_FIXED = 0, ESP_STEP_INV_SQRT = 1 } esp_step_rule;
 
 /* esp_params.flags */
 #define ESP_FLAG_EXACT_ONLY 0x1u       /* evaluate every option in fp64 (no fp32 screen); same results, slower */
-#define ESP_FLAG_PER_ROUND_LAUNCH 0x2u /* one kernel launch per round (CUDA graph) instead of the persistent loop */
-#define ESP_FLAG_PASS_EVENTS 0x4u      /* record a CUDA event pair around every evaluation-pass launch
-                                          (direct launches, no graph); read with esp_pass_times */
+#define ESP_FLAG_PER_ROUND_LAUNCH 0x2u /* price update as its own launch after every evaluation pass, instead of
+                                          by the pass's last warp per scenario (same results) */
+#define ESP_FLAG_PASS_EVENTS 0x4u      /* record a CUDA event pair around every evaluation-pass launch (inside the
+                                          solve's CUDA graph on a non-default stream); read with esp_pass_times */
 
 typedef struct {
     double eta0;            /* > 0, finite */
@@ -180,7 +181,9 @@ esp_status esp_last_launch_count(esp_ctx *ctx, int64_t *out);
 
 /* Device time of the evaluation passes recorded with ESP_FLAG_PASS_EVENTS since the last reset:
  * *total_ms receives the summed CUDA-event durations (measured on the context's stream) and *count
- * the number of passes. Waits for the stream. reset != 0 clears the record afterwards. */
+ * the number of passes. Solves on the legacy default stream contribute every pass; solves replayed
+ * from a CUDA graph contribute the passes of the latest replay. Waits for the stream. reset != 0
+ * clears the record afterwards. */
 esp_status esp_pass_times(esp_ctx *ctx, double *total_ms, int64_t *count, int32_t reset);
 
 /* Static description of a string for a status. Never NULL. */

@@ -85,9 +85,14 @@ struct esp_ctx {
     int64_t last_launches = 0;
     int32_t last_T = 0;
 
-    // ESP_FLAG_PASS_EVENTS: event pairs around evaluation passes; pool reused after a reset
+    // ESP_FLAG_PASS_EVENTS: event pairs around evaluation passes. Direct launches use ev_pool
+    // (reused after a reset); a captured graph records into graph_pool, and every replay rewrites
+    // those events, so they always hold the passes of the graph's latest replay.
     std::vector<cudaEvent_t> ev_pool;
     size_t ev_used = 0;
+    std::vector<cudaEvent_t> graph_pool;
+    size_t graph_pairs = 0;        // event pairs inside the cached graph
+    bool graph_timed_run = false;  // a timed graph ran since the last reset
 };
 
 namespace {
@@ -463,18 +468,21 @@ esp_status enqueue_solve(esp_ctx *ctx, const esp_params *p, const DevState &st, 
     const int T = p->max_rounds;
 
     const bool timed = (p->flags & ESP_FLAG_PASS_EVENTS) != 0;
+    const bool use_graph = ctx->stream != nullptr;   // the legacy default stream cannot be captured
+    std::vector<cudaEvent_t> &pool = use_graph ? ctx->graph_pool : ctx->ev_pool;
+    size_t pool_used = use_graph ? 0 : ctx->ev_used;
     auto pass = [&](int r, PassKind kind) -> cudaError_t {
         if (!timed)
             return launch_pass(t, st, pl, a, r, kind, ctx->grid, ctx->stream);
-        while (ctx->ev_pool.size() < ctx->ev_used + 2) {
+        while (pool.size() < pool_used + 2) {
             cudaEvent_t ev;
             cudaError_t e = cudaEventCreate(&ev);
             if (e != cudaSuccess)
                 return e;
-            ctx->ev_pool.push_back(ev);
+            pool.push_back(ev);
         }
-        cudaEvent_t e0 = ctx->ev_pool[ctx->ev_used], e1 = ctx->ev_pool[ctx->ev_used + 1];
-        ctx->ev_used += 2;
+        cudaEvent_t e0 = pool[pool_used], e1 = pool[pool_used + 1];
+        pool_used += 2;
         cudaError_t e = cudaEventRecord(e0, ctx->stream);
         if (e == cudaSuccess)
             e = launch_pass(t, st, pl, a, r, kind, ctx->grid, ctx->stream);
@@ -512,8 +520,9 @@ esp_status enqueue_solve(esp_ctx *ctx, const esp_params *p, const DevState &st, 
     key.gt = st.dual_trace;
     key.has_l0 = has_l0;
 
-    if (ctx->stream == nullptr || timed) {   // the legacy default stream cannot be captured
+    if (!use_graph) {
         ESP_CUDA(issue());
+        ctx->ev_used = pool_used;
         return ESP_OK;
     }
     if (!(ctx->gexec && ctx->gkey == key)) {
@@ -537,8 +546,11 @@ esp_status enqueue_solve(esp_ctx *ctx, const esp_params *p, const DevState &st, 
             return cuda_fail(ctx, e);
         }
         ctx->gkey = key;
+        ctx->graph_pairs = timed ? pool_used / 2 : 0;
     }
     ESP_CUDA(cudaGraphLaunch(ctx->gexec, ctx->stream));
+    if (timed)
+        ctx->graph_timed_run = true;
     return ESP_OK;
 }
 
@@ -867,15 +879,25 @@ esp_status esp_pass_times(esp_ctx *ctx, double *total_ms, int64_t *count, int32_
         return ESP_ERR_INVALID_ARG;
     ESP_CUDA(cudaStreamSynchronize(ctx->stream));
     double sum = 0.0;
-    for (size_t i = 0; i + 1 < ctx->ev_used; i += 2) {
+    int64_t n = 0;
+    for (size_t i = 0; i + 1 < ctx->ev_used; i += 2, ++n) {
         float ms = 0.0f;
         ESP_CUDA(cudaEventElapsedTime(&ms, ctx->ev_pool[i], ctx->ev_pool[i + 1]));
         sum += ms;
     }
+    if (ctx->graph_timed_run) {   // the latest replay of the timed graph
+        for (size_t i = 0; i < ctx->graph_pairs; ++i, ++n) {
+            float ms = 0.0f;
+            ESP_CUDA(cudaEventElapsedTime(&ms, ctx->graph_pool[2 * i], ctx->graph_pool[2 * i + 1]));
+            sum += ms;
+        }
+    }
     *total_ms = sum;
-    *count = (int64_t)(ctx->ev_used / 2);
-    if (reset)
+    *count = n;
+    if (reset) {
         ctx->ev_used = 0;
+        ctx->graph_timed_run = false;
+    }
     return ESP_OK;
 }
 
@@ -892,6 +914,8 @@ void esp_destroy(esp_ctx *ctx)
     if (ctx->ht.p) cudaFree(ctx->ht.p);
     if (ctx->gt.p) cudaFree(ctx->gt.p);
     for (cudaEvent_t e : ctx->ev_pool)
+        cudaEventDestroy(e);
+    for (cudaEvent_t e : ctx->graph_pool)
         cudaEventDestroy(e);
     delete ctx;
 }
