@@ -481,13 +481,14 @@ esp_status enqueue_solve(esp_ctx *ctx, const esp_params *p, const DevState &st, 
                 return e;
             pool.push_back(ev);
         }
+        // external records: inside a stream capture they become event-record nodes of the graph
         cudaEvent_t e0 = pool[pool_used], e1 = pool[pool_used + 1];
         pool_used += 2;
-        cudaError_t e = cudaEventRecord(e0, ctx->stream);
+        cudaError_t e = cudaEventRecordWithFlags(e0, ctx->stream, cudaEventRecordExternal);
         if (e == cudaSuccess)
             e = launch_pass(t, st, pl, a, r, kind, ctx->grid, ctx->stream);
         if (e == cudaSuccess)
-            e = cudaEventRecord(e1, ctx->stream);
+            e = cudaEventRecordWithFlags(e1, ctx->stream, cudaEventRecordExternal);
         return e;
     };
     auto issue = [&]() -> cudaError_t {

@@ -294,3 +294,22 @@ def test_fused_update_equals_separate_update_launch(name):
     assert s.launches() == 2 * 40 + 3
     s.solve(0.05, 40)
     assert s.launches() == 40 + 3
+
+
+def test_pass_event_timing_in_graph_and_direct():
+    """ESP_FLAG_PASS_EVENTS times every evaluation pass: inside the solve's CUDA graph on a
+    non-default stream (latest replay) and with direct launches on the default stream."""
+    import torch
+    t = W.whatif_batch(scenarios=[0, 1], J=256).table
+    st = torch.cuda.Stream()
+    s = esp.Solver(t, stream=st.cuda_stream)
+    prm = s.params(0.02, 10, flags=esp.ESP_FLAG_PASS_EVENTS)
+    for _ in range(3):
+        esp.esp_solve_async(s.ctx, prm)
+    ms, n = esp.esp_pass_times(s.ctx)
+    assert n == 11 and ms > 0.0
+    d = esp.Solver(t)            # legacy default stream: direct launches accumulate
+    for _ in range(2):
+        d.solve(0.02, 10, flags=esp.ESP_FLAG_PASS_EVENTS)
+    ms, n = esp.esp_pass_times(d.ctx)
+    assert n == 22 and ms > 0.0
