@@ -484,11 +484,12 @@ esp_status enqueue_solve(esp_ctx *ctx, const esp_params *p, const DevState &st, 
         // external records: inside a stream capture they become event-record nodes of the graph
         cudaEvent_t e0 = pool[pool_used], e1 = pool[pool_used + 1];
         pool_used += 2;
-        cudaError_t e = cudaEventRecordWithFlags(e0, ctx->stream, cudaEventRecordExternal);
+        const unsigned int rf = use_graph ? cudaEventRecordExternal : cudaEventRecordDefault;
+        cudaError_t e = cudaEventRecordWithFlags(e0, ctx->stream, rf);
         if (e == cudaSuccess)
             e = launch_pass(t, st, pl, a, r, kind, ctx->grid, ctx->stream);
         if (e == cudaSuccess)
-            e = cudaEventRecordWithFlags(e1, ctx->stream, cudaEventRecordExternal);
+            e = cudaEventRecordWithFlags(e1, ctx->stream, rf);
         return e;
     };
     auto issue = [&]() -> cudaError_t {
