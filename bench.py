@@ -69,6 +69,19 @@ def make_workload(name: str, rank: int, per=None) -> W.Workload:
     return W.make(name, scenarios=scenario_ids(name, rank, per))
 
 
+def aggregate(dist, step_seconds: float, evals_local: float, device=None):
+    """Whole-job throughput under weak scaling: evaluations summed over ranks, divided by the slowest
+    rank's step time (max over ranks). dist is torch.distributed or None for one process."""
+    if dist is None:
+        return evals_local / step_seconds, step_seconds, evals_local
+    import torch
+    t = torch.tensor([step_seconds], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    e = torch.tensor([float(evals_local)], dtype=torch.float64, device=device)
+    dist.all_reduce(e, op=dist.ReduceOp.SUM)
+    return float(e.item()) / float(t.item()), float(t.item()), float(e.item())
+
+
 def config_of(w: W.Workload, T: int) -> dict:
     t = w.table
     K = t.option_counts()
@@ -312,17 +325,8 @@ def run_ours(args):
     n_res, n_marked = esp.esp_debug_stats(ctx, reset=True)
 
     evals_step = t.n_opt * (T + 1)
-    ms_max = ms
-    if dist is not None:
-        x = torch.tensor([ms], device="cuda", dtype=torch.float64)
-        dist.all_reduce(x, op=dist.ReduceOp.MAX)
-        ms_max = float(x.item())
-        y = torch.tensor([float(evals_step)], device="cuda", dtype=torch.float64)
-        dist.all_reduce(y)
-        evals_total = float(y.item())
-    else:
-        evals_total = float(evals_step)
-    value = evals_total / (ms_max / 1e3)
+    value, step_s, evals_total = aggregate(dist, ms / 1e3, evals_step, device="cuda")
+    ms_max = step_s * 1e3
 
     # roofline of the dominant kernel (the evaluation pass): algorithmic bytes = the option table
     peak, peak_kind = measured_peak()
@@ -365,14 +369,11 @@ def run_ours(args):
             e2e_step()
         e2e_s = (time.perf_counter() - t0) / args.steps
         barrier()
-        if dist is not None:
-            x = torch.tensor([e2e_s], device="cuda", dtype=torch.float64)
-            dist.all_reduce(x, op=dist.ReduceOp.MAX)
-            e2e_s = float(x.item())
+        e2e_value, e2e_s, _ = aggregate(dist, e2e_s, evals_step, device="cuda")
         h2d = t.job_off.nbytes + t.units.nbytes + t.values.nbytes + t.capacity.nbytes + \
             (0 if t.group is None else t.group.nbytes)
         d2h = h_sel.numel() * 4 + h_lam.numel() * 8 + t.S * esp.RESULT_DTYPE.itemsize
-        e2e = {"value": evals_total / e2e_s, "unit": "option-evals/s", "h2d_bytes_per_step": int(h2d),
+        e2e = {"value": e2e_value, "unit": "option-evals/s", "h2d_bytes_per_step": int(h2d),
                "d2h_bytes_per_step": int(d2h), "ms_per_step": e2e_s * 1e3}
 
     cpu = None
