@@ -467,14 +467,19 @@ __device__ void flush(WarpCtx<RT, G> &c, int lane)
         c.hacc = 0;
     }
     if (c.kind == PASS_ROUND && c.scen_warps != nullptr && !c.sp.skip) {
-        // arrive; the warp that completes the scenario's count applies Eq. price_update to it
-        __threadfence();
+        // arrive; the warp that completes the scenario's count applies Eq. price_update to it. Lane 0
+        // issued this warp's demand and fingerprint atomics, so its release-ordered arrival publishes
+        // them; with the dual traced, every lane's minimal reduced costs are fenced first.
+        if (c.want_min) {
+            __syncwarp();
+            __threadfence();
+        }
         unsigned int old = 0;
         if (lane == 0)
-            old = atomicAdd(c.st.arrive + c.s, 1u);
+            asm volatile("atom.add.release.gpu.u32 %0, [%1], 1;" : "=r"(old) : "l"(c.st.arrive + c.s) : "memory");
         old = __shfl_sync(FULL, old, 0);
         if (old + 1 == (unsigned int)__ldg(c.scen_warps + c.s)) {
-            __threadfence();
+            asm volatile("fence.acq_rel.gpu;" ::: "memory");
             update_scenario(c.t, c.st, c.a, c.s, c.round, lane);
             if (lane == 0)
                 c.st.arrive[c.s] = 0u;     // every warp of this pass has arrived
