@@ -30,6 +30,12 @@ namespace esp {
 #ifndef ESP_WARPS_PER_CTA
 #define ESP_WARPS_PER_CTA 4
 #endif
+#ifndef ESP_GENERAL_TILE_MAX
+#define ESP_GENERAL_TILE_MAX 0   // cap on the tile of general (CSR) tables; 0: the largest that fits
+#endif
+#ifndef ESP_MIN_CTAS_GENERAL
+#define ESP_MIN_CTAS_GENERAL 4
+#endif
 #ifndef ESP_V32_HW
 #define ESP_V32_HW 0          // 1: fp64 -> fp32 of values by the conversion instruction (round to nearest)
 #endif
@@ -43,7 +49,7 @@ constexpr int kStages = ESP_STAGES;  // TMA stages per warp
 constexpr int kPrefetchTiles = ESP_PREFETCH_TILES;  // L2 prefetch distance, in tiles of the warp
 constexpr int kUniform4Tile = ESP_UNIFORM4_TILE;    // tile of the 4-options-per-lane path (0: largest)
 constexpr int kMinCtasPerSm = ESP_MIN_CTAS_UNIFORM; // register budget of the uniform-K evaluation kernel
-constexpr int kMinCtasPerSmGeneral = 4;  // the general kernel: 4 CTAs (16 warps) per SM
+constexpr int kMinCtasPerSmGeneral = ESP_MIN_CTAS_GENERAL;  // register budget of the general kernel
 constexpr int kStageDataBytes = ESP_STAGE_DATA_BYTES;  // option bytes (units + values [+ group]) of a full stage
 
 // Tile flags. A tile is a run of whole jobs of one scenario whose options are contiguous, or one
@@ -83,6 +89,8 @@ ESP_HD int tile_options_for(int R, bool grouped, long long max_k, bool uniform4)
     long long t = (max_k + 31) & ~31LL;
     if (t < 128)
         t = 128;
+    if (ESP_GENERAL_TILE_MAX > 0 && t > ESP_GENERAL_TILE_MAX)
+        t = ESP_GENERAL_TILE_MAX;
     return t > cap ? cap : (int)t;
 }
 
