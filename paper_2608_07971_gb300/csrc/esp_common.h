@@ -31,7 +31,7 @@ namespace esp {
 #define ESP_WARPS_PER_CTA 4
 #endif
 #ifndef ESP_GENERAL_TILE_MAX
-#define ESP_GENERAL_TILE_MAX 0   // cap on the tile of general (CSR) tables; 0: the largest that fits
+#define ESP_GENERAL_TILE_MAX 128 // cap on the tile of general (CSR) tables (larger jobs become chunk tiles)
 #endif
 #ifndef ESP_MIN_CTAS_GENERAL
 #define ESP_MIN_CTAS_GENERAL 4
