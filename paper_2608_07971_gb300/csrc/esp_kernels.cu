@@ -1034,6 +1034,48 @@ __device__ __forceinline__ void prefetch_tile(const DevTable &t, const TileDesc 
     prefetch_l2(reinterpret_cast<const unsigned char *>(t.values) + vlo, (uint32_t)(vhi - vlo));
 }
 
+// Chunk tile of a job larger than a tile: all its options belong to one job, so no segmentation is
+// needed. Each lane folds the options it owns (lane-strided: conflict-free shared loads) into a
+// lane-private state carried across the job's chunks; the job's last chunk reduces the states across
+// the warp once and records the winner (exact resolution from global memory when ambiguous).
+template <int RT, bool G>
+__device__ void process_tile_bigchunk(WarpCtx<RT, G> &c, const TileDesc &d, const StagePtrs &sp, int64_t &big_first,
+                                      Best &big_priv, int lane)
+{
+    const int R = c.R;
+    const int n = d.n_opt;
+    if (d.flags & TILE_BIG_FIRST) {
+        big_first = d.opt_begin;
+        big_priv = best_none();
+    }
+    const int chunk_base = (int)(d.opt_begin - big_first);
+    for (int i = lane; i < n; i += 32) {
+        int32_t u[Cols<RT>::N];
+        const bool dup = load_units_smem<RT>(sp.units + (size_t)i * R, u, R);
+        const double v = sp.vals[i];
+        const int g = G ? (int)sp.grp[i] : 0;
+        const float q = dup ? INFINITY : screen_score<RT, G>(u, v, g, c.sp, R, c.rg);
+        big_priv = combine(big_priv, Best{q, dup ? kIdxNone : chunk_base + i, INFINITY});
+    }
+    if (!(d.flags & TILE_BIG_LAST))
+        return;
+    const Best x = allreduce_best(big_priv);
+    const float thr = __fadd_ru(x.m1, c.sp.e2);
+    const bool amb = c.sp.exact || !(x.m2 > thr);
+    const int K = chunk_base + n;
+    if (!amb) {
+        if (lane == 0) {
+            int32_t uw[Cols<RT>::N];
+            double vw;
+            int gw;
+            load_option<RT, G>(c, false, sp.units, sp.vals, sp.grp, x.idx, big_first, uw, vw, gw);
+            take_winner<RT, G>(c, d.job_begin, x.idx, uw, vw, gw, false, 0.0);
+        }
+    } else {
+        resolve_row<RT, G>(c, lane, 1u, true, sp.units, sp.vals, sp.grp, 0, K, thr, d.job_begin, big_first);
+    }
+}
+
 // Issues the bulk copies of tile d into a stage; lane 0 only. Uniform tables need no job offsets.
 __device__ __forceinline__ void issue_tile(const DevTable &t, const TileDesc &d, unsigned char *stage,
                                            const StageLayout &SL, uint32_t bar, bool need_offsets)
@@ -1151,6 +1193,7 @@ __global__ void __launch_bounds__(kWarpsPerCta * 32, UNI ? kMinCtasPerSm : kMinC
             prefetch_tile(t, pl.tiles[k]);
     int64_t big_first = 0;
     Best big_carry = best_none();
+    Best big_priv = best_none();     // lane-private state of a chunked job
     int failed_at = -1;
     for (int k = k_begin; k < k_end; ++k) {
         if (issued < k_end) {   // refill the stage the previous tile used
@@ -1183,6 +1226,8 @@ __global__ void __launch_bounds__(kWarpsPerCta * 32, UNI ? kMinCtasPerSm : kMinC
                 process_tile_uniform4<RT, G>(c, d, ptrs, lane);
             else if (UNI)
                 process_tile_uniform<RT, G>(c, d, ptrs, lane);
+            else if (d.flags & TILE_BIG)
+                process_tile_bigchunk<RT, G>(c, d, ptrs, big_first, big_priv, lane);
             else
                 process_tile_general<RT, G>(c, d, ptrs, big_first, big_carry, lane);
         }
