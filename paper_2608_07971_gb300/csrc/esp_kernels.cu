@@ -101,8 +101,8 @@ __device__ __forceinline__ void fence_proxy_async()
 // finish instead of hanging.
 __device__ __forceinline__ bool wait_stage(uint32_t bar, uint32_t parity, unsigned int *err)
 {
-    for (uint32_t it = 0; it < 4096u; ++it)
-        if (mbar_try_wait(bar, parity, 1000000u))
+    for (uint32_t it = 0; it < kWaitPolls; ++it)
+        if (mbar_try_wait(bar, parity, kWaitSuspendNs))
             return true;
     atomicOr(err, DEV_ERR_TIMEOUT);
     return false;
