@@ -53,10 +53,10 @@ constexpr int kPrefetchTiles = ESP_PREFETCH_TILES;  // L2 prefetch distance, in 
 constexpr int kUniform4Tile = ESP_UNIFORM4_TILE;    // tile of the 4-options-per-lane path (0: largest)
 constexpr int kMinCtasPerSm = ESP_MIN_CTAS_UNIFORM; // register budget of the uniform-K evaluation kernel
 constexpr int kMinCtasPerSmGeneral = ESP_MIN_CTAS_GENERAL;  // register budget of the general kernel
-constexpr int kStageDataBytes = ESP_STAGE_DATA_BYTES;
+constexpr int kStageDataBytes = ESP_STAGE_DATA_BYTES;  // option bytes (units + values [+ group]) of a full stage
 constexpr uint32_t kWaitSuspendNs = ESP_WAIT_SUSPEND_NS;
 // bound on stage-wait attempts: about 4 s of waiting in total before a timeout is reported
-constexpr uint32_t kWaitPolls = (uint32_t)(4000000000ull / (ESP_WAIT_SUSPEND_NS > 1000 ? ESP_WAIT_SUSPEND_NS : 1000));  // option bytes (units + values [+ group]) of a full stage
+constexpr uint32_t kWaitPolls = (uint32_t)(4000000000ull / (ESP_WAIT_SUSPEND_NS > 1000 ? ESP_WAIT_SUSPEND_NS : 1000));
 
 // Tile flags. A tile is a run of whole jobs of one scenario whose options are contiguous, or one
 // chunk of a job with more options than a tile holds ("big" job).
