@@ -106,15 +106,26 @@ def measured_peak():
         return 6800.0, "fallback"
 
 
+PASS_KERNEL_SOURCES = ("esp_kernels.cu", "esp_device.cuh", "esp_common.h", "esp_kernels.h")
+
+
+def pass_kernel_sha256() -> str:
+    """SHA-256 over the sources the evaluation-pass kernel is compiled from, in a fixed order."""
+    h = hashlib.sha256()
+    for name in PASS_KERNEL_SOURCES:
+        with open(os.path.join(ROOT, "paper_2608_07971_gb300", "csrc", name), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()
+
+
 def kernel_traffic(n_opt_launch: int):
     """DRAM bytes per evaluation pass from the committed ncu summary, scaled to this workload's
     option count, or None when the kernel source changed since the counters were taken."""
     path = os.path.join(ROOT, "profiles", "k_pass_traffic.json")
-    src = os.path.join(ROOT, "paper_2608_07971_gb300", "csrc", "esp_kernels.cu")
     try:
         with open(path) as f:
             rec = json.load(f)
-        sha = hashlib.sha256(open(src, "rb").read()).hexdigest()
+        sha = pass_kernel_sha256()
         if rec.get("kernel_source_sha256") != sha:
             return None
         return float(rec["dram_bytes_per_launch"]) / float(rec["options_per_launch"]) * n_opt_launch

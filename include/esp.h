@@ -63,6 +63,13 @@ typedef enum { ESP_STEP_FIXED = 0, ESP_STEP_INV_SQRT = 1 } esp_step_rule;
                                           by the pass's last warp per scenario (same results) */
 #define ESP_FLAG_PASS_EVENTS 0x4u      /* record a CUDA event pair around every evaluation-pass launch (inside the
                                           solve's CUDA graph on a non-default stream); read with esp_pass_times */
+#define ESP_FLAG_RESIDENT 0x8u         /* run all rounds of a scenario in one launch, its table held in the shared
+                                          memory of one thread-block cluster for the whole solve (no table bytes
+                                          read from HBM after the first round). Taken when the table has no group
+                                          column and each scenario fits in a cluster (up to 16 CTAs of up to about
+                                          227 KB); otherwise the streaming path runs. Same results either way.
+                                          esp_last_launch_count tells which ran (3: resident); with
+                                          ESP_FLAG_PASS_EVENTS the one resident launch counts as one pass */
 
 typedef struct {
     double eta0;            /* > 0, finite */

@@ -33,6 +33,13 @@ esp_status esp_debug_plan(const int64_t *job_offsets, int32_t S, int32_t J, int3
                           int32_t *tiles, int32_t tiles_cap, int32_t *warp_begin, int32_t warps_cap,
                           int32_t *n_tiles, int32_t *n_warps);
 
+/* Cluster size of the resident kernel (ESP_FLAG_RESIDENT) for the loaded table. force_cs: 0 keeps the
+ * automatic choice; 1, 2, 4, 8 or 16 forces that many CTAs per scenario for later solves (the size must
+ * fit the table). *cs receives the size solves use and *clusters how many such clusters the device
+ * holds at once (either may be NULL). ESP_ERR_UNSUPPORTED: the table cannot run resident at all;
+ * ESP_ERR_INVALID_ARG: force_cs is not a size that fits. */
+esp_status esp_debug_resident(esp_ctx *ctx, int32_t force_cs, int32_t *cs, int32_t *clusters);
+
 #ifdef __cplusplus
 }
 #endif

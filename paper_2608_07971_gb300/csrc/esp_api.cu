@@ -23,10 +23,11 @@ struct GraphKey {
     uint32_t flags = 0;
     const void *lt = nullptr, *dt = nullptr, *ht = nullptr, *gt = nullptr;
     bool has_l0 = false;
+    int res = -1;   // resident option in use, -1: streaming
     bool operator==(const GraphKey &o) const
     {
         return eta0 == o.eta0 && tol == o.tol && step == o.step && mode == o.mode && T == o.T && flags == o.flags &&
-               lt == o.lt && dt == o.dt && ht == o.ht && gt == o.gt && has_l0 == o.has_l0;
+               lt == o.lt && dt == o.dt && ht == o.ht && gt == o.gt && has_l0 == o.has_l0 && res == o.res;
     }
 };
 
@@ -63,6 +64,18 @@ struct esp_ctx {
     int32_t *scen_warps = nullptr;   // warps owning tiles of each scenario
     unsigned int *arrive = nullptr;  // per-scenario arrivals of the round pass in flight
     int32_t n_warps = 0, tile_opt = 0, grid = 0, uniform_k = 0;
+
+    // cluster-resident kernel (tables without a group column): every cluster size that fits
+    struct ResOption {
+        ResPlan plan = {};
+        int64_t smem = 0;
+        int64_t n_max = 0;      // most options in one CTA's slice
+        int32_t clusters = 0;   // clusters the device holds at once
+    };
+    std::vector<ResOption> res;
+    int32_t *res_cuts = nullptr;
+    int res_auto = -1;     // index into res of the automatic choice (-1: none fits)
+    int res_force = -1;    // index forced through esp_debug_resident (-1: automatic)
 
     double *lam = nullptr, *p64 = nullptr, *job_val = nullptr, *job_min = nullptr;
     double *best_dual = nullptr, *primal = nullptr, *dual = nullptr, *lambda0 = nullptr;
@@ -144,6 +157,10 @@ void release_table(esp_ctx *ctx)
     for (void *p : ctx->table_bufs)
         cudaFree(p);
     ctx->table_bufs.clear();
+    ctx->res.clear();
+    ctx->res_cuts = nullptr;
+    ctx->res_auto = -1;
+    ctx->res_force = -1;
     ctx->loaded = false;
     ctx->solved = false;
 }
@@ -389,6 +406,62 @@ esp_status load_common(esp_ctx *ctx, int32_t S, int32_t J, int32_t R, int32_t P,
     ESP_CUDA(cudaMemcpyAsync(ctx->warp_begin, plan.warp_begin.data(), plan.warp_begin.size() * sizeof(int32_t),
                              cudaMemcpyHostToDevice, ctx->stream));
 
+    // resident kernel: every cluster size whose slices fit one CTA's shared memory
+    if (!grouped && J >= 1) {
+        int optin = 0;
+        ESP_CUDA(cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, ctx->device));
+        const int32_t rk = (min_k == max_k) ? (int32_t)max_k : 0;
+        std::vector<ResShape> shapes;
+        for (int32_t cs = 1; cs <= kResMaxCluster; cs *= 2) {
+            ResShape sh;
+            if (!plan_resident(off_host, S, J, cs, sh) || sh.n_max > (1 << 24))
+                continue;
+            esp_ctx::ResOption o;
+            o.plan.cs = cs;
+            o.plan.k = rk;
+            o.plan.m_pad = (sh.m_max + 31) & ~31;
+            o.plan.n_cap = (sh.n_max + 1) & ~1LL;
+            o.smem = res_smem_bytes(R, o.plan);
+            o.n_max = sh.n_max;
+            if (o.smem > optin)
+                continue;
+            int nc = 0;
+            ESP_CUDA(res_max_clusters(dev_table(ctx), o.plan, ctx->small_units != 0, &nc));
+            if (nc < 1)
+                continue;
+            o.clusters = nc;
+            ctx->res.push_back(o);
+            shapes.push_back(std::move(sh));
+        }
+        if (!ctx->res.empty()) {
+            size_t total = 0;
+            for (const ResShape &sh : shapes)
+                total += sh.cuts.size();
+            ALLOC(ctx->res_cuts, total);
+            size_t at = 0;
+            for (size_t i = 0; i < shapes.size(); ++i) {
+                ESP_CUDA(cudaMemcpyAsync(ctx->res_cuts + at, shapes[i].cuts.data(), shapes[i].cuts.size() * sizeof(int32_t),
+                                         cudaMemcpyHostToDevice, ctx->stream));
+                ctx->res[i].plan.cuts = ctx->res_cuts + at;
+                at += shapes[i].cuts.size();
+            }
+            ESP_CUDA(cudaStreamSynchronize(ctx->stream));
+            // automatic size: most scenario-rounds per microsecond under a simple cost model, a fixed
+            // cost per round (barriers and the price update; smaller without a cluster) plus the
+            // slice's options at the SM's screening rate; ties keep the smaller cluster
+            double best = -1.0;
+            for (size_t i = 0; i < ctx->res.size(); ++i) {
+                const esp_ctx::ResOption &o = ctx->res[i];
+                const double round_us = (o.plan.cs == 1 ? 0.6 : 1.0) + 7.8e-5 * (double)o.n_max;
+                const double rate = (double)std::min<int64_t>(S, o.clusters) / round_us;
+                if (rate > best * 1.02) {
+                    best = rate;
+                    ctx->res_auto = (int)i;
+                }
+            }
+        }
+    }
+
     // solve state
     const size_t SP = (size_t)S * P, SJ = (size_t)n_jobs;
     ALLOC(ctx->lam, SP);
@@ -432,7 +505,7 @@ esp_status check_params(const esp_ctx *ctx, const esp_params *p)
         return ESP_ERR_INVALID_ARG;
     if (!(p->tol >= 0.0) || !std::isfinite(p->tol))
         return ESP_ERR_INVALID_ARG;
-    if (p->flags & ~(uint32_t)(ESP_FLAG_EXACT_ONLY | ESP_FLAG_PER_ROUND_LAUNCH | ESP_FLAG_PASS_EVENTS))
+    if (p->flags & ~(uint32_t)(ESP_FLAG_EXACT_ONLY | ESP_FLAG_PER_ROUND_LAUNCH | ESP_FLAG_PASS_EVENTS | ESP_FLAG_RESIDENT))
         return ESP_ERR_INVALID_ARG;
     if (p->lambda0) {
         const size_t n = (size_t)ctx->S * ctx->P;
@@ -471,9 +544,10 @@ esp_status enqueue_solve(esp_ctx *ctx, const esp_params *p, const DevState &st, 
     const bool use_graph = ctx->stream != nullptr;   // the legacy default stream cannot be captured
     std::vector<cudaEvent_t> &pool = use_graph ? ctx->graph_pool : ctx->ev_pool;
     size_t pool_used = use_graph ? 0 : ctx->ev_used;
-    auto pass = [&](int r, PassKind kind) -> cudaError_t {
+    const int ri = (p->flags & ESP_FLAG_RESIDENT) ? (ctx->res_force >= 0 ? ctx->res_force : ctx->res_auto) : -1;
+    auto timed_launch = [&](auto &&launch) -> cudaError_t {
         if (!timed)
-            return launch_pass(t, st, pl, a, r, kind, ctx->grid, ctx->stream);
+            return launch();
         while (pool.size() < pool_used + 2) {
             cudaEvent_t ev;
             cudaError_t e = cudaEventCreate(&ev);
@@ -487,13 +561,24 @@ esp_status enqueue_solve(esp_ctx *ctx, const esp_params *p, const DevState &st, 
         const unsigned int rf = use_graph ? cudaEventRecordExternal : cudaEventRecordDefault;
         cudaError_t e = cudaEventRecordWithFlags(e0, ctx->stream, rf);
         if (e == cudaSuccess)
-            e = launch_pass(t, st, pl, a, r, kind, ctx->grid, ctx->stream);
+            e = launch();
         if (e == cudaSuccess)
             e = cudaEventRecordWithFlags(e1, ctx->stream, rf);
         return e;
     };
+    auto pass = [&](int r, PassKind kind) -> cudaError_t {
+        return timed_launch([&]() { return launch_pass(t, st, pl, a, r, kind, ctx->grid, ctx->stream); });
+    };
     auto issue = [&]() -> cudaError_t {
         cudaError_t e = launch_init(t, st, a, has_l0 ? ctx->lambda0 : nullptr, ctx->stream);
+        if (ri >= 0) {
+            const ResPlan &rp = ctx->res[ri].plan;
+            if (e == cudaSuccess)
+                e = timed_launch([&]() { return launch_resident(t, st, rp, a, ctx->stream); });
+            if (e == cudaSuccess)
+                e = launch_objectives(t, st, a, ctx->stream);
+            return e;
+        }
         for (int r = 0; r < T && e == cudaSuccess; ++r) {
             if (ctx->grid > 0)
                 e = pass(r, PASS_ROUND);
@@ -506,7 +591,7 @@ esp_status enqueue_solve(esp_ctx *ctx, const esp_params *p, const DevState &st, 
             e = launch_objectives(t, st, a, ctx->stream);
         return e;
     };
-    ctx->last_launches = 3 + (fused ? 1LL : 2LL) * T - (ctx->grid > 0 ? 0 : (T + 1));
+    ctx->last_launches = ri >= 0 ? 3 : 3 + (fused ? 1LL : 2LL) * T - (ctx->grid > 0 ? 0 : (T + 1));
     ctx->last_T = T;
 
     GraphKey key;
@@ -521,6 +606,7 @@ esp_status enqueue_solve(esp_ctx *ctx, const esp_params *p, const DevState &st, 
     key.ht = st.hash_trace;
     key.gt = st.dual_trace;
     key.has_l0 = has_l0;
+    key.res = ri;
 
     if (!use_graph) {
         ESP_CUDA(issue());
@@ -942,6 +1028,34 @@ esp_status esp_debug_stats(esp_ctx *ctx, int64_t *resolutions, int64_t *marked, 
 int32_t esp_debug_tile_options(int32_t R, int32_t grouped)
 {
     return tile_options(R, grouped != 0);
+}
+
+esp_status esp_debug_resident(esp_ctx *ctx, int32_t force_cs, int32_t *cs, int32_t *clusters)
+{
+    esp_status st = check_ctx(ctx);
+    if (st != ESP_OK)
+        return st;
+    if (!ctx->loaded)
+        return ESP_ERR_NOT_LOADED;
+    if (ctx->res.empty())
+        return ESP_ERR_UNSUPPORTED;
+    if (force_cs != 0) {
+        int found = -1;
+        for (size_t i = 0; i < ctx->res.size(); ++i)
+            if (ctx->res[i].plan.cs == force_cs)
+                found = (int)i;
+        if (found < 0)
+            return ESP_ERR_INVALID_ARG;
+        ctx->res_force = found;
+    } else {
+        ctx->res_force = -1;
+    }
+    const esp_ctx::ResOption &o = ctx->res[ctx->res_force >= 0 ? ctx->res_force : ctx->res_auto];
+    if (cs)
+        *cs = o.plan.cs;
+    if (clusters)
+        *clusters = o.clusters;
+    return ESP_OK;
 }
 
 esp_status esp_debug_plan(const int64_t *job_offsets, int32_t S, int32_t J, int32_t tile_opt, int32_t max_warps,

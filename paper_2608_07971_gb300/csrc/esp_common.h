@@ -42,6 +42,12 @@ namespace esp {
 #ifndef ESP_V32_HW
 #define ESP_V32_HW 0          // 1: fp64 -> fp32 of values by the conversion instruction (round to nearest)
 #endif
+#ifndef ESP_RES_WARPS
+#define ESP_RES_WARPS 8       // warps per CTA of the cluster-resident kernel
+#endif
+#ifndef ESP_RES_MIN_CTAS
+#define ESP_RES_MIN_CTAS 2    // register budget of the resident kernel: CTAs per SM it must allow
+#endif
 #ifndef ESP_I2F_COLS
 #define ESP_I2F_COLS 16       // unit columns r < ESP_I2F_COLS use the int-to-float instruction
 #endif
@@ -57,6 +63,32 @@ constexpr int kStageDataBytes = ESP_STAGE_DATA_BYTES;  // option bytes (units + 
 constexpr uint32_t kWaitSuspendNs = ESP_WAIT_SUSPEND_NS;
 // bound on stage-wait attempts: about 4 s of waiting in total before a timeout is reported
 constexpr uint32_t kWaitPolls = (uint32_t)(4000000000ull / (ESP_WAIT_SUSPEND_NS > 1000 ? ESP_WAIT_SUSPEND_NS : 1000));
+
+constexpr int kResWarps = ESP_RES_WARPS;
+constexpr int kResMaxCluster = 16;   // CTAs per cluster of the resident kernel (16 is non-portable)
+constexpr int kResCols = kMaxR + 2;  // words of a demand partial: R columns, fingerprint, dual sum
+
+// Shared-memory layout of one CTA of the resident kernel: the CTA's slice of a scenario's table
+// (uniform K: option k of slice job jj at slot k * m_pad + jj, so a warp reading one option of 32
+// consecutive jobs touches 32 consecutive words; general: CSR order with local job offsets), the
+// per-warp and per-cluster demand partials, and the prices of the current round.
+struct ResLayout {
+    int64_t vals, units, loff, wpart, cpart, prices, bytes;
+};
+
+ESP_HD ResLayout res_layout(int R, int K, int m_pad, long long n_cap, int cs)
+{
+    ResLayout L;
+    const long long slots = K > 0 ? (long long)K * m_pad : n_cap;
+    L.vals = 0;
+    L.units = (slots * 8 + 15) & ~15LL;
+    L.loff = L.units + ((slots * R * 4 + 15) & ~15LL);
+    L.wpart = L.loff + (K > 0 ? 0 : (((long long)m_pad + 1) * 4 + 15) & ~15LL);
+    L.cpart = L.wpart + (long long)kResWarps * kResCols * 8;
+    L.prices = L.cpart + 2LL * cs * kResCols * 8;
+    L.bytes = L.prices + kMaxR * 8 + kMaxR * 4 + 16;
+    return L;
+}
 
 // Tile flags. A tile is a run of whole jobs of one scenario whose options are contiguous, or one
 // chunk of a job with more options than a tile holds ("big" job).

@@ -29,22 +29,15 @@
 #include <cstdint>
 #include <cuda_runtime.h>
 
+#include "esp_device.cuh"
 #include "esp_kernels.h"
 
 namespace esp {
 
 namespace {
 
-constexpr unsigned FULL = 0xffffffffu;
-constexpr int kIdxNone = 0x7fffffff;
-
 // ---------------------------------------------------------------------------------------------
 // PTX helpers: mbarrier + 1-D bulk copy (TMA engine), sm_90+ forms that sm_103a accepts.
-
-__device__ __forceinline__ uint32_t smem_u32(const void *p)
-{
-    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
 
 __device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count)
 {
@@ -108,13 +101,6 @@ __device__ __forceinline__ bool wait_stage(uint32_t bar, uint32_t parity, unsign
     return false;
 }
 
-__device__ __forceinline__ uint64_t splitmix64_mix(uint64_t z)
-{
-    z = (z ^ (z >> 30)) * 0xbf58476d1ce4e5b9ULL;
-    z = (z ^ (z >> 27)) * 0x94d049bb133111ebULL;
-    return z ^ (z >> 31);
-}
-
 // ---------------------------------------------------------------------------------------------
 // Scoring. Both chains run r = 0 .. R-1 with one correctly rounded fused multiply-add per column.
 
@@ -132,38 +118,6 @@ struct ScenarioPrices {
     bool skip;             // scenario already stopped
     bool small_units;      // every unit of the table is below 2^23
 };
-
-// fp32 value of v truncated toward zero (relative error < 2^-23) for 2^-100 <= |v| <= 2^100, and 0
-// (absolute error < 2^-100) below; integer ops only (a double-to-float conversion would run on the
-// fp64 pipe). Scenarios with larger values are evaluated exactly and never use the result.
-__device__ __forceinline__ float f32_of_f64(double v)
-{
-    const uint32_t hi = (uint32_t)__double2hiint(v);
-    const uint32_t lo = (uint32_t)__double2loint(v);
-    // rebase the exponent (1023 -> 127); the sign bit is untouched for |v| >= 2^-127
-    const uint32_t t = hi - (896u << 20);
-    // 8 exponent and 23 mantissa bits; bit 31 comes out 0 because the rebased exponent is < 256
-    const uint32_t bits = __funnelshift_l(lo, t, 3) | (hi & 0x80000000u);
-    return ((hi << 1) >= (923u << 21)) ? __uint_as_float(bits) : 0.0f;
-}
-
-// Exact fp32 value of a unit count: 2^23 + u is exact in fp32 for 0 <= u < 2^23, so one OR and one
-// subtraction replace the int-to-float conversion; larger tables use the conversion instruction.
-__device__ __forceinline__ float f32_of_units(int32_t u, bool small)
-{
-    return small ? (__uint_as_float(0x4b000000u | (uint32_t)u) - 8388608.0f) : __int2float_rn(u);
-}
-
-// The fp32 value used by the screen: truncated by integer ops, or (ESP_V32_HW) rounded by the
-// conversion instruction; both are within 2^-23 relative (or 2^-100 absolute) of v in range.
-__device__ __forceinline__ float screen_value(double v)
-{
-#if ESP_V32_HW
-    return __double2float_rn(v);
-#else
-    return f32_of_f64(v);
-#endif
-}
 
 template <int RT, bool G>
 __device__ __forceinline__ float screen_score(const int32_t *u, double v, int g, const ScenarioPrices &sp, int R,
@@ -237,22 +191,6 @@ __device__ __forceinline__ bool load_units_global(const int32_t *p, int32_t *u, 
 // ---------------------------------------------------------------------------------------------
 // Price update (Eq. price_update), one warp per scenario, and the screen bound of the new prices.
 
-__device__ __forceinline__ double warp_sum_fixed(double x)
-{
-#pragma unroll
-    for (int d = 16; d >= 1; d >>= 1)
-        x += __shfl_xor_sync(FULL, x, d);
-    return x;
-}
-
-__device__ __forceinline__ double warp_max(double x)
-{
-#pragma unroll
-    for (int d = 16; d >= 1; d >>= 1)
-        x = fmax(x, __shfl_xor_sync(FULL, x, d));
-    return x;
-}
-
 // Effective prices p = lambda (RAW) or lambda / C (NORMALIZED), their fp32 copy, and the bound E.
 __device__ void set_prices(const DevTable &t, const DevState &st, const SolveArgs &a, int s, int lane)
 {
@@ -260,7 +198,7 @@ __device__ void set_prices(const DevTable &t, const DevState &st, const SolveArg
     bool huge = false;
     for (int k = lane; k < P; k += 32) {
         const double lam = st.lam[(size_t)s * P + k];
-        const double p = (a.mode == 1) ? lam / (double)t.cap[(size_t)s * P + k] : lam;
+        const double p = effective_price(lam, t.cap[(size_t)s * P + k], a.mode);
         st.p64[(size_t)s * P + k] = p;
         st.p32[(size_t)s * P + k] = __double2float_rn(p);
         huge |= !(p <= 0x1p100);
@@ -280,16 +218,8 @@ __device__ void set_prices(const DevTable &t, const DevState &st, const SolveArg
     }
     const double M = st.vmax[s] + warp_sum_fixed(term);
     huge = __any_sync(FULL, huge);
-    if (lane == 0) {
-        float e;
-        if (a.exact_only || huge || !(M <= 0x1p100)) {
-            e = INFINITY;
-        } else {
-            const double eb = (4.0 * R + 16.0) * 0x1p-24 * M * (1.0 + 0x1p-20) + 0x1p-99;
-            e = __double2float_ru(eb);
-        }
-        st.ebound[s] = e;
-    }
+    if (lane == 0)
+        st.ebound[s] = screen_bound(M, R, a.exact_only || huge);
 }
 
 __global__ void k_init(DevTable t, DevState st, SolveArgs a, const double *lambda0)
@@ -348,9 +278,7 @@ __device__ void update_scenario(const DevTable &t, const DevState &st, const Sol
         st.hash[s] = 0ull;
     }
 
-    double eta = a.eta0;
-    if (a.step == 1)
-        eta = a.eta0 / sqrt((double)(round + 1));
+    const double eta = step_size(a.eta0, a.step, round);
     bool bad = false;
     double dmax = 0.0, amax = 0.0;
     for (int k = lane; k < P; k += 32) {
@@ -358,12 +286,8 @@ __device__ void update_scenario(const DevTable &t, const DevState &st, const Sol
         const long long C = t.cap[sp + k];
         if (st.dem_trace)
             st.dem_trace[((size_t)s * T + round) * P + k] = U;
-        double excess = (double)(U - C);
-        if (a.mode == 1)
-            excess = excess / (double)C;
         const double lam = st.lam[sp + k];
-        const double moved = __fma_rn(eta, excess, lam);
-        const double nl = moved > 0.0 ? moved : 0.0;
+        const double nl = price_step(lam, U, C, eta, a.mode);
         bad |= !isfinite(nl);
         dmax = fmax(dmax, fabs(nl - lam));
         amax = fmax(amax, fabs(lam));
@@ -383,11 +307,7 @@ __device__ void update_scenario(const DevTable &t, const DevState &st, const Sol
     for (int k = lane; k < P; k += 32) {
         const long long U = (long long)__ldcg(st.U + sp + k);
         const long long C = t.cap[sp + k];
-        double excess = (double)(U - C);
-        if (a.mode == 1)
-            excess = excess / (double)C;
-        const double moved = __fma_rn(eta, excess, st.lam[sp + k]);
-        const double nl = moved > 0.0 ? moved : 0.0;
+        const double nl = price_step(st.lam[sp + k], U, C, eta, a.mode);
         st.lam[sp + k] = nl;
         st.U[sp + k] = 0ull;
         if (st.lam_trace)
@@ -554,20 +474,6 @@ __device__ __forceinline__ void take_winner(WarpCtx<RT, G> &c, int64_t job, int 
         }
     }
     take_winner_extras<RT, G>(c, job, local, u, v, g, have_s64, s64);
-}
-
-// Signed-integer key with the order of the doubles (no NaN occurs); -0.0 and +0.0 share key 0.
-__device__ __forceinline__ long long order_key(double x)
-{
-    long long b = __double_as_longlong(x);
-    if ((b << 1) == 0)
-        b = 0;
-    return b ^ ((b >> 63) & 0x7fffffffffffffffLL);
-}
-
-__device__ __forceinline__ double key_value(long long k)
-{
-    return __longlong_as_double(k ^ ((k >> 63) & 0x7fffffffffffffffLL));
 }
 
 // Data of tile-local option o (stage) or of job option o (global, gfirst = the job's first option).

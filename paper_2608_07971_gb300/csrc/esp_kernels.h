@@ -68,6 +68,16 @@ struct SolveArgs {
 
 enum PassKind : int32_t { PASS_ROUND = 0, PASS_FINAL = 1 };
 
+// Plan of the cluster-resident kernel: one cluster of cs CTAs per scenario; CTA c of scenario s holds
+// the scenario-local jobs [cuts[s*(cs+1) + c], cuts[s*(cs+1) + c + 1]) in shared memory.
+struct ResPlan {
+    const int32_t *cuts;
+    int32_t cs;
+    int32_t k;          // > 0: every job has k options (interleaved layout); 0: CSR layout
+    int32_t m_pad;      // job slots of a slice, a multiple of 32
+    int64_t n_cap;      // option slots of a slice (CSR layout)
+};
+
 // Dynamic shared memory per CTA of the evaluation kernel.
 int pass_smem_bytes(int R, bool grouped, int P, int tile_opt);
 
@@ -86,6 +96,15 @@ cudaError_t launch_pass(const DevTable &t, const DevState &st, const DevPlan &pl
                         int round, PassKind kind, int grid, cudaStream_t stream);
 cudaError_t launch_update(const DevTable &t, const DevState &st, const SolveArgs &a, int round,
                           cudaStream_t stream);
+// Dynamic shared memory of one resident CTA, and the clusters of the resident kernel that can be
+// resident at once (0: the shape cannot run; needs the device). res_max_clusters also sets the
+// kernel's function attributes and must run (at load time) before its first launch.
+int64_t res_smem_bytes(int R, const ResPlan &rp);
+cudaError_t res_max_clusters(const DevTable &t, const ResPlan &rp, bool small_units, int *n);
+// init must have run; writes everything the final pass and the price updates of the streaming path
+// write (prices, selection, values, minimal reduced costs, final demand, counters, traces).
+cudaError_t launch_resident(const DevTable &t, const DevState &st, const ResPlan &rp, const SolveArgs &a,
+                            cudaStream_t stream);
 cudaError_t launch_objectives(const DevTable &t, const DevState &st, const SolveArgs &a, cudaStream_t stream);
 
 }  // namespace esp

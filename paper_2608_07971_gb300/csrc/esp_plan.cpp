@@ -134,4 +134,33 @@ bool check_plan(const int64_t *off, int32_t S, int32_t J, const Plan &p)
     return big_next_opt < 0 && next_job == n_jobs;
 }
 
+bool plan_resident(const int64_t *off, int32_t S, int32_t J, int32_t cs, ResShape &out)
+{
+    out.cs = cs;
+    out.m_max = 0;
+    out.n_max = 0;
+    out.cuts.assign((size_t)S * (cs + 1), 0);
+    if (cs < 1 || S < 1 || J < 1)
+        return false;
+    for (int32_t s = 0; s < S; ++s) {
+        const int64_t *o = off + (int64_t)s * J;   // o[0 .. J]
+        const int64_t N = o[J] - o[0];
+        if (N < J)
+            return false;
+        int32_t *cut = out.cuts.data() + (size_t)s * (cs + 1);
+        cut[0] = 0;
+        cut[cs] = J;
+        for (int32_t c = 1; c < cs; ++c) {
+            const int64_t target = o[0] + (int64_t)((__int128)N * c / cs);
+            int32_t j = (int32_t)(std::lower_bound(o, o + J, target) - o);
+            cut[c] = std::max(j, cut[c - 1]);
+        }
+        for (int32_t c = 0; c < cs; ++c) {
+            out.m_max = std::max(out.m_max, cut[c + 1] - cut[c]);
+            out.n_max = std::max<int64_t>(out.n_max, o[cut[c + 1]] - o[cut[c]]);
+        }
+    }
+    return true;
+}
+
 }  // namespace esp

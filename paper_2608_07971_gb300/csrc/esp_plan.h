@@ -25,4 +25,17 @@ bool plan_tiles(const int64_t *job_off, int32_t S, int32_t J, int32_t tile_opt, 
 // every tile inside the table. Returns false on the first violation.
 bool check_plan(const int64_t *job_off, int32_t S, int32_t J, const Plan &p);
 
+// Slices of the cluster-resident kernel: every scenario's jobs split into cs contiguous runs of about
+// equal option counts, run c starting at the first job whose first option lies at least
+// floor(c * N_s / cs) options into the scenario (N_s = options of scenario s).
+struct ResShape {
+    int32_t cs = 0;
+    int32_t m_max = 0;                // most jobs in one slice
+    int64_t n_max = 0;                // most options in one slice
+    std::vector<int32_t> cuts;        // S * (cs + 1) scenario-local job indices
+};
+
+// Fills out for cs CTAs per scenario. Returns false on inconsistent offsets.
+bool plan_resident(const int64_t *job_off, int32_t S, int32_t J, int32_t cs, ResShape &out);
+
 }  // namespace esp

@@ -21,13 +21,13 @@ ESP_OK, ESP_ERR_INVALID_ARG, ESP_ERR_OVERFLOW, ESP_ERR_OOM, ESP_ERR_CUDA = 0, 1,
 ESP_ERR_NOT_LOADED, ESP_ERR_TIMEOUT, ESP_ERR_STATE, ESP_ERR_UNSUPPORTED = 5, 6, 7, 8
 ESP_PRICE_RAW, ESP_PRICE_NORMALIZED = 0, 1
 ESP_STEP_FIXED, ESP_STEP_INV_SQRT = 0, 1
-ESP_FLAG_EXACT_ONLY, ESP_FLAG_PER_ROUND_LAUNCH, ESP_FLAG_PASS_EVENTS = 0x1, 0x2, 0x4
+ESP_FLAG_EXACT_ONLY, ESP_FLAG_PER_ROUND_LAUNCH, ESP_FLAG_PASS_EVENTS, ESP_FLAG_RESIDENT = 0x1, 0x2, 0x4, 0x8
 
 EXPORTED = [
     "esp_create", "esp_set_stream", "esp_load_options", "esp_load_options_device", "esp_solve",
     "esp_solve_async", "esp_get_result", "esp_get_prices", "esp_get_selection", "esp_get_demand",
     "esp_evaluate", "esp_last_launch_count", "esp_pass_times", "esp_status_string", "esp_destroy",
-    "esp_debug_tile_options", "esp_debug_plan", "esp_debug_stats", "esp_evaluate_noalloc",
+    "esp_debug_tile_options", "esp_debug_plan", "esp_debug_stats", "esp_debug_resident", "esp_evaluate_noalloc",
 ]
 
 
@@ -84,6 +84,7 @@ def load_library(path: Optional[str] = None):
         "esp_destroy": ([vp], None),
         "esp_debug_tile_options": ([i32, i32], i32),
         "esp_debug_stats": ([vp, ctypes.POINTER(i64), ctypes.POINTER(i64), i32], st),
+        "esp_debug_resident": ([vp, i32, ctypes.POINTER(i32), ctypes.POINTER(i32)], st),
         "esp_debug_plan": ([vp, i32, i32, i32, i32, vp, i32, vp, i32, ctypes.POINTER(i32), ctypes.POINTER(i32)], st),
         "esp_evaluate_noalloc": ([i32, i32, i32, vp, vp, vp, vp, vp, i32, vp, vp, vp, vp], st),
     }
@@ -196,6 +197,18 @@ def esp_debug_stats(ctx: int, reset: bool = True):
     _check(load_library().esp_debug_stats(ctx, ctypes.byref(r), ctypes.byref(m), 1 if reset else 0),
            "esp_debug_stats")
     return r.value, m.value
+
+
+def esp_debug_resident(ctx: int, force_cs: int = 0):
+    """(cluster size, co-resident clusters) of the resident kernel for the loaded table; force_cs
+    1/2/4/8/16 forces that size for later solves, 0 restores the automatic choice. None when the
+    table cannot run resident."""
+    cs, nc = ctypes.c_int32(), ctypes.c_int32()
+    status = load_library().esp_debug_resident(ctx, int(force_cs), ctypes.byref(cs), ctypes.byref(nc))
+    if status == ESP_ERR_UNSUPPORTED:
+        return None
+    _check(status, "esp_debug_resident")
+    return cs.value, nc.value
 
 
 def esp_destroy(ctx: int) -> None:
