@@ -33,6 +33,29 @@ esp_status esp_debug_plan(const int64_t *job_offsets, int32_t S, int32_t J, int3
                           int32_t *tiles, int32_t tiles_cap, int32_t *warp_begin, int32_t warps_cap,
                           int32_t *n_tiles, int32_t *n_warps);
 
+/* Sorted layout of a general table (jobs of varying size, no group column), as esp_load_options
+ * builds it for the evaluation pass: per scenario the jobs of 3..128 options padded to a multiple
+ * of 4 and ordered by padded size (this part first for every scenario), then per scenario the
+ * larger jobs, then per scenario the 2-option and the 1-option jobs. Host buffers:
+ *   off   S*J + 1 int64: padded option offsets in sorted order
+ *   jmap  S*J int32: original global job index of each sorted job
+ *   scen  S*J int32: scenario of each sorted job
+ *   runk  S*J int32: options (padded) of the jobs of the sorted job's run, 0 for a large job
+ * Returns ESP_ERR_INVALID_ARG for inconsistent offsets or more than 2^31 - 1 jobs. */
+esp_status esp_debug_sort_layout(const int64_t *job_offsets, int32_t S, int32_t J, int64_t *off, int32_t *jmap,
+                                 int32_t *scen, int32_t *runk);
+
+/* esp_debug_plan for a sorted layout (the arrays esp_debug_sort_layout returns): tiles never mix
+ * scenarios or runs, and a tile of a run has flag bit 3 set and its jobs' option count in bits 8..15
+ * of its flags. Same buffers and errors as esp_debug_plan. */
+esp_status esp_debug_plan_runs(const int64_t *off, const int32_t *scen, const int32_t *runk, int32_t S, int32_t J,
+                               int32_t tile_opt, int32_t max_warps, int32_t *tiles, int32_t tiles_cap,
+                               int32_t *warp_begin, int32_t warps_cap, int32_t *n_tiles, int32_t *n_warps);
+
+/* enable = 0 makes later esp_load_options calls on this context evaluate general tables in their
+ * original layout (the segmented path) instead of the sorted one; 1 restores the default. */
+esp_status esp_debug_set_sorted_layout(esp_ctx *ctx, int32_t enable);
+
 /* Cluster size of the resident kernel (ESP_FLAG_RESIDENT) for the loaded table. force_cs: 0 keeps the
  * automatic choice; 1, 2, 4, 8 or 16 forces that many CTAs per scenario for later solves (the size must
  * fit the table). *cs receives the size solves use and *clusters how many such clusters the device

@@ -54,6 +54,14 @@ struct esp_ctx {
     int32_t *units = nullptr;
     double *values = nullptr;
     int64_t *off = nullptr;
+    // sorted layout of a general table (the evaluation pass reads it; outputs use jmap)
+    bool sorted_enabled = ESP_SORTED_LAYOUT != 0;   // later loads build it (esp_debug_set_sorted_layout)
+    bool sorted = false;
+    int64_t s_n_opt = 0;
+    int32_t *s_units = nullptr;
+    double *s_values = nullptr;
+    int64_t *s_off = nullptr;
+    int32_t *s_jmap = nullptr;
     uint16_t *group = nullptr;
     int64_t *cap = nullptr;
     double *vmax = nullptr;
@@ -159,6 +167,12 @@ void release_table(esp_ctx *ctx)
     ctx->table_bufs.clear();
     ctx->res.clear();
     ctx->res_cuts = nullptr;
+    ctx->sorted = false;
+    ctx->s_n_opt = 0;
+    ctx->s_units = nullptr;
+    ctx->s_values = nullptr;
+    ctx->s_off = nullptr;
+    ctx->s_jmap = nullptr;
     ctx->res_auto = -1;
     ctx->res_force = -1;
     ctx->loaded = false;
@@ -203,6 +217,21 @@ DevTable dev_table(const esp_ctx *c)
     t.r_global = c->rg;
     t.n_groups = c->n_groups;
     t.small_units = c->small_units;
+    t.jmap = nullptr;
+    return t;
+}
+
+// The table the evaluation pass reads: the sorted layout when there is one, else the original.
+DevTable pass_table(const esp_ctx *c)
+{
+    DevTable t = dev_table(c);
+    if (c->sorted) {
+        t.units = c->s_units;
+        t.values = c->s_values;
+        t.job_off = c->s_off;
+        t.n_opt = c->s_n_opt;
+        t.jmap = c->s_jmap;
+    }
     return t;
 }
 
@@ -367,6 +396,28 @@ esp_status load_common(esp_ctx *ctx, int32_t S, int32_t J, int32_t R, int32_t P,
         min_k = std::min<int64_t>(min_k, k);
     }
     ctx->uniform_k = (!grouped && min_k == max_k && max_k <= 32 && (max_k & (max_k - 1)) == 0) ? (int32_t)max_k : 0;
+
+    // general tables without a group column: the evaluation pass reads the sorted layout (runs of
+    // equal-size jobs take the uniform paths). Jobs keep their option order, so the copy inherits
+    // the duplicate marks of the original; its padding is marked as it is written.
+    SortedLayout lay;
+    if (ctx->sorted_enabled && !grouped && ctx->uniform_k == 0 && J >= 1 && sort_layout(off_host, S, J, lay)) {
+        const int64_t sn = lay.off.back();
+        ALLOC(ctx->s_units, (size_t)sn * R);
+        ALLOC(ctx->s_values, (size_t)sn);
+        ALLOC(ctx->s_off, (size_t)n_jobs + 1);
+        ALLOC(ctx->s_jmap, (size_t)n_jobs);
+        ESP_CUDA(cudaMemcpyAsync(ctx->s_off, lay.off.data(), lay.off.size() * sizeof(int64_t), cudaMemcpyHostToDevice,
+                                 ctx->stream));
+        ESP_CUDA(cudaMemcpyAsync(ctx->s_jmap, lay.jmap.data(), lay.jmap.size() * sizeof(int32_t),
+                                 cudaMemcpyHostToDevice, ctx->stream));
+        ctx->s_n_opt = sn;
+        ctx->sorted = true;
+        ESP_CUDA(launch_gather_sorted(dev_table(ctx), pass_table(ctx), ctx->s_units, ctx->s_values, ctx->stream));
+    }
+    const int64_t *plan_off = ctx->sorted ? lay.off.data() : off_host;
+    const int32_t *plan_scen = ctx->sorted ? lay.scen.data() : nullptr;
+    const int32_t *plan_runk = ctx->sorted ? lay.runk.data() : nullptr;
     const int tile_opt = tile_options_for(R, grouped, max_k, ctx->uniform_k >= 4);
     const int per_sm = pass_ctas_per_sm(R, grouped, ctx->uniform_k > 0, P, tile_opt);
     if (per_sm < 1) {
@@ -375,7 +426,8 @@ esp_status load_common(esp_ctx *ctx, int32_t S, int32_t J, int32_t R, int32_t P,
     }
     const int max_warps = ctx->sm_count * per_sm * kWarpsPerCta;
     Plan plan;
-    if (!plan_tiles(off_host, S, J, tile_opt, max_warps, plan) || !check_plan(off_host, S, J, plan)) {
+    if (!plan_tiles(plan_off, S, J, tile_opt, max_warps, plan, plan_scen, plan_runk) ||
+        !check_plan(plan_off, S, J, plan, plan_scen, plan_runk)) {
         release_table(ctx);
         return ESP_ERR_INVALID_ARG;
     }
@@ -519,7 +571,8 @@ esp_status check_params(const esp_ctx *ctx, const esp_params *p)
 // Queues one whole solve on the stream (captured into a graph when the stream allows it).
 esp_status enqueue_solve(esp_ctx *ctx, const esp_params *p, const DevState &st, bool has_l0)
 {
-    const DevTable t = dev_table(ctx);
+    const DevTable t = pass_table(ctx);
+    const DevTable t_orig = dev_table(ctx);   // the resident kernel reads the original layout
     DevPlan pl;
     pl.tiles = ctx->tiles;
     pl.warp_begin = ctx->warp_begin;
@@ -574,7 +627,7 @@ esp_status enqueue_solve(esp_ctx *ctx, const esp_params *p, const DevState &st, 
         if (ri >= 0) {
             const ResPlan &rp = ctx->res[ri].plan;
             if (e == cudaSuccess)
-                e = timed_launch([&]() { return launch_resident(t, st, rp, a, ctx->stream); });
+                e = timed_launch([&]() { return launch_resident(t_orig, st, rp, a, ctx->stream); });
             if (e == cudaSuccess)
                 e = launch_objectives(t, st, a, ctx->stream);
             return e;
@@ -916,7 +969,7 @@ esp_status esp_evaluate(esp_ctx *ctx, const double *lambda, int32_t mode, uint32
             return ESP_ERR_INVALID_ARG;
     ESP_CUDA(cudaSetDevice(ctx->device));
     ESP_CUDA(cudaMemcpyAsync(ctx->lambda0, lambda, SP * sizeof(double), cudaMemcpyHostToDevice, ctx->stream));
-    const DevTable t = dev_table(ctx);
+    const DevTable t = pass_table(ctx);
     DevState ds = dev_state(ctx);
     DevPlan pl;
     pl.tiles = ctx->tiles;
@@ -1058,15 +1111,11 @@ esp_status esp_debug_resident(esp_ctx *ctx, int32_t force_cs, int32_t *cs, int32
     return ESP_OK;
 }
 
-esp_status esp_debug_plan(const int64_t *job_offsets, int32_t S, int32_t J, int32_t tile_opt, int32_t max_warps,
-                          int32_t *tiles, int32_t tiles_cap, int32_t *warp_begin, int32_t warps_cap,
-                          int32_t *n_tiles, int32_t *n_warps)
+namespace {
+
+esp_status export_plan(const Plan &p, int32_t *tiles, int32_t tiles_cap, int32_t *warp_begin, int32_t warps_cap,
+                       int32_t *n_tiles, int32_t *n_warps)
 {
-    if (!job_offsets || S < 1 || J < 0 || !n_tiles || !n_warps)
-        return ESP_ERR_INVALID_ARG;
-    Plan p;
-    if (!plan_tiles(job_offsets, S, J, tile_opt, max_warps, p) || !check_plan(job_offsets, S, J, p))
-        return ESP_ERR_INVALID_ARG;
     *n_tiles = (int32_t)p.tiles.size();
     *n_warps = p.n_warps;
     if ((int32_t)p.tiles.size() > tiles_cap || p.n_warps + 1 > warps_cap + 1 || !tiles || !warp_begin)
@@ -1085,6 +1134,56 @@ esp_status esp_debug_plan(const int64_t *job_offsets, int32_t S, int32_t J, int3
     }
     for (int32_t w = 0; w <= p.n_warps; ++w)
         warp_begin[w] = p.warp_begin[w];
+    return ESP_OK;
+}
+
+}  // namespace
+
+esp_status esp_debug_plan(const int64_t *job_offsets, int32_t S, int32_t J, int32_t tile_opt, int32_t max_warps,
+                          int32_t *tiles, int32_t tiles_cap, int32_t *warp_begin, int32_t warps_cap,
+                          int32_t *n_tiles, int32_t *n_warps)
+{
+    if (!job_offsets || S < 1 || J < 0 || !n_tiles || !n_warps)
+        return ESP_ERR_INVALID_ARG;
+    Plan p;
+    if (!plan_tiles(job_offsets, S, J, tile_opt, max_warps, p) || !check_plan(job_offsets, S, J, p))
+        return ESP_ERR_INVALID_ARG;
+    return export_plan(p, tiles, tiles_cap, warp_begin, warps_cap, n_tiles, n_warps);
+}
+
+esp_status esp_debug_plan_runs(const int64_t *off, const int32_t *scen, const int32_t *runk, int32_t S, int32_t J,
+                               int32_t tile_opt, int32_t max_warps, int32_t *tiles, int32_t tiles_cap,
+                               int32_t *warp_begin, int32_t warps_cap, int32_t *n_tiles, int32_t *n_warps)
+{
+    if (!off || !scen || !runk || S < 1 || J < 0 || !n_tiles || !n_warps)
+        return ESP_ERR_INVALID_ARG;
+    Plan p;
+    if (!plan_tiles(off, S, J, tile_opt, max_warps, p, scen, runk) || !check_plan(off, S, J, p, scen, runk))
+        return ESP_ERR_INVALID_ARG;
+    return export_plan(p, tiles, tiles_cap, warp_begin, warps_cap, n_tiles, n_warps);
+}
+
+esp_status esp_debug_sort_layout(const int64_t *job_offsets, int32_t S, int32_t J, int64_t *off, int32_t *jmap,
+                                 int32_t *scen, int32_t *runk)
+{
+    if (!job_offsets || !off || !jmap || !scen || !runk || S < 1 || J < 1)
+        return ESP_ERR_INVALID_ARG;
+    SortedLayout lay;
+    if (!sort_layout(job_offsets, S, J, lay))
+        return ESP_ERR_INVALID_ARG;
+    std::memcpy(off, lay.off.data(), lay.off.size() * sizeof(int64_t));
+    std::memcpy(jmap, lay.jmap.data(), lay.jmap.size() * sizeof(int32_t));
+    std::memcpy(scen, lay.scen.data(), lay.scen.size() * sizeof(int32_t));
+    std::memcpy(runk, lay.runk.data(), lay.runk.size() * sizeof(int32_t));
+    return ESP_OK;
+}
+
+esp_status esp_debug_set_sorted_layout(esp_ctx *ctx, int32_t enable)
+{
+    esp_status st = check_ctx(ctx);
+    if (st != ESP_OK)
+        return st;
+    ctx->sorted_enabled = enable != 0;
     return ESP_OK;
 }
 

@@ -48,6 +48,12 @@ namespace esp {
 #ifndef ESP_RES_MIN_CTAS
 #define ESP_RES_MIN_CTAS 2    // register budget of the resident kernel: CTAs per SM it must allow
 #endif
+#ifndef ESP_BIGCHUNK4
+#define ESP_BIGCHUNK4 1       // chunks of large jobs: four independent options per lane and step
+#endif
+#ifndef ESP_SORTED_LAYOUT
+#define ESP_SORTED_LAYOUT 1   // general tables: evaluate a load-time layout sorted into runs of equal-size jobs
+#endif
 #ifndef ESP_I2F_COLS
 #define ESP_I2F_COLS 16       // unit columns r < ESP_I2F_COLS use the int-to-float instruction
 #endif
@@ -96,7 +102,15 @@ enum : uint32_t {
     TILE_BIG = 1u,        // chunk of a big job
     TILE_BIG_FIRST = 2u,  // first chunk of its job
     TILE_BIG_LAST = 4u,   // last chunk of its job
+    TILE_RUN = 8u,        // whole jobs that all have tile_run_k(flags) options (sorted layout)
 };
+
+// Options per job of a TILE_RUN tile (bits 8..15 of the flags).
+ESP_HD int tile_run_k(uint32_t flags) { return (int)((flags >> 8) & 0xffu); }
+ESP_HD uint32_t tile_run_flags(int k) { return TILE_RUN | ((uint32_t)k << 8); }
+
+// Largest padded job of the sorted layout's runs; larger jobs are evaluated in chunks.
+constexpr int kRunMaxK = 128;
 
 struct TileDesc {
     int64_t opt_begin;    // first global option of the tile

@@ -99,19 +99,20 @@ __device__ __forceinline__ double step_size(double eta0, int step, int round)
 
 // Eq. price_update for one resource: lambda' = max(0, lambda + eta d), d = U - C (RAW) or
 // (U - C) / C (NORMALIZED: the same step on capacity-fraction units), one fused multiply-add.
-__device__ __forceinline__ double price_step(double lam, long long U, long long C, double eta, int mode)
+// Cd = (double)C, converted once by the caller.
+__device__ __forceinline__ double price_step(double lam, long long U, long long C, double Cd, double eta, int mode)
 {
     double excess = (double)(U - C);
     if (mode == 1)
-        excess = excess / (double)C;
+        excess = excess / Cd;
     const double moved = __fma_rn(eta, excess, lam);
     return moved > 0.0 ? moved : 0.0;
 }
 
-// Per-unit price of a resource: lambda (RAW) or lambda / C (NORMALIZED).
-__device__ __forceinline__ double effective_price(double lam, long long C, int mode)
+// Per-unit price of a resource: lambda (RAW) or lambda / C (NORMALIZED); Cd = (double)C.
+__device__ __forceinline__ double effective_price(double lam, double Cd, int mode)
 {
-    return mode == 1 ? lam / (double)C : lam;
+    return mode == 1 ? lam / Cd : lam;
 }
 
 // Screen bound E of a scenario (fp32, rounded up) from M = max|v| + sum_r max p_r * max u_r, or

@@ -25,6 +25,7 @@
 // across the warp and added with one 64-bit atomic per priced resource per warp and scenario:
 // integer addition is associative, so U is identical on every run.
 
+#include <algorithm>
 #include <cmath>
 #include <cstdint>
 #include <cuda_runtime.h>
@@ -198,7 +199,7 @@ __device__ void set_prices(const DevTable &t, const DevState &st, const SolveArg
     bool huge = false;
     for (int k = lane; k < P; k += 32) {
         const double lam = st.lam[(size_t)s * P + k];
-        const double p = effective_price(lam, t.cap[(size_t)s * P + k], a.mode);
+        const double p = effective_price(lam, (double)t.cap[(size_t)s * P + k], a.mode);
         st.p64[(size_t)s * P + k] = p;
         st.p32[(size_t)s * P + k] = __double2float_rn(p);
         huge |= !(p <= 0x1p100);
@@ -287,7 +288,7 @@ __device__ void update_scenario(const DevTable &t, const DevState &st, const Sol
         if (st.dem_trace)
             st.dem_trace[((size_t)s * T + round) * P + k] = U;
         const double lam = st.lam[sp + k];
-        const double nl = price_step(lam, U, C, eta, a.mode);
+        const double nl = price_step(lam, U, C, (double)C, eta, a.mode);
         bad |= !isfinite(nl);
         dmax = fmax(dmax, fabs(nl - lam));
         amax = fmax(amax, fabs(lam));
@@ -307,7 +308,7 @@ __device__ void update_scenario(const DevTable &t, const DevState &st, const Sol
     for (int k = lane; k < P; k += 32) {
         const long long U = (long long)__ldcg(st.U + sp + k);
         const long long C = t.cap[sp + k];
-        const double nl = price_step(st.lam[sp + k], U, C, eta, a.mode);
+        const double nl = price_step(st.lam[sp + k], U, C, (double)C, eta, a.mode);
         st.lam[sp + k] = nl;
         st.U[sp + k] = 0ull;
         if (st.lam_trace)
@@ -442,6 +443,8 @@ template <int RT, bool G>
 __device__ __forceinline__ void take_winner_extras(WarpCtx<RT, G> &c, int64_t job, int local, const int32_t *u,
                                                    double v, int g, bool have_s64 = false, double s64 = 0.0)
 {
+    if (c.t.jmap != nullptr && (c.want_hash || c.want_min || c.kind == PASS_FINAL))
+        job = __ldg(c.t.jmap + job);     // sorted layout: outputs go to the caller's job order
     if (c.want_hash)
         c.hacc += splitmix64_mix(((uint64_t)(uint32_t)(job - (int64_t)c.s * c.t.J) << 32) | (uint32_t)local);
     if (c.kind == PASS_FINAL) {
@@ -638,11 +641,11 @@ __device__ __forceinline__ StagePtrs stage_ptrs(const TileDesc &d, const unsigne
 // job is unambiguous the unique lane holding the smallest value is the winner and records it from
 // its own registers.
 template <int RT, bool G>
-__device__ void process_tile_uniform(WarpCtx<RT, G> &c, const TileDesc &d, const StagePtrs &sp, int lane)
+__device__ void process_tile_uniform(WarpCtx<RT, G> &c, const TileDesc &d, const StagePtrs &sp, int lane, int K,
+                                     int log2_k)
 {
     const int R = c.R;
     const int n = d.n_opt;
-    const int K = c.uniform_k;
     for (int b = 0; b < n; b += 32) {
         const int i = b + lane;
         const bool valid = i < n;
@@ -667,7 +670,7 @@ __device__ void process_tile_uniform(WarpCtx<RT, G> &c, const TileDesc &d, const
         }
         const float thr = __fadd_ru(m1, c.sp.e2);
         const bool amb = c.sp.exact || !(m2 > thr);
-        const int64_t job = d.job_begin + (i >> c.log2_k);
+        const int64_t job = d.job_begin + (i >> log2_k);
         if (valid && !amb && q == m1)
             take_winner<RT, G>(c, job, i & (K - 1), u, v, g, false, 0.0);
         const uint32_t amask = __ballot_sync(FULL, valid && amb && (i & (K - 1)) == 0);
@@ -767,6 +770,69 @@ __device__ void process_tile_uniform4(WarpCtx<RT, G> &c, const TileDesc &d, cons
         const uint32_t amask = __ballot_sync(FULL, valid && amb && base == jstart);
         if (amask)
             resolve_row<RT, G>(c, lane, amask, false, sp.units, sp.vals, sp.grp, jstart, jstart + K, thr, job, 0);
+    }
+}
+
+// Tile of a run of the sorted layout whose jobs all have K = 4m options (m <= 32). Every job owns
+// L = 2^ceil(log2 m) lanes; lane `sub` of a job evaluates its options 4 sub .. 4 sub + 3 (16-byte
+// shared loads: the run starts on a 4-option boundary), lanes with sub >= m idle, and a
+// log2(L)-step xor butterfly completes the job as in the uniform path.
+template <int RT, bool G>
+__device__ void process_tile_run4(WarpCtx<RT, G> &c, const TileDesc &d, const StagePtrs &sp, int lane, int K)
+{
+    const int R = c.R;
+    const int m = K >> 2;
+    const int log2L = 32 - __clz(m - 1);
+    const int L = 1 << log2L;
+    const int jobs_per_row = 32 >> log2L;
+    const int jslot = lane >> log2L, sub = lane & (L - 1);
+    const int n_job = d.n_job;
+    for (int jb = 0; jb < n_job; jb += jobs_per_row) {
+        const int jl = jb + jslot;
+        const bool valid = jl < n_job && sub < m;
+        const int base = jl * K + 4 * sub;
+        float q[4] = {INFINITY, INFINITY, INFINITY, INFINITY};
+        if (valid) {
+            int32_t u[4][Cols<RT>::N];
+            bool dup[4];
+            load_units4_smem<RT>(sp.units + (size_t)base * R, u, dup, R);
+            const double2 va = reinterpret_cast<const double2 *>(sp.vals + base)[0];
+            const double2 vb = reinterpret_cast<const double2 *>(sp.vals + base)[1];
+            const double v[4] = {va.x, va.y, vb.x, vb.y};
+#pragma unroll
+            for (int o = 0; o < 4; ++o)
+                if (!dup[o])
+                    q[o] = screen_score<RT, G>(u[o], v[o], 0, c.sp, R, c.rg);
+        }
+        float a0 = fminf(q[0], q[1]), a1 = fmaxf(q[0], q[1]);
+        float b0 = fminf(q[2], q[3]), b1 = fmaxf(q[2], q[3]);
+        float m1 = fminf(a0, b0);
+        float m2 = fminf(fmaxf(a0, b0), fminf(a1, b1));
+        for (int dd = 1; dd < L; dd <<= 1) {
+            const float o1 = __shfl_xor_sync(FULL, m1, dd);
+            const float o2 = __shfl_xor_sync(FULL, m2, dd);
+            m2 = fminf(fminf(m2, o2), fmaxf(m1, o1));
+            m1 = fminf(m1, o1);
+        }
+        const float thr = __fadd_ru(m1, c.sp.e2);
+        const bool amb = c.sp.exact || !(m2 > thr);
+        const int64_t job = d.job_begin + jl;
+        if (valid && !amb) {
+            int w = -1;
+#pragma unroll
+            for (int o = 3; o >= 0; --o)
+                if (q[o] == m1)
+                    w = o;
+            if (w >= 0) {
+                const int i = base + w;
+                int32_t uw[Cols<RT>::N];
+                load_units_smem<RT>(sp.units + (size_t)i * R, uw, R);
+                take_winner<RT, G>(c, job, 4 * sub + w, uw, sp.vals[i], 0, false, 0.0);
+            }
+        }
+        const uint32_t amask = __ballot_sync(FULL, valid && amb && sub == 0);
+        if (amask)
+            resolve_row<RT, G>(c, lane, amask, false, sp.units, sp.vals, sp.grp, jl * K, jl * K + K, thr, job, 0);
     }
 }
 
@@ -955,6 +1021,34 @@ __device__ void process_tile_bigchunk(WarpCtx<RT, G> &c, const TileDesc &d, cons
         big_priv = best_none();
     }
     const int chunk_base = (int)(d.opt_begin - big_first);
+#if ESP_BIGCHUNK4
+    // four options per step (lane, lane + 32, lane + 64, lane + 96): their loads and screens are
+    // independent; the lane's state then takes them in increasing index order (strict <, so the
+    // lowest index keeps a tie)
+    for (int i0 = lane; i0 < n; i0 += 128) {
+        float q[4];
+#pragma unroll
+        for (int o = 0; o < 4; ++o) {
+            const int i = i0 + 32 * o;
+            q[o] = INFINITY;
+            if (i < n) {
+                int32_t u[Cols<RT>::N];
+                const bool dup = load_units_smem<RT>(sp.units + (size_t)i * R, u, R);
+                const double v = sp.vals[i];
+                const int g = G ? (int)sp.grp[i] : 0;
+                if (!dup)
+                    q[o] = screen_score<RT, G>(u, v, g, c.sp, R, c.rg);
+            }
+        }
+#pragma unroll
+        for (int o = 0; o < 4; ++o) {
+            const bool better = q[o] < big_priv.m1;
+            big_priv.m2 = better ? big_priv.m1 : fminf(big_priv.m2, q[o]);
+            big_priv.idx = better ? chunk_base + i0 + 32 * o : big_priv.idx;
+            big_priv.m1 = fminf(big_priv.m1, q[o]);
+        }
+    }
+#else
     for (int i = lane; i < n; i += 32) {
         int32_t u[Cols<RT>::N];
         const bool dup = load_units_smem<RT>(sp.units + (size_t)i * R, u, R);
@@ -963,6 +1057,7 @@ __device__ void process_tile_bigchunk(WarpCtx<RT, G> &c, const TileDesc &d, cons
         const float q = dup ? INFINITY : screen_score<RT, G>(u, v, g, c.sp, R, c.rg);
         big_priv = combine(big_priv, Best{q, dup ? kIdxNone : chunk_base + i, INFINITY});
     }
+#endif
     if (!(d.flags & TILE_BIG_LAST))
         return;
     const Best x = allreduce_best(big_priv);
@@ -993,7 +1088,7 @@ __device__ __forceinline__ void issue_tile(const DevTable &t, const TileDesc &d,
     const int64_t vlo = vb & ~int64_t(15), vhi = (ve + 15) & ~int64_t(15);
     uint32_t total = (uint32_t)(uhi - ulo) + (uint32_t)(vhi - vlo);
     int64_t olo = 0, ohi = 0, glo = 0, ghi = 0;
-    const bool offs = need_offsets && !(d.flags & TILE_BIG);
+    const bool offs = need_offsets && !(d.flags & (TILE_BIG | TILE_RUN));
     if (offs) {
         const int64_t ob = d.job_begin * 8, oe = (d.job_begin + d.n_job + 1) * 8;
         olo = ob & ~int64_t(15);
@@ -1131,9 +1226,13 @@ __global__ void __launch_bounds__(kWarpsPerCta * 32, UNI ? kMinCtasPerSm : kMinC
             if (UNI && c.uniform_k >= 4)
                 process_tile_uniform4<RT, G>(c, d, ptrs, lane);
             else if (UNI)
-                process_tile_uniform<RT, G>(c, d, ptrs, lane);
+                process_tile_uniform<RT, G>(c, d, ptrs, lane, c.uniform_k, c.log2_k);
             else if (d.flags & TILE_BIG)
                 process_tile_bigchunk<RT, G>(c, d, ptrs, big_first, big_priv, lane);
+            else if (!G && (d.flags & TILE_RUN) && tile_run_k(d.flags) >= 4)
+                process_tile_run4<RT, G>(c, d, ptrs, lane, tile_run_k(d.flags));
+            else if (!G && (d.flags & TILE_RUN))
+                process_tile_uniform<RT, G>(c, d, ptrs, lane, tile_run_k(d.flags), tile_run_k(d.flags) >> 1);
             else
                 process_tile_general<RT, G>(c, d, ptrs, big_first, big_carry, lane);
         }
@@ -1207,6 +1306,34 @@ __global__ void __launch_bounds__(kDedupWarps * 32) k_mark_duplicates(DevTable t
             }
         }
         __syncwarp();
+    }
+}
+
+// Sorted layout: one warp per job copies the job's options from the original table and writes its
+// padding (units 0 with the duplicate mark on column 0, value 0), so padding never wins.
+__global__ void k_gather_sorted(DevTable orig, DevTable sorted, int32_t *units, double *values)
+{
+    const int lane = threadIdx.x & 31;
+    const int64_t n_jobs = (int64_t)sorted.S * sorted.J;
+    const int R = sorted.R;
+    for (int64_t j = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); j < n_jobs;
+         j += (int64_t)gridDim.x * (blockDim.x >> 5)) {
+        const int64_t dst = sorted.job_off[j];
+        const int kp = (int)(sorted.job_off[j + 1] - dst);
+        const int64_t oj = sorted.jmap[j];
+        const int64_t src = orig.job_off[oj];
+        const int k = (int)(orig.job_off[oj + 1] - src);
+        for (int i = lane; i < kp * R; i += 32) {
+            const int o = i / R, r = i - o * R;
+            int32_t u = 0;
+            if (o < k)
+                u = orig.units[(src + o) * R + r];
+            else if (r == 0)
+                u = (int32_t)0x80000000;
+            units[dst * R + i] = u;
+        }
+        for (int o = lane; o < kp; o += 32)
+            values[dst + o] = (o < k) ? orig.values[src + o] : 0.0;
     }
 }
 
@@ -1383,6 +1510,17 @@ cudaError_t launch_validate(const DevTable &t, double *vmax, int32_t *umax, unsi
         k_validate_options<<<grid, 256, 0, stream>>>(t, vmax, umax, flags);
     }
     k_validate_offsets<<<256, 256, 0, stream>>>(t, flags);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_gather_sorted(const DevTable &orig, const DevTable &sorted, int32_t *units, double *values,
+                                 cudaStream_t stream)
+{
+    const int64_t n_jobs = (int64_t)sorted.S * sorted.J;
+    if (n_jobs == 0)
+        return cudaSuccess;
+    const int64_t blocks = std::min<int64_t>((n_jobs + 7) / 8, 1 << 20);
+    k_gather_sorted<<<(int)blocks, 256, 0, stream>>>(orig, sorted, units, values);
     return cudaGetLastError();
 }
 

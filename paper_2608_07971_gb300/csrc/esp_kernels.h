@@ -17,6 +17,7 @@ struct DevTable {
     int64_t n_opt;
     int32_t S, J, R, P, r_global, n_groups;
     int32_t small_units;      // 1 if every unit is below 2^23
+    const int32_t *jmap;      // sorted layout: original global index of each job of this table; nullptr: identity
 };
 
 struct DevState {
@@ -90,6 +91,11 @@ cudaError_t launch_validate(const DevTable &t, double *vmax, int32_t *umax, unsi
 // setting the sign bit of its column-0 unit in `units` (the device copy of t.units).
 cudaError_t launch_mark_duplicates(const DevTable &t, int32_t *units, unsigned long long *marked, cudaStream_t stream);
 
+// Fills the sorted layout of a general table: job j of `sorted` (offsets sorted.job_off, original
+// job sorted.jmap[j]) receives the options of that original job of `orig`, followed by padding
+// options (units 0 with the duplicate mark, value 0) up to its padded size.
+cudaError_t launch_gather_sorted(const DevTable &orig, const DevTable &sorted, int32_t *units, double *values,
+                                 cudaStream_t stream);
 cudaError_t launch_init(const DevTable &t, const DevState &st, const SolveArgs &a, const double *lambda0,
                         cudaStream_t stream);
 cudaError_t launch_pass(const DevTable &t, const DevState &st, const DevPlan &pl, const SolveArgs &a,

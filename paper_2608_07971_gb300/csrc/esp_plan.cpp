@@ -5,7 +5,8 @@
 
 namespace esp {
 
-bool plan_tiles(const int64_t *off, int32_t S, int32_t J, int32_t tile_opt, int32_t max_warps, Plan &out)
+bool plan_tiles(const int64_t *off, int32_t S, int32_t J, int32_t tile_opt, int32_t max_warps, Plan &out,
+                const int32_t *scen, const int32_t *runk)
 {
     out.tiles.clear();
     out.warp_begin.clear();
@@ -43,7 +44,7 @@ bool plan_tiles(const int64_t *off, int32_t S, int32_t J, int32_t tile_opt, int3
         int64_t j = jb[w];
         const int64_t jend = jb[w + 1];
         while (j < jend) {
-            const int32_t s = (int32_t)(j / J);
+            const int32_t s = scen ? scen[j] : (int32_t)(j / J);
             const int64_t K = off[j + 1] - off[j];
             if (K < 1)
                 return false;
@@ -63,9 +64,10 @@ bool plan_tiles(const int64_t *off, int32_t S, int32_t J, int32_t tile_opt, int3
                 continue;
             }
             const int64_t opt0 = off[j];
-            const int64_t s_end = (int64_t)(s + 1) * J;
+            const int32_t rk = runk ? runk[j] : 0;
             int64_t jj = j;
-            while (jj < jend && jj < s_end && off[jj + 1] - opt0 <= tile_opt)
+            while (jj < jend && (scen ? scen[jj] == s : jj / J == s) && (runk ? runk[jj] == rk : true) &&
+                   off[jj + 1] - opt0 <= tile_opt)
                 ++jj;
             TileDesc d;
             d.opt_begin = opt0;
@@ -73,7 +75,7 @@ bool plan_tiles(const int64_t *off, int32_t S, int32_t J, int32_t tile_opt, int3
             d.n_opt = (int32_t)(off[jj] - opt0);
             d.n_job = (int32_t)(jj - j);
             d.scenario = s;
-            d.flags = 0;
+            d.flags = rk > 0 ? tile_run_flags(rk) : 0u;
             out.tiles.push_back(d);
             j = jj;
         }
@@ -83,8 +85,10 @@ bool plan_tiles(const int64_t *off, int32_t S, int32_t J, int32_t tile_opt, int3
     return true;
 }
 
-bool check_plan(const int64_t *off, int32_t S, int32_t J, const Plan &p)
+bool check_plan(const int64_t *off, int32_t S, int32_t J, const Plan &p, const int32_t *scen,
+                const int32_t *runk)
 {
+    auto scen_of = [&](int64_t j) -> int64_t { return scen ? scen[j] : j / J; };
     const int64_t n_jobs = (int64_t)S * J;
     if ((int32_t)p.warp_begin.size() != p.n_warps + 1)
         return false;
@@ -108,7 +112,7 @@ bool check_plan(const int64_t *off, int32_t S, int32_t J, const Plan &p)
             } else if (d.opt_begin != big_next_opt || d.n_job != 0 || j != next_job) {
                 return false;
             }
-            if (j / J != d.scenario || d.opt_begin + d.n_opt > off[j + 1])
+            if (scen_of(j) != d.scenario || d.opt_begin + d.n_opt > off[j + 1])
                 return false;
             if (d.flags & TILE_BIG_LAST) {
                 if (d.opt_begin + d.n_opt != off[j + 1])
@@ -126,8 +130,19 @@ bool check_plan(const int64_t *off, int32_t S, int32_t J, const Plan &p)
             const int64_t j1 = d.job_begin + d.n_job;
             if (j1 > n_jobs || d.opt_begin != off[d.job_begin] || d.opt_begin + d.n_opt != off[j1])
                 return false;
-            if (d.job_begin / J != d.scenario || (j1 - 1) / J != d.scenario)
-                return false;
+            for (int64_t j = d.job_begin; j < j1; ++j) {
+                if (scen_of(j) != d.scenario)
+                    return false;
+                if (d.flags & TILE_RUN) {
+                    const int k = tile_run_k(d.flags);
+                    if (!runk || runk[j] != k || off[j + 1] - off[j] != k)
+                        return false;
+                } else if (runk && runk[j] != 0) {
+                    return false;
+                }
+            }
+            if ((d.flags & TILE_RUN) && (d.opt_begin & 3) != 0 && tile_run_k(d.flags) >= 4)
+                return false;   // a run of 4m-option jobs starts on a 4-option boundary
             next_job = j1;
         }
     }
@@ -161,6 +176,52 @@ bool plan_resident(const int64_t *off, int32_t S, int32_t J, int32_t cs, ResShap
         }
     }
     return true;
+}
+
+bool sort_layout(const int64_t *off, int32_t S, int32_t J, SortedLayout &out)
+{
+    const int64_t n_jobs = (int64_t)S * J;
+    out.off.assign(1, 0);
+    out.jmap.clear();
+    out.scen.clear();
+    out.runk.clear();
+    if (n_jobs < 1 || n_jobs >= INT32_MAX)
+        return false;
+    out.off.reserve(n_jobs + 1);
+    out.jmap.reserve(n_jobs);
+    out.scen.reserve(n_jobs);
+    out.runk.reserve(n_jobs);
+    auto push = [&](int64_t j, int32_t s, int64_t kp, int32_t rk) {
+        out.off.push_back(out.off.back() + kp);
+        out.jmap.push_back((int32_t)j);
+        out.scen.push_back(s);
+        out.runk.push_back(rk);
+    };
+    std::vector<std::vector<int32_t>> bucket(kRunMaxK / 4 + 1);
+    for (int32_t s = 0; s < S; ++s) {       // jobs of 3 .. kRunMaxK options, padded to 4m
+        for (auto &b : bucket)
+            b.clear();
+        for (int64_t j = (int64_t)s * J; j < (int64_t)(s + 1) * J; ++j) {
+            const int64_t K = off[j + 1] - off[j];
+            if (K < 1)
+                return false;
+            if (K >= 3 && K <= kRunMaxK)
+                bucket[(K + 3) / 4].push_back((int32_t)j);
+        }
+        for (int b = 1; b <= kRunMaxK / 4; ++b)
+            for (int32_t j : bucket[b])
+                push(j, s, 4 * b, 4 * b);
+    }
+    for (int32_t s = 0; s < S; ++s)         // large jobs, unpadded
+        for (int64_t j = (int64_t)s * J; j < (int64_t)(s + 1) * J; ++j)
+            if (off[j + 1] - off[j] > kRunMaxK)
+                push(j, s, off[j + 1] - off[j], 0);
+    for (int32_t s = 0; s < S; ++s)         // runs of 2- and 1-option jobs
+        for (int64_t k = 2; k >= 1; --k)
+            for (int64_t j = (int64_t)s * J; j < (int64_t)(s + 1) * J; ++j)
+                if (off[j + 1] - off[j] == k)
+                    push(j, s, k, (int32_t)k);
+    return (int64_t)out.jmap.size() == n_jobs;
 }
 
 }  // namespace esp

@@ -58,6 +58,16 @@ __device__ __forceinline__ void cluster_sync()
         "barrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
 
+// The round barrier: the cluster barrier, or the CTA barrier when the cluster is one CTA (its
+// partials then stay in its own shared memory, which the CTA barrier orders).
+__device__ __forceinline__ void round_sync(int cs)
+{
+    if (cs == 1)
+        __syncthreads();
+    else
+        cluster_sync();
+}
+
 // Shared-memory address of the same location in CTA `rank` of the cluster.
 __device__ __forceinline__ uint32_t map_rank(uint32_t addr, uint32_t rank)
 {
@@ -165,8 +175,77 @@ struct ResAcc {
     unsigned int resolved;
 };
 
+// Exact resolution of one job: the lexicographic minimum of (s, k) over its survivors (options
+// with q <= thr that are not load-time duplicates; every non-duplicate option in exact mode).
+// Lane-serial form: the calling lane scans the job's options in order.
+template <int RT, bool UNI, bool SMALL>
+__device__ __forceinline__ int res_resolve_lane(const ResSlice<RT, UNI> &sl, int jj, int ob, int K, float thr,
+                                                double &s_out)
+{
+    long long best = 0x7fffffffffffffffLL;
+    int bi = kIdxNone;
+    double bs = 0.0;
+    for (int k = 0; k < K; ++k) {
+        const int bu = sl.ucol0(jj, ob, k);
+        const double v = sl.V[sl.vslot(jj, ob, k)];
+        bool dup;
+        const float q = res_screen<RT, UNI, SMALL>(sl, bu, v, dup);
+        if (dup || (!sl.exact && q > thr))
+            continue;
+        const double sc = res_exact<RT, UNI, SMALL>(sl, bu, v);
+        const long long key = order_key(sc);
+        if (key < best) {
+            best = key;
+            bi = k;
+            bs = sc;
+        }
+    }
+    s_out = bs;
+    return bi;
+}
+
+// The same minimum computed by the whole warp: lanes take options k = lane, lane + 32, ... and a
+// butterfly keeps the smallest (key, k). Every lane returns the answer.
+template <int RT, bool UNI, bool SMALL>
+__device__ __forceinline__ int res_resolve_warp(const ResSlice<RT, UNI> &sl, int jj, int ob, int K, float thr,
+                                                double &s_out, int lane)
+{
+    long long best = 0x7fffffffffffffffLL;
+    int bi = kIdxNone;
+    double bs = 0.0;
+    for (int k = lane; k < K; k += 32) {
+        const int bu = sl.ucol0(jj, ob, k);
+        const double v = sl.V[sl.vslot(jj, ob, k)];
+        bool dup;
+        const float q = res_screen<RT, UNI, SMALL>(sl, bu, v, dup);
+        if (dup || (!sl.exact && q > thr))
+            continue;
+        const double sc = res_exact<RT, UNI, SMALL>(sl, bu, v);
+        const long long key = order_key(sc);
+        if (key < best) {
+            best = key;
+            bi = k;
+            bs = sc;
+        }
+    }
+#pragma unroll
+    for (int d = 16; d >= 1; d >>= 1) {
+        const long long ok = __shfl_xor_sync(FULL, best, d);
+        const int oi = __shfl_xor_sync(FULL, bi, d);
+        const double os = __shfl_xor_sync(FULL, bs, d);
+        if (ok < best || (ok == best && oi < bi)) {
+            best = ok;
+            bi = oi;
+            bs = os;
+        }
+    }
+    s_out = bs;
+    return bi;
+}
+
 // Best responses of the slice's jobs: lane = job. FINAL writes the selection outputs; otherwise the
-// demand (and, when asked, fingerprint and dual sum) of the winners accumulate in acc.
+// demand (and, when asked, fingerprint and dual sum) of the winners accumulate in acc. Ambiguous
+// jobs are resolved by the whole warp one after the other when they are few, else each by its lane.
 template <int RT, bool UNI, bool SMALL, bool FINAL>
 __device__ void res_evaluate(const DevState &st, const ResSlice<RT, UNI> &sl, bool want_hash, bool want_min,
                              ResAcc<RT> &acc, int warp, int lane)
@@ -174,10 +253,9 @@ __device__ void res_evaluate(const DevState &st, const ResSlice<RT, UNI> &sl, bo
     const int R = RT ? RT : sl.R;
     for (int jb = warp * 32; jb < sl.m; jb += kResWarps * 32) {
         const int jj = jb + lane;
-        if (jj >= sl.m)
-            break;
-        int ob = 0, K = sl.K;
-        if (!UNI) {
+        const bool act = jj < sl.m;
+        int ob = 0, K = act ? sl.K : 0;
+        if (!UNI && act) {
             ob = sl.loff[jj];
             K = sl.loff[jj + 1] - ob;
         }
@@ -194,34 +272,37 @@ __device__ void res_evaluate(const DevState &st, const ResSlice<RT, UNI> &sl, bo
             m1 = fminf(m1, q);
         }
         const float thr = __fadd_ru(m1, sl.e2);
+        const bool amb = act && (sl.exact || !(m2 > thr));
         int w = i1;
         double s_w = 0.0;
         bool have_s = false;
-        if (sl.exact || !(m2 > thr)) {
-            // exact resolution on this lane: lexicographic minimum of (s, k) over the survivors
-            long long best = 0x7fffffffffffffffLL;
-            int bi = kIdxNone;
-            double bs = 0.0;
-            for (int k = 0; k < K; ++k) {
-                const int bu = sl.ucol0(jj, ob, k);
-                const double v = sl.V[sl.vslot(jj, ob, k)];
-                bool dup;
-                const float q = res_screen<RT, UNI, SMALL>(sl, bu, v, dup);
-                if (dup || (!sl.exact && q > thr))
-                    continue;
-                const double s = res_exact<RT, UNI, SMALL>(sl, bu, v);
-                const long long key = order_key(s);
-                if (key < best) {
-                    best = key;
-                    bi = k;
-                    bs = s;
+        uint32_t amask = __ballot_sync(FULL, amb);
+        if (__popc(amask) > 4) {
+            if (amb) {
+                const int bi = res_resolve_lane<RT, UNI, SMALL>(sl, jj, ob, K, thr, s_w);
+                w = (bi == kIdxNone) ? i1 : bi;    // the option of m1 always survives; defensive only
+                have_s = true;
+                ++acc.resolved;
+            }
+        } else {
+            while (amask) {
+                const int cl = __ffs(amask) - 1;
+                amask &= amask - 1;
+                const int cob = __shfl_sync(FULL, ob, cl);
+                const int cK = __shfl_sync(FULL, K, cl);
+                const float cthr = __shfl_sync(FULL, thr, cl);
+                double cs_w;
+                const int bi = res_resolve_warp<RT, UNI, SMALL>(sl, jb + cl, cob, cK, cthr, cs_w, lane);
+                if (lane == cl) {
+                    w = (bi == kIdxNone) ? i1 : bi;
+                    s_w = cs_w;
+                    have_s = true;
+                    ++acc.resolved;
                 }
             }
-            w = (bi == kIdxNone) ? i1 : bi;   // the option of m1 always survives; defensive only
-            s_w = bs;
-            have_s = true;
-            ++acc.resolved;
         }
+        if (!act)
+            continue;
         const int bw = sl.ucol0(jj, ob, w);
 #pragma unroll
         for (int r = 0; r < ResCols<RT>::N; ++r) {
@@ -250,31 +331,46 @@ __device__ void res_evaluate(const DevState &st, const ResSlice<RT, UNI> &sl, bo
     }
 }
 
-__device__ __forceinline__ long long warp_sum_i64(long long v)
+// Wrapping sum over the warp of 64-bit words by three 32-bit hardware reductions of 22-bit chunks
+// (a chunk sum over 32 lanes stays below 2^27); exact for the int64 demand, whose totals are below
+// 2^63, and for the fingerprint, which wraps by definition.
+__device__ __forceinline__ unsigned long long warp_sum_u64(unsigned long long v)
 {
-#pragma unroll
-    for (int d = 16; d >= 1; d >>= 1)
-        v += __shfl_xor_sync(FULL, v, d);
-    return v;
+    const unsigned long long c0 = __reduce_add_sync(FULL, (unsigned)(v & 0x3fffffu));
+    const unsigned long long c1 = __reduce_add_sync(FULL, (unsigned)((v >> 22) & 0x3fffffu));
+    const unsigned long long c2 = __reduce_add_sync(FULL, (unsigned)(v >> 44));
+    return c0 + (c1 << 22) + (c2 << 44);
 }
 
-// Prices of lambda (lanes c < R of warp 0 hold lambda_c): the fp64 and fp32 per-unit prices and
-// the screen bound, written to shared memory. Same arithmetic as the streaming path's set_prices.
-__device__ __forceinline__ void res_set_prices(double lam, long long cap, int umax, double vmax, int R, int mode,
-                                               bool exact_only, double *p64s, float *p32s, float *e2s, int lane)
+// Prices of lambda (lanes c < R of warp 0 hold lambda_c, R <= 16): the fp64 and fp32 per-unit prices
+// (the same values as the streaming path's) and the screen bound 2E, written to shared memory. E
+// only has to bound the screen error from above, so it is computed in fp32 with every operation
+// rounded up: p <= p32 (1 + 2^-23) + 2^-149, M = max|v| + sum_r p_r max u_r and
+// E = (4R + 16) 2^-24 M + 2^-99, each replaced by an upper bound; no fp64 operation beyond the
+// prices themselves. A price bound above 2^100, or M above 2^100, selects exact mode.
+__device__ __forceinline__ void res_set_prices(double lam, double capd, float umax_up, float vmax_up, int R,
+                                               int mode, bool exact_only, double *p64s, float *p32s, float *e2s,
+                                               int lane)
 {
     const bool mine = lane < R;
-    const double p = mine ? effective_price(lam, cap, mode) : 0.0;
-    const bool huge = __any_sync(FULL, mine && !(p <= 0x1p100));
-    const double term = mine ? p * (double)umax : 0.0;
-    const double M = vmax + warp_sum_fixed(term);
+    const double p = mine ? effective_price(lam, capd, mode) : 0.0;
+    const float p32 = __double2float_rn(p);
+    const float p_up = __fadd_ru(__fmul_ru(p32, 1.0f + 0x1p-23f), 0x1p-149f);
+    float term = mine ? __fmul_ru(p_up, umax_up) : 0.0f;
+#pragma unroll
+    for (int d = 8; d >= 1; d >>= 1)    // lanes 0 .. 15 hold the terms
+        term = __fadd_ru(term, __shfl_xor_sync(FULL, term, d));
+    const bool huge = __any_sync(FULL, mine && !(p_up <= 0x1p100f));
     if (mine) {
         p64s[lane] = p;
-        p32s[lane] = __double2float_rn(p);
+        p32s[lane] = p32;
     }
     if (lane == 0) {
-        const float e = screen_bound(M, R, exact_only || huge);
-        *e2s = (e < INFINITY) ? 2.0f * e : INFINITY;
+        const float M = __fadd_ru(vmax_up, term);
+        float e2 = INFINITY;
+        if (!exact_only && !huge && M <= 0x1p100f)
+            e2 = 2.0f * __fadd_ru(__fmul_ru(M, (4.0f * R + 16.0f) * 0x1p-24f), 0x1p-99f);
+        *e2s = e2;
     }
 }
 
@@ -329,17 +425,18 @@ __global__ void __launch_bounds__(kResThreads, ESP_RES_MIN_CTAS) k_resident(DevT
 
     // ---- price state: warp 0 of every CTA holds lambda_c, C_c and max u_c in lane c
     const size_t sp = (size_t)s * P;
-    double lam = 0.0;
+    double lam = 0.0, capd = 1.0;
     long long cap = 1;
-    int umax = 0;
-    const double vmax = st.vmax[s];
+    float umax_up = 0.0f;
+    const float vmax_up = __double2float_ru(st.vmax[s]);
     if (warp == 0) {
         if (lane < R) {
             lam = st.lam[sp + lane];
             cap = t.cap[sp + lane];
-            umax = st.umax[(size_t)s * R + lane];
+            capd = (double)cap;
+            umax_up = __int2float_ru(st.umax[(size_t)s * R + lane]);
         }
-        res_set_prices(lam, cap, umax, vmax, R, a.mode, a.exact_only != 0, p64s, p32s, e2s, lane);
+        res_set_prices(lam, capd, umax_up, vmax_up, R, a.mode, a.exact_only != 0, p64s, p32s, e2s, lane);
         if (lane == 0)
             *stops = 0;
     }
@@ -390,12 +487,12 @@ __global__ void __launch_bounds__(kResThreads, ESP_RES_MIN_CTAS) k_resident(DevT
             for (int r = 0; r < ResCols<RT>::N; ++r) {
                 if (RT == 0 && r >= R)
                     break;
-                const long long v = warp_sum_i64(acc.dem[r]);
+                const long long v = (long long)warp_sum_u64((unsigned long long)acc.dem[r]);
                 if (lane == 0)
                     wpart[warp * kResCols + r] = (unsigned long long)v;
             }
             if (want_hash) {
-                const long long h = warp_sum_i64((long long)acc.hash);
+                const long long h = (long long)warp_sum_u64(acc.hash);
                 if (lane == 0)
                     wpart[warp * kResCols + kColHash] = (unsigned long long)h;
             }
@@ -419,6 +516,7 @@ __global__ void __launch_bounds__(kResThreads, ESP_RES_MIN_CTAS) k_resident(DevT
                         d += __longlong_as_double((long long)wpart[w * kResCols + c]);
                     tot = (unsigned long long)__double_as_longlong(d);
                 } else {
+#pragma unroll
                     for (int w = 0; w < kResWarps; ++w)
                         tot += wpart[w * kResCols + c];
                 }
@@ -427,23 +525,26 @@ __global__ void __launch_bounds__(kResThreads, ESP_RES_MIN_CTAS) k_resident(DevT
                     st_cluster_u64(map_rank(slot, (uint32_t)rk), tot);
             }
         }
-        cluster_sync();
+        round_sync(cs);
 
         // 4. every CTA: the scenario's totals in rank order, then Eq. price_update
         if (!stopped && warp == 0) {
             const int c = lane;
             const unsigned long long *cp = cpart + (size_t)par * cs * kResCols;
             long long Uc = 0;
-            if (c < R)
-                for (int rk = 0; rk < cs; ++rk)
-                    Uc += (long long)cp[rk * kResCols + c];
+            if (c < R) {
+#pragma unroll
+                for (int rk = 0; rk < kResMaxCluster; ++rk)   // independent loads, summed in rank order
+                    if (rk < cs)
+                        Uc += (long long)cp[rk * kResCols + c];
+            }
             const bool lead = rank == 0;
             if (want_min) {
                 double d = 0.0;
                 if (c == 0)
                     for (int rk = 0; rk < cs; ++rk)
                         d += __longlong_as_double((long long)cp[rk * kResCols + kColDual]);
-                const double lc = (c < R) ? ((a.mode == 1) ? lam : lam * (double)cap) : 0.0;
+                const double lc = (c < R) ? ((a.mode == 1) ? lam : lam * capd) : 0.0;
                 const double g = __shfl_sync(FULL, d, 0) + warp_sum_fixed(lc);
                 if (g < best_dual)
                     best_dual = g;
@@ -459,22 +560,25 @@ __global__ void __launch_bounds__(kResThreads, ESP_RES_MIN_CTAS) k_resident(DevT
             if (st.dem_trace && lead && c < R)
                 st.dem_trace[((size_t)s * T + round) * P + c] = Uc;
             const double eta = step_size(a.eta0, a.step, round);
-            const double nl = (c < R) ? price_step(lam, Uc, cap, eta, a.mode) : 0.0;
+            const double nl = (c < R) ? price_step(lam, Uc, cap, capd, eta, a.mode) : 0.0;
             const bool bad = __any_sync(FULL, c < R && !isfinite(nl));
-            const double dmax = warp_max((c < R) ? fabs(nl - lam) : 0.0);
-            const double amax = warp_max((c < R) ? fabs(lam) : 0.0);
             bool stop;
             if (bad) {
                 status = 2;    // the prices stay at the last finite lambda
                 stop = true;
             } else {
-                lam = nl;
                 rounds = round + 1;
                 if (st.lam_trace && lead && c < R)
                     st.lam_trace[((size_t)s * (T + 1) + round + 1) * P + c] = nl;
-                stop = (a.tol > 0.0) && (dmax <= a.tol * fmax(1.0, amax));
+                stop = false;
+                if (a.tol > 0.0) {   // the stopping rule on the step just taken
+                    const double dmax = warp_max((c < R) ? fabs(nl - lam) : 0.0);
+                    const double amax = warp_max((c < R) ? fabs(lam) : 0.0);
+                    stop = dmax <= a.tol * fmax(1.0, amax);
+                }
+                lam = nl;
                 converged = stop ? 1 : 0;
-                res_set_prices(lam, cap, umax, vmax, R, a.mode, a.exact_only != 0, p64s, p32s, e2s, lane);
+                res_set_prices(lam, capd, umax_up, vmax_up, R, a.mode, a.exact_only != 0, p64s, p32s, e2s, lane);
             }
             if (lane == 0)
                 *stops = stop ? 1 : 0;
@@ -496,7 +600,7 @@ __global__ void __launch_bounds__(kResThreads, ESP_RES_MIN_CTAS) k_resident(DevT
     for (int r = 0; r < ResCols<RT>::N; ++r) {
         if (RT == 0 && r >= R)
             break;
-        const long long v = warp_sum_i64(acc.dem[r]);
+        const long long v = (long long)warp_sum_u64((unsigned long long)acc.dem[r]);
         if (lane == 0 && v != 0)
             atomicAdd(st.U_final + sp + r, (unsigned long long)v);
     }

@@ -27,7 +27,8 @@ EXPORTED = [
     "esp_create", "esp_set_stream", "esp_load_options", "esp_load_options_device", "esp_solve",
     "esp_solve_async", "esp_get_result", "esp_get_prices", "esp_get_selection", "esp_get_demand",
     "esp_evaluate", "esp_last_launch_count", "esp_pass_times", "esp_status_string", "esp_destroy",
-    "esp_debug_tile_options", "esp_debug_plan", "esp_debug_stats", "esp_debug_resident", "esp_evaluate_noalloc",
+    "esp_debug_tile_options", "esp_debug_plan", "esp_debug_stats", "esp_debug_resident",
+    "esp_debug_sort_layout", "esp_debug_plan_runs", "esp_debug_set_sorted_layout", "esp_evaluate_noalloc",
 ]
 
 
@@ -85,6 +86,10 @@ def load_library(path: Optional[str] = None):
         "esp_debug_tile_options": ([i32, i32], i32),
         "esp_debug_stats": ([vp, ctypes.POINTER(i64), ctypes.POINTER(i64), i32], st),
         "esp_debug_resident": ([vp, i32, ctypes.POINTER(i32), ctypes.POINTER(i32)], st),
+        "esp_debug_sort_layout": ([vp, i32, i32, vp, vp, vp, vp], st),
+        "esp_debug_plan_runs": ([vp, vp, vp, i32, i32, i32, i32, vp, i32, vp, i32, ctypes.POINTER(i32),
+                                 ctypes.POINTER(i32)], st),
+        "esp_debug_set_sorted_layout": ([vp, i32], st),
         "esp_debug_plan": ([vp, i32, i32, i32, i32, vp, i32, vp, i32, ctypes.POINTER(i32), ctypes.POINTER(i32)], st),
         "esp_evaluate_noalloc": ([i32, i32, i32, vp, vp, vp, vp, vp, i32, vp, vp, vp, vp], st),
     }
@@ -328,3 +333,37 @@ def plan(job_off: np.ndarray, S: int, J: int, tile_opt: int, max_warps: int):
     _check(lib.esp_debug_plan(_p(job_off), S, J, tile_opt, max_warps, _p(tiles), nt.value, _p(wb), nw.value,
                               ctypes.byref(nt), ctypes.byref(nw)), "esp_debug_plan")
     return tiles[:nt.value], wb
+
+
+def sort_layout(job_off: np.ndarray, S: int, J: int):
+    """Sorted layout of a general table (no GPU): (padded offsets, jmap, scen, runk)."""
+    lib = load_library()
+    job_off = np.ascontiguousarray(job_off, np.int64)
+    off = np.zeros(S * J + 1, np.int64)
+    jmap, scen, runk = (np.zeros(S * J, np.int32) for _ in range(3))
+    _check(lib.esp_debug_sort_layout(_p(job_off), S, J, _p(off), _p(jmap), _p(scen), _p(runk)),
+           "esp_debug_sort_layout")
+    return off, jmap, scen, runk
+
+
+def plan_runs(off, scen, runk, S: int, J: int, tile_opt: int, max_warps: int):
+    """Host tile planner over a sorted layout (no GPU): (tiles n x 8 int32, warp_begin)."""
+    lib = load_library()
+    off = np.ascontiguousarray(off, np.int64)
+    scen = np.ascontiguousarray(scen, np.int32)
+    runk = np.ascontiguousarray(runk, np.int32)
+    nt, nw = ctypes.c_int32(), ctypes.c_int32()
+    st = lib.esp_debug_plan_runs(_p(off), _p(scen), _p(runk), S, J, tile_opt, max_warps, None, 0, None, 0,
+                                 ctypes.byref(nt), ctypes.byref(nw))
+    if st not in (ESP_OK, ESP_ERR_OOM):
+        raise EspError(st, "esp_debug_plan_runs")
+    tiles = np.zeros((max(nt.value, 1), 8), np.int32)
+    wb = np.zeros(nw.value + 1, np.int32)
+    _check(lib.esp_debug_plan_runs(_p(off), _p(scen), _p(runk), S, J, tile_opt, max_warps, _p(tiles), nt.value,
+                                   _p(wb), nw.value, ctypes.byref(nt), ctypes.byref(nw)), "esp_debug_plan_runs")
+    return tiles[:nt.value], wb
+
+
+def esp_debug_set_sorted_layout(ctx: int, enable: bool) -> None:
+    _check(load_library().esp_debug_set_sorted_layout(ctx, 1 if enable else 0), "esp_debug_set_sorted_layout")
+

@@ -120,3 +120,72 @@ def test_tile_options(lib):
     assert lib.esp_debug_tile_options(6, 0) == 256
     assert lib.esp_debug_tile_options(4, 0) % 32 == 0
     assert lib.esp_debug_tile_options(8, 1) % 32 == 0
+
+
+def expected_sorted_order(K, S, J):
+    """The sorted layout's job order, restated: per scenario the 3..128-option jobs by padded size
+    (4 * ceil(K / 4)), stable; then per scenario the larger jobs; then per scenario the 2-option and
+    the 1-option jobs."""
+    order, padded, runk = [], [], []
+    for s in range(S):
+        js = range(s * J, (s + 1) * J)
+        small = sorted((j for j in js if 3 <= K[j] <= 128), key=lambda j: (-(-K[j] // 4), j))
+        for j in small:
+            order.append(j); padded.append(4 * -(-K[j] // 4)); runk.append(4 * -(-K[j] // 4))
+    for s in range(S):
+        for j in range(s * J, (s + 1) * J):
+            if K[j] > 128:
+                order.append(j); padded.append(K[j]); runk.append(0)
+    for s in range(S):
+        for k in (2, 1):
+            for j in range(s * J, (s + 1) * J):
+                if K[j] == k:
+                    order.append(j); padded.append(k); runk.append(k)
+    return np.array(order), np.array(padded), np.array(runk)
+
+
+@pytest.mark.parametrize("case", ["zipf", "mixed", "small", "big"])
+def test_sorted_layout(lib, case):
+    rng = np.random.default_rng(11)
+    S, J = 3, 400
+    if case == "zipf":
+        K = np.minimum(256, rng.zipf(1.3, S * J))
+    elif case == "mixed":
+        K = rng.integers(1, 300, S * J)
+    elif case == "small":
+        K = rng.integers(1, 6, S * J)
+    else:
+        K = rng.choice([129, 700, 3], S * J)
+    off = np.zeros(S * J + 1, np.int64)
+    off[1:] = np.cumsum(K)
+    soff, jmap, scen, runk = esp.sort_layout(off, S, J)
+    order, padded, want_runk = expected_sorted_order(K, S, J)
+    assert np.array_equal(jmap, order)                       # a permutation in the stated order
+    assert np.array_equal(np.diff(soff), padded)             # padding to a multiple of 4 (3..128)
+    assert np.array_equal(runk, want_runk)
+    assert np.array_equal(scen, order // J)
+    part_a = runk >= 4
+    assert np.all(soff[:-1][part_a] % 4 == 0)               # every padded job starts 4-aligned
+    assert np.all(np.diff(soff) >= K[jmap])
+    for tile_opt in (128,):
+        for warps in (1, 9, 200):
+            tiles, wb = esp.plan_runs(soff, scen, runk, S, J, tile_opt, warps)
+            opt_begin = tiles[:, 0].astype(np.int64) & 0xFFFFFFFF | (tiles[:, 1].astype(np.int64) << 32)
+            job_begin = tiles[:, 2].astype(np.int64) & 0xFFFFFFFF | (tiles[:, 3].astype(np.int64) << 32)
+            covered = np.zeros(S * J, np.int64)
+            for k in range(len(tiles)):
+                fl = tiles[k, 7]
+                if fl & 1:
+                    covered[job_begin[k]] += tiles[k, 4]
+                    continue
+                j0, j1 = job_begin[k], job_begin[k] + tiles[k, 5]
+                covered[j0:j1] += np.diff(soff[j0:j1 + 1])
+                assert np.all(scen[j0:j1] == tiles[k, 6])
+                if fl & 8:                                   # a run tile: one option count
+                    kk = (fl >> 8) & 0xFF
+                    assert np.all(runk[j0:j1] == kk) and tiles[k, 4] == kk * (j1 - j0)
+                    if kk >= 4:
+                        assert opt_begin[k] % 4 == 0
+                else:
+                    assert np.all(runk[j0:j1] == 0)
+            assert np.array_equal(covered, np.diff(soff))
