@@ -27,6 +27,9 @@ namespace esp {
 #ifndef ESP_MIN_CTAS_UNIFORM
 #define ESP_MIN_CTAS_UNIFORM 5
 #endif
+#ifndef ESP_MIN_CTAS_UNIFORM_NARROW
+#define ESP_MIN_CTAS_UNIFORM_NARROW 6   // the same for R = 4 and R = 6 (80 registers, no spills)
+#endif
 #ifndef ESP_WARPS_PER_CTA
 #define ESP_WARPS_PER_CTA 4
 #endif
@@ -64,6 +67,7 @@ constexpr int kStages = ESP_STAGES;  // TMA stages per warp
 constexpr int kPrefetchTiles = ESP_PREFETCH_TILES;  // L2 prefetch distance, in tiles of the warp
 constexpr int kUniform4Tile = ESP_UNIFORM4_TILE;    // tile of the 4-options-per-lane path (0: largest)
 constexpr int kMinCtasPerSm = ESP_MIN_CTAS_UNIFORM; // register budget of the uniform-K evaluation kernel
+constexpr int kMinCtasPerSmNarrow = ESP_MIN_CTAS_UNIFORM_NARROW;  // ... for R = 4 and R = 6
 constexpr int kMinCtasPerSmGeneral = ESP_MIN_CTAS_GENERAL;  // register budget of the general kernel
 constexpr int kStageDataBytes = ESP_STAGE_DATA_BYTES;  // option bytes (units + values [+ group]) of a full stage
 constexpr uint32_t kWaitSuspendNs = ESP_WAIT_SUSPEND_NS;
@@ -154,30 +158,36 @@ struct StageLayout {
     int off, units, vals, grp, bytes;
 };
 
-ESP_HD StageLayout stage_layout(int tile_opt, int R, bool grouped)
+ESP_HD StageLayout stage_layout(int tile_opt, int R, bool grouped, bool offsets)
 {
     StageLayout L;
     L.off = 0;
-    L.units = round16((tile_opt + 1) * 8 + 32);
+    L.units = offsets ? round16((tile_opt + 1) * 8 + 32) : 0;   // uniform tables need no job offsets
     L.vals = L.units + round16(tile_opt * R * 4 + 32);
     L.grp = L.vals + round16(tile_opt * 8 + 32);
     L.bytes = L.grp + (grouped ? round16(tile_opt * 2 + 32) : 0);
     return L;
 }
 
-// Per-warp shared memory: kStages stages with their tile descriptors, the fp32 prices of the
-// current scenario (grouped tables) and the stage barriers.
+// Tile descriptors a warp keeps in shared memory: a ring refilled kDescBlock at a time, one block
+// ahead of the block being issued.
+constexpr int kDescRing = 16;
+constexpr int kDescBlock = 8;
+static_assert(kDescRing == 2 * kDescBlock, "two blocks in the descriptor ring");
+
+// Per-warp shared memory: kStages stages, the tile-descriptor ring, the fp32 prices of the current
+// scenario (grouped tables) and the stage barriers.
 struct WarpSmem {
     int stage_bytes, descs, p32, bars, bytes;
 };
 
-ESP_HD WarpSmem warp_smem(int tile_opt, int R, bool grouped, int P)
+ESP_HD WarpSmem warp_smem(int tile_opt, int R, bool grouped, int P, bool offsets)
 {
     WarpSmem W;
-    StageLayout L = stage_layout(tile_opt, R, grouped);
+    StageLayout L = stage_layout(tile_opt, R, grouped, offsets);
     W.stage_bytes = L.bytes;
-    W.descs = kStages * L.bytes;          // the descriptor of the tile in each stage
-    W.p32 = W.descs + 32 * kStages;
+    W.descs = kStages * L.bytes;          // the descriptor ring (32 bytes per tile)
+    W.p32 = W.descs + 32 * kDescRing;
     W.bars = W.p32 + (grouped ? round16(P * 4) : 0);
     W.bytes = W.bars + 16 * kStages;
     return W;

@@ -712,6 +712,50 @@ __device__ __forceinline__ void load_units4_smem(const int32_t *p, int32_t (*u)[
     }
 }
 
+// Exact resolution inside a row of the four-options-per-lane layout: every lane of an ambiguous job
+// rescores in fp64 its own survivors among the four options it screened (q <= thr; every option
+// but the duplicates in exact mode), then an xor butterfly over the job's L lanes keeps the
+// lexicographic minimum of (s, job-local index), and the lane holding that option records it.
+// The options are still in the stage, so no option is read twice from memory. base: tile-local
+// index of the lane's first option; loc0: its job-local index; lamb: the lane's job is ambiguous.
+template <int RT, bool G>
+__device__ __forceinline__ void resolve4_in_row(WarpCtx<RT, G> &c, const StagePtrs &sp, bool lamb, const float *q,
+                                                uint32_t dupmask, float thr, int base, int loc0, int64_t job, int L)
+{
+    long long key = 0x7fffffffffffffffLL;
+    int bi = kIdxNone;
+    if (lamb) {
+#pragma unroll
+        for (int o = 0; o < 4; ++o) {
+            const bool cand = c.sp.exact ? !((dupmask >> o) & 1u) : (q[o] <= thr);
+            if (!cand)
+                continue;
+            int32_t u[Cols<RT>::N];
+            load_units_smem<RT>(sp.units + (size_t)(base + o) * c.R, u, c.R);
+            const long long k = order_key(exact_score<RT, G>(u, sp.vals[base + o], 0, c.sp, c.R, c.rg));
+            if (k < key) {
+                key = k;
+                bi = loc0 + o;
+            }
+        }
+    }
+    for (int dd = 1; dd < L; dd <<= 1) {
+        const long long ok = __shfl_xor_sync(FULL, key, dd);
+        const int oi = __shfl_xor_sync(FULL, bi, dd);
+        if (ok < key || (ok == key && oi < bi)) {
+            key = ok;
+            bi = oi;
+        }
+    }
+    if (lamb && bi >= loc0 && bi < loc0 + 4) {
+        const int i = base + (bi - loc0);
+        int32_t uw[Cols<RT>::N];
+        load_units_smem<RT>(sp.units + (size_t)i * c.R, uw, c.R);
+        take_winner<RT, G>(c, job, bi, uw, sp.vals[i], 0, true, key_value(key));
+        atomicAdd(c.st.stats, 1ull);
+    }
+}
+
 // Tile of a table whose jobs all have K options, K in {4, 8, 16, 32}. Each lane evaluates 4
 // consecutive options of one job (a tile row block is 128 options), keeps their smallest and
 // second-smallest screen values, and a log2(K / 4)-step xor butterfly over the job's K / 4 lanes
@@ -727,6 +771,7 @@ __device__ void process_tile_uniform4(WarpCtx<RT, G> &c, const TileDesc &d, cons
         const int base = b + 4 * lane;
         const bool valid = base < n;        // n is a multiple of K, hence of 4
         float q[4] = {INFINITY, INFINITY, INFINITY, INFINITY};
+        uint32_t dupmask = 0;
         if (valid) {
             int32_t u[4][Cols<RT>::N];
             bool dup[4];
@@ -735,9 +780,11 @@ __device__ void process_tile_uniform4(WarpCtx<RT, G> &c, const TileDesc &d, cons
             const double2 vb = reinterpret_cast<const double2 *>(sp.vals + base)[1];
             const double v[4] = {va.x, va.y, vb.x, vb.y};
 #pragma unroll
-            for (int o = 0; o < 4; ++o)
+            for (int o = 0; o < 4; ++o) {
+                dupmask |= dup[o] ? (1u << o) : 0u;
                 if (!dup[o])
                     q[o] = screen_score<RT, G>(u[o], v[o], 0, c.sp, R, c.rg);
+            }
         }
         // smallest and second smallest of the lane's four values
         float a0 = fminf(q[0], q[1]), a1 = fmaxf(q[0], q[1]);
@@ -765,11 +812,10 @@ __device__ void process_tile_uniform4(WarpCtx<RT, G> &c, const TileDesc &d, cons
                 take_winner<RT, G>(c, d.job_begin + (i >> c.log2_k), i & (K - 1), uw, sp.vals[i], 0, false, 0.0);
             }
         }
-        const int jstart = base & ~(K - 1);
-        const int64_t job = d.job_begin + (base >> c.log2_k);
-        const uint32_t amask = __ballot_sync(FULL, valid && amb && base == jstart);
-        if (amask)
-            resolve_row<RT, G>(c, lane, amask, false, sp.units, sp.vals, sp.grp, jstart, jstart + K, thr, job, 0);
+        const bool lamb = valid && amb;
+        if (__any_sync(FULL, lamb))
+            resolve4_in_row<RT, G>(c, sp, lamb, q, dupmask, thr, base, base & (K - 1),
+                                   d.job_begin + (base >> c.log2_k), KL);
     }
 }
 
@@ -792,6 +838,7 @@ __device__ void process_tile_run4(WarpCtx<RT, G> &c, const TileDesc &d, const St
         const bool valid = jl < n_job && sub < m;
         const int base = jl * K + 4 * sub;
         float q[4] = {INFINITY, INFINITY, INFINITY, INFINITY};
+        uint32_t dupmask = 0;
         if (valid) {
             int32_t u[4][Cols<RT>::N];
             bool dup[4];
@@ -800,9 +847,11 @@ __device__ void process_tile_run4(WarpCtx<RT, G> &c, const TileDesc &d, const St
             const double2 vb = reinterpret_cast<const double2 *>(sp.vals + base)[1];
             const double v[4] = {va.x, va.y, vb.x, vb.y};
 #pragma unroll
-            for (int o = 0; o < 4; ++o)
+            for (int o = 0; o < 4; ++o) {
+                dupmask |= dup[o] ? (1u << o) : 0u;
                 if (!dup[o])
                     q[o] = screen_score<RT, G>(u[o], v[o], 0, c.sp, R, c.rg);
+            }
         }
         float a0 = fminf(q[0], q[1]), a1 = fmaxf(q[0], q[1]);
         float b0 = fminf(q[2], q[3]), b1 = fmaxf(q[2], q[3]);
@@ -830,9 +879,9 @@ __device__ void process_tile_run4(WarpCtx<RT, G> &c, const TileDesc &d, const St
                 take_winner<RT, G>(c, job, 4 * sub + w, uw, sp.vals[i], 0, false, 0.0);
             }
         }
-        const uint32_t amask = __ballot_sync(FULL, valid && amb && sub == 0);
-        if (amask)
-            resolve_row<RT, G>(c, lane, amask, false, sp.units, sp.vals, sp.grp, jl * K, jl * K + K, thr, job, 0);
+        const bool lamb = valid && amb;
+        if (__any_sync(FULL, lamb))
+            resolve4_in_row<RT, G>(c, sp, lamb, q, dupmask, thr, base, 4 * sub, job, L);
     }
 }
 
@@ -1072,12 +1121,43 @@ __device__ void process_tile_bigchunk(WarpCtx<RT, G> &c, const TileDesc &d, cons
             load_option<RT, G>(c, false, sp.units, sp.vals, sp.grp, x.idx, big_first, uw, vw, gw);
             take_winner<RT, G>(c, d.job_begin, x.idx, uw, vw, gw, false, 0.0);
         }
+    } else if (!c.sp.exact && !__any_sync(FULL, big_priv.m2 <= thr)) {
+        // every lane holds at most one survivor (q <= thr), its own smallest: those are rescored in
+        // fp64 from global memory, one per lane, and the warp keeps the minimum of (s, index)
+        long long key = 0x7fffffffffffffffLL;
+        int bi = kIdxNone;
+        if (big_priv.m1 <= thr) {
+            int32_t u[Cols<RT>::N];
+            double v;
+            int g;
+            load_option<RT, G>(c, false, sp.units, sp.vals, sp.grp, big_priv.idx, big_first, u, v, g);
+            key = order_key(exact_score<RT, G>(u, v, g, c.sp, c.R, c.rg));
+            bi = big_priv.idx;
+        }
+#pragma unroll
+        for (int dd = 16; dd >= 1; dd >>= 1) {
+            const long long ok = __shfl_xor_sync(FULL, key, dd);
+            const int oi = __shfl_xor_sync(FULL, bi, dd);
+            if (ok < key || (ok == key && oi < bi)) {
+                key = ok;
+                bi = oi;
+            }
+        }
+        if (lane == 0) {
+            int32_t uw[Cols<RT>::N];
+            double vw;
+            int gw;
+            load_option<RT, G>(c, false, sp.units, sp.vals, sp.grp, bi, big_first, uw, vw, gw);
+            take_winner<RT, G>(c, d.job_begin, bi, uw, vw, gw, true, key_value(key));
+            atomicAdd(c.st.stats, 1ull);
+        }
     } else {
         resolve_row<RT, G>(c, lane, 1u, true, sp.units, sp.vals, sp.grp, 0, K, thr, d.job_begin, big_first);
     }
 }
 
-// Issues the bulk copies of tile d into a stage; lane 0 only. Uniform tables need no job offsets.
+// Issues the bulk copies of tile d into a stage; lane 0 only (issuing the copies from several lanes
+// at once measured slower). Uniform tables and runs of the sorted layout need no job offsets.
 __device__ __forceinline__ void issue_tile(const DevTable &t, const TileDesc &d, unsigned char *stage,
                                            const StageLayout &SL, uint32_t bar, bool need_offsets)
 {
@@ -1115,11 +1195,15 @@ __device__ __forceinline__ void issue_tile(const DevTable &t, const TileDesc &d,
                  (uint32_t)(ghi - glo), bar);
 }
 
-// One evaluation pass over every tile: a best response of every job of every (non-stopped) scenario.
-// UNI selects the uniform-K row reduction (tables whose jobs all have the same power-of-two size up
-// to 32, never grouped); otherwise the general segmented path runs.
+// CTAs per SM the evaluation kernel's register budget must allow.
+template <int RT, bool UNI>
+constexpr int pass_min_ctas()
+{
+    return UNI ? ((RT == 4 || RT == 6) ? kMinCtasPerSmNarrow : kMinCtasPerSm) : kMinCtasPerSmGeneral;
+}
+
 template <int RT, bool G, bool UNI, bool PLAIN>
-__global__ void __launch_bounds__(kWarpsPerCta * 32, UNI ? kMinCtasPerSm : kMinCtasPerSmGeneral) k_pass(DevTable t, DevState st, DevPlan pl,
+__global__ void __launch_bounds__(kWarpsPerCta * 32, pass_min_ctas<RT, UNI>()) k_pass(DevTable t, DevState st, DevPlan pl,
                                                                           SolveArgs a, int round, int kind)
 {
     extern __shared__ __align__(128) unsigned char smem[];
@@ -1131,8 +1215,8 @@ __global__ void __launch_bounds__(kWarpsPerCta * 32, UNI ? kMinCtasPerSm : kMinC
     if (k_begin >= k_end)
         return;
 
-    const WarpSmem WS = warp_smem(pl.tile_opt, t.R, G, t.P);
-    const StageLayout SL = stage_layout(pl.tile_opt, t.R, G);
+    const WarpSmem WS = warp_smem(pl.tile_opt, t.R, G, t.P, !UNI);
+    const StageLayout SL = stage_layout(pl.tile_opt, t.R, G, !UNI);
     unsigned char *wsm = smem + (size_t)wid * WS.bytes;
     float *p32s = reinterpret_cast<float *>(wsm + WS.p32);
     const uint32_t bar0 = smem_u32(wsm + WS.bars);
@@ -1165,27 +1249,36 @@ __global__ void __launch_bounds__(kWarpsPerCta * 32, UNI ? kMinCtasPerSm : kMinC
     }
     __syncwarp();
 
-    // prologue: the first kStages-1 tiles in flight. Lane 0 owns the descriptor stream: it reads
-    // each descriptor one tile before issuing it and leaves a copy beside the stage for the warp.
-    TileDesc *descs = reinterpret_cast<TileDesc *>(wsm + WS.descs);
-    const int4 *tiles4 = reinterpret_cast<const int4 *>(pl.tiles);   // a descriptor is two int4
-    int issued = k_begin;
-    int4 dn0 = make_int4(0, 0, 0, 0), dn1 = dn0;
-    if (lane == 0) {
-        dn0 = __ldg(tiles4 + 2 * issued);
-        dn1 = __ldg(tiles4 + 2 * issued + 1);
-    }
-    while (issued < k_end && issued < k_begin + kStages - 1) {
-        if (lane == 0) {
-            const int sidx = (issued - k_begin) % kStages;
-            reinterpret_cast<int4 *>(descs + sidx)[0] = dn0;
-            reinterpret_cast<int4 *>(descs + sidx)[1] = dn1;
-            issue_tile(t, descs[sidx], wsm + sidx * SL.bytes, SL, bar0 + 8 * sidx, need_offsets);
-            if (issued + 1 < k_end) {
-                dn0 = __ldg(tiles4 + 2 * (issued + 1));
-                dn1 = __ldg(tiles4 + 2 * (issued + 1) + 1);
-            }
+    // Tile descriptors reach the warp's ring in blocks of kDescBlock: one cp.async of 16 bytes per
+    // lane fetches a block, issued a whole block before its first tile is issued, so no global
+    // load sits on the per-tile path. Block b uses ring slots (b & 1) * kDescBlock onwards.
+    TileDesc *ring = reinterpret_cast<TileDesc *>(wsm + WS.descs);
+    const unsigned char *tiles_b = reinterpret_cast<const unsigned char *>(pl.tiles);
+    auto fetch_block = [&](int first) {
+        const int ti = first + (lane >> 1);
+        if (lane < 2 * kDescBlock && ti < k_end) {
+            const uint32_t dst = smem_u32(ring + ((ti - k_begin) & (kDescRing - 1))) + 16u * (lane & 1);
+            asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst),
+                         "l"(tiles_b + (size_t)ti * sizeof(TileDesc) + 16 * (lane & 1))
+                         : "memory");
         }
+        asm volatile("cp.async.commit_group;" ::: "memory");
+    };
+    auto wait_blocks = [&]() {
+        asm volatile("cp.async.wait_group 0;" ::: "memory");
+        __syncwarp();
+    };
+    fetch_block(k_begin);
+    fetch_block(k_begin + kDescBlock);
+    wait_blocks();
+
+    // prologue: the first kStages-1 tiles in flight (lane 0 issues every copy)
+    int issued = k_begin;
+    while (issued < k_end && issued < k_begin + kStages - 1) {
+        const int sidx = (issued - k_begin) % kStages;
+        if (lane == 0)
+            issue_tile(t, ring[(issued - k_begin) & (kDescRing - 1)], wsm + sidx * SL.bytes, SL, bar0 + 8 * sidx,
+                       need_offsets);
         ++issued;
     }
     __syncwarp();
@@ -1198,21 +1291,18 @@ __global__ void __launch_bounds__(kWarpsPerCta * 32, UNI ? kMinCtasPerSm : kMinC
     int failed_at = -1;
     for (int k = k_begin; k < k_end; ++k) {
         if (issued < k_end) {   // refill the stage the previous tile used
+            if (((issued - k_begin) & (kDescBlock - 1)) == 0)
+                wait_blocks();  // the block that starts with tile `issued` has landed
             if (lane == 0) {
                 const int sidx = (issued - k_begin) % kStages;
-                reinterpret_cast<int4 *>(descs + sidx)[0] = dn0;
-                reinterpret_cast<int4 *>(descs + sidx)[1] = dn1;
-                issue_tile(t, descs[sidx], wsm + sidx * SL.bytes, SL, bar0 + 8 * sidx, need_offsets);
-                if (issued + 1 < k_end) {
-                    dn0 = __ldg(tiles4 + 2 * (issued + 1));
-                    dn1 = __ldg(tiles4 + 2 * (issued + 1) + 1);
-                }
+                issue_tile(t, ring[(issued - k_begin) & (kDescRing - 1)], wsm + sidx * SL.bytes, SL,
+                           bar0 + 8 * sidx, need_offsets);
                 if (kPrefetchTiles > 0 && k + kPrefetchTiles < k_end)
                     prefetch_tile(t, pl.tiles[k + kPrefetchTiles]);
             }
             ++issued;
         }
-        const TileDesc d = descs[(k - k_begin) % kStages];
+        const TileDesc d = ring[(k - k_begin) & (kDescRing - 1)];
         const int sidx = (k - k_begin) % kStages;
         const uint32_t parity = (uint32_t)(((k - k_begin) / kStages) & 1);
         if (!__all_sync(FULL, wait_stage(bar0 + 8 * sidx, parity, st.err))) {   // uniform decision
@@ -1237,7 +1327,11 @@ __global__ void __launch_bounds__(kWarpsPerCta * 32, UNI ? kMinCtasPerSm : kMinC
                 process_tile_general<RT, G>(c, d, ptrs, big_first, big_carry, lane);
         }
         __syncwarp();
+        // the last tile of a block is done (issued and evaluated): its slots take the block after next
+        if (((k - k_begin) & (kDescBlock - 1)) == kDescBlock - 1)
+            fetch_block(k + 1 + kDescBlock);
     }
+    asm volatile("cp.async.wait_group 0;" ::: "memory");
     if (failed_at < 0) {
         flush<RT, G>(c, lane);
     } else {
@@ -1477,14 +1571,14 @@ auto dispatch_shape(int R, bool grouped, bool uni, F &&f)
 
 }  // namespace
 
-int pass_smem_bytes(int R, bool grouped, int P, int tile_opt)
+int pass_smem_bytes(int R, bool grouped, bool uniform, int P, int tile_opt)
 {
-    return kWarpsPerCta * warp_smem(tile_opt, R, grouped, P).bytes;
+    return kWarpsPerCta * warp_smem(tile_opt, R, grouped, P, !uniform).bytes;
 }
 
 int pass_ctas_per_sm(int R, bool grouped, bool uniform, int P, int tile_opt)
 {
-    const int smem = pass_smem_bytes(R, grouped, P, tile_opt);
+    const int smem = pass_smem_bytes(R, grouped, uniform && !grouped, P, tile_opt);
     return dispatch_shape(R, grouped, uniform && !grouped, [&](auto k) -> int {
         using K = decltype(k);
         if (cudaFuncSetAttribute(K::plain(), cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess ||
@@ -1536,7 +1630,7 @@ cudaError_t launch_pass(const DevTable &t, const DevState &st, const DevPlan &pl
                         PassKind kind, int grid, cudaStream_t stream)
 {
     const bool grouped = t.group != nullptr;
-    const int smem = pass_smem_bytes(t.R, grouped, t.P, pl.tile_opt);
+    const int smem = pass_smem_bytes(t.R, grouped, pl.uniform_k > 0, t.P, pl.tile_opt);
     const bool plain = kind == PASS_ROUND && st.hash_trace == nullptr && st.dual_trace == nullptr;
     dispatch_shape(t.R, grouped, pl.uniform_k > 0, [&](auto k) -> int {
         decltype(k)::launch(plain, grid, smem, stream, t, st, pl, a, round, kind);

@@ -80,7 +80,7 @@ struct ResPlan {
 };
 
 // Dynamic shared memory per CTA of the evaluation kernel.
-int pass_smem_bytes(int R, bool grouped, int P, int tile_opt);
+int pass_smem_bytes(int R, bool grouped, bool uniform, int P, int tile_opt);
 
 // Maximum resident CTAs per SM of the evaluation kernel for this table shape (0 if it cannot run).
 int pass_ctas_per_sm(int R, bool grouped, bool uniform, int P, int tile_opt);

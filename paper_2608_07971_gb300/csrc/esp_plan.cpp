@@ -1,9 +1,34 @@
-// Host tile planner: static work split of one evaluation pass over warps and tiles.
+// Host tile planner: static work split of one evaluation pass over tiles and warps.
 #include "esp_plan.h"
 
 #include <algorithm>
 
 namespace esp {
+
+// Estimated cost of evaluating a tile, in SM cycles of one warp, from clock64 probes of the pass on
+// GB300. A tile costs a fixed part (stage wait, copy issue, bookkeeping) plus one warp-wide step per
+// "row": 128 options four per lane for uniform runs and chunks of large jobs (a run of jobs with K =
+// 4m options gives each job 2^ceil(log2 m) lanes, so 32 / that many jobs share a row), 32 options
+// one per lane otherwise; closing a chunked job adds its cross-warp reduction and winner read.
+static int64_t tile_rows(const TileDesc &d)
+{
+    if (d.flags & TILE_BIG)
+        return (d.n_opt + 127) / 128;
+    if ((d.flags & TILE_RUN) && tile_run_k(d.flags) >= 4) {
+        const int m = tile_run_k(d.flags) / 4;
+        int lanes = 1;
+        while (lanes < m)
+            lanes <<= 1;
+        const int per_row = 32 / lanes;
+        return (d.n_job + per_row - 1) / per_row;
+    }
+    return (d.n_opt + 31) / 32;
+}
+
+static int64_t tile_cost(const TileDesc &d)
+{
+    return 1050 + 1650 * tile_rows(d) + ((d.flags & TILE_BIG_LAST) ? 850 : 0);
+}
 
 bool plan_tiles(const int64_t *off, int32_t S, int32_t J, int32_t tile_opt, int32_t max_warps, Plan &out,
                 const int32_t *scen, const int32_t *runk)
@@ -25,62 +50,72 @@ bool plan_tiles(const int64_t *off, int32_t S, int32_t J, int32_t tile_opt, int3
     for (int64_t j = 0; j < n_jobs; ++j)   // every job needs at least one option
         if (off[j + 1] <= off[j])
             return false;
-    int64_t want = (total + tile_opt - 1) / tile_opt;  // at least a full tile of work per warp
-    int32_t W = (int32_t)std::min<int64_t>(max_warps, std::max<int64_t>(1, want));
-    W = (int32_t)std::min<int64_t>(W, n_jobs);
 
-    std::vector<int64_t> jb(W + 1);
-    jb[0] = 0;
-    jb[W] = n_jobs;
-    for (int32_t w = 1; w < W; ++w) {
-        const int64_t target = (int64_t)((__int128)total * w / W);
-        jb[w] = std::lower_bound(off, off + n_jobs, target) - off;
-        if (jb[w] < jb[w - 1])
-            jb[w] = jb[w - 1];
-    }
-    out.warp_begin.resize(W + 1);
-    for (int32_t w = 0; w < W; ++w) {
-        out.warp_begin[w] = (int32_t)out.tiles.size();
-        int64_t j = jb[w];
-        const int64_t jend = jb[w + 1];
-        while (j < jend) {
-            const int32_t s = scen ? scen[j] : (int32_t)(j / J);
-            const int64_t K = off[j + 1] - off[j];
-            if (K < 1)
-                return false;
-            if (K > tile_opt) {
-                const int64_t nch = (K + tile_opt - 1) / tile_opt;
-                for (int64_t c = 0; c < nch; ++c) {
-                    TileDesc d;
-                    d.opt_begin = off[j] + c * tile_opt;
-                    d.job_begin = j;
-                    d.n_opt = (int32_t)std::min<int64_t>(tile_opt, K - c * tile_opt);
-                    d.n_job = (c == 0) ? 1 : 0;
-                    d.scenario = s;
-                    d.flags = TILE_BIG | (c == 0 ? TILE_BIG_FIRST : 0u) | (c == nch - 1 ? TILE_BIG_LAST : 0u);
-                    out.tiles.push_back(d);
-                }
-                ++j;
-                continue;
+    // 1. tiles in job order: whole jobs of one scenario (and one run) up to tile_opt options, or the
+    //    chunks of a job larger than a tile
+    int64_t j = 0;
+    while (j < n_jobs) {
+        const int32_t s = scen ? scen[j] : (int32_t)(j / J);
+        const int64_t K = off[j + 1] - off[j];
+        if (K > tile_opt) {
+            const int64_t nch = (K + tile_opt - 1) / tile_opt;
+            for (int64_t c = 0; c < nch; ++c) {
+                TileDesc d;
+                d.opt_begin = off[j] + c * tile_opt;
+                d.job_begin = j;
+                d.n_opt = (int32_t)std::min<int64_t>(tile_opt, K - c * tile_opt);
+                d.n_job = (c == 0) ? 1 : 0;
+                d.scenario = s;
+                d.flags = TILE_BIG | (c == 0 ? TILE_BIG_FIRST : 0u) | (c == nch - 1 ? TILE_BIG_LAST : 0u);
+                out.tiles.push_back(d);
             }
-            const int64_t opt0 = off[j];
-            const int32_t rk = runk ? runk[j] : 0;
-            int64_t jj = j;
-            while (jj < jend && (scen ? scen[jj] == s : jj / J == s) && (runk ? runk[jj] == rk : true) &&
-                   off[jj + 1] - opt0 <= tile_opt)
-                ++jj;
-            TileDesc d;
-            d.opt_begin = opt0;
-            d.job_begin = j;
-            d.n_opt = (int32_t)(off[jj] - opt0);
-            d.n_job = (int32_t)(jj - j);
-            d.scenario = s;
-            d.flags = rk > 0 ? tile_run_flags(rk) : 0u;
-            out.tiles.push_back(d);
-            j = jj;
+            ++j;
+            continue;
         }
+        const int64_t opt0 = off[j];
+        const int32_t rk = runk ? runk[j] : 0;
+        int64_t jj = j;
+        while (jj < n_jobs && (scen ? scen[jj] == s : jj / J == s) && (runk ? runk[jj] == rk : true) &&
+               off[jj + 1] - opt0 <= tile_opt)
+            ++jj;
+        TileDesc d;
+        d.opt_begin = opt0;
+        d.job_begin = j;
+        d.n_opt = (int32_t)(off[jj] - opt0);
+        d.n_job = (int32_t)(jj - j);
+        d.scenario = s;
+        d.flags = rk > 0 ? tile_run_flags(rk) : 0u;
+        out.tiles.push_back(d);
+        j = jj;
     }
-    out.warp_begin[W] = (int32_t)out.tiles.size();
+
+    // 2. warps: contiguous tile ranges of about equal estimated cost, at least one full tile of work
+    //    per warp; a range never starts inside the chunks of a large job (its state is per warp)
+    const int64_t n_tiles = (int64_t)out.tiles.size();
+    std::vector<int64_t> pre(n_tiles + 1, 0);
+    for (int64_t k = 0; k < n_tiles; ++k)
+        pre[k + 1] = pre[k] + tile_cost(out.tiles[k]);
+    const int64_t full = 1050 + 1650;     // one row
+    const int64_t want = (pre[n_tiles] + full - 1) / full;
+    const int32_t W = (int32_t)std::min<int64_t>(std::min<int64_t>(max_warps, std::max<int64_t>(1, want)), n_tiles);
+    out.warp_begin.assign(W + 1, 0);
+    out.warp_begin[W] = (int32_t)n_tiles;
+    for (int32_t w = 1; w < W; ++w) {
+        const int64_t target = (int64_t)((__int128)pre[n_tiles] * w / W);
+        int64_t k = std::lower_bound(pre.begin(), pre.end(), target) - pre.begin();
+        if (k > 0 && target - pre[k - 1] < pre[k] - target)   // the nearer tile boundary
+            --k;
+        if (k < n_tiles && (out.tiles[k].flags & TILE_BIG) && !(out.tiles[k].flags & TILE_BIG_FIRST)) {
+            int64_t a = k, b = k;                            // the chunked job's first tile, the next job's
+            while (!(out.tiles[a].flags & TILE_BIG_FIRST))
+                --a;
+            while (b < n_tiles && (out.tiles[b].flags & TILE_BIG) && !(out.tiles[b].flags & TILE_BIG_FIRST))
+                ++b;
+            k = (target - pre[a] < pre[b] - target) ? a : b;
+        }
+        k = std::min<int64_t>(std::max<int64_t>(k, out.warp_begin[w - 1]), n_tiles);
+        out.warp_begin[w] = (int32_t)k;
+    }
     out.n_warps = W;
     return true;
 }

@@ -102,12 +102,41 @@ def test_planner_covers_every_job(lib, case):
             tiles_cover(off, S, J, tiles, wb, tile_opt)
 
 
-def test_planner_balances_options(lib):
+def tile_cost(tiles):
+    """The planner's cost estimate, restated: 1050 + 1650 per row (+850 for the last chunk of a large
+    job); a row is 128 options (chunks, runs of 4m-option jobs: 32 / 2^ceil(log2 m) jobs) or 32."""
+    fl, n_opt, n_job = tiles[:, 7], tiles[:, 4].astype(np.int64), tiles[:, 5].astype(np.int64)
+    big, run = (fl & 1) != 0, (fl & 8) != 0
+    k = (fl >> 8) & 255
+    lanes = np.array([1 << int(np.ceil(np.log2(max(1, kk // 4)))) if kk >= 4 else 1 for kk in k])
+    rows = np.where(big, (n_opt + 127) // 128,
+                    np.where(run & (k >= 4), (n_job + 32 // lanes - 1) // (32 // lanes), (n_opt + 31) // 32))
+    return 1050 + 1650 * rows + np.where((fl & 4) != 0, 850, 0)
+
+
+def test_planner_balances_cost(lib):
+    """Warp ranges have about equal estimated cost: the spread is at most a few tiles' cost, every
+    option is covered, and no range starts inside the chunks of a large job."""
     t = W.whatif_batch(scenarios=range(16), J=2048).table
-    tiles, wb = esp.plan(t.job_off, t.S, t.J, 256, 600)
-    per_warp = np.array([tiles[wb[w]:wb[w + 1], 4].sum() for w in range(len(wb) - 1)])
-    assert per_warp.sum() == t.n_opt
-    assert per_warp.max() - per_warp.min() <= 32
+    for tile_opt, warps in ((256, 600), (128, 3000)):
+        tiles, wb = esp.plan(t.job_off, t.S, t.J, tile_opt, warps)
+        cost = tile_cost(tiles)
+        per_warp = np.array([cost[wb[w]:wb[w + 1]].sum() for w in range(len(wb) - 1)])
+        assert tiles[:, 4].sum() == t.n_opt
+        assert per_warp.max() - per_warp.min() <= cost.max()
+    rng = np.random.default_rng(3)
+    S, J = 4, 3000
+    K = np.minimum(256, rng.zipf(1.3, S * J))
+    off = np.zeros(K.size + 1, np.int64)
+    off[1:] = np.cumsum(K)
+    soff, jmap, scen, runk = esp.sort_layout(off, S, J)
+    tiles, wb = esp.plan_runs(soff, scen, runk, S, J, 128, 257)
+    cost = tile_cost(tiles)
+    per_warp = np.array([cost[wb[w]:wb[w + 1]].sum() for w in range(len(wb) - 1)])
+    # each boundary sits within about one job of two chunks of its target
+    assert per_warp.max() - per_warp.min() <= 4 * cost.max()
+    for w in range(1, len(wb) - 1):
+        assert not (tiles[wb[w], 7] & 1) or (tiles[wb[w], 7] & 2)
 
 
 def test_planner_rejects_bad_offsets(lib):
