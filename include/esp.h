@@ -183,6 +183,43 @@ esp_status esp_evaluate_noalloc(int32_t S, int32_t J, int32_t R, const int64_t *
                                 const double *values, const int64_t *capacity, const double *lambda, int32_t mode,
                                 int32_t *sel, int64_t *demand, double *min_score, void *cuda_stream);
 
+/* The Gamma term of Eq. esp_score for later solves and evaluations. Option c of job j then scores
+ *     rent - v + Gamma_j(c),   Gamma_j(c) = gamma0 * [c != c_cur[j]] + alpha * max(0, s_hat[o] - tau[j]),
+ * the switching cost from the job's current configuration plus the interference penalty of the
+ * predicted co-location slowdown above the job's tolerance (Sec. 3.2.2 and Sec. 3.3; Alg. 1 updates
+ * the slowdowns between ESP rounds). Gamma is computed in fp64 as (c != c_cur ? gamma0 : 0) +
+ * alpha * max(0, s_hat - tau) and applied as the effective value v' = v - Gamma, one correctly
+ * rounded operation per step; every output and objective (primal = sum of v') then refers to v'.
+ *   gamma0  >= 0, finite: switching cost
+ *   c_cur   host, S*J int32: current configuration of each job (local index), -1 for a job without
+ *           one; NULL: no switching cost
+ *   alpha   >= 0, finite: weight of the interference penalty
+ *   s_hat   host, n_opt fp64: predicted slowdown of each option (IAC's output, Eq. dnn_pred); NULL:
+ *           no interference penalty
+ *   tau     host, S*J fp64: tolerance thresholds tau_j(t) (esp_adaptive_threshold); required with
+ *           s_hat, ignored without
+ * gamma0 = 0 with s_hat = NULL restores the loaded values. Errors: ESP_ERR_NOT_LOADED,
+ * ESP_ERR_INVALID_ARG (bad weights, a c_cur at or beyond its job's option count, a non-finite
+ * effective value; the context then holds the loaded values, without penalties). */
+esp_status esp_set_penalties(esp_ctx *ctx, double gamma0, const int32_t *c_cur, double alpha, const double *s_hat,
+                             const double *tau);
+
+/* tau_j(t) of Eq. adaptive_threshold for n jobs (host only, no context):
+ *     tau_out[j] = tau_base[j] + min(beta * (util / util_target - 1), beta_max),
+ * util = U(t) the cluster utilization, util_target = U_target > 0; the additive term is clamped from
+ * above only (Sec. 3.3). Errors: ESP_ERR_INVALID_ARG for null pointers, n < 0 or util_target <= 0. */
+esp_status esp_adaptive_threshold(int64_t n, const double *tau_base, double beta, double util, double util_target,
+                                  double beta_max, double *tau_out);
+
+/* Effective capacity of Eq. effective_capacity (host only): for each of R resources
+ *     c_eff[r] = floor(capacity[r] - gamma * sum over queued jobs q of min over q's options of units[o*R + r]),
+ * at least 1 (a capacity must stay positive). The queue is a CSR table of Q jobs: q_offsets (Q + 1,
+ * q_offsets[0] = 0, every job >= 1 option) and q_units (rows of R int32 >= 0). gamma in [0, 1]
+ * reserves capacity for the queued jobs at their componentwise smallest footprint (Sec. 3.4).
+ * Errors: ESP_ERR_INVALID_ARG. */
+esp_status esp_effective_capacity(int32_t R, const int64_t *capacity, int32_t Q, const int64_t *q_offsets,
+                                  const int32_t *q_units, double gamma, int64_t *c_eff);
+
 /* Number of kernel launches the last esp_solve / esp_solve_async issued. */
 esp_status esp_last_launch_count(esp_ctx *ctx, int64_t *out);
 

@@ -79,6 +79,12 @@ def load(path: Optional[str] = None):
     lib.esp_oracle_solve.argtypes = [T, i32, ctypes.POINTER(_Params), vp, vp, vp, vp, vp,
                                      ctypes.POINTER(_Result), vp, vp, vp, vp, vp]
     lib.esp_oracle_solve.restype = ctypes.c_int
+    lib.esp_oracle_adaptive_threshold.argtypes = [dbl, dbl, dbl, dbl, dbl]
+    lib.esp_oracle_adaptive_threshold.restype = dbl
+    lib.esp_oracle_penalty.argtypes = [i32, i32, dbl, dbl, dbl, dbl]
+    lib.esp_oracle_penalty.restype = dbl
+    lib.esp_oracle_penalized_values.argtypes = [T, dbl, vp, dbl, vp, vp, vp]
+    lib.esp_oracle_effective_capacity.argtypes = [i32, vp, i32, vp, vp, dbl, vp]
     _lib_cache[path] = lib
     return lib
 
@@ -211,3 +217,40 @@ def solve(table, eta0: float, rounds: int, mode: int = NORMALIZED, step: int = S
         l0 = None if lambda0 is None else lambda0[s]
         out.append(solve_scenario(ot, s, eta0, rounds, mode, step, tol, l0, traces, lib=lib))
     return out
+
+
+def adaptive_threshold(tau_base: float, beta: float, util: float, util_target: float, beta_max: float,
+                       lib=None) -> float:
+    """tau_j(t) of Eq. adaptive_threshold."""
+    return (lib or load()).esp_oracle_adaptive_threshold(tau_base, beta, util, util_target, beta_max)
+
+
+def penalty(c: int, c_cur: int, gamma0: float, alpha: float, s_hat: float, tau: float, lib=None) -> float:
+    """Gamma_j(c) of Eq. esp_score: switching cost plus interference penalty."""
+    return (lib or load()).esp_oracle_penalty(c, c_cur, gamma0, alpha, s_hat, tau)
+
+
+def penalized_values(table, gamma0: float = 0.0, c_cur=None, alpha: float = 0.0, s_hat=None, tau=None,
+                     lib=None) -> np.ndarray:
+    """v - Gamma for every option (Eq. esp_score with the Gamma term)."""
+    lib = lib or load()
+    ot = table if isinstance(table, OracleTable) else OracleTable(table)
+    out = np.zeros(ot.values.size)
+    cc = None if c_cur is None else np.ascontiguousarray(c_cur, np.int32)
+    sh = None if s_hat is None else np.ascontiguousarray(s_hat, np.float64)
+    ta = None if tau is None else np.ascontiguousarray(tau, np.float64)
+    lib.esp_oracle_penalized_values(ctypes.byref(ot.c), gamma0, _ptr(cc), alpha, _ptr(sh), _ptr(ta), _ptr(out))
+    return out
+
+
+def effective_capacity(capacity, q_off, q_units, gamma: float, lib=None) -> np.ndarray:
+    """C_eff of Eq. effective_capacity (componentwise minimum footprint of each queued job)."""
+    lib = lib or load()
+    cap = np.ascontiguousarray(capacity, np.int64)
+    qo = np.ascontiguousarray(q_off, np.int64)
+    qu = np.ascontiguousarray(q_units, np.int32)
+    R = cap.size
+    out = np.zeros(R, np.int64)
+    lib.esp_oracle_effective_capacity(R, _ptr(cap), qo.size - 1, _ptr(qo), _ptr(qu), gamma, _ptr(out))
+    return out
+

@@ -240,3 +240,60 @@ int esp_oracle_solve(const esp_oracle_table *t, int32_t s, const esp_oracle_para
     free(score);
     return status;
 }
+
+/* Eq. adaptive_threshold (Sec. 3.3, interference-aware co-location). */
+double esp_oracle_adaptive_threshold(double tau_base, double beta, double util, double util_target,
+                                     double beta_max)
+{
+    double add = beta * (util / util_target - 1.0);
+    if (add > beta_max)
+        add = beta_max;
+    return tau_base + add;
+}
+
+/* Gamma of Eq. esp_score (Sec. 3.2.2): switching cost and interference penalty. */
+double esp_oracle_penalty(int32_t c, int32_t c_cur, double gamma0, double alpha, double s_hat, double tau)
+{
+    const double sw = (c_cur >= 0 && c != c_cur) ? gamma0 : 0.0;
+    double excess = s_hat - tau;
+    if (excess < 0.0)
+        excess = 0.0;
+    const double interference = alpha * excess;
+    return sw + interference;
+}
+
+void esp_oracle_penalized_values(const esp_oracle_table *t, double gamma0, const int32_t *c_cur, double alpha,
+                                 const double *s_hat, const double *tau, double *values_out)
+{
+    const int64_t n_jobs = (int64_t)t->S * t->J;
+    for (int64_t j = 0; j < n_jobs; ++j) {
+        const int32_t cur = c_cur ? c_cur[j] : -1;
+        for (int64_t o = t->job_off[j]; o < t->job_off[j + 1]; ++o) {
+            const int32_t c = (int32_t)(o - t->job_off[j]);
+            const double gamma = esp_oracle_penalty(c, cur, gamma0, s_hat ? alpha : 0.0, s_hat ? s_hat[o] : 0.0,
+                                                    s_hat ? tau[j] : 0.0);
+            values_out[o] = t->values[o] - gamma;
+        }
+    }
+}
+
+/* Eq. effective_capacity (Sec. 3.4, queue-aware capacity reservation). */
+void esp_oracle_effective_capacity(int32_t R, const int64_t *capacity, int32_t Q, const int64_t *q_off,
+                                   const int32_t *q_units, double gamma, int64_t *c_eff)
+{
+    for (int32_t r = 0; r < R; ++r) {
+        int64_t reserved = 0;
+        for (int32_t q = 0; q < Q; ++q) {
+            int32_t m = q_units[q_off[q] * R + r];
+            for (int64_t o = q_off[q] + 1; o < q_off[q + 1]; ++o)
+                if (q_units[o * R + r] < m)
+                    m = q_units[o * R + r];
+            reserved += m;
+        }
+        const double left = (double)capacity[r] - gamma * (double)reserved;
+        int64_t c = (int64_t)floor(left);
+        if (c < 1)
+            c = 1;
+        c_eff[r] = c;
+    }
+}

@@ -98,6 +98,30 @@ int esp_oracle_solve(const esp_oracle_table *t, int32_t s, const esp_oracle_para
                      double *lambda_trace, int64_t *demand_trace, uint64_t *selhash_trace,
                      double *dual_trace, int32_t *sel_trace);
 
+/* tau_j(t) of Eq. adaptive_threshold: tau_base + beta * (U(t) / U_target - 1), the additive term
+ * clamped from above at beta_max (Sec. 3.3: tau_j(t) <= tau_base + beta_max). */
+double esp_oracle_adaptive_threshold(double tau_base, double beta, double util, double util_target,
+                                     double beta_max);
+
+/* Gamma_j^(m)(c) of Eq. esp_score for option c of a job: the switching cost gamma0 * [c != c_cur]
+ * (no switching cost when c_cur < 0, a job without a current configuration) plus the interference
+ * penalty alpha * max(0, s_hat - tau) with s_hat the predicted co-location slowdown of the option
+ * and tau the job's threshold. */
+double esp_oracle_penalty(int32_t c, int32_t c_cur, double gamma0, double alpha, double s_hat, double tau);
+
+/* Values of Eq. esp_score with the Gamma term: v'_o = v_o - Gamma_j(c) for every option of the table
+ * (the score becomes rent - v' = rent - v + Gamma). c_cur: S*J current configurations (local index,
+ * -1 none) or NULL (no switching cost); s_hat: n_opt predicted slowdowns or NULL (no interference
+ * penalty); tau: S*J thresholds (needed with s_hat). values_out: n_opt. */
+void esp_oracle_penalized_values(const esp_oracle_table *t, double gamma0, const int32_t *c_cur, double alpha,
+                                 const double *s_hat, const double *tau, double *values_out);
+
+/* Eq. effective_capacity for P = R priced columns: C_eff_r = C_r - gamma * sum over the queued jobs q
+ * of min over q's options of R_q(c)[r] (componentwise minimum footprint), rounded down to an
+ * integer and kept at least 1. queue: CSR offsets q_off (Q + 1) and units q_units (rows of R). */
+void esp_oracle_effective_capacity(int32_t R, const int64_t *capacity, int32_t Q, const int64_t *q_off,
+                                   const int32_t *q_units, double gamma, int64_t *c_eff);
+
 #ifdef __cplusplus
 }
 #endif

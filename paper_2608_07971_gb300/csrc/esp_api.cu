@@ -62,6 +62,8 @@ struct esp_ctx {
     double *s_values = nullptr;
     int64_t *s_off = nullptr;
     int32_t *s_jmap = nullptr;
+    // Gamma term (esp_set_penalties): the loaded values, kept once penalties are first set
+    double *values0 = nullptr;
     uint16_t *group = nullptr;
     int64_t *cap = nullptr;
     double *vmax = nullptr;
@@ -173,6 +175,7 @@ void release_table(esp_ctx *ctx)
     ctx->s_values = nullptr;
     ctx->s_off = nullptr;
     ctx->s_jmap = nullptr;
+    ctx->values0 = nullptr;
     ctx->res_auto = -1;
     ctx->res_force = -1;
     ctx->loaded = false;
@@ -1001,6 +1004,113 @@ esp_status esp_evaluate(esp_ctx *ctx, const double *lambda, int32_t mode, uint32
         ESP_CUDA(cudaMemcpyAsync(min_score, ctx->job_min, SJ * 8, cudaMemcpyDeviceToHost, ctx->stream));
     ESP_CUDA(cudaStreamSynchronize(ctx->stream));
     return ESP_OK;
+}
+
+namespace {
+
+// After the values changed: clear and redo the duplicate marks, the per-scenario maxima (and the
+// validation they come with) and the sorted copy. Returns the validation flags.
+esp_status refresh_after_values(esp_ctx *ctx, unsigned int *vflags)
+{
+    const DevTable t = dev_table(ctx);
+    ESP_CUDA(launch_clear_marks(ctx->units, ctx->n_opt, ctx->R, ctx->stream));
+    ESP_CUDA(cudaMemsetAsync(ctx->vmax, 0, (size_t)ctx->S * sizeof(double), ctx->stream));
+    ESP_CUDA(cudaMemsetAsync(ctx->umax, 0, (size_t)ctx->S * ctx->R * sizeof(int32_t), ctx->stream));
+    ESP_CUDA(cudaMemsetAsync(ctx->valflags, 0, sizeof(unsigned int), ctx->stream));
+    ESP_CUDA(launch_validate(t, ctx->vmax, ctx->umax, ctx->valflags, ctx->stream));
+    ESP_CUDA(cudaMemsetAsync(ctx->stats + 1, 0, sizeof(unsigned long long), ctx->stream));
+    ESP_CUDA(launch_mark_duplicates(t, ctx->units, ctx->stats + 1, ctx->stream));
+    if (ctx->sorted)
+        ESP_CUDA(launch_gather_sorted(t, pass_table(ctx), ctx->s_units, ctx->s_values, ctx->stream));
+    ESP_CUDA(cudaMemcpyAsync(vflags, ctx->valflags, sizeof(unsigned int), cudaMemcpyDeviceToHost, ctx->stream));
+    ESP_CUDA(cudaStreamSynchronize(ctx->stream));
+    return ESP_OK;
+}
+
+}  // namespace
+
+esp_status esp_set_penalties(esp_ctx *ctx, double gamma0, const int32_t *c_cur, double alpha, const double *s_hat,
+                             const double *tau)
+{
+    esp_status st = check_ctx(ctx);
+    if (st != ESP_OK)
+        return st;
+    if (!ctx->loaded)
+        return ESP_ERR_NOT_LOADED;
+    if (!(gamma0 >= 0.0) || !std::isfinite(gamma0) || !(alpha >= 0.0) || !std::isfinite(alpha) || (s_hat && !tau))
+        return ESP_ERR_INVALID_ARG;
+    ESP_CUDA(cudaSetDevice(ctx->device));
+    const size_t n_jobs = (size_t)ctx->S * ctx->J, n_opt = (size_t)ctx->n_opt;
+    if (!ctx->values0) {
+        void *q = nullptr;
+        cudaError_t e = cudaMalloc(&q, n_opt * sizeof(double) + 64);
+        if (e == cudaErrorMemoryAllocation) {
+            cudaGetLastError();
+            return ESP_ERR_OOM;
+        }
+        ESP_CUDA(e);
+        ctx->table_bufs.push_back(q);
+        ctx->values0 = static_cast<double *>(q);
+        ESP_CUDA(cudaMemcpyAsync(ctx->values0, ctx->values, n_opt * sizeof(double), cudaMemcpyDeviceToDevice,
+                                 ctx->stream));
+    }
+    // inputs on the device, for this call only
+    void *buf = nullptr;
+    const size_t cur_b = c_cur ? n_jobs * sizeof(int32_t) : 0, sh_b = s_hat ? n_opt * sizeof(double) : 0,
+                 tau_b = s_hat ? n_jobs * sizeof(double) : 0;
+    const size_t a1 = (cur_b + 255) & ~size_t(255), a2 = (sh_b + 255) & ~size_t(255);
+    if (cur_b + sh_b + tau_b > 0) {
+        cudaError_t e = cudaMalloc(&buf, a1 + a2 + tau_b + 64);
+        if (e == cudaErrorMemoryAllocation) {
+            cudaGetLastError();
+            return ESP_ERR_OOM;
+        }
+        ESP_CUDA(e);
+    }
+    unsigned char *b = static_cast<unsigned char *>(buf);
+    int32_t *d_cur = c_cur ? reinterpret_cast<int32_t *>(b) : nullptr;
+    double *d_sh = s_hat ? reinterpret_cast<double *>(b + a1) : nullptr;
+    double *d_tau = s_hat ? reinterpret_cast<double *>(b + a1 + a2) : nullptr;
+    auto done = [&](esp_status r) {
+        if (buf) {
+            cudaStreamSynchronize(ctx->stream);
+            cudaFree(buf);
+        }
+        return r;
+    };
+#define ESP_PEN_CUDA(call)                          \
+    do {                                            \
+        cudaError_t e_ = (call);                    \
+        if (e_ != cudaSuccess) {                    \
+            cudaGetLastError();                     \
+            return done(cuda_fail(ctx, e_));        \
+        }                                           \
+    } while (0)
+    if (c_cur)
+        ESP_PEN_CUDA(cudaMemcpyAsync(d_cur, c_cur, cur_b, cudaMemcpyHostToDevice, ctx->stream));
+    if (s_hat) {
+        ESP_PEN_CUDA(cudaMemcpyAsync(d_sh, s_hat, sh_b, cudaMemcpyHostToDevice, ctx->stream));
+        ESP_PEN_CUDA(cudaMemcpyAsync(d_tau, tau, tau_b, cudaMemcpyHostToDevice, ctx->stream));
+    }
+    ESP_PEN_CUDA(cudaMemsetAsync(ctx->valflags, 0, sizeof(unsigned int), ctx->stream));
+    ESP_PEN_CUDA(launch_apply_penalties(dev_table(ctx), ctx->values0, d_cur, d_sh, d_tau, gamma0, alpha, ctx->values,
+                                        ctx->valflags, ctx->stream));
+    unsigned int pflags = 0;
+    ESP_PEN_CUDA(cudaMemcpyAsync(&pflags, ctx->valflags, sizeof(unsigned int), cudaMemcpyDeviceToHost, ctx->stream));
+    ESP_PEN_CUDA(cudaStreamSynchronize(ctx->stream));
+#undef ESP_PEN_CUDA
+    if (pflags) {   // back to the loaded values
+        cudaError_t e = cudaMemcpyAsync(ctx->values, ctx->values0, n_opt * sizeof(double), cudaMemcpyDeviceToDevice,
+                                        ctx->stream);
+        if (e != cudaSuccess)
+            return done(cuda_fail(ctx, e));
+    }
+    unsigned int vflags = 0;
+    st = refresh_after_values(ctx, &vflags);
+    if (st != ESP_OK)
+        return done(st);
+    ctx->solved = false;
+    return done((pflags || vflags) ? ESP_ERR_INVALID_ARG : ESP_OK);
 }
 
 esp_status esp_last_launch_count(esp_ctx *ctx, int64_t *out)

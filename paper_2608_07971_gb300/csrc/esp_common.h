@@ -207,6 +207,7 @@ enum : uint32_t {
     VAL_OFFSETS = 4u,
     VAL_GROUP_RANGE = 8u,
     VAL_CAPACITY = 16u,
+    VAL_PENALTY = 32u,    // a current configuration outside its job, or a non-finite effective value
 };
 
 }  // namespace esp

@@ -1431,6 +1431,45 @@ __global__ void k_gather_sorted(DevTable orig, DevTable sorted, int32_t *units, 
     }
 }
 
+// Gamma term of Eq. esp_score folded into the values (one warp per job): v' = v0 - Gamma with
+// Gamma = (c != c_cur ? gamma0 : 0) + alpha * max(0, s_hat - tau), every step one correctly rounded
+// fp64 operation (no contraction), so v' is the oracle's to the bit. Flags a current configuration
+// outside its job or a non-finite result.
+__global__ void k_apply_penalties(DevTable t, const double *values0, const int32_t *c_cur, const double *s_hat,
+                                  const double *tau, double gamma0, double alpha, double *values,
+                                  unsigned int *flags)
+{
+    const int lane = threadIdx.x & 31;
+    const int64_t n_jobs = (int64_t)t.S * t.J;
+    for (int64_t j = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); j < n_jobs;
+         j += (int64_t)gridDim.x * (blockDim.x >> 5)) {
+        const int64_t a = t.job_off[j];
+        const int K = (int)(t.job_off[j + 1] - a);
+        const int32_t cur = c_cur ? c_cur[j] : -1;
+        if (lane == 0 && cur >= K)
+            atomicOr(flags, VAL_PENALTY);
+        const double tj = s_hat ? tau[j] : 0.0;
+        for (int c = lane; c < K; c += 32) {
+            const double sw = (cur >= 0 && c != cur) ? gamma0 : 0.0;
+            double excess = s_hat ? __dsub_rn(s_hat[a + c], tj) : 0.0;
+            if (excess < 0.0)
+                excess = 0.0;
+            const double gamma = __dadd_rn(sw, __dmul_rn(alpha, excess));
+            const double v = __dsub_rn(values0[a + c], gamma);
+            if (!isfinite(v))
+                atomicOr(flags, VAL_PENALTY);
+            values[a + c] = v;
+        }
+    }
+}
+
+// Clears the load-time duplicate marks (sign bit of each option's column-0 unit).
+__global__ void k_clear_marks(int32_t *units, int64_t n_opt, int R)
+{
+    for (int64_t o = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; o < n_opt; o += (int64_t)gridDim.x * blockDim.x)
+        units[o * R] &= 0x7fffffff;
+}
+
 // Final objectives: primal = sum of chosen values, dual g(lambda) at the final prices, feasibility.
 __global__ void k_objectives(DevTable t, DevState st, SolveArgs a)
 {
@@ -1615,6 +1654,27 @@ cudaError_t launch_gather_sorted(const DevTable &orig, const DevTable &sorted, i
         return cudaSuccess;
     const int64_t blocks = std::min<int64_t>((n_jobs + 7) / 8, 1 << 20);
     k_gather_sorted<<<(int)blocks, 256, 0, stream>>>(orig, sorted, units, values);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_apply_penalties(const DevTable &t, const double *values0, const int32_t *c_cur, const double *s_hat,
+                                   const double *tau, double gamma0, double alpha, double *values, unsigned int *flags,
+                                   cudaStream_t stream)
+{
+    const int64_t n_jobs = (int64_t)t.S * t.J;
+    if (n_jobs == 0)
+        return cudaSuccess;
+    const int64_t blocks = std::min<int64_t>((n_jobs + 7) / 8, 1 << 20);
+    k_apply_penalties<<<(int)blocks, 256, 0, stream>>>(t, values0, c_cur, s_hat, tau, gamma0, alpha, values, flags);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_clear_marks(int32_t *units, int64_t n_opt, int R, cudaStream_t stream)
+{
+    if (n_opt == 0)
+        return cudaSuccess;
+    const int64_t blocks = std::min<int64_t>((n_opt + 255) / 256, 1 << 20);
+    k_clear_marks<<<(int)blocks, 256, 0, stream>>>(units, n_opt, R);
     return cudaGetLastError();
 }
 

@@ -96,6 +96,12 @@ cudaError_t launch_mark_duplicates(const DevTable &t, int32_t *units, unsigned l
 // options (units 0 with the duplicate mark, value 0) up to its padded size.
 cudaError_t launch_gather_sorted(const DevTable &orig, const DevTable &sorted, int32_t *units, double *values,
                                  cudaStream_t stream);
+// v' = values0 - Gamma (Eq. esp_score's Gamma term) for every option; flags VAL_PENALTY.
+cudaError_t launch_apply_penalties(const DevTable &t, const double *values0, const int32_t *c_cur, const double *s_hat,
+                                   const double *tau, double gamma0, double alpha, double *values, unsigned int *flags,
+                                   cudaStream_t stream);
+// Clears every duplicate mark of a units array.
+cudaError_t launch_clear_marks(int32_t *units, int64_t n_opt, int R, cudaStream_t stream);
 cudaError_t launch_init(const DevTable &t, const DevState &st, const SolveArgs &a, const double *lambda0,
                         cudaStream_t stream);
 cudaError_t launch_pass(const DevTable &t, const DevState &st, const DevPlan &pl, const SolveArgs &a,

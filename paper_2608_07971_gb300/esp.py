@@ -29,6 +29,7 @@ EXPORTED = [
     "esp_evaluate", "esp_last_launch_count", "esp_pass_times", "esp_status_string", "esp_destroy",
     "esp_debug_tile_options", "esp_debug_plan", "esp_debug_stats", "esp_debug_resident",
     "esp_debug_sort_layout", "esp_debug_plan_runs", "esp_debug_set_sorted_layout", "esp_evaluate_noalloc",
+    "esp_set_penalties", "esp_adaptive_threshold", "esp_effective_capacity",
 ]
 
 
@@ -90,6 +91,10 @@ def load_library(path: Optional[str] = None):
         "esp_debug_plan_runs": ([vp, vp, vp, i32, i32, i32, i32, vp, i32, vp, i32, ctypes.POINTER(i32),
                                  ctypes.POINTER(i32)], st),
         "esp_debug_set_sorted_layout": ([vp, i32], st),
+        "esp_set_penalties": ([vp, ctypes.c_double, vp, ctypes.c_double, vp, vp], st),
+        "esp_adaptive_threshold": ([i64, vp, ctypes.c_double, ctypes.c_double, ctypes.c_double, ctypes.c_double, vp],
+                                   st),
+        "esp_effective_capacity": ([i32, vp, i32, vp, vp, ctypes.c_double, vp], st),
         "esp_debug_plan": ([vp, i32, i32, i32, i32, vp, i32, vp, i32, ctypes.POINTER(i32), ctypes.POINTER(i32)], st),
         "esp_evaluate_noalloc": ([i32, i32, i32, vp, vp, vp, vp, vp, i32, vp, vp, vp, vp], st),
     }
@@ -214,6 +219,35 @@ def esp_debug_resident(ctx: int, force_cs: int = 0):
         return None
     _check(status, "esp_debug_resident")
     return cs.value, nc.value
+
+
+def esp_set_penalties(ctx: int, gamma0: float = 0.0, c_cur=None, alpha: float = 0.0, s_hat=None, tau=None) -> None:
+    """Gamma term of Eq. esp_score for later solves (see include/esp.h)."""
+    cc = None if c_cur is None else np.ascontiguousarray(c_cur, np.int32)
+    sh = None if s_hat is None else np.ascontiguousarray(s_hat, np.float64)
+    ta = None if tau is None else np.ascontiguousarray(tau, np.float64)
+    _check(load_library().esp_set_penalties(ctx, float(gamma0), _p(cc), float(alpha), _p(sh), _p(ta)),
+           "esp_set_penalties")
+
+
+def esp_adaptive_threshold(tau_base, beta: float, util: float, util_target: float, beta_max: float) -> np.ndarray:
+    """tau_j(t) of Eq. adaptive_threshold (host)."""
+    tb = np.ascontiguousarray(tau_base, np.float64)
+    out = np.zeros_like(tb)
+    _check(load_library().esp_adaptive_threshold(tb.size, _p(tb), beta, util, util_target, beta_max, _p(out)),
+           "esp_adaptive_threshold")
+    return out
+
+
+def esp_effective_capacity(capacity, q_offsets, q_units, gamma: float) -> np.ndarray:
+    """C_eff of Eq. effective_capacity (host)."""
+    cap = np.ascontiguousarray(capacity, np.int64)
+    qo = np.ascontiguousarray(q_offsets, np.int64)
+    qu = np.ascontiguousarray(q_units, np.int32)
+    out = np.zeros(cap.size, np.int64)
+    _check(load_library().esp_effective_capacity(cap.size, _p(cap), qo.size - 1, _p(qo), _p(qu), gamma, _p(out)),
+           "esp_effective_capacity")
+    return out
 
 
 def esp_destroy(ctx: int) -> None:

@@ -218,3 +218,25 @@ def test_sorted_layout(lib, case):
                 else:
                     assert np.all(runk[j0:j1] == 0)
             assert np.array_equal(covered, np.diff(soff))
+
+
+def test_host_formulas_match_the_oracle(lib):
+    """esp_adaptive_threshold and esp_effective_capacity (host code of the library) give the oracle's
+    values bit for bit."""
+    import oracle
+    rng = np.random.default_rng(21)
+    tb = rng.random(50) + 1.0
+    for util, beta_max in ((0.93, 0.05), (0.4, 0.2), (1.7, 0.1)):
+        got = esp.esp_adaptive_threshold(tb, 0.3, util, 0.8, beta_max)
+        want = np.array([oracle.adaptive_threshold(x, 0.3, util, 0.8, beta_max) for x in tb])
+        assert np.array_equal(got, want)
+    K = rng.integers(1, 5, 40)
+    q_off = np.zeros(41, np.int64)
+    q_off[1:] = np.cumsum(K)
+    q_units = rng.integers(0, 1000, (int(q_off[-1]), 6)).astype(np.int32)
+    cap = rng.integers(10000, 40000, 6).astype(np.int64)
+    for gamma in (0.0, 0.37, 1.0):
+        assert np.array_equal(esp.esp_effective_capacity(cap, q_off, q_units, gamma),
+                              oracle.effective_capacity(cap, q_off, q_units, gamma))
+    with pytest.raises(esp.EspError):
+        esp.esp_effective_capacity(cap, np.array([0, 0], np.int64), q_units, 0.5)   # an empty queued job

@@ -10,6 +10,7 @@ import numpy as np
 import pytest
 
 import oracle
+from tests import test_oracle_penalties as pen
 from tests import test_oracle_pins as pins
 
 SRC = os.path.join(os.path.dirname(oracle.__file__), "esp_oracle.c")
@@ -31,6 +32,11 @@ MUTANTS = {
     "demand_wrong_column": ("demand[esp_oracle_price_index(t, best, r)] +=", "demand[r % t->P] +="),
     "primal_first_option": ("primal += t->values[t->job_off[(int64_t)s * J + j] + sel[j]];",
                             "primal += t->values[t->job_off[(int64_t)s * J + j]];"),
+    "switching_cost_inverted": ("(c_cur >= 0 && c != c_cur) ? gamma0", "(c_cur >= 0 && c == c_cur) ? gamma0"),
+    "interference_not_clamped": ("    if (excess < 0.0)\n        excess = 0.0;\n", ""),
+    "penalty_added_to_value": ("values_out[o] = t->values[o] - gamma;", "values_out[o] = t->values[o] + gamma;"),
+    "threshold_not_clamped": ("    if (add > beta_max)\n        add = beta_max;\n", ""),
+    "capacity_largest_footprint": ("if (q_units[o * R + r] < m)", "if (q_units[o * R + r] > m)"),
 }
 
 
@@ -58,6 +64,11 @@ def pin_suite():
     yield pins.test_fixed_point_complementary_slackness
     yield pins.test_tolerance_stops_early_and_freezes
     yield pins.test_tolerance_rule_boundary_is_inclusive
+    yield pen.test_adaptive_threshold_closed_form
+    yield pen.test_switching_cost_shifts_switch_price
+    yield pen.test_interference_penalty_only_above_threshold
+    yield pen.test_large_switching_cost_keeps_current_configuration
+    yield pen.test_effective_capacity_hand_example
 
 
 def failing_pins(lib):
