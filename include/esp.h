@@ -183,6 +183,28 @@ esp_status esp_evaluate_noalloc(int32_t S, int32_t J, int32_t R, const int64_t *
                                 const double *values, const int64_t *capacity, const double *lambda, int32_t mode,
                                 int32_t *sel, int64_t *demand, double *min_score, void *cuda_stream);
 
+/* Loads a placement-expanded table in factored form (Sec. 3.3: configurations crossed with nodes,
+ * the co-location slowdown folded into the value), replacing any loaded table. Job j of scenario s
+ * (global job index s*J + j) has KC configurations and KC * N options; option (k, n) has local index
+ * k * N + n, the units of configuration k — columns r < r_global priced by lambda_r, columns
+ * r >= r_global by lambda[r_global + (R - r_global)*n + (r - r_global)], so P = r_global +
+ * (R - r_global) * N — and the value
+ *     cfg_values[j*KC + k] - (double)(sens[j] * D[job_type[j]*NT + node_type[n]])
+ * with the product taken in fp32. The solve is the one esp_load_options would give for the
+ * expanded table (same selections, demands, prices, objectives), computed from the factors:
+ *   cfg_units   host, S*J*KC*R int32 >= 0      cfg_values host, S*J*KC fp64, finite
+ *   sens        host, S*J fp32, finite           job_type   host, S*J int32 in [0, NT)
+ *   node_type   host, N int32 in [0, NT)          D          host, NT*NT fp32, finite
+ *   capacity    host, S*P int64 > 0
+ * 1 <= KC <= 32, 1 <= N <= 64, 1 <= NT <= 64, 1 <= R <= 16, 0 <= r_global < R. esp_set_penalties
+ * and ESP_FLAG_RESIDENT do not apply (ESP_ERR_UNSUPPORTED / the streaming path). Errors:
+ * ESP_ERR_INVALID_ARG, ESP_ERR_UNSUPPORTED (shape beyond the limits of the device), ESP_ERR_OOM,
+ * ESP_ERR_CUDA. */
+esp_status esp_load_placement(esp_ctx *ctx, int32_t S, int32_t J, int32_t KC, int32_t N, int32_t R, int32_t r_global,
+                              const int32_t *cfg_units, const double *cfg_values, const float *sens,
+                              const int32_t *job_type, int32_t NT, const int32_t *node_type, const float *D,
+                              const int64_t *capacity);
+
 /* The Gamma term of Eq. esp_score for later solves and evaluations. Option c of job j then scores
  *     rent - v + Gamma_j(c),   Gamma_j(c) = gamma0 * [c != c_cur[j]] + alpha * max(0, s_hat[o] - tau[j]),
  * the switching cost from the job's current configuration plus the interference penalty of the

@@ -64,6 +64,11 @@ struct esp_ctx {
     int32_t *s_jmap = nullptr;
     // Gamma term (esp_set_penalties): the loaded values, kept once penalties are first set
     double *values0 = nullptr;
+
+    // factored placement table (esp_load_placement): no stored option table
+    bool placement = false;
+    DevPlace place = {};
+    int32_t place_grid = 0;
     uint16_t *group = nullptr;
     int64_t *cap = nullptr;
     double *vmax = nullptr;
@@ -176,6 +181,9 @@ void release_table(esp_ctx *ctx)
     ctx->s_off = nullptr;
     ctx->s_jmap = nullptr;
     ctx->values0 = nullptr;
+    ctx->placement = false;
+    ctx->place = DevPlace{};
+    ctx->place_grid = 0;
     ctx->res_auto = -1;
     ctx->res_force = -1;
     ctx->loaded = false;
@@ -300,6 +308,38 @@ esp_status check_shape(int32_t S, int32_t J, int32_t R, int32_t P, int32_t rg, b
         return ESP_ERR_INVALID_ARG;
     *n_groups = ng;
     return ESP_OK;
+}
+
+// Per-scenario and per-job state of a solve (prices, demands, selections, objectives, status).
+esp_status alloc_solve_state(esp_ctx *ctx)
+{
+    const size_t S = (size_t)ctx->S, SP = (size_t)ctx->S * ctx->P, SJ = (size_t)ctx->S * ctx->J;
+    esp_status a = ESP_OK;
+    auto al = [&](auto **p, size_t n) {
+        if (a == ESP_OK)
+            a = dev_alloc(ctx, p, n);
+    };
+    al(&ctx->lam, SP);
+    al(&ctx->p64, SP);
+    al(&ctx->p32, SP);
+    al(&ctx->ebound, S);
+    al(&ctx->U, SP);
+    al(&ctx->U_final, SP);
+    al(&ctx->hash, S);
+    al(&ctx->sel, SJ);
+    al(&ctx->job_val, SJ);
+    al(&ctx->job_min, SJ);
+    al(&ctx->rounds_run, S);
+    al(&ctx->converged, S);
+    al(&ctx->status, S);
+    al(&ctx->frozen, S);
+    al(&ctx->feasible, S);
+    al(&ctx->best_dual, S);
+    al(&ctx->primal, S);
+    al(&ctx->dual, S);
+    al(&ctx->lambda0, SP);
+    al(&ctx->err, 4);
+    return a;
 }
 
 // Upload (host or device source), validate on the device, plan, allocate the solve state.
@@ -517,29 +557,11 @@ esp_status load_common(esp_ctx *ctx, int32_t S, int32_t J, int32_t R, int32_t P,
         }
     }
 
-    // solve state
-    const size_t SP = (size_t)S * P, SJ = (size_t)n_jobs;
-    ALLOC(ctx->lam, SP);
-    ALLOC(ctx->p64, SP);
-    ALLOC(ctx->p32, SP);
-    ALLOC(ctx->ebound, (size_t)S);
-    ALLOC(ctx->U, SP);
-    ALLOC(ctx->U_final, SP);
-    ALLOC(ctx->hash, (size_t)S);
-    ALLOC(ctx->sel, SJ);
-    ALLOC(ctx->job_val, SJ);
-    ALLOC(ctx->job_min, SJ);
-    ALLOC(ctx->rounds_run, (size_t)S);
-    ALLOC(ctx->converged, (size_t)S);
-    ALLOC(ctx->status, (size_t)S);
-    ALLOC(ctx->frozen, (size_t)S);
-    ALLOC(ctx->feasible, (size_t)S);
-    ALLOC(ctx->best_dual, (size_t)S);
-    ALLOC(ctx->primal, (size_t)S);
-    ALLOC(ctx->dual, (size_t)S);
-    ALLOC(ctx->lambda0, SP);
-    ALLOC(ctx->err, 4);
 #undef ALLOC
+    if ((st = alloc_solve_state(ctx)) != ESP_OK) {
+        release_table(ctx);
+        return st;
+    }
     ESP_CUDA(cudaStreamSynchronize(ctx->stream));
     ctx->loaded = true;
     ctx->solved = false;
@@ -571,9 +593,28 @@ esp_status check_params(const esp_ctx *ctx, const esp_params *p)
     return ESP_OK;
 }
 
+// Every device buffer the solve kernels touch exists (an internal inconsistency is reported on the
+// host instead of reaching a kernel as a null pointer).
+bool state_ready(const esp_ctx *c)
+{
+    const void *need[] = {c->lam, c->p64, c->p32, c->ebound, c->U, c->U_final, c->hash, c->sel, c->job_val,
+                          c->job_min, c->rounds_run, c->converged, c->status, c->frozen, c->feasible,
+                          c->best_dual, c->primal, c->dual, c->lambda0, c->err, c->vmax, c->umax, c->stats,
+                          c->arrive, c->cap, c->scen_warps};
+    for (const void *p : need)
+        if (!p)
+            return false;
+    if (c->placement)
+        return c->place.cfg_units && c->place.cfg_values && c->place.sens && c->place.job_type &&
+               c->place.node_type && c->place.D && c->place.cfg_dup && c->place.warp_job && c->place.n_warps > 0;
+    return c->grid == 0 || (c->tiles && c->warp_begin && c->units && c->values && c->off);
+}
+
 // Queues one whole solve on the stream (captured into a graph when the stream allows it).
 esp_status enqueue_solve(esp_ctx *ctx, const esp_params *p, const DevState &st, bool has_l0)
 {
+    if (!state_ready(ctx))
+        return ESP_ERR_STATE;
     const DevTable t = pass_table(ctx);
     const DevTable t_orig = dev_table(ctx);   // the resident kernel reads the original layout
     DevPlan pl;
@@ -622,7 +663,11 @@ esp_status enqueue_solve(esp_ctx *ctx, const esp_params *p, const DevState &st, 
             e = cudaEventRecordWithFlags(e1, ctx->stream, rf);
         return e;
     };
+    DevPlace pp = ctx->place;
+    pp.scen_warps = fused ? ctx->scen_warps : nullptr;
     auto pass = [&](int r, PassKind kind) -> cudaError_t {
+        if (ctx->placement)
+            return timed_launch([&]() { return launch_place(t, st, pp, a, r, kind, ctx->place_grid, ctx->stream); });
         return timed_launch([&]() { return launch_pass(t, st, pl, a, r, kind, ctx->grid, ctx->stream); });
     };
     auto issue = [&]() -> cudaError_t {
@@ -971,6 +1016,8 @@ esp_status esp_evaluate(esp_ctx *ctx, const double *lambda, int32_t mode, uint32
         if (!(lambda[i] >= 0.0) || !std::isfinite(lambda[i]))
             return ESP_ERR_INVALID_ARG;
     ESP_CUDA(cudaSetDevice(ctx->device));
+    if (!state_ready(ctx))
+        return ESP_ERR_STATE;
     ESP_CUDA(cudaMemcpyAsync(ctx->lambda0, lambda, SP * sizeof(double), cudaMemcpyHostToDevice, ctx->stream));
     const DevTable t = pass_table(ctx);
     DevState ds = dev_state(ctx);
@@ -990,7 +1037,9 @@ esp_status esp_evaluate(esp_ctx *ctx, const double *lambda, int32_t mode, uint32
     a.flags = flags;
     a.exact_only = (flags & ESP_FLAG_EXACT_ONLY) ? 1 : 0;
     ESP_CUDA(launch_init(t, ds, a, ctx->lambda0, ctx->stream));
-    if (ctx->grid > 0)
+    if (ctx->placement)
+        ESP_CUDA(launch_place(t, ds, ctx->place, a, 0, PASS_FINAL, ctx->place_grid, ctx->stream));
+    else if (ctx->grid > 0)
         ESP_CUDA(launch_pass(t, ds, pl, a, 0, PASS_FINAL, ctx->grid, ctx->stream));
     ESP_CUDA(launch_objectives(t, ds, a, ctx->stream));
     ctx->solved = true;
@@ -1003,6 +1052,167 @@ esp_status esp_evaluate(esp_ctx *ctx, const double *lambda, int32_t mode, uint32
     if (min_score)
         ESP_CUDA(cudaMemcpyAsync(min_score, ctx->job_min, SJ * 8, cudaMemcpyDeviceToHost, ctx->stream));
     ESP_CUDA(cudaStreamSynchronize(ctx->stream));
+    return ESP_OK;
+}
+
+esp_status esp_load_placement(esp_ctx *ctx, int32_t S, int32_t J, int32_t KC, int32_t N, int32_t R, int32_t r_global,
+                              const int32_t *cfg_units, const double *cfg_values, const float *sens,
+                              const int32_t *job_type, int32_t NT, const int32_t *node_type, const float *D,
+                              const int64_t *capacity)
+{
+    esp_status st = check_ctx(ctx);
+    if (st != ESP_OK)
+        return st;
+    if (S < 1 || J < 1 || KC < 1 || KC > kPlaceMaxKC || N < 1 || N > kPlaceMaxN || R < 1 || R > kMaxR ||
+        r_global < 0 || r_global >= R || NT < 1 || NT > kPlaceMaxNT || !cfg_units || !cfg_values || !sens ||
+        !job_type || !node_type || !D || !capacity)
+        return ESP_ERR_INVALID_ARG;
+    const int64_t n_jobs = (int64_t)S * J;
+    const int32_t P = r_global + (R - r_global) * N;
+    if (n_jobs >= INT32_MAX)
+        return ESP_ERR_INVALID_ARG;
+    // validation and the per-scenario maxima on the host (the factored table is small)
+    double dmax = 0.0;
+    for (int32_t i = 0; i < NT * NT; ++i) {
+        if (!std::isfinite(D[i]))
+            return ESP_ERR_INVALID_ARG;
+        dmax = std::max(dmax, (double)std::fabs(D[i]));
+    }
+    for (int32_t n = 0; n < N; ++n)
+        if (node_type[n] < 0 || node_type[n] >= NT)
+            return ESP_ERR_INVALID_ARG;
+    for (int64_t i = 0; i < (int64_t)S * P; ++i)
+        if (capacity[i] <= 0)
+            return ESP_ERR_INVALID_ARG;
+    std::vector<double> vmax((size_t)S, 0.0);
+    std::vector<int32_t> umax((size_t)S * R, 0);
+    std::vector<uint32_t> dup((size_t)n_jobs, 0u);
+    int32_t small = 1;
+    for (int64_t j = 0; j < n_jobs; ++j) {
+        const int64_t s = j / J;
+        if (!std::isfinite(sens[j]) || job_type[j] < 0 || job_type[j] >= NT)
+            return ESP_ERR_INVALID_ARG;
+        double vm = 0.0;
+        for (int32_t k = 0; k < KC; ++k) {
+            const double v = cfg_values[j * KC + k];
+            if (!std::isfinite(v))
+                return ESP_ERR_INVALID_ARG;
+            vm = std::max(vm, std::fabs(v));
+            const int32_t *u = cfg_units + (j * KC + k) * R;
+            for (int32_t r = 0; r < R; ++r) {
+                if (u[r] < 0)
+                    return ESP_ERR_INVALID_ARG;
+                umax[(size_t)s * R + r] = std::max(umax[(size_t)s * R + r], u[r]);
+                if (u[r] >= (1 << 23))
+                    small = 0;
+            }
+            for (int32_t k2 = 0; k2 < k; ++k2) {   // configuration k repeats configuration k2
+                if (std::memcmp(&cfg_values[j * KC + k2], &v, sizeof(double)) == 0 &&
+                    std::memcmp(cfg_units + (j * KC + k2) * R, u, sizeof(int32_t) * (size_t)R) == 0) {
+                    dup[(size_t)j] |= 1u << k;
+                    break;
+                }
+            }
+        }
+        // |v_kn| <= |v_k| + |sens * D| (the fp32 product rounds by at most 2^-24 relative)
+        const double bound = vm + std::fabs((double)sens[j]) * dmax * (1.0 + 0x1p-20);
+        vmax[(size_t)s] = std::max(vmax[(size_t)s], bound);
+    }
+    const int smem = place_smem_bytes(R, P, KC, N, NT);
+    int optin = 0;
+    ESP_CUDA(cudaSetDevice(ctx->device));
+    ESP_CUDA(cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, ctx->device));
+    if (smem > optin)
+        return ESP_ERR_UNSUPPORTED;
+    const int per_sm = place_ctas_per_sm(R, P, KC, N, NT);
+    if (per_sm < 1)
+        return ESP_ERR_UNSUPPORTED;
+    release_table(ctx);
+    ctx->S = S;
+    ctx->J = J;
+    ctx->R = R;
+    ctx->P = P;
+    ctx->rg = r_global;
+    ctx->n_groups = N;
+    ctx->n_opt = n_jobs * KC * N;
+    ctx->small_units = small;
+    ctx->placement = true;
+
+    // warps: contiguous job ranges; the warps touching a scenario arrive once for its price update
+    const int32_t W = (int32_t)std::min<int64_t>(n_jobs, (int64_t)ctx->sm_count * per_sm * kPlaceWarps);
+    std::vector<int32_t> wj((size_t)W + 1), sw((size_t)S, 0);
+    for (int32_t w = 0; w <= W; ++w)
+        wj[(size_t)w] = (int32_t)((__int128)n_jobs * w / W);
+    for (int32_t w = 0; w < W; ++w)
+        if (wj[w + 1] > wj[w])
+            for (int64_t sc = wj[w] / J; sc <= (wj[w + 1] - 1) / J; ++sc)
+                ++sw[(size_t)sc];
+
+#define PALLOC(ptr, count)                                \
+    do {                                                  \
+        esp_status a_ = dev_alloc(ctx, &(ptr), (count));  \
+        if (a_ != ESP_OK) {                               \
+            release_table(ctx);                           \
+            return a_;                                    \
+        }                                                 \
+    } while (0)
+    int32_t *d_units = nullptr, *d_jt = nullptr, *d_nt = nullptr, *d_wj = nullptr;
+    double *d_vals = nullptr;
+    float *d_sens = nullptr, *d_D = nullptr;
+    uint32_t *d_dup = nullptr;
+    PALLOC(d_units, (size_t)n_jobs * KC * R);
+    PALLOC(d_vals, (size_t)n_jobs * KC);
+    PALLOC(d_sens, (size_t)n_jobs);
+    PALLOC(d_jt, (size_t)n_jobs);
+    PALLOC(d_nt, (size_t)N);
+    PALLOC(d_D, (size_t)NT * NT);
+    PALLOC(d_dup, (size_t)n_jobs);
+    PALLOC(d_wj, (size_t)W + 1);
+    PALLOC(ctx->scen_warps, (size_t)S);
+    PALLOC(ctx->arrive, (size_t)S);
+    PALLOC(ctx->cap, (size_t)S * P);
+    PALLOC(ctx->vmax, (size_t)S);
+    PALLOC(ctx->umax, (size_t)S * R);
+    PALLOC(ctx->valflags, 4);
+    PALLOC(ctx->stats, 2);
+#undef PALLOC
+    auto h2d = [&](void *dst, const void *src, size_t bytes) {
+        return cudaMemcpyAsync(dst, src, bytes, cudaMemcpyHostToDevice, ctx->stream);
+    };
+    ESP_CUDA(h2d(d_units, cfg_units, (size_t)n_jobs * KC * R * sizeof(int32_t)));
+    ESP_CUDA(h2d(d_vals, cfg_values, (size_t)n_jobs * KC * sizeof(double)));
+    ESP_CUDA(h2d(d_sens, sens, (size_t)n_jobs * sizeof(float)));
+    ESP_CUDA(h2d(d_jt, job_type, (size_t)n_jobs * sizeof(int32_t)));
+    ESP_CUDA(h2d(d_nt, node_type, (size_t)N * sizeof(int32_t)));
+    ESP_CUDA(h2d(d_D, D, (size_t)NT * NT * sizeof(float)));
+    ESP_CUDA(h2d(d_dup, dup.data(), dup.size() * sizeof(uint32_t)));
+    ESP_CUDA(h2d(d_wj, wj.data(), wj.size() * sizeof(int32_t)));
+    ESP_CUDA(h2d(ctx->scen_warps, sw.data(), sw.size() * sizeof(int32_t)));
+    ESP_CUDA(h2d(ctx->cap, capacity, (size_t)S * P * sizeof(int64_t)));
+    ESP_CUDA(h2d(ctx->vmax, vmax.data(), vmax.size() * sizeof(double)));
+    ESP_CUDA(h2d(ctx->umax, umax.data(), umax.size() * sizeof(int32_t)));
+    ctx->place.cfg_units = d_units;
+    ctx->place.cfg_values = d_vals;
+    ctx->place.sens = d_sens;
+    ctx->place.job_type = d_jt;
+    ctx->place.node_type = d_nt;
+    ctx->place.D = d_D;
+    ctx->place.cfg_dup = d_dup;
+    ctx->place.warp_job = d_wj;
+    ctx->place.scen_warps = nullptr;
+    ctx->place.KC = KC;
+    ctx->place.N = N;
+    ctx->place.NT = NT;
+    ctx->place.n_warps = W;
+    ctx->place_grid = (W + kPlaceWarps - 1) / kPlaceWarps;
+    ctx->grid = ctx->place_grid;
+    if ((st = alloc_solve_state(ctx)) != ESP_OK) {
+        release_table(ctx);
+        return st;
+    }
+    ESP_CUDA(cudaStreamSynchronize(ctx->stream));
+    ctx->loaded = true;
+    ctx->solved = false;
     return ESP_OK;
 }
 
@@ -1037,6 +1247,8 @@ esp_status esp_set_penalties(esp_ctx *ctx, double gamma0, const int32_t *c_cur, 
         return st;
     if (!ctx->loaded)
         return ESP_ERR_NOT_LOADED;
+    if (ctx->placement)
+        return ESP_ERR_UNSUPPORTED;
     if (!(gamma0 >= 0.0) || !std::isfinite(gamma0) || !(alpha >= 0.0) || !std::isfinite(alpha) || (s_hat && !tau))
         return ESP_ERR_INVALID_ARG;
     ESP_CUDA(cudaSetDevice(ctx->device));

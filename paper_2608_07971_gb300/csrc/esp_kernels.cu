@@ -209,7 +209,7 @@ __device__ void set_prices(const DevTable &t, const DevState &st, const SolveArg
     double term = 0.0;
     if (lane < R) {
         double pmax = 0.0;
-        if (t.group == nullptr || lane < t.r_global) {
+        if (t.n_groups == 0 || lane < t.r_global) {
             pmax = st.p64[(size_t)s * P + lane];
         } else {
             for (int gi = 0; gi < t.n_groups; ++gi)
@@ -1344,6 +1344,192 @@ __global__ void __launch_bounds__(kWarpsPerCta * 32, pass_min_ctas<RT, UNI>()) k
 }
 
 // ---------------------------------------------------------------------------------------------
+// Factored placement evaluation (esp_load_placement). A job's options are its KC configurations
+// crossed with N nodes, and only the configurations are stored (Sec. 3.3's slowdown enters the
+// value of (k, n) as the fp32 penalty sens_j * D[a_j][b_n]): a pass reads a few hundred bytes per
+// job instead of KC * N options. One warp per job at a time; lane l takes nodes l and l + 32.
+//
+// Screen. G_k = the fp32 chain over the globally priced columns from -v32_k (v truncated as for a
+// stored option), and candidate (k, n) scores q = the fp32 chain over the node's columns from
+// fl(G_k + pen_n). Against the exact s (the fp64 chain from -(v_k - (double)pen_n)) this is one
+// rounding more than the screen of a stored option; with M_s >= max|v_k| + max pen + sum_r max p_r
+// max u_r the error stays within the same E (which has a factor of about 4 to spare), so the
+// screen rule and the exact rule are those of the streaming kernel. Candidates are visited in
+// increasing local index k * N + n on every lane, and configurations that repeat an earlier one
+// of their job (marked at load) are skipped: their twins have lower indices and equal scores.
+
+__host__ __device__ inline int place_warp_bytes(int R, int P, int KC)
+{
+    return round16(KC * R * 4) + round16(KC * 8) + round16(P * 4);
+}
+
+template <int RT>
+__device__ __forceinline__ float place_global_part(const int32_t *u, double v, const ScenarioPrices &sp, int rg)
+{
+    float g = -screen_value(v);
+#pragma unroll
+    for (int r = 0; r < Cols<RT>::N; ++r) {
+        if (r >= rg)
+            break;
+        g = __fmaf_rn(sp.pf[r], __int2float_rn(u[r]), g);
+    }
+    return g;
+}
+
+template <int RT>
+__device__ __forceinline__ float place_node_part(const int32_t *u, float base, const float *p32s, int rg, int R, int n)
+{
+    float q = base;
+    for (int r = rg; r < R; ++r)
+        q = __fmaf_rn(p32s[rg + (R - rg) * n + (r - rg)], __int2float_rn(u[r]), q);
+    return q;
+}
+
+template <int RT, bool PLAIN>
+__global__ void __launch_bounds__(kPlaceWarps * 32, 4) k_place(DevTable t, DevState st, DevPlace pl, SolveArgs a,
+                                                            int round, int kind)
+{
+    extern __shared__ __align__(16) unsigned char smem[];
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+    const int KC = pl.KC, N = pl.N, NT = pl.NT;
+    const int R = RT ? RT : t.R, rg = t.r_global;
+    float *Ds = reinterpret_cast<float *>(smem);
+    int32_t *nts = reinterpret_cast<int32_t *>(smem + round16(NT * NT * 4));
+    unsigned char *wbase = smem + round16(NT * NT * 4) + round16(N * 4) + (size_t)wid * place_warp_bytes(R, t.P, KC);
+    int32_t *us = reinterpret_cast<int32_t *>(wbase);
+    double *vs = reinterpret_cast<double *>(wbase + round16(KC * R * 4));
+    float *p32s = reinterpret_cast<float *>(wbase + round16(KC * R * 4) + round16(KC * 8));
+    for (int i = threadIdx.x; i < NT * NT; i += blockDim.x)
+        Ds[i] = __ldg(pl.D + i);
+    for (int i = threadIdx.x; i < N; i += blockDim.x)
+        nts[i] = __ldg(pl.node_type + i);
+    __syncthreads();
+    const int w = blockIdx.x * kPlaceWarps + wid;
+    if (w >= pl.n_warps)
+        return;
+
+    WarpCtx<RT, true> c;
+    c.t = t;
+    c.st = st;
+    c.scen_warps = pl.scen_warps;
+    c.a = a;
+    c.round = round;
+    c.R = R;
+    c.rg = rg;
+    c.kind = PLAIN ? (int)PASS_ROUND : kind;
+    c.want_min = PLAIN ? false : ((kind == PASS_FINAL) || (st.dual_trace != nullptr));
+    c.want_hash = PLAIN ? false : ((kind == PASS_ROUND) && (st.hash_trace != nullptr));
+    c.uniform_k = 0;
+    c.log2_k = 0;
+    c.s = -1;
+#pragma unroll
+    for (int r = 0; r < Cols<RT>::N; ++r)
+        c.acc[r] = 0;
+    c.hacc = 0;
+
+    const int64_t j_end = pl.warp_job[w + 1];
+    for (int64_t j = pl.warp_job[w]; j < j_end; ++j) {
+        const int sc = (int)(j / t.J);
+        if (sc != c.s)
+            enter_scenario<RT, true>(c, sc, p32s, lane);
+        if (c.sp.skip)
+            continue;
+        __syncwarp();
+        for (int i = lane; i < KC * R; i += 32)
+            us[i] = __ldg(pl.cfg_units + j * KC * R + i);
+        for (int k = lane; k < KC; k += 32)
+            vs[k] = __ldg(pl.cfg_values + j * KC + k);
+        const float sens = __ldg(pl.sens + j);
+        const int aj = __ldg(pl.job_type + j);
+        const uint32_t dup = __ldg(pl.cfg_dup + j);
+        __syncwarp();
+
+        const int n0 = lane, n1 = lane + 32;
+        const bool h0 = n0 < N, h1 = n1 < N;
+        const float pen0 = h0 ? __fmul_rn(sens, Ds[aj * NT + nts[n0]]) : 0.0f;
+        const float pen1 = h1 ? __fmul_rn(sens, Ds[aj * NT + nts[n1]]) : 0.0f;
+        float m1 = INFINITY, m2 = INFINITY;
+        int i1 = kIdxNone;
+        auto fold = [&](float q, int idx) {
+            const bool better = q < m1;
+            m2 = better ? m1 : fminf(m2, q);
+            i1 = better ? idx : i1;
+            m1 = fminf(m1, q);
+        };
+        for (int k = 0; k < KC; ++k) {
+            if ((dup >> k) & 1u)
+                continue;
+            const int32_t *uk = us + k * R;
+            const float g = place_global_part<RT>(uk, vs[k], c.sp, rg);
+            if (h0)
+                fold(place_node_part<RT>(uk, __fadd_rn(g, pen0), p32s, rg, R, n0), k * N + n0);
+            if (h1)
+                fold(place_node_part<RT>(uk, __fadd_rn(g, pen1), p32s, rg, R, n1), k * N + n1);
+        }
+        const Best x = allreduce_best(Best{m1, i1, m2});
+        const float thr = __fadd_ru(x.m1, c.sp.e2);
+        int win = x.idx;
+        double s_w = 0.0;
+        bool has_s = false;
+        if (c.sp.exact || !(x.m2 > thr)) {
+            // survivors rescored in fp64: v_kn = v_k - (double)pen_n, then the chain of Eq. esp_score
+            long long key = 0x7fffffffffffffffLL;
+            int bi = kIdxNone;
+            for (int k = 0; k < KC; ++k) {
+                if ((dup >> k) & 1u)
+                    continue;
+                const int32_t *uk = us + k * R;
+                int32_t u[Cols<RT>::N];
+#pragma unroll
+                for (int r = 0; r < Cols<RT>::N; ++r)
+                    u[r] = (RT != 0 || r < R) ? uk[r] : 0;
+                const float g = place_global_part<RT>(uk, vs[k], c.sp, rg);
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    const int n = h ? n1 : n0;
+                    if (!(h ? h1 : h0))
+                        continue;
+                    const float pen = h ? pen1 : pen0;
+                    const float q = place_node_part<RT>(uk, __fadd_rn(g, pen), p32s, rg, R, n);
+                    if (!c.sp.exact && !(q <= thr))
+                        continue;
+                    const double v = __dsub_rn(vs[k], (double)pen);
+                    const long long kk = order_key(exact_score<RT, true>(u, v, n, c.sp, R, rg));
+                    if (kk < key) {
+                        key = kk;
+                        bi = k * N + n;
+                    }
+                }
+            }
+#pragma unroll
+            for (int dd = 16; dd >= 1; dd >>= 1) {
+                const long long ok = __shfl_xor_sync(FULL, key, dd);
+                const int oi = __shfl_xor_sync(FULL, bi, dd);
+                if (ok < key || (ok == key && oi < bi)) {
+                    key = ok;
+                    bi = oi;
+                }
+            }
+            win = bi;
+            s_w = key_value(key);
+            has_s = true;
+            if (lane == 0)
+                atomicAdd(st.stats, 1ull);
+        }
+        if (lane == 0) {
+            const int k = win / N, n = win - k * N;
+            int32_t u[Cols<RT>::N];
+#pragma unroll
+            for (int r = 0; r < Cols<RT>::N; ++r)
+                u[r] = (RT != 0 || r < R) ? us[k * R + r] : 0;
+            const double v = __dsub_rn(vs[k], (double)__fmul_rn(sens, Ds[aj * NT + nts[n]]));
+            take_winner<RT, true>(c, j, win, u, v, n, has_s, s_w);
+        }
+    }
+    flush<RT, true>(c, lane);
+}
+
+// ---------------------------------------------------------------------------------------------
 // Load-time marking of exact duplicates: option o of a job is marked (sign bit of its column-0
 // unit) when an earlier option of the same job has the same units, value and group. Such an option
 // ties its twin in every round and loses the tie on index, so it never changes a best response;
@@ -1696,6 +1882,56 @@ cudaError_t launch_pass(const DevTable &t, const DevState &st, const DevPlan &pl
         decltype(k)::launch(plain, grid, smem, stream, t, st, pl, a, round, kind);
         return 0;
     });
+    return cudaGetLastError();
+}
+
+int place_smem_bytes(int R, int P, int KC, int N, int NT)
+{
+    return round16(NT * NT * 4) + round16(N * 4) + kPlaceWarps * place_warp_bytes(R, P, KC);
+}
+
+template <typename F>
+static auto place_dispatch(int R, bool plain, F &&f)
+{
+    if (R == 8)
+        return plain ? f(reinterpret_cast<const void *>(&k_place<8, true>)) : f(reinterpret_cast<const void *>(&k_place<8, false>));
+    return plain ? f(reinterpret_cast<const void *>(&k_place<0, true>)) : f(reinterpret_cast<const void *>(&k_place<0, false>));
+}
+
+int place_ctas_per_sm(int R, int P, int KC, int N, int NT)
+{
+    const int smem = place_smem_bytes(R, P, KC, N, NT);
+    int best = 1 << 30;
+    for (int plain = 0; plain < 2; ++plain) {
+        const int n = place_dispatch(R, plain != 0, [&](const void *fn) -> int {
+            if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess)
+                return 0;
+            int m = 0;
+            if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&m, fn, kPlaceWarps * 32, smem) != cudaSuccess)
+                return 0;
+            return m;
+        });
+        best = n < best ? n : best;
+    }
+    return best;
+}
+
+cudaError_t launch_place(const DevTable &t, const DevState &st, const DevPlace &pl, const SolveArgs &a, int round,
+                         PassKind kind, int grid, cudaStream_t stream)
+{
+    const int smem = place_smem_bytes(t.R, t.P, pl.KC, pl.N, pl.NT);
+    const bool plain = kind == PASS_ROUND && st.hash_trace == nullptr && st.dual_trace == nullptr;
+    if (t.R == 8) {
+        if (plain)
+            k_place<8, true><<<grid, kPlaceWarps * 32, smem, stream>>>(t, st, pl, a, round, kind);
+        else
+            k_place<8, false><<<grid, kPlaceWarps * 32, smem, stream>>>(t, st, pl, a, round, kind);
+    } else {
+        if (plain)
+            k_place<0, true><<<grid, kPlaceWarps * 32, smem, stream>>>(t, st, pl, a, round, kind);
+        else
+            k_place<0, false><<<grid, kPlaceWarps * 32, smem, stream>>>(t, st, pl, a, round, kind);
+    }
     return cudaGetLastError();
 }
 

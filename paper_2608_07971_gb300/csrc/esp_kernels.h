@@ -69,6 +69,34 @@ struct SolveArgs {
 
 enum PassKind : int32_t { PASS_ROUND = 0, PASS_FINAL = 1 };
 
+// A placement table in factored form (esp_load_placement): option (k, n) of job j, local index
+// k * N + n, has the units of configuration k (columns r >= r_global priced per node n, as a group)
+// and the value cfg_values[j*KC + k] - (double)(sens[j] *fp32 D[job_type[j]*NT + node_type[n]]).
+// Warps own contiguous job ranges.
+struct DevPlace {
+    const int32_t *cfg_units;     // n_jobs * KC * R
+    const double *cfg_values;     // n_jobs * KC
+    const float *sens;            // n_jobs
+    const int32_t *job_type;      // n_jobs
+    const int32_t *node_type;     // N
+    const float *D;               // NT * NT
+    const uint32_t *cfg_dup;      // n_jobs: bit k = configuration k repeats an earlier one of its job
+    const int32_t *warp_job;      // n_warps + 1: first job of each warp
+    const int32_t *scen_warps;    // S warps owning jobs of each scenario; non-null: round passes update prices
+    int32_t KC, N, NT, n_warps;
+};
+
+constexpr int kPlaceMaxKC = 32;
+constexpr int kPlaceMaxN = 64;
+constexpr int kPlaceMaxNT = 64;
+constexpr int kPlaceWarps = 4;
+
+// Dynamic shared memory and resident CTAs per SM of the placement kernel (0 if it cannot run).
+int place_smem_bytes(int R, int P, int KC, int N, int NT);
+int place_ctas_per_sm(int R, int P, int KC, int N, int NT);
+cudaError_t launch_place(const DevTable &t, const DevState &st, const DevPlace &pl, const SolveArgs &a, int round,
+                         PassKind kind, int grid, cudaStream_t stream);
+
 // Plan of the cluster-resident kernel: one cluster of cs CTAs per scenario; CTA c of scenario s holds
 // the scenario-local jobs [cuts[s*(cs+1) + c], cuts[s*(cs+1) + c + 1]) in shared memory.
 struct ResPlan {

@@ -29,7 +29,7 @@ EXPORTED = [
     "esp_evaluate", "esp_last_launch_count", "esp_pass_times", "esp_status_string", "esp_destroy",
     "esp_debug_tile_options", "esp_debug_plan", "esp_debug_stats", "esp_debug_resident",
     "esp_debug_sort_layout", "esp_debug_plan_runs", "esp_debug_set_sorted_layout", "esp_evaluate_noalloc",
-    "esp_set_penalties", "esp_adaptive_threshold", "esp_effective_capacity",
+    "esp_set_penalties", "esp_adaptive_threshold", "esp_effective_capacity", "esp_load_placement",
 ]
 
 
@@ -92,6 +92,7 @@ def load_library(path: Optional[str] = None):
                                  ctypes.POINTER(i32)], st),
         "esp_debug_set_sorted_layout": ([vp, i32], st),
         "esp_set_penalties": ([vp, ctypes.c_double, vp, ctypes.c_double, vp, vp], st),
+        "esp_load_placement": ([vp, i32, i32, i32, i32, i32, i32, vp, vp, vp, vp, i32, vp, vp, vp], st),
         "esp_adaptive_threshold": ([i64, vp, ctypes.c_double, ctypes.c_double, ctypes.c_double, ctypes.c_double, vp],
                                    st),
         "esp_effective_capacity": ([i32, vp, i32, vp, vp, ctypes.c_double, vp], st),
@@ -221,6 +222,18 @@ def esp_debug_resident(ctx: int, force_cs: int = 0):
     return cs.value, nc.value
 
 
+def esp_load_placement(ctx: int, f) -> None:
+    """Loads a workloads.PlacementFactors-like factored placement table (see include/esp.h)."""
+    arrs = [np.ascontiguousarray(f.cfg_units, np.int32), np.ascontiguousarray(f.cfg_values, np.float64),
+            np.ascontiguousarray(f.sens, np.float32), np.ascontiguousarray(f.job_type, np.int32),
+            np.ascontiguousarray(f.node_type, np.int32), np.ascontiguousarray(f.D, np.float32),
+            np.ascontiguousarray(f.capacity, np.int64)]
+    NT = int(arrs[5].shape[0])
+    _check(load_library().esp_load_placement(ctx, f.S, f.J, f.KC, f.N, f.R, f.r_global, _p(arrs[0]), _p(arrs[1]),
+                                             _p(arrs[2]), _p(arrs[3]), NT, _p(arrs[4]), _p(arrs[5]), _p(arrs[6])),
+           "esp_load_placement")
+
+
 def esp_set_penalties(ctx: int, gamma0: float = 0.0, c_cur=None, alpha: float = 0.0, s_hat=None, tau=None) -> None:
     """Gamma term of Eq. esp_score for later solves (see include/esp.h)."""
     cc = None if c_cur is None else np.ascontiguousarray(c_cur, np.int32)
@@ -304,6 +317,11 @@ class Solver:
         esp_load_options(self.ctx, t.S, t.J, t.R, t.P, t.r_global, arrs["job_off"], arrs["units"],
                          arrs["values"], arrs["group"], arrs["cap"])
         self.shape = (t.S, t.J, t.R, t.P)
+
+    def load_placement(self, f):
+        """Factored placement table (workloads.PlacementFactors)."""
+        esp_load_placement(self.ctx, f)
+        self.shape = (f.S, f.J, f.R, f.r_global + (f.R - f.r_global) * f.N)
 
     def load_device(self, S, J, R, P, r_global, job_off, units, values, group, cap):
         """Table given as device tensors (torch); copied device-to-device."""

@@ -129,6 +129,27 @@ class Workload:
     step: int = STEP_FIXED
     mode: int = NORMALIZED
     seed: int = 0
+    factors: Optional["PlacementFactors"] = None   # placement_expanded: the table before expansion
+
+
+@dataclasses.dataclass
+class PlacementFactors:
+    """A placement-expanded table in factored form: option (k, n) of job j (local index k * N + n)
+    has the units of configuration k (columns r >= r_global priced per node n) and the value
+    cfg_values[j, k] - (double)(sens[j] *fp32 D[job_type[j], node_type[n]])."""
+    S: int
+    J: int
+    KC: int                   # configurations per job
+    N: int                    # nodes
+    R: int
+    r_global: int
+    cfg_units: np.ndarray     # (S*J, KC, R) int32
+    cfg_values: np.ndarray    # (S*J, KC) fp64
+    sens: np.ndarray          # (S*J,) fp32
+    job_type: np.ndarray      # (S*J,) int32
+    node_type: np.ndarray     # (N,) int32
+    D: np.ndarray             # (NT, NT) fp32
+    capacity: np.ndarray      # (S, r_global + (R - r_global) * N) int64
 
 
 # Capacities (Sec. 5.1's testbed scaled to the named clusters): GPU milli-share, GPU memory MiB,
@@ -306,7 +327,13 @@ def placement_expanded(scenarios: Optional[Sequence[int]] = None, J: int = 4096)
     cap = np.tile(cap_row, (S, 1))
     t = OptionTable(S, J, R, P, 6, job_off, units.reshape(-1, R), values.reshape(-1),
                     np.ascontiguousarray(group.reshape(-1)), cap)
-    return Workload("placement_expanded", t, eta0=0.02, rounds=400, seed=seed)
+    cfg_units = np.empty((nj, KC, R), dtype=np.int32)
+    cfg_units[:, :, :6] = cols12
+    cfg_units[:, :, 6] = cols12[:, :, 0]
+    cfg_units[:, :, 7] = cols12[:, :, 1]
+    factors = PlacementFactors(S, J, KC, NODES, R, 6, cfg_units, np.ascontiguousarray(v12, np.float64), sens,
+                               job_type.astype(np.int32), node_type.astype(np.int32), D, cap)
+    return Workload("placement_expanded", t, eta0=0.02, rounds=400, seed=seed, factors=factors)
 
 
 def heavy_tail(scenarios: Optional[Sequence[int]] = None, J: int = 65536) -> Workload:

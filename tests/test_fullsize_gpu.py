@@ -104,3 +104,25 @@ def test_cluster_and_tiny_full(torch):
         lam, sel, dem, res = solve_like_bench(torch, w, T)
         check_properties(w.table, lam, sel, dem, res, T)
         check_against_oracle(w.table, w, T, lam, sel, dem, res, [0])
+
+
+def test_placement_factored_full(torch):
+    """The benchmark's placement workload loaded in factored form, full size, against the oracle."""
+    w = W.placement_expanded()
+    T = w.rounds
+    stream = torch.cuda.Stream()
+    s = esp.Solver(stream=stream.cuda_stream)
+    s.load_placement(w.factors)
+    prm = s.params(w.eta0, T, mode=w.mode, step=w.step)
+    esp.esp_solve_async(s.ctx, prm)
+    t = w.table
+    res = np.zeros(t.S, esp.RESULT_DTYPE)
+    esp.esp_get_result(s.ctx, res)
+    lam = np.zeros((t.S, t.P))
+    sel = np.zeros((t.S, t.J), np.int32)
+    dem = np.zeros((t.S, t.P), np.int64)
+    esp.esp_get_prices(s.ctx, lam)
+    esp.esp_get_selection(s.ctx, sel)
+    esp.esp_get_demand(s.ctx, dem)
+    s.close()
+    check_against_oracle(t, w, T, lam, sel, dem, res, [0])

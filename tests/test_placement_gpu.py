@@ -1,0 +1,104 @@
+"""Factored placement tables (esp_load_placement): the solve computed from configurations x nodes
+without storing the expanded options equals the oracle's solve of the expanded table (and the
+streaming solve of that table) bit for bit."""
+
+import zlib
+
+import numpy as np
+import pytest
+
+import oracle
+from paper_2608_07971_gb300 import esp, workloads as W
+from tests.parity_util import check_solution
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    import torch
+    if not torch.cuda.is_available():
+        pytest.skip("needs a GPU")
+    from paper_2608_07971_gb300 import build
+    build.build()
+    esp.load_library()
+
+
+def expand(f):
+    """The expanded table the factors stand for (include/esp.h's definition, restated)."""
+    nj = f.S * f.J
+    pen = (f.sens[:, None] * f.D[f.job_type][:, f.node_type]).astype(np.float32)
+    values = f.cfg_values[:, :, None] - pen[:, None, :].astype(np.float64)
+    units = np.broadcast_to(f.cfg_units[:, :, None, :], (nj, f.KC, f.N, f.R))
+    group = np.broadcast_to(np.arange(f.N, dtype=np.uint16)[None, None, :], (nj, f.KC, f.N))
+    P = f.r_global + (f.R - f.r_global) * f.N
+    off = np.arange(nj + 1, dtype=np.int64) * (f.KC * f.N)
+    return W.OptionTable(f.S, f.J, f.R, P, f.r_global, off, np.ascontiguousarray(units.reshape(-1, f.R)),
+                         np.ascontiguousarray(values.reshape(-1)), np.ascontiguousarray(group.reshape(-1)),
+                         f.capacity)
+
+
+def random_factors(seed, S=2, J=150, KC=7, N=40, R=5, rg=3, NT=10, dups=True):
+    rng = np.random.default_rng(seed)
+    nj = S * J
+    cu = rng.integers(0, 60, (nj, KC, R)).astype(np.int32)
+    cv = np.exp(rng.standard_normal((nj, KC)))
+    if dups:                                   # some configurations repeat an earlier one
+        cu[::3, KC - 1] = cu[::3, 0]
+        cv[::3, KC - 1] = cv[::3, 0]
+    P = rg + (R - rg) * N
+    cap = np.maximum(1, (0.4 * J * 30 * np.ones((S, P)))).astype(np.int64)
+    cap[:, rg:] //= N
+    return W.PlacementFactors(S, J, KC, N, R, rg, cu, cv, rng.random(nj).astype(np.float32),
+                              rng.integers(0, NT, nj).astype(np.int32), rng.integers(0, NT, N).astype(np.int32),
+                              rng.random((NT, NT)).astype(np.float32), cap)
+
+
+@pytest.mark.parametrize("case", ["bench_shape", "generic"])
+@pytest.mark.parametrize("mode", [esp.ESP_PRICE_NORMALIZED, esp.ESP_PRICE_RAW])
+def test_factored_placement_matches_oracle(case, mode):
+    if case == "bench_shape":
+        f = W.placement_expanded(scenarios=[0, 3], J=256).factors
+    else:
+        f = random_factors(zlib.crc32(b"generic"))
+    t = expand(f)
+    eta = 0.05 if mode == esp.ESP_PRICE_NORMALIZED else 2e-5
+    T = 40
+    s = esp.Solver()
+    s.load_placement(f)
+    sol = s.solve(eta, T, mode=mode, traces=True)
+    assert s.launches() == T + 3
+    check_solution(t, sol, list(range(t.S)), eta, T, mode, esp.ESP_STEP_FIXED)
+    ref = esp.Solver(t).solve(eta, T, mode=mode, traces=True)       # the expanded table, streamed
+    for fld in ("lam", "sel", "demand", "lambda_trace", "demand_trace", "selhash_trace"):
+        assert np.array_equal(getattr(sol, fld), getattr(ref, fld), equal_nan=True), fld
+    ex = s.solve(eta, T, mode=mode, flags=esp.ESP_FLAG_EXACT_ONLY, traces=True)
+    assert np.array_equal(ex.lambda_trace, sol.lambda_trace) and np.array_equal(ex.sel, sol.sel)
+    sep = s.solve(eta, T, mode=mode, flags=esp.ESP_FLAG_PER_ROUND_LAUNCH, traces=True)
+    assert np.array_equal(sep.lambda_trace, sol.lambda_trace)
+
+
+def test_factored_placement_evaluate_at_oracle_prices():
+    f = random_factors(7, S=1, J=300)
+    t = expand(f)
+    s = esp.Solver()
+    s.load_placement(f)
+    ref = oracle.solve_scenario(t, 0, 0.05, 25, traces=True)
+    for ti in (0, 9, 24):
+        lam = ref.lambda_trace[ti][None, :]
+        sel, dem, ms = s.evaluate(lam)
+        rsel, rdem, rms = oracle.best_response(t, 0, lam[0], oracle.NORMALIZED)
+        assert np.array_equal(sel[0], rsel) and np.array_equal(dem[0], rdem) and np.array_equal(ms[0], rms)
+
+
+def test_factored_placement_rejects_bad_input():
+    f = random_factors(3, S=1, J=20)
+    bad = W.PlacementFactors(**{**f.__dict__, "job_type": f.job_type.copy()})
+    bad.job_type[4] = 99
+    s = esp.Solver()
+    with pytest.raises(esp.EspError):
+        s.load_placement(bad)
+    s.load_placement(f)
+    with pytest.raises(esp.EspError) as e:
+        esp.esp_set_penalties(s.ctx, gamma0=0.1)
+    assert e.value.status == esp.ESP_ERR_UNSUPPORTED
