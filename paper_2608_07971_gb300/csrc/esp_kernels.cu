@@ -193,29 +193,41 @@ __device__ __forceinline__ bool load_units_global(const int32_t *p, int32_t *u, 
 // Price update (Eq. price_update), one warp per scenario, and the screen bound of the new prices.
 
 // Effective prices p = lambda (RAW) or lambda / C (NORMALIZED), their fp32 copy, and the bound E.
+// A lane's first KEEP prices are unrolled so that their loads and divides overlap (KEEP = 1 where a
+// table has at most 32 prices, keeping the evaluation kernels' register budget).
+template <int KEEP>
 __device__ void set_prices(const DevTable &t, const DevState &st, const SolveArgs &a, int s, int lane)
 {
     const int P = t.P, R = t.R;
     bool huge = false;
-    for (int k = lane; k < P; k += 32) {
+    auto price_of = [&](int k) {
         const double lam = st.lam[(size_t)s * P + k];
         const double p = effective_price(lam, (double)t.cap[(size_t)s * P + k], a.mode);
         st.p64[(size_t)s * P + k] = p;
         st.p32[(size_t)s * P + k] = __double2float_rn(p);
         huge |= !(p <= 0x1p100);
-    }
+    };
+#pragma unroll
+    for (int i = 0; i < KEEP; ++i)
+        if (lane + 32 * i < P)
+            price_of(lane + 32 * i);
+    for (int k = lane + 32 * KEEP; k < P; k += 32)
+        price_of(k);
     __syncwarp();
-    // M_s = max|v| + sum_r (max price of column r over groups) * (max unit of column r)
+    // M_s = max|v| + sum_r (max price of column r over groups) * (max unit of column r); lane r
+    // holds column r's term. The maxima over groups are taken lane-parallel (a max is exact, so the
+    // order does not matter).
     double term = 0.0;
-    if (lane < R) {
-        double pmax = 0.0;
-        if (t.n_groups == 0 || lane < t.r_global) {
-            pmax = st.p64[(size_t)s * P + lane];
-        } else {
-            for (int gi = 0; gi < t.n_groups; ++gi)
-                pmax = fmax(pmax, st.p64[(size_t)s * P + t.r_global + (R - t.r_global) * gi + (lane - t.r_global)]);
-        }
-        term = pmax * (double)st.umax[(size_t)s * R + lane];
+    const int rg = (t.n_groups == 0) ? R : t.r_global;
+    if (lane < rg)
+        term = st.p64[(size_t)s * P + lane] * (double)st.umax[(size_t)s * R + lane];
+    for (int c2 = 0; c2 < R - rg; ++c2) {
+        double pm = 0.0;
+        for (int gi = lane; gi < t.n_groups; gi += 32)
+            pm = fmax(pm, st.p64[(size_t)s * P + rg + (R - rg) * gi + c2]);
+        pm = warp_max(pm);
+        if (lane == rg + c2)
+            term = pm * (double)st.umax[(size_t)s * R + lane];
     }
     const double M = st.vmax[s] + warp_sum_fixed(term);
     huge = __any_sync(FULL, huge);
@@ -248,12 +260,15 @@ __global__ void k_init(DevTable t, DevState st, SolveArgs a, const double *lambd
         st.best_dual[s] = INFINITY;
     }
     __syncwarp();
-    set_prices(t, st, a, s, lane);
+    set_prices<8>(t, st, a, s, lane);
 }
 
 // Eq. price_update for scenario s after round `round` (one warp): traces, the projected step, the
 // stopping rule, and the prices and screen bound of the next round. Reads what other warps of the
-// same launch wrote (demand, minimal reduced costs, fingerprint) through L2.
+// same launch wrote (demand, minimal reduced costs, fingerprint) through L2. A lane's first KEEP
+// new prices are computed once, unrolled (their loads and divides overlap), and kept in registers
+// for the write; the rest are recomputed.
+template <int KEEP>
 __device__ void update_scenario(const DevTable &t, const DevState &st, const SolveArgs &a, int s, int round,
                                 int lane)
 {
@@ -282,13 +297,31 @@ __device__ void update_scenario(const DevTable &t, const DevState &st, const Sol
     const double eta = step_size(a.eta0, a.step, round);
     bool bad = false;
     double dmax = 0.0, amax = 0.0;
-    for (int k = lane; k < P; k += 32) {
+    double keep[KEEP];
+    auto step_of = [&](int k, double &lam_out) {
         const long long U = (long long)__ldcg(st.U + sp + k);
         const long long C = t.cap[sp + k];
         if (st.dem_trace)
             st.dem_trace[((size_t)s * T + round) * P + k] = U;
-        const double lam = st.lam[sp + k];
-        const double nl = price_step(lam, U, C, (double)C, eta, a.mode);
+        lam_out = st.lam[sp + k];
+        return price_step(lam_out, U, C, (double)C, eta, a.mode);
+    };
+#pragma unroll
+    for (int i = 0; i < KEEP; ++i) {
+        const int k = lane + 32 * i;
+        keep[i] = 0.0;
+        if (k < P) {
+            double lam;
+            const double nl = step_of(k, lam);
+            keep[i] = nl;
+            bad |= !isfinite(nl);
+            dmax = fmax(dmax, fabs(nl - lam));
+            amax = fmax(amax, fabs(lam));
+        }
+    }
+    for (int k = lane + 32 * KEEP; k < P; k += 32) {
+        double lam;
+        const double nl = step_of(k, lam);
         bad |= !isfinite(nl);
         dmax = fmax(dmax, fabs(nl - lam));
         amax = fmax(amax, fabs(lam));
@@ -305,10 +338,18 @@ __device__ void update_scenario(const DevTable &t, const DevState &st, const Sol
         }
         return;
     }
-    for (int k = lane; k < P; k += 32) {
-        const long long U = (long long)__ldcg(st.U + sp + k);
-        const long long C = t.cap[sp + k];
-        const double nl = price_step(st.lam[sp + k], U, C, (double)C, eta, a.mode);
+    for (int k = lane, i = 0; k < P; k += 32, ++i) {
+        double nl;
+        if (i < KEEP) {
+#pragma unroll
+            for (int q = 0; q < KEEP; ++q)
+                if (q == i)
+                    nl = keep[q];
+        } else {
+            const long long U = (long long)__ldcg(st.U + sp + k);
+            const long long C = t.cap[sp + k];
+            nl = price_step(st.lam[sp + k], U, C, (double)C, eta, a.mode);
+        }
         st.lam[sp + k] = nl;
         st.U[sp + k] = 0ull;
         if (st.lam_trace)
@@ -323,7 +364,7 @@ __device__ void update_scenario(const DevTable &t, const DevState &st, const Sol
         }
     }
     __syncwarp();
-    set_prices(t, st, a, s, lane);
+    set_prices<KEEP>(t, st, a, s, lane);
 }
 
 // Separate price-update launch (used when no warp owns tiles, e.g. J = 0).
@@ -333,7 +374,7 @@ __global__ void k_update(DevTable t, DevState st, SolveArgs a, int round)
     const int s = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
     if (s >= t.S || st.frozen[s])
         return;
-    update_scenario(t, st, a, s, round, lane);
+    update_scenario<8>(t, st, a, s, round, lane);
 }
 
 
@@ -401,7 +442,7 @@ __device__ void flush(WarpCtx<RT, G> &c, int lane)
         old = __shfl_sync(FULL, old, 0);
         if (old + 1 == (unsigned int)__ldg(c.scen_warps + c.s)) {
             asm volatile("fence.acq_rel.gpu;" ::: "memory");
-            update_scenario(c.t, c.st, c.a, c.s, c.round, lane);
+            update_scenario<G ? 8 : 1>(c.t, c.st, c.a, c.s, c.round, lane);
             if (lane == 0)
                 c.st.arrive[c.s] = 0u;     // every warp of this pass has arrived
         }
@@ -1360,7 +1401,8 @@ __global__ void __launch_bounds__(kWarpsPerCta * 32, pass_min_ctas<RT, UNI>()) k
 
 __host__ __device__ inline int place_warp_bytes(int R, int P, int KC)
 {
-    return round16(KC * R * 4) + round16(KC * 8) + round16(P * 4);
+    // configuration units, values, fp32 global parts, fp32 node-column units, fp32 prices
+    return round16(KC * R * 4) + round16(KC * 8) + round16(KC * 4) + round16(KC * R * 4) + round16(P * 4);
 }
 
 template <int RT>
@@ -1376,12 +1418,13 @@ __device__ __forceinline__ float place_global_part(const int32_t *u, double v, c
     return g;
 }
 
+// uf: the configuration's units in fp32 (exact below 2^24, rounded above, as the stored screen does)
 template <int RT>
-__device__ __forceinline__ float place_node_part(const int32_t *u, float base, const float *p32s, int rg, int R, int n)
+__device__ __forceinline__ float place_node_part(const float *uf, float base, const float *p32s, int rg, int R, int n)
 {
     float q = base;
     for (int r = rg; r < R; ++r)
-        q = __fmaf_rn(p32s[rg + (R - rg) * n + (r - rg)], __int2float_rn(u[r]), q);
+        q = __fmaf_rn(p32s[rg + (R - rg) * n + (r - rg)], uf[r], q);
     return q;
 }
 
@@ -1393,17 +1436,12 @@ __global__ void __launch_bounds__(kPlaceWarps * 32, 4) k_place(DevTable t, DevSt
     const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
     const int KC = pl.KC, N = pl.N, NT = pl.NT;
     const int R = RT ? RT : t.R, rg = t.r_global;
-    float *Ds = reinterpret_cast<float *>(smem);
-    int32_t *nts = reinterpret_cast<int32_t *>(smem + round16(NT * NT * 4));
-    unsigned char *wbase = smem + round16(NT * NT * 4) + round16(N * 4) + (size_t)wid * place_warp_bytes(R, t.P, KC);
+    unsigned char *wbase = smem + (size_t)wid * place_warp_bytes(R, t.P, KC);
     int32_t *us = reinterpret_cast<int32_t *>(wbase);
     double *vs = reinterpret_cast<double *>(wbase + round16(KC * R * 4));
-    float *p32s = reinterpret_cast<float *>(wbase + round16(KC * R * 4) + round16(KC * 8));
-    for (int i = threadIdx.x; i < NT * NT; i += blockDim.x)
-        Ds[i] = __ldg(pl.D + i);
-    for (int i = threadIdx.x; i < N; i += blockDim.x)
-        nts[i] = __ldg(pl.node_type + i);
-    __syncthreads();
+    float *gs = reinterpret_cast<float *>(wbase + round16(KC * R * 4) + round16(KC * 8));
+    float *ufs = reinterpret_cast<float *>(wbase + round16(KC * R * 4) + round16(KC * 8) + round16(KC * 4));
+    float *p32s = reinterpret_cast<float *>(wbase + 2 * round16(KC * R * 4) + round16(KC * 8) + round16(KC * 4));
     const int w = blockIdx.x * kPlaceWarps + wid;
     if (w >= pl.n_warps)
         return;
@@ -1443,11 +1481,18 @@ __global__ void __launch_bounds__(kPlaceWarps * 32, 4) k_place(DevTable t, DevSt
         const int aj = __ldg(pl.job_type + j);
         const uint32_t dup = __ldg(pl.cfg_dup + j);
         __syncwarp();
+        // the global part of every configuration once (lane k), and the node columns' units in fp32;
+        // a repeated configuration gets +inf and never survives the screen
+        for (int k = lane; k < KC; k += 32)
+            gs[k] = ((dup >> k) & 1u) ? INFINITY : place_global_part<RT>(us + k * R, vs[k], c.sp, rg);
+        for (int i = lane; i < KC * R; i += 32)
+            ufs[i] = __int2float_rn(us[i]);
+        __syncwarp();
 
         const int n0 = lane, n1 = lane + 32;
         const bool h0 = n0 < N, h1 = n1 < N;
-        const float pen0 = h0 ? __fmul_rn(sens, Ds[aj * NT + nts[n0]]) : 0.0f;
-        const float pen1 = h1 ? __fmul_rn(sens, Ds[aj * NT + nts[n1]]) : 0.0f;
+        const float pen0 = h0 ? __fmul_rn(sens, __ldg(pl.D + aj * NT + __ldg(pl.node_type + n0))) : 0.0f;
+        const float pen1 = h1 ? __fmul_rn(sens, __ldg(pl.D + aj * NT + __ldg(pl.node_type + n1))) : 0.0f;
         float m1 = INFINITY, m2 = INFINITY;
         int i1 = kIdxNone;
         auto fold = [&](float q, int idx) {
@@ -1457,10 +1502,8 @@ __global__ void __launch_bounds__(kPlaceWarps * 32, 4) k_place(DevTable t, DevSt
             m1 = fminf(m1, q);
         };
         for (int k = 0; k < KC; ++k) {
-            if ((dup >> k) & 1u)
-                continue;
-            const int32_t *uk = us + k * R;
-            const float g = place_global_part<RT>(uk, vs[k], c.sp, rg);
+            const float g = gs[k];
+            const float *uk = ufs + k * R;
             if (h0)
                 fold(place_node_part<RT>(uk, __fadd_rn(g, pen0), p32s, rg, R, n0), k * N + n0);
             if (h1)
@@ -1483,14 +1526,14 @@ __global__ void __launch_bounds__(kPlaceWarps * 32, 4) k_place(DevTable t, DevSt
 #pragma unroll
                 for (int r = 0; r < Cols<RT>::N; ++r)
                     u[r] = (RT != 0 || r < R) ? uk[r] : 0;
-                const float g = place_global_part<RT>(uk, vs[k], c.sp, rg);
+                const float g = gs[k];
 #pragma unroll
                 for (int h = 0; h < 2; ++h) {
                     const int n = h ? n1 : n0;
                     if (!(h ? h1 : h0))
                         continue;
                     const float pen = h ? pen1 : pen0;
-                    const float q = place_node_part<RT>(uk, __fadd_rn(g, pen), p32s, rg, R, n);
+                    const float q = place_node_part<RT>(ufs + k * R, __fadd_rn(g, pen), p32s, rg, R, n);
                     if (!c.sp.exact && !(q <= thr))
                         continue;
                     const double v = __dsub_rn(vs[k], (double)pen);
@@ -1522,7 +1565,7 @@ __global__ void __launch_bounds__(kPlaceWarps * 32, 4) k_place(DevTable t, DevSt
 #pragma unroll
             for (int r = 0; r < Cols<RT>::N; ++r)
                 u[r] = (RT != 0 || r < R) ? us[k * R + r] : 0;
-            const double v = __dsub_rn(vs[k], (double)__fmul_rn(sens, Ds[aj * NT + nts[n]]));
+            const double v = __dsub_rn(vs[k], (double)__fmul_rn(sens, __ldg(pl.D + aj * NT + __ldg(pl.node_type + n))));
             take_winner<RT, true>(c, j, win, u, v, n, has_s, s_w);
         }
     }
@@ -1887,7 +1930,9 @@ cudaError_t launch_pass(const DevTable &t, const DevState &st, const DevPlan &pl
 
 int place_smem_bytes(int R, int P, int KC, int N, int NT)
 {
-    return round16(NT * NT * 4) + round16(N * 4) + kPlaceWarps * place_warp_bytes(R, P, KC);
+    (void)N;
+    (void)NT;
+    return kPlaceWarps * place_warp_bytes(R, P, KC);
 }
 
 template <typename F>
