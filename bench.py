@@ -50,6 +50,7 @@ def parse_args():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-resident", action="store_true", help="skip the cluster-resident measurement")
     ap.add_argument("--no-factored", action="store_true", help="skip the factored placement measurement")
+    ap.add_argument("--no-iac", action="store_true", help="skip the IAC predictor measurement")
     ap.add_argument("--cpu-seconds", type=float, default=12.0, help="oracle time budget of the CPU baseline")
     return ap.parse_args()
 
@@ -133,6 +134,53 @@ def kernel_traffic(n_opt_launch: int):
         return float(rec["dram_bytes_per_launch"]) / float(rec["options_per_launch"]) * n_opt_launch
     except Exception:
         return None
+
+
+# fp32 FMA units of a GB300 (152 SMs x 128 lanes) at the maximum SM clock, 2 flops per FMA
+FP32_PEAK_TFLOPS = 152 * 128 * 2 * 2070e6 / 1e12
+
+
+def bench_iac(esp, stream, args, dist, barrier):
+    """Times esp_iac_predict on the IAC what-if batch (S=1024 scenarios x 2048 jobs x 16
+    configurations = 33.5 M pairs, 64 hidden units); one launch per batch."""
+    import torch
+    from paper_2608_07971_gb300 import workloads as W
+    w = W.iac_batch()
+    dev = torch.device("cuda", torch.cuda.current_device())
+    rows = torch.from_numpy(w.rows).to(dev)
+    pairs = torch.from_numpy(w.pairs).to(dev)
+    out = torch.empty(len(w.pairs), dtype=torch.float32, device=dev)
+    pr = esp.Predictor(w.model, stream=stream.cuda_stream)
+    torch.cuda.synchronize()
+    for _ in range(max(3, args.warmup)):
+        pr.predict(rows, pairs, w.c_mem, out)
+    barrier()
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        pr.predict(rows, pairs, w.c_mem, out)
+    e1.record(stream)
+    stream.synchronize()
+    barrier()
+    ms = e0.elapsed_time(e1) / args.steps
+    n = len(w.pairs)
+    value, step_s, _ = aggregate(dist, ms / 1e3, n, device="cuda")
+    H = w.model.W1.shape[0]
+    flops = 2 * (36 * H + H * H + H)
+    achieved = n * flops / (ms / 1e3) / 1e12
+    line = {"value": value, "unit": "pairs/s", "ms_per_step": step_s * 1e3, "pairs_per_step": n,
+            "hidden": H, "launches_per_step": esp.esp_iac_last_launch_count(pr.h),
+            "roofline": {"bound": "alu", "kernel": "k_iac (pair features + 36-H-H-1 network, fp32 FMA)",
+                         "achieved": achieved, "peak": FP32_PEAK_TFLOPS, "unit": "TFLOP/s",
+                         "frac": achieved / FP32_PEAK_TFLOPS, "traffic": None,
+                         "peak_kind": "derived: 152 SMs x 128 fp32 lanes x 2 flops x 2070 MHz",
+                         "flops_per_pair": flops},
+            "workload": f"iac_whatif S={w.S} J={w.J} K={w.K}, pair list {w.pairs.nbytes} B (> L2)"}
+    pr.close()
+    del rows, pairs, out
+    return line
 
 
 class ClockSampler:
@@ -421,6 +469,9 @@ def run_ours(args):
                             "options are never stored; evaluations counted over the expanded options"}
         fs.close()
 
+    # the IAC slowdown predictor (Eq. dnn_pred) over the what-if batch's co-location pairs
+    iac_line = None if args.no_iac else bench_iac(esp, stream, args, dist, barrier)
+
     # end to end through the public API with host inputs
     e2e = None
     if not args.no_e2e:
@@ -472,6 +523,7 @@ def run_ours(args):
         "e2e": e2e,
         "resident": resident,
         "factored": factored,
+        "iac": iac_line,
         "clocks": {k: clocks.get(k) for k in ("sm_mhz", "sm_max_mhz", "reasons")},
         "gpu_launches": int(launches_per_step * args.steps),
     }

@@ -30,6 +30,8 @@ EXPORTED = [
     "esp_debug_tile_options", "esp_debug_plan", "esp_debug_stats", "esp_debug_resident",
     "esp_debug_sort_layout", "esp_debug_plan_runs", "esp_debug_set_sorted_layout", "esp_evaluate_noalloc",
     "esp_set_penalties", "esp_adaptive_threshold", "esp_effective_capacity", "esp_load_placement",
+    "esp_iac_create", "esp_iac_set_stream", "esp_iac_load_model", "esp_iac_predict", "esp_iac_predict_host",
+    "esp_iac_last_launch_count", "esp_iac_destroy",
 ]
 
 
@@ -98,6 +100,13 @@ def load_library(path: Optional[str] = None):
         "esp_effective_capacity": ([i32, vp, i32, vp, vp, ctypes.c_double, vp], st),
         "esp_debug_plan": ([vp, i32, i32, i32, i32, vp, i32, vp, i32, ctypes.POINTER(i32), ctypes.POINTER(i32)], st),
         "esp_evaluate_noalloc": ([i32, i32, i32, vp, vp, vp, vp, vp, i32, vp, vp, vp, vp], st),
+        "esp_iac_create": ([ctypes.POINTER(vp), ctypes.c_int, vp], st),
+        "esp_iac_set_stream": ([vp, vp], st),
+        "esp_iac_load_model": ([vp, i32, vp, vp, vp, vp, vp, vp, vp, ctypes.c_float, ctypes.c_float], st),
+        "esp_iac_predict": ([vp, i32, vp, i64, vp, ctypes.c_float, vp], st),
+        "esp_iac_predict_host": ([vp, i32, vp, i64, vp, ctypes.c_float, vp], st),
+        "esp_iac_last_launch_count": ([vp, ctypes.POINTER(i64)], st),
+        "esp_iac_destroy": ([vp], None),
     }
     for name, (args, res) in sig.items():
         fn = getattr(lib, name)
@@ -419,3 +428,82 @@ def plan_runs(off, scen, runk, S: int, J: int, tile_opt: int, max_warps: int):
 def esp_debug_set_sorted_layout(ctx: int, enable: bool) -> None:
     _check(load_library().esp_debug_set_sorted_layout(ctx, 1 if enable else 0), "esp_debug_set_sorted_layout")
 
+
+
+# --- IAC slowdown predictor (include/esp_iac.h) ------------------------------------------------
+
+def esp_iac_create(device: int = -1, stream: Optional[int] = None) -> int:
+    h = ctypes.c_void_p()
+    _check(load_library().esp_iac_create(ctypes.byref(h), device, stream), "esp_iac_create")
+    return h.value
+
+
+def esp_iac_set_stream(h: int, stream: Optional[int]) -> None:
+    _check(load_library().esp_iac_set_stream(h, stream), "esp_iac_set_stream")
+
+
+def esp_iac_load_model(h: int, model) -> None:
+    """Loads W1, b1, bn1 (4 x H), W2, b2, bn2, W3, b3, eps from any object with those fields."""
+    f32 = lambda a: np.ascontiguousarray(a, np.float32)
+    W1, b1, bn1, W2, b2, bn2, W3 = (f32(getattr(model, n)) for n in ("W1", "b1", "bn1", "W2", "b2", "bn2", "W3"))
+    H = int(W1.shape[0])
+    _check(load_library().esp_iac_load_model(h, H, _p(W1), _p(b1), _p(bn1), _p(W2), _p(b2), _p(bn2), _p(W3),
+                                             float(model.b3), float(model.eps)), "esp_iac_load_model")
+
+
+def esp_iac_predict(h: int, rows, pairs, c_mem: float, out) -> None:
+    """Device variant: rows (n, 14) fp32, pairs (m, 2) int32 and out (m,) fp32 are CUDA tensors;
+    queued on the handle's stream."""
+    n_rows = int(rows.shape[0]) if rows is not None else 0
+    n_pairs = int(pairs.shape[0]) if pairs is not None else 0
+    _check(load_library().esp_iac_predict(h, n_rows, _p(rows), n_pairs, _p(pairs), float(c_mem), _p(out)),
+           "esp_iac_predict")
+
+
+def esp_iac_predict_host(h: int, rows: np.ndarray, pairs: np.ndarray, c_mem: float) -> np.ndarray:
+    rows = np.ascontiguousarray(rows, np.float32).reshape(-1, 14)
+    pairs = np.ascontiguousarray(pairs, np.int32).reshape(-1, 2)
+    out = np.empty(pairs.shape[0], np.float32)
+    _check(load_library().esp_iac_predict_host(h, rows.shape[0], _p(rows), pairs.shape[0], _p(pairs), float(c_mem),
+                                               _p(out)), "esp_iac_predict_host")
+    return out
+
+
+def esp_iac_last_launch_count(h: int) -> int:
+    n = ctypes.c_int64()
+    _check(load_library().esp_iac_last_launch_count(h, ctypes.byref(n)), "esp_iac_last_launch_count")
+    return n.value
+
+
+def esp_iac_destroy(h: int) -> None:
+    load_library().esp_iac_destroy(h)
+
+
+class Predictor:
+    """One esp_iac handle: load a model, then predict slowdowns of co-location pairs."""
+
+    def __init__(self, model=None, device: int = -1, stream: Optional[int] = None):
+        self.h = esp_iac_create(device, stream)
+        if model is not None:
+            esp_iac_load_model(self.h, model)
+
+    def load(self, model) -> None:
+        esp_iac_load_model(self.h, model)
+
+    def predict(self, rows, pairs, c_mem: float, out=None):
+        """numpy inputs: host call, returns numpy; torch CUDA tensors: device call into `out`."""
+        if isinstance(rows, np.ndarray) or isinstance(pairs, np.ndarray):
+            return esp_iac_predict_host(self.h, rows, pairs, c_mem)
+        esp_iac_predict(self.h, rows, pairs, c_mem, out)
+        return out
+
+    def close(self) -> None:
+        if self.h:
+            esp_iac_destroy(self.h)
+            self.h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass

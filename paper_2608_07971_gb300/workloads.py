@@ -33,6 +33,7 @@ _M2 = np.uint64(0x94D049BB133111EB)
 _TAG_NODE = np.uint64(1 << 62)
 _TAG_MATRIX = np.uint64(1 << 61)
 _TAG_CAP = np.uint64(1 << 60)
+_TAG_IAC = np.uint64(1 << 59)
 
 # Field numbers inside a job's stream; configuration k uses 16 + 8k + field.
 F_BASE_Z1, F_BASE_Z2, F_MEM, F_CPU, F_HOST, F_NVL, F_NET, F_K, F_TYPE, F_SENS = range(10)
@@ -354,6 +355,127 @@ def heavy_tail(scenarios: Optional[Sequence[int]] = None, J: int = 65536) -> Wor
     cap = np.maximum(cap, 1)
     t = OptionTable(S, J, R, R, R, job_off, units, value, None, cap)
     return Workload("heavy_tail", t, eta0=0.02, rounds=1000, seed=seed)
+
+
+# ---- IAC co-location pairs (Sec. 3.4.1) ---------------------------------------------------------
+#
+# Profile rows of 14 features per (job, configuration), row index j*K + k, in the order of
+# Sec. 3.4.1: SM Active, SM Occupancy, DRAM Active, Framebuffer Used (MB), Tensor Core Active,
+# workload type (0 training, 1 inference), log-scaled parameter count, isolated throughput,
+# micro-batch, checkpointing flag, mixed-precision flag, ISL, OSL, prefix caching ratio. The
+# paper's profiled co-location experiments are not available; these draws give each feature a
+# plausible range (type, parameter count and the task-level attributes are per job, the hardware
+# metrics and throughput per configuration).
+
+IAC_ROW = 14
+IAC_C_MEM = 81920.0     # MB: an 80 GB device, the paper's example capacity
+# Approximate mean and standard deviation of each of the 36 network inputs under these draws (the
+# pairwise block from two independent rows); used only to scale the synthetic weights.
+IAC_INPUT_MEAN = np.asarray([0.55, 0.36, 0.475, 40024, 0.45, 0.5, 22, 1.13, 5.25, 0.25, 0.4, 2080, 516, 0.225] * 2 +
+                            [0.55, 0.36, 0.475, 0.45, 1.0, 0.977, 0.6, 1.5])
+IAC_INPUT_STD = np.asarray([0.26, 0.2, 0.245, 21925, 0.26, 0.5, 2.31, 0.6, 8.0, 0.43, 0.49, 2700, 660, 0.3] * 2 +
+                           [0.18, 0.14, 0.17, 0.18, 0.71, 0.38, 0.25, 2.0])
+
+
+def iac_rows(seed: int, J: int, K: int) -> np.ndarray:
+    """(J*K, 14) fp32 profile rows."""
+    js = np.repeat(np.arange(J, dtype=np.uint64), K)
+    ks = np.tile(np.arange(K, dtype=np.uint64), J)
+    job = _TAG_IAC | js
+    cfg = _TAG_IAC | (np.uint64(1) << np.uint64(40)) | (js * np.uint64(K) + ks)
+    f = np.zeros((J * K, IAC_ROW), np.float64)
+    wtype = randint(seed, job, 0, 0, 1)
+    f[:, 0] = 0.1 + 0.9 * uniform(seed, cfg, 0)
+    f[:, 1] = f[:, 0] * (0.3 + 0.7 * uniform(seed, cfg, 1))
+    f[:, 2] = 0.05 + 0.85 * uniform(seed, cfg, 2)
+    f[:, 3] = randint(seed, cfg, 3, 2048, 78000)
+    f[:, 4] = 0.9 * uniform(seed, cfg, 4)
+    f[:, 5] = wtype
+    f[:, 6] = 18.0 + 8.0 * uniform(seed, job, 1)
+    f[:, 7] = np.exp(0.5 * normal(seed, cfg, 5, 6))
+    train = wtype == 0
+    f[:, 8] = np.where(train, 2.0 ** randint(seed, job, 2, 0, 5), 0.0)
+    f[:, 9] = np.where(train, randint(seed, cfg, 7, 0, 1), 0)
+    f[:, 10] = np.where(train, (uniform(seed, job, 3) < 0.8).astype(np.float64), 0.0)
+    f[:, 11] = np.where(train, 0, randint(seed, job, 4, 128, 8192))
+    f[:, 12] = np.where(train, 0, randint(seed, job, 5, 16, 2048))
+    f[:, 13] = np.where(train, 0.0, 0.9 * uniform(seed, cfg, 8))
+    return f.astype(np.float32)
+
+
+def iac_pairs(seed: int, S: int, J: int, K: int) -> np.ndarray:
+    """(S*J*K, 2) int32: for what-if scenario s, every configuration k of every job j (row j*K + k)
+    against its co-located partner's current configuration: partner (j + 1 + d) mod J with
+    d ~ U{0..J-2}, at configuration c ~ U{0..K-1}, drawn per (s, j)."""
+    s = np.repeat(np.arange(S, dtype=np.uint64), J)
+    j = np.tile(np.arange(J, dtype=np.uint64), S)
+    st = _TAG_IAC | (np.uint64(2) << np.uint64(40)) | (s << np.uint64(20)) | j
+    d = randint(seed, st, 0, 0, max(J - 2, 0))
+    c = randint(seed, st, 1, 0, K - 1)
+    partner = ((j.astype(np.int64) + 1 + d) % J) * K + c
+    out = np.empty((S * J, K, 2), np.int32)
+    out[:, :, 0] = (j.astype(np.int64) * K)[:, None] + np.arange(K)[None, :]
+    out[:, :, 1] = partner[:, None]
+    return out.reshape(-1, 2)
+
+
+@dataclasses.dataclass
+class IacParams:
+    """Synthetic parameters of the IAC network (the trained weights are not available): W1 (H, 36),
+    b1 (H), bn1 (4, H) = gamma, beta, running mean, running variance; W2 (H, H), b2, bn2; W3 (H), b3;
+    eps. W1 is scaled per input by the inputs' spread so that the first layer sees inputs of order
+    one, as a trained first layer would."""
+
+    W1: np.ndarray
+    b1: np.ndarray
+    bn1: np.ndarray
+    W2: np.ndarray
+    b2: np.ndarray
+    bn2: np.ndarray
+    W3: np.ndarray
+    b3: float
+    eps: float
+
+
+def iac_model(seed: int, H: int = 64, eps: float = 1e-5) -> IacParams:
+    def nrm(layer, n):
+        st = _TAG_IAC | (np.uint64(3 + layer) << np.uint64(40)) | np.arange(n, dtype=np.uint64)
+        return normal(seed, st, 0, 1)
+
+    def uni(layer, n, lo, hi):
+        st = _TAG_IAC | (np.uint64(3 + layer) << np.uint64(40)) | np.arange(n, dtype=np.uint64)
+        return lo + (hi - lo) * uniform(seed, st, 2)
+
+    n_in = 2 * IAC_ROW + 8
+    W1 = nrm(0, H * n_in).reshape(H, n_in) * np.sqrt(2.0 / n_in) / IAC_INPUT_STD
+    b1 = -(W1 @ IAC_INPUT_MEAN) + 0.1 * nrm(1, H)          # inputs centred on their mean
+    bn1 = np.stack([uni(2, H, 0.8, 1.2), 0.2 * nrm(3, H), 0.1 * nrm(4, H), uni(5, H, 0.8, 1.5)])
+    W2 = nrm(6, H * H).reshape(H, H) * np.sqrt(2.0 / H)
+    b2 = 0.1 * nrm(7, H)
+    bn2 = np.stack([uni(8, H, 0.8, 1.2), 0.2 * nrm(9, H), 0.3 * nrm(10, H), uni(11, H, 0.8, 1.5)])
+    W3 = np.abs(nrm(12, H)) * np.sqrt(2.0 / H) * np.where(np.arange(H) % 2 == 0, 1.0, -1.0)
+    f32 = lambda a: np.ascontiguousarray(a, np.float32)
+    return IacParams(W1=f32(W1), b1=f32(b1), bn1=f32(bn1), W2=f32(W2), b2=f32(b2), bn2=f32(bn2), W3=f32(W3),
+                     b3=float(np.float32(0.05)), eps=eps)
+
+
+@dataclasses.dataclass
+class IacWorkload:
+    name: str
+    rows: np.ndarray
+    pairs: np.ndarray
+    c_mem: float
+    model: IacParams
+    S: int
+    J: int
+    K: int
+
+
+def iac_batch(S: int = 1024, J: int = 2048, K: int = 16, H: int = 64, seed: int = 6) -> IacWorkload:
+    """IAC slowdowns for S what-if scenarios of the 512-GPU cluster's shape (J=2048 jobs, K=16
+    configurations): every option against its partner, S*J*K pairs (33.5 M at the defaults)."""
+    return IacWorkload("iac_whatif", iac_rows(seed, J, K), iac_pairs(seed, S, J, K), IAC_C_MEM,
+                       iac_model(seed, H), S, J, K)
 
 
 WORKLOADS = {

@@ -22,7 +22,7 @@ def lib():
 
 def declared_functions():
     names = []
-    for h in ("esp.h", "esp_debug.h"):
+    for h in ("esp.h", "esp_debug.h", "esp_iac.h"):
         src = open(os.path.join(ROOT, "include", h)).read()
         src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
         names += re.findall(r"^\s*(?:const\s+)?\w+\s*\*?\s*(esp_\w+)\s*\(", src, flags=re.M)
