@@ -138,11 +138,23 @@ def kernel_traffic(n_opt_launch: int):
 
 # fp32 FMA units of a GB300 (152 SMs x 128 lanes) at the maximum SM clock, 2 flops per FMA
 FP32_PEAK_TFLOPS = 152 * 128 * 2 * 2070e6 / 1e12
+# nominal dense tf32 / bf16 tensor rate of a GB300 (1.1 / 2.25 PFLOP/s)
+TF32_PER_BF16 = 1.1 / 2.25
+
+
+def tensor_peak_tf32():
+    """tf32 tensor peak: the measured bf16 burst peak x the nominal tf32/bf16 ratio."""
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f)["bf16_tflops"]) * TF32_PER_BF16, "measured bf16_tflops x nominal tf32/bf16"
+    except Exception:
+        return 1900.0 * TF32_PER_BF16, "fallback bf16 x nominal tf32/bf16"
 
 
 def bench_iac(esp, stream, args, dist, barrier):
     """Times esp_iac_predict on the IAC what-if batch (S=1024 scenarios x 2048 jobs x 16
-    configurations = 33.5 M pairs, 64 hidden units); one launch per batch."""
+    configurations = 33.5 M pairs, 64 hidden units), one launch per batch: the tensor-core kernel
+    (the default) and the CUDA-core kernel beside it."""
     import torch
     from paper_2608_07971_gb300 import workloads as W
     w = W.iac_batch()
@@ -150,35 +162,47 @@ def bench_iac(esp, stream, args, dist, barrier):
     rows = torch.from_numpy(w.rows).to(dev)
     pairs = torch.from_numpy(w.pairs).to(dev)
     out = torch.empty(len(w.pairs), dtype=torch.float32, device=dev)
-    pr = esp.Predictor(w.model, stream=stream.cuda_stream)
-    torch.cuda.synchronize()
-    for _ in range(max(3, args.warmup)):
-        pr.predict(rows, pairs, w.c_mem, out)
-    barrier()
-    torch.cuda.synchronize()
-    e0 = torch.cuda.Event(enable_timing=True)
-    e1 = torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    for _ in range(args.steps):
-        pr.predict(rows, pairs, w.c_mem, out)
-    e1.record(stream)
-    stream.synchronize()
-    barrier()
-    ms = e0.elapsed_time(e1) / args.steps
     n = len(w.pairs)
-    value, step_s, _ = aggregate(dist, ms / 1e3, n, device="cuda")
     H = w.model.W1.shape[0]
-    flops = 2 * (36 * H + H * H + H)
-    achieved = n * flops / (ms / 1e3) / 1e12
+
+    def timed(path):
+        pr = esp.Predictor(w.model, stream=stream.cuda_stream, path=path)
+        for _ in range(max(3, args.warmup)):
+            pr.predict(rows, pairs, w.c_mem, out)
+        esp.esp_iac_synchronize(pr.h)
+        barrier()
+        torch.cuda.synchronize()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(args.steps):
+            pr.predict(rows, pairs, w.c_mem, out)
+        e1.record(stream)
+        esp.esp_iac_synchronize(pr.h)
+        barrier()
+        launches = esp.esp_iac_last_launch_count(pr.h)
+        pr.close()
+        return e0.elapsed_time(e1) / args.steps, launches
+
+    flops = 2 * (36 * H + H * H + H)            # algorithmic flops per pair
+    ms_tc, launches = timed(esp.ESP_IAC_PATH_TENSOR)
+    ms_fma, _ = timed(esp.ESP_IAC_PATH_FMA)
+    value, step_s, _ = aggregate(dist, ms_tc / 1e3, n, device="cuda")
+    peak, peak_kind = tensor_peak_tf32()
+    achieved = n * flops / (ms_tc / 1e3) / 1e12
+    mma_flops = 3 * 2 * (40 * 64 + 64 * 64)      # issued by the split (padded K and N)
+    fma_tflops = n * flops / (ms_fma / 1e3) / 1e12
     line = {"value": value, "unit": "pairs/s", "ms_per_step": step_s * 1e3, "pairs_per_step": n,
-            "hidden": H, "launches_per_step": esp.esp_iac_last_launch_count(pr.h),
-            "roofline": {"bound": "alu", "kernel": "k_iac (pair features + 36-H-H-1 network, fp32 FMA)",
-                         "achieved": achieved, "peak": FP32_PEAK_TFLOPS, "unit": "TFLOP/s",
-                         "frac": achieved / FP32_PEAK_TFLOPS, "traffic": None,
-                         "peak_kind": "derived: 152 SMs x 128 fp32 lanes x 2 flops x 2070 MHz",
-                         "flops_per_pair": flops},
+            "hidden": H, "launches_per_step": launches, "dtype": "f32 (tf32x3 tensor-core products)",
+            "roofline": {"bound": "tensor", "kernel": "k_iac_tc (tcgen05 kind::tf32, three-term split)",
+                         "achieved": achieved, "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak,
+                         "traffic": None, "peak_kind": peak_kind, "flops_per_pair": flops,
+                         "mma_flops_per_pair": mma_flops,
+                         "tensor_pipe_frac": n * mma_flops / (ms_tc / 1e3) / 1e12 / peak},
+            "fma_path": {"ms_per_step": ms_fma, "value": n / (ms_fma / 1e3), "achieved": fma_tflops,
+                         "peak": FP32_PEAK_TFLOPS, "unit": "TFLOP/s", "frac": fma_tflops / FP32_PEAK_TFLOPS,
+                         "peak_kind": "derived: 152 SMs x 128 fp32 lanes x 2 flops x 2070 MHz"},
             "workload": f"iac_whatif S={w.S} J={w.J} K={w.K}, pair list {w.pairs.nbytes} B (> L2)"}
-    pr.close()
     del rows, pairs, out
     return line
 

@@ -23,8 +23,9 @@
  * Network (inference: dropout off, Batch Normalization with its running statistics):
  *     h1 = ReLU(BN1(W1 x + b1)),  h2 = ReLU(BN2(W2 h1 + b2)),  S_hat = 1 + ReLU(W3 h2 + b3)
  * (Eq. dnn_pred), BN(z) = gamma (z - mean) / sqrt(var + eps) + beta per unit. Each BN is folded
- * into the preceding layer when the model is loaded; the kernel computes in fp32 with fused
- * multiply-adds in input order.
+ * into the preceding layer when the model is loaded; the kernels compute in fp32 (the hidden layers
+ * on the tensor cores with a three-term tf32 split, or as fused multiply-adds; see
+ * esp_iac_set_path).
  *
  * Conventions are those of esp.h: every function returns an esp_status, "host" pointers are copied
  * during the call, "device" pointers are CUDA device pointers owned by the caller, a handle is used
@@ -46,6 +47,16 @@ extern "C" {
 #define ESP_IAC_MAX_HIDDEN 64
 
 typedef struct esp_iac esp_iac;
+
+/* Kernels of esp_iac_predict (esp_iac_set_path):
+ * ESP_IAC_PATH_TENSOR (default): the two hidden layers as tcgen05 tensor-core MMAs (kind::tf32,
+ *     fp32 accumulators in tensor memory) on a three-term split of every operand, a = a_hi + a_lo
+ *     with a_hi = a truncated to tf32 and a_lo = tf32(a - a_hi): a_hi b_hi + a_hi b_lo + a_lo b_hi,
+ *     which keeps each product within 2^-19 relative of the fp32 product; biases, ReLU and the
+ *     output layer on the CUDA cores.
+ * ESP_IAC_PATH_FMA: everything as fp32 fused multiply-adds on the CUDA cores. */
+#define ESP_IAC_PATH_TENSOR 0
+#define ESP_IAC_PATH_FMA 1
 
 /* Creates a predictor on `device` (-1: the current device) whose work runs on `cuda_stream`
  * (NULL: the legacy default stream). Errors: ESP_ERR_INVALID_ARG, ESP_ERR_UNSUPPORTED (no GPU, or
@@ -80,6 +91,15 @@ esp_status esp_iac_predict(esp_iac *m, int32_t n_rows, const float *job_features
  * host (ESP_ERR_INVALID_ARG for one outside [0, n_rows)). */
 esp_status esp_iac_predict_host(esp_iac *m, int32_t n_rows, const float *job_features, int64_t n_pairs,
                                 const int32_t *pairs, float c_mem, float *s_hat);
+
+/* Selects the kernel of later predictions (ESP_IAC_PATH_TENSOR or ESP_IAC_PATH_FMA). Errors:
+ * ESP_ERR_INVALID_ARG for another value. */
+esp_status esp_iac_set_path(esp_iac *m, int32_t path);
+
+/* Waits for the handle's stream and reports a device-side failure of the queued predictions:
+ * ESP_ERR_TIMEOUT when a bounded wait of the tensor path gave up (the handle then refuses further
+ * work with ESP_ERR_STATE), ESP_ERR_CUDA on a CUDA error. esp_iac_predict_host does this itself. */
+esp_status esp_iac_synchronize(esp_iac *m);
 
 /* Number of kernel launches of the last esp_iac_predict / esp_iac_predict_host. */
 esp_status esp_iac_last_launch_count(esp_iac *m, int64_t *out);

@@ -1,7 +1,8 @@
 // IAC slowdown predictor (include/esp_iac.h): the pair features of Sec. 3.4.1 and the three-layer
 // network of Sec. 3.4.2 / Eq. dnn_pred, batched over co-location pairs.
 //
-// One thread per pair. The folded parameters (at most 64 hidden units: 6,593 fp32, 26 KB) travel
+// Two kernels compute it. k_iac_tc (the default) runs the hidden layers on the tensor cores
+// (esp_iac_tc.cuh). k_iac is the CUDA-core kernel: one thread per pair. The folded parameters (at most 64 hidden units: 6,593 fp32, 26 KB) travel
 // as the kernel's own __grid_constant__ argument, which lives in the constant bank: with every loop
 // unrolled each weight is a compile-time constant-bank operand of its fused multiply-add, so the
 // two hidden layers are a straight run of FFMAs with no loads (no shared-memory staging, no global
@@ -17,6 +18,7 @@
 #include <cuda_runtime.h>
 
 #include "esp_iac.h"
+#include "esp_iac_tc.cuh"
 
 namespace {
 
@@ -116,6 +118,341 @@ void fill_params(IacParams<H> &dst, int hp, const std::vector<float> &w1, const 
     dst.b3 = b3;
 }
 
+
+// ---- tensor-core path (esp_iac_tc.cuh)
+
+struct IacEpilogue {
+    float b1[iac_tc::kN];   // folded layer-1 bias (zero beyond H)
+    float b2[iac_tc::kN];
+    float w3[iac_tc::kN];
+    float b3;
+};
+
+constexpr uint32_t kIacWaitSuspendNs = 1000000;
+constexpr uint32_t kIacWaitPolls = 4096;     // about 4 s of waiting before a timeout is reported
+constexpr unsigned int kIacErrTimeout = 1u;
+
+__device__ __forceinline__ uint32_t smem_addr(const void *p)
+{
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+// Shared-memory matrix descriptor: start address, leading and stride byte offsets (16-byte units),
+// descriptor version 1 (bits 46-47), no swizzle (bits 61-63 = 0).
+__device__ __forceinline__ uint64_t smem_desc(uint32_t addr, uint32_t lbo, uint32_t sbo)
+{
+    return (uint64_t)((addr >> 4) & 0x3fffu) | ((uint64_t)((lbo >> 4) & 0x3fffu) << 16) |
+           ((uint64_t)((sbo >> 4) & 0x3fffu) << 32) | (1ull << 46);
+}
+
+__device__ __forceinline__ void mma_tf32(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t accumulate)
+{
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::tf32 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(a), "l"(b), "r"(iac_tc::kIdesc), "r"(accumulate)
+        : "memory");
+}
+
+__device__ __forceinline__ void mma_commit(uint32_t bar)
+{
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+                 : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before()
+{
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+
+__device__ __forceinline__ void tc_fence_after()
+{
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+
+__device__ __forceinline__ void fence_async_smem()
+{
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+// Barrier of one warpgroup (named barrier id, 128 threads) that also ANDs a predicate over it.
+__device__ __forceinline__ bool wg_sync_and(int id, bool v)
+{
+    uint32_t r;
+    asm volatile(
+        "{\n\t.reg .pred p, q;\n\t"
+        "setp.ne.b32 p, %1, 0;\n\t"
+        "bar.red.and.pred q, %2, 128, p;\n\t"
+        "selp.u32 %0, 1, 0, q;\n\t}"
+        : "=r"(r)
+        : "r"((uint32_t)v), "r"(id)
+        : "memory");
+    return r != 0;
+}
+
+__device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity)
+{
+    for (uint32_t it = 0; it < kIacWaitPolls; ++it) {
+        uint32_t done;
+        asm volatile(
+            "{\n\t.reg .pred p;\n\t"
+            "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+            "selp.u32 %0, 1, 0, p;\n\t}"
+            : "=r"(done)
+            : "r"(bar), "r"(parity), "r"(kIacWaitSuspendNs)
+            : "memory");
+        if (done)
+            return true;
+    }
+    return false;
+}
+
+// 32 consecutive fp32 columns of this thread's TMEM lane.
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float *v)
+{
+    uint32_t r[32];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, "
+        "%15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+          "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+          "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+        : "r"(taddr)
+        : "memory");
+#pragma unroll
+    for (int i = 0; i < 32; ++i)
+        v[i] = __uint_as_float(r[i]);
+}
+
+__device__ __forceinline__ void tmem_wait_ld()
+{
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+// Four consecutive values of a row, split into tf32 high and low parts, stored as one 16-byte chunk
+// of each part.
+__device__ __forceinline__ void store_split4(unsigned char *hi, unsigned char *lo, int off, float a, float b, float c,
+                                             float d)
+{
+    using namespace iac_tc;
+    const uint32_t ha = tf32_trunc_bits(__float_as_uint(a)), hb = tf32_trunc_bits(__float_as_uint(b));
+    const uint32_t hc = tf32_trunc_bits(__float_as_uint(c)), hd = tf32_trunc_bits(__float_as_uint(d));
+    const uint32_t la = tf32_round_bits(__float_as_uint(__fsub_rn(a, __uint_as_float(ha))));
+    const uint32_t lb = tf32_round_bits(__float_as_uint(__fsub_rn(b, __uint_as_float(hb))));
+    const uint32_t lc = tf32_round_bits(__float_as_uint(__fsub_rn(c, __uint_as_float(hc))));
+    const uint32_t ld = tf32_round_bits(__float_as_uint(__fsub_rn(d, __uint_as_float(hd))));
+    *reinterpret_cast<uint4 *>(hi + off) = make_uint4(ha, hb, hc, hd);
+    *reinterpret_cast<uint4 *>(lo + off) = make_uint4(la, lb, lc, ld);
+}
+
+__global__ void __launch_bounds__(iac_tc::kThreads, 1) k_iac_tc(const __grid_constant__ IacEpilogue ep,
+                                                                 const uint4 *bimg, const float *jf, int32_t n_rows,
+                                                                 const int2 *pairs, int64_t n_pairs, float c_mem,
+                                                                 float *out, unsigned int *err)
+{
+    using namespace iac_tc;
+    extern __shared__ unsigned char smem_raw[];
+    unsigned char *sm = reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                                          ~static_cast<uintptr_t>(1023));
+    const int tid = threadIdx.x, wg = tid >> 7, row = tid & 127, warp = tid >> 5;
+    uint64_t *bars = reinterpret_cast<uint64_t *>(sm + kOffBar);
+    uint32_t *slot = reinterpret_cast<uint32_t *>(sm + kOffSlot);
+
+    // the split weights, once per CTA
+    for (int i = tid; i < kBImgBytes / 16; i += kThreads)
+        reinterpret_cast<uint4 *>(sm)[i] = __ldg(bimg + i);
+    if (tid == 0) {
+        for (int g = 0; g < kWG; ++g)
+            asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_addr(bars + g)) : "memory");
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    if (warp == 0) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_addr(slot)),
+                     "r"(kTmemCols)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    fence_async_smem();
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *slot;
+    const uint32_t d1 = tmem + (uint32_t)(wg * 128), d2 = d1 + kN;
+    const uint32_t lane_sel = (uint32_t)(32 * (warp & 3)) << 16;   // this warp's quarter of the lanes
+    unsigned char *a_hi = sm + kOffA + wg * 2 * kABytes, *a_lo = a_hi + kABytes;
+    const uint32_t a_hi_s = smem_addr(a_hi), a_lo_s = smem_addr(a_lo), sm_s = smem_addr(sm);
+    const uint32_t bar = smem_addr(bars + wg);
+    const int bar_id = 1 + wg;
+    uint32_t phase = 0;
+    bool ok = true;
+
+    for (int64_t tile = (int64_t)blockIdx.x * kWG + wg; tile * kM < n_pairs; tile += (int64_t)gridDim.x * kWG) {
+        const int64_t p = tile * kM + row;
+        // ---- the pair's 36 inputs (Sec. 3.4.1), zero for a pair past the end or out of range
+        float x[kK1];
+#pragma unroll
+        for (int i = 0; i < kK1; ++i)
+            x[i] = 0.0f;
+        bool valid = false;
+        if (p < n_pairs) {
+            const int2 ij = __ldg(pairs + p);
+            valid = (uint32_t)ij.x < (uint32_t)n_rows && (uint32_t)ij.y < (uint32_t)n_rows;
+            if (valid) {
+                const float2 *ra = reinterpret_cast<const float2 *>(jf + (size_t)ij.x * kFeat);
+                const float2 *rb = reinterpret_cast<const float2 *>(jf + (size_t)ij.y * kFeat);
+#pragma unroll
+                for (int q = 0; q < kFeat / 2; ++q) {
+                    const float2 va = __ldg(ra + q), vb = __ldg(rb + q);
+                    x[2 * q] = va.x;
+                    x[2 * q + 1] = va.y;
+                    x[kFeat + 2 * q] = vb.x;
+                    x[kFeat + 2 * q + 1] = vb.y;
+                }
+                const float *a = x, *b = x + kFeat;
+                x[28] = __fmul_rn(__fadd_rn(a[0], b[0]), 0.5f);
+                x[29] = __fmul_rn(__fadd_rn(a[1], b[1]), 0.5f);
+                x[30] = __fmul_rn(__fadd_rn(a[2], b[2]), 0.5f);
+                x[31] = __fmul_rn(__fadd_rn(a[4], b[4]), 0.5f);
+                x[32] = __fadd_rn(a[5], b[5]);
+                x[33] = __fdiv_rn(__fadd_rn(a[3], b[3]), c_mem);
+                const float lo = fminf(a[0], b[0]), hi = fmaxf(a[0], b[0]);
+                x[34] = hi == 0.0f ? 1.0f : __fdiv_rn(lo, hi);
+                x[35] = fabsf(__fsub_rn(intensity(a[0], a[2]), intensity(b[0], b[2])));
+            }
+        }
+#pragma unroll
+        for (int c = 0; c < kK1 / 4; ++c)
+            store_split4(a_hi, a_lo, cm_off(row, 4 * c, kK1), x[4 * c], x[4 * c + 1], x[4 * c + 2], x[4 * c + 3]);
+        fence_async_smem();
+        tc_fence_before();
+        asm volatile("bar.sync %0, 128;" ::"r"(bar_id) : "memory");
+        tc_fence_after();
+
+        // ---- layer 1: D1 = X W1'^T, three split products per k-step
+        if (row == 0) {
+#pragma unroll
+            for (int ks = 0; ks < kK1 / 8; ++ks) {
+                const uint64_t ah = smem_desc(a_hi_s + ks * 256, 128, kK1 / 4 * 128);
+                const uint64_t al = smem_desc(a_lo_s + ks * 256, 128, kK1 / 4 * 128);
+                const uint64_t bh = smem_desc(sm_s + kOffB1Hi + ks * 256, 128, kK1 / 4 * 128);
+                const uint64_t bl = smem_desc(sm_s + kOffB1Lo + ks * 256, 128, kK1 / 4 * 128);
+                mma_tf32(d1, ah, bh, ks > 0 ? 1u : 0u);
+                mma_tf32(d1, ah, bl, 1u);
+                mma_tf32(d1, al, bh, 1u);
+            }
+            mma_commit(bar);
+        }
+        __syncwarp();
+        ok = wg_sync_and(bar_id, mbar_wait_bounded(bar, phase));
+        phase ^= 1u;
+        if (!ok)
+            break;
+        tc_fence_after();
+
+        // ---- epilogue 1: h1 = ReLU(D1 + b1'), split into operand A of layer 2
+        {
+            float v[32];
+#pragma unroll
+            for (int half = 0; half < 2; ++half) {
+                tmem_ld32((d1 + 32 * half) | lane_sel, v);
+                tmem_wait_ld();
+#pragma unroll
+                for (int c = 0; c < 8; ++c) {
+                    const int o = 32 * half + 4 * c;
+                    store_split4(a_hi, a_lo, cm_off(row, o, kK2), fmaxf(__fadd_rn(v[4 * c], ep.b1[o]), 0.0f),
+                                 fmaxf(__fadd_rn(v[4 * c + 1], ep.b1[o + 1]), 0.0f),
+                                 fmaxf(__fadd_rn(v[4 * c + 2], ep.b1[o + 2]), 0.0f),
+                                 fmaxf(__fadd_rn(v[4 * c + 3], ep.b1[o + 3]), 0.0f));
+                }
+            }
+        }
+        fence_async_smem();
+        tc_fence_before();
+        asm volatile("bar.sync %0, 128;" ::"r"(bar_id) : "memory");
+        tc_fence_after();
+
+        // ---- layer 2: D2 = H1 W2'^T
+        if (row == 0) {
+#pragma unroll
+            for (int ks = 0; ks < kK2 / 8; ++ks) {
+                const uint64_t ah = smem_desc(a_hi_s + ks * 256, 128, kK2 / 4 * 128);
+                const uint64_t al = smem_desc(a_lo_s + ks * 256, 128, kK2 / 4 * 128);
+                const uint64_t bh = smem_desc(sm_s + kOffB2Hi + ks * 256, 128, kK2 / 4 * 128);
+                const uint64_t bl = smem_desc(sm_s + kOffB2Lo + ks * 256, 128, kK2 / 4 * 128);
+                mma_tf32(d2, ah, bh, ks > 0 ? 1u : 0u);
+                mma_tf32(d2, ah, bl, 1u);
+                mma_tf32(d2, al, bh, 1u);
+            }
+            mma_commit(bar);
+        }
+        __syncwarp();
+        ok = wg_sync_and(bar_id, mbar_wait_bounded(bar, phase));
+        phase ^= 1u;
+        if (!ok)
+            break;
+        tc_fence_after();
+
+        // ---- epilogue 2: S_hat = 1 + ReLU(b3 + sum_o w3_o ReLU(D2_o + b2'_o)), o in order
+        float y = ep.b3;
+        {
+            float v[32];
+#pragma unroll
+            for (int half = 0; half < 2; ++half) {
+                tmem_ld32((d2 + 32 * half) | lane_sel, v);
+                tmem_wait_ld();
+#pragma unroll
+                for (int i = 0; i < 32; ++i) {
+                    const int o = 32 * half + i;
+                    y = __fmaf_rn(ep.w3[o], fmaxf(__fadd_rn(v[i], ep.b2[o]), 0.0f), y);
+                }
+            }
+        }
+        if (p < n_pairs)
+            out[p] = valid ? __fadd_rn(1.0f, fmaxf(y, 0.0f)) : __int_as_float(0x7fffffff);
+        // the next tile rewrites operand A (its MMAs have completed) and D1/D2 (read above: the
+        // tcgen05.fence before the next warpgroup barrier orders those reads before the next MMAs)
+    }
+    if (!ok) {
+        // an MMA group did not complete in time: give it one more bounded wait before the tensor
+        // memory is released, and report the timeout
+        mbar_wait_bounded(bar, phase ^ 1u);
+        if (row == 0)
+            atomicOr(err, kIacErrTimeout);
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 0)
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols) : "memory");
+}
+
+// Split images of W1' (64 x 40) and W2' (64 x 64) in the canonical layout, hi then lo of each.
+void build_bimg(int H, const std::vector<float> &w1, const std::vector<float> &w2, std::vector<uint32_t> &img)
+{
+    using namespace iac_tc;
+    img.assign(kBImgBytes / 4, 0u);
+    auto put = [&](int base, int K, int o, int k, float v) {
+        uint32_t bits;
+        std::memcpy(&bits, &v, 4);
+        const uint32_t hi = tf32_trunc_bits(bits);
+        float hf;
+        std::memcpy(&hf, &hi, 4);
+        const float lo = v - hf;   // exact: the bits below the tf32 mantissa
+        uint32_t lb;
+        std::memcpy(&lb, &lo, 4);
+        const int B = (base == 0) ? kB1Bytes : kB2Bytes;
+        img[(base + cm_off(o, k, K)) / 4] = hi;
+        img[(base + B + cm_off(o, k, K)) / 4] = tf32_round_bits(lb);
+    };
+    for (int o = 0; o < H; ++o) {
+        for (int k = 0; k < kIn; ++k)
+            put(kOffB1Hi, kK1, o, k, w1[(size_t)o * kIn + k]);
+        for (int i = 0; i < H; ++i)
+            put(kOffB2Hi, kK2, o, i, w2[(size_t)o * H + i]);
+    }
+}
 }  // namespace
 
 struct esp_iac {
@@ -131,6 +468,11 @@ struct esp_iac {
     IacParams<64> p64;
     int grid_cap = 0;
     int64_t launches = 0;
+    int path = ESP_IAC_PATH_TENSOR;
+    IacEpilogue ep;                       // tensor path: biases and output weights
+    std::vector<uint32_t> h_bimg;         // tensor path: split W1', W2' (host copy of the upload)
+    uint4 *d_bimg = nullptr;
+    unsigned int *d_err = nullptr;        // device error word (timeouts of the tensor path)
     // buffers of esp_iac_predict_host
     float *d_rows = nullptr, *d_out = nullptr;
     int2 *d_pairs = nullptr;
@@ -163,6 +505,16 @@ esp_status check_handle(esp_iac *m)
     return ESP_OK;
 }
 
+cudaError_t launch_iac_tc(esp_iac *m, int32_t n_rows, const float *rows, int64_t n_pairs, const int2 *pairs,
+                         float c_mem, float *out)
+{
+    const int64_t tiles = (n_pairs + iac_tc::kM - 1) / iac_tc::kM;
+    const int grid = (int)std::min<int64_t>((tiles + iac_tc::kWG - 1) / iac_tc::kWG, m->sm_count);
+    k_iac_tc<<<grid, iac_tc::kThreads, iac_tc::kSmemBytes, m->stream>>>(m->ep, m->d_bimg, rows, n_rows, pairs,
+                                                                       n_pairs, c_mem, out, m->d_err);
+    return cudaGetLastError();
+}
+
 template <int H>
 cudaError_t launch_iac(esp_iac *m, const IacParams<H> &w, int32_t n_rows, const float *rows, int64_t n_pairs,
                        const int2 *pairs, float c_mem, float *out)
@@ -181,7 +533,9 @@ esp_status enqueue(esp_iac *m, int32_t n_rows, const float *rows, int64_t n_pair
         return ESP_OK;
     IAC_CUDA(cudaSetDevice(m->device));
     cudaError_t e;
-    if (m->Hk == 16)
+    if (m->path == ESP_IAC_PATH_TENSOR)
+        e = launch_iac_tc(m, n_rows, rows, n_pairs, pairs, c_mem, out);
+    else if (m->Hk == 16)
         e = launch_iac<16>(m, m->p16, n_rows, rows, n_pairs, pairs, c_mem, out);
     else if (m->Hk == 32)
         e = launch_iac<32>(m, m->p32, n_rows, rows, n_pairs, pairs, c_mem, out);
@@ -281,7 +635,49 @@ esp_status esp_iac_create(esp_iac **out, int device, void *cuda_stream)
         delete m;
         return ESP_ERR_CUDA;
     }
+    void *e = nullptr, *b = nullptr;
+    if (cudaMalloc(&e, sizeof(unsigned int)) != cudaSuccess || cudaMalloc(&b, iac_tc::kBImgBytes) != cudaSuccess ||
+        cudaMemset(e, 0, sizeof(unsigned int)) != cudaSuccess ||
+        cudaFuncSetAttribute(k_iac_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, iac_tc::kSmemBytes) !=
+            cudaSuccess) {
+        cudaGetLastError();
+        if (e)
+            cudaFree(e);
+        if (b)
+            cudaFree(b);
+        delete m;
+        return ESP_ERR_CUDA;
+    }
+    m->d_err = static_cast<unsigned int *>(e);
+    m->d_bimg = static_cast<uint4 *>(b);
     *out = m;
+    return ESP_OK;
+}
+
+esp_status esp_iac_set_path(esp_iac *m, int32_t path)
+{
+    const esp_status st = check_handle(m);
+    if (st != ESP_OK)
+        return st;
+    if (path != ESP_IAC_PATH_TENSOR && path != ESP_IAC_PATH_FMA)
+        return ESP_ERR_INVALID_ARG;
+    m->path = path;
+    return ESP_OK;
+}
+
+esp_status esp_iac_synchronize(esp_iac *m)
+{
+    const esp_status st = check_handle(m);
+    if (st != ESP_OK)
+        return st;
+    IAC_CUDA(cudaSetDevice(m->device));
+    IAC_CUDA(cudaStreamSynchronize(m->stream));
+    unsigned int err = 0;
+    IAC_CUDA(cudaMemcpy(&err, m->d_err, sizeof(err), cudaMemcpyDeviceToHost));
+    if (err) {
+        m->poisoned = true;
+        return ESP_ERR_TIMEOUT;
+    }
     return ESP_OK;
 }
 
@@ -312,6 +708,18 @@ esp_status esp_iac_load_model(esp_iac *m, int32_t H, const float *W1, const floa
         return ESP_ERR_INVALID_ARG;
     std::vector<float> w3(W3, W3 + H);
     m->loaded = false;
+    // tensor path: biases and output weights for the epilogue, split weight images for the MMAs
+    std::memset(&m->ep, 0, sizeof(m->ep));
+    for (int o = 0; o < H; ++o) {
+        m->ep.b1[o] = b1f[o];
+        m->ep.b2[o] = b2f[o];
+        m->ep.w3[o] = w3[o];
+    }
+    m->ep.b3 = b3;
+    build_bimg(H, w1f, w2f, m->h_bimg);
+    IAC_CUDA(cudaSetDevice(m->device));
+    IAC_CUDA(cudaMemcpyAsync(m->d_bimg, m->h_bimg.data(), iac_tc::kBImgBytes, cudaMemcpyHostToDevice, m->stream));
+    IAC_CUDA(cudaStreamSynchronize(m->stream));
     m->H = H;
     m->Hk = H <= 16 ? 16 : (H <= 32 ? 32 : 64);
     if (m->Hk == 16)
@@ -385,8 +793,7 @@ esp_status esp_iac_predict_host(esp_iac *m, int32_t n_rows, const float *job_fea
     if ((st = enqueue(m, n_rows, m->d_rows, n_pairs, m->d_pairs, c_mem, m->d_out)) != ESP_OK)
         return st;
     IAC_CUDA(cudaMemcpyAsync(s_hat, m->d_out, (size_t)n_pairs * sizeof(float), cudaMemcpyDeviceToHost, m->stream));
-    IAC_CUDA(cudaStreamSynchronize(m->stream));
-    return ESP_OK;
+    return esp_iac_synchronize(m);
 }
 
 esp_status esp_iac_last_launch_count(esp_iac *m, int64_t *out)
@@ -408,6 +815,10 @@ void esp_iac_destroy(esp_iac *m)
         cudaFree(m->d_pairs);
     if (m->d_out)
         cudaFree(m->d_out);
+    if (m->d_bimg)
+        cudaFree(m->d_bimg);
+    if (m->d_err)
+        cudaFree(m->d_err);
     cudaGetLastError();
     delete m;
 }

@@ -31,7 +31,7 @@ EXPORTED = [
     "esp_debug_sort_layout", "esp_debug_plan_runs", "esp_debug_set_sorted_layout", "esp_evaluate_noalloc",
     "esp_set_penalties", "esp_adaptive_threshold", "esp_effective_capacity", "esp_load_placement",
     "esp_iac_create", "esp_iac_set_stream", "esp_iac_load_model", "esp_iac_predict", "esp_iac_predict_host",
-    "esp_iac_last_launch_count", "esp_iac_destroy",
+    "esp_iac_last_launch_count", "esp_iac_destroy", "esp_iac_set_path", "esp_iac_synchronize",
 ]
 
 
@@ -107,6 +107,8 @@ def load_library(path: Optional[str] = None):
         "esp_iac_predict_host": ([vp, i32, vp, i64, vp, ctypes.c_float, vp], st),
         "esp_iac_last_launch_count": ([vp, ctypes.POINTER(i64)], st),
         "esp_iac_destroy": ([vp], None),
+        "esp_iac_set_path": ([vp, i32], st),
+        "esp_iac_synchronize": ([vp], st),
     }
     for name, (args, res) in sig.items():
         fn = getattr(lib, name)
@@ -469,6 +471,17 @@ def esp_iac_predict_host(h: int, rows: np.ndarray, pairs: np.ndarray, c_mem: flo
     return out
 
 
+ESP_IAC_PATH_TENSOR, ESP_IAC_PATH_FMA = 0, 1
+
+
+def esp_iac_set_path(h: int, path: int) -> None:
+    _check(load_library().esp_iac_set_path(h, path), "esp_iac_set_path")
+
+
+def esp_iac_synchronize(h: int) -> None:
+    _check(load_library().esp_iac_synchronize(h), "esp_iac_synchronize")
+
+
 def esp_iac_last_launch_count(h: int) -> int:
     n = ctypes.c_int64()
     _check(load_library().esp_iac_last_launch_count(h, ctypes.byref(n)), "esp_iac_last_launch_count")
@@ -482,8 +495,9 @@ def esp_iac_destroy(h: int) -> None:
 class Predictor:
     """One esp_iac handle: load a model, then predict slowdowns of co-location pairs."""
 
-    def __init__(self, model=None, device: int = -1, stream: Optional[int] = None):
+    def __init__(self, model=None, device: int = -1, stream: Optional[int] = None, path: int = 0):
         self.h = esp_iac_create(device, stream)
+        esp_iac_set_path(self.h, path)
         if model is not None:
             esp_iac_load_model(self.h, model)
 
