@@ -247,6 +247,34 @@ __device__ __forceinline__ void store_split4(unsigned char *hi, unsigned char *l
     *reinterpret_cast<uint4 *>(lo + off) = make_uint4(la, lb, lc, ld);
 }
 
+// A pair's two feature rows (zero when the pair is past the end or out of range).
+struct PairRows {
+    float2 a[kFeat / 2], b[kFeat / 2];
+    bool valid;
+};
+
+__device__ __forceinline__ void fetch_pair(PairRows &r, int64_t p, int64_t n_pairs, const int2 *pairs,
+                                           const float *jf, int32_t n_rows)
+{
+#pragma unroll
+    for (int q = 0; q < kFeat / 2; ++q)
+        r.a[q] = r.b[q] = make_float2(0.0f, 0.0f);
+    r.valid = false;
+    if (p < n_pairs) {
+        const int2 ij = __ldg(pairs + p);
+        r.valid = (uint32_t)ij.x < (uint32_t)n_rows && (uint32_t)ij.y < (uint32_t)n_rows;
+        if (r.valid) {
+            const float2 *ra = reinterpret_cast<const float2 *>(jf + (size_t)ij.x * kFeat);
+            const float2 *rb = reinterpret_cast<const float2 *>(jf + (size_t)ij.y * kFeat);
+#pragma unroll
+            for (int q = 0; q < kFeat / 2; ++q) {
+                r.a[q] = __ldg(ra + q);
+                r.b[q] = __ldg(rb + q);
+            }
+        }
+    }
+}
+
 __global__ void __launch_bounds__(iac_tc::kThreads, 1) k_iac_tc(const __grid_constant__ IacEpilogue ep,
                                                                  const uint4 *bimg, const float *jf, int32_t n_rows,
                                                                  const int2 *pairs, int64_t n_pairs, float c_mem,
@@ -288,39 +316,35 @@ __global__ void __launch_bounds__(iac_tc::kThreads, 1) k_iac_tc(const __grid_con
     uint32_t phase = 0;
     bool ok = true;
 
-    for (int64_t tile = (int64_t)blockIdx.x * kWG + wg; tile * kM < n_pairs; tile += (int64_t)gridDim.x * kWG) {
+    const int64_t tile_stride = (int64_t)gridDim.x * kWG;
+    PairRows cur;
+    fetch_pair(cur, ((int64_t)blockIdx.x * kWG + wg) * kM + row, n_pairs, pairs, jf, n_rows);
+    for (int64_t tile = (int64_t)blockIdx.x * kWG + wg; tile * kM < n_pairs; tile += tile_stride) {
         const int64_t p = tile * kM + row;
         // ---- the pair's 36 inputs (Sec. 3.4.1), zero for a pair past the end or out of range
         float x[kK1];
 #pragma unroll
-        for (int i = 0; i < kK1; ++i)
-            x[i] = 0.0f;
-        bool valid = false;
-        if (p < n_pairs) {
-            const int2 ij = __ldg(pairs + p);
-            valid = (uint32_t)ij.x < (uint32_t)n_rows && (uint32_t)ij.y < (uint32_t)n_rows;
-            if (valid) {
-                const float2 *ra = reinterpret_cast<const float2 *>(jf + (size_t)ij.x * kFeat);
-                const float2 *rb = reinterpret_cast<const float2 *>(jf + (size_t)ij.y * kFeat);
+        for (int q = 0; q < kFeat / 2; ++q) {
+            x[2 * q] = cur.a[q].x;
+            x[2 * q + 1] = cur.a[q].y;
+            x[kFeat + 2 * q] = cur.b[q].x;
+            x[kFeat + 2 * q + 1] = cur.b[q].y;
+        }
 #pragma unroll
-                for (int q = 0; q < kFeat / 2; ++q) {
-                    const float2 va = __ldg(ra + q), vb = __ldg(rb + q);
-                    x[2 * q] = va.x;
-                    x[2 * q + 1] = va.y;
-                    x[kFeat + 2 * q] = vb.x;
-                    x[kFeat + 2 * q + 1] = vb.y;
-                }
-                const float *a = x, *b = x + kFeat;
-                x[28] = __fmul_rn(__fadd_rn(a[0], b[0]), 0.5f);
-                x[29] = __fmul_rn(__fadd_rn(a[1], b[1]), 0.5f);
-                x[30] = __fmul_rn(__fadd_rn(a[2], b[2]), 0.5f);
-                x[31] = __fmul_rn(__fadd_rn(a[4], b[4]), 0.5f);
-                x[32] = __fadd_rn(a[5], b[5]);
-                x[33] = __fdiv_rn(__fadd_rn(a[3], b[3]), c_mem);
-                const float lo = fminf(a[0], b[0]), hi = fmaxf(a[0], b[0]);
-                x[34] = hi == 0.0f ? 1.0f : __fdiv_rn(lo, hi);
-                x[35] = fabsf(__fsub_rn(intensity(a[0], a[2]), intensity(b[0], b[2])));
-            }
+        for (int i = 2 * kFeat; i < kK1; ++i)
+            x[i] = 0.0f;
+        const bool valid = cur.valid;
+        if (valid) {
+            const float *a = x, *b = x + kFeat;
+            x[28] = __fmul_rn(__fadd_rn(a[0], b[0]), 0.5f);
+            x[29] = __fmul_rn(__fadd_rn(a[1], b[1]), 0.5f);
+            x[30] = __fmul_rn(__fadd_rn(a[2], b[2]), 0.5f);
+            x[31] = __fmul_rn(__fadd_rn(a[4], b[4]), 0.5f);
+            x[32] = __fadd_rn(a[5], b[5]);
+            x[33] = __fdiv_rn(__fadd_rn(a[3], b[3]), c_mem);
+            const float lo = fminf(a[0], b[0]), hi = fmaxf(a[0], b[0]);
+            x[34] = hi == 0.0f ? 1.0f : __fdiv_rn(lo, hi);
+            x[35] = fabsf(__fsub_rn(intensity(a[0], a[2]), intensity(b[0], b[2])));
         }
 #pragma unroll
         for (int c = 0; c < kK1 / 4; ++c)
@@ -345,6 +369,9 @@ __global__ void __launch_bounds__(iac_tc::kThreads, 1) k_iac_tc(const __grid_con
             mma_commit(bar);
         }
         __syncwarp();
+        // the next tile's pair and rows: their latency overlaps this tile's MMAs and epilogues
+        PairRows nxt;
+        fetch_pair(nxt, p + tile_stride * kM, n_pairs, pairs, jf, n_rows);
         ok = wg_sync_and(bar_id, mbar_wait_bounded(bar, phase));
         phase ^= 1u;
         if (!ok)
@@ -413,6 +440,7 @@ __global__ void __launch_bounds__(iac_tc::kThreads, 1) k_iac_tc(const __grid_con
             out[p] = valid ? __fadd_rn(1.0f, fmaxf(y, 0.0f)) : __int_as_float(0x7fffffff);
         // the next tile rewrites operand A (its MMAs have completed) and D1/D2 (read above: the
         // tcgen05.fence before the next warpgroup barrier orders those reads before the next MMAs)
+        cur = nxt;
     }
     if (!ok) {
         // an MMA group did not complete in time: give it one more bounded wait before the tensor
