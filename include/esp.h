@@ -69,7 +69,11 @@ typedef enum { ESP_STEP_FIXED = 0, ESP_STEP_INV_SQRT = 1 } esp_step_rule;
                                           column and each scenario fits in a cluster (up to 16 CTAs of up to about
                                           227 KB); otherwise the streaming path runs. Same results either way.
                                           esp_last_launch_count tells which ran (3: resident); with
-                                          ESP_FLAG_PASS_EVENTS the one resident launch counts as one pass */
+                                          ESP_FLAG_PASS_EVENTS the one resident launch counts as one pass.
+                                          For a table loaded with esp_load_placement it selects the
+                                          grid-resident solve instead: all rounds in one cooperative launch
+                                          with a grid-wide barrier per round (4 launches; S*P <= 4096, no
+                                          fingerprint or dual trace; otherwise per-round launches) */
 
 typedef struct {
     double eta0;            /* > 0, finite */
@@ -197,7 +201,8 @@ esp_status esp_evaluate_noalloc(int32_t S, int32_t J, int32_t R, const int64_t *
  *   node_type   host, N int32 in [0, NT)          D          host, NT*NT fp32, finite
  *   capacity    host, S*P int64 > 0
  * 1 <= KC <= 32, 1 <= N <= 64, 1 <= NT <= 64, 1 <= R <= 16, 0 <= r_global < R. esp_set_penalties
- * and ESP_FLAG_RESIDENT do not apply (ESP_ERR_UNSUPPORTED / the streaming path). Errors:
+ * does not apply (ESP_ERR_UNSUPPORTED); ESP_FLAG_RESIDENT selects the grid-resident solve (see the
+ * flag). Errors:
  * ESP_ERR_INVALID_ARG, ESP_ERR_UNSUPPORTED (shape beyond the limits of the device), ESP_ERR_OOM,
  * ESP_ERR_CUDA. */
 esp_status esp_load_placement(esp_ctx *ctx, int32_t S, int32_t J, int32_t KC, int32_t N, int32_t R, int32_t r_global,

@@ -69,6 +69,8 @@ struct esp_ctx {
     bool placement = false;
     DevPlace place = {};
     int32_t place_grid = 0;
+    PlaceRes place_res = {};         // grid-resident placement solve (ESP_FLAG_RESIDENT), when allocated
+    bool place_res_ok = false;
     uint16_t *group = nullptr;
     int64_t *cap = nullptr;
     double *vmax = nullptr;
@@ -184,6 +186,8 @@ void release_table(esp_ctx *ctx)
     ctx->placement = false;
     ctx->place = DevPlace{};
     ctx->place_grid = 0;
+    ctx->place_res = PlaceRes{};
+    ctx->place_res_ok = false;
     ctx->res_auto = -1;
     ctx->res_force = -1;
     ctx->loaded = false;
@@ -641,7 +645,13 @@ esp_status enqueue_solve(esp_ctx *ctx, const esp_params *p, const DevState &st, 
     const bool use_graph = ctx->stream != nullptr;   // the legacy default stream cannot be captured
     std::vector<cudaEvent_t> &pool = use_graph ? ctx->graph_pool : ctx->ev_pool;
     size_t pool_used = use_graph ? 0 : ctx->ev_used;
-    const int ri = (p->flags & ESP_FLAG_RESIDENT) ? (ctx->res_force >= 0 ? ctx->res_force : ctx->res_auto) : -1;
+    const int ri = (p->flags & ESP_FLAG_RESIDENT) && !ctx->placement
+                       ? (ctx->res_force >= 0 ? ctx->res_force : ctx->res_auto)
+                       : -1;
+    // a placement table solves all rounds in one cooperative launch when asked, unless the
+    // fingerprint or dual trace is wanted (those need the per-round launches)
+    const bool place_res = ctx->placement && (p->flags & ESP_FLAG_RESIDENT) && ctx->place_res_ok &&
+                           st.hash_trace == nullptr && st.dual_trace == nullptr;
     auto timed_launch = [&](auto &&launch) -> cudaError_t {
         if (!timed)
             return launch();
@@ -672,6 +682,17 @@ esp_status enqueue_solve(esp_ctx *ctx, const esp_params *p, const DevState &st, 
     };
     auto issue = [&]() -> cudaError_t {
         cudaError_t e = launch_init(t, st, a, has_l0 ? ctx->lambda0 : nullptr, ctx->stream);
+        if (place_res) {
+            if (e == cudaSuccess && T > 0)
+                e = timed_launch([&]() {
+                    return launch_place_res(t, st, pp, a, ctx->place_res, ctx->place_grid, ctx->stream);
+                });
+            if (e == cudaSuccess)
+                e = pass(T, PASS_FINAL);
+            if (e == cudaSuccess)
+                e = launch_objectives(t, st, a, ctx->stream);
+            return e;
+        }
         if (ri >= 0) {
             const ResPlan &rp = ctx->res[ri].plan;
             if (e == cudaSuccess)
@@ -692,7 +713,8 @@ esp_status enqueue_solve(esp_ctx *ctx, const esp_params *p, const DevState &st, 
             e = launch_objectives(t, st, a, ctx->stream);
         return e;
     };
-    ctx->last_launches = ri >= 0 ? 3 : 3 + (fused ? 1LL : 2LL) * T - (ctx->grid > 0 ? 0 : (T + 1));
+    ctx->last_launches = place_res ? 3 + (T > 0 ? 1 : 0)
+                         : ri >= 0 ? 3 : 3 + (fused ? 1LL : 2LL) * T - (ctx->grid > 0 ? 0 : (T + 1));
     ctx->last_T = T;
 
     GraphKey key;
@@ -707,7 +729,7 @@ esp_status enqueue_solve(esp_ctx *ctx, const esp_params *p, const DevState &st, 
     key.ht = st.hash_trace;
     key.gt = st.dual_trace;
     key.has_l0 = has_l0;
-    key.res = ri;
+    key.res = place_res ? -2 : ri;
 
     if (!use_graph) {
         ESP_CUDA(issue());
@@ -1175,7 +1197,6 @@ esp_status esp_load_placement(esp_ctx *ctx, int32_t S, int32_t J, int32_t KC, in
     PALLOC(ctx->umax, (size_t)S * R);
     PALLOC(ctx->valflags, 4);
     PALLOC(ctx->stats, 2);
-#undef PALLOC
     auto h2d = [&](void *dst, const void *src, size_t bytes) {
         return cudaMemcpyAsync(dst, src, bytes, cudaMemcpyHostToDevice, ctx->stream);
     };
@@ -1210,6 +1231,25 @@ esp_status esp_load_placement(esp_ctx *ctx, int32_t S, int32_t J, int32_t KC, in
         release_table(ctx);
         return st;
     }
+    // scratch of the grid-resident solve: every CTA keeps a copy of the price state, so it is kept
+    // for small price vectors only (S * P <= kPlaceResMaxPrices)
+    if ((int64_t)S * P <= kPlaceResMaxPrices) {
+        const size_t g = (size_t)ctx->place_grid;
+        PlaceRes &pr = ctx->place_res;
+        PALLOC(pr.U3, 3 * (size_t)S * P);
+        PALLOC(pr.lam, g * S * P);
+        PALLOC(pr.p64, g * S * P);
+        PALLOC(pr.p32, g * S * P);
+        PALLOC(pr.ebound, g * S);
+        PALLOC(pr.frozen, g * S);
+        PALLOC(pr.status, g * S);
+        PALLOC(pr.converged, g * S);
+        PALLOC(pr.rounds_run, g * S);
+        PALLOC(pr.bar, 2);
+        ESP_CUDA(cudaMemsetAsync(pr.U3, 0, 3 * (size_t)S * P * sizeof(unsigned long long), ctx->stream));
+        ctx->place_res_ok = true;
+    }
+#undef PALLOC
     ESP_CUDA(cudaStreamSynchronize(ctx->stream));
     ctx->loaded = true;
     ctx->solved = false;

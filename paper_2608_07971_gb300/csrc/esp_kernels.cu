@@ -268,7 +268,9 @@ __global__ void k_init(DevTable t, DevState st, SolveArgs a, const double *lambd
 // same launch wrote (demand, minimal reduced costs, fingerprint) through L2. A lane's first KEEP
 // new prices are computed once, unrolled (their loads and divides overlap), and kept in registers
 // for the write; the rest are recomputed.
-template <int KEEP>
+// ZERO_U = false leaves the demand in place (a grid-resident solve reads it from every CTA and
+// clears it later).
+template <int KEEP, bool ZERO_U = true>
 __device__ void update_scenario(const DevTable &t, const DevState &st, const SolveArgs &a, int s, int round,
                                 int lane)
 {
@@ -330,8 +332,9 @@ __device__ void update_scenario(const DevTable &t, const DevState &st, const Sol
     dmax = warp_max(dmax);
     amax = warp_max(amax);
     if (bad) {
-        for (int k = lane; k < P; k += 32)
-            st.U[sp + k] = 0ull;
+        if (ZERO_U)
+            for (int k = lane; k < P; k += 32)
+                st.U[sp + k] = 0ull;
         if (lane == 0) {
             st.status[s] = 2;
             st.frozen[s] = 1;
@@ -351,7 +354,8 @@ __device__ void update_scenario(const DevTable &t, const DevState &st, const Sol
             nl = price_step(st.lam[sp + k], U, C, (double)C, eta, a.mode);
         }
         st.lam[sp + k] = nl;
-        st.U[sp + k] = 0ull;
+        if (ZERO_U)
+            st.U[sp + k] = 0ull;
         if (st.lam_trace)
             st.lam_trace[((size_t)s * (T + 1) + round + 1) * P + k] = nl;
     }
@@ -1428,45 +1432,44 @@ __device__ __forceinline__ float place_node_part(const float *uf, float base, co
     return q;
 }
 
-template <int RT, bool PLAIN>
-__global__ void __launch_bounds__(kPlaceWarps * 32, 4) k_place(DevTable t, DevState st, DevPlace pl, SolveArgs a,
-                                                            int round, int kind)
+// Shared-memory areas of one warp of the placement kernels: configuration units, values, fp32
+// global parts, fp32 node-column units, fp32 prices.
+struct PlaceWarpSmem {
+    int32_t *us;
+    double *vs;
+    float *gs;
+    float *ufs;
+    float *p32s;
+};
+
+__device__ __forceinline__ PlaceWarpSmem place_warp_smem(unsigned char *smem, int wid, int R, int P, int KC)
 {
-    extern __shared__ __align__(16) unsigned char smem[];
-    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+    unsigned char *wbase = smem + (size_t)wid * place_warp_bytes(R, P, KC);
+    PlaceWarpSmem w;
+    w.us = reinterpret_cast<int32_t *>(wbase);
+    w.vs = reinterpret_cast<double *>(wbase + round16(KC * R * 4));
+    w.gs = reinterpret_cast<float *>(wbase + round16(KC * R * 4) + round16(KC * 8));
+    w.ufs = reinterpret_cast<float *>(wbase + round16(KC * R * 4) + round16(KC * 8) + round16(KC * 4));
+    w.p32s = reinterpret_cast<float *>(wbase + 2 * round16(KC * R * 4) + round16(KC * 8) + round16(KC * 4));
+    return w;
+}
+
+// Best responses of the jobs [j_begin, j_end) (global job indices) over their configurations x
+// nodes at the prices of c, the winners' demand into c's accumulators, then a flush.
+template <int RT>
+__device__ void place_jobs(WarpCtx<RT, true> &c, const DevPlace &pl, const PlaceWarpSmem &ws, int64_t j_begin,
+                           int64_t j_end, int lane)
+{
+    const DevTable &t = c.t;
+    const DevState &st = c.st;
     const int KC = pl.KC, N = pl.N, NT = pl.NT;
-    const int R = RT ? RT : t.R, rg = t.r_global;
-    unsigned char *wbase = smem + (size_t)wid * place_warp_bytes(R, t.P, KC);
-    int32_t *us = reinterpret_cast<int32_t *>(wbase);
-    double *vs = reinterpret_cast<double *>(wbase + round16(KC * R * 4));
-    float *gs = reinterpret_cast<float *>(wbase + round16(KC * R * 4) + round16(KC * 8));
-    float *ufs = reinterpret_cast<float *>(wbase + round16(KC * R * 4) + round16(KC * 8) + round16(KC * 4));
-    float *p32s = reinterpret_cast<float *>(wbase + 2 * round16(KC * R * 4) + round16(KC * 8) + round16(KC * 4));
-    const int w = blockIdx.x * kPlaceWarps + wid;
-    if (w >= pl.n_warps)
-        return;
-
-    WarpCtx<RT, true> c;
-    c.t = t;
-    c.st = st;
-    c.scen_warps = pl.scen_warps;
-    c.a = a;
-    c.round = round;
-    c.R = R;
-    c.rg = rg;
-    c.kind = PLAIN ? (int)PASS_ROUND : kind;
-    c.want_min = PLAIN ? false : ((kind == PASS_FINAL) || (st.dual_trace != nullptr));
-    c.want_hash = PLAIN ? false : ((kind == PASS_ROUND) && (st.hash_trace != nullptr));
-    c.uniform_k = 0;
-    c.log2_k = 0;
-    c.s = -1;
-#pragma unroll
-    for (int r = 0; r < Cols<RT>::N; ++r)
-        c.acc[r] = 0;
-    c.hacc = 0;
-
-    const int64_t j_end = pl.warp_job[w + 1];
-    for (int64_t j = pl.warp_job[w]; j < j_end; ++j) {
+    const int R = c.R, rg = c.rg;
+    int32_t *us = ws.us;
+    double *vs = ws.vs;
+    float *gs = ws.gs;
+    float *ufs = ws.ufs;
+    float *p32s = ws.p32s;
+    for (int64_t j = j_begin; j < j_end; ++j) {
         const int sc = (int)(j / t.J);
         if (sc != c.s)
             enter_scenario<RT, true>(c, sc, p32s, lane);
@@ -1570,6 +1573,186 @@ __global__ void __launch_bounds__(kPlaceWarps * 32, 4) k_place(DevTable t, DevSt
         }
     }
     flush<RT, true>(c, lane);
+}
+
+template <int RT, bool PLAIN>
+__global__ void __launch_bounds__(kPlaceWarps * 32, 4) k_place(DevTable t, DevState st, DevPlace pl, SolveArgs a,
+                                                            int round, int kind)
+{
+    extern __shared__ __align__(16) unsigned char smem[];
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+    const int R = RT ? RT : t.R, rg = t.r_global;
+    const PlaceWarpSmem ws = place_warp_smem(smem, wid, R, t.P, pl.KC);
+    const int w = blockIdx.x * kPlaceWarps + wid;
+    if (w >= pl.n_warps)
+        return;
+
+    WarpCtx<RT, true> c;
+    c.t = t;
+    c.st = st;
+    c.scen_warps = pl.scen_warps;
+    c.a = a;
+    c.round = round;
+    c.R = R;
+    c.rg = rg;
+    c.kind = PLAIN ? (int)PASS_ROUND : kind;
+    c.want_min = PLAIN ? false : ((kind == PASS_FINAL) || (st.dual_trace != nullptr));
+    c.want_hash = PLAIN ? false : ((kind == PASS_ROUND) && (st.hash_trace != nullptr));
+    c.uniform_k = 0;
+    c.log2_k = 0;
+    c.s = -1;
+#pragma unroll
+    for (int r = 0; r < Cols<RT>::N; ++r)
+        c.acc[r] = 0;
+    c.hacc = 0;
+    place_jobs<RT>(c, pl, ws, pl.warp_job[w], pl.warp_job[w + 1], lane);
+}
+
+// Grid-wide barrier of a cooperative launch: every CTA adds 1 to *bar and waits until it reaches
+// target (= CTAs x barriers so far). Thread 0 waits, bounded (about 4 s); on expiry, or when
+// another CTA gave up (bar[1] != 0), the barrier fails for the whole CTA, the device error word is
+// flagged and bar[1] set so that no CTA waits for it any longer.
+__device__ bool grid_barrier(unsigned int *bar, unsigned int target, unsigned int *err, int *ok_s)
+{
+    __threadfence();
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        atomicAdd(bar, 1u);
+        uint64_t t0;
+        asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t0));
+        bool ok = false;
+        for (uint32_t it = 0;; ++it) {
+            unsigned int v, ab;
+            asm volatile("ld.acquire.gpu.u32 %0, [%1];" : "=r"(v) : "l"(bar) : "memory");
+            if ((int)(v - target) >= 0) {
+                ok = true;
+                break;
+            }
+            asm volatile("ld.relaxed.gpu.u32 %0, [%1];" : "=r"(ab) : "l"(bar + 1) : "memory");
+            if (ab != 0u)
+                break;
+            if (it > 64) {
+                uint64_t t1;
+                asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t1));
+                if (t1 - t0 > 4000000000ull)
+                    break;
+                __nanosleep(200);
+            }
+        }
+        if (!ok) {
+            atomicOr(err, DEV_ERR_TIMEOUT);
+            atomicExch(bar + 1, 1u);
+        }
+        *ok_s = ok ? 1 : 0;
+    }
+    __syncthreads();
+    return *ok_s != 0;
+}
+
+// All T rounds of a placement solve in one cooperative launch (the single-scenario placement
+// table is too small per round to fill the GPU efficiently with one launch per round). Every CTA
+// keeps its own copy of the price state (in global scratch, identical in every CTA); a round is:
+// best responses of the CTA's warps at the copy's prices, demand into buffer round % 3 of U3, a
+// grid barrier, then Eq. price_update applied by every CTA to its own copy from the same totals
+// (identical inputs, identical prices). CTA 0 writes the traces and clears buffer (round + 2) % 3,
+// whose last readers finished before they arrived at this round's barrier. Hash and dual traces
+// are not supported here (the host then uses the per-round launches).
+template <int RT>
+__global__ void __launch_bounds__(kPlaceWarps * 32, 4) k_place_res(DevTable t, DevState st, DevPlace pl,
+                                                                SolveArgs a, PlaceRes pr)
+{
+    extern __shared__ __align__(16) unsigned char smem[];
+    __shared__ int ok_s;
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+    const int R = RT ? RT : t.R, rg = t.r_global;
+    const int S = t.S, P = t.P;
+    const PlaceWarpSmem ws = place_warp_smem(smem, wid, R, P, pl.KC);
+    const size_t cb = blockIdx.x;
+
+    // this CTA's copy of the price state, from the state k_init set up
+    DevState cs = st;
+    cs.lam = pr.lam + cb * S * P;
+    cs.p64 = pr.p64 + cb * S * P;
+    cs.p32 = pr.p32 + cb * S * P;
+    cs.ebound = pr.ebound + cb * S;
+    cs.frozen = pr.frozen + cb * S;
+    cs.status = pr.status + cb * S;
+    cs.converged = pr.converged + cb * S;
+    cs.rounds_run = pr.rounds_run + cb * S;
+    cs.hash_trace = nullptr;
+    cs.dual_trace = nullptr;
+    if (blockIdx.x != 0) {
+        cs.lam_trace = nullptr;
+        cs.dem_trace = nullptr;
+    }
+    for (int i = threadIdx.x; i < S * P; i += blockDim.x) {
+        cs.lam[i] = st.lam[i];
+        cs.p64[i] = st.p64[i];
+        cs.p32[i] = st.p32[i];
+    }
+    for (int i = threadIdx.x; i < S; i += blockDim.x) {
+        cs.ebound[i] = st.ebound[i];
+        cs.frozen[i] = st.frozen[i];
+        cs.status[i] = 0;
+        cs.converged[i] = 0;
+        cs.rounds_run[i] = 0;
+    }
+    __syncthreads();
+
+    const int w = blockIdx.x * kPlaceWarps + wid;
+    WarpCtx<RT, true> c;
+    c.t = t;
+    c.st = cs;
+    c.scen_warps = nullptr;
+    c.a = a;
+    c.R = R;
+    c.rg = rg;
+    c.kind = PASS_ROUND;
+    c.want_min = false;
+    c.want_hash = false;
+    c.uniform_k = 0;
+    c.log2_k = 0;
+#pragma unroll
+    for (int r = 0; r < Cols<RT>::N; ++r)
+        c.acc[r] = 0;
+    c.hacc = 0;
+
+    for (int round = 0; round < a.T; ++round) {
+        unsigned long long *Ub = pr.U3 + (size_t)(round % 3) * S * P;
+        c.st.U = Ub;
+        c.round = round;
+        c.s = -1;
+        if (w < pl.n_warps)
+            place_jobs<RT>(c, pl, ws, pl.warp_job[w], pl.warp_job[w + 1], lane);
+        if (!grid_barrier(pr.bar, (unsigned int)(round + 1) * gridDim.x, st.err, &ok_s))
+            break;
+        DevState us = cs;
+        us.U = Ub;
+        for (int sc = wid; sc < S; sc += kPlaceWarps)
+            if (!us.frozen[sc])
+                update_scenario<8, false>(t, us, a, sc, round, lane);
+        if (blockIdx.x == 0) {
+            unsigned long long *Uz = pr.U3 + (size_t)((round + 2) % 3) * S * P;
+            for (int i = threadIdx.x; i < S * P; i += blockDim.x)
+                Uz[i] = 0ull;
+        }
+        __syncthreads();
+    }
+    // CTA 0 publishes the final price state for the final pass and the objectives
+    if (blockIdx.x == 0) {
+        for (int i = threadIdx.x; i < S * P; i += blockDim.x) {
+            st.lam[i] = cs.lam[i];
+            st.p64[i] = cs.p64[i];
+            st.p32[i] = cs.p32[i];
+        }
+        for (int i = threadIdx.x; i < S; i += blockDim.x) {
+            st.ebound[i] = cs.ebound[i];
+            st.frozen[i] = cs.frozen[i];
+            st.status[i] = cs.status[i];
+            st.converged[i] = cs.converged[i];
+            st.rounds_run[i] = cs.rounds_run[i];
+        }
+    }
 }
 
 // ---------------------------------------------------------------------------------------------
@@ -1947,6 +2130,16 @@ int place_ctas_per_sm(int R, int P, int KC, int N, int NT)
 {
     const int smem = place_smem_bytes(R, P, KC, N, NT);
     int best = 1 << 30;
+    // the grid-resident kernel runs on the same warp ranges, so its co-residency bounds them too
+    {
+        const void *fn = R == 8 ? reinterpret_cast<const void *>(&k_place_res<8>)
+                                : reinterpret_cast<const void *>(&k_place_res<0>);
+        int m = 0;
+        if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess ||
+            cudaOccupancyMaxActiveBlocksPerMultiprocessor(&m, fn, kPlaceWarps * 32, smem) != cudaSuccess)
+            return 0;
+        best = m;
+    }
     for (int plain = 0; plain < 2; ++plain) {
         const int n = place_dispatch(R, plain != 0, [&](const void *fn) -> int {
             if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess)
@@ -1978,6 +2171,29 @@ cudaError_t launch_place(const DevTable &t, const DevState &st, const DevPlace &
             k_place<0, false><<<grid, kPlaceWarps * 32, smem, stream>>>(t, st, pl, a, round, kind);
     }
     return cudaGetLastError();
+}
+
+cudaError_t launch_place_res(const DevTable &t, const DevState &st, const DevPlace &pl, const SolveArgs &a,
+                             const PlaceRes &pr, int grid, cudaStream_t stream)
+{
+    cudaError_t e = cudaMemsetAsync(pr.bar, 0, 2 * sizeof(unsigned int), stream);
+    if (e == cudaSuccess)   // the last rounds of the previous solve leave demand in two buffers
+        e = cudaMemsetAsync(pr.U3, 0, 3 * (size_t)t.S * t.P * sizeof(unsigned long long), stream);
+    if (e != cudaSuccess)
+        return e;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)grid);
+    cfg.blockDim = dim3(kPlaceWarps * 32);
+    cfg.dynamicSmemBytes = (size_t)place_smem_bytes(t.R, t.P, pl.KC, pl.N, pl.NT);
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeCooperative;   // every CTA co-resident: the grid barrier can complete
+    attr[0].val.cooperative = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    if (t.R == 8)
+        return cudaLaunchKernelEx(&cfg, k_place_res<8>, t, st, pl, a, pr);
+    return cudaLaunchKernelEx(&cfg, k_place_res<0>, t, st, pl, a, pr);
 }
 
 cudaError_t launch_mark_duplicates(const DevTable &t, int32_t *units, unsigned long long *marked, cudaStream_t stream)

@@ -90,6 +90,23 @@ constexpr int kPlaceMaxKC = 32;
 constexpr int kPlaceMaxN = 64;
 constexpr int kPlaceMaxNT = 64;
 constexpr int kPlaceWarps = 4;
+constexpr int kPlaceResMaxPrices = 4096;   // S * P limit of the grid-resident placement solve
+
+// Scratch of the grid-resident placement solve (k_place_res): the demand of round r in buffer
+// r % 3 of U3, every CTA's own copy of the price state, and the grid barrier words.
+struct PlaceRes {
+    unsigned long long *U3;     // 3 * S * P
+    double *lam, *p64;          // grid * S * P
+    float *p32;                 // grid * S * P
+    float *ebound;              // grid * S
+    int32_t *frozen, *status, *converged, *rounds_run;   // grid * S each
+    unsigned int *bar;          // [0] arrivals, [1] abort; zeroed before each launch
+};
+
+// All rounds of a placement solve in one cooperative launch of `grid` CTAs (the placement grid;
+// place_ctas_per_sm covers this kernel's occupancy). Zeroes pr.bar and pr.U3 first.
+cudaError_t launch_place_res(const DevTable &t, const DevState &st, const DevPlace &pl, const SolveArgs &a,
+                             const PlaceRes &pr, int grid, cudaStream_t stream);
 
 // Dynamic shared memory and resident CTAs per SM of the placement kernel (0 if it cannot run).
 int place_smem_bytes(int R, int P, int KC, int N, int NT);

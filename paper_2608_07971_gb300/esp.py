@@ -353,12 +353,14 @@ class Solver:
         l0 = None if lambda0 is None else np.ascontiguousarray(lambda0, np.float64).reshape(S, P)
         prm = self.params(eta0, rounds, mode, step, tol, flags, l0)
         lt = dt = ht = gt = None
-        if traces:
+        if traces:          # True: every trace; "prices": the price and demand trajectories only
             lt = np.full((S, T + 1, P), np.nan)
             dt = np.zeros((S, T, P), np.int64)
-            ht = np.zeros((S, T), np.uint64)
-            gt = np.full((S, T + 1), np.nan)
-            prm.lambda_trace, prm.demand_trace, prm.selhash_trace, prm.dual_trace = _p(lt), _p(dt), _p(ht), _p(gt)
+            prm.lambda_trace, prm.demand_trace = _p(lt), _p(dt)
+            if traces is True:
+                ht = np.zeros((S, T), np.uint64)
+                gt = np.full((S, T + 1), np.nan)
+                prm.selhash_trace, prm.dual_trace = _p(ht), _p(gt)
         res = np.zeros(S, RESULT_DTYPE)
         status = esp_solve(self.ctx, prm, res)
         lam = np.zeros((S, P))

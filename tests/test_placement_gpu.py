@@ -102,3 +102,64 @@ def test_factored_placement_rejects_bad_input():
     with pytest.raises(esp.EspError) as e:
         esp.esp_set_penalties(s.ctx, gamma0=0.1)
     assert e.value.status == esp.ESP_ERR_UNSUPPORTED
+
+
+def same_solution(a, b, fields=("lam", "sel", "demand", "lambda_trace", "demand_trace")):
+    for fld in fields:
+        x, y = getattr(a, fld), getattr(b, fld)
+        if x is None and y is None:
+            continue
+        assert np.array_equal(x, y, equal_nan=True), fld
+    for k in ("rounds_run", "converged", "feasible", "status", "primal", "dual"):
+        assert np.array_equal(a.result[k], b.result[k]), k
+
+
+@pytest.mark.parametrize("case", ["bench_shape", "generic", "one_job_per_warp"])
+@pytest.mark.parametrize("mode", [esp.ESP_PRICE_NORMALIZED, esp.ESP_PRICE_RAW])
+def test_grid_resident_placement_equals_per_round_launches(case, mode):
+    """ESP_FLAG_RESIDENT on a placement table: every round in one cooperative launch with a grid
+    barrier per round; every CTA applies Eq. price_update to its own copy of the prices. The result
+    equals the per-round launches bit for bit (and so the expanded table's streaming solve)."""
+    if case == "bench_shape":
+        f = W.placement_expanded(scenarios=[0, 3], J=256).factors
+    elif case == "generic":
+        f = random_factors(zlib.crc32(b"resident"), S=3, J=97)
+    else:
+        f = random_factors(5, S=1, J=7, KC=3, N=9)
+    eta = 0.05 if mode == esp.ESP_PRICE_NORMALIZED else 2e-5
+    T = 37
+    s = esp.Solver()
+    s.load_placement(f)
+    ref = s.solve(eta, T, mode=mode, traces="prices")
+    assert s.launches() == T + 3
+    res = s.solve(eta, T, mode=mode, flags=esp.ESP_FLAG_RESIDENT, traces="prices")
+    assert s.launches() == 4
+    same_solution(res, ref)
+    again = s.solve(eta, T, mode=mode, flags=esp.ESP_FLAG_RESIDENT)      # buffers reused, graph replayed
+    same_solution(again, ref, fields=("lam", "sel", "demand"))
+    full = s.solve(eta, T, mode=mode, flags=esp.ESP_FLAG_RESIDENT, traces=True)   # hash / dual traces:
+    assert s.launches() == T + 3                                                    # per-round launches
+    same_solution(full, ref)
+
+
+def test_grid_resident_placement_stops_like_per_round_launches():
+    f = random_factors(11, S=2, J=120)
+    s = esp.Solver()
+    s.load_placement(f)
+    for tol, T in ((5e-2, 300), (2e-2, 300), (0.0, 0), (0.0, 1)):
+        ref = s.solve(0.05, T, tol=tol, traces="prices")
+        res = s.solve(0.05, T, tol=tol, flags=esp.ESP_FLAG_RESIDENT, traces="prices")
+        same_solution(res, ref)
+        if tol > 0:
+            assert (res.result["converged"] == 1).any() and (res.result["rounds_run"] < T).any()  # oracle: 170, 134 at 5e-2; 293 and no stop at 2e-2
+
+
+def test_grid_resident_placement_full_size():
+    """The benchmark placement table (4096 jobs x 12 configurations x 64 nodes, 400 rounds)."""
+    w = W.placement_expanded()
+    s = esp.Solver()
+    s.load_placement(w.factors)
+    ref = s.solve(w.eta0, w.rounds)
+    res = s.solve(w.eta0, w.rounds, flags=esp.ESP_FLAG_RESIDENT)
+    assert s.launches() == 4
+    same_solution(res, ref, fields=("lam", "sel", "demand"))
