@@ -685,7 +685,7 @@ esp_status enqueue_solve(esp_ctx *ctx, const esp_params *p, const DevState &st, 
         if (place_res) {
             if (e == cudaSuccess && T > 0)
                 e = timed_launch([&]() {
-                    return launch_place_res(t, st, pp, a, ctx->place_res, ctx->place_grid, ctx->stream);
+                    return launch_place_res(t, st, pp, a, ctx->place_res, ctx->stream);
                 });
             if (e == cudaSuccess)
                 e = pass(T, PASS_FINAL);
@@ -1231,22 +1231,24 @@ esp_status esp_load_placement(esp_ctx *ctx, int32_t S, int32_t J, int32_t KC, in
         release_table(ctx);
         return st;
     }
-    // scratch of the grid-resident solve: every CTA keeps a copy of the price state, so it is kept
-    // for small price vectors only (S * P <= kPlaceResMaxPrices)
-    if ((int64_t)S * P <= kPlaceResMaxPrices) {
-        const size_t g = (size_t)ctx->place_grid;
+    // the grid-resident solve (ESP_FLAG_RESIDENT): one CTA per SM holds the price state of every
+    // scenario and each warp at most kPlaceResJobs jobs, all in shared memory
+    if ((int64_t)S * P <= kPlaceResMaxPrices &&
+        n_jobs <= (int64_t)kPlaceResJobs * kPlaceResWarps * ctx->sm_count &&
+        place_res_smem_bytes(S, P, KC, R) <= optin && place_res_ctas_per_sm(S, P, KC, R) >= 1) {
         PlaceRes &pr = ctx->place_res;
+        const int32_t Wr = (int32_t)std::min<int64_t>(n_jobs, (int64_t)kPlaceResWarps * ctx->sm_count);
+        std::vector<int32_t> wr((size_t)Wr + 1);
+        for (int32_t w = 0; w <= Wr; ++w)
+            wr[(size_t)w] = (int32_t)((__int128)n_jobs * w / Wr);
+        int32_t *d_wr = nullptr;
         PALLOC(pr.U3, 3 * (size_t)S * P);
-        PALLOC(pr.lam, g * S * P);
-        PALLOC(pr.p64, g * S * P);
-        PALLOC(pr.p32, g * S * P);
-        PALLOC(pr.ebound, g * S);
-        PALLOC(pr.frozen, g * S);
-        PALLOC(pr.status, g * S);
-        PALLOC(pr.converged, g * S);
-        PALLOC(pr.rounds_run, g * S);
         PALLOC(pr.bar, 2);
-        ESP_CUDA(cudaMemsetAsync(pr.U3, 0, 3 * (size_t)S * P * sizeof(unsigned long long), ctx->stream));
+        PALLOC(d_wr, (size_t)Wr + 1);
+        ESP_CUDA(h2d(d_wr, wr.data(), wr.size() * sizeof(int32_t)));
+        pr.warp_job = d_wr;
+        pr.n_warps = Wr;
+        pr.grid = (Wr + kPlaceResWarps - 1) / kPlaceResWarps;
         ctx->place_res_ok = true;
     }
 #undef PALLOC

@@ -90,23 +90,63 @@ constexpr int kPlaceMaxKC = 32;
 constexpr int kPlaceMaxN = 64;
 constexpr int kPlaceMaxNT = 64;
 constexpr int kPlaceWarps = 4;
-constexpr int kPlaceResMaxPrices = 4096;   // S * P limit of the grid-resident placement solve
+constexpr int kPlaceResMaxPrices = 1024;   // S * P limit of the grid-resident placement solve
+constexpr int kPlaceResWarps = 16;         // warps per CTA of the grid-resident placement solve
+constexpr int kPlaceResJobs = 2;           // jobs per warp it holds in shared memory
 
-// Scratch of the grid-resident placement solve (k_place_res): the demand of round r in buffer
-// r % 3 of U3, every CTA's own copy of the price state, and the grid barrier words.
+// The grid-resident placement solve (k_place_res): one CTA of kPlaceResWarps warps per SM, each warp
+// holding at most kPlaceResJobs jobs; warp w owns the jobs [warp_job[w], warp_job[w + 1]).
 struct PlaceRes {
-    unsigned long long *U3;     // 3 * S * P
-    double *lam, *p64;          // grid * S * P
-    float *p32;                 // grid * S * P
-    float *ebound;              // grid * S
-    int32_t *frozen, *status, *converged, *rounds_run;   // grid * S each
-    unsigned int *bar;          // [0] arrivals, [1] abort; zeroed before each launch
+    unsigned long long *U3;     // 3 * S * P: the demand of round r in buffer r % 3
+    unsigned int *bar;          // [0] barrier arrivals, [1] abort; zeroed before each launch
+    const int32_t *warp_job;    // n_warps + 1
+    int32_t n_warps, grid;
 };
 
-// All rounds of a placement solve in one cooperative launch of `grid` CTAs (the placement grid;
-// place_ctas_per_sm covers this kernel's occupancy). Zeroes pr.bar and pr.U3 first.
+// Shared-memory layout of k_place_res (byte offsets): the CTA's demand, price state and per-scenario
+// reductions, then per warp the gs scratch and its cached jobs.
+struct PlaceResLayout {
+    int u, lam, p64, capd, cap, p32, eb, flags, maxes, warps;
+    int warp_bytes, job_bytes, job_units, job_ufs, job_vals, job_pens, cand;
+    int total;
+};
+
+__host__ __device__ inline PlaceResLayout place_res_layout(int S, int P, int KC, int R)
+{
+    auto up16 = [](int x) { return (x + 15) & ~15; };
+    PlaceResLayout L;
+    const int SP = S * P;
+    L.u = 0;
+    L.lam = L.u + up16(SP * 8);
+    L.p64 = L.lam + up16(SP * 8);
+    L.capd = L.p64 + up16(SP * 8);
+    L.cap = L.capd + up16(SP * 8);
+    L.p32 = L.cap + up16(SP * 8);
+    L.eb = L.p32 + up16(SP * 4);
+    L.flags = L.eb + up16(S * 4);
+    L.maxes = L.flags + up16(6 * S * 4);
+    L.warps = L.maxes + up16(2 * S * 8);
+    // per warp: gs (KC floats), 32 candidate slots, then per job: units, fp32 units, values and the
+    // fp32 penalty of every node
+    const int head = up16(KC * 4) + 32 * 4;
+    L.cand = up16(KC * 4);
+    L.job_units = head;
+    L.job_ufs = head + up16(KC * R * 4);
+    L.job_vals = head + 2 * up16(KC * R * 4);
+    L.job_pens = head + 2 * up16(KC * R * 4) + up16(KC * 8);
+    L.job_bytes = 2 * up16(KC * R * 4) + up16(KC * 8) + kPlaceMaxN * 4;
+    L.warp_bytes = head + kPlaceResJobs * L.job_bytes;
+    L.total = L.warps + kPlaceResWarps * L.warp_bytes;
+    return L;
+}
+
+int place_res_smem_bytes(int S, int P, int KC, int R);
+int place_res_ctas_per_sm(int S, int P, int KC, int R);   // 0 if it cannot run
+
+// All rounds of a placement solve in one cooperative launch of pr.grid CTAs (at most one per SM).
+// Zeroes pr.bar and pr.U3 first.
 cudaError_t launch_place_res(const DevTable &t, const DevState &st, const DevPlace &pl, const SolveArgs &a,
-                             const PlaceRes &pr, int grid, cudaStream_t stream);
+                             const PlaceRes &pr, cudaStream_t stream);
 
 // Dynamic shared memory and resident CTAs per SM of the placement kernel (0 if it cannot run).
 int place_smem_bytes(int R, int P, int KC, int N, int NT);
