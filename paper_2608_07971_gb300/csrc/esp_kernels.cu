@@ -1729,12 +1729,15 @@ __global__ void __launch_bounds__(kPlaceResWarps * 32, 1) k_place_res(DevTable t
     const bool h0 = n0 < N, h1 = n1 < N;
     float pen0[kPlaceResJobs], pen1[kPlaceResJobs];
     uint32_t dup[kPlaceResJobs];
+    int scen[kPlaceResJobs];
 #pragma unroll
     for (int q = 0; q < kPlaceResJobs; ++q) {
         pen0[q] = pen1[q] = 0.0f;
         dup[q] = 0u;
+        scen[q] = 0;
         if (q < nj) {
             const int64_t j = j0 + q;
+            scen[q] = (int)(j / t.J);
             int32_t *us = reinterpret_cast<int32_t *>(wb + L.job_units + q * L.job_bytes);
             float *ufs = reinterpret_cast<float *>(wb + L.job_ufs + q * L.job_bytes);
             double *vs = reinterpret_cast<double *>(wb + L.job_vals + q * L.job_bytes);
@@ -1765,8 +1768,7 @@ __global__ void __launch_bounds__(kPlaceResWarps * 32, 1) k_place_res(DevTable t
         for (int q = 0; q < kPlaceResJobs; ++q) {
             if (q >= nj)
                 break;
-            const int64_t j = j0 + q;
-            const int sc = (int)(j / t.J);
+            const int sc = scen[q];
             if (frozen_s[sc])
                 continue;
             const int32_t *us = reinterpret_cast<const int32_t *>(wb + L.job_units + q * L.job_bytes);
@@ -1818,6 +1820,7 @@ __global__ void __launch_bounds__(kPlaceResWarps * 32, 1) k_place_res(DevTable t
                 i1 = better ? idx : i1;
                 m1 = fminf(m1, qv);
             };
+#pragma unroll 4
             for (int k = 0; k < KC; ++k) {
                 float q0, q1;
                 node_q(k, q0, q1);
@@ -1933,10 +1936,17 @@ __global__ void __launch_bounds__(kPlaceResWarps * 32, 1) k_place_res(DevTable t
         if (!grid_barrier(pr.bar, (unsigned int)(round + 1) * gridDim.x, st.err, &ok_s))
             break;
 
-        // ---- Eq. price_update of every scenario, one price per thread
+        // ---- Eq. price_update of every scenario, one price per thread: the new prices are computed
+        // into registers, and written once no price of the scenario became non-finite
         const double eta = step_size(a.eta0, a.step, round);
         const bool lead = blockIdx.x == 0;
-        for (int i = tid; i < SP; i += blockDim.x) {
+        double nl_r[kPlaceResPricesPerThread], pe_r[kPlaceResPricesPerThread];
+#pragma unroll
+        for (int m = 0; m < kPlaceResPricesPerThread; ++m) {
+            const int i = tid + m * kPlaceResWarps * 32;
+            nl_r[m] = pe_r[m] = 0.0;
+            if (i >= SP)
+                break;
             const int sc = i / P;
             if (frozen_s[sc])
                 continue;
@@ -1945,25 +1955,30 @@ __global__ void __launch_bounds__(kPlaceResWarps * 32, 1) k_place_res(DevTable t
                 st.dem_trace[((size_t)sc * T + round) * P + (i - sc * P)] = U;
             const double lam = lam_s[i];
             const double nl = price_step(lam, U, cap_s[i], capd_s[i], eta, a.mode);
+            nl_r[m] = nl;
+            pe_r[m] = effective_price(nl, capd_s[i], a.mode);
             if (!isfinite(nl))
                 atomicOr(bad_s + sc, 1);
-            atomicMax(dmax_s + sc, (unsigned long long)__double_as_longlong(fabs(nl - lam)));
-            atomicMax(amax_s + sc, (unsigned long long)__double_as_longlong(fabs(lam)));
+            if (a.tol > 0.0) {   // maxima of the stopping rule (non-negative doubles order as integers)
+                atomicMax(dmax_s + sc, (unsigned long long)__double_as_longlong(fabs(nl - lam)));
+                atomicMax(amax_s + sc, (unsigned long long)__double_as_longlong(fabs(lam)));
+            }
         }
         __syncthreads();
-        for (int i = tid; i < SP; i += blockDim.x) {
+#pragma unroll
+        for (int m = 0; m < kPlaceResPricesPerThread; ++m) {
+            const int i = tid + m * kPlaceResWarps * 32;
+            if (i >= SP)
+                break;
             const int sc = i / P;
             if (frozen_s[sc] || bad_s[sc])
                 continue;
-            const long long U = (long long)__ldcg(Ub + i);
-            const double nl = price_step(lam_s[i], U, cap_s[i], capd_s[i], eta, a.mode);
-            lam_s[i] = nl;
+            lam_s[i] = nl_r[m];
             if (lead && st.lam_trace)
-                st.lam_trace[((size_t)sc * (T + 1) + round + 1) * P + (i - sc * P)] = nl;
-            const double pe = effective_price(nl, capd_s[i], a.mode);
-            p64_s[i] = pe;
-            p32_s[i] = __double2float_rn(pe);
-            if (!(pe <= 0x1p100))
+                st.lam_trace[((size_t)sc * (T + 1) + round + 1) * P + (i - sc * P)] = nl_r[m];
+            p64_s[i] = pe_r[m];
+            p32_s[i] = __double2float_rn(pe_r[m]);
+            if (!(pe_r[m] <= 0x1p100))
                 atomicOr(huge_s + sc, 1);
         }
         __syncthreads();

@@ -93,6 +93,7 @@ constexpr int kPlaceWarps = 4;
 constexpr int kPlaceResMaxPrices = 1024;   // S * P limit of the grid-resident placement solve
 constexpr int kPlaceResWarps = 16;         // warps per CTA of the grid-resident placement solve
 constexpr int kPlaceResJobs = 2;           // jobs per warp it holds in shared memory
+constexpr int kPlaceResPricesPerThread = (kPlaceResMaxPrices + kPlaceResWarps * 32 - 1) / (kPlaceResWarps * 32);
 
 // The grid-resident placement solve (k_place_res): one CTA of kPlaceResWarps warps per SM, each warp
 // holding at most kPlaceResJobs jobs; warp w owns the jobs [warp_job[w], warp_job[w + 1]).
