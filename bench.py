@@ -51,6 +51,7 @@ def parse_args():
     ap.add_argument("--no-resident", action="store_true", help="skip the cluster-resident measurement")
     ap.add_argument("--no-factored", action="store_true", help="skip the factored placement measurement")
     ap.add_argument("--no-iac", action="store_true", help="skip the IAC predictor measurement")
+    ap.add_argument("--iac-scenarios", type=int, default=1024, help="what-if scenarios of the IAC batch")
     ap.add_argument("--cpu-seconds", type=float, default=12.0, help="oracle time budget of the CPU baseline")
     return ap.parse_args()
 
@@ -157,7 +158,7 @@ def bench_iac(esp, stream, args, dist, barrier):
     (the default) and the CUDA-core kernel beside it."""
     import torch
     from paper_2608_07971_gb300 import workloads as W
-    w = W.iac_batch()
+    w = W.iac_batch(S=args.iac_scenarios)
     dev = torch.device("cuda", torch.cuda.current_device())
     rows = torch.from_numpy(w.rows).to(dev)
     pairs = torch.from_numpy(w.pairs).to(dev)
@@ -483,14 +484,36 @@ def run_ours(args):
         f_value, f_s, _ = aggregate(dist, f_ms / 1e3, evals_step, device="cuda")
         lam_f = np.zeros((t.S, t.P))
         esp.esp_get_prices(fs.ctx, lam_f)
+        f_launches = esp.esp_last_launch_count(fs.ctx)
+        # the grid-resident variant (ESP_FLAG_RESIDENT: all rounds in one cooperative launch)
+        prm_fr = fs.params(w.eta0, T, mode=w.mode, step=w.step, flags=esp.ESP_FLAG_RESIDENT)
+        for _ in range(args.warmup):
+            esp.esp_solve_async(fs.ctx, prm_fr)
+        barrier()
+        torch.cuda.synchronize()
+        f0.record(stream)
+        for _ in range(args.steps):
+            esp.esp_solve_async(fs.ctx, prm_fr)
+        f1.record(stream)
+        stream.synchronize()
+        barrier()
+        fr_ms = f0.elapsed_time(f1) / args.steps
+        fr_value, fr_s, _ = aggregate(dist, fr_ms / 1e3, evals_step, device="cuda")
+        lam_fr = np.zeros((t.S, t.P))
+        esp.esp_get_prices(fs.ctx, lam_fr)
+        fr_launches = esp.esp_last_launch_count(fs.ctx)
         f = w.factors
         fbytes = f.cfg_units.nbytes + f.cfg_values.nbytes + f.sens.nbytes + f.job_type.nbytes
         factored = {"value": f_value, "unit": "option-evals/s", "ms_per_step": f_s * 1e3,
                     "rounds_per_sec": T / f_s, "bytes_per_pass": int(fbytes),
-                    "launches_per_step": esp.esp_last_launch_count(fs.ctx),
+                    "launches_per_step": f_launches,
                     "same_prices_as_streaming": bool(np.array_equal(lam_f, lam_stream)),
+                    "grid_resident": {"value": fr_value, "ms_per_step": fr_s * 1e3, "rounds_per_sec": T / fr_s,
+                                      "launches_per_step": fr_launches,
+                                      "same_prices_as_streaming": bool(np.array_equal(lam_fr, lam_stream))},
                     "note": "esp_load_placement: configurations x nodes scored from the factors, the expanded "
-                            "options are never stored; evaluations counted over the expanded options"}
+                            "options are never stored; evaluations counted over the expanded options; "
+                            "grid_resident = ESP_FLAG_RESIDENT, every round in one cooperative launch"}
         fs.close()
 
     # the IAC slowdown predictor (Eq. dnn_pred) over the what-if batch's co-location pairs
