@@ -39,6 +39,19 @@ struct DevArr {
 
 }  // namespace
 
+// The host plan of a load (option counts, sorted layout, tiles and warp ranges), kept for the next
+// load of a table with the same shape and offsets.
+struct PlanCache {
+    bool valid = false;
+    int32_t S = 0, J = 0, R = 0, P = 0, max_warps = 0, tile_opt = 0;
+    bool grouped = false, sorted_enabled = false;
+    std::vector<int64_t> off;
+    int64_t min_k = 0, max_k = 0;
+    bool sorted = false;
+    esp::SortedLayout lay;
+    esp::Plan plan;
+};
+
 struct esp_ctx {
     int device = 0;
     cudaStream_t stream = nullptr;
@@ -50,7 +63,11 @@ struct esp_ctx {
     int32_t S = 0, J = 0, R = 0, P = 0, rg = 0, n_groups = 0;
     int64_t n_opt = 0;
     int32_t small_units = 0;
-    std::vector<void *> table_bufs;  // everything freed on reload
+    PlanCache pc;
+    // device buffers of the loaded table and solve state (pointer, bytes); a reload hands them to
+    // `pool`, from which the new table's allocations are served when the sizes fit
+    std::vector<std::pair<void *, size_t>> table_bufs;
+    std::vector<std::pair<void *, size_t>> pool;
     int32_t *units = nullptr;
     double *values = nullptr;
     int64_t *off = nullptr;
@@ -149,30 +166,63 @@ esp_status dev_alloc(esp_ctx *ctx, T **p, size_t count, size_t pad_bytes = 64)
 {
     void *q = nullptr;
     const size_t bytes = count * sizeof(T) + pad_bytes;
-    cudaError_t e = cudaMalloc(&q, bytes);
-    if (e == cudaErrorMemoryAllocation) {
-        cudaGetLastError();
-        return ESP_ERR_OOM;
+    // reuse the smallest pooled buffer that fits and is at most about twice the size (a reload of a
+    // table of the same shape gets every buffer back, without cudaMalloc / cudaFree; work still
+    // queued on the context's stream that used it is ordered before the new contents)
+    size_t best = SIZE_MAX, bi = SIZE_MAX;
+    for (size_t i = 0; i < ctx->pool.size(); ++i) {
+        const size_t have = ctx->pool[i].second;
+        if (have >= bytes && have <= 2 * bytes + 4096 && have < best) {
+            best = have;
+            bi = i;
+        }
     }
+    size_t have = bytes;
+    if (bi != SIZE_MAX) {
+        q = ctx->pool[bi].first;
+        have = ctx->pool[bi].second;
+        ctx->pool.erase(ctx->pool.begin() + (std::ptrdiff_t)bi);
+    } else {
+        cudaError_t e = cudaMalloc(&q, bytes);
+        if (e == cudaErrorMemoryAllocation) {
+            cudaGetLastError();
+            return ESP_ERR_OOM;
+        }
+        if (e != cudaSuccess)
+            return cuda_fail(ctx, e);
+    }
+    ctx->table_bufs.emplace_back(q, have);
+    cudaError_t e = cudaMemsetAsync(q, 0, bytes, ctx->stream);
     if (e != cudaSuccess)
         return cuda_fail(ctx, e);
-    e = cudaMemsetAsync(q, 0, bytes, ctx->stream);
-    if (e != cudaSuccess)
-        return cuda_fail(ctx, e);
-    ctx->table_bufs.push_back(q);
     *p = static_cast<T *>(q);
     return ESP_OK;
 }
 
-void release_table(esp_ctx *ctx)
+// Frees the pooled buffers that the current table did not take.
+void trim_pool(esp_ctx *ctx)
+{
+    for (auto &b : ctx->pool)
+        cudaFree(b.first);
+    ctx->pool.clear();
+}
+
+// Drops the loaded table. keep = true (the start of a reload) moves its buffers to the pool, from which
+// the next table's allocations are served; keep = false frees everything.
+void release_table(esp_ctx *ctx, bool keep = false)
 {
     if (ctx->gexec) {
         cudaGraphExecDestroy(ctx->gexec);
         ctx->gexec = nullptr;
         ctx->gkey = GraphKey();
     }
-    for (void *p : ctx->table_bufs)
-        cudaFree(p);
+    if (keep) {
+        ctx->pool.insert(ctx->pool.end(), ctx->table_bufs.begin(), ctx->table_bufs.end());
+    } else {
+        for (auto &b : ctx->table_bufs)
+            cudaFree(b.first);
+        trim_pool(ctx);
+    }
     ctx->table_bufs.clear();
     ctx->res.clear();
     ctx->res_cuts = nullptr;
@@ -363,7 +413,7 @@ esp_status load_common(esp_ctx *ctx, int32_t S, int32_t J, int32_t R, int32_t P,
     if (!grouped)
         rg = R;
     ESP_CUDA(cudaSetDevice(ctx->device));
-    release_table(ctx);
+    release_table(ctx, true);
 
     const int64_t n_jobs = (int64_t)S * J;
     std::vector<int64_t> h_off;
@@ -416,6 +466,8 @@ esp_status load_common(esp_ctx *ctx, int32_t S, int32_t J, int32_t R, int32_t P,
         ESP_CUDA(cudaMemcpyAsync(ctx->group, group, (size_t)n_opt * sizeof(uint16_t), kind, ctx->stream));
     ESP_CUDA(cudaMemcpyAsync(ctx->cap, capacity, (size_t)S * P * sizeof(int64_t), kind, ctx->stream));
 
+    // validation, then (stream-ordered after it) the marking of duplicates in the device copy; the
+    // host plans the pass meanwhile, and checks the validation result before anything uses the plan
     const DevTable t = dev_table(ctx);
     ESP_CUDA(launch_validate(t, ctx->vmax, ctx->umax, ctx->valflags, ctx->stream));
     unsigned int vflags = 0;
@@ -423,32 +475,45 @@ esp_status load_common(esp_ctx *ctx, int32_t S, int32_t J, int32_t R, int32_t P,
     ESP_CUDA(cudaMemcpyAsync(&vflags, ctx->valflags, sizeof(unsigned int), cudaMemcpyDeviceToHost, ctx->stream));
     ESP_CUDA(cudaMemcpyAsync(h_umax.data(), ctx->umax, h_umax.size() * sizeof(int32_t), cudaMemcpyDeviceToHost,
                              ctx->stream));
-    ESP_CUDA(cudaStreamSynchronize(ctx->stream));
-    if (vflags != 0) {
+    // the plan of the previous load serves when the shape and offsets are the same
+    PlanCache &pc = ctx->pc;
+    const bool cached = pc.valid && pc.S == S && pc.J == J && pc.R == R && pc.P == P && pc.grouped == grouped &&
+                        pc.sorted_enabled == ctx->sorted_enabled && (int64_t)pc.off.size() == n_jobs + 1 &&
+                        std::memcmp(pc.off.data(), off_host, (size_t)(n_jobs + 1) * sizeof(int64_t)) == 0;
+    // option counts, on the host meanwhile: every job non-empty makes the offsets strictly
+    // increasing up to n_opt, so no kernel below can index outside the table
+    int64_t max_k = 1, min_k = n_jobs ? INT64_MAX : 1;
+    if (cached) {
+        max_k = pc.max_k;
+        min_k = pc.min_k;
+    } else {
+        for (int64_t j = 0; j < n_jobs; ++j) {
+            const int64_t k = off_host[j + 1] - off_host[j];
+            max_k = std::max<int64_t>(max_k, k);
+            min_k = std::min<int64_t>(min_k, k);
+        }
+    }
+    if (min_k < 1) {
+        cudaStreamSynchronize(ctx->stream);
         release_table(ctx);
         return ESP_ERR_INVALID_ARG;
     }
-    ctx->small_units = 1;
-    for (int32_t x : h_umax)
-        if (x >= (1 << 23))
-            ctx->small_units = 0;
-    // duplicates are marked in the device copy only (validation has already read the units)
-    ESP_CUDA(launch_mark_duplicates(dev_table(ctx), ctx->units, ctx->stats + 1, ctx->stream));
+    ESP_CUDA(launch_mark_duplicates(t, ctx->units, ctx->stats + 1, ctx->stream));
 
     // plan the evaluation pass
-    int64_t max_k = 1, min_k = n_jobs ? INT64_MAX : 1;
-    for (int64_t j = 0; j < n_jobs; ++j) {
-        const int64_t k = off_host[j + 1] - off_host[j];
-        max_k = std::max<int64_t>(max_k, k);
-        min_k = std::min<int64_t>(min_k, k);
-    }
     ctx->uniform_k = (!grouped && min_k == max_k && max_k <= 32 && (max_k & (max_k - 1)) == 0) ? (int32_t)max_k : 0;
 
     // general tables without a group column: the evaluation pass reads the sorted layout (runs of
     // equal-size jobs take the uniform paths). Jobs keep their option order, so the copy inherits
     // the duplicate marks of the original; its padding is marked as it is written.
-    SortedLayout lay;
-    if (ctx->sorted_enabled && !grouped && ctx->uniform_k == 0 && J >= 1 && sort_layout(off_host, S, J, lay)) {
+    SortedLayout lay_new;
+    bool use_sorted = false;
+    if (cached)
+        use_sorted = pc.sorted;
+    else
+        use_sorted = ctx->sorted_enabled && !grouped && ctx->uniform_k == 0 && J >= 1 && sort_layout(off_host, S, J, lay_new);
+    const SortedLayout &lay = cached ? pc.lay : lay_new;
+    if (use_sorted) {
         const int64_t sn = lay.off.back();
         ALLOC(ctx->s_units, (size_t)sn * R);
         ALLOC(ctx->s_values, (size_t)sn);
@@ -472,12 +537,25 @@ esp_status load_common(esp_ctx *ctx, int32_t S, int32_t J, int32_t R, int32_t P,
         return ESP_ERR_UNSUPPORTED;
     }
     const int max_warps = ctx->sm_count * per_sm * kWarpsPerCta;
-    Plan plan;
-    if (!plan_tiles(plan_off, S, J, tile_opt, max_warps, plan, plan_scen, plan_runk) ||
-        !check_plan(plan_off, S, J, plan, plan_scen, plan_runk)) {
+    Plan plan_new;
+    const bool plan_cached = cached && pc.max_warps == max_warps && pc.tile_opt == tile_opt;
+    if (!plan_cached && (!plan_tiles(plan_off, S, J, tile_opt, max_warps, plan_new, plan_scen, plan_runk) ||
+                         !check_plan(plan_off, S, J, plan_new, plan_scen, plan_runk))) {
+        cudaStreamSynchronize(ctx->stream);
         release_table(ctx);
         return ESP_ERR_INVALID_ARG;
     }
+    const Plan &plan = plan_cached ? pc.plan : plan_new;
+    // the validation result (the copies, validation and duplicate marking ran during the planning)
+    ESP_CUDA(cudaStreamSynchronize(ctx->stream));
+    if (vflags != 0) {
+        release_table(ctx);
+        return ESP_ERR_INVALID_ARG;
+    }
+    ctx->small_units = 1;
+    for (int32_t x : h_umax)
+        if (x >= (1 << 23))
+            ctx->small_units = 0;
     ctx->n_warps = plan.n_warps;
     ctx->tile_opt = plan.tile_opt;
     ctx->grid = (plan.n_warps + kWarpsPerCta - 1) / kWarpsPerCta;
@@ -567,6 +645,26 @@ esp_status load_common(esp_ctx *ctx, int32_t S, int32_t J, int32_t R, int32_t P,
         return st;
     }
     ESP_CUDA(cudaStreamSynchronize(ctx->stream));
+    if (!plan_cached) {   // keep this load's plan for the next load of the same offsets
+        pc.valid = true;
+        pc.S = S;
+        pc.J = J;
+        pc.R = R;
+        pc.P = P;
+        pc.grouped = grouped;
+        pc.sorted_enabled = ctx->sorted_enabled;
+        if (!cached) {
+            pc.off.assign(off_host, off_host + n_jobs + 1);
+            pc.min_k = min_k;
+            pc.max_k = max_k;
+            pc.sorted = use_sorted;
+            pc.lay = std::move(lay_new);
+        }
+        pc.max_warps = max_warps;
+        pc.tile_opt = tile_opt;
+        pc.plan = std::move(plan_new);
+    }
+    trim_pool(ctx);
     ctx->loaded = true;
     ctx->solved = false;
     return ESP_OK;
@@ -864,10 +962,15 @@ esp_status esp_set_stream(esp_ctx *ctx, void *cuda_stream)
     esp_status st = check_ctx(ctx);
     if (st != ESP_OK)
         return st;
-    if (ctx->stream != static_cast<cudaStream_t>(cuda_stream) && ctx->gexec) {
-        cudaGraphExecDestroy(ctx->gexec);
-        ctx->gexec = nullptr;
-        ctx->gkey = GraphKey();
+    if (ctx->stream != static_cast<cudaStream_t>(cuda_stream)) {
+        // work queued on the old stream finishes before another stream can reuse the buffers
+        ESP_CUDA(cudaSetDevice(ctx->device));
+        ESP_CUDA(cudaStreamSynchronize(ctx->stream));
+        if (ctx->gexec) {
+            cudaGraphExecDestroy(ctx->gexec);
+            ctx->gexec = nullptr;
+            ctx->gkey = GraphKey();
+        }
     }
     ctx->stream = static_cast<cudaStream_t>(cuda_stream);
     return ESP_OK;
@@ -1149,7 +1252,7 @@ esp_status esp_load_placement(esp_ctx *ctx, int32_t S, int32_t J, int32_t KC, in
     const int per_sm = place_ctas_per_sm(R, P, KC, N, NT);
     if (per_sm < 1)
         return ESP_ERR_UNSUPPORTED;
-    release_table(ctx);
+    release_table(ctx, true);
     ctx->S = S;
     ctx->J = J;
     ctx->R = R;
@@ -1253,6 +1356,7 @@ esp_status esp_load_placement(esp_ctx *ctx, int32_t S, int32_t J, int32_t KC, in
     }
 #undef PALLOC
     ESP_CUDA(cudaStreamSynchronize(ctx->stream));
+    trim_pool(ctx);
     ctx->loaded = true;
     ctx->solved = false;
     return ESP_OK;
@@ -1303,7 +1407,7 @@ esp_status esp_set_penalties(esp_ctx *ctx, double gamma0, const int32_t *c_cur, 
             return ESP_ERR_OOM;
         }
         ESP_CUDA(e);
-        ctx->table_bufs.push_back(q);
+        ctx->table_bufs.emplace_back(q, n_opt * sizeof(double) + 64);
         ctx->values0 = static_cast<double *>(q);
         ESP_CUDA(cudaMemcpyAsync(ctx->values0, ctx->values, n_opt * sizeof(double), cudaMemcpyDeviceToDevice,
                                  ctx->stream));

@@ -2209,39 +2209,72 @@ __global__ void k_objectives(DevTable t, DevState st, SolveArgs a)
 // ---------------------------------------------------------------------------------------------
 // Load-time validation and per-scenario maxima (max |v|, max unit per column).
 
-__global__ void k_validate_options(DevTable t, double *vmax, int32_t *umax, unsigned int *flags)
+constexpr int kValidateThreads = 256;
+
+// Per scenario (blockIdx.y): finite values, non-negative units, groups in range, and the maxima
+// max |v| and max u_r, reduced per warp and per block before one atomic per block and quantity.
+__global__ void __launch_bounds__(kValidateThreads) k_validate_options(DevTable t, double *vmax, int32_t *umax,
+                                                                       unsigned int *flags)
 {
-  for (int s = blockIdx.y; s < t.S; s += gridDim.y) {
-    const int64_t a = t.job_off[(int64_t)s * t.J];
-    const int64_t b = t.job_off[(int64_t)(s + 1) * t.J];
+    __shared__ unsigned long long s_vm[kValidateThreads / 32];
+    __shared__ int32_t s_um[kValidateThreads / 32][kMaxR];
+    __shared__ unsigned int s_bad[kValidateThreads / 32];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int R = t.R;
-    double vm = 0.0;
-    int32_t um[kMaxR];
-    for (int r = 0; r < kMaxR; ++r)
-        um[r] = 0;
-    unsigned int bad = 0;
-    for (int64_t o = a + (int64_t)blockIdx.x * blockDim.x + threadIdx.x; o < b; o += (int64_t)gridDim.x * blockDim.x) {
-        const double v = t.values[o];
-        if (!isfinite(v))
-            bad |= VAL_VALUE_NONFINITE;
-        else
-            vm = fmax(vm, fabs(v));
-        for (int r = 0; r < R; ++r) {
-            const int32_t u = t.units[o * R + r];
-            if (u < 0)
-                bad |= VAL_UNITS_NEG;
-            um[r] = max(um[r], u);
+    for (int s = blockIdx.y; s < t.S; s += gridDim.y) {
+        const int64_t a = t.job_off[(int64_t)s * t.J];
+        const int64_t b = t.job_off[(int64_t)(s + 1) * t.J];
+        unsigned long long vm = 0ull;   // non-negative doubles order like their bit patterns
+        int32_t um[kMaxR];
+        for (int r = 0; r < kMaxR; ++r)
+            um[r] = 0;
+        unsigned int bad = 0;
+        for (int64_t o = a + (int64_t)blockIdx.x * blockDim.x + threadIdx.x; o < b;
+             o += (int64_t)gridDim.x * blockDim.x) {
+            const double v = t.values[o];
+            if (!isfinite(v))
+                bad |= VAL_VALUE_NONFINITE;
+            else
+                vm = max(vm, (unsigned long long)__double_as_longlong(fabs(v)));
+            for (int r = 0; r < R; ++r) {
+                const int32_t u = t.units[o * R + r];
+                if (u < 0)
+                    bad |= VAL_UNITS_NEG;
+                um[r] = max(um[r], u);
+            }
+            if (t.group && (int)t.group[o] >= t.n_groups)
+                bad |= VAL_GROUP_RANGE;
         }
-        if (t.group && (int)t.group[o] >= t.n_groups)
-            bad |= VAL_GROUP_RANGE;
+#pragma unroll
+        for (int d = 16; d >= 1; d >>= 1)
+            vm = max(vm, __shfl_xor_sync(FULL, vm, d));
+        bad = __reduce_or_sync(FULL, bad);
+        for (int r = 0; r < R; ++r)
+            um[r] = __reduce_max_sync(FULL, um[r]);
+        if (lane == 0) {
+            s_vm[warp] = vm;
+            s_bad[warp] = bad;
+            for (int r = 0; r < R; ++r)
+                s_um[warp][r] = um[r];
+        }
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            for (int w = 1; w < kValidateThreads / 32; ++w) {
+                vm = max(vm, s_vm[w]);
+                bad |= s_bad[w];
+            }
+            if (bad)
+                atomicOr(flags, bad);
+            atomicMax(reinterpret_cast<unsigned long long *>(vmax + s), vm);
+        }
+        if (threadIdx.x < R) {
+            int32_t m = s_um[0][threadIdx.x];
+            for (int w = 1; w < kValidateThreads / 32; ++w)
+                m = max(m, s_um[w][threadIdx.x]);
+            atomicMax(umax + (size_t)s * R + threadIdx.x, m);
+        }
+        __syncthreads();
     }
-    if (bad)
-        atomicOr(flags, bad);
-    // non-negative doubles order like their bit patterns
-    atomicMax(reinterpret_cast<unsigned long long *>(vmax + s), (unsigned long long)__double_as_longlong(vm));
-    for (int r = 0; r < R; ++r)
-        atomicMax(umax + (size_t)s * R + r, um[r]);
-  }
 }
 
 __global__ void k_validate_offsets(DevTable t, unsigned int *flags)
@@ -2336,11 +2369,12 @@ int pass_ctas_per_sm(int R, bool grouped, bool uniform, int P, int tile_opt)
 cudaError_t launch_validate(const DevTable &t, double *vmax, int32_t *umax, unsigned int *flags, cudaStream_t stream)
 {
     if (t.S > 0) {
+        // about 8 options per thread, so each block's reduction and atomics cover a few thousand
         const int64_t per = t.n_opt / (t.S > 0 ? t.S : 1) + 1;
-        int gx = (int)((per + 255) / 256);
+        int gx = (int)((per + 8 * kValidateThreads - 1) / (8 * kValidateThreads));
         gx = gx < 1 ? 1 : (gx > 256 ? 256 : gx);
         dim3 grid(gx, t.S < 65535 ? t.S : 65535);
-        k_validate_options<<<grid, 256, 0, stream>>>(t, vmax, umax, flags);
+        k_validate_options<<<grid, kValidateThreads, 0, stream>>>(t, vmax, umax, flags);
     }
     k_validate_offsets<<<256, 256, 0, stream>>>(t, flags);
     return cudaGetLastError();

@@ -52,10 +52,18 @@ bool plan_tiles(const int64_t *off, int32_t S, int32_t J, int32_t tile_opt, int3
             return false;
 
     // 1. tiles in job order: whole jobs of one scenario (and one run) up to tile_opt options, or the
-    //    chunks of a job larger than a tile
+    //    chunks of a job larger than a tile. Without scen, job j belongs to scenario j / J, tracked
+    //    incrementally (s_cur, s_end) instead of dividing per job.
+    out.tiles.reserve((size_t)std::min<int64_t>(n_jobs, total / std::max(1, tile_opt / 4) + S + 1));
+    int32_t s_cur = 0;
+    int64_t s_end = J;
     int64_t j = 0;
     while (j < n_jobs) {
-        const int32_t s = scen ? scen[j] : (int32_t)(j / J);
+        while (!scen && j >= s_end) {
+            ++s_cur;
+            s_end += J;
+        }
+        const int32_t s = scen ? scen[j] : s_cur;
         const int64_t K = off[j + 1] - off[j];
         if (K > tile_opt) {
             const int64_t nch = (K + tile_opt - 1) / tile_opt;
@@ -75,8 +83,8 @@ bool plan_tiles(const int64_t *off, int32_t S, int32_t J, int32_t tile_opt, int3
         const int64_t opt0 = off[j];
         const int32_t rk = runk ? runk[j] : 0;
         int64_t jj = j;
-        while (jj < n_jobs && (scen ? scen[jj] == s : jj / J == s) && (runk ? runk[jj] == rk : true) &&
-               off[jj + 1] - opt0 <= tile_opt)
+        const int64_t jlim = scen ? n_jobs : std::min<int64_t>(n_jobs, s_end);
+        while (jj < jlim && (!scen || scen[jj] == s) && (!runk || runk[jj] == rk) && off[jj + 1] - opt0 <= tile_opt)
             ++jj;
         TileDesc d;
         d.opt_begin = opt0;
@@ -165,16 +173,24 @@ bool check_plan(const int64_t *off, int32_t S, int32_t J, const Plan &p, const i
             const int64_t j1 = d.job_begin + d.n_job;
             if (j1 > n_jobs || d.opt_begin != off[d.job_begin] || d.opt_begin + d.n_opt != off[j1])
                 return false;
-            for (int64_t j = d.job_begin; j < j1; ++j) {
-                if (scen_of(j) != d.scenario)
+            if (!scen) {   // a contiguous range lies in one scenario iff its ends do
+                if (scen_of(d.job_begin) != d.scenario || scen_of(j1 - 1) != d.scenario)
                     return false;
-                if (d.flags & TILE_RUN) {
-                    const int k = tile_run_k(d.flags);
-                    if (!runk || runk[j] != k || off[j + 1] - off[j] != k)
+            }
+            if (scen || runk) {
+                for (int64_t j = d.job_begin; j < j1; ++j) {
+                    if (scen && scen[j] != d.scenario)
                         return false;
-                } else if (runk && runk[j] != 0) {
-                    return false;
+                    if (d.flags & TILE_RUN) {
+                        const int k = tile_run_k(d.flags);
+                        if (!runk || runk[j] != k || off[j + 1] - off[j] != k)
+                            return false;
+                    } else if (runk && runk[j] != 0) {
+                        return false;
+                    }
                 }
+            } else if (d.flags & TILE_RUN) {
+                return false;
             }
             if ((d.flags & TILE_RUN) && (d.opt_begin & 3) != 0 && tile_run_k(d.flags) >= 4)
                 return false;   // a run of 4m-option jobs starts on a 4-option boundary
