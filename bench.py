@@ -531,15 +531,23 @@ def run_ours(args):
         prm_e2e = solver.params(w.eta0, T, mode=w.mode, step=w.step, flags=0)
         res_e = np.zeros(t.S, esp.RESULT_DTYPE)
 
+        parts = np.zeros(3)
+
         def e2e_step():
+            p0 = time.perf_counter()
             esp.esp_load_options(ctx, t.S, t.J, t.R, t.P, t.r_global, h_off, h_units, h_vals, h_grp, h_cap)
+            p1 = time.perf_counter()
             esp.esp_solve(ctx, prm_e2e, res_e)
+            p2 = time.perf_counter()
             esp.esp_get_selection(ctx, h_sel)
             esp.esp_get_prices(ctx, h_lam)
+            p3 = time.perf_counter()
+            parts[:] += (p1 - p0, p2 - p1, p3 - p2)
 
         for _ in range(max(1, args.warmup)):
             e2e_step()
         barrier()
+        parts[:] = 0.0
         t0 = time.perf_counter()
         for _ in range(args.steps):
             e2e_step()
@@ -550,7 +558,8 @@ def run_ours(args):
             (0 if t.group is None else t.group.nbytes)
         d2h = h_sel.numel() * 4 + h_lam.numel() * 8 + t.S * esp.RESULT_DTYPE.itemsize
         e2e = {"value": e2e_value, "unit": "option-evals/s", "h2d_bytes_per_step": int(h2d),
-               "d2h_bytes_per_step": int(d2h), "ms_per_step": e2e_s * 1e3}
+               "d2h_bytes_per_step": int(d2h), "ms_per_step": e2e_s * 1e3,
+               "ms_load_solve_read": [round(1e3 * x / args.steps, 3) for x in parts]}
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:

@@ -2081,6 +2081,7 @@ __global__ void __launch_bounds__(kDedupWarps * 32) k_mark_duplicates(DevTable t
     __shared__ uint64_t hs[kDedupWarps][kDedupMaxK];
     const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
     const int64_t n_jobs = (int64_t)t.S * t.J;
+    unsigned int n_marked = 0;   // counted per lane, one atomic per warp at the end
     for (int64_t j = (int64_t)blockIdx.x * kDedupWarps + wid; j < n_jobs; j += (int64_t)gridDim.x * kDedupWarps) {
         const int64_t a = t.job_off[j];
         const int K = (int)(t.job_off[j + 1] - a);
@@ -2094,13 +2095,16 @@ __global__ void __launch_bounds__(kDedupWarps * 32) k_mark_duplicates(DevTable t
             for (int k2 = 0; k2 < k; ++k2) {
                 if (hs[wid][k2] == h && same_option(t, a + k, a + k2)) {
                     units[(a + k) * t.R] |= (int32_t)0x80000000;
-                    atomicAdd(marked, 1ull);
+                    ++n_marked;
                     break;
                 }
             }
         }
         __syncwarp();
     }
+    n_marked = __reduce_add_sync(FULL, n_marked);
+    if (lane == 0 && n_marked != 0)
+        atomicAdd(marked, (unsigned long long)n_marked);
 }
 
 // Sorted layout: one warp per job copies the job's options from the original table and writes its
