@@ -776,7 +776,9 @@ esp_status enqueue_solve(esp_ctx *ctx, const esp_params *p, const DevState &st, 
     auto pass = [&](int r, PassKind kind) -> cudaError_t {
         if (ctx->placement)
             return timed_launch([&]() { return launch_place(t, st, pp, a, r, kind, ctx->place_grid, ctx->stream); });
-        return timed_launch([&]() { return launch_pass(t, st, pl, a, r, kind, ctx->grid, ctx->stream); });
+        // without per-pass events the previous operation is always a kernel: the pass overlaps its
+        // start with that kernel's tail (programmatic dependent launch)
+        return timed_launch([&]() { return launch_pass(t, st, pl, a, r, kind, ctx->grid, ctx->stream, !timed); });
     };
     auto issue = [&]() -> cudaError_t {
         cudaError_t e = launch_init(t, st, a, has_l0 ? ctx->lambda0 : nullptr, ctx->stream);

@@ -1252,6 +1252,9 @@ __global__ void __launch_bounds__(kWarpsPerCta * 32, pass_min_ctas<RT, UNI>()) k
                                                                           SolveArgs a, int round, int kind)
 {
     extern __shared__ __align__(128) unsigned char smem[];
+    // a pass launched as a programmatic dependent of this one may start its CTAs as soon as slots
+    // free up; it waits (griddepcontrol.wait below) for this grid's completion before reading state
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
     const int w = blockIdx.x * kWarpsPerCta + wid;
     if (w >= pl.n_warps)
@@ -1330,6 +1333,10 @@ __global__ void __launch_bounds__(kWarpsPerCta * 32, pass_min_ctas<RT, UNI>()) k
     if (lane == 0)
         for (int k = issued; k < k_end && k < k_begin + kPrefetchTiles; ++k)
             prefetch_tile(t, pl.tiles[k]);
+    // everything above reads only the table and the plan; prices, flags and the demand accumulators
+    // were written by the previous kernel on the stream, which is complete after this wait (a no-op
+    // for an ordinary launch)
+    asm volatile("griddepcontrol.wait;" ::: "memory");
     int64_t big_first = 0;
     Best big_carry = best_none();
     Best big_priv = best_none();     // lane-private state of a chunked job
@@ -2307,13 +2314,25 @@ template <int RT, bool G, bool UNI>
 struct PassKernels {
     static const void *plain() { return reinterpret_cast<const void *>(&k_pass<RT, G, UNI, true>); }
     static const void *other() { return reinterpret_cast<const void *>(&k_pass<RT, G, UNI, false>); }
+    // pdl: programmatic dependent launch, so the pass's CTAs may start (and stage their first tiles)
+    // while the previous kernel on the stream finishes; the kernel waits for it before reading state
     static void launch(bool plain, int grid, int smem, cudaStream_t stream, const DevTable &t, const DevState &st,
-                       const DevPlan &pl, const SolveArgs &a, int round, int kind)
+                       const DevPlan &pl, const SolveArgs &a, int round, int kind, bool pdl)
     {
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3((unsigned)grid);
+        cfg.blockDim = dim3(kWarpsPerCta * 32);
+        cfg.dynamicSmemBytes = (size_t)smem;
+        cfg.stream = stream;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[0].val.programmaticStreamSerializationAllowed = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = pdl ? 1 : 0;
         if (plain)
-            k_pass<RT, G, UNI, true><<<grid, kWarpsPerCta * 32, smem, stream>>>(t, st, pl, a, round, kind);
+            cudaLaunchKernelEx(&cfg, k_pass<RT, G, UNI, true>, t, st, pl, a, round, kind);
         else
-            k_pass<RT, G, UNI, false><<<grid, kWarpsPerCta * 32, smem, stream>>>(t, st, pl, a, round, kind);
+            cudaLaunchKernelEx(&cfg, k_pass<RT, G, UNI, false>, t, st, pl, a, round, kind);
     }
 };
 
@@ -2425,13 +2444,13 @@ cudaError_t launch_init(const DevTable &t, const DevState &st, const SolveArgs &
 }
 
 cudaError_t launch_pass(const DevTable &t, const DevState &st, const DevPlan &pl, const SolveArgs &a, int round,
-                        PassKind kind, int grid, cudaStream_t stream)
+                        PassKind kind, int grid, cudaStream_t stream, bool pdl)
 {
     const bool grouped = t.group != nullptr;
     const int smem = pass_smem_bytes(t.R, grouped, pl.uniform_k > 0, t.P, pl.tile_opt);
     const bool plain = kind == PASS_ROUND && st.hash_trace == nullptr && st.dual_trace == nullptr;
     dispatch_shape(t.R, grouped, pl.uniform_k > 0, [&](auto k) -> int {
-        decltype(k)::launch(plain, grid, smem, stream, t, st, pl, a, round, kind);
+        decltype(k)::launch(plain, grid, smem, stream, t, st, pl, a, round, kind, pdl);
         return 0;
     });
     return cudaGetLastError();

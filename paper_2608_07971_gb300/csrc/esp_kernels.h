@@ -190,8 +190,10 @@ cudaError_t launch_apply_penalties(const DevTable &t, const double *values0, con
 cudaError_t launch_clear_marks(int32_t *units, int64_t n_opt, int R, cudaStream_t stream);
 cudaError_t launch_init(const DevTable &t, const DevState &st, const SolveArgs &a, const double *lambda0,
                         cudaStream_t stream);
+// pdl: launch as a programmatic dependent of the previous kernel on the stream (the pass stages its
+// first tiles before waiting for that kernel); only when the previous operation is a kernel.
 cudaError_t launch_pass(const DevTable &t, const DevState &st, const DevPlan &pl, const SolveArgs &a,
-                        int round, PassKind kind, int grid, cudaStream_t stream);
+                        int round, PassKind kind, int grid, cudaStream_t stream, bool pdl = false);
 cudaError_t launch_update(const DevTable &t, const DevState &st, const SolveArgs &a, int round,
                           cudaStream_t stream);
 // Dynamic shared memory of one resident CTA, and the clusters of the resident kernel that can be
