@@ -56,6 +56,11 @@ esp_status esp_debug_plan_runs(const int64_t *off, const int32_t *scen, const in
  * original layout (the segmented path) instead of the sorted one; 1 restores the default. */
 esp_status esp_debug_set_sorted_layout(esp_ctx *ctx, int32_t enable);
 
+/* Programmatic dependent launch of the evaluation passes (each pass stages its first tiles while the
+ * kernel before it finishes): mode -1 automatic (the library's choice per table), 0 off, 1 on. Takes
+ * effect from the next solve; results are the same either way. */
+esp_status esp_debug_set_pdl(esp_ctx *ctx, int32_t mode);
+
 /* Cluster size of the resident kernel (ESP_FLAG_RESIDENT) for the loaded table. force_cs: 0 keeps the
  * automatic choice; 1, 2, 4, 8 or 16 forces that many CTAs per scenario for later solves (the size must
  * fit the table). *cs receives the size solves use and *clusters how many such clusters the device

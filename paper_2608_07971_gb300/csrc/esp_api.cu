@@ -73,6 +73,7 @@ struct esp_ctx {
     int64_t *off = nullptr;
     // sorted layout of a general table (the evaluation pass reads it; outputs use jmap)
     bool sorted_enabled = ESP_SORTED_LAYOUT != 0;   // later loads build it (esp_debug_set_sorted_layout)
+    int pdl_mode = -1;   // programmatic dependent launch of the passes: -1 automatic, 0 off, 1 on
     bool sorted = false;
     int64_t s_n_opt = 0;
     int32_t *s_units = nullptr;
@@ -712,6 +713,14 @@ bool state_ready(const esp_ctx *c)
     return c->grid == 0 || (c->tiles && c->warp_begin && c->units && c->values && c->off);
 }
 
+// Whether the passes of this table are launched as programmatic dependents by default: measured
+// on GB300 it pays for large uniform tables (what-if batch: -1.2% per solve) and costs on others
+// (one 2048-job scenario: +10%; the ragged 16-scenario table: +12%), so only the former use it.
+bool pdl_default(const esp_ctx *c)
+{
+    return !c->placement && c->uniform_k > 0 && (int64_t)c->S * c->J >= (1 << 16);
+}
+
 // Queues one whole solve on the stream (captured into a graph when the stream allows it).
 esp_status enqueue_solve(esp_ctx *ctx, const esp_params *p, const DevState &st, bool has_l0)
 {
@@ -771,6 +780,9 @@ esp_status enqueue_solve(esp_ctx *ctx, const esp_params *p, const DevState &st, 
             e = cudaEventRecordWithFlags(e1, ctx->stream, rf);
         return e;
     };
+    // programmatic dependent launch of the passes (never with per-pass events, whose record nodes sit
+    // between the passes)
+    const bool pdl = !timed && (ctx->pdl_mode == 1 || (ctx->pdl_mode < 0 && pdl_default(ctx)));
     DevPlace pp = ctx->place;
     pp.scen_warps = fused ? ctx->scen_warps : nullptr;
     auto pass = [&](int r, PassKind kind) -> cudaError_t {
@@ -778,7 +790,7 @@ esp_status enqueue_solve(esp_ctx *ctx, const esp_params *p, const DevState &st, 
             return timed_launch([&]() { return launch_place(t, st, pp, a, r, kind, ctx->place_grid, ctx->stream); });
         // without per-pass events the previous operation is always a kernel: the pass overlaps its
         // start with that kernel's tail (programmatic dependent launch)
-        return timed_launch([&]() { return launch_pass(t, st, pl, a, r, kind, ctx->grid, ctx->stream, !timed); });
+        return timed_launch([&]() { return launch_pass(t, st, pl, a, r, kind, ctx->grid, ctx->stream, pdl); });
     };
     auto issue = [&]() -> cudaError_t {
         cudaError_t e = launch_init(t, st, a, has_l0 ? ctx->lambda0 : nullptr, ctx->stream);
@@ -1654,6 +1666,22 @@ esp_status esp_debug_set_sorted_layout(esp_ctx *ctx, int32_t enable)
     if (st != ESP_OK)
         return st;
     ctx->sorted_enabled = enable != 0;
+    return ESP_OK;
+}
+
+esp_status esp_debug_set_pdl(esp_ctx *ctx, int32_t mode)
+{
+    esp_status st = check_ctx(ctx);
+    if (st != ESP_OK)
+        return st;
+    if (mode < -1 || mode > 1)
+        return ESP_ERR_INVALID_ARG;
+    ctx->pdl_mode = mode;
+    if (ctx->gexec) {   // the graph holds the launches of the previous setting
+        cudaGraphExecDestroy(ctx->gexec);
+        ctx->gexec = nullptr;
+        ctx->gkey = GraphKey();
+    }
     return ESP_OK;
 }
 
