@@ -110,7 +110,7 @@ def measured_peak():
         return 6800.0, "fallback"
 
 
-PASS_KERNEL_SOURCES = ("esp_kernels.cu", "esp_device.cuh", "esp_common.h", "esp_kernels.h")
+PASS_KERNEL_SOURCES = ("esp_kernels.cu", "esp_warp.cuh", "esp_device.cuh", "esp_common.h", "esp_kernels.h")
 
 
 def pass_kernel_sha256() -> str:
