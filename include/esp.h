@@ -213,7 +213,7 @@ esp_status esp_load_placement(esp_ctx *ctx, int32_t S, int32_t J, int32_t KC, in
 /* The Gamma term of Eq. esp_score for later solves and evaluations. Option c of job j then scores
  *     rent - v + Gamma_j(c),   Gamma_j(c) = gamma0 * [c != c_cur[j]] + alpha * max(0, s_hat[o] - tau[j]),
  * the switching cost from the job's current configuration plus the interference penalty of the
- * predicted co-location slowdown above the job's tolerance (Sec. 3.2.2 and Sec. 3.3; Alg. 1 updates
+ * predicted co-location slowdown above the job's tolerance (Sec. 3.2.3 and Sec. 3.3; Alg. 1 updates
  * the slowdowns between ESP rounds). Gamma is computed in fp64 as (c != c_cur ? gamma0 : 0) +
  * alpha * max(0, s_hat - tau) and applied as the effective value v' = v - Gamma, one correctly
  * rounded operation per step; every output and objective (primal = sum of v') then refers to v'.

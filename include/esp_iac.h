@@ -1,10 +1,10 @@
 /*
- * esp_iac.h - C ABI of the IAC slowdown predictor (Sec. 3.4 of the paper, "Interference-Aware
+ * esp_iac.h - C ABI of the IAC slowdown predictor (Sec. 3.3 of the paper, "Interference-Aware
  * Co-location") on one GB300 (sm_103a): batched inference of the three-layer network of
- * Sec. 3.4.2 over co-location pairs, producing the predicted slowdowns S_hat that feed the
+ * Sec. 3.3.2 over co-location pairs, producing the predicted slowdowns S_hat that feed the
  * interference penalty of Eq. esp_score (esp_set_penalties in esp.h).
  *
- * Per-job features (Sec. 3.4.1), 14 fp32 per row, in this order:
+ * Per-job features (Sec. 3.3.1), 14 fp32 per row, in this order:
  *    0 SM Active (fraction of cycles)   1 SM Occupancy   2 DRAM Active   3 Framebuffer Used (MB)
  *    4 Tensor Core Active   5 workload type (0 training, 1 inference)   6 log-scaled parameter count
  *    7 isolated throughput T_j(c)   8 micro-batch size   9 activation checkpointing flag

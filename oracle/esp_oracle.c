@@ -251,7 +251,7 @@ double esp_oracle_adaptive_threshold(double tau_base, double beta, double util, 
     return tau_base + add;
 }
 
-/* Gamma of Eq. esp_score (Sec. 3.2.2): switching cost and interference penalty. */
+/* Gamma of Eq. esp_score (Sec. 3.2.3): switching cost and interference penalty. */
 double esp_oracle_penalty(int32_t c, int32_t c_cur, double gamma0, double alpha, double s_hat, double tau)
 {
     const double sw = (c_cur >= 0 && c != c_cur) ? gamma0 : 0.0;

@@ -1,10 +1,10 @@
-"""Oracle of the IAC interference predictor (Sec. 3.4): the 36-dimensional pair feature vector of
-Sec. 3.4.1 and the three-layer network of Sec. 3.4.2 / Eq. dnn_pred, in numpy fp64.
+"""Oracle of the IAC interference predictor (Sec. 3.3): the 36-dimensional pair feature vector of
+Sec. 3.3.1 and the three-layer network of Sec. 3.3.2 / Eq. dnn_pred, in numpy fp64.
 
 TEST INFRASTRUCTURE: only tests/, __graft_entry__.smoke() and bench.py's CPU-baseline and reference
 legs may import this module. It imports nothing from the library under paper_2608_07971_gb300/.
 
-Per-job features, in this order (Sec. 3.4.1; 14 = 5 hardware + 3 common + 3 training + 3 inference):
+Per-job features, in this order (Sec. 3.3.1; 14 = 5 hardware + 3 common + 3 training + 3 inference):
    0 SM Active        1 SM Occupancy     2 DRAM Active      3 Framebuffer Used (MB)   4 Tensor Core Active
    5 workload type (0 training, 1 inference)    6 log-scaled parameter count    7 isolated throughput T_j(c)
    8 micro-batch size   9 activation checkpointing flag   10 mixed-precision flag
@@ -12,7 +12,7 @@ Per-job features, in this order (Sec. 3.4.1; 14 = 5 hardware + 3 common + 3 trai
 A training job's inference slots and an inference job's training slots hold 0.
 
 Pair (i, j), predicting the slowdown of i next to j: x[0:14] = f_i, x[14:28] = f_j, then the 8 pairwise
-features (Sec. 3.4.1):
+features (Sec. 3.3.1):
   28-31 the mean over the two jobs of SM Active, SM Occupancy, DRAM Active, Tensor Core Active
   32    co-location type: type_i + type_j (0 training-training, 1 training-inference, 2 inference-inference)
   33    memory pressure (fb_i + fb_j) / C_mem
@@ -23,7 +23,7 @@ means are taken over the four utilization metrics (fractions of cycles), the fra
 through the memory pressure ratio, which gives the stated 36. A zero SM Active (undefined ratios)
 takes the values above.
 
-Network (Sec. 3.4.2, inference mode: dropout is the identity, Batch Normalization uses its running
+Network (Sec. 3.3.2, inference mode: dropout is the identity, Batch Normalization uses its running
 statistics):  h1 = ReLU(BN1(W1 x + b1)),  h2 = ReLU(BN2(W2 h1 + b2)),  S_hat = 1 + ReLU(W3 h2 + b3)
 (Eq. dnn_pred), BN(z) = gamma (z - mean) / sqrt(var + eps) + beta per unit. Parameters are given in
 fp32 (as a trained model stores them) and used exactly, converted to fp64.
@@ -64,7 +64,7 @@ class IacModel:
 
 
 def pair_features(f_i: np.ndarray, f_j: np.ndarray, c_mem: float) -> np.ndarray:
-    """The 36 features of the pair (i, j) (Sec. 3.4.1), fp64."""
+    """The 36 features of the pair (i, j) (Sec. 3.3.1), fp64."""
     a = np.asarray(f_i, dtype=np.float64)
     b = np.asarray(f_j, dtype=np.float64)
     x = np.zeros(N_FEAT)

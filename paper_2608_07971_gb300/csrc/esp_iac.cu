@@ -1,5 +1,5 @@
-// IAC slowdown predictor (include/esp_iac.h): the pair features of Sec. 3.4.1 and the three-layer
-// network of Sec. 3.4.2 / Eq. dnn_pred, batched over co-location pairs.
+// IAC slowdown predictor (include/esp_iac.h): the pair features of Sec. 3.3.1 and the three-layer
+// network of Sec. 3.3.2 / Eq. dnn_pred, batched over co-location pairs.
 //
 // Two kernels compute it. k_iac_tc (the default) runs the hidden layers on the tensor cores
 // (esp_iac_tc.cuh). k_iac is the CUDA-core kernel: one thread per pair. The folded parameters (at most 64 hidden units: 6,593 fp32, 26 KB) travel
@@ -321,7 +321,7 @@ __global__ void __launch_bounds__(iac_tc::kThreads, 1) k_iac_tc(const __grid_con
     fetch_pair(cur, ((int64_t)blockIdx.x * kWG + wg) * kM + row, n_pairs, pairs, jf, n_rows);
     for (int64_t tile = (int64_t)blockIdx.x * kWG + wg; tile * kM < n_pairs; tile += tile_stride) {
         const int64_t p = tile * kM + row;
-        // ---- the pair's 36 inputs (Sec. 3.4.1), zero for a pair past the end or out of range
+        // ---- the pair's 36 inputs (Sec. 3.3.1), zero for a pair past the end or out of range
         float x[kK1];
 #pragma unroll
         for (int q = 0; q < kFeat / 2; ++q) {

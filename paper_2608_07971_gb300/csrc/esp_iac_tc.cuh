@@ -1,4 +1,4 @@
-// Tensor-core path of the IAC predictor (Sec. 3.4.2, Eq. dnn_pred): the two hidden layers as
+// Tensor-core path of the IAC predictor (Sec. 3.3.2, Eq. dnn_pred): the two hidden layers as
 // tcgen05 MMAs (kind::tf32, accumulators in tensor memory) with a three-term split that keeps
 // fp32-level accuracy.
 //

@@ -357,10 +357,10 @@ def heavy_tail(scenarios: Optional[Sequence[int]] = None, J: int = 65536) -> Wor
     return Workload("heavy_tail", t, eta0=0.02, rounds=1000, seed=seed)
 
 
-# ---- IAC co-location pairs (Sec. 3.4.1) ---------------------------------------------------------
+# ---- IAC co-location pairs (Sec. 3.3.1) ---------------------------------------------------------
 #
 # Profile rows of 14 features per (job, configuration), row index j*K + k, in the order of
-# Sec. 3.4.1: SM Active, SM Occupancy, DRAM Active, Framebuffer Used (MB), Tensor Core Active,
+# Sec. 3.3.1: SM Active, SM Occupancy, DRAM Active, Framebuffer Used (MB), Tensor Core Active,
 # workload type (0 training, 1 inference), log-scaled parameter count, isolated throughput,
 # micro-batch, checkpointing flag, mixed-precision flag, ISL, OSL, prefix caching ratio. The
 # paper's profiled co-location experiments are not available; these draws give each feature a

@@ -1,4 +1,4 @@
-"""Pins of the IAC oracle (Sec. 3.4.1 features, Sec. 3.4.2 network and Eq. dnn_pred) against what
+"""Pins of the IAC oracle (Sec. 3.3.1 features, Sec. 3.3.2 network and Eq. dnn_pred) against what
 does not come from the oracle itself: the hand-worked dyadic example in tests/golden/iac_hand.json,
 PyTorch's own Linear / BatchNorm1d (eval) / ReLU / Dropout (eval) layers in fp64, and the invariants
 S_hat >= 1 and the symmetry of the pairwise block. Every check takes the oracle module as an

@@ -1,5 +1,5 @@
 """The outer ESP-IAC loop of Alg. 1 on the GPU: warm-started tatonnement, the IAC predictor's
-slowdowns for every option against its co-located partner's current configuration (Sec. 3.4,
+slowdowns for every option against its co-located partner's current configuration (Sec. 3.3,
 Eq. dnn_pred), the adaptive thresholds (Eq. adaptive_threshold) and the Gamma term of Eq.
 esp_score set for the next round (esp_set_penalties). Every outer round is compared with the oracle
 running the same loop on the same predicted slowdowns: selections and prices bit-exact. The
