@@ -61,6 +61,7 @@ struct esp_ctx {
     bool solved = false;
 
     int32_t S = 0, J = 0, R = 0, P = 0, rg = 0, n_groups = 0;
+    int64_t max_k = 0;   // largest option count of the loaded table
     int64_t n_opt = 0;
     int32_t small_units = 0;
     PlanCache pc;
@@ -499,7 +500,8 @@ esp_status load_common(esp_ctx *ctx, int32_t S, int32_t J, int32_t R, int32_t P,
         release_table(ctx);
         return ESP_ERR_INVALID_ARG;
     }
-    ESP_CUDA(launch_mark_duplicates(t, ctx->units, ctx->stats + 1, ctx->stream));
+    ctx->max_k = max_k;
+    ESP_CUDA(launch_mark_duplicates(t, ctx->units, ctx->stats + 1, ctx->stream, max_k));
 
     // plan the evaluation pass
     ctx->uniform_k = (!grouped && min_k == max_k && max_k <= 32 && (max_k & (max_k - 1)) == 0) ? (int32_t)max_k : 0;
@@ -1389,7 +1391,7 @@ esp_status refresh_after_values(esp_ctx *ctx, unsigned int *vflags)
     ESP_CUDA(cudaMemsetAsync(ctx->valflags, 0, sizeof(unsigned int), ctx->stream));
     ESP_CUDA(launch_validate(t, ctx->vmax, ctx->umax, ctx->valflags, ctx->stream));
     ESP_CUDA(cudaMemsetAsync(ctx->stats + 1, 0, sizeof(unsigned long long), ctx->stream));
-    ESP_CUDA(launch_mark_duplicates(t, ctx->units, ctx->stats + 1, ctx->stream));
+    ESP_CUDA(launch_mark_duplicates(t, ctx->units, ctx->stats + 1, ctx->stream, ctx->max_k));
     if (ctx->sorted)
         ESP_CUDA(launch_gather_sorted(t, pass_table(ctx), ctx->s_units, ctx->s_values, ctx->stream));
     ESP_CUDA(cudaMemcpyAsync(vflags, ctx->valflags, sizeof(unsigned int), cudaMemcpyDeviceToHost, ctx->stream));

@@ -175,7 +175,9 @@ cudaError_t launch_validate(const DevTable &t, double *vmax, int32_t *umax, unsi
                             cudaStream_t stream);
 // Marks every option that repeats an earlier option of its job (units, value and group equal) by
 // setting the sign bit of its column-0 unit in `units` (the device copy of t.units).
-cudaError_t launch_mark_duplicates(const DevTable &t, int32_t *units, unsigned long long *marked, cudaStream_t stream);
+// max_k: the table's largest option count (jobs above 1024 options stay unmarked).
+cudaError_t launch_mark_duplicates(const DevTable &t, int32_t *units, unsigned long long *marked, cudaStream_t stream,
+                                   int64_t max_k);
 
 // Fills the sorted layout of a general table: job j of `sorted` (offsets sorted.job_off, original
 // job sorted.jmap[j]) receives the options of that original job of `orig`, followed by padding
