@@ -75,6 +75,7 @@ struct esp_ctx {
     // sorted layout of a general table (the evaluation pass reads it; outputs use jmap)
     bool sorted_enabled = ESP_SORTED_LAYOUT != 0;   // later loads build it (esp_debug_set_sorted_layout)
     int pdl_mode = -1;   // programmatic dependent launch of the passes: -1 automatic, 0 off, 1 on
+    bool res_planned = false;   // resident options planned for the loaded table
     bool sorted = false;
     int64_t s_n_opt = 0;
     int32_t *s_units = nullptr;
@@ -586,61 +587,8 @@ esp_status load_common(esp_ctx *ctx, int32_t S, int32_t J, int32_t R, int32_t P,
     ESP_CUDA(cudaMemcpyAsync(ctx->warp_begin, plan.warp_begin.data(), plan.warp_begin.size() * sizeof(int32_t),
                              cudaMemcpyHostToDevice, ctx->stream));
 
-    // resident kernel: every cluster size whose slices fit one CTA's shared memory
-    if (!grouped && J >= 1) {
-        int optin = 0;
-        ESP_CUDA(cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, ctx->device));
-        const int32_t rk = (min_k == max_k) ? (int32_t)max_k : 0;
-        std::vector<ResShape> shapes;
-        for (int32_t cs = 1; cs <= kResMaxCluster; cs *= 2) {
-            ResShape sh;
-            if (!plan_resident(off_host, S, J, cs, sh) || sh.n_max > (1 << 24))
-                continue;
-            esp_ctx::ResOption o;
-            o.plan.cs = cs;
-            o.plan.k = rk;
-            o.plan.m_pad = (sh.m_max + 31) & ~31;
-            o.plan.n_cap = (sh.n_max + 1) & ~1LL;
-            o.smem = res_smem_bytes(R, o.plan);
-            o.n_max = sh.n_max;
-            if (o.smem > optin)
-                continue;
-            int nc = 0;
-            ESP_CUDA(res_max_clusters(dev_table(ctx), o.plan, ctx->small_units != 0, &nc));
-            if (nc < 1)
-                continue;
-            o.clusters = nc;
-            ctx->res.push_back(o);
-            shapes.push_back(std::move(sh));
-        }
-        if (!ctx->res.empty()) {
-            size_t total = 0;
-            for (const ResShape &sh : shapes)
-                total += sh.cuts.size();
-            ALLOC(ctx->res_cuts, total);
-            size_t at = 0;
-            for (size_t i = 0; i < shapes.size(); ++i) {
-                ESP_CUDA(cudaMemcpyAsync(ctx->res_cuts + at, shapes[i].cuts.data(), shapes[i].cuts.size() * sizeof(int32_t),
-                                         cudaMemcpyHostToDevice, ctx->stream));
-                ctx->res[i].plan.cuts = ctx->res_cuts + at;
-                at += shapes[i].cuts.size();
-            }
-            ESP_CUDA(cudaStreamSynchronize(ctx->stream));
-            // automatic size: most scenario-rounds per microsecond under a simple cost model, a fixed
-            // cost per round (barriers and the price update; smaller without a cluster) plus the
-            // slice's options at the SM's screening rate; ties keep the smaller cluster
-            double best = -1.0;
-            for (size_t i = 0; i < ctx->res.size(); ++i) {
-                const esp_ctx::ResOption &o = ctx->res[i];
-                const double round_us = (o.plan.cs == 1 ? 0.6 : 1.0) + 7.8e-5 * (double)o.n_max;
-                const double rate = (double)std::min<int64_t>(S, o.clusters) / round_us;
-                if (rate > best * 1.02) {
-                    best = rate;
-                    ctx->res_auto = (int)i;
-                }
-            }
-        }
-    }
+    // the resident kernel's options are planned on first use (plan_resident_options)
+    ctx->res_planned = false;
 
 #undef ALLOC
     if ((st = alloc_solve_state(ctx)) != ESP_OK) {
@@ -715,6 +663,79 @@ bool state_ready(const esp_ctx *c)
     return c->grid == 0 || (c->tiles && c->warp_begin && c->units && c->values && c->off);
 }
 
+// Options of the cluster-resident kernel (ESP_FLAG_RESIDENT) for the loaded table: every cluster
+// size whose slices fit one CTA's shared memory, with the automatic choice. Planned on first use
+// (not every load needs them), from the host copy of the offsets kept with the plan.
+esp_status plan_resident_options(esp_ctx *ctx)
+{
+    if (ctx->res_planned)
+        return ESP_OK;
+    ctx->res_planned = true;
+    ctx->res.clear();
+    ctx->res_auto = -1;
+    const int32_t S = ctx->S, J = ctx->J, R = ctx->R;
+    esp_status st = ESP_OK;
+    if (!ctx->pc.valid || (int64_t)ctx->pc.off.size() != (int64_t)S * J + 1)
+        return ESP_OK;
+    if (ctx->group == nullptr && J >= 1) {
+        int optin = 0;
+        ESP_CUDA(cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, ctx->device));
+        const int32_t rk = (ctx->pc.min_k == ctx->pc.max_k) ? (int32_t)ctx->pc.max_k : 0;
+        std::vector<ResShape> shapes;
+        for (int32_t cs = 1; cs <= kResMaxCluster; cs *= 2) {
+            ResShape sh;
+            if (!plan_resident(ctx->pc.off.data(), S, J, cs, sh) || sh.n_max > (1 << 24))
+                continue;
+            esp_ctx::ResOption o;
+            o.plan.cs = cs;
+            o.plan.k = rk;
+            o.plan.m_pad = (sh.m_max + 31) & ~31;
+            o.plan.n_cap = (sh.n_max + 1) & ~1LL;
+            o.smem = res_smem_bytes(R, o.plan);
+            o.n_max = sh.n_max;
+            if (o.smem > optin)
+                continue;
+            int nc = 0;
+            ESP_CUDA(res_max_clusters(dev_table(ctx), o.plan, ctx->small_units != 0, &nc));
+            if (nc < 1)
+                continue;
+            o.clusters = nc;
+            ctx->res.push_back(o);
+            shapes.push_back(std::move(sh));
+        }
+        if (!ctx->res.empty()) {
+            size_t total = 0;
+            for (const ResShape &sh : shapes)
+                total += sh.cuts.size();
+            if ((st = dev_alloc(ctx, &ctx->res_cuts, total)) != ESP_OK)
+                return st;
+            size_t at = 0;
+            for (size_t i = 0; i < shapes.size(); ++i) {
+                ESP_CUDA(cudaMemcpyAsync(ctx->res_cuts + at, shapes[i].cuts.data(), shapes[i].cuts.size() * sizeof(int32_t),
+                                         cudaMemcpyHostToDevice, ctx->stream));
+                ctx->res[i].plan.cuts = ctx->res_cuts + at;
+                at += shapes[i].cuts.size();
+            }
+            ESP_CUDA(cudaStreamSynchronize(ctx->stream));
+            // automatic size: most scenario-rounds per microsecond under a simple cost model, a fixed
+            // cost per round (barriers and the price update; smaller without a cluster) plus the
+            // slice's options at the SM's screening rate; ties keep the smaller cluster
+            double best = -1.0;
+            for (size_t i = 0; i < ctx->res.size(); ++i) {
+                const esp_ctx::ResOption &o = ctx->res[i];
+                const double round_us = (o.plan.cs == 1 ? 0.6 : 1.0) + 7.8e-5 * (double)o.n_max;
+                const double rate = (double)std::min<int64_t>(S, o.clusters) / round_us;
+                if (rate > best * 1.02) {
+                    best = rate;
+                    ctx->res_auto = (int)i;
+                }
+            }
+        }
+    }
+
+    return ESP_OK;
+}
+
 // Whether the passes of this table are launched as programmatic dependents by default: measured
 // on GB300 it pays for large uniform tables (what-if batch: -1.2% per solve) and costs on others
 // (one 2048-job scenario: +10%; the ragged 16-scenario table: +12%), so only the former use it.
@@ -754,6 +775,11 @@ esp_status enqueue_solve(esp_ctx *ctx, const esp_params *p, const DevState &st, 
     const bool use_graph = ctx->stream != nullptr;   // the legacy default stream cannot be captured
     std::vector<cudaEvent_t> &pool = use_graph ? ctx->graph_pool : ctx->ev_pool;
     size_t pool_used = use_graph ? 0 : ctx->ev_used;
+    if ((p->flags & ESP_FLAG_RESIDENT) && !ctx->placement) {
+        const esp_status rs = plan_resident_options(ctx);
+        if (rs != ESP_OK)
+            return rs;
+    }
     const int ri = (p->flags & ESP_FLAG_RESIDENT) && !ctx->placement
                        ? (ctx->res_force >= 0 ? ctx->res_force : ctx->res_auto)
                        : -1;
@@ -1574,6 +1600,8 @@ esp_status esp_debug_resident(esp_ctx *ctx, int32_t force_cs, int32_t *cs, int32
         return st;
     if (!ctx->loaded)
         return ESP_ERR_NOT_LOADED;
+    if (!ctx->placement && (st = plan_resident_options(ctx)) != ESP_OK)
+        return st;
     if (ctx->res.empty())
         return ESP_ERR_UNSUPPORTED;
     if (force_cs != 0) {
