@@ -311,3 +311,23 @@ def test_sorted_layout_equals_original_layout(case):
     sel, dem, ms = a.evaluate(lam)
     rsel, rdem, rms = oracle.best_response(t, 0, lam[0], oracle.NORMALIZED)
     assert np.array_equal(sel[0], rsel) and np.array_equal(dem[0], rdem) and np.array_equal(ms[0], rms)
+
+
+@pytest.mark.parametrize("graph", [True, False])
+def test_programmatic_dependent_launch_is_transparent(graph):
+    """Passes launched as programmatic dependents (forced on for a small table, where the default
+    keeps them off) give the oracle's solve, and the same bits as ordinary launches."""
+    import torch
+    t = W.whatif_batch(scenarios=[1, 4, 6], J=300).table
+    stream = torch.cuda.Stream() if graph else None
+    s = esp.Solver(t, stream=None if stream is None else stream.cuda_stream)
+    T = 30
+    sols = {}
+    for mode in (1, 0):
+        esp.esp_debug_set_pdl(s.ctx, mode)
+        sols[mode] = s.solve(0.02, T, traces=True)
+    check_solution(t, sols[1], [0, 1, 2], 0.02, T, esp.ESP_PRICE_NORMALIZED, esp.ESP_STEP_FIXED)
+    for f in ("lam", "sel", "demand", "lambda_trace", "demand_trace", "selhash_trace", "dual_trace"):
+        assert np.array_equal(getattr(sols[1], f), getattr(sols[0], f), equal_nan=True), f
+    esp.esp_debug_set_pdl(s.ctx, -1)
+    s.close()
