@@ -440,6 +440,7 @@ def run_ours(args):
                 "achieved": achieved, "peak": peak, "unit": "GB/s",
                 "frac": (achieved / peak) if achieved else None, "traffic": traffic,
                 "peak_kind": f"{peak_kind} hbm_gbs (copy)",
+                "frac_of_nominal_8tbs": (achieved / 8000.0) if achieved else None,
                 "bytes_per_launch": bytes_pass, "avg_launch_ms": pass_avg_ms, "launches_timed": n_pass,
                 "share_of_step": pass_ms / ms_ev if ms_ev else None,
                 "event_timed_ms_per_step": ms_ev,
