@@ -380,19 +380,17 @@ __global__ void __launch_bounds__(iac_tc::kThreads, 1) k_iac_tc(const __grid_con
 
         // ---- epilogue 1: h1 = ReLU(D1 + b1'), split into operand A of layer 2
         {
-            float v[32];
+            float v[64];   // both halves requested before one wait, so their latencies overlap
+            tmem_ld32(d1 | lane_sel, v);
+            tmem_ld32((d1 + 32) | lane_sel, v + 32);
+            tmem_wait_ld();
 #pragma unroll
-            for (int half = 0; half < 2; ++half) {
-                tmem_ld32((d1 + 32 * half) | lane_sel, v);
-                tmem_wait_ld();
-#pragma unroll
-                for (int c = 0; c < 8; ++c) {
-                    const int o = 32 * half + 4 * c;
-                    store_split4(a_hi, a_lo, cm_off(row, o, kK2), fmaxf(__fadd_rn(v[4 * c], ep.b1[o]), 0.0f),
-                                 fmaxf(__fadd_rn(v[4 * c + 1], ep.b1[o + 1]), 0.0f),
-                                 fmaxf(__fadd_rn(v[4 * c + 2], ep.b1[o + 2]), 0.0f),
-                                 fmaxf(__fadd_rn(v[4 * c + 3], ep.b1[o + 3]), 0.0f));
-                }
+            for (int c = 0; c < 16; ++c) {
+                const int o = 4 * c;
+                store_split4(a_hi, a_lo, cm_off(row, o, kK2), fmaxf(__fadd_rn(v[o], ep.b1[o]), 0.0f),
+                             fmaxf(__fadd_rn(v[o + 1], ep.b1[o + 1]), 0.0f),
+                             fmaxf(__fadd_rn(v[o + 2], ep.b1[o + 2]), 0.0f),
+                             fmaxf(__fadd_rn(v[o + 3], ep.b1[o + 3]), 0.0f));
             }
         }
         fence_async_smem();
@@ -424,17 +422,13 @@ __global__ void __launch_bounds__(iac_tc::kThreads, 1) k_iac_tc(const __grid_con
         // ---- epilogue 2: S_hat = 1 + ReLU(b3 + sum_o w3_o ReLU(D2_o + b2'_o)), o in order
         float y = ep.b3;
         {
-            float v[32];
+            float v[64];
+            tmem_ld32(d2 | lane_sel, v);
+            tmem_ld32((d2 + 32) | lane_sel, v + 32);
+            tmem_wait_ld();
 #pragma unroll
-            for (int half = 0; half < 2; ++half) {
-                tmem_ld32((d2 + 32 * half) | lane_sel, v);
-                tmem_wait_ld();
-#pragma unroll
-                for (int i = 0; i < 32; ++i) {
-                    const int o = 32 * half + i;
-                    y = __fmaf_rn(ep.w3[o], fmaxf(__fadd_rn(v[i], ep.b2[o]), 0.0f), y);
-                }
-            }
+            for (int o = 0; o < kN; ++o)
+                y = __fmaf_rn(ep.w3[o], fmaxf(__fadd_rn(v[o], ep.b2[o]), 0.0f), y);
         }
         if (p < n_pairs)
             out[p] = valid ? __fadd_rn(1.0f, fmaxf(y, 0.0f)) : __int_as_float(0x7fffffff);
