@@ -61,6 +61,11 @@ esp_status esp_debug_set_sorted_layout(esp_ctx *ctx, int32_t enable);
  * effect from the next solve; results are the same either way. */
 esp_status esp_debug_set_pdl(esp_ctx *ctx, int32_t mode);
 
+/* Warps of the evaluation pass planned by later loads, as a number of waves of resident CTAs
+ * (1..8; 0 = the library's choice, two waves): more waves give smaller warp ranges that the hardware
+ * schedules as CTAs finish. Results are the same for any setting. */
+esp_status esp_debug_set_plan_waves(esp_ctx *ctx, int32_t waves);
+
 /* Cluster size of the resident kernel (ESP_FLAG_RESIDENT) for the loaded table. force_cs: 0 keeps the
  * automatic choice; 1, 2, 4, 8 or 16 forces that many CTAs per scenario for later solves (the size must
  * fit the table). *cs receives the size solves use and *clusters how many such clusters the device
