@@ -55,7 +55,33 @@ def test_create_without_gpu_is_unsupported(lib):
 def test_null_context_rejected(lib):
     assert lib.esp_solve(None, None, None) == esp.ESP_ERR_INVALID_ARG
     assert lib.esp_get_prices(None, None) == esp.ESP_ERR_INVALID_ARG
+    assert lib.esp_debug_set_pdl(None, 1) == esp.ESP_ERR_INVALID_ARG
+    assert lib.esp_debug_set_plan_waves(None, 2) == esp.ESP_ERR_INVALID_ARG
+    assert lib.esp_load_placement(None, 1, 1, 1, 1, 2, 1, None, None, None, None, 1, None, None, None) \
+        == esp.ESP_ERR_INVALID_ARG
     lib.esp_destroy(None)
+
+
+def test_null_predictor_rejected(lib):
+    assert lib.esp_iac_create(None, -1, None) == esp.ESP_ERR_INVALID_ARG
+    assert lib.esp_iac_set_path(None, 0) == esp.ESP_ERR_INVALID_ARG
+    assert lib.esp_iac_synchronize(None) == esp.ESP_ERR_INVALID_ARG
+    assert lib.esp_iac_load_model(None, 8, None, None, None, None, None, None, None, 0.0, 1e-5) \
+        == esp.ESP_ERR_INVALID_ARG
+    assert lib.esp_iac_predict(None, 0, None, 0, None, 1.0, None) == esp.ESP_ERR_INVALID_ARG
+    assert lib.esp_iac_predict_host(None, 0, None, 0, None, 1.0, None) == esp.ESP_ERR_INVALID_ARG
+    n = ctypes.c_int64(5)
+    assert lib.esp_iac_last_launch_count(None, ctypes.byref(n)) == esp.ESP_ERR_INVALID_ARG
+    lib.esp_iac_destroy(None)
+
+
+def test_create_predictor_without_gpu_is_unsupported(lib):
+    import torch
+    if torch.cuda.is_available():
+        pytest.skip("a GPU is present")
+    h = ctypes.c_void_p()
+    assert lib.esp_iac_create(ctypes.byref(h), -1, None) == esp.ESP_ERR_UNSUPPORTED
+    assert h.value is None
 
 
 def tiles_cover(job_off, S, J, tiles, wb, tile_opt):
