@@ -90,3 +90,45 @@ def test_placement_structure():
     assert np.array_equal(t.units[:n, 6], t.units[:n, 0]) and np.array_equal(t.units[:n, 7], t.units[:n, 1])
     # the interference penalty is in [0, 1) and varies by node
     assert t.r_global == 6 and t.P == 134
+
+
+def test_iac_rows_ranges_and_job_level_fields():
+    J, K = 300, 16
+    f = W.iac_rows(6, J, K).astype(np.float64)
+    assert f.shape == (J * K, 14) and np.all(np.isfinite(f))
+    sm, occ, dram, fb, tc, typ = f[:, 0], f[:, 1], f[:, 2], f[:, 3], f[:, 4], f[:, 5]
+    assert np.all((sm >= 0.1) & (sm <= 1.0)) and np.all((occ > 0) & (occ <= sm))
+    assert np.all((dram >= 0.05) & (dram <= 0.9)) and np.all((tc >= 0) & (tc <= 0.9))
+    assert np.all((fb >= 2048) & (fb <= 78000))
+    rows = f.reshape(J, K, 14)
+    # type, parameter count, micro-batch, mixed precision, ISL and OSL are per job
+    for c in (5, 6, 8, 10, 11, 12):
+        assert np.all(rows[:, :, c] == rows[:, :1, c]), c
+    train = rows[:, 0, 5] == 0
+    assert 0.3 < train.mean() < 0.7
+    assert np.all(rows[train][:, :, 11:14] == 0) and np.all(rows[~train][:, :, 8:11] == 0)
+    assert np.array_equal(W.iac_rows(6, J, K), W.iac_rows(6, J, K))
+
+
+def test_iac_pairs_partners_and_scenario_subset():
+    S, J, K = 4, 50, 8
+    p = W.iac_pairs(6, S, J, K).reshape(S, J, K, 2)
+    assert np.all(p[..., 0] == (np.arange(J)[:, None] * K + np.arange(K)[None, :])[None])
+    partner_job, partner_cfg = p[..., 1] // K, p[..., 1] % K
+    assert np.all(partner_job != np.arange(J)[None, :, None])           # never the job itself
+    assert np.all(partner_job == partner_job[..., :1]) and np.all(partner_cfg == partner_cfg[..., :1])
+    assert np.all((p >= 0) & (p < J * K))
+    # the first scenarios of a larger batch are the smaller batch
+    assert np.array_equal(W.iac_pairs(6, 2, J, K), W.iac_pairs(6, S, J, K)[: 2 * J * K])
+
+
+def test_iac_model_shapes_and_scaling():
+    m = W.iac_model(6, 48)
+    assert m.W1.shape == (48, 36) and m.W2.shape == (48, 48) and m.W3.shape == (48,)
+    assert m.bn1.shape == (4, 48) and m.bn2.shape == (4, 48)
+    assert np.all(m.bn1[3] > 0) and np.all(m.bn2[3] > 0)       # running variances
+    for a in (m.W1, m.b1, m.bn1, m.W2, m.b2, m.bn2, m.W3):
+        assert a.dtype == np.float32 and np.all(np.isfinite(a))
+    # the first layer sees inputs of order one: W1 scaled by the inputs' spread
+    z = (W.IAC_INPUT_MEAN[None, :] + W.IAC_INPUT_STD[None, :]) @ m.W1.T.astype(np.float64) + m.b1
+    assert np.all(np.abs(z) < 20.0)
