@@ -240,10 +240,11 @@ esp_status esp_adaptive_threshold(int64_t n, const double *tau_base, double beta
 
 /* Effective capacity of Eq. effective_capacity (host only): for each of R resources
  *     c_eff[r] = floor(capacity[r] - gamma * sum over queued jobs q of min over q's options of units[o*R + r]),
- * at least 1 (a capacity must stay positive). The queue is a CSR table of Q jobs: q_offsets (Q + 1,
- * q_offsets[0] = 0, every job >= 1 option) and q_units (rows of R int32 >= 0). gamma in [0, 1]
- * reserves capacity for the queued jobs at their componentwise smallest footprint (Sec. 3.4).
- * Errors: ESP_ERR_INVALID_ARG. */
+ * at least 1 (a capacity must stay positive). capacity[r] lies in [1, 2^53] (exact in fp64). The queue
+ * is a CSR table of Q jobs: q_offsets (Q + 1, q_offsets[0] = 0, every job >= 1 option) and q_units
+ * (rows of R int32 >= 0). gamma in [0, 1] reserves capacity for the queued jobs at their componentwise
+ * smallest footprint (Sec. 3.4). Errors: ESP_ERR_INVALID_ARG (also for a capacity outside that range
+ * or a negative unit). */
 esp_status esp_effective_capacity(int32_t R, const int64_t *capacity, int32_t Q, const int64_t *q_offsets,
                                   const int32_t *q_units, double gamma, int64_t *c_eff);
 

@@ -5,6 +5,10 @@
 
 #include "esp.h"
 
+namespace {
+constexpr int64_t kMaxCapacity = (int64_t)1 << 53;
+}
+
 esp_status esp_adaptive_threshold(int64_t n, const double *tau_base, double beta, double util, double util_target,
                                   double beta_max, double *tau_out)
 {
@@ -27,6 +31,10 @@ esp_status esp_effective_capacity(int32_t R, const int64_t *capacity, int32_t Q,
         return ESP_ERR_INVALID_ARG;
     for (int32_t q = 0; q < Q; ++q)
         if (q_offsets[q + 1] <= q_offsets[q])
+            return ESP_ERR_INVALID_ARG;
+    // Capacities up to 2^53 convert to double exactly, so the floor below stays within int64.
+    for (int32_t r = 0; r < R; ++r)
+        if (capacity[r] < 1 || capacity[r] > kMaxCapacity)
             return ESP_ERR_INVALID_ARG;
     for (int32_t r = 0; r < R; ++r) {
         int64_t reserved = 0;

@@ -266,3 +266,11 @@ def test_host_formulas_match_the_oracle(lib):
                               oracle.effective_capacity(cap, q_off, q_units, gamma))
     with pytest.raises(esp.EspError):
         esp.esp_effective_capacity(cap, np.array([0, 0], np.int64), q_units, 0.5)   # an empty queued job
+    # capacities must be exact in fp64 (the floor then stays inside int64) and positive
+    edge = cap.copy()
+    edge[2] = 1 << 53
+    assert np.array_equal(esp.esp_effective_capacity(edge, q_off, q_units, 0.0), edge)
+    for bad in (0, -5, (1 << 53) + 1, np.iinfo(np.int64).max):
+        edge[2] = bad
+        with pytest.raises(esp.EspError):
+            esp.esp_effective_capacity(edge, q_off, q_units, 0.5)
