@@ -73,6 +73,14 @@ esp_status esp_debug_set_plan_waves(esp_ctx *ctx, int32_t waves);
  * ESP_ERR_INVALID_ARG: force_cs is not a size that fits. */
 esp_status esp_debug_resident(esp_ctx *ctx, int32_t force_cs, int32_t *cs, int32_t *clusters);
 
+/* Failure-detection hook of the grid-resident placement solve (the bounded grid barrier): the next
+ * esp_solve with ESP_FLAG_RESIDENT starts the barrier's arrival counter far short of its targets, so
+ * no CTA passes the first barrier. Every CTA's wait gives up after its time limit (4 s of the GPU's
+ * global timer) or when another CTA has given up; the solve returns ESP_ERR_TIMEOUT and the context
+ * answers ESP_ERR_STATE from then on (destroy it; the device stays usable). One solve only.
+ * ESP_ERR_UNSUPPORTED: no placement table is loaded, or it cannot run grid-resident. */
+esp_status esp_debug_hold_barrier(esp_ctx *ctx);
+
 #ifdef __cplusplus
 }
 #endif

@@ -24,10 +24,12 @@ struct GraphKey {
     const void *lt = nullptr, *dt = nullptr, *ht = nullptr, *gt = nullptr;
     bool has_l0 = false;
     int res = -1;   // resident option in use, -1: streaming
+    bool hold = false;
     bool operator==(const GraphKey &o) const
     {
         return eta0 == o.eta0 && tol == o.tol && step == o.step && mode == o.mode && T == o.T && flags == o.flags &&
-               lt == o.lt && dt == o.dt && ht == o.ht && gt == o.gt && has_l0 == o.has_l0 && res == o.res;
+               lt == o.lt && dt == o.dt && ht == o.ht && gt == o.gt && has_l0 == o.has_l0 && res == o.res &&
+               hold == o.hold;
     }
 };
 
@@ -92,6 +94,7 @@ struct esp_ctx {
     int32_t place_grid = 0;
     PlaceRes place_res = {};         // grid-resident placement solve (ESP_FLAG_RESIDENT), when allocated
     bool place_res_ok = false;
+    bool hold_barrier = false;       // test hook: the next grid-resident solve's barrier never completes
     uint16_t *group = nullptr;
     int64_t *cap = nullptr;
     double *vmax = nullptr;
@@ -791,6 +794,8 @@ esp_status enqueue_solve(esp_ctx *ctx, const esp_params *p, const DevState &st, 
     // fingerprint or dual trace is wanted (those need the per-round launches)
     const bool place_res = ctx->placement && (p->flags & ESP_FLAG_RESIDENT) && ctx->place_res_ok &&
                            st.hash_trace == nullptr && st.dual_trace == nullptr;
+    const bool hold = place_res && ctx->hold_barrier;
+    ctx->hold_barrier = false;
     auto timed_launch = [&](auto &&launch) -> cudaError_t {
         if (!timed)
             return launch();
@@ -829,7 +834,7 @@ esp_status enqueue_solve(esp_ctx *ctx, const esp_params *p, const DevState &st, 
         if (place_res) {
             if (e == cudaSuccess && T > 0)
                 e = timed_launch([&]() {
-                    return launch_place_res(t, st, pp, a, ctx->place_res, ctx->stream);
+                    return launch_place_res(t, st, pp, a, ctx->place_res, ctx->stream, hold);
                 });
             if (e == cudaSuccess)
                 e = pass(T, PASS_FINAL);
@@ -874,6 +879,7 @@ esp_status enqueue_solve(esp_ctx *ctx, const esp_params *p, const DevState &st, 
     key.gt = st.dual_trace;
     key.has_l0 = has_l0;
     key.res = place_res ? -2 : ri;
+    key.hold = hold;
 
     if (!use_graph) {
         ESP_CUDA(issue());
@@ -1727,6 +1733,17 @@ esp_status esp_debug_set_pdl(esp_ctx *ctx, int32_t mode)
         ctx->gexec = nullptr;
         ctx->gkey = GraphKey();
     }
+    return ESP_OK;
+}
+
+esp_status esp_debug_hold_barrier(esp_ctx *ctx)
+{
+    esp_status st = check_ctx(ctx);
+    if (st != ESP_OK)
+        return st;
+    if (!ctx->loaded || !ctx->placement || !ctx->place_res_ok)
+        return ESP_ERR_UNSUPPORTED;
+    ctx->hold_barrier = true;
     return ESP_OK;
 }
 

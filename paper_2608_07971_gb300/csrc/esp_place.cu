@@ -744,9 +744,13 @@ int place_res_ctas_per_sm(int S, int P, int KC, int R)
 }
 
 cudaError_t launch_place_res(const DevTable &t, const DevState &st, const DevPlace &pl, const SolveArgs &a,
-                             const PlaceRes &pr, cudaStream_t stream)
+                             const PlaceRes &pr, cudaStream_t stream, bool hold_barrier)
 {
     cudaError_t e = cudaMemsetAsync(pr.bar, 0, 2 * sizeof(unsigned int), stream);
+    // held: the arrival counter starts at 0xC0C0C0C0, about 2^30 arrivals short of any target the
+    // kernel waits for, so no CTA passes the first barrier and every wait runs out
+    if (e == cudaSuccess && hold_barrier)
+        e = cudaMemsetAsync(pr.bar, 0xC0, sizeof(unsigned int), stream);
     if (e == cudaSuccess)   // the last rounds of the previous solve leave demand in two buffers
         e = cudaMemsetAsync(pr.U3, 0, 3 * (size_t)t.S * t.P * sizeof(unsigned long long), stream);
     if (e != cudaSuccess)

@@ -29,6 +29,7 @@ EXPORTED = [
     "esp_evaluate", "esp_last_launch_count", "esp_pass_times", "esp_status_string", "esp_destroy",
     "esp_debug_tile_options", "esp_debug_plan", "esp_debug_stats", "esp_debug_resident",
     "esp_debug_sort_layout", "esp_debug_plan_runs", "esp_debug_set_sorted_layout", "esp_debug_set_pdl", "esp_debug_set_plan_waves",
+    "esp_debug_hold_barrier",
     "esp_evaluate_noalloc",
     "esp_set_penalties", "esp_adaptive_threshold", "esp_effective_capacity", "esp_load_placement",
     "esp_iac_create", "esp_iac_set_stream", "esp_iac_load_model", "esp_iac_predict", "esp_iac_predict_host",
@@ -96,6 +97,7 @@ def load_library(path: Optional[str] = None):
         "esp_debug_set_sorted_layout": ([vp, i32], st),
         "esp_debug_set_pdl": ([vp, i32], st),
         "esp_debug_set_plan_waves": ([vp, i32], st),
+        "esp_debug_hold_barrier": ([vp], st),
         "esp_set_penalties": ([vp, ctypes.c_double, vp, ctypes.c_double, vp, vp], st),
         "esp_load_placement": ([vp, i32, i32, i32, i32, i32, i32, vp, vp, vp, vp, i32, vp, vp, vp], st),
         "esp_adaptive_threshold": ([i64, vp, ctypes.c_double, ctypes.c_double, ctypes.c_double, ctypes.c_double, vp],
@@ -435,6 +437,12 @@ def plan_runs(off, scen, runk, S: int, J: int, tile_opt: int, max_warps: int):
 def esp_debug_set_plan_waves(ctx: int, waves: int) -> None:
     """Warps of the evaluation pass as this many waves of resident CTAs (0: the library's choice)."""
     _check(load_library().esp_debug_set_plan_waves(ctx, waves), "esp_debug_set_plan_waves")
+
+
+def esp_debug_hold_barrier(ctx: int) -> None:
+    """Test hook: the next grid-resident placement solve's barrier never completes, so it ends in
+    ESP_ERR_TIMEOUT and poisons the context (see include/esp_debug.h)."""
+    _check(load_library().esp_debug_hold_barrier(ctx), "esp_debug_hold_barrier")
 
 
 def esp_debug_set_pdl(ctx: int, mode: int) -> None:

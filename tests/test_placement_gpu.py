@@ -2,6 +2,7 @@
 without storing the expanded options equals the oracle's solve of the expanded table (and the
 streaming solve of that table) bit for bit."""
 
+import time
 import zlib
 
 import numpy as np
@@ -163,3 +164,32 @@ def test_grid_resident_placement_full_size():
     res = s.solve(w.eta0, w.rounds, flags=esp.ESP_FLAG_RESIDENT)
     assert s.launches() == 4
     same_solution(res, ref, fields=("lam", "sel", "demand"))
+
+
+def test_grid_barrier_timeout_is_reported_and_poisons_the_context():
+    """Failure detection of the grid-resident solve without a GPU fault: with the barrier held (its
+    arrival counter far short of every target, a count that nothing completes) each CTA's bounded
+    wait gives up, at its 4 s limit or on the abort word of the first CTA that gave up; the solve
+    returns ESP_ERR_TIMEOUT, the context answers ESP_ERR_STATE, and a new context on the same device
+    solves correctly."""
+    f = random_factors(zlib.crc32(b"resident"), S=3, J=97)    # 291 jobs: 19 CTAs share the barrier
+    s = esp.Solver()
+    s.load_placement(f)
+    ref = s.solve(0.05, 9)
+    esp.esp_debug_hold_barrier(s.ctx)
+    t0 = time.monotonic()
+    with pytest.raises(esp.EspError) as e:
+        s.solve(0.05, 9, flags=esp.ESP_FLAG_RESIDENT)
+    assert e.value.status == esp.ESP_ERR_TIMEOUT
+    assert time.monotonic() - t0 < 60
+    with pytest.raises(esp.EspError) as e:
+        s.solve(0.05, 9)
+    assert e.value.status == esp.ESP_ERR_STATE
+    s.close()
+    s2 = esp.Solver()
+    with pytest.raises(esp.EspError) as e:
+        esp.esp_debug_hold_barrier(s2.ctx)                       # nothing loaded
+    assert e.value.status == esp.ESP_ERR_UNSUPPORTED
+    s2.load_placement(f)
+    same_solution(s2.solve(0.05, 9, flags=esp.ESP_FLAG_RESIDENT), ref, fields=("lam", "sel", "demand"))
+    s2.close()
