@@ -14,7 +14,7 @@ import pytest
 import oracle
 from paper_2608_07971_gb300 import esp, workloads as W
 
-from tests.parity_util import MODES, STEPS, check_solution, rel_err  # noqa: F401
+from tests.parity_util import check_solution
 
 pytestmark = pytest.mark.gpu
 
