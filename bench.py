@@ -306,7 +306,6 @@ def run_reference(args):
     ot = oracle.OracleTable(t)
     lib = oracle.load()
     # one step = the oracle's full solve of a fixed number of scenarios, about 1-2 s of CPU work
-    per_scen = t.n_opt / t.S * (T + 1)
     t0 = time.perf_counter()
     oracle.solve_scenario(ot, 0, w.eta0, T, mode=w.mode, step=w.step, lib=lib)
     one = time.perf_counter() - t0

@@ -1,0 +1,53 @@
+"""bench.py's contract on the host (no GPU): the reference arm (the oracle as it stands, timed on the
+host cores) prints one JSON line with the same metric, unit and config keys as the GPU arm plus its
+cpu_baseline and e2e objects; under torchrun only rank 0 prints; and the GPU arm refuses to run
+without a GPU instead of falling back to the CPU."""
+
+import json
+import os
+import subprocess
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def run_bench(*args, env=None):
+    return subprocess.run([sys.executable, "bench.py", *args], cwd=ROOT, capture_output=True, text=True,
+                          timeout=600, env=dict(os.environ, **(env or {})))
+
+
+def test_reference_arm_prints_one_contract_line():
+    r = run_bench("--impl", "reference", "--workload", "tiny_cluster", "--steps", "2", "--warmup", "1")
+    assert r.returncode == 0, r.stderr[-2000:]
+    lines = [ln for ln in r.stdout.splitlines() if ln.startswith("{")]
+    assert len(lines) == 1
+    d = json.loads(lines[0])
+    assert d["impl"] == "reference"
+    assert d["metric"] == "option-evaluations/sec" and d["unit"] == "option-evals/s"
+    assert d["higher_is_better"] is True and d["n_gpus"] == 1 and d["steps"] == 2 and d["warmup"] == 1
+    assert d["value"] > 0 and d["ms_per_step"] > 0 and d["vs_baseline"] is None
+    assert d["config"]["workload"] == "tiny_cluster" and d["config"]["rounds"] == 200
+    cb = d["cpu_baseline"]
+    assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["value"] == d["value"] and cb["sample"]
+    e2e = d["e2e"]
+    assert e2e["value"] == d["value"] and e2e["unit"] == d["unit"]
+    assert e2e["h2d_bytes_per_step"] == 0 and e2e["d2h_bytes_per_step"] == 0
+
+
+def test_reference_arm_other_ranks_exit_without_work():
+    r = run_bench("--impl", "reference", "--workload", "tiny_cluster", "--steps", "1", "--warmup", "0",
+                  env={"RANK": "1", "WORLD_SIZE": "2", "LOCAL_RANK": "1"})
+    assert r.returncode == 0, r.stderr[-2000:]
+    assert not [ln for ln in r.stdout.splitlines() if ln.startswith("{")]
+
+
+def test_gpu_arm_refuses_to_run_without_a_gpu():
+    import torch
+    if torch.cuda.is_available():
+        pytest.skip("a GPU is present")
+    r = run_bench("--workload", "tiny_cluster", "--steps", "1", "--warmup", "0")
+    assert r.returncode != 0
+    assert "no CPU fallback" in r.stderr
+    assert not [ln for ln in r.stdout.splitlines() if ln.startswith("{")]
