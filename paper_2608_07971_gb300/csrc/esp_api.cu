@@ -11,6 +11,7 @@
 #include "esp.h"
 #include "esp_debug.h"
 #include "esp_kernels.h"
+#include "esp_place.h"
 #include "esp_plan.h"
 
 using namespace esp;
@@ -834,7 +835,8 @@ esp_status enqueue_solve(esp_ctx *ctx, const esp_params *p, const DevState &st, 
         if (place_res) {
             if (e == cudaSuccess && T > 0)
                 e = timed_launch([&]() {
-                    return launch_place_res(t, st, pp, a, ctx->place_res, ctx->stream, hold);
+                    return hold ? launch_place_res_held(t, st, pp, a, ctx->place_res, ctx->stream)
+                                : launch_place_res(t, st, pp, a, ctx->place_res, ctx->stream);
                 });
             if (e == cudaSuccess)
                 e = pass(T, PASS_FINAL);

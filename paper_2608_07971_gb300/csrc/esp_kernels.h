@@ -145,11 +145,9 @@ int place_res_smem_bytes(int S, int P, int KC, int R);
 int place_res_ctas_per_sm(int S, int P, int KC, int R);   // 0 if it cannot run
 
 // All rounds of a placement solve in one cooperative launch of pr.grid CTAs (at most one per SM).
-// Zeroes pr.bar and pr.U3 first. hold_barrier (a test hook) starts the barrier's arrival counter far
-// short of its targets instead, so that every CTA's bounded wait runs out and the solve reports a
-// timeout.
+// Zeroes pr.bar and pr.U3 first.
 cudaError_t launch_place_res(const DevTable &t, const DevState &st, const DevPlace &pl, const SolveArgs &a,
-                             const PlaceRes &pr, cudaStream_t stream, bool hold_barrier = false);
+                             const PlaceRes &pr, cudaStream_t stream);
 
 // Dynamic shared memory and resident CTAs per SM of the placement kernel (0 if it cannot run).
 int place_smem_bytes(int R, int P, int KC, int N, int NT);

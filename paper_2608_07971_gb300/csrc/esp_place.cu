@@ -9,6 +9,7 @@
 
 #include "esp_device.cuh"
 #include "esp_kernels.h"
+#include "esp_place.h"
 #include "esp_warp.cuh"
 
 namespace esp {
@@ -743,13 +744,11 @@ int place_res_ctas_per_sm(int S, int P, int KC, int R)
     return m;
 }
 
-cudaError_t launch_place_res(const DevTable &t, const DevState &st, const DevPlace &pl, const SolveArgs &a,
-                             const PlaceRes &pr, cudaStream_t stream, bool hold_barrier)
+static cudaError_t place_res_launch(const DevTable &t, const DevState &st, const DevPlace &pl, const SolveArgs &a,
+                                    const PlaceRes &pr, cudaStream_t stream, bool hold_barrier)
 {
     cudaError_t e = cudaMemsetAsync(pr.bar, 0, 2 * sizeof(unsigned int), stream);
-    // held: the arrival counter starts at 0xC0C0C0C0, about 2^30 arrivals short of any target the
-    // kernel waits for, so no CTA passes the first barrier and every wait runs out
-    if (e == cudaSuccess && hold_barrier)
+    if (e == cudaSuccess && hold_barrier)   // every byte 0xC0: the counter far short of its targets
         e = cudaMemsetAsync(pr.bar, 0xC0, sizeof(unsigned int), stream);
     if (e == cudaSuccess)   // the last rounds of the previous solve leave demand in two buffers
         e = cudaMemsetAsync(pr.U3, 0, 3 * (size_t)t.S * t.P * sizeof(unsigned long long), stream);
@@ -768,6 +767,18 @@ cudaError_t launch_place_res(const DevTable &t, const DevState &st, const DevPla
     if (t.R == 8)
         return cudaLaunchKernelEx(&cfg, k_place_res<8>, t, st, pl, a, pr);
     return cudaLaunchKernelEx(&cfg, k_place_res<0>, t, st, pl, a, pr);
+}
+
+cudaError_t launch_place_res(const DevTable &t, const DevState &st, const DevPlace &pl, const SolveArgs &a,
+                             const PlaceRes &pr, cudaStream_t stream)
+{
+    return place_res_launch(t, st, pl, a, pr, stream, false);
+}
+
+cudaError_t launch_place_res_held(const DevTable &t, const DevState &st, const DevPlace &pl, const SolveArgs &a,
+                                  const PlaceRes &pr, cudaStream_t stream)
+{
+    return place_res_launch(t, st, pl, a, pr, stream, true);
 }
 
 }  // namespace esp
