@@ -1,0 +1,211 @@
+"""The fp32 screen's error bound, checked on the CPU (no GPU).
+
+The evaluation kernels score every option first in fp32,
+    q = fma32(p32_{R-1}, u32_{R-1}, ... fma32(p32_0, u32_0, -v32)),
+with p32 the prices rounded to fp32, u32 the units converted to fp32 and v32 the value truncated to
+fp32 by integer operations (0 below 2^-100), and rely on |q - s| <= E for the fp64 reduced cost s
+of Eq. esp_score, with E = (4R + 16) 2^-24 M_s + 2^-99 computed per scenario from
+M_s = max|v| + sum_r max p_r max u_r and rounded up to fp32. Each step is restated here with exact
+IEEE single-precision rounding (an fp32 fused multiply-add is emulated through fp64 with an
+error-free sum, so ties are decided exactly), and E the way the scenario's warp computes it (lane
+terms, xor-butterfly sum in fp64). The distance to the exact rational value of s must stay within E
+less the fp64 chain's own rounding (R 2^-52 M), on typical, extreme and adversarial inputs."""
+
+import zlib
+from fractions import Fraction
+
+import numpy as np
+import pytest
+
+TWO = Fraction(2)
+
+
+def fma32(a, b, c):
+    """Correctly rounded fp32 a * b + c for fp32 arrays a, b, c (a * b is exact in fp64)."""
+    a, b, c = (np.asarray(x, np.float32).astype(np.float64) for x in (a, b, c))
+    t = a * b
+    s = t + c
+    bb = s - t
+    e = (t - (s - bb)) + (c - bb)              # t + c = s + e exactly
+    r = s.astype(np.float32)
+    rd = r.astype(np.float64)
+    up = np.nextafter(r, np.float32(np.inf)).astype(np.float64)
+    dn = np.nextafter(r, np.float32(-np.inf)).astype(np.float64)
+    # the only ambiguous case: s exactly halfway between two fp32 neighbours, e breaking the tie
+    mid_hi = (rd + up) / 2.0
+    mid_lo = (rd + dn) / 2.0
+    fix_up = (s == mid_hi) & (e > 0)
+    fix_dn = (s == mid_lo) & (e < 0)
+    out = r.copy()
+    out[fix_up] = up[fix_up].astype(np.float32)
+    out[fix_dn] = dn[fix_dn].astype(np.float32)
+    return out
+
+
+def v32_of(v):
+    """fp32 of v truncated toward zero (24-bit significand); 0 when |v| < 2^-100."""
+    bits = np.asarray(v, np.float64).view(np.uint64) & ~np.uint64((1 << 29) - 1)
+    t = bits.view(np.float64)
+    return np.where(np.abs(v) < 2.0 ** -100, 0.0, t).astype(np.float32)
+
+
+def screen(units, values, p64):
+    """q of every option (rows of units) at fp64 prices p64."""
+    p32 = p64.astype(np.float32)
+    q = -v32_of(values)
+    for r in range(units.shape[1]):
+        q = fma32(np.full(len(q), p32[r], np.float32), units[:, r].astype(np.float32), q)
+    return q
+
+
+def bound(units, values, p64):
+    """E of the scenario as its warp computes it: lane r's term p_r * max u_r, an xor-butterfly sum
+    over 32 lanes in fp64, M = max|v| + sum, then (4R + 16) 2^-24 M (1 + 2^-20) + 2^-99 rounded up
+    to fp32."""
+    R = units.shape[1]
+    x = np.zeros(32)
+    x[:R] = p64 * units.max(axis=0).astype(np.float64)
+    for d in (16, 8, 4, 2, 1):
+        x = x + x[np.arange(32) ^ d]
+    M = np.abs(values).max() + x[0]
+    eb = (4.0 * R + 16.0) * 2.0 ** -24 * M * (1.0 + 2.0 ** -20) + 2.0 ** -99
+    e32 = np.float32(eb)
+    if float(e32) < eb:
+        e32 = np.nextafter(e32, np.float32(np.inf))
+    return float(e32), M
+
+
+def exact_s(u_row, v, p64):
+    s = -Fraction(float(v))
+    for r in range(len(u_row)):
+        s += Fraction(float(p64[r])) * int(u_row[r])
+    return s
+
+
+def check(units, values, p64, sample=None):
+    """Largest |q - s| / (E - R 2^-52 M) over the options (at most `sample` of them, exactly)."""
+    q = screen(units, values, p64)
+    E, M = bound(units, values, p64)
+    R = units.shape[1]
+    budget = Fraction(E) - R * Fraction(M) * TWO ** -52
+    assert budget > 0
+    idx = np.arange(len(values)) if sample is None else np.random.default_rng(0).choice(len(values), sample, False)
+    worst = Fraction(0)
+    for i in idx:
+        d = abs(Fraction(float(q[i])) - exact_s(units[i], values[i], p64))
+        worst = max(worst, d / budget)
+    return float(worst)
+
+
+def test_fp32_fma_emulation_is_correctly_rounded():
+    """Against exact rationals on random operands and on exact halfway cases: (1 + 2^-23) * 1.5 has
+    25 significant bits, so it lies midway between two fp32 numbers; adding 0 leaves the tie to the
+    even neighbour, adding +-2^-60 (lost in the fp64 sum, kept in its error term) must round up or
+    down."""
+    rng = np.random.default_rng(1)
+    n = 4000
+    a = rng.standard_normal(n).astype(np.float32)
+    b = rng.integers(0, 1 << 24, n).astype(np.float32)
+    c = (rng.standard_normal(n) * 1e6).astype(np.float32)
+    c[:500] = -(a[:500].astype(np.float64) * b[:500].astype(np.float64)).astype(np.float32)   # cancellation
+    ties = np.float32(1.0 + 2.0 ** -23), np.float32(1.5)
+    a[500:530], b[500:530] = ties
+    c[500:510] = 0.0
+    c[510:520] = np.float32(2.0 ** -60)
+    c[520:530] = np.float32(-2.0 ** -60)
+    a[530:540], b[530:540] = -ties[0], ties[1]
+    c[530:540] = np.float32(2.0 ** -60)
+    got = fma32(a, b, c)
+    for i in range(n):
+        x = Fraction(float(a[i])) * Fraction(float(b[i])) + Fraction(float(c[i]))
+        f = float(x)
+        if Fraction(f) == x:
+            want = np.float32(f)                # exact in fp64: one rounding to fp32
+        else:                                   # the fp32 neighbours, nearest first
+            lo = np.float32(f)
+            cand = [np.nextafter(lo, np.float32(-np.inf)), lo, np.nextafter(lo, np.float32(np.inf))]
+            want = min(cand, key=lambda y: abs(Fraction(float(y)) - x))
+        assert got[i] == want, (i, a[i], b[i], c[i])
+    t = float(ties[0]) * 1.5                                           # exact in fp64
+    assert float(got[500]) == float(np.float32(t))                      # the tie, to even
+    assert float(got[510]) > t > float(got[520])                        # decided by the error term
+    assert float(got[510]) - float(got[520]) == 2.0 ** -23               # neighbours
+
+
+def test_value_truncation_and_range():
+    v = np.array([1.0, -1.0 - 2.0 ** -30, 3.141592653589793, 2.0 ** -100, 2.0 ** -101, -2.0 ** 100, 0.0])
+    got = v32_of(v)
+    assert got[0] == 1.0 and got[1] == -1.0 and got[3] == np.float32(2.0 ** -100) and got[4] == 0.0
+    assert abs(float(got[2]) - v[2]) < 2.0 ** -22 * v[2] and float(got[2]) <= v[2]
+    assert got[5] == np.float32(-2.0 ** 100) and got[6] == 0.0
+
+
+@pytest.mark.parametrize("case", ["whatif_like", "large_units", "values_near_2e100", "values_near_2em100",
+                                  "cancellation", "r16_mixed_scales", "r1", "subnormal_prices"])
+def test_screen_within_bound(case):
+    rng = np.random.default_rng(zlib.crc32(case.encode()))
+    n = 3000
+    if case == "whatif_like":
+        R = 6
+        units = rng.integers(0, 163841, (n, R)).astype(np.int64)
+        values = np.exp(rng.standard_normal(n))
+        p64 = rng.random(R) * 1e-5
+    elif case == "large_units":
+        R = 8
+        units = rng.integers((1 << 31) - (1 << 20), (1 << 31) - 1, (n, R)).astype(np.int64)
+        values = rng.random(n) * 1e9
+        p64 = rng.random(R) * 1e-3
+    elif case == "values_near_2e100":
+        R = 4
+        units = rng.integers(0, 1000, (n, R)).astype(np.int64)
+        values = (0.5 + 0.5 * rng.random(n)) * 2.0 ** 100
+        p64 = rng.random(R) * 2.0 ** 80
+    elif case == "values_near_2em100":
+        R = 4
+        units = rng.integers(0, 1000, (n, R)).astype(np.int64)
+        values = rng.random(n) * 2.0 ** -98
+        p64 = rng.random(R) * 2.0 ** -110
+    elif case == "cancellation":
+        # value equal to the rent up to a few ulps: q and s are tiny differences of large terms
+        R = 6
+        units = rng.integers(1, 1 << 22, (n, R)).astype(np.int64)
+        p64 = rng.random(R)
+        values = units.astype(np.float64) @ p64 * (1.0 + rng.standard_normal(n) * 1e-15)
+    elif case == "r16_mixed_scales":
+        R = 16
+        units = rng.integers(0, 1 << 24, (n, R)).astype(np.int64)
+        values = np.exp(rng.standard_normal(n) * 10)
+        p64 = np.exp(rng.standard_normal(R) * 8)
+    elif case == "r1":
+        R = 1
+        units = rng.integers(0, 1 << 31, (n, R)).astype(np.int64)
+        values = rng.random(n) * 1e6
+        p64 = np.array([rng.random() * 1e-3])
+    else:
+        R = 5
+        units = rng.integers(0, 1 << 20, (n, R)).astype(np.int64)
+        values = rng.random(n) * 2.0 ** -90
+        p64 = rng.random(R) * 2.0 ** -135      # fp32 subnormals
+    worst = check(units, values, p64)
+    assert worst <= 1.0, worst
+    assert worst <= 0.5 or case in ("cancellation", "values_near_2em100", "subnormal_prices"), worst
+
+
+def test_bound_is_reached_within_its_stated_margin():
+    """Errors aligned on purpose (R = 1): values whose truncation to fp32 drops almost a whole fp32
+    ulp (2^-23 |v|), prices just above a midpoint of the fp32 grid (rounded up by 2^-24 p), and a
+    rent p u equal to v to within p, so that both errors add with the same sign and the final
+    rounding is negligible: |q - s| is close to 3 2^-24 v. With M ~ 2 max v the ratio to
+    E = 20 2^-24 M is about 3/40 (0.066 measured), and the derivation's own worst case
+    (R + 4) 2^-24 M is 1/4 of E: a bound too small by a factor of 15 would fail here."""
+    rng = np.random.default_rng(7)
+    n = 3000
+    # values at the bottom of the binade [2^20, 2^21), where one fp32 ulp is 2^-23 |v|
+    mant = (rng.integers(0, 1 << 10, n).astype(np.uint64) << np.uint64(29)) | np.uint64((1 << 29) - 1)
+    values = ((np.uint64(1023 + 20) << np.uint64(52)) | mant).view(np.float64)
+    p32 = np.float32(1.0 + rng.integers(0, 1 << 23) * 2.0 ** -23)
+    p64 = np.array([float(p32) + 2.0 ** -24 + 2.0 ** -40])                             # rounds up
+    assert np.float32(p64[0]) == np.nextafter(p32, np.float32(2))
+    units = np.rint(values / p64[0]).astype(np.int64)[:, None]
+    worst = check(units, values, p64)
+    assert 0.05 <= worst <= 0.25, worst
