@@ -209,3 +209,57 @@ def test_bound_is_reached_within_its_stated_margin():
     units = np.rint(values / p64[0]).astype(np.int64)[:, None]
     worst = check(units, values, p64)
     assert 0.05 <= worst <= 0.25, worst
+
+
+def test_placement_screen_within_bound():
+    """The factored placement screen: the global columns of configuration k scored once,
+    g_k = chain over r < rg from -v32_k, then per node n the fp32 sum g_k + pen_n with
+    pen_n = fp32(sigma_j * D[a_j][b_n]) (one rounding more than a stored option), then the
+    node-priced columns. The fp64 score it must bound is the chain of the expanded option, from
+    v_kn = v_k - pen_n rounded to fp64. M takes |v_k| + |sigma_j| max D (1 + 2^-20) as the value
+    bound, and for each node-priced column the largest price over the nodes."""
+    rng = np.random.default_rng(11)
+    J, KC, N, R, rg, NT = 10, 12, 64, 8, 6, 8
+    units = rng.integers(0, 200000, (J, KC, R)).astype(np.int64)
+    values = np.exp(rng.standard_normal((J, KC)))
+    sens = (rng.random(J) * 0.5).astype(np.float32)
+    D = rng.beta(2, 8, (NT, NT)).astype(np.float32)
+    a = rng.integers(0, NT, J)
+    b = rng.integers(0, NT, N)
+    P = rg + (R - rg) * N
+    p64 = rng.random(P) * 1e-5
+    p32 = p64.astype(np.float32)
+    dmax = float(D.max())
+    vmax = max(float(np.abs(values[j]).max()) + abs(float(sens[j])) * dmax * (1.0 + 2.0 ** -20) for j in range(J))
+    umax = units.reshape(-1, R).max(axis=0).astype(np.float64)
+    x = np.zeros(32)
+    x[:rg] = p64[:rg] * umax[:rg]
+    for c2 in range(R - rg):
+        x[rg + c2] = p64[rg + c2::R - rg].max() * umax[rg + c2]
+    for d in (16, 8, 4, 2, 1):
+        x = x + x[np.arange(32) ^ d]
+    M = vmax + x[0]
+    eb = (4.0 * R + 16.0) * 2.0 ** -24 * M * (1.0 + 2.0 ** -20) + 2.0 ** -99
+    E = np.float32(eb)
+    if float(E) < eb:
+        E = np.nextafter(E, np.float32(np.inf))
+    budget = Fraction(float(E)) - R * Fraction(M) * TWO ** -52
+    worst = Fraction(0)
+    for j in range(J):
+        pen = (sens[j] * D[a[j], b]).astype(np.float32)                 # fp32 products, per node
+        for k in range(KC):
+            g = -v32_of(np.array([values[j, k]]))
+            for r in range(rg):
+                g = fma32(p32[r:r + 1], units[j, k, r:r + 1].astype(np.float32), g)
+            q = (np.full(N, g[0], np.float32) + pen).astype(np.float32)  # fp32 sum, one rounding
+            cols = [rg + (R - rg) * np.arange(N) + (r - rg) for r in range(rg, R)]
+            for i, r in enumerate(range(rg, R)):
+                q = fma32(p32[cols[i]], np.full(N, units[j, k, r], np.float32), q)
+            for n in range(N):
+                v_kn = float(values[j, k]) - float(pen[n])               # the expanded option's value
+                s = -Fraction(v_kn)
+                for r in range(R):
+                    col = r if r < rg else rg + (R - rg) * n + (r - rg)
+                    s += Fraction(float(p64[col])) * int(units[j, k, r])
+                worst = max(worst, abs(Fraction(float(q[n])) - s) / budget)
+    assert float(worst) <= 0.5, float(worst)
