@@ -263,3 +263,58 @@ def test_placement_screen_within_bound():
                     s += Fraction(float(p64[col])) * int(units[j, k, r])
                 worst = max(worst, abs(Fraction(float(q[n])) - s) / budget)
     assert float(worst) <= 0.5, float(worst)
+
+
+def ru32(x: Fraction) -> np.float32:
+    """The smallest fp32 number >= x."""
+    c = np.float32(float(x))
+    while Fraction(float(c)) < x:
+        c = np.nextafter(c, np.float32(np.inf))
+    while True:
+        d = np.nextafter(c, np.float32(-np.inf))
+        if Fraction(float(d)) >= x:
+            c = d
+        else:
+            return c
+
+
+def resident_bound(p64, umax, vmax, R):
+    """E of the cluster-resident kernel: every fp32 operation rounded up (p <= p32 (1 + 2^-23) +
+    2^-149, lane terms p_up * max u summed by a 16-lane xor butterfly, M = max|v| + sum, then
+    (4R + 16) 2^-24 M + 2^-99); returns 2E / 2."""
+    F = lambda v: Fraction(float(v))                                   # noqa: E731
+    p32 = p64.astype(np.float32)
+    terms = [np.float32(0.0)] * 16
+    for r in range(R):
+        p_up = ru32(F(ru32(F(p32[r]) * F(np.float32(1.0 + 2.0 ** -23)))) + TWO ** -149)
+        terms[r] = ru32(F(p_up) * F(ru32(Fraction(int(umax[r])))))
+    for d in (8, 4, 2, 1):
+        terms = [ru32(F(terms[i]) + F(terms[i ^ d])) for i in range(16)]
+    M = ru32(F(ru32(Fraction(float(vmax)))) + F(terms[0]))
+    coef = np.float32((4.0 * R + 16.0) * 2.0 ** -24)
+    return F(ru32(F(ru32(F(M) * F(coef))) + TWO ** -99))
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_bound_computations_never_undercut_the_exact_bound(seed):
+    """Both computed bounds (the streaming path's fp64 M with a (1 + 2^-20) factor, rounded up to
+    fp32 at the end; the resident path's fp32 arithmetic rounded up at every step) are at least the
+    exact (4R + 16) 2^-24 M + 2^-99 with M = max|v| + sum_r p_r max u_r in exact arithmetic."""
+    rng = np.random.default_rng(100 + seed)
+    checked = 0
+    for _ in range(50):
+        R = int(rng.integers(1, 17))
+        umax = rng.integers(0, 1 << 31, R) if seed % 2 else rng.integers(0, 1 << 18, R)
+        p64 = np.exp(rng.standard_normal(R) * (4 + 4 * seed)) * rng.random(R)
+        vmax = float(np.exp(rng.standard_normal() * (4 + 4 * seed)))
+        M = Fraction(vmax) + sum(Fraction(float(p64[r])) * int(umax[r]) for r in range(R))
+        if M > TWO ** 90:
+            continue
+        exact = (4 * R + 16) * TWO ** -24 * M + TWO ** -99
+        units = np.zeros((2, R), np.int64)
+        units[0] = umax
+        E_stream, _ = bound(units, np.array([vmax, 0.0]), p64)
+        assert Fraction(E_stream) >= exact
+        assert resident_bound(p64, umax, vmax, R) >= exact
+        checked += 1
+    assert checked >= 10
