@@ -97,6 +97,7 @@ def config_of(w: W.Workload, T: int) -> dict:
         "l2": "inputs larger than L2 (table %.2f GB vs 129 MB L2)" % (t.table_bytes() / 1e9)
         if t.table_bytes() > L2_BYTES else "table fits in L2 (latency-bound workload)",
         "evals_per_step": t.n_opt * (T + 1),
+        "table_sha256": t.digest(),
     }
 
 

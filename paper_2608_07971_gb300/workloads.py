@@ -110,6 +110,19 @@ class OptionTable:
         per = 4 * self.R + 8 + (2 if self.group is not None else 0)
         return self.n_opt * per
 
+    def digest(self) -> str:
+        """SHA-256 of the table: shape, then job offsets, units, values, group column and capacities
+        as little-endian bytes, so that two runs (or two arms of a benchmark) can show they read the
+        same synthetic table."""
+        import hashlib
+        h = hashlib.sha256()
+        h.update(np.asarray([self.S, self.J, self.R, self.P, self.r_global, self.group is not None], "<i8").tobytes())
+        for a, dt in ((self.job_off, "<i8"), (self.units, "<i4"), (self.values, "<f8"), (self.capacity, "<i8")):
+            h.update(np.ascontiguousarray(a, dt).tobytes())
+        if self.group is not None:
+            h.update(np.ascontiguousarray(self.group, "<u2").tobytes())
+        return h.hexdigest()
+
     def scenario(self, s: int) -> "OptionTable":
         """Scenario s alone, re-based to option index 0."""
         a, b = int(self.job_off[s * self.J]), int(self.job_off[(s + 1) * self.J])

@@ -29,6 +29,8 @@ def test_reference_arm_prints_one_contract_line():
     assert d["higher_is_better"] is True and d["n_gpus"] == 1 and d["steps"] == 2 and d["warmup"] == 1
     assert d["value"] > 0 and d["ms_per_step"] > 0 and d["vs_baseline"] is None
     assert d["config"]["workload"] == "tiny_cluster" and d["config"]["rounds"] == 200
+    from paper_2608_07971_gb300 import workloads as W
+    assert d["config"]["table_sha256"] == W.tiny_cluster().table.digest()
     cb = d["cpu_baseline"]
     assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["value"] == d["value"] and cb["sample"]
     e2e = d["e2e"]

@@ -132,3 +132,19 @@ def test_iac_model_shapes_and_scaling():
     # the first layer sees inputs of order one: W1 scaled by the inputs' spread
     z = (W.IAC_INPUT_MEAN[None, :] + W.IAC_INPUT_STD[None, :]) @ m.W1.T.astype(np.float64) + m.b1
     assert np.all(np.abs(z) < 20.0)
+
+
+def test_table_digest_identifies_the_table():
+    a = W.whatif_batch(scenarios=[0, 3], J=64).table
+    b = W.whatif_batch(scenarios=[0, 3], J=64).table
+    assert a.digest() == b.digest() and len(a.digest()) == 64
+    # a scenario drawn alone is the same table as that scenario cut from a batch
+    assert W.whatif_batch(scenarios=[3], J=64).table.digest() == a.scenario(1).digest()
+    units = a.units.copy()
+    units[5, 2] += 1
+    assert W.OptionTable(**{**a.__dict__, "units": units}).digest() != a.digest()
+    values = a.values.copy()
+    values[7] = np.nextafter(values[7], np.inf)
+    assert W.OptionTable(**{**a.__dict__, "values": values}).digest() != a.digest()
+    g = W.placement_expanded(scenarios=[0], J=8).table
+    assert g.group is not None and g.digest() != W.OptionTable(**{**g.__dict__, "group": g.group[::-1].copy()}).digest()
