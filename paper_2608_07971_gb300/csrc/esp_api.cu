@@ -715,8 +715,11 @@ esp_status plan_resident_options(esp_ctx *ctx)
             size_t total = 0;
             for (const ResShape &sh : shapes)
                 total += sh.cuts.size();
-            if ((st = dev_alloc(ctx, &ctx->res_cuts, total)) != ESP_OK)
+            if ((st = dev_alloc(ctx, &ctx->res_cuts, total)) != ESP_OK) {
+                ctx->res.clear();            // no option without its slices; a later solve plans again
+                ctx->res_planned = false;
                 return st;
+            }
             size_t at = 0;
             for (size_t i = 0; i < shapes.size(); ++i) {
                 ESP_CUDA(cudaMemcpyAsync(ctx->res_cuts + at, shapes[i].cuts.data(), shapes[i].cuts.size() * sizeof(int32_t),
