@@ -37,6 +37,11 @@ MUTANTS = {
     "penalty_added_to_value": ("values_out[o] = t->values[o] - gamma;", "values_out[o] = t->values[o] + gamma;"),
     "threshold_not_clamped": ("    if (add > beta_max)\n        add = beta_max;\n", ""),
     "capacity_largest_footprint": ("if (q_units[o * R + r] < m)", "if (q_units[o * R + r] > m)"),
+    "best_dual_tracks_largest": ("        if (g < best_dual)\n            best_dual = g;\n        if (dual_trace)\n            dual_trace[it] = g;",
+                                 "        if (g > best_dual || best_dual == INFINITY)\n            best_dual = g;\n        if (dual_trace)\n            dual_trace[it] = g;"),
+    "feasible_only_below_capacity": ("if (demand[k] > cap[k])", "if (demand[k] >= cap[k])"),
+    "stopping_scale_from_new_prices": ("if (fabs(lambda[k]) > scale)\n                    scale = fabs(lambda[k]);",
+                                       "if (fabs(next[k]) > scale)\n                    scale = fabs(next[k]);"),
 }
 
 
@@ -64,6 +69,7 @@ def pin_suite():
     yield pins.test_fixed_point_complementary_slackness
     yield pins.test_tolerance_stops_early_and_freezes
     yield pins.test_tolerance_rule_boundary_is_inclusive
+    yield pins.test_tolerance_scale_is_the_current_price
     yield pen.test_adaptive_threshold_closed_form
     yield pen.test_switching_cost_shifts_switch_price
     yield pen.test_interference_penalty_only_above_threshold

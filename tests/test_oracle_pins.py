@@ -397,3 +397,13 @@ def test_tolerance_rule_boundary_is_inclusive():
     assert sol.converged == 1 and sol.rounds_run == 1 and sol.lam[0] == 1.0 / 32
     sol = oracle.solve_scenario(t, 0, 1.0 / 256, 20, mode=oracle.RAW, tol=1.0 / 32 - 2**-40)
     assert sol.converged == 0 and sol.rounds_run == 20 and sol.lam[0] == 20.0 / 32
+
+
+def test_tolerance_scale_is_the_current_price():
+    # the stopping rule compares the move with tol * max(1, |lambda^t|), the prices before the
+    # update. Constant excess d = 2 at eta = 1/2 (raw): lambda^t = t, every move is 1. With tol = 1/8
+    # the move reaches the threshold once lambda^t = 8, so the update from 8 to 9 is the last (9
+    # updates); scaling by the new prices instead would stop one update earlier.
+    t = table_from_jobs([[(1.0, (12,))]], [10])
+    sol = oracle.solve_scenario(t, 0, 0.5, 50, mode=oracle.RAW, tol=0.125)
+    assert sol.converged == 1 and sol.rounds_run == 9 and sol.lam[0] == 9.0
