@@ -70,6 +70,8 @@ def pin_suite():
     yield pins.test_tolerance_stops_early_and_freezes
     yield pins.test_tolerance_rule_boundary_is_inclusive
     yield pins.test_tolerance_scale_is_the_current_price
+    yield pins.test_scenarios_are_independent
+    yield pins.test_warm_start_resumes_the_trajectory
     yield pen.test_adaptive_threshold_closed_form
     yield pen.test_switching_cost_shifts_switch_price
     yield pen.test_interference_penalty_only_above_threshold

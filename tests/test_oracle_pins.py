@@ -407,3 +407,47 @@ def test_tolerance_scale_is_the_current_price():
     t = table_from_jobs([[(1.0, (12,))]], [10])
     sol = oracle.solve_scenario(t, 0, 0.5, 50, mode=oracle.RAW, tol=0.125)
     assert sol.converged == 1 and sol.rounds_run == 9 and sol.lam[0] == 9.0
+
+
+def test_scenarios_are_independent():
+    """Scenario s of a batch solves exactly as the same scenario alone (offsets re-based to 0), with
+    capacities that differ between scenarios, so that any mistake in the per-scenario offsets of
+    the capacities, prices or options changes the result."""
+    rng = np.random.default_rng(61)
+    t = W.random_table(rng, S=3, J=25, R=3, kmin=1, kmax=6, cap_frac=0.5)
+    cap = t.capacity.copy()
+    cap[1] = cap[1] * 100                  # never binding: feasible
+    cap[2] = np.maximum(1, cap[2] // 3)
+    t = W.OptionTable(**{**t.__dict__, "capacity": cap})
+    flags = set()
+    for mode in (oracle.RAW, oracle.NORMALIZED):
+        eta = 0.002 if mode == oracle.RAW else 0.3
+        for s in range(t.S):
+            a = oracle.solve_scenario(t, s, eta, 30, mode=mode, traces=True)
+            b = oracle.solve_scenario(t.scenario(s), 0, eta, 30, mode=mode, traces=True)
+            for f in ("lam", "sel", "demand", "min_score", "lambda_trace", "demand_trace", "dual_trace"):
+                assert np.array_equal(getattr(a, f), getattr(b, f)), (mode, s, f)
+            assert (a.primal, a.dual, a.best_dual, a.feasible) == (b.primal, b.dual, b.best_dual, b.feasible)
+            assert a.feasible == int(np.all(a.demand <= cap[s]))
+            flags.add((s, a.feasible, int(np.all(a.demand <= cap[0]))))
+    # some scenario is feasible under its own capacities and not under scenario 0's, or the reverse
+    assert any(own != first for _, own, first in flags), flags
+    # the scenarios do differ
+    assert not np.array_equal(oracle.solve_scenario(t, 1, 0.3, 30).lam, oracle.solve_scenario(t, 2, 0.3, 30).lam)
+
+
+def test_warm_start_resumes_the_trajectory():
+    """With a fixed step, T1 updates followed by T2 more from the prices reached (lambda0) are the
+    trajectory of T1 + T2 updates; the solve's minimal reduced costs are those of a best response at
+    its final prices."""
+    rng = np.random.default_rng(62)
+    t = W.random_table(rng, S=1, J=30, R=4, kmin=1, kmax=7, cap_frac=0.4)
+    full = oracle.solve_scenario(t, 0, 0.25, 24, traces=True)
+    head = oracle.solve_scenario(t, 0, 0.25, 10)
+    tail = oracle.solve_scenario(t, 0, 0.25, 14, lambda0=head.lam, traces=True)
+    assert np.array_equal(tail.lam, full.lam) and np.array_equal(tail.sel, full.sel)
+    assert np.array_equal(tail.lambda_trace, full.lambda_trace[10:])
+    assert np.array_equal(tail.demand_trace, full.demand_trace[10:])
+    assert len(np.unique(full.lam)) > 1
+    sel, dem, ms = oracle.best_response(t, 0, full.lam)
+    assert np.array_equal(full.min_score, ms) and np.array_equal(full.sel, sel) and np.array_equal(full.demand, dem)
