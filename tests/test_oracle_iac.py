@@ -14,7 +14,7 @@ from oracle import iac_oracle
 
 GOLDEN = os.path.join(os.path.dirname(__file__), "golden", "iac_hand.json")
 PAIR_NAMES = {"a|b": ("a", "b"), "b|a": ("b", "a"), "a|a": ("a", "a"), "b|b": ("b", "b"),
-              "a|c": ("a", "c"), "c|c": ("c", "c")}
+              "a|c": ("a", "c"), "b|c": ("b", "c"), "c|c": ("c", "c")}
 
 
 def golden():

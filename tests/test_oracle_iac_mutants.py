@@ -25,6 +25,7 @@ MUTANTS = {
     "balance_zero_case": ("x[k + 2] = 1.0 if sm_hi == 0.0", "x[k + 2] = 0.0 if sm_hi == 0.0"),
     "intensity_inverted": ("f[DRAM_ACTIVE] / f[SM_ACTIVE]", "f[SM_ACTIVE] / max(f[DRAM_ACTIVE], 1e-300)"),
     "intensity_no_abs": ("abs(intensity(a) - intensity(b))", "(intensity(a) - intensity(b))"),
+    "intensity_zero_case": ("return 0.0 if f[SM_ACTIVE] == 0.0", "return 1.0 if f[SM_ACTIVE] == 0.0"),
     "pairwise_order": ("x[k + 2] = 1.0 if", "x[k + 3] = 1.0 if"),
     "bn_no_sqrt": ("np.sqrt(var + float(eps))", "(var + float(eps))"),
     "bn_no_eps": ("np.sqrt(var + float(eps))", "np.sqrt(var)"),
