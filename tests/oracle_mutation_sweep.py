@@ -8,7 +8,10 @@ either equivalent to the original (the change only matters at an equality where 
 give the same value, or for a sign of zero) or read or write out of bounds, which
 tests/test_host_sanitized.py reports when it runs the same pins under AddressSanitizer.
 
-    python -m tests.oracle_mutation_sweep [--child LIB]
+    python -m tests.oracle_mutation_sweep [--sanitize-survivors]
+
+With --sanitize-survivors every mutant that the pins miss is also run under the sanitizers, and the
+first report (or its absence) is printed beneath it.
 """
 
 from __future__ import annotations
@@ -54,6 +57,7 @@ def child(lib_path: str) -> int:
 def main() -> int:
     if len(sys.argv) == 3 and sys.argv[1] == "--child":
         return child(sys.argv[2])
+    sanitize = "--sanitize-survivors" in sys.argv
     sys.path.insert(0, ROOT)
     import oracle
     src_path = os.path.join(ROOT, "oracle", "esp_oracle.c")
@@ -77,9 +81,34 @@ def main() -> int:
         if not caught:
             survivors += 1
             print(f"not caught, line {i + 1}: {lines[i].strip()}  =>  {new_line.strip()}", flush=True)
+            if sanitize:
+                print("    sanitizers: " + sanitized_verdict(mutated, tmp, n), flush=True)
     shutil.rmtree(tmp, ignore_errors=True)
     print(f"{survivors} of {total} compiled mutants not caught by the pins")
     return 0
+
+
+def sanitized_verdict(mutated_lines, tmp, n):
+    """Runs the pins on the mutant built with AddressSanitizer and UndefinedBehaviorSanitizer (as
+    tests/test_host_sanitized.py does) and returns the first report, or says there was none."""
+    from tests import test_host_sanitized as san
+    rt = san._runtime("libasan.so")
+    if rt is None:
+        return "unavailable (no AddressSanitizer runtime)"
+    d = os.path.join(tmp, f"san{n}")
+    os.makedirs(d, exist_ok=True)
+    src = "\n".join(mutated_lines)
+    c = os.path.join(d, "esp_oracle.c")
+    open(c, "w").write(src)
+    shutil.copy(os.path.join(ROOT, "oracle", "esp_oracle.h"), d)
+    import oracle
+    so = os.path.join(d, "liboracle_san.so")
+    subprocess.check_call(["gcc", *oracle.CFLAGS, *san.SAN, c, "-o", so, "-lm"])
+    r = san.run_child(rt, so, os.path.join(d, "out.npz"), pins=True)
+    reports = [ln.strip() for ln in r.stderr.splitlines() if "ERROR: AddressSanitizer" in ln or "runtime error" in ln]
+    if r.returncode != 0 and reports:
+        return "reported: " + reports[0][:120]
+    return "no report (equivalent to the original, or undetected)"
 
 
 if __name__ == "__main__":
