@@ -9,7 +9,7 @@
 //   the tile plan of the table:            ok, n_tiles, n_warps, 6 fields per tile, warp_begin [n_warps + 1]
 //   the sorted layout:                     ok, then off [S*J + 1], jmap, scen, runk [S*J each]
 //   the tile plan of the sorted layout:    ok, n_tiles, n_warps, tiles, warp_begin (only after a sorted layout)
-//   the cluster-resident slices:           ok, m_max, n_max, cuts [S * (cs + 1)]
+//   the cluster-resident slices:           ok, m_max, n_max, n, cuts [n = S * (cs + 1)]
 // then: status, tau_out [n] (bit patterns); status, c_eff [R].
 // A plan that the planner accepts but its own check rejects exits with status 3.
 #include <cstdint>
@@ -134,6 +134,7 @@ int main(int argc, char **argv)
         if (res) {
             out.put(rs.m_max);
             out.put(rs.n_max);
+            out.put((int64_t)rs.cuts.size());
             for (int32_t v : rs.cuts)
                 out.put(v);
         }
