@@ -7,9 +7,12 @@ the final best response, for every scenario of the batch. `value` is measured wi
 resident in HBM; `e2e` repeats the step through the public API with host inputs (pinned), i.e. the
 upload, validation and planning of the table, the solve, and the read-back of selections and prices.
 
-Default workload: whatif_batch (1024 independent 512-GPU scenarios, J=2048, K=16, R=6, T=300).
-Multi-GPU (torchrun): every rank solves its own 1024 scenarios (weak scaling, no data-path collective).
---impl reference times the oracle (the plain single-threaded C restatement of the method) instead.
+Default workload: heavy_tail (16 scenarios of J=65536 jobs with K_j = min(256, Zipf 1.3) options,
+R=6, T=1000: 61.3 M options, 1.96 GB per round), the largest single-GPU configuration; whatif_batch
+(1024 independent 512-GPU scenarios, J=2048, K=16, R=6, T=300) is measured beside it as a keyed
+second line with its own roofline. Multi-GPU (torchrun): every rank solves its own block of
+scenarios (weak scaling, no data-path collective). --impl reference times the oracle (the plain
+single-threaded C restatement of the method) instead.
 """
 
 from __future__ import annotations
@@ -43,7 +46,9 @@ def parse_args():
     ap.add_argument("--steps", type=int, default=5)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", default="whatif_batch", choices=sorted(W.WORKLOADS))
+    ap.add_argument("--workload", default="heavy_tail", choices=sorted(W.WORKLOADS))
+    ap.add_argument("--second", default="whatif_batch",
+                    help="workload measured beside the main one as a keyed line ('none' to skip)")
     ap.add_argument("--rounds", type=int, default=None, help="override T (changes the workload)")
     ap.add_argument("--scenarios", type=int, default=None, help="override S (profiling of a smaller case)")
     ap.add_argument("--no-e2e", action="store_true")
@@ -111,7 +116,8 @@ def measured_peak():
         return 6800.0, "fallback"
 
 
-PASS_KERNEL_SOURCES = ("esp_kernels.cu", "esp_warp.cuh", "esp_device.cuh", "esp_common.h", "esp_kernels.h")
+PASS_KERNEL_SOURCES = ("esp_stream.cu", "esp_kernels.cu", "esp_tile.cuh", "esp_ptx.cuh", "esp_warp.cuh",
+                       "esp_device.cuh", "esp_common.h", "esp_kernels.h")
 
 
 def pass_kernel_sha256() -> str:
@@ -123,15 +129,15 @@ def pass_kernel_sha256() -> str:
     return h.hexdigest()
 
 
-def kernel_traffic(n_opt_launch: int):
-    """DRAM bytes per evaluation pass from the committed ncu summary, scaled to this workload's
-    option count, or None when the kernel source changed since the counters were taken."""
-    path = os.path.join(ROOT, "profiles", "k_pass_traffic.json")
+def kernel_traffic(workload: str, n_opt_launch: int):
+    """DRAM bytes per evaluation pass from the committed ncu summary of this workload's shape (a
+    smaller capture of the same table shape), scaled to this workload's option count, or None when
+    there is none or the kernel sources changed since the counters were taken."""
+    path = os.path.join(ROOT, "profiles", "pass_traffic.json")
     try:
         with open(path) as f:
-            rec = json.load(f)
-        sha = pass_kernel_sha256()
-        if rec.get("kernel_source_sha256") != sha:
+            rec = json.load(f)[workload]
+        if rec.get("kernel_source_sha256") != pass_kernel_sha256():
             return None
         return float(rec["dram_bytes_per_launch"]) / float(rec["options_per_launch"]) * n_opt_launch
     except Exception:
@@ -344,6 +350,134 @@ def run_reference(args):
     return 0
 
 
+def time_streaming(esp, solver, w, T, args, dist, barrier, stream, clk=None):
+    """Times args.steps whole solves of the loaded table (one CUDA graph each, CUDA events on the
+    library's stream), then the evaluation passes alone (separate solves with an event pair around
+    every pass). Returns the measured line: value, ms per step, roofline of the pass kernel."""
+    import torch
+    import contextlib
+    t = w.table
+    ctx = solver.ctx
+    prm = solver.params(w.eta0, T, mode=w.mode, step=w.step)
+    prm_ev = solver.params(w.eta0, T, mode=w.mode, step=w.step, flags=esp.ESP_FLAG_PASS_EVENTS)
+    for _ in range(args.warmup):
+        esp.esp_solve_async(ctx, prm)
+    stream.synchronize()
+    esp.esp_debug_stats(ctx, reset=True)
+    launches_per_step = esp.esp_last_launch_count(ctx)
+    barrier()
+    torch.cuda.synchronize()
+    ev0 = torch.cuda.Event(enable_timing=True)
+    ev1 = torch.cuda.Event(enable_timing=True)
+    with (clk if clk is not None else contextlib.nullcontext()):
+        ev0.record(stream)
+        for _ in range(args.steps):
+            esp.esp_solve_async(ctx, prm)
+        ev1.record(stream)
+        stream.synchronize()
+    torch.cuda.synchronize()
+    barrier()
+    ms = ev0.elapsed_time(ev1) / args.steps
+    res = np.zeros(t.S, esp.RESULT_DTYPE)
+    st = esp.esp_get_result(ctx, res)
+    assert np.all(res["rounds_run"] == T) or st != 0, "unexpected early stop"
+    n_res, n_marked = esp.esp_debug_stats(ctx, reset=True)
+    # the pass durations: solves with an event pair around every pass (the last solve's passes)
+    for _ in range(2):
+        esp.esp_solve_async(ctx, prm_ev)
+    stream.synchronize()
+    esp.esp_pass_times(ctx, reset=True)
+    ev0.record(stream)
+    esp.esp_solve_async(ctx, prm_ev)
+    ev1.record(stream)
+    stream.synchronize()
+    ms_ev = ev0.elapsed_time(ev1)
+    pass_ms, n_pass = esp.esp_pass_times(ctx, reset=True)
+
+    evals_step = t.n_opt * (T + 1)
+    value, step_s, _ = aggregate(dist, ms / 1e3, evals_step, device="cuda")
+    peak, peak_kind = measured_peak()
+    pass_avg_ms = pass_ms / max(n_pass, 1)
+    bytes_pass = t.table_bytes()
+    achieved = bytes_pass / (pass_avg_ms / 1e3) / 1e9 if n_pass else None
+    kind = {1: "k_stream (streaming pass: producer warp + consumer warps)", 0: "k_pass (per-warp pass)"}.get(
+        esp.esp_debug_pass_kernel(ctx), "k_place")
+    roofline = {"bound": "hbm", "kernel": kind + ": best response + demand aggregation + fused price update",
+                "achieved": achieved, "peak": peak, "unit": "GB/s",
+                "frac": (achieved / peak) if achieved else None, "traffic": kernel_traffic(w.name, t.n_opt),
+                "peak_kind": f"{peak_kind} hbm_gbs (copy)",
+                "frac_of_nominal_8tbs": (achieved / 8000.0) if achieved else None,
+                "bytes_per_launch": bytes_pass, "avg_launch_ms": pass_avg_ms, "launches_timed": n_pass,
+                "share_of_step": pass_ms / ms_ev if ms_ev else None,
+                "event_timed_ms_per_step": ms_ev,
+                "achieved_over_step": bytes_pass * (T + 1) / (ms / 1e3) / 1e9,
+                "exact_resolutions_per_pass": n_res / max(1, (args.warmup + args.steps) * (T + 1)),
+                "duplicates_marked": n_marked}
+    return {"value": value, "unit": "option-evals/s", "ms_per_step": step_s * 1e3,
+            "rounds_per_sec": T / step_s, "evals_per_step": evals_step, "roofline": roofline,
+            "launches_per_step": launches_per_step, "device_ms_last_solve": float(res["device_ms"][0])}
+
+
+def time_e2e(esp, solver, w, T, args, dist, barrier, stream, local):
+    """The step through the public API from pinned host buffers: every step uploads its table
+    (esp_load_options: copy, validation, planning, duplicate marks), solves it, and reads back the
+    selections and prices. Two contexts alternate so that step i+1's upload overlaps step i's solve
+    (esp_solve_async); every step still pays its own copies, inside the timed region."""
+    import torch
+    t = w.table
+    pin = lambda a: torch.from_numpy(np.ascontiguousarray(a)).pin_memory()  # noqa: E731
+    h_off, h_units, h_vals = pin(t.job_off), pin(t.units), pin(t.values)
+    h_grp = None if t.group is None else pin(t.group.view(np.int16))
+    h_cap = pin(t.capacity)
+    h_sel = [torch.empty((t.S, t.J), dtype=torch.int32).pin_memory() for _ in range(2)]
+    h_lam = [torch.empty((t.S, t.P), dtype=torch.float64).pin_memory() for _ in range(2)]
+    # a cold load: a new context (fresh buffers, nothing planned yet)
+    torch.cuda.synchronize()
+    c0 = time.perf_counter()
+    other = esp.Solver(device=local, stream=stream.cuda_stream)
+    esp.esp_load_options(other.ctx, t.S, t.J, t.R, t.P, t.r_global, h_off, h_units, h_vals, h_grp, h_cap)
+    torch.cuda.synchronize()
+    cold_ms = (time.perf_counter() - c0) * 1e3
+    ctxs = [solver.ctx, other.ctx]
+    prm = [s.params(w.eta0, T, mode=w.mode, step=w.step) for s in (solver, other)]
+
+    def load(i):
+        esp.esp_load_options(ctxs[i], t.S, t.J, t.R, t.P, t.r_global, h_off, h_units, h_vals, h_grp, h_cap)
+
+    def run(steps):
+        load(0)
+        esp.esp_solve_async(ctxs[0], prm[0])
+        for i in range(steps):
+            cur, nxt = i % 2, (i + 1) % 2
+            if i + 1 < steps:
+                load(nxt)          # overlaps the current solve
+            esp.esp_get_selection(ctxs[cur], h_sel[cur])
+            esp.esp_get_prices(ctxs[cur], h_lam[cur])
+            if i + 1 < steps:
+                esp.esp_solve_async(ctxs[nxt], prm[nxt])
+
+    run(max(2, args.warmup))
+    barrier()
+    t0 = time.perf_counter()
+    run(args.steps)
+    e2e_s = (time.perf_counter() - t0) / args.steps
+    barrier()
+    # a warm load alone (same offsets: the host plan is reused), for the split of a step
+    w0 = time.perf_counter()
+    load(1)
+    warm_ms = (time.perf_counter() - w0) * 1e3
+    evals_step = t.n_opt * (T + 1)
+    e2e_value, e2e_s, _ = aggregate(dist, e2e_s, evals_step, device="cuda")
+    h2d = t.job_off.nbytes + t.units.nbytes + t.values.nbytes + t.capacity.nbytes + \
+        (0 if t.group is None else t.group.nbytes)
+    d2h = h_sel[0].numel() * 4 + h_lam[0].numel() * 8
+    other.close()
+    return {"value": e2e_value, "unit": "option-evals/s", "h2d_bytes_per_step": int(h2d),
+            "d2h_bytes_per_step": int(d2h), "ms_per_step": e2e_s * 1e3,
+            "cold_load_ms": cold_ms, "warm_load_ms": warm_ms,
+            "pipeline": "two contexts: step i+1's upload overlaps step i's solve"}
+
+
 def run_ours(args):
     import torch
     rank, world, local = rank_info()
@@ -360,32 +494,16 @@ def run_ours(args):
         build.build()
     esp.load_library()
 
+    def barrier():
+        if dist is not None:
+            dist.barrier()
+
     w = make_workload(args.workload, rank, args.scenarios)
     T = args.rounds if args.rounds is not None else w.rounds
     t = w.table
     stream = torch.cuda.Stream()
     solver = esp.Solver(t, device=local, stream=stream.cuda_stream)
-
-    # the timed solves replay one CUDA graph per solve with an event pair around every evaluation pass
-    # (event-record nodes of the graph), so the pass timings come from the timed region itself
-    # the timed solves replay one CUDA graph per solve; a second, separately timed set of solves puts
-    # an event pair around every evaluation pass (event-record nodes of the graph) for the kernel's
-    # own duration. Without the events each pass is a programmatic dependent of the kernel before
-    # it, so the step time is the one to report.
-    prm = solver.params(w.eta0, T, mode=w.mode, step=w.step)
-    prm_ev = solver.params(w.eta0, T, mode=w.mode, step=w.step, flags=esp.ESP_FLAG_PASS_EVENTS)
     ctx = solver.ctx
-
-    def barrier():
-        if dist is not None:
-            dist.barrier()
-
-    # warm-up (also builds the CUDA graph when --graph)
-    for _ in range(args.warmup):
-        esp.esp_solve_async(ctx, prm)
-    stream.synchronize()
-    esp.esp_pass_times(ctx, reset=True)
-    launches_per_step = esp.esp_last_launch_count(ctx)
 
     uuid = None
     try:
@@ -395,58 +513,9 @@ def run_ours(args):
     except Exception:
         uuid = None
 
-    barrier()
-    torch.cuda.synchronize()
-    ev0 = torch.cuda.Event(enable_timing=True)
-    ev1 = torch.cuda.Event(enable_timing=True)
-    with ClockSampler(uuid) as clk:
-        ev0.record(stream)
-        for _ in range(args.steps):
-            esp.esp_solve_async(ctx, prm)
-        ev1.record(stream)
-        stream.synchronize()
-    torch.cuda.synchronize()
-    barrier()
-    ms = ev0.elapsed_time(ev1) / args.steps
-    res = np.zeros(t.S, esp.RESULT_DTYPE)
-    st = esp.esp_get_result(ctx, res)
-    assert np.all(res["rounds_run"] == T) or st != 0, "unexpected early stop"
-
-    n_res, n_marked = esp.esp_debug_stats(ctx, reset=True)
-    # the pass durations: solves with an event pair around every pass (the last solve's passes)
-    n_ev = max(1, min(args.steps, 3))
-    for _ in range(1 + n_ev):
-        esp.esp_solve_async(ctx, prm_ev)
-    stream.synchronize()
-    pass_ms, n_pass = esp.esp_pass_times(ctx, reset=True)
-    ev0.record(stream)
-    esp.esp_solve_async(ctx, prm_ev)
-    ev1.record(stream)
-    stream.synchronize()
-    ms_ev = ev0.elapsed_time(ev1)
-    pass_ms, n_pass = esp.esp_pass_times(ctx, reset=True)
-
-    evals_step = t.n_opt * (T + 1)
-    value, step_s, evals_total = aggregate(dist, ms / 1e3, evals_step, device="cuda")
-    ms_max = step_s * 1e3
-
-    # roofline of the dominant kernel (the evaluation pass): algorithmic bytes = the option table
-    peak, peak_kind = measured_peak()
-    pass_avg_ms = pass_ms / max(n_pass, 1)
-    bytes_pass = t.table_bytes()
-    achieved = bytes_pass / (pass_avg_ms / 1e3) / 1e9 if n_pass else None
-    traffic = kernel_traffic(t.n_opt)
-    roofline = {"bound": "hbm", "kernel": "k_pass (best response + demand aggregation)",
-                "achieved": achieved, "peak": peak, "unit": "GB/s",
-                "frac": (achieved / peak) if achieved else None, "traffic": traffic,
-                "peak_kind": f"{peak_kind} hbm_gbs (copy)",
-                "frac_of_nominal_8tbs": (achieved / 8000.0) if achieved else None,
-                "bytes_per_launch": bytes_pass, "avg_launch_ms": pass_avg_ms, "launches_timed": n_pass,
-                "share_of_step": pass_ms / ms_ev if ms_ev else None,
-                "event_timed_ms_per_step": ms_ev,
-                "achieved_over_step": bytes_pass * (T + 1) / (ms / 1e3) / 1e9,
-                "exact_resolutions_per_pass": n_res / max(1, (args.warmup + args.steps) * (T + 1)),
-                "duplicates_marked": n_marked}
+    clk = ClockSampler(uuid)
+    main = time_streaming(esp, solver, w, T, args, dist, barrier, stream, clk)
+    value, ms_max = main["value"], main["ms_per_step"]
 
     # the cluster-resident path (all rounds in one launch, tables in shared memory) on the same
     # workload, when the table qualifies: a second measured line beside the streaming one
@@ -469,7 +538,7 @@ def run_ours(args):
         stream.synchronize()
         barrier()
         res_ms = r0.elapsed_time(r1) / args.steps
-        res_value, res_s, _ = aggregate(dist, res_ms / 1e3, evals_step, device="cuda")
+        res_value, res_s, _ = aggregate(dist, res_ms / 1e3, t.n_opt * (T + 1), device="cuda")
         lam_res = np.zeros((t.S, t.P))
         esp.esp_get_prices(ctx, lam_res)
         resident = {"value": res_value, "unit": "option-evals/s", "ms_per_step": res_s * 1e3,
@@ -477,16 +546,76 @@ def run_ours(args):
                     "launches_per_step": esp.esp_last_launch_count(ctx),
                     "same_prices_as_streaming": bool(np.array_equal(lam_res, lam_stream)),
                     "note": "ESP_FLAG_RESIDENT: each scenario's table read from HBM once per solve, then held "
-                            "in the shared memory of one thread-block cluster for all rounds"}
+                            "in the shared memory of one thread-block cluster for all rounds (the library "
+                            "falls back to streaming where its cost model predicts the resident solve slower)"}
 
     # the factored placement path (configurations x nodes computed on the fly, esp_load_placement)
     factored = None
     if w.factors is not None and not args.no_factored:
-        lam_stream = np.zeros((t.S, t.P))
-        esp.esp_get_prices(ctx, lam_stream)
-        fs = esp.Solver(device=local, stream=stream.cuda_stream)
-        fs.load_placement(w.factors)
-        prm_f = fs.params(w.eta0, T, mode=w.mode, step=w.step)
+        factored = bench_factored(esp, w, T, args, dist, barrier, stream, local, ctx)
+
+    # the IAC slowdown predictor (Eq. dnn_pred) over the what-if batch's co-location pairs
+    iac_line = None if args.no_iac else bench_iac(esp, stream, args, dist, barrier)
+
+    # end to end through the public API with host inputs
+    e2e = None if args.no_e2e else time_e2e(esp, solver, w, T, args, dist, barrier, stream, local)
+    solver.close()
+
+    # the second batched workload, measured the same way, as a keyed line
+    second = None
+    if args.second != "none" and args.second != args.workload and args.scenarios is None and args.rounds is None:
+        w2 = make_workload(args.second, rank)
+        s2 = esp.Solver(w2.table, device=local, stream=stream.cuda_stream)
+        second = time_streaming(esp, s2, w2, w2.rounds, args, dist, barrier, stream)
+        second["config"] = config_of(w2, w2.rounds)
+        s2.close()
+        del w2, s2
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(w, T, args.cpu_seconds)
+
+    clocks = clk.summary()
+    line = {
+        "metric": "option-evaluations/sec", "value": value, "unit": "option-evals/s",
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_max,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic (seeded generator, shapes of the named workload)",
+        "config": config_of(w, T),
+        "run": {"parallelism": f"scenarios sharded over {world} GPU(s), no collective",
+                "launch": "one CUDA graph per solve: T+3 launches; pass durations from separate solves with an "
+                          "event pair around every pass"},
+        "rounds_per_sec": main["rounds_per_sec"],
+        "roofline": main["roofline"],
+        "device_ms_last_solve": main["device_ms_last_solve"],
+        "cpu_baseline": cpu,
+        "e2e": e2e,
+        args.second if second is not None else "second": second,
+        "resident": resident,
+        "factored": factored,
+        "iac": iac_line,
+        "clocks": {k: clocks.get(k) for k in ("sm_mhz", "sm_max_mhz", "reasons")},
+        "gpu_launches": int(main["launches_per_step"] * args.steps),
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if dist is not None:
+        dist.destroy_process_group()
+    return 0
+
+
+def bench_factored(esp, w, T, args, dist, barrier, stream, local, ctx):
+    """esp_load_placement on the placement workload: per-round launches and the grid-resident solve."""
+    import torch
+    t = w.table
+    evals_step = t.n_opt * (T + 1)
+    lam_stream = np.zeros((t.S, t.P))
+    esp.esp_get_prices(ctx, lam_stream)
+    fs = esp.Solver(device=local, stream=stream.cuda_stream)
+    fs.load_placement(w.factors)
+
+    def timed(flags):
+        prm_f = fs.params(w.eta0, T, mode=w.mode, step=w.step, flags=flags)
         for _ in range(args.warmup):
             esp.esp_solve_async(fs.ctx, prm_f)
         barrier()
@@ -503,112 +632,21 @@ def run_ours(args):
         f_value, f_s, _ = aggregate(dist, f_ms / 1e3, evals_step, device="cuda")
         lam_f = np.zeros((t.S, t.P))
         esp.esp_get_prices(fs.ctx, lam_f)
-        f_launches = esp.esp_last_launch_count(fs.ctx)
-        # the grid-resident variant (ESP_FLAG_RESIDENT: all rounds in one cooperative launch)
-        prm_fr = fs.params(w.eta0, T, mode=w.mode, step=w.step, flags=esp.ESP_FLAG_RESIDENT)
-        for _ in range(args.warmup):
-            esp.esp_solve_async(fs.ctx, prm_fr)
-        barrier()
-        torch.cuda.synchronize()
-        f0.record(stream)
-        for _ in range(args.steps):
-            esp.esp_solve_async(fs.ctx, prm_fr)
-        f1.record(stream)
-        stream.synchronize()
-        barrier()
-        fr_ms = f0.elapsed_time(f1) / args.steps
-        fr_value, fr_s, _ = aggregate(dist, fr_ms / 1e3, evals_step, device="cuda")
-        lam_fr = np.zeros((t.S, t.P))
-        esp.esp_get_prices(fs.ctx, lam_fr)
-        fr_launches = esp.esp_last_launch_count(fs.ctx)
-        f = w.factors
-        fbytes = f.cfg_units.nbytes + f.cfg_values.nbytes + f.sens.nbytes + f.job_type.nbytes
-        factored = {"value": f_value, "unit": "option-evals/s", "ms_per_step": f_s * 1e3,
-                    "rounds_per_sec": T / f_s, "bytes_per_pass": int(fbytes),
-                    "launches_per_step": f_launches,
-                    "same_prices_as_streaming": bool(np.array_equal(lam_f, lam_stream)),
-                    "grid_resident": {"value": fr_value, "ms_per_step": fr_s * 1e3, "rounds_per_sec": T / fr_s,
-                                      "launches_per_step": fr_launches,
-                                      "same_prices_as_streaming": bool(np.array_equal(lam_fr, lam_stream))},
-                    "note": "esp_load_placement: configurations x nodes scored from the factors, the expanded "
-                            "options are never stored; evaluations counted over the expanded options; "
-                            "grid_resident = ESP_FLAG_RESIDENT, every round in one cooperative launch"}
-        fs.close()
+        return f_value, f_s, esp.esp_last_launch_count(fs.ctx), bool(np.array_equal(lam_f, lam_stream))
 
-    # the IAC slowdown predictor (Eq. dnn_pred) over the what-if batch's co-location pairs
-    iac_line = None if args.no_iac else bench_iac(esp, stream, args, dist, barrier)
-
-    # end to end through the public API with host inputs
-    e2e = None
-    if not args.no_e2e:
-        pin = lambda a: torch.from_numpy(np.ascontiguousarray(a)).pin_memory()  # noqa: E731
-        h_off, h_units, h_vals = pin(t.job_off), pin(t.units), pin(t.values)
-        h_grp = None if t.group is None else pin(t.group.view(np.int16))
-        h_cap = pin(t.capacity)
-        h_sel = torch.empty((t.S, t.J), dtype=torch.int32).pin_memory()
-        h_lam = torch.empty((t.S, t.P), dtype=torch.float64).pin_memory()
-        prm_e2e = solver.params(w.eta0, T, mode=w.mode, step=w.step, flags=0)
-        res_e = np.zeros(t.S, esp.RESULT_DTYPE)
-
-        parts = np.zeros(3)
-
-        def e2e_step():
-            p0 = time.perf_counter()
-            esp.esp_load_options(ctx, t.S, t.J, t.R, t.P, t.r_global, h_off, h_units, h_vals, h_grp, h_cap)
-            p1 = time.perf_counter()
-            esp.esp_solve(ctx, prm_e2e, res_e)
-            p2 = time.perf_counter()
-            esp.esp_get_selection(ctx, h_sel)
-            esp.esp_get_prices(ctx, h_lam)
-            p3 = time.perf_counter()
-            parts[:] += (p1 - p0, p2 - p1, p3 - p2)
-
-        for _ in range(max(1, args.warmup)):
-            e2e_step()
-        barrier()
-        parts[:] = 0.0
-        t0 = time.perf_counter()
-        for _ in range(args.steps):
-            e2e_step()
-        e2e_s = (time.perf_counter() - t0) / args.steps
-        barrier()
-        e2e_value, e2e_s, _ = aggregate(dist, e2e_s, evals_step, device="cuda")
-        h2d = t.job_off.nbytes + t.units.nbytes + t.values.nbytes + t.capacity.nbytes + \
-            (0 if t.group is None else t.group.nbytes)
-        d2h = h_sel.numel() * 4 + h_lam.numel() * 8 + t.S * esp.RESULT_DTYPE.itemsize
-        e2e = {"value": e2e_value, "unit": "option-evals/s", "h2d_bytes_per_step": int(h2d),
-               "d2h_bytes_per_step": int(d2h), "ms_per_step": e2e_s * 1e3,
-               "ms_load_solve_read": [round(1e3 * x / args.steps, 3) for x in parts]}
-
-    cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        cpu = cpu_baseline(w, T, args.cpu_seconds)
-
-    clocks = clk.summary()
-    line = {
-        "metric": "option-evaluations/sec", "value": value, "unit": "option-evals/s",
-        "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_max,
-        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-        "data": "synthetic (seeded generator, shapes of the named workload)",
-        "config": {**config_of(w, T), "parallelism": f"scenarios sharded over {world} GPU(s), no collective",
-                   "launch": "one CUDA graph per solve: T+3 launches, each pass a programmatic dependent "
-                             "of the kernel before it; pass durations from a separate event-timed solve"},
-        "rounds_per_sec": T / (ms_max / 1e3),
-        "roofline": roofline,
-        "cpu_baseline": cpu,
-        "e2e": e2e,
-        "resident": resident,
-        "factored": factored,
-        "iac": iac_line,
-        "clocks": {k: clocks.get(k) for k in ("sm_mhz", "sm_max_mhz", "reasons")},
-        "gpu_launches": int(launches_per_step * args.steps),
-    }
-    if rank == 0:
-        print(json.dumps(line), flush=True)
-    solver.close()
-    if dist is not None:
-        dist.destroy_process_group()
-    return 0
+    f_value, f_s, f_launches, same_f = timed(0)
+    fr_value, fr_s, fr_launches, same_fr = timed(esp.ESP_FLAG_RESIDENT)
+    f = w.factors
+    fbytes = f.cfg_units.nbytes + f.cfg_values.nbytes + f.sens.nbytes + f.job_type.nbytes
+    fs.close()
+    return {"value": f_value, "unit": "option-evals/s", "ms_per_step": f_s * 1e3,
+            "rounds_per_sec": T / f_s, "bytes_per_pass": int(fbytes), "launches_per_step": f_launches,
+            "same_prices_as_streaming": same_f,
+            "grid_resident": {"value": fr_value, "ms_per_step": fr_s * 1e3, "rounds_per_sec": T / fr_s,
+                              "launches_per_step": fr_launches, "same_prices_as_streaming": same_fr},
+            "note": "esp_load_placement: configurations x nodes scored from the factors, the expanded "
+                    "options are never stored; evaluations counted over the expanded options; "
+                    "grid_resident = ESP_FLAG_RESIDENT, every round in one cooperative launch"}
 
 
 def main():

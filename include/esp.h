@@ -66,8 +66,10 @@ typedef enum { ESP_STEP_FIXED = 0, ESP_STEP_INV_SQRT = 1 } esp_step_rule;
 #define ESP_FLAG_RESIDENT 0x8u         /* run all rounds of a scenario in one launch, its table held in the shared
                                           memory of one thread-block cluster for the whole solve (no table bytes
                                           read from HBM after the first round). Taken when the table has no group
-                                          column and each scenario fits in a cluster (up to 16 CTAs of up to about
-                                          227 KB); otherwise the streaming path runs. Same results either way.
+                                          column, each scenario fits in a cluster (up to 16 CTAs of up to about
+                                          227 KB) and the library's cost model predicts it faster than streaming
+                                          (a batch of many scenarios needs many waves of clusters and usually is
+                                          not); otherwise the streaming path runs. Same results either way.
                                           esp_last_launch_count tells which ran (3: resident); with
                                           ESP_FLAG_PASS_EVENTS the one resident launch counts as one pass.
                                           For a table loaded with esp_load_placement it selects the
@@ -103,6 +105,8 @@ typedef struct {
     double dual;            /* g(lambda) at the final prices (Eq. lagrangian maximised over x) */
     double best_dual;       /* min over evaluated rounds of g(lambda^t) when dual_trace is given,
                                else equal to dual */
+    float device_ms;        /* device time of the whole solve (every launch of it, all scenarios),
+                               from a CUDA event pair around it on the context's stream */
 } esp_result;
 
 /* Creates a context on `device` (-1: the current device) that issues all work on `cuda_stream`
@@ -172,7 +176,8 @@ esp_status esp_evaluate(esp_ctx *ctx, const double *lambda, int32_t mode, uint32
  * framework's caching allocator owns the device, or a scheduler loop that must not stall on the
  * device synchronisation that cudaMalloc / cudaFree imply and works from memory reserved up front.
  * Every pointer is a device pointer owned by the caller: the table (job_offsets S*J+1 int64,
- * units n_opt*R int32 >= 0, values n_opt fp64 finite; every job non-empty; R <= 16, no groups),
+ * units n_opt*R int32 >= 0, values n_opt fp64 finite; R <= 16, no groups; a job with no options
+ * gets sel = -1, min_score = +inf and adds no demand),
  * capacity S*R int64 > 0, lambda S*R (>= 0, finite, in the units of `mode`), and the outputs sel
  * S*J, demand S*R (overwritten; int64), min_score S*J (may be NULL). The inputs are not validated.
  * The per-unit prices go to one fixed scratch array of 65536 fp64 in the library's device memory,
@@ -180,7 +185,8 @@ esp_status esp_evaluate(esp_ctx *ctx, const double *lambda, int32_t mode, uint32
  * shared by every call and keeps the last call's contents; calls that may overlap on the GPU (on
  * different streams, or from different threads) race on it and must be serialised by the caller.
  * The first call on a device looks up the array's device address (once per device, under a lock);
- * make that first call before any stream capture. Work is queued on `cuda_stream` (NULL: the legacy
+ * make that first call before any stream capture. The address is kept until the process exits, so
+ * the entry point must not be used across a cudaDeviceReset of that device. Work is queued on `cuda_stream` (NULL: the legacy
  * default stream); the call returns without waiting. Results equal esp_evaluate's.
  * Errors: ESP_ERR_INVALID_ARG, ESP_ERR_UNSUPPORTED (device index >= 64), ESP_ERR_CUDA. */
 esp_status esp_evaluate_noalloc(int32_t S, int32_t J, int32_t R, const int64_t *job_offsets, const int32_t *units,

@@ -26,11 +26,12 @@ struct GraphKey {
     bool has_l0 = false;
     int res = -1;   // resident option in use, -1: streaming
     bool hold = false;
+    uint32_t hold_tx = 0, wait_ms = 0;
     bool operator==(const GraphKey &o) const
     {
         return eta0 == o.eta0 && tol == o.tol && step == o.step && mode == o.mode && T == o.T && flags == o.flags &&
                lt == o.lt && dt == o.dt && ht == o.ht && gt == o.gt && has_l0 == o.has_l0 && res == o.res &&
-               hold == o.hold;
+               hold == o.hold && hold_tx == o.hold_tx && wait_ms == o.wait_ms;
     }
 };
 
@@ -53,6 +54,10 @@ struct PlanCache {
     bool sorted = false;
     esp::SortedLayout lay;
     esp::Plan plan;
+    bool stream_enabled = false;   // the load that made this plan allowed the streaming pass
+    bool stream = false;           // ... and the table took it
+    int32_t stream_grid = 0;
+    esp::StreamPlan splan;
 };
 
 struct esp_ctx {
@@ -103,6 +108,17 @@ struct esp_ctx {
 
     TileDesc *tiles = nullptr;
     int32_t *warp_begin = nullptr;
+    // streaming pass (k_stream): per-CTA block ranges (the blocks are the tiles), when the loaded table
+    // takes it
+    bool stream_enabled = false;     // later loads may use the streaming pass (esp_debug_set_stream_pass)
+    bool stream_pass = false;
+    int32_t *cta_begin = nullptr;
+    // failure-detection hooks (esp_debug.h): limit of a bounded wait of the evaluation passes in ms
+    // (0: the default, 4 s), extra bytes announced on the next solve's first stage, allocations left
+    // before an injected failure (-1: none)
+    uint32_t wait_ms = 0;
+    uint32_t hold_tx = 0;
+    int64_t fail_alloc_in = -1;
     int32_t *scen_warps = nullptr;   // warps owning tiles of each scenario
     unsigned int *arrive = nullptr;  // per-scenario arrivals of the round pass in flight
     int32_t n_warps = 0, tile_opt = 0, grid = 0, uniform_k = 0;
@@ -117,6 +133,7 @@ struct esp_ctx {
     std::vector<ResOption> res;
     int32_t *res_cuts = nullptr;
     int res_auto = -1;     // index into res of the automatic choice (-1: none fits)
+    bool res_slower = false;   // the automatic choice is predicted slower than streaming: streaming runs
     int res_force = -1;    // index forced through esp_debug_resident (-1: automatic)
 
     double *lam = nullptr, *p64 = nullptr, *job_val = nullptr, *job_min = nullptr;
@@ -137,6 +154,9 @@ struct esp_ctx {
 
     cudaGraphExec_t gexec = nullptr;
     GraphKey gkey;
+    // an event pair around the last solve or evaluation (esp_result::device_ms)
+    cudaEvent_t solve_ev[2] = {nullptr, nullptr};
+    bool solve_timed = false;
     int64_t last_launches = 0;
     int32_t last_T = 0;
 
@@ -186,6 +206,8 @@ esp_status dev_alloc(esp_ctx *ctx, T **p, size_t count, size_t pad_bytes = 64)
         }
     }
     size_t have = bytes;
+    if (ctx->fail_alloc_in >= 0 && ctx->fail_alloc_in-- == 0)
+        return ESP_ERR_OOM;   // injected failure (esp_debug_fail_alloc)
     if (bi != SIZE_MAX) {
         q = ctx->pool[bi].first;
         have = ctx->pool[bi].second;
@@ -248,6 +270,8 @@ void release_table(esp_ctx *ctx, bool keep = false)
     ctx->place_res_ok = false;
     ctx->res_auto = -1;
     ctx->res_force = -1;
+    ctx->stream_pass = false;
+    ctx->cta_begin = nullptr;
     ctx->loaded = false;
     ctx->solved = false;
 }
@@ -486,7 +510,8 @@ esp_status load_common(esp_ctx *ctx, int32_t S, int32_t J, int32_t R, int32_t P,
     // the plan of the previous load serves when the shape and offsets are the same
     PlanCache &pc = ctx->pc;
     const bool cached = pc.valid && pc.S == S && pc.J == J && pc.R == R && pc.P == P && pc.grouped == grouped &&
-                        pc.sorted_enabled == ctx->sorted_enabled && (int64_t)pc.off.size() == n_jobs + 1 &&
+                        pc.sorted_enabled == ctx->sorted_enabled && pc.stream_enabled == ctx->stream_enabled &&
+                        (int64_t)pc.off.size() == n_jobs + 1 &&
                         std::memcmp(pc.off.data(), off_host, (size_t)(n_jobs + 1) * sizeof(int64_t)) == 0;
     // option counts, on the host meanwhile: every job non-empty makes the offsets strictly
     // increasing up to n_opt, so no kernel below can index outside the table
@@ -511,6 +536,10 @@ esp_status load_common(esp_ctx *ctx, int32_t S, int32_t J, int32_t R, int32_t P,
 
     // plan the evaluation pass
     ctx->uniform_k = (!grouped && min_k == max_k && max_k <= 32 && (max_k & (max_k - 1)) == 0) ? (int32_t)max_k : 0;
+    // the streaming pass (k_stream) takes uniform tables and ragged tables whose jobs have at most
+    // kStreamRunMaxK options (through the sorted layout); every other table the per-warp pass
+    const bool stream_try = ctx->stream_enabled && !grouped && J >= 1 &&
+                            (ctx->uniform_k > 0 || (ctx->sorted_enabled && max_k <= kStreamRunMaxK));
 
     // general tables without a group column: the evaluation pass reads the sorted layout (runs of
     // equal-size jobs take the uniform paths). Jobs keep their option order, so the copy inherits
@@ -520,7 +549,8 @@ esp_status load_common(esp_ctx *ctx, int32_t S, int32_t J, int32_t R, int32_t P,
     if (cached)
         use_sorted = pc.sorted;
     else
-        use_sorted = ctx->sorted_enabled && !grouped && ctx->uniform_k == 0 && J >= 1 && sort_layout(off_host, S, J, lay_new);
+        use_sorted = ctx->sorted_enabled && !grouped && ctx->uniform_k == 0 && J >= 1 &&
+                     sort_layout(off_host, S, J, lay_new, stream_try ? kStreamRunMaxK : kRunMaxK);
     const SortedLayout &lay = cached ? pc.lay : lay_new;
     if (use_sorted) {
         const int64_t sn = lay.off.back();
@@ -539,25 +569,42 @@ esp_status load_common(esp_ctx *ctx, int32_t S, int32_t J, int32_t R, int32_t P,
     const int64_t *plan_off = ctx->sorted ? lay.off.data() : off_host;
     const int32_t *plan_scen = ctx->sorted ? lay.scen.data() : nullptr;
     const int32_t *plan_runk = ctx->sorted ? lay.runk.data() : nullptr;
-    const int tile_opt = tile_options_for(R, grouped, max_k, ctx->uniform_k >= 4);
-    const int per_sm = pass_ctas_per_sm(R, grouped, ctx->uniform_k > 0, P, tile_opt);
-    if (per_sm < 1) {
-        release_table(ctx);
-        return ESP_ERR_UNSUPPORTED;
-    }
-    // two waves of resident CTAs by default: CTAs that finish early take the second wave's ranges,
-    // which halves the pass's tail (measured: what-if batch -2.1%, heavy-tailed table -2.5%)
-    const int waves = ctx->plan_waves > 0 ? ctx->plan_waves : 2;
-    const int max_warps = ctx->sm_count * per_sm * kWarpsPerCta * waves;
+
     Plan plan_new;
-    const bool plan_cached = cached && pc.max_warps == max_warps && pc.tile_opt == tile_opt;
-    if (!plan_cached && (!plan_tiles(plan_off, S, J, tile_opt, max_warps, plan_new, plan_scen, plan_runk) ||
-                         !check_plan(plan_off, S, J, plan_new, plan_scen, plan_runk))) {
-        cudaStreamSynchronize(ctx->stream);
-        release_table(ctx);
-        return ESP_ERR_INVALID_ARG;
+    StreamPlan splan_new;
+    bool plan_cached = false, stream = false;
+    int tile_opt = 0, max_warps = 0, s_grid = 0;
+    const int s_per_sm = stream_try ? stream_ctas_per_sm(R) : 0;
+    if (stream_try && s_per_sm >= 1 && (ctx->uniform_k > 0 || use_sorted)) {
+        s_grid = ctx->sm_count * std::min(s_per_sm, (int)ESP_STREAM_CTAS_PER_SM);
+        plan_cached = cached && pc.stream && pc.stream_grid == s_grid;
+        stream = plan_cached ||
+                 (plan_stream(plan_off, S, J, plan_scen, plan_runk, ctx->uniform_k, R, stream_stage_opt(R), s_grid,
+                              splan_new) &&
+                  check_stream_plan(plan_off, S, J, plan_scen, plan_runk, ctx->uniform_k, R, splan_new));
+    }
+    if (!stream) {
+        tile_opt = tile_options_for(R, grouped, max_k, ctx->uniform_k >= 4);
+        const int per_sm = pass_ctas_per_sm(R, grouped, ctx->uniform_k > 0, P, tile_opt);
+        if (per_sm < 1) {
+            cudaStreamSynchronize(ctx->stream);
+            release_table(ctx);
+            return ESP_ERR_UNSUPPORTED;
+        }
+        // two waves of resident CTAs by default: CTAs that finish early take the second wave's ranges,
+        // which halves the pass's tail (measured: what-if batch -2.1%, heavy-tailed table -2.5%)
+        const int waves = ctx->plan_waves > 0 ? ctx->plan_waves : 2;
+        max_warps = ctx->sm_count * per_sm * kWarpsPerCta * waves;
+        plan_cached = cached && !pc.stream && pc.max_warps == max_warps && pc.tile_opt == tile_opt;
+        if (!plan_cached && (!plan_tiles(plan_off, S, J, tile_opt, max_warps, plan_new, plan_scen, plan_runk) ||
+                             !check_plan(plan_off, S, J, plan_new, plan_scen, plan_runk))) {
+            cudaStreamSynchronize(ctx->stream);
+            release_table(ctx);
+            return ESP_ERR_INVALID_ARG;
+        }
     }
     const Plan &plan = plan_cached ? pc.plan : plan_new;
+    const StreamPlan &splan = plan_cached ? pc.splan : splan_new;
     // the validation result (the copies, validation and duplicate marking ran during the planning)
     ESP_CUDA(cudaStreamSynchronize(ctx->stream));
     if (vflags != 0) {
@@ -568,14 +615,29 @@ esp_status load_common(esp_ctx *ctx, int32_t S, int32_t J, int32_t R, int32_t P,
     for (int32_t x : h_umax)
         if (x >= (1 << 23))
             ctx->small_units = 0;
-    ctx->n_warps = plan.n_warps;
-    ctx->tile_opt = plan.tile_opt;
-    ctx->grid = (plan.n_warps + kWarpsPerCta - 1) / kWarpsPerCta;
-    ALLOC(ctx->tiles, plan.tiles.size() + 1);
-    ALLOC(ctx->warp_begin, plan.warp_begin.size());
     ALLOC(ctx->scen_warps, (size_t)S);
     ALLOC(ctx->arrive, (size_t)S);
-    {
+    ctx->stream_pass = stream;
+    if (stream) {
+        ctx->n_warps = 0;
+        ctx->tile_opt = splan.stage_opt;
+        ctx->grid = splan.grid;
+        ALLOC(ctx->tiles, splan.tiles.size() + 1);
+        ALLOC(ctx->warp_begin, 1);
+        ALLOC(ctx->cta_begin, splan.cta_begin.size());
+        if (!splan.tiles.empty())
+            ESP_CUDA(cudaMemcpyAsync(ctx->tiles, splan.tiles.data(), splan.tiles.size() * sizeof(TileDesc),
+                                     cudaMemcpyHostToDevice, ctx->stream));
+        ESP_CUDA(cudaMemcpyAsync(ctx->cta_begin, splan.cta_begin.data(), splan.cta_begin.size() * sizeof(int32_t),
+                                 cudaMemcpyHostToDevice, ctx->stream));
+        ESP_CUDA(cudaMemcpyAsync(ctx->scen_warps, splan.arrivals.data(), (size_t)S * sizeof(int32_t),
+                                 cudaMemcpyHostToDevice, ctx->stream));
+    } else {
+        ctx->n_warps = plan.n_warps;
+        ctx->tile_opt = plan.tile_opt;
+        ctx->grid = (plan.n_warps + kWarpsPerCta - 1) / kWarpsPerCta;
+        ALLOC(ctx->tiles, plan.tiles.size() + 1);
+        ALLOC(ctx->warp_begin, plan.warp_begin.size());
         std::vector<int32_t> sw((size_t)S, 0);
         for (int32_t w = 0; w < plan.n_warps; ++w) {
             int32_t last = -1;
@@ -588,12 +650,12 @@ esp_status load_common(esp_ctx *ctx, int32_t S, int32_t J, int32_t R, int32_t P,
         ESP_CUDA(cudaMemcpyAsync(ctx->scen_warps, sw.data(), sw.size() * sizeof(int32_t), cudaMemcpyHostToDevice,
                                  ctx->stream));
         ESP_CUDA(cudaStreamSynchronize(ctx->stream));
-    }
-    if (!plan.tiles.empty())
-        ESP_CUDA(cudaMemcpyAsync(ctx->tiles, plan.tiles.data(), plan.tiles.size() * sizeof(TileDesc),
+        if (!plan.tiles.empty())
+            ESP_CUDA(cudaMemcpyAsync(ctx->tiles, plan.tiles.data(), plan.tiles.size() * sizeof(TileDesc),
+                                     cudaMemcpyHostToDevice, ctx->stream));
+        ESP_CUDA(cudaMemcpyAsync(ctx->warp_begin, plan.warp_begin.data(), plan.warp_begin.size() * sizeof(int32_t),
                                  cudaMemcpyHostToDevice, ctx->stream));
-    ESP_CUDA(cudaMemcpyAsync(ctx->warp_begin, plan.warp_begin.data(), plan.warp_begin.size() * sizeof(int32_t),
-                             cudaMemcpyHostToDevice, ctx->stream));
+    }
 
     // the resident kernel's options are planned on first use (plan_resident_options)
     ctx->res_planned = false;
@@ -622,6 +684,10 @@ esp_status load_common(esp_ctx *ctx, int32_t S, int32_t J, int32_t R, int32_t P,
         pc.max_warps = max_warps;
         pc.tile_opt = tile_opt;
         pc.plan = std::move(plan_new);
+        pc.stream_enabled = ctx->stream_enabled;
+        pc.stream = stream;
+        pc.stream_grid = s_grid;
+        pc.splan = std::move(splan_new);
     }
     trim_pool(ctx);
     ctx->loaded = true;
@@ -668,7 +734,38 @@ bool state_ready(const esp_ctx *c)
     if (c->placement)
         return c->place.cfg_units && c->place.cfg_values && c->place.sens && c->place.job_type &&
                c->place.node_type && c->place.D && c->place.cfg_dup && c->place.warp_job && c->place.n_warps > 0;
-    return c->grid == 0 || (c->tiles && c->warp_begin && c->units && c->values && c->off);
+    return c->grid == 0 || (c->tiles && c->warp_begin && c->units && c->values && c->off &&
+                            (!c->stream_pass || c->cta_begin));
+}
+
+// The plan of the evaluation pass as the kernels take it.
+DevPlan dev_plan(const esp_ctx *c, bool fused)
+{
+    DevPlan pl;
+    pl.tiles = c->tiles;
+    pl.warp_begin = c->warp_begin;
+    pl.n_warps = c->n_warps;
+    pl.tile_opt = c->tile_opt;
+    pl.uniform_k = c->uniform_k;
+    pl.scen_warps = fused ? c->scen_warps : nullptr;
+    pl.cta_begin = c->stream_pass ? c->cta_begin : nullptr;
+    return pl;
+}
+
+// Solve arguments common to every launch of a solve or evaluation.
+SolveArgs solve_args(const esp_ctx *c, double eta0, int32_t step, int32_t mode, int32_t T, double tol, uint32_t flags)
+{
+    SolveArgs a;
+    a.eta0 = eta0;
+    a.step = step;
+    a.mode = mode;
+    a.T = T;
+    a.tol = tol;
+    a.flags = flags;
+    a.exact_only = (flags & ESP_FLAG_EXACT_ONLY) ? 1 : 0;
+    a.wait_ms = c->wait_ms ? c->wait_ms : kWaitLimitMs;
+    a.hold_tx = c->hold_tx;
+    return a;
 }
 
 // Options of the cluster-resident kernel (ESP_FLAG_RESIDENT) for the loaded table: every cluster
@@ -681,6 +778,7 @@ esp_status plan_resident_options(esp_ctx *ctx)
     ctx->res_planned = true;
     ctx->res.clear();
     ctx->res_auto = -1;
+    ctx->res_slower = false;
     const int32_t S = ctx->S, J = ctx->J, R = ctx->R;
     esp_status st = ESP_OK;
     if (!ctx->pc.valid || (int64_t)ctx->pc.off.size() != (int64_t)S * J + 1)
@@ -741,6 +839,19 @@ esp_status plan_resident_options(esp_ctx *ctx)
                     ctx->res_auto = (int)i;
                 }
             }
+            // the automatic choice runs only where it is predicted faster than streaming. Absolute
+            // times per round measured on GB300: a resident round of one wave of clusters costs about
+            // 2.6 + 0.135 cs + 7.8e-5 n_max us (2.7 us at 1 CTA, 4.75 us at 16 CTAs), and S scenarios
+            // take ceil(S / clusters) waves; a streaming round reads the table at about 5.6 TB/s
+            // plus 3 us, and no streaming round takes less than about 9 us (launch and update latency)
+            if (ctx->res_auto >= 0) {
+                const esp_ctx::ResOption &o = ctx->res[ctx->res_auto];
+                const double waves = std::ceil((double)S / (double)o.clusters);
+                const double res_us = waves * (2.6 + 0.135 * o.plan.cs + 7.8e-5 * (double)o.n_max);
+                const double bytes = (double)ctx->n_opt * (4.0 * R + 8.0);
+                const double stream_us = std::max(9.0, 3.0 + bytes / 5.6e6);
+                ctx->res_slower = res_us > stream_us;
+            }
         }
     }
 
@@ -755,6 +866,18 @@ bool pdl_default(const esp_ctx *c)
     return !c->placement && c->uniform_k > 0 && (int64_t)c->S * c->J >= (1 << 16);
 }
 
+// Records event i of the pair around a solve on the context's stream (outside any capture).
+cudaError_t record_solve_event(esp_ctx *ctx, int i)
+{
+    if (!ctx->solve_ev[i]) {
+        const cudaError_t e = cudaEventCreate(&ctx->solve_ev[i]);
+        if (e != cudaSuccess)
+            return e;
+    }
+    ctx->solve_timed = (i == 1);
+    return cudaEventRecord(ctx->solve_ev[i], ctx->stream);
+}
+
 // Queues one whole solve on the stream (captured into a graph when the stream allows it).
 esp_status enqueue_solve(esp_ctx *ctx, const esp_params *p, const DevState &st, bool has_l0)
 {
@@ -762,24 +885,12 @@ esp_status enqueue_solve(esp_ctx *ctx, const esp_params *p, const DevState &st, 
         return ESP_ERR_STATE;
     const DevTable t = pass_table(ctx);
     const DevTable t_orig = dev_table(ctx);   // the resident kernel reads the original layout
-    DevPlan pl;
-    pl.tiles = ctx->tiles;
-    pl.warp_begin = ctx->warp_begin;
-    pl.n_warps = ctx->n_warps;
-    pl.tile_opt = ctx->tile_opt;
-    pl.uniform_k = ctx->uniform_k;
     // the last warp to finish a scenario in a round pass updates its prices (one launch per round);
     // ESP_FLAG_PER_ROUND_LAUNCH keeps a separate update launch (also used when no warp has tiles)
     const bool fused = ctx->grid > 0 && !(p->flags & ESP_FLAG_PER_ROUND_LAUNCH);
-    pl.scen_warps = fused ? ctx->scen_warps : nullptr;
-    SolveArgs a;
-    a.eta0 = p->eta0;
-    a.step = p->step;
-    a.mode = p->mode;
-    a.T = p->max_rounds;
-    a.tol = p->tol;
-    a.flags = p->flags;
-    a.exact_only = (p->flags & ESP_FLAG_EXACT_ONLY) ? 1 : 0;
+    const DevPlan pl = dev_plan(ctx, fused);
+    const SolveArgs a = solve_args(ctx, p->eta0, p->step, p->mode, p->max_rounds, p->tol, p->flags);
+    ctx->hold_tx = 0;   // the hook holds one solve only
     const int T = p->max_rounds;
 
     const bool timed = (p->flags & ESP_FLAG_PASS_EVENTS) != 0;
@@ -792,7 +903,7 @@ esp_status enqueue_solve(esp_ctx *ctx, const esp_params *p, const DevState &st, 
             return rs;
     }
     const int ri = (p->flags & ESP_FLAG_RESIDENT) && !ctx->placement
-                       ? (ctx->res_force >= 0 ? ctx->res_force : ctx->res_auto)
+                       ? (ctx->res_force >= 0 ? ctx->res_force : (ctx->res_slower ? -1 : ctx->res_auto))
                        : -1;
     // a placement table solves all rounds in one cooperative launch when asked, unless the
     // fingerprint or dual trace is wanted (those need the per-round launches)
@@ -885,9 +996,13 @@ esp_status enqueue_solve(esp_ctx *ctx, const esp_params *p, const DevState &st, 
     key.has_l0 = has_l0;
     key.res = place_res ? -2 : ri;
     key.hold = hold;
+    key.hold_tx = a.hold_tx;
+    key.wait_ms = a.wait_ms;
 
     if (!use_graph) {
+        ESP_CUDA(record_solve_event(ctx, 0));
         ESP_CUDA(issue());
+        ESP_CUDA(record_solve_event(ctx, 1));
         ctx->ev_used = pool_used;
         return ESP_OK;
     }
@@ -914,7 +1029,9 @@ esp_status enqueue_solve(esp_ctx *ctx, const esp_params *p, const DevState &st, 
         ctx->gkey = key;
         ctx->graph_pairs = timed ? pool_used / 2 : 0;
     }
+    ESP_CUDA(record_solve_event(ctx, 0));
     ESP_CUDA(cudaGraphLaunch(ctx->gexec, ctx->stream));
+    ESP_CUDA(record_solve_event(ctx, 1));
     if (timed)
         ctx->graph_timed_run = true;
     return ESP_OK;
@@ -933,8 +1050,14 @@ esp_status read_results(esp_ctx *ctx, esp_result *out)
     ESP_CUDA(cudaMemcpyAsync(du.data(), ctx->dual, S * 8, cudaMemcpyDeviceToHost, ctx->stream));
     ESP_CUDA(cudaMemcpyAsync(bd.data(), ctx->best_dual, S * 8, cudaMemcpyDeviceToHost, ctx->stream));
     ESP_CUDA(cudaStreamSynchronize(ctx->stream));
+    float ms = 0.0f;
+    if (ctx->solve_timed && cudaEventElapsedTime(&ms, ctx->solve_ev[0], ctx->solve_ev[1]) != cudaSuccess) {
+        cudaGetLastError();
+        ms = 0.0f;
+    }
     bool overflow = false;
     for (int s = 0; s < S; ++s) {
+        out[s].device_ms = ms;
         out[s].rounds_run = rr[s];
         out[s].converged = cv[s];
         out[s].feasible = fe[s];
@@ -1203,27 +1326,16 @@ esp_status esp_evaluate(esp_ctx *ctx, const double *lambda, int32_t mode, uint32
     ESP_CUDA(cudaMemcpyAsync(ctx->lambda0, lambda, SP * sizeof(double), cudaMemcpyHostToDevice, ctx->stream));
     const DevTable t = pass_table(ctx);
     DevState ds = dev_state(ctx);
-    DevPlan pl;
-    pl.tiles = ctx->tiles;
-    pl.warp_begin = ctx->warp_begin;
-    pl.n_warps = ctx->n_warps;
-    pl.tile_opt = ctx->tile_opt;
-    pl.uniform_k = ctx->uniform_k;
-    pl.scen_warps = nullptr;
-    SolveArgs a;
-    a.eta0 = 1.0;
-    a.step = 0;
-    a.mode = mode;
-    a.T = 0;
-    a.tol = 0.0;
-    a.flags = flags;
-    a.exact_only = (flags & ESP_FLAG_EXACT_ONLY) ? 1 : 0;
+    const DevPlan pl = dev_plan(ctx, false);
+    const SolveArgs a = solve_args(ctx, 1.0, 0, mode, 0, 0.0, flags);
+    ESP_CUDA(record_solve_event(ctx, 0));
     ESP_CUDA(launch_init(t, ds, a, ctx->lambda0, ctx->stream));
     if (ctx->placement)
         ESP_CUDA(launch_place(t, ds, ctx->place, a, 0, PASS_FINAL, ctx->place_grid, ctx->stream));
     else if (ctx->grid > 0)
         ESP_CUDA(launch_pass(t, ds, pl, a, 0, PASS_FINAL, ctx->grid, ctx->stream));
     ESP_CUDA(launch_objectives(t, ds, a, ctx->stream));
+    ESP_CUDA(record_solve_event(ctx, 1));
     ctx->solved = true;
     if ((st = check_device_error(ctx)) != ESP_OK)
         return st;
@@ -1583,6 +1695,9 @@ void esp_destroy(esp_ctx *ctx)
         cudaEventDestroy(e);
     for (cudaEvent_t e : ctx->graph_pool)
         cudaEventDestroy(e);
+    for (cudaEvent_t e : ctx->solve_ev)
+        if (e)
+            cudaEventDestroy(e);
     delete ctx;
 }
 
@@ -1738,6 +1853,107 @@ esp_status esp_debug_set_pdl(esp_ctx *ctx, int32_t mode)
         ctx->gexec = nullptr;
         ctx->gkey = GraphKey();
     }
+    return ESP_OK;
+}
+
+esp_status esp_debug_set_wait_limit(esp_ctx *ctx, uint32_t limit_ms)
+{
+    esp_status st = check_ctx(ctx);
+    if (st != ESP_OK)
+        return st;
+    ctx->wait_ms = limit_ms;
+    return ESP_OK;
+}
+
+esp_status esp_debug_hold_stage(esp_ctx *ctx)
+{
+    esp_status st = check_ctx(ctx);
+    if (st != ESP_OK)
+        return st;
+    if (!ctx->loaded || ctx->placement || ctx->grid == 0)
+        return ESP_ERR_UNSUPPORTED;
+    ctx->hold_tx = 16;
+    return ESP_OK;
+}
+
+esp_status esp_debug_fail_alloc(esp_ctx *ctx, int64_t n)
+{
+    if (!ctx)
+        return ESP_ERR_INVALID_ARG;
+    ctx->fail_alloc_in = n < 0 ? -1 : n;
+    return ESP_OK;
+}
+
+esp_status esp_debug_set_stream_pass(esp_ctx *ctx, int32_t enable)
+{
+    esp_status st = check_ctx(ctx);
+    if (st != ESP_OK)
+        return st;
+    ctx->stream_enabled = enable != 0;
+    return ESP_OK;
+}
+
+esp_status esp_debug_pass_kernel(esp_ctx *ctx, int32_t *kind)
+{
+    esp_status st = check_ctx(ctx);
+    if (st != ESP_OK)
+        return st;
+    if (!kind)
+        return ESP_ERR_INVALID_ARG;
+    if (!ctx->loaded)
+        return ESP_ERR_NOT_LOADED;
+    *kind = ctx->placement ? 2 : ctx->stream_pass ? 1 : 0;
+    return ESP_OK;
+}
+
+esp_status esp_debug_plan_stream(const int64_t *job_offsets, int32_t S, int32_t J, const int32_t *scen,
+                                 const int32_t *runk, int32_t uniform_k, int32_t R, int32_t grid, int32_t *tiles,
+                                 int32_t tiles_cap, int32_t *cta_begin, int32_t *arrivals, int32_t *n_tiles,
+                                 int32_t *n_ctas, int32_t *stage_opt)
+{
+    if (!job_offsets || S < 1 || J < 0 || R < 1 || R > kMaxR || grid < 1 || (!scen) != (!runk) || !n_tiles ||
+        !n_ctas || !stage_opt)
+        return ESP_ERR_INVALID_ARG;
+    StreamPlan p;
+    const int32_t so = stream_stage_opt(R);
+    if (!plan_stream(job_offsets, S, J, scen, runk, uniform_k, R, so, grid, p) ||
+        !check_stream_plan(job_offsets, S, J, scen, runk, uniform_k, R, p))
+        return ESP_ERR_INVALID_ARG;
+    *n_tiles = (int32_t)p.tiles.size();
+    *n_ctas = p.grid;
+    *stage_opt = so;
+    if ((int32_t)p.tiles.size() > tiles_cap || !tiles || !cta_begin || !arrivals)
+        return ESP_ERR_OOM;
+    for (size_t i = 0; i < p.tiles.size(); ++i) {
+        const TileDesc &d = p.tiles[i];
+        int32_t *w = tiles + 8 * i;
+        w[0] = (int32_t)(uint32_t)(d.opt_begin & 0xffffffff);
+        w[1] = (int32_t)(d.opt_begin >> 32);
+        w[2] = (int32_t)(uint32_t)(d.job_begin & 0xffffffff);
+        w[3] = (int32_t)(d.job_begin >> 32);
+        w[4] = d.n_opt;
+        w[5] = d.n_job;
+        w[6] = d.scenario;
+        w[7] = (int32_t)d.flags;
+    }
+    std::memcpy(cta_begin, p.cta_begin.data(), p.cta_begin.size() * sizeof(int32_t));
+    std::memcpy(arrivals, p.arrivals.data(), p.arrivals.size() * sizeof(int32_t));
+    return ESP_OK;
+}
+
+esp_status esp_debug_sort_layout_k(const int64_t *job_offsets, int32_t S, int32_t J, int32_t run_max_k, int64_t *off,
+                                   int32_t *jmap, int32_t *scen, int32_t *runk)
+{
+    if (!job_offsets || !off || !jmap || !scen || !runk || S < 1 || J < 1 || run_max_k < 4 || (run_max_k & 3) ||
+        run_max_k > 4096)
+        return ESP_ERR_INVALID_ARG;
+    SortedLayout lay;
+    if (!sort_layout(job_offsets, S, J, lay, run_max_k))
+        return ESP_ERR_INVALID_ARG;
+    std::memcpy(off, lay.off.data(), lay.off.size() * sizeof(int64_t));
+    std::memcpy(jmap, lay.jmap.data(), lay.jmap.size() * sizeof(int32_t));
+    std::memcpy(scen, lay.scen.data(), lay.scen.size() * sizeof(int32_t));
+    std::memcpy(runk, lay.runk.data(), lay.runk.size() * sizeof(int32_t));
     return ESP_OK;
 }
 

@@ -39,9 +39,6 @@ namespace esp {
 #ifndef ESP_MIN_CTAS_GENERAL
 #define ESP_MIN_CTAS_GENERAL 4
 #endif
-#ifndef ESP_WAIT_SUSPEND_NS
-#define ESP_WAIT_SUSPEND_NS 1000000   // longest sleep of one stage-wait attempt
-#endif
 #ifndef ESP_V32_HW
 #define ESP_V32_HW 0          // 1: fp64 -> fp32 of values by the conversion instruction (round to nearest)
 #endif
@@ -61,6 +58,25 @@ namespace esp {
 #define ESP_I2F_COLS 16       // unit columns r < ESP_I2F_COLS use the int-to-float instruction
 #endif
 
+#ifndef ESP_STREAM_CONSUMERS
+#define ESP_STREAM_CONSUMERS 12   // consumer warps per CTA of the streaming pass (plus one producer warp)
+#endif
+#ifndef ESP_STREAM_SMEM
+#define ESP_STREAM_SMEM 200704    // dynamic shared memory budget of a streaming-pass CTA (stages + barriers)
+#endif
+#ifndef ESP_STREAM_MAX_STAGES
+#define ESP_STREAM_MAX_STAGES 32  // most stages of the streaming pass's copy ring (one block each)
+#endif
+#ifndef ESP_STREAM_STAGE_OPT
+#define ESP_STREAM_STAGE_OPT 256  // options one stage holds (a multiple of 128, at least 256)
+#endif
+#ifndef ESP_STREAM_PRODUCERS
+#define ESP_STREAM_PRODUCERS 2    // producer warps per CTA of the streaming pass (each issues every P-th block)
+#endif
+#ifndef ESP_STREAM_CTAS_PER_SM
+#define ESP_STREAM_CTAS_PER_SM 1  // CTAs per SM the streaming pass is planned for (limited by its shared memory)
+#endif
+
 constexpr int kMaxR = 16;            // stored resource columns per option
 constexpr int kWarpsPerCta = ESP_WARPS_PER_CTA;  // warps of a CTA; each warp owns its own stage ring
 constexpr int kStages = ESP_STAGES;  // TMA stages per warp
@@ -70,9 +86,8 @@ constexpr int kMinCtasPerSm = ESP_MIN_CTAS_UNIFORM; // register budget of the un
 constexpr int kMinCtasPerSmNarrow = ESP_MIN_CTAS_UNIFORM_NARROW;  // ... for R = 4 and R = 6
 constexpr int kMinCtasPerSmGeneral = ESP_MIN_CTAS_GENERAL;  // register budget of the general kernel
 constexpr int kStageDataBytes = ESP_STAGE_DATA_BYTES;  // option bytes (units + values [+ group]) of a full stage
-constexpr uint32_t kWaitSuspendNs = ESP_WAIT_SUSPEND_NS;
-// bound on stage-wait attempts: about 4 s of waiting in total before a timeout is reported
-constexpr uint32_t kWaitPolls = (uint32_t)(4000000000ull / (ESP_WAIT_SUSPEND_NS > 1000 ? ESP_WAIT_SUSPEND_NS : 1000));
+// limit of a bounded stage wait of the evaluation passes, in milliseconds of the GPU's global timer
+constexpr uint32_t kWaitLimitMs = 4000;
 
 constexpr int kResWarps = ESP_RES_WARPS;
 constexpr int kResMaxCluster = 16;   // CTAs per cluster of the resident kernel (16 is non-portable)
@@ -109,12 +124,72 @@ enum : uint32_t {
     TILE_RUN = 8u,        // whole jobs that all have tile_run_k(flags) options (sorted layout)
 };
 
-// Options per job of a TILE_RUN tile (bits 8..15 of the flags).
-ESP_HD int tile_run_k(uint32_t flags) { return (int)((flags >> 8) & 0xffu); }
+ESP_HD int round16(int x) { return (x + 15) & ~15; }
+
+// Options per job of a TILE_RUN tile (bits 8..19 of the flags).
+ESP_HD int tile_run_k(uint32_t flags) { return (int)((flags >> 8) & 0xfffu); }
 ESP_HD uint32_t tile_run_flags(int k) { return TILE_RUN | ((uint32_t)k << 8); }
 
-// Largest padded job of the sorted layout's runs; larger jobs are evaluated in chunks.
+// Largest padded job of the sorted layout's runs for the per-warp pass (k_pass); larger jobs are
+// evaluated in chunks.
 constexpr int kRunMaxK = 128;
+// The same for the streaming pass (k_stream), whose runs take up to 256 options per job (two groups
+// of four options per lane); a table with a larger job uses the per-warp pass.
+constexpr int kStreamRunMaxK = 256;
+
+// ---------------------------------------------------------------------------------------------
+// Streaming pass (k_stream): per CTA kStreamProducers producer warps fill a ring of stream_stages()
+// stages by bulk copies, one block per stage, and kStreamConsumers consumer warps evaluate them. A
+// block is whole jobs of one run and scenario, at most a stage's options, described by one TileDesc
+// (flags: TILE_RUN and the jobs' option count); each block is taken by one consumer warp (the next
+// free one: a shared counter), which releases its stage alone.
+constexpr int kStreamConsumers = ESP_STREAM_CONSUMERS;
+constexpr int kStreamProducers = ESP_STREAM_PRODUCERS;
+
+// Options a stage holds (the same for every R): a multiple of 128, at least 256 (a whole job of the
+// largest run).
+ESP_HD int stream_stage_opt(int R)
+{
+    (void)R;
+    const int t = ESP_STREAM_STAGE_OPT & ~127;
+    return t < 256 ? 256 : t;
+}
+
+// Byte layout of one stage: the block's descriptor (32 bytes) and the block's index in its CTA's
+// range (the stage's sequence word), the units and the values; the regions have room for the up-to-15
+// bytes the bulk copies read before and after their data to keep both ends 16-byte aligned.
+struct StreamStageLayout {
+    int hdr, seq, units, vals, bytes;
+};
+
+ESP_HD StreamStageLayout stream_stage_layout(int stage_opt, int R)
+{
+    StreamStageLayout L;
+    L.hdr = 0;
+    L.seq = 32;
+    L.units = 48;
+    L.vals = L.units + round16(stage_opt * R * 4 + 32);
+    L.bytes = (L.vals + round16(stage_opt * 8 + 32) + 127) & ~127;
+    return L;
+}
+
+// Stages of the ring for R stored columns: as many as the shared-memory budget holds, at most
+// ESP_STREAM_MAX_STAGES, a multiple of kStreamProducers (stage s is filled only by producer
+// s % kStreamProducers, so each stage's blocks are issued in order by one warp).
+ESP_HD int stream_stages(int stage_opt, int R)
+{
+    int n = (ESP_STREAM_SMEM - 16) / (stream_stage_layout(stage_opt, R).bytes + 16);
+    n = n > ESP_STREAM_MAX_STAGES ? ESP_STREAM_MAX_STAGES : n;
+    return n - n % kStreamProducers;
+}
+
+// Dynamic shared memory of a CTA of the streaming pass: the stages, then a full and an empty
+// barrier per stage, then the consumers' block counter.
+ESP_HD int stream_smem_bytes(int stage_opt, int R)
+{
+    const int n = stream_stages(stage_opt, R);
+    return n * stream_stage_layout(stage_opt, R).bytes + 16 * n + 16;
+}
 
 struct TileDesc {
     int64_t opt_begin;    // first global option of the tile
@@ -150,7 +225,6 @@ ESP_HD int tile_options_for(int R, bool grouped, long long max_k, bool uniform4)
     return t > cap ? cap : (int)t;
 }
 
-ESP_HD int round16(int x) { return (x + 15) & ~15; }
 
 // Byte layout of one stage. Every region starts 16-byte aligned and has room for the up-to-15
 // bytes the bulk copy reads before and after its data to keep source and size 16-byte aligned.

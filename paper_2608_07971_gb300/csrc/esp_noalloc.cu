@@ -33,7 +33,9 @@ std::mutex g_setup_mutex;
 double *g_prices_ptr[kMaxDevices] = {};
 
 // Device address of the scratch array on the current device; looked up once per device (the host
-// name of the array is only a stand-in and must never be passed to a kernel).
+// name of the array is only a stand-in and must never be passed to a kernel). The address is kept
+// for the life of the process: after cudaDeviceReset (or any teardown of the device's primary
+// context) it is stale, so the entry point must not be used across a device reset.
 esp_status scratch_for_current_device(double **out)
 {
     int dev = 0;
@@ -97,11 +99,18 @@ __global__ void k_noalloc_best_response(int32_t S, int32_t J, int32_t R, const i
             }
         }
         if (lane == 0) {
-            sel[j] = (int32_t)(best_i - a);
-            if (min_score)
-                min_score[j] = best;
-            for (int r = 0; r < R; ++r)
-                atomicAdd(demand + s * R + r, (unsigned long long)(long long)units[best_i * R + r]);
+            if (b <= a) {
+                // an empty job chooses nothing, and no option of it is read
+                sel[j] = -1;
+                if (min_score)
+                    min_score[j] = INFINITY;
+            } else {
+                sel[j] = (int32_t)(best_i - a);
+                if (min_score)
+                    min_score[j] = best;
+                for (int r = 0; r < R; ++r)
+                    atomicAdd(demand + s * R + r, (unsigned long long)(long long)units[best_i * R + r]);
+            }
         }
     }
 }

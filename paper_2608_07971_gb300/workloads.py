@@ -248,7 +248,8 @@ def _build(seed, scenarios, J, R, K_of_job):
     n_opt = int(job_off[-1])
     units = np.empty((n_opt, R), dtype=np.int32)
     values = np.empty(n_opt, dtype=np.float64)
-    for si in range(S):
+
+    def one(si):
         K, st = Ks[si], streams[si]
         a, b = int(job_off[si * J]), int(job_off[(si + 1) * J])
         loc = job_off[si * J:(si + 1) * J + 1] - a
@@ -260,6 +261,17 @@ def _build(seed, scenarios, J, R, K_of_job):
             k_local = np.arange(c0, c1, dtype=np.int64) - loc[:-1][ji]
             _configs(seed, st[ji], k_local, bj[ji], mem[ji], cpu[ji], host[ji], nvl[ji], net[ji], R,
                      units[a + c0:a + c1], values[a + c0:a + c1])
+
+    # scenarios write disjoint slices; numpy releases the GIL inside its array loops, so threads
+    # overlap them (every draw is a function of its counter: the result does not depend on the order)
+    if S > 1 and n_opt > (1 << 20):
+        from concurrent.futures import ThreadPoolExecutor
+        import os
+        with ThreadPoolExecutor(max_workers=min(S, os.cpu_count() or 1, 16)) as ex:
+            list(ex.map(one, range(S)))
+    else:
+        for si in range(S):
+            one(si)
     return job_off, units, values
 
 
@@ -358,13 +370,20 @@ def heavy_tail(scenarios: Optional[Sequence[int]] = None, J: int = 65536) -> Wor
     job_off, units, value = _build(seed, scenarios, J, R, lambda st: _zipf_counts(seed, st))
     S = len(scenarios)
     cap = np.zeros((S, R), dtype=np.int64)
-    for si in range(S):
+
+    def one(si):
         a, b = int(job_off[si * J]), int(job_off[(si + 1) * J])
         loc_off = job_off[si * J:(si + 1) * J + 1] - a
         loc_job = np.repeat(np.arange(J, dtype=np.int64), np.diff(loc_off))
         for r in range(R):
             med = _lower_median_per_job(units[a:b, r], loc_job, loc_off)
             cap[si, r] = (6 * int(med.sum())) // 10
+
+    # scenarios are independent (numpy's sort releases the GIL, so threads overlap them)
+    from concurrent.futures import ThreadPoolExecutor
+    import os
+    with ThreadPoolExecutor(max_workers=max(1, min(S, os.cpu_count() or 1, 16))) as ex:
+        list(ex.map(one, range(S)))
     cap = np.maximum(cap, 1)
     t = OptionTable(S, J, R, R, R, job_off, units, value, None, cap)
     return Workload("heavy_tail", t, eta0=0.02, rounds=1000, seed=seed)

@@ -1,10 +1,14 @@
 """Parity at the full benchmark sizes, in the launch configuration bench.py times (a non-default stream,
 one CUDA graph per solve, the price update fused into the evaluation pass, no traces).
 
-Sampled scenarios are compared with the oracle's complete trajectory (selections, demands and prices
-bit-exact / 1e-12, objectives 1e-9); every scenario of the batch is checked against properties that
-hold at any size: prices finite and non-negative, selections inside each job, the final demand equal to
-the units of the selected options, the primal equal to their values, feasibility consistent.
+The two batched workloads are compared with the oracle scenario by scenario, every scenario of the
+batch (1024 what-if scenarios, 16 heavy-tailed ones): the final selections, demands and prices of the
+timed launch configuration bit-exact / 1e-12, objectives 1e-9, and, from a second solve that records
+the trajectories, the prices of every round within 1e-12 and the demand of every round bit-exact (the
+oracle runs in a pool of spawned processes, started before the GPU solves, tests/oracle_batch.py).
+The other workloads are compared on their scenario. Every scenario is also checked against properties
+that hold at any size: prices finite and non-negative, selections inside each job, the final demand
+equal to the units of the selected options, the primal equal to their values, feasibility consistent.
 """
 
 import numpy as np
@@ -74,20 +78,44 @@ def check_against_oracle(t, w, T, lam, sel, dem, res, scenarios):
         assert abs(res["dual"][s] - ref.dual) <= 1e-9 * max(1.0, abs(ref.dual))
 
 
-def test_whatif_batch_full(torch):
-    w = W.whatif_batch()
-    T = w.rounds
+def check_every_scenario(torch, name):
+    """Every scenario of a batched workload against the oracle (started first, in the background)."""
+    from tests.oracle_batch import Batch
+    w0 = W.make(name, scenarios=[0])
+    T = w0.rounds
+    S = {"whatif_batch": 1024, "heavy_tail": 16}[name]
+    batch = Batch(name, range(S), T)
+    w = W.make(name)
+    t = w.table
     lam, sel, dem, res = solve_like_bench(torch, w, T)
-    check_properties(w.table, lam, sel, dem, res, T)
-    check_against_oracle(w.table, w, T, lam, sel, dem, res, [0, 311, 777, 1023])
+    check_properties(t, lam, sel, dem, res, T)
+    s = esp.Solver(t)
+    tr = s.solve(w.eta0, T, mode=w.mode, step=w.step, traces="prices")
+    s.close()
+    assert np.array_equal(tr.lam, lam) and np.array_equal(tr.sel, sel) and np.array_equal(tr.demand, dem)
+    refs = batch.result()
+    for i in range(S):
+        ref = refs[i]
+        assert np.array_equal(sel[i], ref["sel"]), f"selection differs in scenario {i}"
+        assert np.array_equal(dem[i], ref["demand"]), f"demand differs in scenario {i}"
+        d = np.abs(lam[i] - ref["lam"])
+        assert np.all(d <= 1e-12 * np.maximum(np.abs(ref["lam"]), 1e-300)), f"prices differ in scenario {i}"
+        assert res["rounds_run"][i] == int(ref["rounds_run"]) == T
+        assert res["feasible"][i] == int(ref["feasible"])
+        assert abs(res["primal"][i] - float(ref["primal"])) <= 1e-9 * max(1.0, abs(float(ref["primal"])))
+        assert abs(res["dual"][i] - float(ref["dual"])) <= 1e-9 * max(1.0, abs(float(ref["dual"])))
+        lt = ref["lambda_trace"]
+        d = np.abs(tr.lambda_trace[i] - lt)
+        assert np.all(d <= 1e-12 * np.maximum(np.abs(lt), 1e-300)), f"price trajectory differs in scenario {i}"
+        assert np.array_equal(tr.demand_trace[i], ref["demand_trace"]), f"demand trajectory differs in {i}"
 
 
-def test_heavy_tail_full(torch):
-    w = W.heavy_tail()
-    T = w.rounds
-    lam, sel, dem, res = solve_like_bench(torch, w, T)
-    check_properties(w.table, lam, sel, dem, res, T)
-    check_against_oracle(w.table, w, T, lam, sel, dem, res, [11])
+def test_whatif_batch_every_scenario(torch):
+    check_every_scenario(torch, "whatif_batch")
+
+
+def test_heavy_tail_every_scenario(torch):
+    check_every_scenario(torch, "heavy_tail")
 
 
 def test_placement_expanded_full(torch):
