@@ -34,7 +34,7 @@ esp_status esp_debug_plan(const int64_t *job_offsets, int32_t S, int32_t J, int3
                           int32_t *n_tiles, int32_t *n_warps);
 
 /* Sorted layout of a general table (jobs of varying size, no group column), as esp_load_options
- * builds it for the evaluation pass: per scenario the jobs of 3..128 options padded to a multiple
+ * builds it for the evaluation pass: per scenario the jobs of 3..256 options padded to a multiple
  * of 4 and ordered by padded size (this part first for every scenario), then per scenario the
  * larger jobs, then per scenario the 2-option and the 1-option jobs. Host buffers:
  *   off   S*J + 1 int64: padded option offsets in sorted order
@@ -98,9 +98,16 @@ esp_status esp_debug_fail_alloc(esp_ctx *ctx, int64_t n);
 /* enable = 0 makes later loads evaluate every table with the per-warp pass (k_pass); 1 restores the
  * default, the streaming pass (k_stream) for uniform tables and for ragged tables whose jobs have at
  * most 256 options. *kind (esp_debug_pass_kernel) receives the pass the loaded table uses: 1
- * streaming, 0 per-warp, 2 factored placement. Results are identical either way. */
+ * streaming, 0 per-warp, 3 per-warp on the tile-interleaved table, 2 factored placement. Results are
+ * identical either way. */
 esp_status esp_debug_set_stream_pass(esp_ctx *ctx, int32_t enable);
 esp_status esp_debug_pass_kernel(esp_ctx *ctx, int32_t *kind);
+
+/* enable = 0 makes later loads keep the per-warp pass's table as separate unit and value arrays (two
+ * bulk copies per tile); 1 restores the default, a tile-interleaved copy (each tile's units then its
+ * values, one bulk copy per tile) wherever every tile allows it (esp_debug_pass_kernel then reports
+ * 3). Results are identical either way. */
+esp_status esp_debug_set_interleave(esp_ctx *ctx, int32_t enable);
 
 /* Runs the streaming pass's host planner (no GPU code) on CSR offsets (host, S*J + 1 int64): with
  * scen and runk (host, S*J int32 each, a sorted layout from esp_debug_sort_layout_k) or, with both

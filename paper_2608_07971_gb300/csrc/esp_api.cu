@@ -93,6 +93,10 @@ struct esp_ctx {
     int32_t *s_jmap = nullptr;
     // Gamma term (esp_set_penalties): the loaded values, kept once penalties are first set
     double *values0 = nullptr;
+    // the pass table tile by tile (units then values of each tile; one bulk copy per tile), when every
+    // tile of the per-warp plan allows it; n_tiles: tiles of that plan
+    unsigned char *il = nullptr;
+    int64_t n_tiles = 0;
 
     // factored placement table (esp_load_placement): no stored option table
     bool placement = false;
@@ -111,6 +115,7 @@ struct esp_ctx {
     // streaming pass (k_stream): per-CTA block ranges (the blocks are the tiles), when the loaded table
     // takes it
     bool stream_enabled = false;     // later loads may use the streaming pass (esp_debug_set_stream_pass)
+    bool il_enabled = true;          // later loads may interleave the pass table (esp_debug_set_interleave)
     bool stream_pass = false;
     int32_t *cta_begin = nullptr;
     // failure-detection hooks (esp_debug.h): limit of a bounded wait of the evaluation passes in ms
@@ -263,6 +268,8 @@ void release_table(esp_ctx *ctx, bool keep = false)
     ctx->s_off = nullptr;
     ctx->s_jmap = nullptr;
     ctx->values0 = nullptr;
+    ctx->il = nullptr;
+    ctx->n_tiles = 0;
     ctx->placement = false;
     ctx->place = DevPlace{};
     ctx->place_grid = 0;
@@ -315,6 +322,7 @@ DevTable dev_table(const esp_ctx *c)
     t.n_groups = c->n_groups;
     t.small_units = c->small_units;
     t.jmap = nullptr;
+    t.il = nullptr;
     return t;
 }
 
@@ -329,6 +337,7 @@ DevTable pass_table(const esp_ctx *c)
         t.n_opt = c->s_n_opt;
         t.jmap = c->s_jmap;
     }
+    t.il = c->il;
     return t;
 }
 
@@ -585,7 +594,10 @@ esp_status load_common(esp_ctx *ctx, int32_t S, int32_t J, int32_t R, int32_t P,
     }
     if (!stream) {
         tile_opt = tile_options_for(R, grouped, max_k, ctx->uniform_k >= 4);
-        const int per_sm = pass_ctas_per_sm(R, grouped, ctx->uniform_k > 0, P, tile_opt);
+        // a sorted layout's tiles are runs and chunks only (the sorted layout exists only without a
+        // group column): the runs-only instantiation
+        const int mode = ctx->uniform_k > 0 ? kModeUniform : (use_sorted && !grouped) ? kModeRuns : kModeGeneral;
+        const int per_sm = pass_ctas_per_sm(R, grouped, mode, P, tile_opt);
         if (per_sm < 1) {
             cudaStreamSynchronize(ctx->stream);
             release_table(ctx);
@@ -602,6 +614,14 @@ esp_status load_common(esp_ctx *ctx, int32_t S, int32_t J, int32_t R, int32_t P,
             release_table(ctx);
             return ESP_ERR_INVALID_ARG;
         }
+        // the runs-only instantiation has no path for a general tile
+        if (mode == kModeRuns)
+            for (const TileDesc &d : (plan_cached ? pc.plan : plan_new).tiles)
+                if (!(d.flags & (TILE_RUN | TILE_BIG))) {
+                    cudaStreamSynchronize(ctx->stream);
+                    release_table(ctx);
+                    return ESP_ERR_INVALID_ARG;
+                }
     }
     const Plan &plan = plan_cached ? pc.plan : plan_new;
     const StreamPlan &splan = plan_cached ? pc.splan : splan_new;
@@ -655,6 +675,25 @@ esp_status load_common(esp_ctx *ctx, int32_t S, int32_t J, int32_t R, int32_t P,
                                      cudaMemcpyHostToDevice, ctx->stream));
         ESP_CUDA(cudaMemcpyAsync(ctx->warp_begin, plan.warp_begin.data(), plan.warp_begin.size() * sizeof(int32_t),
                                  cudaMemcpyHostToDevice, ctx->stream));
+        // one bulk copy per tile when every tile can take it: no job offsets needed (uniform tables,
+        // runs and chunks of the sorted layout), every tile 16-byte aligned in the interleaved copy,
+        // and its values aligned in the stage for the loads of its path (16 bytes for the paths of
+        // four options per lane, 8 otherwise)
+        const int64_t W = 4 * (int64_t)R + 8;
+        bool il_ok = ctx->il_enabled && !grouped && (ctx->uniform_k > 0 || ctx->sorted) && !plan.tiles.empty();
+        for (size_t k = 0; il_ok && k < plan.tiles.size(); ++k) {
+            const TileDesc &d = plan.tiles[k];
+            const int kk = (d.flags & TILE_RUN) ? tile_run_k(d.flags) : ctx->uniform_k;
+            const bool vec = (d.flags & TILE_BIG) ? ((d.opt_begin | (int64_t)d.n_opt) & 3) == 0 : kk >= 4;
+            il_ok = (d.opt_begin * W) % 16 == 0 && ((int64_t)d.n_opt * R * 4) % (vec ? 16 : 8) == 0 &&
+                    ((d.flags & (TILE_BIG | TILE_RUN)) || ctx->uniform_k > 0);
+        }
+        if (il_ok) {
+            const int64_t pass_opt = ctx->sorted ? ctx->s_n_opt : n_opt;
+            ALLOC(ctx->il, (size_t)(pass_opt * W));
+            ctx->n_tiles = (int64_t)plan.tiles.size();
+            ESP_CUDA(launch_interleave(pass_table(ctx), ctx->tiles, ctx->n_tiles, ctx->il, ctx->stream));
+        }
     }
 
     // the resident kernel's options are planned on first use (plan_resident_options)
@@ -747,6 +786,7 @@ DevPlan dev_plan(const esp_ctx *c, bool fused)
     pl.n_warps = c->n_warps;
     pl.tile_opt = c->tile_opt;
     pl.uniform_k = c->uniform_k;
+    pl.runs_only = (c->sorted && c->group == nullptr) ? 1 : 0;
     pl.scen_warps = fused ? c->scen_warps : nullptr;
     pl.cta_begin = c->stream_pass ? c->cta_begin : nullptr;
     return pl;
@@ -1547,6 +1587,8 @@ esp_status refresh_after_values(esp_ctx *ctx, unsigned int *vflags)
     ESP_CUDA(launch_mark_duplicates(t, ctx->units, ctx->stats + 1, ctx->stream, ctx->max_k));
     if (ctx->sorted)
         ESP_CUDA(launch_gather_sorted(t, pass_table(ctx), ctx->s_units, ctx->s_values, ctx->stream));
+    if (ctx->il)
+        ESP_CUDA(launch_interleave(pass_table(ctx), ctx->tiles, ctx->n_tiles, ctx->il, ctx->stream));
     ESP_CUDA(cudaMemcpyAsync(vflags, ctx->valflags, sizeof(unsigned int), cudaMemcpyDeviceToHost, ctx->stream));
     ESP_CUDA(cudaStreamSynchronize(ctx->stream));
     return ESP_OK;
@@ -1893,6 +1935,15 @@ esp_status esp_debug_set_stream_pass(esp_ctx *ctx, int32_t enable)
     return ESP_OK;
 }
 
+esp_status esp_debug_set_interleave(esp_ctx *ctx, int32_t enable)
+{
+    esp_status st = check_ctx(ctx);
+    if (st != ESP_OK)
+        return st;
+    ctx->il_enabled = enable != 0;
+    return ESP_OK;
+}
+
 esp_status esp_debug_pass_kernel(esp_ctx *ctx, int32_t *kind)
 {
     esp_status st = check_ctx(ctx);
@@ -1902,7 +1953,7 @@ esp_status esp_debug_pass_kernel(esp_ctx *ctx, int32_t *kind)
         return ESP_ERR_INVALID_ARG;
     if (!ctx->loaded)
         return ESP_ERR_NOT_LOADED;
-    *kind = ctx->placement ? 2 : ctx->stream_pass ? 1 : 0;
+    *kind = ctx->placement ? 2 : ctx->stream_pass ? 1 : ctx->il ? 3 : 0;
     return ESP_OK;
 }
 

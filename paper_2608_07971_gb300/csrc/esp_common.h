@@ -39,6 +39,9 @@ namespace esp {
 #ifndef ESP_MIN_CTAS_GENERAL
 #define ESP_MIN_CTAS_GENERAL 4
 #endif
+#ifndef ESP_MIN_CTAS_RUNS
+#define ESP_MIN_CTAS_RUNS 5       // register budget of the runs-only kernel (sorted layouts): 5 measured best
+#endif
 #ifndef ESP_V32_HW
 #define ESP_V32_HW 0          // 1: fp64 -> fp32 of values by the conversion instruction (round to nearest)
 #endif
@@ -85,6 +88,7 @@ constexpr int kUniform4Tile = ESP_UNIFORM4_TILE;    // tile of the 4-options-per
 constexpr int kMinCtasPerSm = ESP_MIN_CTAS_UNIFORM; // register budget of the uniform-K evaluation kernel
 constexpr int kMinCtasPerSmNarrow = ESP_MIN_CTAS_UNIFORM_NARROW;  // ... for R = 4 and R = 6
 constexpr int kMinCtasPerSmGeneral = ESP_MIN_CTAS_GENERAL;  // register budget of the general kernel
+constexpr int kMinCtasPerSmRuns = ESP_MIN_CTAS_RUNS;        // ... of the runs-only kernel
 constexpr int kStageDataBytes = ESP_STAGE_DATA_BYTES;  // option bytes (units + values [+ group]) of a full stage
 // limit of a bounded stage wait of the evaluation passes, in milliseconds of the GPU's global timer
 constexpr uint32_t kWaitLimitMs = 4000;
@@ -130,12 +134,20 @@ ESP_HD int round16(int x) { return (x + 15) & ~15; }
 ESP_HD int tile_run_k(uint32_t flags) { return (int)((flags >> 8) & 0xfffu); }
 ESP_HD uint32_t tile_run_flags(int k) { return TILE_RUN | ((uint32_t)k << 8); }
 
-// Largest padded job of the sorted layout's runs for the per-warp pass (k_pass); larger jobs are
-// evaluated in chunks.
-constexpr int kRunMaxK = 128;
-// The same for the streaming pass (k_stream), whose runs take up to 256 options per job (two groups
-// of four options per lane); a table with a larger job uses the per-warp pass.
+// Largest padded job of the sorted layout (a multiple of 4): jobs of 3 .. kRunMaxK options are padded
+// to a multiple of 4 and grouped into runs of equal size, which the per-warp pass evaluates as rows of
+// whole jobs; larger jobs stay unpadded and are evaluated in chunks. (Measured on GB300 with the
+// heavy-tailed table: padding the jobs of 129..256 options too, and reading their chunks four
+// consecutive options per lane, was 2.5% and 7% slower than the unpadded, lane-strided chunks.)
+#ifndef ESP_RUN_MAX_K
+#define ESP_RUN_MAX_K 128
+#endif
+constexpr int kRunMaxK = ESP_RUN_MAX_K;
+// The streaming pass's runs take up to 256 options per job (two groups of four options per lane).
 constexpr int kStreamRunMaxK = 256;
+// Largest run tile of the per-warp pass (rows of whole jobs of up to 32 lanes x 4 options); a padded
+// job above it is planned as chunks.
+constexpr int kPassRunMaxK = 128;
 
 // ---------------------------------------------------------------------------------------------
 // Streaming pass (k_stream): per CTA kStreamProducers producer warps fill a ring of stream_stages()

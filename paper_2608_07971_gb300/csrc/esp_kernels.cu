@@ -104,6 +104,14 @@ __device__ __forceinline__ void issue_tile(const DevTable &t, const TileDesc &d,
                                            const StageLayout &SL, uint32_t bar, bool need_offsets, uint32_t extra_tx = 0)
 {
     const int R = t.R;
+    if (t.il) {   // the tile's units and values are adjacent: one copy (its start is 16-byte aligned)
+        const int64_t W = 4 * R + 8;
+        const int64_t b = d.opt_begin * W, e = ((d.opt_begin + d.n_opt) * W + 15) & ~int64_t(15);
+        fence_proxy_async();
+        mbar_arrive_expect_tx(bar, (uint32_t)(e - b) + extra_tx);
+        bulk_g2s(smem_u32(stage + SL.units), t.il + b, (uint32_t)(e - b), bar);
+        return;
+    }
     const int64_t ub = d.opt_begin * R * 4, ue = (d.opt_begin + d.n_opt) * R * 4;
     const int64_t ulo = ub & ~int64_t(15), uhi = (ue + 15) & ~int64_t(15);
     const int64_t vb = d.opt_begin * 8, ve = (d.opt_begin + d.n_opt) * 8;
@@ -138,14 +146,18 @@ __device__ __forceinline__ void issue_tile(const DevTable &t, const TileDesc &d,
 }
 
 // CTAs per SM the evaluation kernel's register budget must allow.
-template <int RT, bool UNI>
+// CTAs per SM the evaluation kernel's register budget must allow: the uniform and runs-only
+// instantiations (no segmented-scan path) as many as the general one's shared memory would.
+template <int RT, int MODE>
 constexpr int pass_min_ctas()
 {
-    return UNI ? ((RT == 4 || RT == 6) ? kMinCtasPerSmNarrow : kMinCtasPerSm) : kMinCtasPerSmGeneral;
+    return MODE == kModeUniform ? ((RT == 4 || RT == 6) ? kMinCtasPerSmNarrow : kMinCtasPerSm)
+           : MODE == kModeRuns  ? kMinCtasPerSmRuns
+                                : kMinCtasPerSmGeneral;
 }
 
-template <int RT, bool G, bool UNI, bool PLAIN>
-__global__ void __launch_bounds__(kWarpsPerCta * 32, pass_min_ctas<RT, UNI>()) k_pass(DevTable t, DevState st, DevPlan pl,
+template <int RT, bool G, int MODE, bool PLAIN>
+__global__ void __launch_bounds__(kWarpsPerCta * 32, pass_min_ctas<RT, MODE>()) k_pass(DevTable t, DevState st, DevPlan pl,
                                                                           SolveArgs a, int round, int kind)
 {
     extern __shared__ __align__(128) unsigned char smem[];
@@ -164,12 +176,13 @@ __global__ void __launch_bounds__(kWarpsPerCta * 32, pass_min_ctas<RT, UNI>()) k
     if (__any_sync(FULL, (*reinterpret_cast<volatile unsigned int *>(st.err) & DEV_ERR_TIMEOUT) != 0))
         return;
 
-    const WarpSmem WS = warp_smem(pl.tile_opt, t.R, G, t.P, !UNI);
-    const StageLayout SL = stage_layout(pl.tile_opt, t.R, G, !UNI);
+    constexpr bool UNI = MODE == kModeUniform;
+    const WarpSmem WS = warp_smem(pl.tile_opt, t.R, G, t.P, MODE == kModeGeneral);
+    const StageLayout SL = stage_layout(pl.tile_opt, t.R, G, MODE == kModeGeneral);
     unsigned char *wsm = smem + (size_t)wid * WS.bytes;
     float *p32s = reinterpret_cast<float *>(wsm + WS.p32);
     const uint32_t bar0 = smem_u32(wsm + WS.bars);
-    const bool need_offsets = !UNI;
+    const bool need_offsets = MODE == kModeGeneral;
 
     WarpCtx<RT, G> c;
     c.t = t;
@@ -269,7 +282,8 @@ __global__ void __launch_bounds__(kWarpsPerCta * 32, pass_min_ctas<RT, UNI>()) k
         if (d.scenario != c.s)
             enter_scenario<RT, G>(c, d.scenario, p32s, lane);
         if (!c.sp.skip) {
-            const StagePtrs ptrs = stage_ptrs(d, wsm + sidx * SL.bytes, SL, c.R);
+            const StagePtrs ptrs = t.il ? stage_ptrs_il(d, wsm + sidx * SL.bytes, SL, c.R)
+                                        : stage_ptrs(d, wsm + sidx * SL.bytes, SL, c.R);
             if (UNI && c.uniform_k >= 4)
                 process_tile_uniform4<RT, G>(c, d, ptrs, lane);
             else if (UNI)
@@ -280,7 +294,7 @@ __global__ void __launch_bounds__(kWarpsPerCta * 32, pass_min_ctas<RT, UNI>()) k
                 process_tile_run4<RT, G, 1>(c, d, ptrs, lane, tile_run_k(d.flags));
             else if (!G && (d.flags & TILE_RUN))
                 process_tile_uniform<RT, G>(c, d, ptrs, lane, tile_run_k(d.flags), tile_run_k(d.flags) >> 1);
-            else
+            else if (MODE == kModeGeneral)
                 process_tile_general<RT, G>(c, d, ptrs, big_first, big_carry, lane);
         }
         __syncwarp();
@@ -335,10 +349,10 @@ __global__ void k_objectives(DevTable t, DevState st, SolveArgs a)
     }
 }
 // Both instantiations (plain round pass and the general one) of a table shape.
-template <int RT, bool G, bool UNI>
+template <int RT, bool G, int MODE>
 struct PassKernels {
-    static const void *plain() { return reinterpret_cast<const void *>(&k_pass<RT, G, UNI, true>); }
-    static const void *other() { return reinterpret_cast<const void *>(&k_pass<RT, G, UNI, false>); }
+    static const void *plain() { return reinterpret_cast<const void *>(&k_pass<RT, G, MODE, true>); }
+    static const void *other() { return reinterpret_cast<const void *>(&k_pass<RT, G, MODE, false>); }
     // pdl: programmatic dependent launch, so the pass's CTAs may start (and stage their first tiles)
     // while the previous kernel on the stream finishes; the kernel waits for it before reading state
     static void launch(bool plain, int grid, int smem, cudaStream_t stream, const DevTable &t, const DevState &st,
@@ -355,51 +369,60 @@ struct PassKernels {
         cfg.attrs = attr;
         cfg.numAttrs = pdl ? 1 : 0;
         if (plain)
-            cudaLaunchKernelEx(&cfg, k_pass<RT, G, UNI, true>, t, st, pl, a, round, kind);
+            cudaLaunchKernelEx(&cfg, k_pass<RT, G, MODE, true>, t, st, pl, a, round, kind);
         else
-            cudaLaunchKernelEx(&cfg, k_pass<RT, G, UNI, false>, t, st, pl, a, round, kind);
+            cudaLaunchKernelEx(&cfg, k_pass<RT, G, MODE, false>, t, st, pl, a, round, kind);
     }
 };
 
-// Calls f.template operator()<RT, G, UNI>() for the instantiation that serves this table shape.
+// Calls f(PassKernels<RT, G, MODE>()) for the instantiation that serves this table shape (grouped
+// tables are always general).
 template <typename F>
-auto dispatch_shape(int R, bool grouped, bool uni, F &&f)
+auto dispatch_shape(int R, bool grouped, int mode, F &&f)
 {
     if (grouped) {
         switch (R) {
-        case 4: return f(PassKernels<4, true, false>());
-        case 6: return f(PassKernels<6, true, false>());
-        case 8: return f(PassKernels<8, true, false>());
-        default: return f(PassKernels<0, true, false>());
+        case 4: return f(PassKernels<4, true, kModeGeneral>());
+        case 6: return f(PassKernels<6, true, kModeGeneral>());
+        case 8: return f(PassKernels<8, true, kModeGeneral>());
+        default: return f(PassKernels<0, true, kModeGeneral>());
         }
     }
-    if (uni) {
+    if (mode == kModeUniform) {
         switch (R) {
-        case 4: return f(PassKernels<4, false, true>());
-        case 6: return f(PassKernels<6, false, true>());
-        case 8: return f(PassKernels<8, false, true>());
-        default: return f(PassKernels<0, false, true>());
+        case 4: return f(PassKernels<4, false, kModeUniform>());
+        case 6: return f(PassKernels<6, false, kModeUniform>());
+        case 8: return f(PassKernels<8, false, kModeUniform>());
+        default: return f(PassKernels<0, false, kModeUniform>());
+        }
+    }
+    if (mode == kModeRuns) {
+        switch (R) {
+        case 4: return f(PassKernels<4, false, kModeRuns>());
+        case 6: return f(PassKernels<6, false, kModeRuns>());
+        case 8: return f(PassKernels<8, false, kModeRuns>());
+        default: return f(PassKernels<0, false, kModeRuns>());
         }
     }
     switch (R) {
-    case 4: return f(PassKernels<4, false, false>());
-    case 6: return f(PassKernels<6, false, false>());
-    case 8: return f(PassKernels<8, false, false>());
-    default: return f(PassKernels<0, false, false>());
+    case 4: return f(PassKernels<4, false, kModeGeneral>());
+    case 6: return f(PassKernels<6, false, kModeGeneral>());
+    case 8: return f(PassKernels<8, false, kModeGeneral>());
+    default: return f(PassKernels<0, false, kModeGeneral>());
     }
 }
 
 }  // namespace
 
-int pass_smem_bytes(int R, bool grouped, bool uniform, int P, int tile_opt)
+int pass_smem_bytes(int R, bool grouped, int mode, int P, int tile_opt)
 {
-    return kWarpsPerCta * warp_smem(tile_opt, R, grouped, P, !uniform).bytes;
+    return kWarpsPerCta * warp_smem(tile_opt, R, grouped, P, grouped || mode == kModeGeneral).bytes;
 }
 
-int pass_ctas_per_sm(int R, bool grouped, bool uniform, int P, int tile_opt)
+int pass_ctas_per_sm(int R, bool grouped, int mode, int P, int tile_opt)
 {
-    const int smem = pass_smem_bytes(R, grouped, uniform && !grouped, P, tile_opt);
-    return dispatch_shape(R, grouped, uniform && !grouped, [&](auto k) -> int {
+    const int smem = pass_smem_bytes(R, grouped, mode, P, tile_opt);
+    return dispatch_shape(R, grouped, mode, [&](auto k) -> int {
         using K = decltype(k);
         if (cudaFuncSetAttribute(K::plain(), cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess ||
             cudaFuncSetAttribute(K::other(), cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess)
@@ -428,9 +451,10 @@ cudaError_t launch_pass(const DevTable &t, const DevState &st, const DevPlan &pl
     if (pl.cta_begin)
         return launch_stream(t, st, pl, a, round, kind, grid, stream, pdl);
     const bool grouped = t.group != nullptr;
-    const int smem = pass_smem_bytes(t.R, grouped, pl.uniform_k > 0, t.P, pl.tile_opt);
+    const int mode = pass_mode(pl);
+    const int smem = pass_smem_bytes(t.R, grouped, mode, t.P, pl.tile_opt);
     const bool plain = kind == PASS_ROUND && st.hash_trace == nullptr && st.dual_trace == nullptr;
-    dispatch_shape(t.R, grouped, pl.uniform_k > 0, [&](auto k) -> int {
+    dispatch_shape(t.R, grouped, mode, [&](auto k) -> int {
         decltype(k)::launch(plain, grid, smem, stream, t, st, pl, a, round, kind, pdl);
         return 0;
     });

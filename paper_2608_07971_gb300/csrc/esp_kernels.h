@@ -18,6 +18,9 @@ struct DevTable {
     int32_t S, J, R, P, r_global, n_groups;
     int32_t small_units;      // 1 if every unit is below 2^23
     const int32_t *jmap;      // sorted layout: original global index of each job of this table; nullptr: identity
+    // evaluation passes only: the table tile by tile, each tile's units then its values, the tile of
+    // options [a, b) at byte a * (4R + 8) (one bulk copy per tile); nullptr: units and values apart
+    const unsigned char *il;
 };
 
 struct DevState {
@@ -56,6 +59,7 @@ struct DevPlan {
     int32_t n_warps;
     int32_t tile_opt;
     int32_t uniform_k;          // > 0: every job has exactly this many options, a power of two <= 32
+    int32_t runs_only;          // 1: every tile is a run of equal-size jobs or a chunk of a large job
     const int32_t *scen_warps;  // S arrivals that complete each scenario in a round pass (one per warp and
                                 // maximal run of the scenario's tiles); non-null: round passes update prices
     // streaming pass (k_stream) when cta_begin is non-null: every tile is one block, and CTA c
@@ -172,8 +176,18 @@ struct ResPlan {
     int64_t n_cap;      // option slots of a slice (CSR layout)
 };
 
+// Instantiations of the per-warp evaluation kernel: general tables (the segmented scan over job
+// offsets), uniform tables (every job the same power-of-two option count), and sorted layouts, whose
+// tiles are all runs of equal-size jobs or chunks of large jobs (no job offsets, no segmented scan).
+enum : int { kModeGeneral = 0, kModeUniform = 1, kModeRuns = 2 };
+
+inline int pass_mode(const DevPlan &pl)
+{
+    return pl.uniform_k > 0 ? kModeUniform : pl.runs_only ? kModeRuns : kModeGeneral;
+}
+
 // Dynamic shared memory per CTA of the evaluation kernel.
-int pass_smem_bytes(int R, bool grouped, bool uniform, int P, int tile_opt);
+int pass_smem_bytes(int R, bool grouped, int mode, int P, int tile_opt);
 
 // Resident CTAs per SM of the streaming pass for R stored columns (0 if it cannot run); sets the
 // kernels' shared-memory attribute, so it runs (at load time) before their first launch.
@@ -183,7 +197,7 @@ cudaError_t launch_stream(const DevTable &t, const DevState &st, const DevPlan &
                           PassKind kind, int grid, cudaStream_t stream, bool pdl);
 
 // Maximum resident CTAs per SM of the evaluation kernel for this table shape (0 if it cannot run).
-int pass_ctas_per_sm(int R, bool grouped, bool uniform, int P, int tile_opt);
+int pass_ctas_per_sm(int R, bool grouped, int mode, int P, int tile_opt);
 
 cudaError_t launch_validate(const DevTable &t, double *vmax, int32_t *umax, unsigned int *flags,
                             cudaStream_t stream);
@@ -202,6 +216,9 @@ cudaError_t launch_gather_sorted(const DevTable &orig, const DevTable &sorted, i
 cudaError_t launch_apply_penalties(const DevTable &t, const double *values0, const int32_t *c_cur, const double *s_hat,
                                    const double *tau, double gamma0, double alpha, double *values, unsigned int *flags,
                                    cudaStream_t stream);
+// Fills the tile-interleaved copy `il` of table t (t.il's layout) for the n_tiles tiles of a plan.
+cudaError_t launch_interleave(const DevTable &t, const TileDesc *tiles, int64_t n_tiles, unsigned char *il,
+                              cudaStream_t stream);
 // Clears every duplicate mark of a units array.
 cudaError_t launch_clear_marks(int32_t *units, int64_t n_opt, int R, cudaStream_t stream);
 cudaError_t launch_init(const DevTable &t, const DevState &st, const SolveArgs &a, const double *lambda0,

@@ -308,4 +308,35 @@ cudaError_t launch_mark_duplicates(const DevTable &t, int32_t *units, unsigned l
     return cudaGetLastError();
 }
 
+// One warp per tile: the tile's units (n R int32, duplicate marks included) then its values (n fp64)
+// at byte opt_begin * (4R + 8) of the interleaved copy.
+__global__ void k_interleave(DevTable t, const TileDesc *tiles, int64_t n_tiles, unsigned char *il)
+{
+    const int lane = threadIdx.x & 31;
+    const int64_t warps = (int64_t)gridDim.x * (blockDim.x >> 5);
+    const int R = t.R;
+    const int64_t W = 4 * R + 8;
+    for (int64_t k = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); k < n_tiles; k += warps) {
+        const TileDesc d = tiles[k];
+        int32_t *u = reinterpret_cast<int32_t *>(il + d.opt_begin * W);
+        double *v = reinterpret_cast<double *>(il + d.opt_begin * W + (int64_t)d.n_opt * R * 4);
+        const int32_t *su = t.units + d.opt_begin * R;
+        const double *sv = t.values + d.opt_begin;
+        for (int64_t i = lane; i < (int64_t)d.n_opt * R; i += 32)
+            u[i] = su[i];
+        for (int i = lane; i < d.n_opt; i += 32)
+            v[i] = sv[i];
+    }
+}
+
+cudaError_t launch_interleave(const DevTable &t, const TileDesc *tiles, int64_t n_tiles, unsigned char *il,
+                              cudaStream_t stream)
+{
+    if (n_tiles <= 0)
+        return cudaSuccess;
+    const int64_t blocks = std::min<int64_t>((n_tiles + 7) / 8, 65536);
+    k_interleave<<<(int)blocks, 256, 0, stream>>>(t, tiles, n_tiles, il);
+    return cudaGetLastError();
+}
+
 }  // namespace esp

@@ -65,7 +65,7 @@ bool plan_tiles(const int64_t *off, int32_t S, int32_t J, int32_t tile_opt, int3
         }
         const int32_t s = scen ? scen[j] : s_cur;
         const int64_t K = off[j + 1] - off[j];
-        if (K > tile_opt) {
+        if (K > tile_opt || (runk && runk[j] > kPassRunMaxK)) {
             const int64_t nch = (K + tile_opt - 1) / tile_opt;
             for (int64_t c = 0; c < nch; ++c) {
                 TileDesc d;
@@ -183,7 +183,7 @@ bool check_plan(const int64_t *off, int32_t S, int32_t J, const Plan &p, const i
                         return false;
                     if (d.flags & TILE_RUN) {
                         const int k = tile_run_k(d.flags);
-                        if (!runk || runk[j] != k || off[j + 1] - off[j] != k)
+                        if (!runk || runk[j] != k || off[j + 1] - off[j] != k || k > kPassRunMaxK)
                             return false;
                     } else if (runk && runk[j] != 0) {
                         return false;

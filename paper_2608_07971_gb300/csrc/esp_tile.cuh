@@ -171,6 +171,19 @@ __device__ __forceinline__ StagePtrs stage_ptrs(const TileDesc &d, const unsigne
     return p;
 }
 
+// Stage pointers of one tile copied from the tile-interleaved table (DevTable::il): its units at the
+// start of the stage's units region, its values right after them.
+__device__ __forceinline__ StagePtrs stage_ptrs_il(const TileDesc &d, const unsigned char *stage,
+                                                   const StageLayout &SL, int R)
+{
+    StagePtrs p;
+    p.units = reinterpret_cast<const int32_t *>(stage + SL.units);
+    p.vals = reinterpret_cast<const double *>(stage + SL.units + (size_t)d.n_opt * R * 4);
+    p.grp = nullptr;
+    p.off = nullptr;
+    return p;
+}
+
 // Tile of a table whose jobs all have K = uniform_k options (a power of two <= 32). Tiles start at
 // job boundaries, so each aligned group of K lanes of a row is one job: a log2(K)-step xor
 // butterfly gives every lane of the group the smallest and second-smallest screen value; when the
@@ -667,10 +680,14 @@ __device__ void process_tile_bigchunk(WarpCtx<RT, G> &c, const TileDesc &d, cons
     const int K = chunk_base + n;
     if (!amb) {
         if (lane == 0) {
+            // the winner's data: from the stage when it lies in this (last) chunk, else from global
+            // memory (the earlier chunks' stages have been refilled)
             int32_t uw[Cols<RT>::N];
             double vw;
             int gw;
-            load_option<RT, G>(c, false, sp.units, sp.vals, sp.grp, x.idx, big_first, uw, vw, gw);
+            const bool here = x.idx >= chunk_base;
+            load_option<RT, G>(c, here, sp.units, sp.vals, sp.grp, here ? x.idx - chunk_base : x.idx, big_first, uw,
+                               vw, gw);
             take_winner<RT, G>(c, d.job_begin, x.idx, uw, vw, gw, false, 0.0);
         }
     } else if (!c.sp.exact && !__any_sync(FULL, big_priv.m2 <= thr)) {

@@ -31,6 +31,7 @@ EXPORTED = [
     "esp_debug_sort_layout", "esp_debug_plan_runs", "esp_debug_set_sorted_layout", "esp_debug_set_pdl", "esp_debug_set_plan_waves",
     "esp_debug_hold_barrier", "esp_debug_set_wait_limit", "esp_debug_hold_stage", "esp_debug_fail_alloc",
     "esp_debug_set_stream_pass", "esp_debug_pass_kernel", "esp_debug_plan_stream", "esp_debug_sort_layout_k",
+    "esp_debug_set_interleave",
     "esp_evaluate_noalloc",
     "esp_set_penalties", "esp_adaptive_threshold", "esp_effective_capacity", "esp_load_placement",
     "esp_iac_create", "esp_iac_set_stream", "esp_iac_load_model", "esp_iac_predict", "esp_iac_predict_host",
@@ -105,6 +106,7 @@ def load_library(path: Optional[str] = None):
         "esp_debug_fail_alloc": ([vp, i64], st),
         "esp_debug_set_stream_pass": ([vp, i32], st),
         "esp_debug_pass_kernel": ([vp, ctypes.POINTER(i32)], st),
+        "esp_debug_set_interleave": ([vp, i32], st),
         "esp_debug_plan_stream": ([vp, i32, i32, vp, vp, i32, i32, i32, vp, i32, vp, vp,
                                    ctypes.POINTER(i32), ctypes.POINTER(i32), ctypes.POINTER(i32)], st),
         "esp_debug_sort_layout_k": ([vp, i32, i32, i32, vp, vp, vp, vp], st),
@@ -485,8 +487,14 @@ def esp_debug_set_stream_pass(ctx: int, enable: bool) -> None:
     _check(load_library().esp_debug_set_stream_pass(ctx, 1 if enable else 0), "esp_debug_set_stream_pass")
 
 
+def esp_debug_set_interleave(ctx: int, enable: bool) -> None:
+    """Later loads interleave the per-warp pass's table tile by tile (True, the default) or not."""
+    _check(load_library().esp_debug_set_interleave(ctx, 1 if enable else 0), "esp_debug_set_interleave")
+
+
 def esp_debug_pass_kernel(ctx: int) -> int:
-    """The evaluation pass the loaded table uses: 1 streaming, 0 per-warp, 2 factored placement."""
+    """The evaluation pass the loaded table uses: 1 streaming, 0 per-warp, 3 per-warp on the
+    tile-interleaved table, 2 factored placement."""
     k = ctypes.c_int32()
     _check(load_library().esp_debug_pass_kernel(ctx, ctypes.byref(k)), "esp_debug_pass_kernel")
     return k.value

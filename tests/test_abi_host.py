@@ -210,7 +210,7 @@ def test_sorted_layout(lib, case):
     elif case == "small":
         K = rng.integers(1, 6, S * J)
     else:
-        K = rng.choice([129, 700, 3], S * J)
+        K = rng.choice([129, 255, 700, 3], S * J)
     off = np.zeros(S * J + 1, np.int64)
     off[1:] = np.cumsum(K)
     soff, jmap, scen, runk = esp.sort_layout(off, S, J)
@@ -237,7 +237,7 @@ def test_sorted_layout(lib, case):
                 covered[j0:j1] += np.diff(soff[j0:j1 + 1])
                 assert np.all(scen[j0:j1] == tiles[k, 6])
                 if fl & 8:                                   # a run tile: one option count
-                    kk = (fl >> 8) & 0xFF
+                    kk = (fl >> 8) & 0xFFF
                     assert np.all(runk[j0:j1] == kk) and tiles[k, 4] == kk * (j1 - j0)
                     if kk >= 4:
                         assert opt_begin[k] % 4 == 0

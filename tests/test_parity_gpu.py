@@ -331,3 +331,37 @@ def test_programmatic_dependent_launch_is_transparent(graph):
         assert np.array_equal(getattr(sols[1], f), getattr(sols[0], f), equal_nan=True), f
     esp.esp_debug_set_pdl(s.ctx, -1)
     s.close()
+
+
+@pytest.mark.parametrize("case", ["whatif", "heavy", "ragged256", "k1", "k2", "r4k8", "r5k4"])
+def test_interleaved_tiles_equal_separate_arrays(case):
+    """The per-warp pass reads each tile's units and values with one bulk copy from a tile-interleaved
+    copy of the table (the default wherever every tile allows it) or with two copies from the separate
+    arrays: the same bits, round by round, and the oracle's at the end."""
+    rng = np.random.default_rng(13)
+    if case == "whatif":
+        t = W.whatif_batch(scenarios=[3, 40], J=1024).table
+    elif case == "heavy":
+        t = W.heavy_tail(scenarios=[1, 2], J=3000).table
+    elif case == "ragged256":
+        t = W.random_table(rng, S=3, J=500, R=6, kmin=1, kmax=256, umax=5000)
+    elif case in ("k1", "k2"):
+        K = int(case[1])
+        t = W.random_table(rng, S=2, J=2000, R=6, kmin=K, kmax=K, umax=5000)
+    elif case == "r4k8":
+        t = W.random_table(rng, S=2, J=900, R=4, kmin=8, kmax=8, umax=5000)
+    else:
+        t = W.random_table(rng, S=2, J=900, R=5, kmin=4, kmax=4, umax=5000)
+    a = esp.Solver(t)
+    b = esp.Solver()
+    esp.esp_debug_set_interleave(b.ctx, False)
+    b.load(t)
+    assert esp.esp_debug_pass_kernel(b.ctx) == 0
+    T = 30
+    sa = a.solve(0.05, T, traces=True)
+    sb = b.solve(0.05, T, traces=True)
+    for f in ("lam", "sel", "demand", "lambda_trace", "demand_trace", "selhash_trace"):
+        assert np.array_equal(getattr(sa, f), getattr(sb, f), equal_nan=True), f
+    check_solution(t, sa, list(range(t.S)), 0.05, T, esp.ESP_PRICE_NORMALIZED, esp.ESP_STEP_FIXED)
+    if case in ("whatif", "heavy", "ragged256", "r4k8", "r5k4"):
+        assert esp.esp_debug_pass_kernel(a.ctx) == 3, "the table should take the interleaved tiles"

@@ -96,7 +96,7 @@ def test_stream_pass_equals_per_warp_pass(name, make):
     T = 40
     a = streaming(t)
     b = streaming(t, stream=False)
-    assert esp.esp_debug_pass_kernel(a.ctx) == 1 and esp.esp_debug_pass_kernel(b.ctx) == 0
+    assert esp.esp_debug_pass_kernel(a.ctx) == 1 and esp.esp_debug_pass_kernel(b.ctx) in (0, 3)
     for flags in (0, esp.ESP_FLAG_EXACT_ONLY):
         sa = a.solve(0.03, T, flags=flags)
         sb = b.solve(0.03, T, flags=flags)
@@ -136,7 +136,7 @@ def test_stage_wait_timeout_reports_and_poisons(stream):
     bit-exactly."""
     t = uniform(21, 4, 2048, 6, 16)
     s = streaming(t, stream)
-    assert esp.esp_debug_pass_kernel(s.ctx) == (1 if stream else 0)
+    assert esp.esp_debug_pass_kernel(s.ctx) in ((1,) if stream else (0, 3))
     ref = s.solve(0.05, 10)
     esp.esp_debug_set_wait_limit(s.ctx, 20)
     esp.esp_debug_hold_stage(s.ctx)

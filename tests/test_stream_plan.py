@@ -119,17 +119,18 @@ def test_ineligible_tables_are_refused():
     check(p, np.arange(11, dtype=np.int64) * 12, 1, 10, None, None, 12)
 
 
-def test_sort_layout_k_matches_the_default_at_128():
+def test_sort_layout_k_default_and_256():
     rng = np.random.default_rng(4)
     S, J = 3, 500
     K = rng.integers(1, 300, size=S * J)
     off0 = np.zeros(S * J + 1, np.int64)
     off0[1:] = np.cumsum(K)
-    a = esp.sort_layout(off0, S, J)
+    a = esp.sort_layout(off0, S, J)            # the library's layout: runs of up to 128 options
     b = esp.sort_layout_k(off0, S, J, 128)
     for x, y in zip(a, b):
         assert np.array_equal(x, y)
-    # with 256: jobs of 129..256 options join padded runs, the others keep their places' rules
+    # with 256 (the streaming pass's runs): jobs of 129..256 options join padded runs, larger ones keep
+    # their size and no run
     off, jmap, scen, runk = esp.sort_layout_k(off0, S, J, 256)
     Kj = K[jmap]
     big = Kj > 256
