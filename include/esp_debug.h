@@ -81,9 +81,9 @@ esp_status esp_debug_resident(esp_ctx *ctx, int32_t force_cs, int32_t *cs, int32
  * ESP_ERR_UNSUPPORTED: no placement table is loaded, or it cannot run grid-resident. */
 esp_status esp_debug_hold_barrier(esp_ctx *ctx);
 
-/* Failure-detection hooks of the evaluation passes. esp_debug_set_wait_limit sets how long a bounded
- * wait of the per-warp and streaming passes polls, in milliseconds of the GPU's global timer, before it
- * gives up: limit_ms = 0 restores the default (4000); a test sets a few to make a timeout short. esp_debug_hold_stage makes the next esp_solve's first round pass announce 16 more
+/* Failure-detection hooks of the evaluation pass. esp_debug_set_wait_limit sets how long a bounded
+ * wait of the pass's stage ring polls, in milliseconds of the GPU's global timer, before it gives up:
+ * limit_ms = 0 restores the default (4000); a test sets a few to make a timeout short. esp_debug_hold_stage makes the next esp_solve's first round pass announce 16 more
  * bytes on the first stage of its first CTA (warp) than its copies bring, so that stage's barrier
  * phase never completes: no memory is accessed out of place, every wait on that phase runs out, and
  * the solve returns ESP_ERR_TIMEOUT; the context then answers ESP_ERR_STATE (destroy it; the device
@@ -95,37 +95,16 @@ esp_status esp_debug_hold_stage(esp_ctx *ctx);
  * very next) reports ESP_ERR_OOM as a failed cudaMalloc would; n < 0 disarms it. */
 esp_status esp_debug_fail_alloc(esp_ctx *ctx, int64_t n);
 
-/* enable = 0 makes later loads evaluate every table with the per-warp pass (k_pass); 1 restores the
- * default, the streaming pass (k_stream) for uniform tables and for ragged tables whose jobs have at
- * most 256 options. *kind (esp_debug_pass_kernel) receives the pass the loaded table uses: 1
- * streaming, 0 per-warp, 3 per-warp on the tile-interleaved table, 2 factored placement. Results are
- * identical either way. */
-esp_status esp_debug_set_stream_pass(esp_ctx *ctx, int32_t enable);
+/* *kind receives how the loaded table is evaluated: 0 the per-warp pass with two bulk copies per tile
+ * (units and values apart), 1 the per-warp pass with one bulk copy per tile (tile-interleaved table),
+ * 2 the factored placement pass. */
 esp_status esp_debug_pass_kernel(esp_ctx *ctx, int32_t *kind);
 
 /* enable = 0 makes later loads keep the per-warp pass's table as separate unit and value arrays (two
  * bulk copies per tile); 1 restores the default, a tile-interleaved copy (each tile's units then its
  * values, one bulk copy per tile) wherever every tile allows it (esp_debug_pass_kernel then reports
- * 3). Results are identical either way. */
+ * 1). Results are identical either way. */
 esp_status esp_debug_set_interleave(esp_ctx *ctx, int32_t enable);
-
-/* Runs the streaming pass's host planner (no GPU code) on CSR offsets (host, S*J + 1 int64): with
- * scen and runk (host, S*J int32 each, a sorted layout from esp_debug_sort_layout_k) or, with both
- * NULL, every job having uniform_k options; R stored columns, grid CTAs. Outputs (host buffers): the
- * blocks as tiles, tiles_cap * 8 int32 (as esp_debug_plan), cta_begin grid + 1 int32 (CTA c takes the
- * blocks [cta_begin[c], cta_begin[c + 1])), arrivals S int32 (blocks per scenario); the counts go
- * to *n_tiles and *n_ctas, and *stage_opt receives the options a stage (a block) holds at most.
- * Returns ESP_OK, ESP_ERR_INVALID_ARG (the table is not eligible, or the plan check failed) or
- * ESP_ERR_OOM (a buffer is too small; the counts are still written). */
-esp_status esp_debug_plan_stream(const int64_t *job_offsets, int32_t S, int32_t J, const int32_t *scen,
-                                 const int32_t *runk, int32_t uniform_k, int32_t R, int32_t grid, int32_t *tiles,
-                                 int32_t tiles_cap, int32_t *cta_begin, int32_t *arrivals, int32_t *n_tiles,
-                                 int32_t *n_ctas, int32_t *stage_opt);
-
-/* esp_debug_sort_layout with runs of up to run_max_k options (a multiple of 4: 128 is the per-warp
- * pass's layout, 256 the streaming pass's). */
-esp_status esp_debug_sort_layout_k(const int64_t *job_offsets, int32_t S, int32_t J, int32_t run_max_k, int64_t *off,
-                                   int32_t *jmap, int32_t *scen, int32_t *runk);
 
 #ifdef __cplusplus
 }

@@ -54,10 +54,6 @@ struct PlanCache {
     bool sorted = false;
     esp::SortedLayout lay;
     esp::Plan plan;
-    bool stream_enabled = false;   // the load that made this plan allowed the streaming pass
-    bool stream = false;           // ... and the table took it
-    int32_t stream_grid = 0;
-    esp::StreamPlan splan;
 };
 
 struct esp_ctx {
@@ -112,12 +108,7 @@ struct esp_ctx {
 
     TileDesc *tiles = nullptr;
     int32_t *warp_begin = nullptr;
-    // streaming pass (k_stream): per-CTA block ranges (the blocks are the tiles), when the loaded table
-    // takes it
-    bool stream_enabled = false;     // later loads may use the streaming pass (esp_debug_set_stream_pass)
     bool il_enabled = true;          // later loads may interleave the pass table (esp_debug_set_interleave)
-    bool stream_pass = false;
-    int32_t *cta_begin = nullptr;
     // failure-detection hooks (esp_debug.h): limit of a bounded wait of the evaluation passes in ms
     // (0: the default, 4 s), extra bytes announced on the next solve's first stage, allocations left
     // before an injected failure (-1: none)
@@ -277,8 +268,6 @@ void release_table(esp_ctx *ctx, bool keep = false)
     ctx->place_res_ok = false;
     ctx->res_auto = -1;
     ctx->res_force = -1;
-    ctx->stream_pass = false;
-    ctx->cta_begin = nullptr;
     ctx->loaded = false;
     ctx->solved = false;
 }
@@ -519,8 +508,7 @@ esp_status load_common(esp_ctx *ctx, int32_t S, int32_t J, int32_t R, int32_t P,
     // the plan of the previous load serves when the shape and offsets are the same
     PlanCache &pc = ctx->pc;
     const bool cached = pc.valid && pc.S == S && pc.J == J && pc.R == R && pc.P == P && pc.grouped == grouped &&
-                        pc.sorted_enabled == ctx->sorted_enabled && pc.stream_enabled == ctx->stream_enabled &&
-                        (int64_t)pc.off.size() == n_jobs + 1 &&
+                        pc.sorted_enabled == ctx->sorted_enabled && (int64_t)pc.off.size() == n_jobs + 1 &&
                         std::memcmp(pc.off.data(), off_host, (size_t)(n_jobs + 1) * sizeof(int64_t)) == 0;
     // option counts, on the host meanwhile: every job non-empty makes the offsets strictly
     // increasing up to n_opt, so no kernel below can index outside the table
@@ -545,10 +533,6 @@ esp_status load_common(esp_ctx *ctx, int32_t S, int32_t J, int32_t R, int32_t P,
 
     // plan the evaluation pass
     ctx->uniform_k = (!grouped && min_k == max_k && max_k <= 32 && (max_k & (max_k - 1)) == 0) ? (int32_t)max_k : 0;
-    // the streaming pass (k_stream) takes uniform tables and ragged tables whose jobs have at most
-    // kStreamRunMaxK options (through the sorted layout); every other table the per-warp pass
-    const bool stream_try = ctx->stream_enabled && !grouped && J >= 1 &&
-                            (ctx->uniform_k > 0 || (ctx->sorted_enabled && max_k <= kStreamRunMaxK));
 
     // general tables without a group column: the evaluation pass reads the sorted layout (runs of
     // equal-size jobs take the uniform paths). Jobs keep their option order, so the copy inherits
@@ -559,7 +543,7 @@ esp_status load_common(esp_ctx *ctx, int32_t S, int32_t J, int32_t R, int32_t P,
         use_sorted = pc.sorted;
     else
         use_sorted = ctx->sorted_enabled && !grouped && ctx->uniform_k == 0 && J >= 1 &&
-                     sort_layout(off_host, S, J, lay_new, stream_try ? kStreamRunMaxK : kRunMaxK);
+                     sort_layout(off_host, S, J, lay_new, kRunMaxK);
     const SortedLayout &lay = cached ? pc.lay : lay_new;
     if (use_sorted) {
         const int64_t sn = lay.off.back();
@@ -580,51 +564,36 @@ esp_status load_common(esp_ctx *ctx, int32_t S, int32_t J, int32_t R, int32_t P,
     const int32_t *plan_runk = ctx->sorted ? lay.runk.data() : nullptr;
 
     Plan plan_new;
-    StreamPlan splan_new;
-    bool plan_cached = false, stream = false;
-    int tile_opt = 0, max_warps = 0, s_grid = 0;
-    const int s_per_sm = stream_try ? stream_ctas_per_sm(R) : 0;
-    if (stream_try && s_per_sm >= 1 && (ctx->uniform_k > 0 || use_sorted)) {
-        s_grid = ctx->sm_count * std::min(s_per_sm, (int)ESP_STREAM_CTAS_PER_SM);
-        plan_cached = cached && pc.stream && pc.stream_grid == s_grid;
-        stream = plan_cached ||
-                 (plan_stream(plan_off, S, J, plan_scen, plan_runk, ctx->uniform_k, R, stream_stage_opt(R), s_grid,
-                              splan_new) &&
-                  check_stream_plan(plan_off, S, J, plan_scen, plan_runk, ctx->uniform_k, R, splan_new));
+    const int tile_opt = tile_options_for(R, grouped, max_k, ctx->uniform_k >= 4);
+    // a sorted layout's tiles are runs and chunks only (the sorted layout exists only without a group
+    // column): the runs-only instantiation
+    const int mode = ctx->uniform_k > 0 ? kModeUniform : (use_sorted && !grouped) ? kModeRuns : kModeGeneral;
+    const int per_sm = pass_ctas_per_sm(R, grouped, mode, P, tile_opt);
+    if (per_sm < 1) {
+        cudaStreamSynchronize(ctx->stream);
+        release_table(ctx);
+        return ESP_ERR_UNSUPPORTED;
     }
-    if (!stream) {
-        tile_opt = tile_options_for(R, grouped, max_k, ctx->uniform_k >= 4);
-        // a sorted layout's tiles are runs and chunks only (the sorted layout exists only without a
-        // group column): the runs-only instantiation
-        const int mode = ctx->uniform_k > 0 ? kModeUniform : (use_sorted && !grouped) ? kModeRuns : kModeGeneral;
-        const int per_sm = pass_ctas_per_sm(R, grouped, mode, P, tile_opt);
-        if (per_sm < 1) {
-            cudaStreamSynchronize(ctx->stream);
-            release_table(ctx);
-            return ESP_ERR_UNSUPPORTED;
-        }
-        // two waves of resident CTAs by default: CTAs that finish early take the second wave's ranges,
-        // which halves the pass's tail (measured: what-if batch -2.1%, heavy-tailed table -2.5%)
-        const int waves = ctx->plan_waves > 0 ? ctx->plan_waves : 2;
-        max_warps = ctx->sm_count * per_sm * kWarpsPerCta * waves;
-        plan_cached = cached && !pc.stream && pc.max_warps == max_warps && pc.tile_opt == tile_opt;
-        if (!plan_cached && (!plan_tiles(plan_off, S, J, tile_opt, max_warps, plan_new, plan_scen, plan_runk) ||
-                             !check_plan(plan_off, S, J, plan_new, plan_scen, plan_runk))) {
-            cudaStreamSynchronize(ctx->stream);
-            release_table(ctx);
-            return ESP_ERR_INVALID_ARG;
-        }
-        // the runs-only instantiation has no path for a general tile
-        if (mode == kModeRuns)
-            for (const TileDesc &d : (plan_cached ? pc.plan : plan_new).tiles)
-                if (!(d.flags & (TILE_RUN | TILE_BIG))) {
-                    cudaStreamSynchronize(ctx->stream);
-                    release_table(ctx);
-                    return ESP_ERR_INVALID_ARG;
-                }
+    // two waves of resident CTAs by default: CTAs that finish early take the second wave's ranges,
+    // which halves the pass's tail (measured: what-if batch -2.1%, heavy-tailed table -2.5%)
+    const int waves = ctx->plan_waves > 0 ? ctx->plan_waves : 2;
+    const int max_warps = ctx->sm_count * per_sm * kWarpsPerCta * waves;
+    const bool plan_cached = cached && pc.max_warps == max_warps && pc.tile_opt == tile_opt;
+    if (!plan_cached && (!plan_tiles(plan_off, S, J, tile_opt, max_warps, plan_new, plan_scen, plan_runk) ||
+                         !check_plan(plan_off, S, J, plan_new, plan_scen, plan_runk))) {
+        cudaStreamSynchronize(ctx->stream);
+        release_table(ctx);
+        return ESP_ERR_INVALID_ARG;
     }
     const Plan &plan = plan_cached ? pc.plan : plan_new;
-    const StreamPlan &splan = plan_cached ? pc.splan : splan_new;
+    // the runs-only instantiation has no path for a general tile
+    if (mode == kModeRuns)
+        for (const TileDesc &d : plan.tiles)
+            if (!(d.flags & (TILE_RUN | TILE_BIG))) {
+                cudaStreamSynchronize(ctx->stream);
+                release_table(ctx);
+                return ESP_ERR_INVALID_ARG;
+            }
     // the validation result (the copies, validation and duplicate marking ran during the planning)
     ESP_CUDA(cudaStreamSynchronize(ctx->stream));
     if (vflags != 0) {
@@ -637,22 +606,7 @@ esp_status load_common(esp_ctx *ctx, int32_t S, int32_t J, int32_t R, int32_t P,
             ctx->small_units = 0;
     ALLOC(ctx->scen_warps, (size_t)S);
     ALLOC(ctx->arrive, (size_t)S);
-    ctx->stream_pass = stream;
-    if (stream) {
-        ctx->n_warps = 0;
-        ctx->tile_opt = splan.stage_opt;
-        ctx->grid = splan.grid;
-        ALLOC(ctx->tiles, splan.tiles.size() + 1);
-        ALLOC(ctx->warp_begin, 1);
-        ALLOC(ctx->cta_begin, splan.cta_begin.size());
-        if (!splan.tiles.empty())
-            ESP_CUDA(cudaMemcpyAsync(ctx->tiles, splan.tiles.data(), splan.tiles.size() * sizeof(TileDesc),
-                                     cudaMemcpyHostToDevice, ctx->stream));
-        ESP_CUDA(cudaMemcpyAsync(ctx->cta_begin, splan.cta_begin.data(), splan.cta_begin.size() * sizeof(int32_t),
-                                 cudaMemcpyHostToDevice, ctx->stream));
-        ESP_CUDA(cudaMemcpyAsync(ctx->scen_warps, splan.arrivals.data(), (size_t)S * sizeof(int32_t),
-                                 cudaMemcpyHostToDevice, ctx->stream));
-    } else {
+    {
         ctx->n_warps = plan.n_warps;
         ctx->tile_opt = plan.tile_opt;
         ctx->grid = (plan.n_warps + kWarpsPerCta - 1) / kWarpsPerCta;
@@ -723,10 +677,6 @@ esp_status load_common(esp_ctx *ctx, int32_t S, int32_t J, int32_t R, int32_t P,
         pc.max_warps = max_warps;
         pc.tile_opt = tile_opt;
         pc.plan = std::move(plan_new);
-        pc.stream_enabled = ctx->stream_enabled;
-        pc.stream = stream;
-        pc.stream_grid = s_grid;
-        pc.splan = std::move(splan_new);
     }
     trim_pool(ctx);
     ctx->loaded = true;
@@ -773,8 +723,7 @@ bool state_ready(const esp_ctx *c)
     if (c->placement)
         return c->place.cfg_units && c->place.cfg_values && c->place.sens && c->place.job_type &&
                c->place.node_type && c->place.D && c->place.cfg_dup && c->place.warp_job && c->place.n_warps > 0;
-    return c->grid == 0 || (c->tiles && c->warp_begin && c->units && c->values && c->off &&
-                            (!c->stream_pass || c->cta_begin));
+    return c->grid == 0 || (c->tiles && c->warp_begin && c->units && c->values && c->off);
 }
 
 // The plan of the evaluation pass as the kernels take it.
@@ -788,7 +737,6 @@ DevPlan dev_plan(const esp_ctx *c, bool fused)
     pl.uniform_k = c->uniform_k;
     pl.runs_only = (c->sorted && c->group == nullptr) ? 1 : 0;
     pl.scen_warps = fused ? c->scen_warps : nullptr;
-    pl.cta_begin = c->stream_pass ? c->cta_begin : nullptr;
     return pl;
 }
 
@@ -1926,15 +1874,6 @@ esp_status esp_debug_fail_alloc(esp_ctx *ctx, int64_t n)
     return ESP_OK;
 }
 
-esp_status esp_debug_set_stream_pass(esp_ctx *ctx, int32_t enable)
-{
-    esp_status st = check_ctx(ctx);
-    if (st != ESP_OK)
-        return st;
-    ctx->stream_enabled = enable != 0;
-    return ESP_OK;
-}
-
 esp_status esp_debug_set_interleave(esp_ctx *ctx, int32_t enable)
 {
     esp_status st = check_ctx(ctx);
@@ -1953,58 +1892,7 @@ esp_status esp_debug_pass_kernel(esp_ctx *ctx, int32_t *kind)
         return ESP_ERR_INVALID_ARG;
     if (!ctx->loaded)
         return ESP_ERR_NOT_LOADED;
-    *kind = ctx->placement ? 2 : ctx->stream_pass ? 1 : ctx->il ? 3 : 0;
-    return ESP_OK;
-}
-
-esp_status esp_debug_plan_stream(const int64_t *job_offsets, int32_t S, int32_t J, const int32_t *scen,
-                                 const int32_t *runk, int32_t uniform_k, int32_t R, int32_t grid, int32_t *tiles,
-                                 int32_t tiles_cap, int32_t *cta_begin, int32_t *arrivals, int32_t *n_tiles,
-                                 int32_t *n_ctas, int32_t *stage_opt)
-{
-    if (!job_offsets || S < 1 || J < 0 || R < 1 || R > kMaxR || grid < 1 || (!scen) != (!runk) || !n_tiles ||
-        !n_ctas || !stage_opt)
-        return ESP_ERR_INVALID_ARG;
-    StreamPlan p;
-    const int32_t so = stream_stage_opt(R);
-    if (!plan_stream(job_offsets, S, J, scen, runk, uniform_k, R, so, grid, p) ||
-        !check_stream_plan(job_offsets, S, J, scen, runk, uniform_k, R, p))
-        return ESP_ERR_INVALID_ARG;
-    *n_tiles = (int32_t)p.tiles.size();
-    *n_ctas = p.grid;
-    *stage_opt = so;
-    if ((int32_t)p.tiles.size() > tiles_cap || !tiles || !cta_begin || !arrivals)
-        return ESP_ERR_OOM;
-    for (size_t i = 0; i < p.tiles.size(); ++i) {
-        const TileDesc &d = p.tiles[i];
-        int32_t *w = tiles + 8 * i;
-        w[0] = (int32_t)(uint32_t)(d.opt_begin & 0xffffffff);
-        w[1] = (int32_t)(d.opt_begin >> 32);
-        w[2] = (int32_t)(uint32_t)(d.job_begin & 0xffffffff);
-        w[3] = (int32_t)(d.job_begin >> 32);
-        w[4] = d.n_opt;
-        w[5] = d.n_job;
-        w[6] = d.scenario;
-        w[7] = (int32_t)d.flags;
-    }
-    std::memcpy(cta_begin, p.cta_begin.data(), p.cta_begin.size() * sizeof(int32_t));
-    std::memcpy(arrivals, p.arrivals.data(), p.arrivals.size() * sizeof(int32_t));
-    return ESP_OK;
-}
-
-esp_status esp_debug_sort_layout_k(const int64_t *job_offsets, int32_t S, int32_t J, int32_t run_max_k, int64_t *off,
-                                   int32_t *jmap, int32_t *scen, int32_t *runk)
-{
-    if (!job_offsets || !off || !jmap || !scen || !runk || S < 1 || J < 1 || run_max_k < 4 || (run_max_k & 3) ||
-        run_max_k > 4096)
-        return ESP_ERR_INVALID_ARG;
-    SortedLayout lay;
-    if (!sort_layout(job_offsets, S, J, lay, run_max_k))
-        return ESP_ERR_INVALID_ARG;
-    std::memcpy(off, lay.off.data(), lay.off.size() * sizeof(int64_t));
-    std::memcpy(jmap, lay.jmap.data(), lay.jmap.size() * sizeof(int32_t));
-    std::memcpy(scen, lay.scen.data(), lay.scen.size() * sizeof(int32_t));
-    std::memcpy(runk, lay.runk.data(), lay.runk.size() * sizeof(int32_t));
+    *kind = ctx->placement ? 2 : ctx->il ? 1 : 0;
     return ESP_OK;
 }
 

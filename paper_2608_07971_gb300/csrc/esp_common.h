@@ -61,25 +61,6 @@ namespace esp {
 #define ESP_I2F_COLS 16       // unit columns r < ESP_I2F_COLS use the int-to-float instruction
 #endif
 
-#ifndef ESP_STREAM_CONSUMERS
-#define ESP_STREAM_CONSUMERS 12   // consumer warps per CTA of the streaming pass (plus one producer warp)
-#endif
-#ifndef ESP_STREAM_SMEM
-#define ESP_STREAM_SMEM 200704    // dynamic shared memory budget of a streaming-pass CTA (stages + barriers)
-#endif
-#ifndef ESP_STREAM_MAX_STAGES
-#define ESP_STREAM_MAX_STAGES 32  // most stages of the streaming pass's copy ring (one block each)
-#endif
-#ifndef ESP_STREAM_STAGE_OPT
-#define ESP_STREAM_STAGE_OPT 256  // options one stage holds (a multiple of 128, at least 256)
-#endif
-#ifndef ESP_STREAM_PRODUCERS
-#define ESP_STREAM_PRODUCERS 2    // producer warps per CTA of the streaming pass (each issues every P-th block)
-#endif
-#ifndef ESP_STREAM_CTAS_PER_SM
-#define ESP_STREAM_CTAS_PER_SM 1  // CTAs per SM the streaming pass is planned for (limited by its shared memory)
-#endif
-
 constexpr int kMaxR = 16;            // stored resource columns per option
 constexpr int kWarpsPerCta = ESP_WARPS_PER_CTA;  // warps of a CTA; each warp owns its own stage ring
 constexpr int kStages = ESP_STAGES;  // TMA stages per warp
@@ -143,65 +124,10 @@ ESP_HD uint32_t tile_run_flags(int k) { return TILE_RUN | ((uint32_t)k << 8); }
 #define ESP_RUN_MAX_K 128
 #endif
 constexpr int kRunMaxK = ESP_RUN_MAX_K;
-// The streaming pass's runs take up to 256 options per job (two groups of four options per lane).
-constexpr int kStreamRunMaxK = 256;
 // Largest run tile of the per-warp pass (rows of whole jobs of up to 32 lanes x 4 options); a padded
 // job above it is planned as chunks.
 constexpr int kPassRunMaxK = 128;
 
-// ---------------------------------------------------------------------------------------------
-// Streaming pass (k_stream): per CTA kStreamProducers producer warps fill a ring of stream_stages()
-// stages by bulk copies, one block per stage, and kStreamConsumers consumer warps evaluate them. A
-// block is whole jobs of one run and scenario, at most a stage's options, described by one TileDesc
-// (flags: TILE_RUN and the jobs' option count); each block is taken by one consumer warp (the next
-// free one: a shared counter), which releases its stage alone.
-constexpr int kStreamConsumers = ESP_STREAM_CONSUMERS;
-constexpr int kStreamProducers = ESP_STREAM_PRODUCERS;
-
-// Options a stage holds (the same for every R): a multiple of 128, at least 256 (a whole job of the
-// largest run).
-ESP_HD int stream_stage_opt(int R)
-{
-    (void)R;
-    const int t = ESP_STREAM_STAGE_OPT & ~127;
-    return t < 256 ? 256 : t;
-}
-
-// Byte layout of one stage: the block's descriptor (32 bytes) and the block's index in its CTA's
-// range (the stage's sequence word), the units and the values; the regions have room for the up-to-15
-// bytes the bulk copies read before and after their data to keep both ends 16-byte aligned.
-struct StreamStageLayout {
-    int hdr, seq, units, vals, bytes;
-};
-
-ESP_HD StreamStageLayout stream_stage_layout(int stage_opt, int R)
-{
-    StreamStageLayout L;
-    L.hdr = 0;
-    L.seq = 32;
-    L.units = 48;
-    L.vals = L.units + round16(stage_opt * R * 4 + 32);
-    L.bytes = (L.vals + round16(stage_opt * 8 + 32) + 127) & ~127;
-    return L;
-}
-
-// Stages of the ring for R stored columns: as many as the shared-memory budget holds, at most
-// ESP_STREAM_MAX_STAGES, a multiple of kStreamProducers (stage s is filled only by producer
-// s % kStreamProducers, so each stage's blocks are issued in order by one warp).
-ESP_HD int stream_stages(int stage_opt, int R)
-{
-    int n = (ESP_STREAM_SMEM - 16) / (stream_stage_layout(stage_opt, R).bytes + 16);
-    n = n > ESP_STREAM_MAX_STAGES ? ESP_STREAM_MAX_STAGES : n;
-    return n - n % kStreamProducers;
-}
-
-// Dynamic shared memory of a CTA of the streaming pass: the stages, then a full and an empty
-// barrier per stage, then the consumers' block counter.
-ESP_HD int stream_smem_bytes(int stage_opt, int R)
-{
-    const int n = stream_stages(stage_opt, R);
-    return n * stream_stage_layout(stage_opt, R).bytes + 16 * n + 16;
-}
 
 struct TileDesc {
     int64_t opt_begin;    // first global option of the tile

@@ -203,10 +203,6 @@ __global__ void __launch_bounds__(kWarpsPerCta * 32, pass_min_ctas<RT, MODE>()) 
     for (int r = 0; r < Cols<RT>::N; ++r)
         c.acc[r] = 0;
     c.hacc = 0;
-    c.defer = false;
-    c.pend_s = -1;
-    c.count_tiles = false;
-    c.ntiles = 0;
 
     if (lane == 0) {
         for (int s = 0; s < kStages; ++s)
@@ -291,7 +287,7 @@ __global__ void __launch_bounds__(kWarpsPerCta * 32, pass_min_ctas<RT, MODE>()) 
             else if (d.flags & TILE_BIG)
                 process_tile_bigchunk<RT, G>(c, d, ptrs, big_first, big_priv, lane);
             else if (!G && (d.flags & TILE_RUN) && tile_run_k(d.flags) >= 4)
-                process_tile_run4<RT, G, 1>(c, d, ptrs, lane, tile_run_k(d.flags));
+                process_tile_run4<RT, G>(c, d, ptrs, lane, tile_run_k(d.flags));
             else if (!G && (d.flags & TILE_RUN))
                 process_tile_uniform<RT, G>(c, d, ptrs, lane, tile_run_k(d.flags), tile_run_k(d.flags) >> 1);
             else if (MODE == kModeGeneral)
@@ -448,8 +444,6 @@ cudaError_t launch_init(const DevTable &t, const DevState &st, const SolveArgs &
 cudaError_t launch_pass(const DevTable &t, const DevState &st, const DevPlan &pl, const SolveArgs &a, int round,
                         PassKind kind, int grid, cudaStream_t stream, bool pdl)
 {
-    if (pl.cta_begin)
-        return launch_stream(t, st, pl, a, round, kind, grid, stream, pdl);
     const bool grouped = t.group != nullptr;
     const int mode = pass_mode(pl);
     const int smem = pass_smem_bytes(t.R, grouped, mode, t.P, pl.tile_opt);

@@ -60,11 +60,7 @@ struct DevPlan {
     int32_t tile_opt;
     int32_t uniform_k;          // > 0: every job has exactly this many options, a power of two <= 32
     int32_t runs_only;          // 1: every tile is a run of equal-size jobs or a chunk of a large job
-    const int32_t *scen_warps;  // S arrivals that complete each scenario in a round pass (one per warp and
-                                // maximal run of the scenario's tiles); non-null: round passes update prices
-    // streaming pass (k_stream) when cta_begin is non-null: every tile is one block, and CTA c
-    // evaluates the tiles [cta_begin[c], cta_begin[c + 1]); tile_opt then holds the options of a stage
-    const int32_t *cta_begin;
+    const int32_t *scen_warps;  // S warps owning tiles of each scenario; non-null: round passes update prices
 };
 
 struct SolveArgs {
@@ -75,7 +71,7 @@ struct SolveArgs {
     int32_t exact_only;
     uint32_t wait_ms;         // limit of a bounded stage wait, ms of the global timer (kWaitLimitMs: 4 s)
     uint32_t hold_tx;         // test hook, 0 normally: extra bytes announced on the first stage of the first
-                              // round pass (CTA 0), so that stage's phase never completes and its waits time out
+                              // round pass (warp 0), so that stage's phase never completes and its waits time out
 };
 
 enum PassKind : int32_t { PASS_ROUND = 0, PASS_FINAL = 1 };
@@ -188,13 +184,6 @@ inline int pass_mode(const DevPlan &pl)
 
 // Dynamic shared memory per CTA of the evaluation kernel.
 int pass_smem_bytes(int R, bool grouped, int mode, int P, int tile_opt);
-
-// Resident CTAs per SM of the streaming pass for R stored columns (0 if it cannot run); sets the
-// kernels' shared-memory attribute, so it runs (at load time) before their first launch.
-int stream_ctas_per_sm(int R);
-// One streaming pass (pl.cta_begin non-null) over `grid` CTAs.
-cudaError_t launch_stream(const DevTable &t, const DevState &st, const DevPlan &pl, const SolveArgs &a, int round,
-                          PassKind kind, int grid, cudaStream_t stream, bool pdl);
 
 // Maximum resident CTAs per SM of the evaluation kernel for this table shape (0 if it cannot run).
 int pass_ctas_per_sm(int R, bool grouped, int mode, int P, int tile_opt);

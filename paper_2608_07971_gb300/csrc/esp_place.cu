@@ -233,10 +233,6 @@ __global__ void __launch_bounds__(kPlaceWarps * 32, 4) k_place(DevTable t, DevSt
     for (int r = 0; r < Cols<RT>::N; ++r)
         c.acc[r] = 0;
     c.hacc = 0;
-    c.defer = false;
-    c.pend_s = -1;
-    c.count_tiles = false;
-    c.ntiles = 0;
     place_jobs<RT>(c, pl, ws, pl.warp_job[w], pl.warp_job[w + 1], lane);
 }
 

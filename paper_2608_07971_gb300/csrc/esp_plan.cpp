@@ -278,149 +278,4 @@ bool sort_layout(const int64_t *off, int32_t S, int32_t J, SortedLayout &out, in
     return (int64_t)out.jmap.size() == n_jobs;
 }
 
-int32_t stream_row_jobs(int64_t K)
-{
-    if (K < 1 || K > kStreamRunMaxK)
-        return 0;
-    if (K < 4)
-        return (int32_t)(128 / K);
-    if (K & 3)
-        return 0;
-    const int64_t m = K / 4;
-    if (m > 32)
-        return 1;
-    int32_t lanes = 1;
-    while (lanes < m)
-        lanes <<= 1;
-    return 32 / lanes;
-}
-
-// Jobs of one block of a run of K options: the most whole rows (stream_row_jobs) that fit a stage.
-static int64_t stream_block_jobs(int64_t K, int32_t stage_opt)
-{
-    const int64_t row = stream_row_jobs(K);
-    const int64_t rows = std::max<int64_t>(1, stage_opt / (row * K));
-    return std::min<int64_t>(row * rows, stage_opt / K);
-}
-
-// Estimated cost of a block for the CTA split: its option bytes plus a fixed part (the consumer's
-// per-block bookkeeping), in bytes of streamed table.
-static int64_t block_cost(const TileDesc &b, int32_t R)
-{
-    return (int64_t)b.n_opt * (4 * R + 8) + 512;
-}
-
-bool plan_stream(const int64_t *off, int32_t S, int32_t J, const int32_t *scen, const int32_t *runk,
-                 int32_t uniform_k, int32_t R, int32_t stage_opt, int32_t grid, StreamPlan &out)
-{
-    out = StreamPlan();
-    out.stage_opt = stage_opt;
-    const int64_t n_jobs = (int64_t)S * J;
-    if (S < 1 || J < 0 || R < 1 || grid < 1 || stage_opt < kStreamRunMaxK || (stage_opt & 127))
-        return false;
-    if (!runk && !(uniform_k >= 1 && stream_row_jobs(uniform_k) > 0))
-        return false;
-    if (off[0] != 0)
-        return false;
-    out.arrivals.assign((size_t)S, 0);
-    if (n_jobs == 0) {
-        out.grid = 0;
-        out.cta_begin.assign(1, 0);
-        return true;
-    }
-
-    // 1. blocks: whole jobs of one run and scenario, up to a stage's options in whole rows
-    int32_t s_cur = 0;
-    int64_t s_end = J;
-    int64_t j = 0;
-    while (j < n_jobs) {
-        while (!scen && j >= s_end) {
-            ++s_cur;
-            s_end += J;
-        }
-        const int32_t s = scen ? scen[j] : s_cur;
-        if (s < 0 || s >= S)
-            return false;
-        const int64_t K = runk ? runk[j] : uniform_k;
-        if (stream_row_jobs(K) < 1 || off[j + 1] - off[j] != K)
-            return false;
-        if (K >= 4 && (off[j] & 3))
-            return false;
-        const int64_t per = stream_block_jobs(K, stage_opt);
-        const int64_t jlim = scen ? n_jobs : std::min<int64_t>(n_jobs, s_end);
-        int64_t jj = j;
-        while (jj < jlim && jj - j < per && (!scen || scen[jj] == s) && (!runk || runk[jj] == K) &&
-               off[jj + 1] - off[jj] == K)
-            ++jj;
-        TileDesc d;
-        d.opt_begin = off[j];
-        d.job_begin = j;
-        d.n_opt = (int32_t)(off[jj] - off[j]);
-        d.n_job = (int32_t)(jj - j);
-        d.scenario = s;
-        d.flags = tile_run_flags((int)K);
-        out.tiles.push_back(d);
-        ++out.arrivals[s];
-        j = jj;
-    }
-    if (out.tiles.size() >= (size_t)INT32_MAX)
-        return false;
-
-    // 2. CTAs: contiguous block ranges of about equal estimated cost
-    const int64_t nb = (int64_t)out.tiles.size();
-    std::vector<int64_t> pre(nb + 1, 0);
-    for (int64_t b = 0; b < nb; ++b)
-        pre[b + 1] = pre[b] + block_cost(out.tiles[b], R);
-    const int32_t G = (int32_t)std::min<int64_t>(grid, nb);
-    out.grid = G;
-    out.cta_begin.assign(G + 1, 0);
-    out.cta_begin[G] = (int32_t)nb;
-    for (int32_t c = 1; c < G; ++c) {
-        const int64_t target = (int64_t)((__int128)pre[nb] * c / G);
-        int64_t b = std::lower_bound(pre.begin(), pre.end(), target) - pre.begin();
-        if (b > 0 && target - pre[b - 1] < pre[b] - target)
-            --b;
-        b = std::min<int64_t>(std::max<int64_t>(b, out.cta_begin[c - 1]), nb);
-        out.cta_begin[c] = (int32_t)b;
-    }
-    return true;
-}
-
-bool check_stream_plan(const int64_t *off, int32_t S, int32_t J, const int32_t *scen, const int32_t *runk,
-                       int32_t uniform_k, int32_t R, const StreamPlan &p)
-{
-    (void)R;
-    const int64_t n_jobs = (int64_t)S * J;
-    if ((int32_t)p.arrivals.size() != S || (int32_t)p.cta_begin.size() != p.grid + 1)
-        return false;
-    std::vector<int32_t> arr((size_t)S, 0);
-    int64_t next_job = 0;
-    for (const TileDesc &d : p.tiles) {
-        if (!(d.flags & TILE_RUN) || d.n_job < 1 || d.job_begin != next_job || d.job_begin + d.n_job > n_jobs)
-            return false;
-        const int64_t K = tile_run_k(d.flags);
-        if (stream_row_jobs(K) < 1 || d.opt_begin != off[d.job_begin] || d.n_opt > p.stage_opt ||
-            off[d.job_begin + d.n_job] - d.opt_begin != (int64_t)d.n_opt || (int64_t)d.n_opt != K * d.n_job)
-            return false;
-        if (K >= 4 && (d.opt_begin & 3))
-            return false;
-        for (int64_t j = d.job_begin; j < d.job_begin + d.n_job; ++j) {
-            const int64_t s = scen ? scen[j] : j / J;
-            const int64_t k = runk ? runk[j] : uniform_k;
-            if (s != d.scenario || k != K || off[j + 1] - off[j] != K)
-                return false;
-        }
-        ++arr[d.scenario];
-        next_job = d.job_begin + d.n_job;
-    }
-    if (next_job != n_jobs)
-        return false;
-    if (p.cta_begin.front() != 0 || p.cta_begin.back() != (int32_t)p.tiles.size())
-        return false;
-    for (int32_t c = 0; c < p.grid; ++c)
-        if (p.cta_begin[c] > p.cta_begin[c + 1])
-            return false;
-    return arr == p.arrivals;
-}
-
 }  // namespace esp

@@ -45,34 +45,10 @@ struct SortedLayout {
 };
 
 // Returns false when the table is not eligible (more than 2^31 - 1 jobs, or inconsistent offsets).
-// run_max_k: the largest padded job of the runs (kRunMaxK for the per-warp pass, kStreamRunMaxK for
-// the streaming pass).
+// run_max_k: the largest padded job of the runs (a multiple of 4; the library uses kRunMaxK).
 bool sort_layout(const int64_t *job_off, int32_t S, int32_t J, SortedLayout &out, int32_t run_max_k = kRunMaxK);
 
-// Plan of the streaming pass (k_stream): blocks of whole jobs of one run and scenario, at most a
-// stage's options (each block one TileDesc with flags tile_run_flags(K)), and a contiguous range of
-// blocks per CTA.
-struct StreamPlan {
-    std::vector<TileDesc> tiles;      // the blocks, in table order
-    std::vector<int32_t> cta_begin;   // grid + 1
-    std::vector<int32_t> arrivals;    // S: blocks per scenario (the count that completes it in a round pass)
-    int32_t grid = 0;
-    int32_t stage_opt = 0;
-};
 
-// Plans the streaming pass. Every job must belong to a run: runk[j] (sorted layout) or uniform_k for
-// every job (scen and runk NULL, uniform_k > 0); a run of K options takes 4m-option jobs (K a
-// multiple of 4, at most kStreamRunMaxK) or jobs of 1 to 3 options. stage_opt: options a stage holds;
-// grid: CTAs. Returns false when the table is not eligible (a job outside such a run, a run of 4 or
-// more options not starting on a 4-option boundary) or inconsistent.
-bool plan_stream(const int64_t *job_off, int32_t S, int32_t J, const int32_t *scen, const int32_t *runk,
-                 int32_t uniform_k, int32_t R, int32_t stage_opt, int32_t grid, StreamPlan &out);
-
-// Checks a stream plan against the table: blocks cover every job once, in order, each a whole number
-// of jobs of one run and scenario within a stage; CTA ranges cover the blocks; the arrival counts are
-// the scenarios' block counts.
-bool check_stream_plan(const int64_t *job_off, int32_t S, int32_t J, const int32_t *scen, const int32_t *runk,
-                       int32_t uniform_k, int32_t R, const StreamPlan &p);
 
 // Slices of the cluster-resident kernel: every scenario's jobs split into cs contiguous runs of about
 // equal option counts, run c starting at the first job whose first option lies at least

@@ -368,45 +368,30 @@ __device__ void process_tile_uniform4(WarpCtx<RT, G> &c, const TileDesc &d, cons
     }
 }
 
-// Exact resolution inside a row of a run with NG groups of 4 options per lane: every lane of an
-// ambiguous job screens its 4 NG options again (the same instructions give the same q) and rescores
-// in fp64 its survivors (q <= thr; every option but the duplicates in exact mode), in increasing index
-// order, then an xor butterfly over the job's L lanes keeps the lexicographic minimum of (s, job-local
-// index), and the lane holding that option records it. base[g]: tile-local index of the lane's group
-// g; loc[g]: its job-local index; valid[g]: the group holds data (jl: the job's index in the tile,
-// sub: the lane's place in the job); lamb: the lane's job is ambiguous.
-template <int RT, bool G, int NG>
-__device__ __forceinline__ void resolve_groups_in_row(WarpCtx<RT, G> &c, const StagePtrs &sp, bool lamb, float thr, int jl,
-                                                   int K, int sub, int n_job, int64_t job, int L)
+// Exact resolution inside a row of a run: every lane of an ambiguous job screens its 4 options again
+// (the same instructions give the same q) and rescores in fp64 its survivors (q <= thr; every option
+// but the duplicates in exact mode), in increasing index order, then an xor butterfly over the job's L
+// lanes keeps the lexicographic minimum of (s, job-local index), and the lane holding that option
+// records it. base: tile-local index of the lane's first option; loc: its job-local index; lamb: the
+// lane's job is ambiguous.
+template <int RT, bool G>
+__device__ __forceinline__ void resolve_run_row(WarpCtx<RT, G> &c, const StagePtrs &sp, bool lamb, float thr,
+                                                int base, int loc, int64_t job, int L)
 {
-    const int m = K >> 2;
-    int base[NG], loc[NG];
-    bool valid[NG];
-#pragma unroll
-    for (int g = 0; g < NG; ++g) {
-        loc[g] = 4 * (sub + 32 * g);
-        valid[g] = jl < n_job && (sub + 32 * g) < m;
-        base[g] = jl * K + loc[g];
-    }
     long long key = 0x7fffffffffffffffLL;
     int bi = kIdxNone;
     if (lamb) {
-#pragma unroll
-        for (int g = 0; g < NG; ++g) {
-            if (!valid[g])
+        for (int o = 0; o < 4; ++o) {
+            int32_t u[Cols<RT>::N];
+            if (load_units_smem<RT>(sp.units + (size_t)(base + o) * c.R, u, c.R))
                 continue;
-            for (int o = 0; o < 4; ++o) {
-                int32_t u[Cols<RT>::N];
-                if (load_units_smem<RT>(sp.units + (size_t)(base[g] + o) * c.R, u, c.R))
-                    continue;
-                const double v = sp.vals[base[g] + o];
-                if (!c.sp.exact && !(screen_score<RT, G>(u, v, 0, c.sp, c.R, c.rg) <= thr))
-                    continue;
-                const long long k = order_key(exact_score<RT, G>(u, v, 0, c.sp, c.R, c.rg));
-                if (k < key) {
-                    key = k;
-                    bi = loc[g] + o;
-                }
+            const double v = sp.vals[base + o];
+            if (!c.sp.exact && !(screen_score<RT, G>(u, v, 0, c.sp, c.R, c.rg) <= thr))
+                continue;
+            const long long k = order_key(exact_score<RT, G>(u, v, 0, c.sp, c.R, c.rg));
+            if (k < key) {
+                key = k;
+                bi = loc + o;
             }
         }
     }
@@ -418,63 +403,52 @@ __device__ __forceinline__ void resolve_groups_in_row(WarpCtx<RT, G> &c, const S
             bi = oi;
         }
     }
-    if (lamb) {
-#pragma unroll
-        for (int g = 0; g < NG; ++g) {
-            if (valid[g] && bi >= loc[g] && bi < loc[g] + 4) {
-                const int i = base[g] + (bi - loc[g]);
-                int32_t uw[Cols<RT>::N];
-                load_units_smem<RT>(sp.units + (size_t)i * c.R, uw, c.R);
-                take_winner<RT, G>(c, job, bi, uw, sp.vals[i], 0, true, key_value(key));
-                atomicAdd(c.st.stats, 1ull);
-            }
-        }
+    if (lamb && bi >= loc && bi < loc + 4) {
+        const int i = base + (bi - loc);
+        int32_t uw[Cols<RT>::N];
+        load_units_smem<RT>(sp.units + (size_t)i * c.R, uw, c.R);
+        take_winner<RT, G>(c, job, bi, uw, sp.vals[i], 0, true, key_value(key));
+        atomicAdd(c.st.stats, 1ull);
     }
 }
 
-// Tile of a run whose jobs all have K = 4m options, m <= 32 NG (NG = 1: up to 128 options, NG = 2:
-// up to 256). A job owns L = 2^ceil(log2 m) lanes (32 when NG = 2); lane `sub` of a job screens its
-// options 4 (sub + 32 g) .. 4 (sub + 32 g) + 3 for g < NG (16-byte shared loads: the run starts on a
-// 4-option boundary) and folds them, in increasing index order, into its smallest value (with its
+// Tile of a run whose jobs all have K = 4m options, m <= 32. A job owns L = 2^ceil(log2 m) lanes;
+// lane `sub` of a job screens its options 4 sub .. 4 sub + 3 (16-byte shared loads: the run starts on
+// a 4-option boundary) and folds them, in increasing index order, into its smallest value (with its
 // index) and second-smallest value; lanes past the job's end idle. A log2(L)-step xor butterfly of
 // (smallest, second smallest) completes the job as in the uniform path; an unambiguous job's winner
 // is the unique option holding the smallest value, recorded by the lane that holds it.
-template <int RT, bool G, int NG>
+template <int RT, bool G>
 __device__ void process_tile_run4(WarpCtx<RT, G> &c, const TileDesc &d, const StagePtrs &sp, int lane, int K)
 {
     const int R = c.R;
     const int m = K >> 2;
-    const int log2L = NG == 1 ? 32 - __clz(m - 1) : 5;
+    const int log2L = 32 - __clz(m - 1);
     const int L = 1 << log2L;
     const int jobs_per_row = 32 >> log2L;
     const int jslot = lane >> log2L, sub = lane & (L - 1);
     const int n_job = d.n_job;
     for (int jb = 0; jb < n_job; jb += jobs_per_row) {
         const int jl = jb + jslot;
-        int base[NG], loc[NG];
-        bool valid[NG];
+        const int loc = 4 * sub;
+        const bool valid = jl < n_job && sub < m;
+        const int base = jl * K + loc;
         float m1 = INFINITY, m2 = INFINITY;
         int i1 = kIdxNone;
+        if (valid) {
+            int32_t u[4][Cols<RT>::N];
+            bool dup[4];
+            load_units4_smem<RT>(sp.units + (size_t)base * R, u, dup, R);
+            const double2 va = reinterpret_cast<const double2 *>(sp.vals + base)[0];
+            const double2 vb = reinterpret_cast<const double2 *>(sp.vals + base)[1];
+            const double v[4] = {va.x, va.y, vb.x, vb.y};
 #pragma unroll
-        for (int g = 0; g < NG; ++g) {
-            loc[g] = 4 * (sub + 32 * g);
-            valid[g] = jl < n_job && (sub + 32 * g) < m;
-            base[g] = jl * K + loc[g];
-            if (valid[g]) {
-                int32_t u[4][Cols<RT>::N];
-                bool dup[4];
-                load_units4_smem<RT>(sp.units + (size_t)base[g] * R, u, dup, R);
-                const double2 va = reinterpret_cast<const double2 *>(sp.vals + base[g])[0];
-                const double2 vb = reinterpret_cast<const double2 *>(sp.vals + base[g])[1];
-                const double v[4] = {va.x, va.y, vb.x, vb.y};
-#pragma unroll
-                for (int o = 0; o < 4; ++o) {
-                    const float q = dup[o] ? INFINITY : screen_score<RT, G>(u[o], v[o], 0, c.sp, R, c.rg);
-                    const bool better = q < m1;
-                    m2 = better ? m1 : fminf(m2, q);
-                    i1 = better ? loc[g] + o : i1;
-                    m1 = fminf(m1, q);
-                }
+            for (int o = 0; o < 4; ++o) {
+                const float q = dup[o] ? INFINITY : screen_score<RT, G>(u[o], v[o], 0, c.sp, R, c.rg);
+                const bool better = q < m1;
+                m2 = better ? m1 : fminf(m2, q);
+                i1 = better ? loc + o : i1;
+                m1 = fminf(m1, q);
             }
         }
         const float lm1 = m1;
@@ -486,17 +460,16 @@ __device__ void process_tile_run4(WarpCtx<RT, G> &c, const TileDesc &d, const St
         }
         const float thr = __fadd_ru(m1, c.sp.e2);
         const bool amb = c.sp.exact || !(m2 > thr);
-        const bool lvalid = valid[0];
         const int64_t job = d.job_begin + jl;
-        if (lvalid && !amb && lm1 == m1) {
+        if (valid && !amb && lm1 == m1) {
             const int i = jl * K + i1;
             int32_t uw[Cols<RT>::N];
             load_units_smem<RT>(sp.units + (size_t)i * R, uw, R);
             take_winner<RT, G>(c, job, i1, uw, sp.vals[i], 0, false, 0.0);
         }
-        const bool lamb = lvalid && amb;
+        const bool lamb = valid && amb;
         if (__any_sync(FULL, lamb))
-            resolve_groups_in_row<RT, G, NG>(c, sp, lamb, thr, jl, K, sub, n_job, job, L);
+            resolve_run_row<RT, G>(c, sp, lamb, thr, base, loc, job, L);
     }
 }
 

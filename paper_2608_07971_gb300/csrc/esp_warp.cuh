@@ -280,35 +280,13 @@ struct WarpCtx {
     ScenarioPrices sp;
     long long acc[Cols<RT>::N];   // per-lane demand of the globally priced columns
     unsigned long long hacc;
-    bool defer;               // the last arriver of a scenario leaves its price update pending (pend_s)
-    int pend_s;               // scenario whose price update is pending, -1: none
-    bool count_tiles;         // arrivals count tiles (scen_warps: tiles per scenario) instead of warps
-    unsigned int ntiles;      // tiles of the current scenario evaluated since the last flush
 };
 
-// Eq. price_update of scenario s by this warp, once every warp of the pass has arrived for it.
 template <int RT, bool G>
-__device__ __forceinline__ void apply_update(WarpCtx<RT, G> &c, int s, int lane)
+__device__ void flush(WarpCtx<RT, G> &c, int lane)
 {
-    update_scenario<G ? 8 : 1>(c.t, c.st, c.a, s, c.round, lane);
-    if (lane == 0)
-        c.st.arrive[s] = 0u;     // every warp of this pass has arrived
-}
-
-// Runs the pending price update, if any (a warp that defers updates calls this once it has released
-// the stage it was evaluating).
-template <int RT, bool G>
-__device__ __forceinline__ void run_pending(WarpCtx<RT, G> &c, int lane)
-{
-    if (c.pend_s >= 0) {
-        apply_update(c, c.pend_s, lane);
-        c.pend_s = -1;
-    }
-}
-
-template <int RT, bool G>
-__device__ void flush_demand(WarpCtx<RT, G> &c, int lane)
-{
+    if (c.s < 0)
+        return;
     const int ncol = G ? c.rg : c.R;
     unsigned long long *dst = (c.kind == PASS_ROUND ? c.st.U : c.st.U_final) + (size_t)c.s * c.t.P;
 #pragma unroll
@@ -340,32 +318,17 @@ __device__ void flush_demand(WarpCtx<RT, G> &c, int lane)
             __syncwarp();
             __threadfence();
         }
-        const unsigned int inc = c.count_tiles ? c.ntiles : 1u;
         unsigned int old = 0;
         if (lane == 0)
-            asm volatile("atom.add.release.gpu.u32 %0, [%1], %2;" : "=r"(old) : "l"(c.st.arrive + c.s), "r"(inc) : "memory");
+            asm volatile("atom.add.release.gpu.u32 %0, [%1], 1;" : "=r"(old) : "l"(c.st.arrive + c.s) : "memory");
         old = __shfl_sync(FULL, old, 0);
-        if (old + inc == (unsigned int)__ldg(c.scen_warps + c.s)) {
+        if (old + 1 == (unsigned int)__ldg(c.scen_warps + c.s)) {
             asm volatile("fence.acq_rel.gpu;" ::: "memory");
-            if (c.defer) {
-                run_pending(c, lane);
-                c.pend_s = c.s;
-            } else {
-                apply_update(c, c.s, lane);
-            }
+            update_scenario<G ? 8 : 1>(c.t, c.st, c.a, c.s, c.round, lane);
+            if (lane == 0)
+                c.st.arrive[c.s] = 0u;     // every warp of this pass has arrived
         }
     }
-}
-
-// Adds the warp's demand of its current scenario to the scenario's accumulator and arrives (a warp
-// that has evaluated nothing yet does nothing).
-template <int RT, bool G>
-__device__ void flush(WarpCtx<RT, G> &c, int lane)
-{
-    if (c.s < 0)
-        return;
-    flush_demand(c, lane);
-    c.ntiles = 0;
 }
 
 template <int RT, bool G>

@@ -30,8 +30,7 @@ EXPORTED = [
     "esp_debug_tile_options", "esp_debug_plan", "esp_debug_stats", "esp_debug_resident",
     "esp_debug_sort_layout", "esp_debug_plan_runs", "esp_debug_set_sorted_layout", "esp_debug_set_pdl", "esp_debug_set_plan_waves",
     "esp_debug_hold_barrier", "esp_debug_set_wait_limit", "esp_debug_hold_stage", "esp_debug_fail_alloc",
-    "esp_debug_set_stream_pass", "esp_debug_pass_kernel", "esp_debug_plan_stream", "esp_debug_sort_layout_k",
-    "esp_debug_set_interleave",
+    "esp_debug_pass_kernel", "esp_debug_set_interleave",
     "esp_evaluate_noalloc",
     "esp_set_penalties", "esp_adaptive_threshold", "esp_effective_capacity", "esp_load_placement",
     "esp_iac_create", "esp_iac_set_stream", "esp_iac_load_model", "esp_iac_predict", "esp_iac_predict_host",
@@ -104,12 +103,8 @@ def load_library(path: Optional[str] = None):
         "esp_debug_set_wait_limit": ([vp, u32], st),
         "esp_debug_hold_stage": ([vp], st),
         "esp_debug_fail_alloc": ([vp, i64], st),
-        "esp_debug_set_stream_pass": ([vp, i32], st),
         "esp_debug_pass_kernel": ([vp, ctypes.POINTER(i32)], st),
         "esp_debug_set_interleave": ([vp, i32], st),
-        "esp_debug_plan_stream": ([vp, i32, i32, vp, vp, i32, i32, i32, vp, i32, vp, vp,
-                                   ctypes.POINTER(i32), ctypes.POINTER(i32), ctypes.POINTER(i32)], st),
-        "esp_debug_sort_layout_k": ([vp, i32, i32, i32, vp, vp, vp, vp], st),
         "esp_set_penalties": ([vp, ctypes.c_double, vp, ctypes.c_double, vp, vp], st),
         "esp_load_placement": ([vp, i32, i32, i32, i32, i32, i32, vp, vp, vp, vp, i32, vp, vp, vp], st),
         "esp_adaptive_threshold": ([i64, vp, ctypes.c_double, ctypes.c_double, ctypes.c_double, ctypes.c_double, vp],
@@ -482,53 +477,17 @@ def esp_debug_fail_alloc(ctx: int, n: int) -> None:
     _check(load_library().esp_debug_fail_alloc(ctx, int(n)), "esp_debug_fail_alloc")
 
 
-def esp_debug_set_stream_pass(ctx: int, enable: bool) -> None:
-    """Later loads use the streaming pass where the table allows it (True, the default) or never."""
-    _check(load_library().esp_debug_set_stream_pass(ctx, 1 if enable else 0), "esp_debug_set_stream_pass")
-
-
 def esp_debug_set_interleave(ctx: int, enable: bool) -> None:
     """Later loads interleave the per-warp pass's table tile by tile (True, the default) or not."""
     _check(load_library().esp_debug_set_interleave(ctx, 1 if enable else 0), "esp_debug_set_interleave")
 
 
 def esp_debug_pass_kernel(ctx: int) -> int:
-    """The evaluation pass the loaded table uses: 1 streaming, 0 per-warp, 3 per-warp on the
-    tile-interleaved table, 2 factored placement."""
+    """How the loaded table is evaluated: 0 per-warp pass, two copies per tile; 1 per-warp pass on the
+    tile-interleaved table, one copy per tile; 2 factored placement."""
     k = ctypes.c_int32()
     _check(load_library().esp_debug_pass_kernel(ctx, ctypes.byref(k)), "esp_debug_pass_kernel")
     return k.value
-
-
-def sort_layout_k(job_off: np.ndarray, S: int, J: int, run_max_k: int):
-    """Sorted layout with runs of up to run_max_k options (no GPU): (padded offsets, jmap, scen, runk)."""
-    lib = load_library()
-    job_off = np.ascontiguousarray(job_off, np.int64)
-    off = np.zeros(S * J + 1, np.int64)
-    jmap, scen, runk = (np.zeros(S * J, np.int32) for _ in range(3))
-    _check(lib.esp_debug_sort_layout_k(_p(job_off), S, J, run_max_k, _p(off), _p(jmap), _p(scen), _p(runk)),
-           "esp_debug_sort_layout_k")
-    return off, jmap, scen, runk
-
-
-def plan_stream(job_off, S: int, J: int, R: int, grid: int, scen=None, runk=None, uniform_k: int = 0):
-    """The streaming pass's host planner (no GPU): dict of its blocks as tiles (n x 8 int32), cta_begin,
-    arrivals and stage_opt."""
-    lib = load_library()
-    job_off = np.ascontiguousarray(job_off, np.int64)
-    sc = None if scen is None else np.ascontiguousarray(scen, np.int32)
-    rk = None if runk is None else np.ascontiguousarray(runk, np.int32)
-    nt, nc, so = (ctypes.c_int32() for _ in range(3))
-    cta = np.zeros(grid + 1, np.int32)
-    arr = np.zeros(S, np.int32)
-    args = lambda tl, tc: (_p(job_off), S, J, _p(sc), _p(rk), uniform_k, R, grid, tl, tc, _p(cta), _p(arr),  # noqa: E731
-                           ctypes.byref(nt), ctypes.byref(nc), ctypes.byref(so))
-    st = lib.esp_debug_plan_stream(*args(None, 0))
-    if st not in (ESP_OK, ESP_ERR_OOM):
-        raise EspError(st, "esp_debug_plan_stream")
-    tiles = np.zeros((max(nt.value, 1), 8), np.int32)
-    _check(lib.esp_debug_plan_stream(*args(_p(tiles), nt.value)), "esp_debug_plan_stream")
-    return {"tiles": tiles[:nt.value], "cta_begin": cta[:nc.value + 1], "arrivals": arr, "stage_opt": so.value}
 
 
 
