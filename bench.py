@@ -116,7 +116,7 @@ def measured_peak():
         return 6800.0, "fallback"
 
 
-PASS_KERNEL_SOURCES = ("esp_kernels.cu", "esp_tile.cuh", "esp_ptx.cuh", "esp_warp.cuh", "esp_device.cuh",
+PASS_KERNEL_SOURCES = ("esp_kernels.cu", "esp_kernels_f32.cu", "esp_pass.cuh", "esp_tile.cuh", "esp_ptx.cuh", "esp_warp.cuh", "esp_device.cuh",
                        "esp_common.h", "esp_kernels.h")
 
 

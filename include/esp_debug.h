@@ -97,8 +97,28 @@ esp_status esp_debug_fail_alloc(esp_ctx *ctx, int64_t n);
 
 /* *kind receives how the loaded table is evaluated: 0 the per-warp pass with two bulk copies per tile
  * (units and values apart), 1 the per-warp pass with one bulk copy per tile (tile-interleaved table),
- * 2 the factored placement pass. */
+ * 2 the factored placement pass, 3 as 1 with the units of the interleaved table stored as fp32 (every
+ * unit below 2^23, so each is exact; the screen then needs no conversion per unit). */
 esp_status esp_debug_pass_kernel(esp_ctx *ctx, int32_t *kind);
+
+/* Persistent pass: every round of a solve in one cooperative launch, each scenario's next round
+ * released by its price update instead of a kernel boundary (tables whose interleaved tiles hold fp32
+ * units; solves without per-pass events, fingerprint or dual trace). mode -1 (the default) uses it on
+ * uniform tables with at least 16 tiles per warp of its launch, 0 never, 1 wherever the table can take
+ * it; later solves of this context follow the mode. Results are identical either way.
+ * esp_debug_persistent: *grid receives the CTAs of the persistent launch that a plain solve of the
+ * loaded table uses under the current mode (0: one launch per round). */
+esp_status esp_debug_set_persistent(esp_ctx *ctx, int32_t mode);
+esp_status esp_debug_persistent(esp_ctx *ctx, int32_t *grid);
+/* Waits of the persistent pass for a scenario's prices that had to poll since the last reset: *ns their
+ * total duration in nanoseconds of the GPU's global timer (summed over warps), *waits their number.
+ * Waits for the context's stream; reset != 0 zeroes both. */
+esp_status esp_debug_persist_waits(esp_ctx *ctx, int64_t *ns, int64_t *waits, int32_t reset);
+
+/* enable = 0 makes later loads keep integer units in the tile-interleaved table; 1 restores the
+ * default (fp32 units where every unit is below 2^23 and the table has no group column, R = 4, 6 or 8,
+ * uniform or sorted). Results are identical either way. */
+esp_status esp_debug_set_stage_f32(esp_ctx *ctx, int32_t enable);
 
 /* enable = 0 makes later loads keep the per-warp pass's table as separate unit and value arrays (two
  * bulk copies per tile); 1 restores the default, a tile-interleaved copy (each tile's units then its

@@ -18,7 +18,7 @@ INCLUDE = os.path.join(ROOT, "include")
 OBJDIR = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libesp.so")
 
-SOURCES = ["esp_api.cu", "esp_kernels.cu", "esp_place.cu", "esp_load.cu", "esp_resident.cu", "esp_plan.cpp",
+SOURCES = ["esp_api.cu", "esp_kernels.cu", "esp_kernels_f32.cu", "esp_place.cu", "esp_load.cu", "esp_resident.cu", "esp_plan.cpp",
            "esp_host.cpp", "esp_noalloc.cu", "esp_iac.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC,-O2,-ffp-contract=off", "-I", INCLUDE, "-I", CSRC,

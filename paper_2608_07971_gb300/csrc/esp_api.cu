@@ -26,10 +26,12 @@ struct GraphKey {
     bool has_l0 = false;
     int res = -1;   // resident option in use, -1: streaming
     bool hold = false;
+    bool persist = false;   // rounds in one persistent launch
     uint32_t hold_tx = 0, wait_ms = 0;
     bool operator==(const GraphKey &o) const
     {
         return eta0 == o.eta0 && tol == o.tol && step == o.step && mode == o.mode && T == o.T && flags == o.flags &&
+               persist == o.persist &&
                lt == o.lt && dt == o.dt && ht == o.ht && gt == o.gt && has_l0 == o.has_l0 && res == o.res &&
                hold == o.hold && hold_tx == o.hold_tx && wait_ms == o.wait_ms;
     }
@@ -93,6 +95,7 @@ struct esp_ctx {
     // tile of the per-warp plan allows it; n_tiles: tiles of that plan
     unsigned char *il = nullptr;
     int64_t n_tiles = 0;
+    bool il_f32 = false;             // il holds the units as fp32 bit patterns (every unit below 2^23)
 
     // factored placement table (esp_load_placement): no stored option table
     bool placement = false;
@@ -109,6 +112,7 @@ struct esp_ctx {
     TileDesc *tiles = nullptr;
     int32_t *warp_begin = nullptr;
     bool il_enabled = true;          // later loads may interleave the pass table (esp_debug_set_interleave)
+    bool il_f32_enabled = true;      // ... with fp32 units where exact (esp_debug_set_stage_f32)
     // failure-detection hooks (esp_debug.h): limit of a bounded wait of the evaluation passes in ms
     // (0: the default, 4 s), extra bytes announced on the next solve's first stage, allocations left
     // before an injected failure (-1: none)
@@ -116,7 +120,17 @@ struct esp_ctx {
     uint32_t hold_tx = 0;
     int64_t fail_alloc_in = -1;
     int32_t *scen_warps = nullptr;   // warps owning tiles of each scenario
+    int32_t *scen_tiles = nullptr;   // tiles of each scenario
+    int32_t *item_order = nullptr;   // the plan's ranges by the scenario of their first tile
     unsigned int *arrive = nullptr;  // per-scenario arrivals of the round pass in flight
+    unsigned int *ver = nullptr;     // per-scenario price versions of the persistent pass
+    unsigned int *work = nullptr;    // work items the persistent pass has handed out
+    // persistent pass (every round in one cooperative launch): CTAs of its launch, 0 when the loaded
+    // table cannot take it; persist_auto: plain solves use it by default; persist_mode: -1 automatic,
+    // 0 never, 1 wherever the table can take it (esp_debug_set_persistent)
+    int32_t persist_grid = 0;
+    bool persist_auto = false;
+    int persist_mode = -1;
     int32_t n_warps = 0, tile_opt = 0, grid = 0, uniform_k = 0;
 
     // cluster-resident kernel (tables without a group column): every cluster size that fits
@@ -140,7 +154,9 @@ struct esp_ctx {
             *feasible = nullptr;
     unsigned int *err = nullptr;
     unsigned int *valflags = nullptr;
-    unsigned long long *stats = nullptr;  // [0] exact resolutions (since the last read), [1] marked duplicates
+    // [0] exact resolutions (since the last read), [1] marked duplicates, [2] nanoseconds and [3] number
+    // of the persistent pass's waits for a scenario's prices that had to poll
+    unsigned long long *stats = nullptr;
 
     // trace buffers (grown on demand, freed on destroy)
     DevArr<double> lt;
@@ -260,6 +276,9 @@ void release_table(esp_ctx *ctx, bool keep = false)
     ctx->s_jmap = nullptr;
     ctx->values0 = nullptr;
     ctx->il = nullptr;
+    ctx->il_f32 = false;
+    ctx->persist_grid = 0;
+    ctx->persist_auto = false;
     ctx->n_tiles = 0;
     ctx->placement = false;
     ctx->place = DevPlace{};
@@ -312,6 +331,7 @@ DevTable dev_table(const esp_ctx *c)
     t.small_units = c->small_units;
     t.jmap = nullptr;
     t.il = nullptr;
+    t.il_f32 = 0;
     return t;
 }
 
@@ -327,6 +347,7 @@ DevTable pass_table(const esp_ctx *c)
         t.jmap = c->s_jmap;
     }
     t.il = c->il;
+    t.il_f32 = (c->il != nullptr && c->il_f32) ? 1 : 0;
     return t;
 }
 
@@ -356,6 +377,8 @@ DevState dev_state(const esp_ctx *c)
     s.err = c->err;
     s.stats = c->stats;
     s.arrive = c->arrive;
+    s.ver = c->ver;
+    s.work = c->work;
     s.lam_trace = nullptr;
     s.dem_trace = nullptr;
     s.hash_trace = nullptr;
@@ -422,6 +445,8 @@ esp_status alloc_solve_state(esp_ctx *ctx)
     al(&ctx->primal, S);
     al(&ctx->dual, S);
     al(&ctx->lambda0, SP);
+    al(&ctx->ver, S);
+    al(&ctx->work, 1);
     al(&ctx->err, 4);
     return a;
 }
@@ -486,7 +511,7 @@ esp_status load_common(esp_ctx *ctx, int32_t S, int32_t J, int32_t R, int32_t P,
     ALLOC(ctx->vmax, (size_t)S);
     ALLOC(ctx->umax, (size_t)S * R);
     ALLOC(ctx->valflags, 4);
-    ALLOC(ctx->stats, 2);
+    ALLOC(ctx->stats, 4);
 
     const cudaMemcpyKind kind = device_src ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice;
     ESP_CUDA(cudaMemcpyAsync(ctx->units, units, (size_t)n_opt * R * sizeof(int32_t), kind, ctx->stream));
@@ -568,15 +593,24 @@ esp_status load_common(esp_ctx *ctx, int32_t S, int32_t J, int32_t R, int32_t P,
     // a sorted layout's tiles are runs and chunks only (the sorted layout exists only without a group
     // column): the runs-only instantiation
     const int mode = ctx->uniform_k > 0 ? kModeUniform : (use_sorted && !grouped) ? kModeRuns : kModeGeneral;
-    const int per_sm = pass_ctas_per_sm(R, grouped, mode, P, tile_opt);
+    int per_sm = pass_ctas_per_sm(R, grouped, mode, P, tile_opt);
+    // a table that may take the persistent pass is planned for its co-resident CTAs, so that each of
+    // its physical warps runs exactly `waves` ranges (its fp32 stage units are decided after the
+    // validation; a table that turns out not to qualify runs the same plan with per-round launches)
+    const int per_sm_persist = (ctx->il_enabled && ctx->il_f32_enabled && pass_f32_shape(R, grouped, mode))
+                                   ? pass_persist_ctas_per_sm(R, mode, P, tile_opt)
+                                   : 0;
+    if (per_sm_persist > 0 && per_sm_persist < per_sm)
+        per_sm = per_sm_persist;
     if (per_sm < 1) {
         cudaStreamSynchronize(ctx->stream);
         release_table(ctx);
         return ESP_ERR_UNSUPPORTED;
     }
-    // two waves of resident CTAs by default: CTAs that finish early take the second wave's ranges,
-    // which halves the pass's tail (measured: what-if batch -2.1%, heavy-tailed table -2.5%)
-    const int waves = ctx->plan_waves > 0 ? ctx->plan_waves : 2;
+    // Ranges of the plan as waves of resident CTAs: two by default (with per-round launches, CTAs that
+    // finish early take the second wave's ranges; the persistent pass hands them out as work items,
+    // two per warp and round), one for a sorted layout (measured 2% faster there).
+    const int waves = ctx->plan_waves > 0 ? ctx->plan_waves : (mode == kModeRuns) ? 1 : 2;
     const int max_warps = ctx->sm_count * per_sm * kWarpsPerCta * waves;
     const bool plan_cached = cached && pc.max_warps == max_warps && pc.tile_opt == tile_opt;
     if (!plan_cached && (!plan_tiles(plan_off, S, J, tile_opt, max_warps, plan_new, plan_scen, plan_runk) ||
@@ -605,6 +639,8 @@ esp_status load_common(esp_ctx *ctx, int32_t S, int32_t J, int32_t R, int32_t P,
         if (x >= (1 << 23))
             ctx->small_units = 0;
     ALLOC(ctx->scen_warps, (size_t)S);
+    ALLOC(ctx->scen_tiles, (size_t)S);
+    ALLOC(ctx->item_order, (size_t)std::max<int32_t>(plan.n_warps, 1));
     ALLOC(ctx->arrive, (size_t)S);
     {
         ctx->n_warps = plan.n_warps;
@@ -621,8 +657,27 @@ esp_status load_common(esp_ctx *ctx, int32_t S, int32_t J, int32_t R, int32_t P,
                     ++sw[last];
                 }
         }
+        std::vector<int32_t> stl((size_t)S, 0);
+        for (const TileDesc &d : plan.tiles)
+            ++stl[d.scenario];
         ESP_CUDA(cudaMemcpyAsync(ctx->scen_warps, sw.data(), sw.size() * sizeof(int32_t), cudaMemcpyHostToDevice,
                                  ctx->stream));
+        ESP_CUDA(cudaMemcpyAsync(ctx->scen_tiles, stl.data(), stl.size() * sizeof(int32_t), cudaMemcpyHostToDevice,
+                                 ctx->stream));
+        // the ranges by the scenario of their first tile, in table order within a scenario (a sorted
+        // layout keeps each scenario's runs, large jobs and one- and two-option jobs apart)
+        std::vector<int32_t> order((size_t)plan.n_warps);
+        for (int32_t w = 0; w < plan.n_warps; ++w)
+            order[w] = w;
+        auto first_scen = [&](int32_t w) {
+            const int32_t k = plan.warp_begin[w];
+            return k < (int32_t)plan.tiles.size() ? plan.tiles[k].scenario : S;
+        };
+        std::stable_sort(order.begin(), order.end(),
+                         [&](int32_t x, int32_t y) { return first_scen(x) < first_scen(y); });
+        if (!order.empty())
+            ESP_CUDA(cudaMemcpyAsync(ctx->item_order, order.data(), order.size() * sizeof(int32_t),
+                                     cudaMemcpyHostToDevice, ctx->stream));
         ESP_CUDA(cudaStreamSynchronize(ctx->stream));
         if (!plan.tiles.empty())
             ESP_CUDA(cudaMemcpyAsync(ctx->tiles, plan.tiles.data(), plan.tiles.size() * sizeof(TileDesc),
@@ -646,7 +701,22 @@ esp_status load_common(esp_ctx *ctx, int32_t S, int32_t J, int32_t R, int32_t P,
             const int64_t pass_opt = ctx->sorted ? ctx->s_n_opt : n_opt;
             ALLOC(ctx->il, (size_t)(pass_opt * W));
             ctx->n_tiles = (int64_t)plan.tiles.size();
-            ESP_CUDA(launch_interleave(pass_table(ctx), ctx->tiles, ctx->n_tiles, ctx->il, ctx->stream));
+            // units as fp32 where every unit converts exactly and the shape has that instantiation
+            ctx->il_f32 = ctx->il_f32_enabled && ctx->small_units && pass_f32_shape(R, grouped, mode);
+            ESP_CUDA(launch_interleave(pass_table(ctx), ctx->tiles, ctx->n_tiles, ctx->il, ctx->il_f32,
+                                       ctx->stream));
+            // the persistent pass: every CTA of its launch co-resident, no more warps than ranges. Used
+            // by default on uniform tables with at least kPersistMinTiles tiles per warp of its launch
+            // (measured on the what-if batch at 1024 and 256 scenarios: 16% and 19% faster per solve;
+            // at 64 scenarios, 4.5 tiles per warp, 5% slower; sorted layouts measured faster with
+            // per-round launches)
+            if (ctx->il_f32 && per_sm_persist > 0 && plan.n_warps > 0) {
+                const int64_t cap_ctas = (int64_t)per_sm_persist * ctx->sm_count;
+                const int64_t need_ctas = ((int64_t)plan.n_warps + kWarpsPerCta - 1) / kWarpsPerCta;
+                ctx->persist_grid = (int32_t)std::min(cap_ctas, need_ctas);
+                ctx->persist_auto = mode == kModeUniform &&
+                                    ctx->n_tiles >= (int64_t)kPersistMinTiles * ctx->persist_grid * kWarpsPerCta;
+            }
         }
     }
 
@@ -716,7 +786,7 @@ bool state_ready(const esp_ctx *c)
     const void *need[] = {c->lam, c->p64, c->p32, c->ebound, c->U, c->U_final, c->hash, c->sel, c->job_val,
                           c->job_min, c->rounds_run, c->converged, c->status, c->frozen, c->feasible,
                           c->best_dual, c->primal, c->dual, c->lambda0, c->err, c->vmax, c->umax, c->stats,
-                          c->arrive, c->cap, c->scen_warps};
+                          c->arrive, c->ver, c->work, c->cap, c->scen_warps};
     for (const void *p : need)
         if (!p)
             return false;
@@ -737,6 +807,8 @@ DevPlan dev_plan(const esp_ctx *c, bool fused)
     pl.uniform_k = c->uniform_k;
     pl.runs_only = (c->sorted && c->group == nullptr) ? 1 : 0;
     pl.scen_warps = fused ? c->scen_warps : nullptr;
+    pl.scen_tiles = c->scen_tiles;
+    pl.item_order = c->item_order;
     return pl;
 }
 
@@ -899,6 +971,12 @@ esp_status enqueue_solve(esp_ctx *ctx, const esp_params *p, const DevState &st, 
                            st.hash_trace == nullptr && st.dual_trace == nullptr;
     const bool hold = place_res && ctx->hold_barrier;
     ctx->hold_barrier = false;
+    // rounds 0 .. T-1 in one persistent launch (fused updates, fp32 stage units, no per-pass events,
+    // no fingerprint or dual trace: those are written by the round passes)
+    const bool persist = ctx->persist_grid > 0 && (ctx->persist_mode > 0 || (ctx->persist_mode < 0 && ctx->persist_auto)) &&
+                         !ctx->placement && ri < 0 && fused &&
+                         !timed && t.il_f32 && T > 0 && st.hash_trace == nullptr && st.dual_trace == nullptr &&
+                         (int64_t)T * ctx->n_tiles < (int64_t)INT32_MAX;   // items and a warp's tiles below 2^31
     auto timed_launch = [&](auto &&launch) -> cudaError_t {
         if (!timed)
             return launch();
@@ -954,6 +1032,16 @@ esp_status enqueue_solve(esp_ctx *ctx, const esp_params *p, const DevState &st, 
                 e = launch_objectives(t, st, a, ctx->stream);
             return e;
         }
+        if (persist) {
+            if (e == cudaSuccess)
+                e = launch_pass_persist(t, st, pl, a, T, ctx->persist_grid, ctx->stream);
+            // after the cooperative launch the final pass starts as an ordinary launch
+            if (e == cudaSuccess)
+                e = launch_pass(t, st, pl, a, T, PASS_FINAL, ctx->grid, ctx->stream, false);
+            if (e == cudaSuccess)
+                e = launch_objectives(t, st, a, ctx->stream);
+            return e;
+        }
         for (int r = 0; r < T && e == cudaSuccess; ++r) {
             if (ctx->grid > 0)
                 e = pass(r, PASS_ROUND);
@@ -967,7 +1055,9 @@ esp_status enqueue_solve(esp_ctx *ctx, const esp_params *p, const DevState &st, 
         return e;
     };
     ctx->last_launches = place_res ? 3 + (T > 0 ? 1 : 0)
-                         : ri >= 0 ? 3 : 3 + (fused ? 1LL : 2LL) * T - (ctx->grid > 0 ? 0 : (T + 1));
+                         : ri >= 0 ? 3
+                         : persist ? 4
+                                   : 3 + (fused ? 1LL : 2LL) * T - (ctx->grid > 0 ? 0 : (T + 1));
     ctx->last_T = T;
 
     GraphKey key;
@@ -984,6 +1074,7 @@ esp_status enqueue_solve(esp_ctx *ctx, const esp_params *p, const DevState &st, 
     key.has_l0 = has_l0;
     key.res = place_res ? -2 : ri;
     key.hold = hold;
+    key.persist = persist;
     key.hold_tx = a.hold_tx;
     key.wait_ms = a.wait_ms;
 
@@ -1456,7 +1547,7 @@ esp_status esp_load_placement(esp_ctx *ctx, int32_t S, int32_t J, int32_t KC, in
     PALLOC(ctx->vmax, (size_t)S);
     PALLOC(ctx->umax, (size_t)S * R);
     PALLOC(ctx->valflags, 4);
-    PALLOC(ctx->stats, 2);
+    PALLOC(ctx->stats, 4);
     auto h2d = [&](void *dst, const void *src, size_t bytes) {
         return cudaMemcpyAsync(dst, src, bytes, cudaMemcpyHostToDevice, ctx->stream);
     };
@@ -1536,7 +1627,7 @@ esp_status refresh_after_values(esp_ctx *ctx, unsigned int *vflags)
     if (ctx->sorted)
         ESP_CUDA(launch_gather_sorted(t, pass_table(ctx), ctx->s_units, ctx->s_values, ctx->stream));
     if (ctx->il)
-        ESP_CUDA(launch_interleave(pass_table(ctx), ctx->tiles, ctx->n_tiles, ctx->il, ctx->stream));
+        ESP_CUDA(launch_interleave(pass_table(ctx), ctx->tiles, ctx->n_tiles, ctx->il, ctx->il_f32, ctx->stream));
     ESP_CUDA(cudaMemcpyAsync(vflags, ctx->valflags, sizeof(unsigned int), cudaMemcpyDeviceToHost, ctx->stream));
     ESP_CUDA(cudaStreamSynchronize(ctx->stream));
     return ESP_OK;
@@ -1705,6 +1796,23 @@ esp_status esp_debug_stats(esp_ctx *ctx, int64_t *resolutions, int64_t *marked, 
     *marked = (int64_t)h[1];
     if (reset)
         ESP_CUDA(cudaMemsetAsync(ctx->stats, 0, sizeof(unsigned long long), ctx->stream));
+    return ESP_OK;
+}
+
+esp_status esp_debug_persist_waits(esp_ctx *ctx, int64_t *ns, int64_t *waits, int32_t reset)
+{
+    esp_status st = check_ctx(ctx);
+    if (st != ESP_OK)
+        return st;
+    if (!ctx->loaded || !ns || !waits)
+        return ESP_ERR_INVALID_ARG;
+    unsigned long long h[2] = {0, 0};
+    ESP_CUDA(cudaMemcpyAsync(h, ctx->stats + 2, sizeof(h), cudaMemcpyDeviceToHost, ctx->stream));
+    ESP_CUDA(cudaStreamSynchronize(ctx->stream));
+    *ns = (int64_t)h[0];
+    *waits = (int64_t)h[1];
+    if (reset)
+        ESP_CUDA(cudaMemsetAsync(ctx->stats + 2, 0, sizeof(h), ctx->stream));
     return ESP_OK;
 }
 
@@ -1892,7 +2000,40 @@ esp_status esp_debug_pass_kernel(esp_ctx *ctx, int32_t *kind)
         return ESP_ERR_INVALID_ARG;
     if (!ctx->loaded)
         return ESP_ERR_NOT_LOADED;
-    *kind = ctx->placement ? 2 : ctx->il ? 1 : 0;
+    *kind = ctx->placement ? 2 : ctx->il ? (ctx->il_f32 ? 3 : 1) : 0;
+    return ESP_OK;
+}
+
+esp_status esp_debug_set_persistent(esp_ctx *ctx, int32_t mode)
+{
+    esp_status st = check_ctx(ctx);
+    if (st != ESP_OK)
+        return st;
+    if (mode < -1 || mode > 1)
+        return ESP_ERR_INVALID_ARG;
+    ctx->persist_mode = mode;
+    return ESP_OK;
+}
+
+esp_status esp_debug_persistent(esp_ctx *ctx, int32_t *grid)
+{
+    esp_status st = check_ctx(ctx);
+    if (st != ESP_OK)
+        return st;
+    if (!grid)
+        return ESP_ERR_INVALID_ARG;
+    if (!ctx->loaded)
+        return ESP_ERR_NOT_LOADED;
+    *grid = (ctx->persist_mode > 0 || (ctx->persist_mode < 0 && ctx->persist_auto)) ? ctx->persist_grid : 0;
+    return ESP_OK;
+}
+
+esp_status esp_debug_set_stage_f32(esp_ctx *ctx, int32_t enable)
+{
+    esp_status st = check_ctx(ctx);
+    if (st != ESP_OK)
+        return st;
+    ctx->il_f32_enabled = enable != 0;
     return ESP_OK;
 }
 

@@ -205,6 +205,15 @@ ESP_HD WarpSmem warp_smem(int tile_opt, int R, bool grouped, int P, bool offsets
     return W;
 }
 
+// Persistent evaluation pass (every round in one cooperative launch): each warp keeps a queue of up to
+// kPersistQueue taken work items (item, first tile, tiles, first virtual tile) in kPersistQueueBytes
+// of shared memory after its WarpSmem.
+constexpr int kPersistQueue = 8;
+constexpr int kPersistMinTiles = 16;   // tiles per warp of the launch for the persistent pass by default
+constexpr int kPersistQueueBytes = 4 * 4 * kPersistQueue;
+// Price version of a scenario that stopped (converged or non-finite): every later round is released.
+constexpr unsigned int kVerStopped = 0x7fffffffu;
+
 // Device status words (bit flags in ctx error word).
 enum : uint32_t {
     DEV_ERR_TIMEOUT = 1u,

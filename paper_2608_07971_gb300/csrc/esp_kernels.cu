@@ -35,6 +35,7 @@
 #include "esp_ptx.cuh"
 #include "esp_tile.cuh"
 #include "esp_warp.cuh"
+#include "esp_pass.cuh"
 
 namespace esp {
 
@@ -60,6 +61,10 @@ __global__ void k_init(DevTable t, DevState st, SolveArgs a, const double *lambd
     if (lane == 0) {
         st.hash[s] = 0ull;
         st.arrive[s] = 0u;
+        if (st.ver)
+            st.ver[s] = 0u;
+        if (st.work && s == 0)
+            *st.work = 0u;
         st.rounds_run[s] = 0;
         st.converged[s] = 0;
         st.status[s] = 0;
@@ -78,236 +83,6 @@ __global__ void k_update(DevTable t, DevState st, SolveArgs a, int round)
     if (s >= t.S || st.frozen[s])
         return;
     update_scenario<8>(t, st, a, s, round, lane);
-}
-
-// Data of tile-local option o (stage) or of job option o (global, gfirst = the job's first option).
-
-// Asks L2 for the option bytes of tile d (lane 0 only), a few tiles before the stage copy of the
-// same bytes is issued: the DRAM latency is then hidden by L2 rather than by shared memory.
-__device__ __forceinline__ void prefetch_tile(const DevTable &t, const TileDesc &d)
-{
-    const int R = t.R;
-    const int64_t ub = d.opt_begin * R * 4, ue = (d.opt_begin + d.n_opt) * R * 4;
-    const int64_t ulo = ub & ~int64_t(15), uhi = (ue + 15) & ~int64_t(15);
-    const int64_t vb = d.opt_begin * 8, ve = (d.opt_begin + d.n_opt) * 8;
-    const int64_t vlo = vb & ~int64_t(15), vhi = (ve + 15) & ~int64_t(15);
-    prefetch_l2(reinterpret_cast<const unsigned char *>(t.units) + ulo, (uint32_t)(uhi - ulo));
-    prefetch_l2(reinterpret_cast<const unsigned char *>(t.values) + vlo, (uint32_t)(vhi - vlo));
-}
-
-// Chunk tile of a job larger than a tile: all its options belong to one job, so no segmentation is
-
-
-// Issues the bulk copies of tile d into a stage; lane 0 only (issuing the copies from several lanes
-// at once measured slower). Uniform tables and runs of the sorted layout need no job offsets.
-__device__ __forceinline__ void issue_tile(const DevTable &t, const TileDesc &d, unsigned char *stage,
-                                           const StageLayout &SL, uint32_t bar, bool need_offsets, uint32_t extra_tx = 0)
-{
-    const int R = t.R;
-    if (t.il) {   // the tile's units and values are adjacent: one copy (its start is 16-byte aligned)
-        const int64_t W = 4 * R + 8;
-        const int64_t b = d.opt_begin * W, e = ((d.opt_begin + d.n_opt) * W + 15) & ~int64_t(15);
-        fence_proxy_async();
-        mbar_arrive_expect_tx(bar, (uint32_t)(e - b) + extra_tx);
-        bulk_g2s(smem_u32(stage + SL.units), t.il + b, (uint32_t)(e - b), bar);
-        return;
-    }
-    const int64_t ub = d.opt_begin * R * 4, ue = (d.opt_begin + d.n_opt) * R * 4;
-    const int64_t ulo = ub & ~int64_t(15), uhi = (ue + 15) & ~int64_t(15);
-    const int64_t vb = d.opt_begin * 8, ve = (d.opt_begin + d.n_opt) * 8;
-    const int64_t vlo = vb & ~int64_t(15), vhi = (ve + 15) & ~int64_t(15);
-    uint32_t total = (uint32_t)(uhi - ulo) + (uint32_t)(vhi - vlo);
-    int64_t olo = 0, ohi = 0, glo = 0, ghi = 0;
-    const bool offs = need_offsets && !(d.flags & (TILE_BIG | TILE_RUN));
-    if (offs) {
-        const int64_t ob = d.job_begin * 8, oe = (d.job_begin + d.n_job + 1) * 8;
-        olo = ob & ~int64_t(15);
-        ohi = (oe + 15) & ~int64_t(15);
-        total += (uint32_t)(ohi - olo);
-    }
-    if (t.group) {
-        const int64_t gb = d.opt_begin * 2, ge = (d.opt_begin + d.n_opt) * 2;
-        glo = gb & ~int64_t(15);
-        ghi = (ge + 15) & ~int64_t(15);
-        total += (uint32_t)(ghi - glo);
-    }
-    fence_proxy_async();
-    mbar_arrive_expect_tx(bar, total + extra_tx);
-    const unsigned char *ubase = reinterpret_cast<const unsigned char *>(t.units);
-    const unsigned char *vbase = reinterpret_cast<const unsigned char *>(t.values);
-    bulk_g2s(smem_u32(stage + SL.units), ubase + ulo, (uint32_t)(uhi - ulo), bar);
-    bulk_g2s(smem_u32(stage + SL.vals), vbase + vlo, (uint32_t)(vhi - vlo), bar);
-    if (offs)
-        bulk_g2s(smem_u32(stage + SL.off), reinterpret_cast<const unsigned char *>(t.job_off) + olo,
-                 (uint32_t)(ohi - olo), bar);
-    if (t.group)
-        bulk_g2s(smem_u32(stage + SL.grp), reinterpret_cast<const unsigned char *>(t.group) + glo,
-                 (uint32_t)(ghi - glo), bar);
-}
-
-// CTAs per SM the evaluation kernel's register budget must allow.
-// CTAs per SM the evaluation kernel's register budget must allow: the uniform and runs-only
-// instantiations (no segmented-scan path) as many as the general one's shared memory would.
-template <int RT, int MODE>
-constexpr int pass_min_ctas()
-{
-    return MODE == kModeUniform ? ((RT == 4 || RT == 6) ? kMinCtasPerSmNarrow : kMinCtasPerSm)
-           : MODE == kModeRuns  ? kMinCtasPerSmRuns
-                                : kMinCtasPerSmGeneral;
-}
-
-template <int RT, bool G, int MODE, bool PLAIN>
-__global__ void __launch_bounds__(kWarpsPerCta * 32, pass_min_ctas<RT, MODE>()) k_pass(DevTable t, DevState st, DevPlan pl,
-                                                                          SolveArgs a, int round, int kind)
-{
-    extern __shared__ __align__(128) unsigned char smem[];
-    // a pass launched as a programmatic dependent of this one may start its CTAs as soon as slots
-    // free up; it waits (griddepcontrol.wait below) for this grid's completion before reading state
-    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
-    const int w = blockIdx.x * kWarpsPerCta + wid;
-    if (w >= pl.n_warps)
-        return;
-    const int k_begin = pl.warp_begin[w], k_end = pl.warp_begin[w + 1];
-    if (k_begin >= k_end)
-        return;
-    // a wait of an earlier pass of this solve gave up: this warp does nothing (a flag set too recently
-    // to be seen here only means the warp runs, with its own bounded waits)
-    if (__any_sync(FULL, (*reinterpret_cast<volatile unsigned int *>(st.err) & DEV_ERR_TIMEOUT) != 0))
-        return;
-
-    constexpr bool UNI = MODE == kModeUniform;
-    const WarpSmem WS = warp_smem(pl.tile_opt, t.R, G, t.P, MODE == kModeGeneral);
-    const StageLayout SL = stage_layout(pl.tile_opt, t.R, G, MODE == kModeGeneral);
-    unsigned char *wsm = smem + (size_t)wid * WS.bytes;
-    float *p32s = reinterpret_cast<float *>(wsm + WS.p32);
-    const uint32_t bar0 = smem_u32(wsm + WS.bars);
-    const bool need_offsets = MODE == kModeGeneral;
-
-    WarpCtx<RT, G> c;
-    c.t = t;
-    c.st = st;
-    c.scen_warps = pl.scen_warps;
-    c.a = a;
-    c.round = round;
-    c.R = RT ? RT : t.R;
-    c.rg = t.r_global;
-    // PLAIN: a round pass without traces (the hot case), with every per-pass choice a constant
-    c.kind = PLAIN ? (int)PASS_ROUND : kind;
-    c.want_min = PLAIN ? false : ((kind == PASS_FINAL) || (st.dual_trace != nullptr));
-    c.want_hash = PLAIN ? false : ((kind == PASS_ROUND) && (st.hash_trace != nullptr));
-    c.uniform_k = pl.uniform_k;
-    c.log2_k = pl.uniform_k > 0 ? __ffs(pl.uniform_k) - 1 : 0;
-    c.s = -1;
-#pragma unroll
-    for (int r = 0; r < Cols<RT>::N; ++r)
-        c.acc[r] = 0;
-    c.hacc = 0;
-
-    if (lane == 0) {
-        for (int s = 0; s < kStages; ++s)
-            mbar_init(bar0 + 8 * s, 1);
-        fence_barrier_init();
-    }
-    __syncwarp();
-
-    // Tile descriptors reach the warp's ring in blocks of kDescBlock: one cp.async of 16 bytes per
-    // lane fetches a block, issued a whole block before its first tile is issued, so no global
-    // load sits on the per-tile path. Block b uses ring slots (b & 1) * kDescBlock onwards.
-    TileDesc *ring = reinterpret_cast<TileDesc *>(wsm + WS.descs);
-    const unsigned char *tiles_b = reinterpret_cast<const unsigned char *>(pl.tiles);
-    auto fetch_block = [&](int first) {
-        const int ti = first + (lane >> 1);
-        if (lane < 2 * kDescBlock && ti < k_end) {
-            const uint32_t dst = smem_u32(ring + ((ti - k_begin) & (kDescRing - 1))) + 16u * (lane & 1);
-            asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst),
-                         "l"(tiles_b + (size_t)ti * sizeof(TileDesc) + 16 * (lane & 1))
-                         : "memory");
-        }
-        asm volatile("cp.async.commit_group;" ::: "memory");
-    };
-    auto wait_blocks = [&]() {
-        asm volatile("cp.async.wait_group 0;" ::: "memory");
-        __syncwarp();
-    };
-    fetch_block(k_begin);
-    fetch_block(k_begin + kDescBlock);
-    wait_blocks();
-
-    // prologue: the first kStages-1 tiles in flight (lane 0 issues every copy)
-    int issued = k_begin;
-    while (issued < k_end && issued < k_begin + kStages - 1) {
-        const int sidx = (issued - k_begin) % kStages;
-        if (lane == 0)
-            issue_tile(t, ring[(issued - k_begin) & (kDescRing - 1)], wsm + sidx * SL.bytes, SL, bar0 + 8 * sidx,
-                       need_offsets, (w == 0 && issued == k_begin && round == 0 && kind == PASS_ROUND) ? a.hold_tx : 0u);
-        ++issued;
-    }
-    __syncwarp();
-    if (lane == 0)
-        for (int k = issued; k < k_end && k < k_begin + kPrefetchTiles; ++k)
-            prefetch_tile(t, pl.tiles[k]);
-    // everything above reads only the table and the plan; prices, flags and the demand accumulators
-    // were written by the previous kernel on the stream, which is complete after this wait (a no-op
-    // for an ordinary launch)
-    asm volatile("griddepcontrol.wait;" ::: "memory");
-    int64_t big_first = 0;
-    Best big_carry = best_none();
-    Best big_priv = best_none();     // lane-private state of a chunked job
-    int failed_at = -1;
-    for (int k = k_begin; k < k_end; ++k) {
-        if (issued < k_end) {   // refill the stage the previous tile used
-            if (((issued - k_begin) & (kDescBlock - 1)) == 0)
-                wait_blocks();  // the block that starts with tile `issued` has landed
-            if (lane == 0) {
-                const int sidx = (issued - k_begin) % kStages;
-                issue_tile(t, ring[(issued - k_begin) & (kDescRing - 1)], wsm + sidx * SL.bytes, SL,
-                           bar0 + 8 * sidx, need_offsets);
-                if (kPrefetchTiles > 0 && k + kPrefetchTiles < k_end)
-                    prefetch_tile(t, pl.tiles[k + kPrefetchTiles]);
-            }
-            ++issued;
-        }
-        const TileDesc d = ring[(k - k_begin) & (kDescRing - 1)];
-        const int sidx = (k - k_begin) % kStages;
-        const uint32_t parity = (uint32_t)(((k - k_begin) / kStages) & 1);
-        if (!__all_sync(FULL, wait_stage(bar0 + 8 * sidx, parity, st.err, a.wait_ms))) {   // uniform decision
-            failed_at = k;
-            break;
-        }
-        if (d.scenario != c.s)
-            enter_scenario<RT, G>(c, d.scenario, p32s, lane);
-        if (!c.sp.skip) {
-            const StagePtrs ptrs = t.il ? stage_ptrs_il(d, wsm + sidx * SL.bytes, SL, c.R)
-                                        : stage_ptrs(d, wsm + sidx * SL.bytes, SL, c.R);
-            if (UNI && c.uniform_k >= 4)
-                process_tile_uniform4<RT, G>(c, d, ptrs, lane);
-            else if (UNI)
-                process_tile_uniform<RT, G>(c, d, ptrs, lane, c.uniform_k, c.log2_k);
-            else if (d.flags & TILE_BIG)
-                process_tile_bigchunk<RT, G>(c, d, ptrs, big_first, big_priv, lane);
-            else if (!G && (d.flags & TILE_RUN) && tile_run_k(d.flags) >= 4)
-                process_tile_run4<RT, G>(c, d, ptrs, lane, tile_run_k(d.flags));
-            else if (!G && (d.flags & TILE_RUN))
-                process_tile_uniform<RT, G>(c, d, ptrs, lane, tile_run_k(d.flags), tile_run_k(d.flags) >> 1);
-            else if (MODE == kModeGeneral)
-                process_tile_general<RT, G>(c, d, ptrs, big_first, big_carry, lane);
-        }
-        __syncwarp();
-        // the last tile of a block is done (issued and evaluated): its slots take the block after next
-        if (((k - k_begin) & (kDescBlock - 1)) == kDescBlock - 1)
-            fetch_block(k + 1 + kDescBlock);
-    }
-    asm volatile("cp.async.wait_group 0;" ::: "memory");
-    if (failed_at < 0) {
-        flush<RT, G>(c, lane);
-    } else {
-        // a copy never completed: wait (bounded) for every copy still in flight, then leave
-        for (int k = failed_at; k < issued; ++k) {
-            const int sidx = (k - k_begin) % kStages;
-            wait_stage(bar0 + 8 * sidx, (uint32_t)(((k - k_begin) / kStages) & 1), st.err, a.wait_ms);
-        }
-    }
 }
 
 __global__ void k_objectives(DevTable t, DevState st, SolveArgs a)
@@ -344,32 +119,6 @@ __global__ void k_objectives(DevTable t, DevState st, SolveArgs a)
         }
     }
 }
-// Both instantiations (plain round pass and the general one) of a table shape.
-template <int RT, bool G, int MODE>
-struct PassKernels {
-    static const void *plain() { return reinterpret_cast<const void *>(&k_pass<RT, G, MODE, true>); }
-    static const void *other() { return reinterpret_cast<const void *>(&k_pass<RT, G, MODE, false>); }
-    // pdl: programmatic dependent launch, so the pass's CTAs may start (and stage their first tiles)
-    // while the previous kernel on the stream finishes; the kernel waits for it before reading state
-    static void launch(bool plain, int grid, int smem, cudaStream_t stream, const DevTable &t, const DevState &st,
-                       const DevPlan &pl, const SolveArgs &a, int round, int kind, bool pdl)
-    {
-        cudaLaunchConfig_t cfg = {};
-        cfg.gridDim = dim3((unsigned)grid);
-        cfg.blockDim = dim3(kWarpsPerCta * 32);
-        cfg.dynamicSmemBytes = (size_t)smem;
-        cfg.stream = stream;
-        cudaLaunchAttribute attr[1];
-        attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-        attr[0].val.programmaticStreamSerializationAllowed = 1;
-        cfg.attrs = attr;
-        cfg.numAttrs = pdl ? 1 : 0;
-        if (plain)
-            cudaLaunchKernelEx(&cfg, k_pass<RT, G, MODE, true>, t, st, pl, a, round, kind);
-        else
-            cudaLaunchKernelEx(&cfg, k_pass<RT, G, MODE, false>, t, st, pl, a, round, kind);
-    }
-};
 
 // Calls f(PassKernels<RT, G, MODE>()) for the instantiation that serves this table shape (grouped
 // tables are always general).
@@ -418,19 +167,14 @@ int pass_smem_bytes(int R, bool grouped, int mode, int P, int tile_opt)
 int pass_ctas_per_sm(int R, bool grouped, int mode, int P, int tile_opt)
 {
     const int smem = pass_smem_bytes(R, grouped, mode, P, tile_opt);
-    return dispatch_shape(R, grouped, mode, [&](auto k) -> int {
-        using K = decltype(k);
-        if (cudaFuncSetAttribute(K::plain(), cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess ||
-            cudaFuncSetAttribute(K::other(), cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess)
-            return 0;
-        int n = 0;
-        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, K::plain(), kWarpsPerCta * 32, smem) != cudaSuccess)
-            return 0;
-        int m = 0;
-        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&m, K::other(), kWarpsPerCta * 32, smem) != cudaSuccess)
-            return 0;
-        return n < m ? n : m;
-    });
+    int n = dispatch_shape(R, grouped, mode,
+                           [&](auto k) -> int { return pass_kernels_ctas_per_sm<decltype(k)>(smem); });
+    if (n > 0 && pass_f32_shape(R, grouped, mode)) {
+        // the plan must also suit the instantiation that reads fp32 stage units
+        const int m = pass_ctas_per_sm_f32(R, mode, smem);
+        n = m < n ? m : n;
+    }
+    return n;
 }
 
 cudaError_t launch_init(const DevTable &t, const DevState &st, const SolveArgs &a, const double *lambda0,
@@ -448,6 +192,8 @@ cudaError_t launch_pass(const DevTable &t, const DevState &st, const DevPlan &pl
     const int mode = pass_mode(pl);
     const int smem = pass_smem_bytes(t.R, grouped, mode, t.P, pl.tile_opt);
     const bool plain = kind == PASS_ROUND && st.hash_trace == nullptr && st.dual_trace == nullptr;
+    if (t.il_f32)
+        return launch_pass_f32(t, st, pl, a, round, kind, grid, smem, stream, pdl);
     dispatch_shape(t.R, grouped, mode, [&](auto k) -> int {
         decltype(k)::launch(plain, grid, smem, stream, t, st, pl, a, round, kind, pdl);
         return 0;

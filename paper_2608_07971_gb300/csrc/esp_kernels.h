@@ -21,6 +21,9 @@ struct DevTable {
     // evaluation passes only: the table tile by tile, each tile's units then its values, the tile of
     // options [a, b) at byte a * (4R + 8) (one bulk copy per tile); nullptr: units and values apart
     const unsigned char *il;
+    // 1: il holds each unit as the bit pattern of its fp32 value (exact: every unit is below 2^23),
+    // the duplicate mark still the sign bit of column 0
+    int32_t il_f32;
 };
 
 struct DevState {
@@ -47,6 +50,8 @@ struct DevState {
     unsigned int *err;        // device error word (DEV_ERR_*)
     unsigned long long *stats;  // [0] exact resolutions since the last reset, [1] duplicates marked at load
     unsigned int *arrive;     // S   warps of the current round pass that finished the scenario
+    unsigned int *ver;        // S   persistent pass: price updates applied to the scenario (kVerStopped once stopped)
+    unsigned int *work;       // 1   persistent pass: work items handed out
     double *lam_trace;        // S*(T+1)*P or nullptr
     long long *dem_trace;     // S*T*P or nullptr
     unsigned long long *hash_trace; // S*T or nullptr
@@ -61,6 +66,8 @@ struct DevPlan {
     int32_t uniform_k;          // > 0: every job has exactly this many options, a power of two <= 32
     int32_t runs_only;          // 1: every tile is a run of equal-size jobs or a chunk of a large job
     const int32_t *scen_warps;  // S warps owning tiles of each scenario; non-null: round passes update prices
+    const int32_t *scen_tiles;  // S tiles of each scenario (the persistent pass counts arrivals in tiles)
+    const int32_t *item_order;  // n_warps: the persistent pass's ranges in the order it hands them out
 };
 
 struct SolveArgs {
@@ -188,6 +195,26 @@ int pass_smem_bytes(int R, bool grouped, int mode, int P, int tile_opt);
 // Maximum resident CTAs per SM of the evaluation kernel for this table shape (0 if it cannot run).
 int pass_ctas_per_sm(int R, bool grouped, int mode, int P, int tile_opt);
 
+// Table shapes with an instantiation of the evaluation kernel that reads the units of its
+// tile-interleaved stage as fp32 (DevTable::il_f32; esp_kernels_f32.cu).
+inline bool pass_f32_shape(int R, bool grouped, int mode)
+{
+    return !grouped && (R == 4 || R == 6 || R == 8) && (mode == kModeUniform || mode == kModeRuns);
+}
+// Resident CTAs per SM of that instantiation (0: the shape has none, or it cannot run).
+int pass_ctas_per_sm_f32(int R, int mode, int smem);
+// The persistent pass (rounds 0 .. n_rounds - 1 in one cooperative launch, esp_pass.cuh) exists for
+// the same shapes, reading fp32 stage units. Its dynamic shared memory per CTA, its resident CTAs per
+// SM (0: no such kernel or it cannot run) and its launch (grid at most the co-resident CTAs; fused
+// updates; n_rounds * pl.n_warps below 2^31; k_init resets its item counter and versions).
+int pass_persist_smem_bytes(int R, int P, int tile_opt);
+int pass_persist_ctas_per_sm(int R, int mode, int P, int tile_opt);
+cudaError_t launch_pass_persist(const DevTable &t, const DevState &st, const DevPlan &pl, const SolveArgs &a,
+                                int n_rounds, int grid, cudaStream_t stream);
+// Launches it (pass_f32_shape must hold for the table and plan).
+cudaError_t launch_pass_f32(const DevTable &t, const DevState &st, const DevPlan &pl, const SolveArgs &a, int round,
+                            PassKind kind, int grid, int smem, cudaStream_t stream, bool pdl);
+
 cudaError_t launch_validate(const DevTable &t, double *vmax, int32_t *umax, unsigned int *flags,
                             cudaStream_t stream);
 // Marks every option that repeats an earlier option of its job (units, value and group equal) by
@@ -205,9 +232,10 @@ cudaError_t launch_gather_sorted(const DevTable &orig, const DevTable &sorted, i
 cudaError_t launch_apply_penalties(const DevTable &t, const double *values0, const int32_t *c_cur, const double *s_hat,
                                    const double *tau, double gamma0, double alpha, double *values, unsigned int *flags,
                                    cudaStream_t stream);
-// Fills the tile-interleaved copy `il` of table t (t.il's layout) for the n_tiles tiles of a plan.
+// Fills the tile-interleaved copy `il` of table t (t.il's layout) for the n_tiles tiles of a plan;
+// f32: units as fp32 bit patterns (DevTable::il_f32).
 cudaError_t launch_interleave(const DevTable &t, const TileDesc *tiles, int64_t n_tiles, unsigned char *il,
-                              cudaStream_t stream);
+                              bool f32, cudaStream_t stream);
 // Clears every duplicate mark of a units array.
 cudaError_t launch_clear_marks(int32_t *units, int64_t n_opt, int R, cudaStream_t stream);
 cudaError_t launch_init(const DevTable &t, const DevState &st, const SolveArgs &a, const double *lambda0,

@@ -309,8 +309,9 @@ cudaError_t launch_mark_duplicates(const DevTable &t, int32_t *units, unsigned l
 }
 
 // One warp per tile: the tile's units (n R int32, duplicate marks included) then its values (n fp64)
-// at byte opt_begin * (4R + 8) of the interleaved copy.
-__global__ void k_interleave(DevTable t, const TileDesc *tiles, int64_t n_tiles, unsigned char *il)
+// at byte opt_begin * (4R + 8) of the interleaved copy. f32: each unit is written as the bit pattern
+// of its fp32 value (exact below 2^24), the duplicate mark kept as the sign bit.
+__global__ void k_interleave(DevTable t, const TileDesc *tiles, int64_t n_tiles, unsigned char *il, int f32)
 {
     const int lane = threadIdx.x & 31;
     const int64_t warps = (int64_t)gridDim.x * (blockDim.x >> 5);
@@ -322,20 +323,24 @@ __global__ void k_interleave(DevTable t, const TileDesc *tiles, int64_t n_tiles,
         double *v = reinterpret_cast<double *>(il + d.opt_begin * W + (int64_t)d.n_opt * R * 4);
         const int32_t *su = t.units + d.opt_begin * R;
         const double *sv = t.values + d.opt_begin;
-        for (int64_t i = lane; i < (int64_t)d.n_opt * R; i += 32)
-            u[i] = su[i];
+        for (int64_t i = lane; i < (int64_t)d.n_opt * R; i += 32) {
+            const int32_t x = su[i];
+            u[i] = f32 ? (int32_t)(((uint32_t)x & 0x80000000u) |
+                                   (uint32_t)__float_as_int(__int2float_rn(x & 0x7fffffff)))
+                       : x;
+        }
         for (int i = lane; i < d.n_opt; i += 32)
             v[i] = sv[i];
     }
 }
 
 cudaError_t launch_interleave(const DevTable &t, const TileDesc *tiles, int64_t n_tiles, unsigned char *il,
-                              cudaStream_t stream)
+                              bool f32, cudaStream_t stream)
 {
     if (n_tiles <= 0)
         return cudaSuccess;
     const int64_t blocks = std::min<int64_t>((n_tiles + 7) / 8, 65536);
-    k_interleave<<<(int)blocks, 256, 0, stream>>>(t, tiles, n_tiles, il);
+    k_interleave<<<(int)blocks, 256, 0, stream>>>(t, tiles, n_tiles, il, f32 ? 1 : 0);
     return cudaGetLastError();
 }
 

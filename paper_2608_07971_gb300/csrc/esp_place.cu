@@ -216,6 +216,9 @@ __global__ void __launch_bounds__(kPlaceWarps * 32, 4) k_place(DevTable t, DevSt
         return;
 
     WarpCtx<RT, true> c;
+    c.persist = false;
+    c.scen_tiles = nullptr;
+    c.ntiles = 0;
     c.t = t;
     c.st = st;
     c.scen_warps = pl.scen_warps;

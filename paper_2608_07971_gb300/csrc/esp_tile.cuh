@@ -16,7 +16,7 @@ namespace esp {
 
 namespace {
 
-template <int RT, bool G>
+template <int RT, bool G, bool F>
 __device__ __forceinline__ bool load_option(const WarpCtx<RT, G> &c, bool in_smem, const int32_t *units_s,
                                             const double *vals_s, const uint16_t *grp_s, int o, int64_t gfirst,
                                             int32_t *u, double &v, int &g)
@@ -25,7 +25,7 @@ __device__ __forceinline__ bool load_option(const WarpCtx<RT, G> &c, bool in_sme
     bool dup;
     g = 0;
     if (in_smem) {
-        dup = load_units_smem<RT>(units_s + (size_t)o * R, u, R);
+        dup = load_units_stage<RT, F>(units_s + (size_t)o * R, u, R);
         v = vals_s[o];
         if (G)
             g = grp_s[o];
@@ -46,7 +46,7 @@ __device__ __forceinline__ bool load_option(const WarpCtx<RT, G> &c, bool in_sme
 // load-time marking did not cover) is skipped for the same reason, so only survivors that differ
 // from c0 are rescored in fp64. q is recomputed with the same instructions as the screen.
 // Returns the job-local index; s_out is set when has_s is true (always when need_s).
-template <int RT, bool G>
+template <int RT, bool G, bool F>
 __device__ void resolve_job(WarpCtx<RT, G> &c, int lane, bool in_smem, const int32_t *units_s, const double *vals_s,
                             const uint16_t *grp_s, int jstart, int jend, int64_t gfirst, float thr, bool need_s,
                             double &s_out, bool &has_s, int &local_out)
@@ -57,7 +57,7 @@ __device__ void resolve_job(WarpCtx<RT, G> &c, int lane, bool in_smem, const int
     int g;
     int first = kIdxNone;
     for (int o = jstart + lane; o < jend; o += 32) {
-        if (load_option<RT, G>(c, in_smem, units_s, vals_s, grp_s, o, gfirst, u, v, g))
+        if (load_option<RT, G, F>(c, in_smem, units_s, vals_s, grp_s, o, gfirst, u, v, g))
             continue;
         if (c.sp.exact || screen_score<RT, G>(u, v, g, c.sp, R, c.rg) <= thr) {
             first = o;
@@ -68,7 +68,7 @@ __device__ void resolve_job(WarpCtx<RT, G> &c, int lane, bool in_smem, const int
     int32_t u0[Cols<RT>::N];
     double v0;
     int g0;
-    load_option<RT, G>(c, in_smem, units_s, vals_s, grp_s, first, gfirst, u0, v0, g0);
+    load_option<RT, G, F>(c, in_smem, units_s, vals_s, grp_s, first, gfirst, u0, v0, g0);
 
     long long best_key = 0x7fffffffffffffffLL;
     int best_i = kIdxNone;
@@ -76,7 +76,7 @@ __device__ void resolve_job(WarpCtx<RT, G> &c, int lane, bool in_smem, const int
     for (int o = jstart + lane; o < jend; o += 32) {
         if (o <= first)
             continue;
-        if (load_option<RT, G>(c, in_smem, units_s, vals_s, grp_s, o, gfirst, u, v, g))
+        if (load_option<RT, G, F>(c, in_smem, units_s, vals_s, grp_s, o, gfirst, u, v, g))
             continue;
         if (!(c.sp.exact || screen_score<RT, G>(u, v, g, c.sp, R, c.rg) <= thr))
             continue;
@@ -124,7 +124,7 @@ __device__ void resolve_job(WarpCtx<RT, G> &c, int lane, bool in_smem, const int
 
 // Resolves, one after the other, the ambiguous jobs whose closing lanes are set in amask, and records
 // each winner (lane 0). big: the job is chunked and read from global memory.
-template <int RT, bool G>
+template <int RT, bool G, bool F>
 __device__ __forceinline__ void resolve_row(WarpCtx<RT, G> &c, int lane, uint32_t amask, bool big,
                                             const int32_t *units_s, const double *vals_s, const uint16_t *grp_s,
                                             int jstart, int jend, float thr, int64_t job, int64_t big_first)
@@ -139,14 +139,14 @@ __device__ __forceinline__ void resolve_row(WarpCtx<RT, G> &c, int lane, uint32_
         double s_w = 0.0;
         bool has_s = false;
         int li;
-        resolve_job<RT, G>(c, lane, !big, units_s, vals_s, grp_s, js, je, big ? big_first : 0, th, c.want_min,
+        resolve_job<RT, G, F>(c, lane, !big, units_s, vals_s, grp_s, js, je, big ? big_first : 0, th, c.want_min,
                            s_w, has_s, li);
         if (lane == 0) {
             atomicAdd(c.st.stats, 1ull);
             int32_t uw[Cols<RT>::N];
             double vw;
             int gw;
-            load_option<RT, G>(c, !big, units_s, vals_s, grp_s, js + li, big ? big_first : 0, uw, vw, gw);
+            load_option<RT, G, F>(c, !big, units_s, vals_s, grp_s, js + li, big ? big_first : 0, uw, vw, gw);
             take_winner<RT, G>(c, jb, li, uw, vw, gw, has_s, s_w);
         }
     }
@@ -189,7 +189,7 @@ __device__ __forceinline__ StagePtrs stage_ptrs_il(const TileDesc &d, const unsi
 // butterfly gives every lane of the group the smallest and second-smallest screen value; when the
 // job is unambiguous the unique lane holding the smallest value is the winner and records it from
 // its own registers.
-template <int RT, bool G>
+template <int RT, bool G, bool F>
 __device__ void process_tile_uniform(WarpCtx<RT, G> &c, const TileDesc &d, const StagePtrs &sp, int lane, int K,
                                      int log2_k)
 {
@@ -208,7 +208,7 @@ __device__ void process_tile_uniform(WarpCtx<RT, G> &c, const TileDesc &d, const
             if (G)
                 g = sp.grp[i];
             if (!dup)
-                q = screen_score<RT, G>(u, v, g, c.sp, R, c.rg);
+                q = screen_score_st<RT, G, F>(u, v, g, c.sp, R, c.rg);
         }
         float m1 = q, m2 = INFINITY;
         for (int dd = 1; dd < K; dd <<= 1) {
@@ -220,20 +220,54 @@ __device__ void process_tile_uniform(WarpCtx<RT, G> &c, const TileDesc &d, const
         const float thr = __fadd_ru(m1, c.sp.e2);
         const bool amb = c.sp.exact || !(m2 > thr);
         const int64_t job = d.job_begin + (i >> log2_k);
-        if (valid && !amb && q == m1)
+        if (valid && !amb && q == m1) {
+            stage_units_to_int<RT, F>(u, R);
             take_winner<RT, G>(c, job, i & (K - 1), u, v, g, false, 0.0);
+        }
         const uint32_t amask = __ballot_sync(FULL, valid && amb && (i & (K - 1)) == 0);
         if (amask)
-            resolve_row<RT, G>(c, lane, amask, false, sp.units, sp.vals, sp.grp, i, i + K, thr, job, 0);
+            resolve_row<RT, G, F>(c, lane, amask, false, sp.units, sp.vals, sp.grp, i, i + K, thr, job, 0);
     }
 }
 
-// Units of the 4 consecutive options starting at p (16-byte aligned): six, four or eight 16-byte
-// shared loads for R = 6, 4, 8. Duplicate marks are removed and returned in dup[].
+// Half-swap of a lane's four options (R = 6 only). A lane's 4 options span 96 bytes, so in each
+// quarter-warp phase of a 16-byte shared load lanes l and l + 4 start in the same bank (96 bytes is
+// 24 banks; four such strides wrap the 32 banks): a two-way conflict on every load. A lane whose
+// group of four options has (group >> 2) odd reads the second half of its group (options 2, 3:
+// 48 bytes = 12 banks further) first, which moves its 16-byte window off the other lanes' windows
+// for every pair of the phase; its register slot s then holds option s ^ 2. The same swap of the two
+// 16-byte value halves removes the two-way conflict of the value loads (32-byte lane stride).
+// `opt0` is the tile-local index of the lane's first option (a multiple of 4).
 template <int RT>
-__device__ __forceinline__ void load_units4_smem(const int32_t *p, int32_t (*u)[Cols<RT>::N], bool *dup, int R)
+__device__ __forceinline__ int half_swap(int opt0)
 {
-    if constexpr (RT == 4 || RT == 6 || RT == 8) {
+    return RT == 6 ? (opt0 >> 4) & 1 : 0;
+}
+
+// Units of the 4 consecutive options starting at p (16-byte aligned): six, four or eight 16-byte
+// shared loads for R = 6, 4, 8. Duplicate marks are removed and returned in dup[]. With rot = 1
+// (R = 6, half_swap) slot s receives option s ^ 2.
+template <int RT>
+__device__ __forceinline__ void load_units4_smem(const int32_t *p, int32_t (*u)[Cols<RT>::N], bool *dup, int R,
+                                                 int rot = 0)
+{
+    if constexpr (RT == 6) {
+        int32_t raw[24];
+        const int4 *q4 = reinterpret_cast<const int4 *>(p);
+        const int4 *pa = q4 + 3 * rot, *pb = q4 + (3 - 3 * rot);
+#pragma unroll
+        for (int k = 0; k < 3; ++k) {
+            const int4 x = pa[k];
+            raw[4 * k] = x.x; raw[4 * k + 1] = x.y; raw[4 * k + 2] = x.z; raw[4 * k + 3] = x.w;
+            const int4 y = pb[k];
+            raw[12 + 4 * k] = y.x; raw[12 + 4 * k + 1] = y.y; raw[12 + 4 * k + 2] = y.z; raw[12 + 4 * k + 3] = y.w;
+        }
+#pragma unroll
+        for (int o = 0; o < 4; ++o)
+#pragma unroll
+            for (int r = 0; r < 6; ++r)
+                u[o][r] = raw[o * 6 + r];
+    } else if constexpr (RT == 4 || RT == 8) {
         constexpr int W = RT;
         int32_t raw[4 * W];
         const int4 *q4 = reinterpret_cast<const int4 *>(p);
@@ -267,22 +301,24 @@ __device__ __forceinline__ void load_units4_smem(const int32_t *p, int32_t (*u)[
 // lexicographic minimum of (s, job-local index), and the lane holding that option records it.
 // The options are still in the stage, so no option is read twice from memory. base: tile-local
 // index of the lane's first option; loc0: its job-local index; lamb: the lane's job is ambiguous.
-template <int RT, bool G>
+template <int RT, bool G, bool F>
 __device__ __forceinline__ void resolve4_in_row(WarpCtx<RT, G> &c, const StagePtrs &sp, bool lamb, const float *q,
-                                                uint32_t dupmask, float thr, int base, int loc0, int64_t job, int L)
+                                                uint32_t dupmask, float thr, int base, int loc0, int64_t job, int L,
+                                                int rot)
 {
     long long key = 0x7fffffffffffffffLL;
     int bi = kIdxNone;
     if (lamb) {
 #pragma unroll
-        for (int o = 0; o < 4; ++o) {
-            const bool cand = c.sp.exact ? !((dupmask >> o) & 1u) : (q[o] <= thr);
+        for (int s = 0; s < 4; ++s) {   // slot s holds option s ^ (2 rot)
+            const bool cand = c.sp.exact ? !((dupmask >> s) & 1u) : (q[s] <= thr);
             if (!cand)
                 continue;
+            const int o = s ^ (rot << 1);
             int32_t u[Cols<RT>::N];
-            load_units_smem<RT>(sp.units + (size_t)(base + o) * c.R, u, c.R);
+            load_units_stage<RT, F>(sp.units + (size_t)(base + o) * c.R, u, c.R);
             const long long k = order_key(exact_score<RT, G>(u, sp.vals[base + o], 0, c.sp, c.R, c.rg));
-            if (k < key) {
+            if (k < key || (k == key && loc0 + o < bi)) {
                 key = k;
                 bi = loc0 + o;
             }
@@ -299,7 +335,7 @@ __device__ __forceinline__ void resolve4_in_row(WarpCtx<RT, G> &c, const StagePt
     if (lamb && bi >= loc0 && bi < loc0 + 4) {
         const int i = base + (bi - loc0);
         int32_t uw[Cols<RT>::N];
-        load_units_smem<RT>(sp.units + (size_t)i * c.R, uw, c.R);
+        load_units_stage<RT, F>(sp.units + (size_t)i * c.R, uw, c.R);
         take_winner<RT, G>(c, job, bi, uw, sp.vals[i], 0, true, key_value(key));
         atomicAdd(c.st.stats, 1ull);
     }
@@ -309,7 +345,7 @@ __device__ __forceinline__ void resolve4_in_row(WarpCtx<RT, G> &c, const StagePt
 // consecutive options of one job (a tile row block is 128 options), keeps their smallest and
 // second-smallest screen values, and a log2(K / 4)-step xor butterfly over the job's K / 4 lanes
 // completes the job. An unambiguous job's winner is the unique option holding the smallest value.
-template <int RT, bool G>
+template <int RT, bool G, bool F>
 __device__ void process_tile_uniform4(WarpCtx<RT, G> &c, const TileDesc &d, const StagePtrs &sp, int lane)
 {
     const int R = c.R;
@@ -319,20 +355,21 @@ __device__ void process_tile_uniform4(WarpCtx<RT, G> &c, const TileDesc &d, cons
     for (int b = 0; b < n; b += 128) {
         const int base = b + 4 * lane;
         const bool valid = base < n;        // n is a multiple of K, hence of 4
+        const int rot = 0;   // measured slower with the half swap on this path
         float q[4] = {INFINITY, INFINITY, INFINITY, INFINITY};
         uint32_t dupmask = 0;
         if (valid) {
             int32_t u[4][Cols<RT>::N];
             bool dup[4];
-            load_units4_smem<RT>(sp.units + (size_t)base * R, u, dup, R);
-            const double2 va = reinterpret_cast<const double2 *>(sp.vals + base)[0];
-            const double2 vb = reinterpret_cast<const double2 *>(sp.vals + base)[1];
+            load_units4_smem<RT>(sp.units + (size_t)base * R, u, dup, R, rot);
+            const double2 va = reinterpret_cast<const double2 *>(sp.vals + base)[rot];
+            const double2 vb = reinterpret_cast<const double2 *>(sp.vals + base)[rot ^ 1];
             const double v[4] = {va.x, va.y, vb.x, vb.y};
 #pragma unroll
             for (int o = 0; o < 4; ++o) {
                 dupmask |= dup[o] ? (1u << o) : 0u;
                 if (!dup[o])
-                    q[o] = screen_score<RT, G>(u[o], v[o], 0, c.sp, R, c.rg);
+                    q[o] = screen_score_st<RT, G, F>(u[o], v[o], 0, c.sp, R, c.rg);
             }
         }
         // smallest and second smallest of the lane's four values
@@ -349,22 +386,23 @@ __device__ void process_tile_uniform4(WarpCtx<RT, G> &c, const TileDesc &d, cons
         const float thr = __fadd_ru(m1, c.sp.e2);
         const bool amb = c.sp.exact || !(m2 > thr);
         if (valid && !amb) {
+            // an unambiguous job's smallest value is held by one slot only (a tie would make m2 = m1)
             int w = -1;
 #pragma unroll
             for (int o = 3; o >= 0; --o)
                 if (q[o] == m1)
-                    w = o;
+                    w = o ^ (rot << 1);
             if (w >= 0) {
                 const int i = base + w;
                 int32_t uw[Cols<RT>::N];
-                load_units_smem<RT>(sp.units + (size_t)i * R, uw, R);
+                load_units_stage<RT, F>(sp.units + (size_t)i * R, uw, R);
                 take_winner<RT, G>(c, d.job_begin + (i >> c.log2_k), i & (K - 1), uw, sp.vals[i], 0, false, 0.0);
             }
         }
         const bool lamb = valid && amb;
         if (__any_sync(FULL, lamb))
-            resolve4_in_row<RT, G>(c, sp, lamb, q, dupmask, thr, base, base & (K - 1),
-                                   d.job_begin + (base >> c.log2_k), KL);
+            resolve4_in_row<RT, G, F>(c, sp, lamb, q, dupmask, thr, base, base & (K - 1),
+                                   d.job_begin + (base >> c.log2_k), KL, rot);
     }
 }
 
@@ -374,7 +412,7 @@ __device__ void process_tile_uniform4(WarpCtx<RT, G> &c, const TileDesc &d, cons
 // lanes keeps the lexicographic minimum of (s, job-local index), and the lane holding that option
 // records it. base: tile-local index of the lane's first option; loc: its job-local index; lamb: the
 // lane's job is ambiguous.
-template <int RT, bool G>
+template <int RT, bool G, bool F>
 __device__ __forceinline__ void resolve_run_row(WarpCtx<RT, G> &c, const StagePtrs &sp, bool lamb, float thr,
                                                 int base, int loc, int64_t job, int L)
 {
@@ -383,7 +421,7 @@ __device__ __forceinline__ void resolve_run_row(WarpCtx<RT, G> &c, const StagePt
     if (lamb) {
         for (int o = 0; o < 4; ++o) {
             int32_t u[Cols<RT>::N];
-            if (load_units_smem<RT>(sp.units + (size_t)(base + o) * c.R, u, c.R))
+            if (load_units_stage<RT, F>(sp.units + (size_t)(base + o) * c.R, u, c.R))
                 continue;
             const double v = sp.vals[base + o];
             if (!c.sp.exact && !(screen_score<RT, G>(u, v, 0, c.sp, c.R, c.rg) <= thr))
@@ -406,7 +444,7 @@ __device__ __forceinline__ void resolve_run_row(WarpCtx<RT, G> &c, const StagePt
     if (lamb && bi >= loc && bi < loc + 4) {
         const int i = base + (bi - loc);
         int32_t uw[Cols<RT>::N];
-        load_units_smem<RT>(sp.units + (size_t)i * c.R, uw, c.R);
+        load_units_stage<RT, F>(sp.units + (size_t)i * c.R, uw, c.R);
         take_winner<RT, G>(c, job, bi, uw, sp.vals[i], 0, true, key_value(key));
         atomicAdd(c.st.stats, 1ull);
     }
@@ -418,7 +456,7 @@ __device__ __forceinline__ void resolve_run_row(WarpCtx<RT, G> &c, const StagePt
 // index) and second-smallest value; lanes past the job's end idle. A log2(L)-step xor butterfly of
 // (smallest, second smallest) completes the job as in the uniform path; an unambiguous job's winner
 // is the unique option holding the smallest value, recorded by the lane that holds it.
-template <int RT, bool G>
+template <int RT, bool G, bool F>
 __device__ void process_tile_run4(WarpCtx<RT, G> &c, const TileDesc &d, const StagePtrs &sp, int lane, int K)
 {
     const int R = c.R;
@@ -433,21 +471,24 @@ __device__ void process_tile_run4(WarpCtx<RT, G> &c, const TileDesc &d, const St
         const int loc = 4 * sub;
         const bool valid = jl < n_job && sub < m;
         const int base = jl * K + loc;
+        const int rot = half_swap<RT>(base);   // slot s holds option s ^ (2 rot)
         float m1 = INFINITY, m2 = INFINITY;
         int i1 = kIdxNone;
         if (valid) {
             int32_t u[4][Cols<RT>::N];
             bool dup[4];
-            load_units4_smem<RT>(sp.units + (size_t)base * R, u, dup, R);
-            const double2 va = reinterpret_cast<const double2 *>(sp.vals + base)[0];
-            const double2 vb = reinterpret_cast<const double2 *>(sp.vals + base)[1];
+            load_units4_smem<RT>(sp.units + (size_t)base * R, u, dup, R, rot);
+            const double2 va = reinterpret_cast<const double2 *>(sp.vals + base)[rot];
+            const double2 vb = reinterpret_cast<const double2 *>(sp.vals + base)[rot ^ 1];
             const double v[4] = {va.x, va.y, vb.x, vb.y};
+            // m1 and m2 do not depend on the order the slots are taken in; i1 matters only when the
+            // smallest value is held by one slot (otherwise m2 = m1 and the job is ambiguous)
 #pragma unroll
             for (int o = 0; o < 4; ++o) {
-                const float q = dup[o] ? INFINITY : screen_score<RT, G>(u[o], v[o], 0, c.sp, R, c.rg);
+                const float q = dup[o] ? INFINITY : screen_score_st<RT, G, F>(u[o], v[o], 0, c.sp, R, c.rg);
                 const bool better = q < m1;
                 m2 = better ? m1 : fminf(m2, q);
-                i1 = better ? loc + o : i1;
+                i1 = better ? loc + (o ^ (rot << 1)) : i1;
                 m1 = fminf(m1, q);
             }
         }
@@ -464,12 +505,12 @@ __device__ void process_tile_run4(WarpCtx<RT, G> &c, const TileDesc &d, const St
         if (valid && !amb && lm1 == m1) {
             const int i = jl * K + i1;
             int32_t uw[Cols<RT>::N];
-            load_units_smem<RT>(sp.units + (size_t)i * R, uw, R);
+            load_units_stage<RT, F>(sp.units + (size_t)i * R, uw, R);
             take_winner<RT, G>(c, job, i1, uw, sp.vals[i], 0, false, 0.0);
         }
         const bool lamb = valid && amb;
         if (__any_sync(FULL, lamb))
-            resolve_run_row<RT, G>(c, sp, lamb, thr, base, loc, job, L);
+            resolve_run_row<RT, G, F>(c, sp, lamb, thr, base, loc, job, L);
     }
 }
 
@@ -478,7 +519,7 @@ __device__ void process_tile_run4(WarpCtx<RT, G> &c, const TileDesc &d, const St
 // offsets; a job continuing from the previous row enters as a carry; rows entirely inside one job
 // only fold per lane. A job larger than a tile arrives as consecutive chunk tiles of this warp
 // (big_first / big_carry carry its state across them) and is resolved from global memory.
-template <int RT, bool G>
+template <int RT, bool G, bool F>
 __device__ void process_tile_general(WarpCtx<RT, G> &c, const TileDesc &d, const StagePtrs &sp, int64_t &big_first,
                                      Best &big_carry, int lane)
 {
@@ -507,7 +548,7 @@ __device__ void process_tile_general(WarpCtx<RT, G> &c, const TileDesc &d, const
         int32_t u[Cols<RT>::N];
         float q = INFINITY;
         if (valid) {
-            const bool dup = load_units_smem<RT>(sp.units + (size_t)i * R, u, R);
+            const bool dup = load_units_stage<RT, F>(sp.units + (size_t)i * R, u, R);
             const double v = sp.vals[i];
             const int g = G ? (int)sp.grp[i] : 0;
             if (!dup)
@@ -580,13 +621,13 @@ __device__ void process_tile_general(WarpCtx<RT, G> &c, const TileDesc &d, const
             int32_t uw[Cols<RT>::N];
             double vw;
             int gw;
-            load_option<RT, G>(c, !big, sp.units, sp.vals, sp.grp, big ? x.idx : x.idx, big ? big_first : 0, uw, vw,
+            load_option<RT, G, F>(c, !big, sp.units, sp.vals, sp.grp, big ? x.idx : x.idx, big ? big_first : 0, uw, vw,
                                gw);
             take_winner<RT, G>(c, job, li, uw, vw, gw, false, 0.0);
         }
         const uint32_t amask = __ballot_sync(FULL, amb);
         if (amask)
-            resolve_row<RT, G>(c, lane, amask, big, sp.units, sp.vals, sp.grp, jstart, jend, thr, job, big_first);
+            resolve_row<RT, G, F>(c, lane, amask, big, sp.units, sp.vals, sp.grp, jstart, jend, thr, job, big_first);
     }
     if (big) {
         if (priv_dirty)
@@ -597,7 +638,7 @@ __device__ void process_tile_general(WarpCtx<RT, G> &c, const TileDesc &d, const
 // needed. Each lane folds the options it owns (lane-strided: conflict-free shared loads) into a
 // lane-private state carried across the job's chunks; the job's last chunk reduces the states across
 // the warp once and records the winner (exact resolution from global memory when ambiguous).
-template <int RT, bool G>
+template <int RT, bool G, bool F>
 __device__ void process_tile_bigchunk(WarpCtx<RT, G> &c, const TileDesc &d, const StagePtrs &sp, int64_t &big_first,
                                       Best &big_priv, int lane)
 {
@@ -624,7 +665,7 @@ __device__ void process_tile_bigchunk(WarpCtx<RT, G> &c, const TileDesc &d, cons
                 const double v = sp.vals[i];
                 const int g = G ? (int)sp.grp[i] : 0;
                 if (!dup)
-                    q[o] = screen_score<RT, G>(u, v, g, c.sp, R, c.rg);
+                    q[o] = screen_score_st<RT, G, F>(u, v, g, c.sp, R, c.rg);
             }
         }
 #pragma unroll
@@ -641,7 +682,7 @@ __device__ void process_tile_bigchunk(WarpCtx<RT, G> &c, const TileDesc &d, cons
         const bool dup = load_units_smem<RT>(sp.units + (size_t)i * R, u, R);
         const double v = sp.vals[i];
         const int g = G ? (int)sp.grp[i] : 0;
-        const float q = dup ? INFINITY : screen_score<RT, G>(u, v, g, c.sp, R, c.rg);
+        const float q = dup ? INFINITY : screen_score_st<RT, G, F>(u, v, g, c.sp, R, c.rg);
         big_priv = combine(big_priv, Best{q, dup ? kIdxNone : chunk_base + i, INFINITY});
     }
 #endif
@@ -659,7 +700,7 @@ __device__ void process_tile_bigchunk(WarpCtx<RT, G> &c, const TileDesc &d, cons
             double vw;
             int gw;
             const bool here = x.idx >= chunk_base;
-            load_option<RT, G>(c, here, sp.units, sp.vals, sp.grp, here ? x.idx - chunk_base : x.idx, big_first, uw,
+            load_option<RT, G, F>(c, here, sp.units, sp.vals, sp.grp, here ? x.idx - chunk_base : x.idx, big_first, uw,
                                vw, gw);
             take_winner<RT, G>(c, d.job_begin, x.idx, uw, vw, gw, false, 0.0);
         }
@@ -672,7 +713,7 @@ __device__ void process_tile_bigchunk(WarpCtx<RT, G> &c, const TileDesc &d, cons
             int32_t u[Cols<RT>::N];
             double v;
             int g;
-            load_option<RT, G>(c, false, sp.units, sp.vals, sp.grp, big_priv.idx, big_first, u, v, g);
+            load_option<RT, G, F>(c, false, sp.units, sp.vals, sp.grp, big_priv.idx, big_first, u, v, g);
             key = order_key(exact_score<RT, G>(u, v, g, c.sp, c.R, c.rg));
             bi = big_priv.idx;
         }
@@ -689,12 +730,12 @@ __device__ void process_tile_bigchunk(WarpCtx<RT, G> &c, const TileDesc &d, cons
             int32_t uw[Cols<RT>::N];
             double vw;
             int gw;
-            load_option<RT, G>(c, false, sp.units, sp.vals, sp.grp, bi, big_first, uw, vw, gw);
+            load_option<RT, G, F>(c, false, sp.units, sp.vals, sp.grp, bi, big_first, uw, vw, gw);
             take_winner<RT, G>(c, d.job_begin, bi, uw, vw, gw, true, key_value(key));
             atomicAdd(c.st.stats, 1ull);
         }
     } else {
-        resolve_row<RT, G>(c, lane, 1u, true, sp.units, sp.vals, sp.grp, 0, K, thr, d.job_begin, big_first);
+        resolve_row<RT, G, F>(c, lane, 1u, true, sp.units, sp.vals, sp.grp, 0, K, thr, d.job_begin, big_first);
     }
 }
 }  // namespace

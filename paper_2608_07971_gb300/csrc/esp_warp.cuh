@@ -59,7 +59,8 @@ __device__ __forceinline__ double exact_score(const int32_t *u, double v, int g,
     for (int r = 0; r < Cols<RT>::N; ++r) {
         if (RT == 0 && r >= R)
             break;
-        const double price = __ldg(sp.p64g + ((G && r >= rg) ? rg + (R - rg) * g + (r - rg) : r));
+        // through L2: a persistent pass sees the prices change between rounds
+        const double price = __ldcg(sp.p64g + ((G && r >= rg) ? rg + (R - rg) * g + (r - rg) : r));
         s = __fma_rn(price, __int2double_rn(u[r]), s);
     }
     return s;
@@ -92,6 +93,49 @@ __device__ __forceinline__ bool load_units_smem(const int32_t *p, int32_t *u, in
     return dup;
 }
 
+// Units staged as fp32 bit patterns (F: the tile-interleaved copy of a table whose units are all
+// below 2^23, each converted exactly at load; the duplicate mark stays the sign bit of column 0). The
+// screen takes them as they are: the same fp32 values the conversion of the integers gives, so the
+// same q, without a conversion per unit. Every other use converts them back to the integers.
+template <int RT, bool G, bool F>
+__device__ __forceinline__ float screen_score_st(const int32_t *u, double v, int g, const ScenarioPrices &sp, int R,
+                                                 int rg)
+{
+    if constexpr (F) {
+        static_assert(!G, "fp32 stage units only for tables without a group column");
+        float q = -screen_value(v);
+#pragma unroll
+        for (int r = 0; r < Cols<RT>::N; ++r) {
+            if (RT == 0 && r >= R)
+                break;
+            q = __fmaf_rn(sp.pf[r], __int_as_float(u[r]), q);
+        }
+        return q;
+    } else {
+        return screen_score<RT, G>(u, v, g, sp, R, rg);
+    }
+}
+
+template <int RT, bool F>
+__device__ __forceinline__ void stage_units_to_int(int32_t *u, int R)
+{
+    if constexpr (F) {
+#pragma unroll
+        for (int r = 0; r < Cols<RT>::N; ++r)
+            if (RT != 0 || r < R)
+                u[r] = __float2int_rn(__int_as_float(u[r]));
+    }
+}
+
+// Units of one staged option as integers (duplicate mark removed and returned).
+template <int RT, bool F>
+__device__ __forceinline__ bool load_units_stage(const int32_t *p, int32_t *u, int R)
+{
+    const bool dup = load_units_smem<RT>(p, u, R);
+    stage_units_to_int<RT, F>(u, R);
+    return dup;
+}
+
 template <int RT>
 __device__ __forceinline__ bool load_units_global(const int32_t *p, int32_t *u, int R)
 {
@@ -115,7 +159,7 @@ __device__ void set_prices(const DevTable &t, const DevState &st, const SolveArg
     const int P = t.P, R = t.R;
     bool huge = false;
     auto price_of = [&](int k) {
-        const double lam = st.lam[(size_t)s * P + k];
+        const double lam = __ldcg(st.lam + (size_t)s * P + k);
         const double p = effective_price(lam, (double)t.cap[(size_t)s * P + k], a.mode);
         st.p64[(size_t)s * P + k] = p;
         st.p32[(size_t)s * P + k] = __double2float_rn(p);
@@ -134,11 +178,11 @@ __device__ void set_prices(const DevTable &t, const DevState &st, const SolveArg
     double term = 0.0;
     const int rg = (t.n_groups == 0) ? R : t.r_global;
     if (lane < rg)
-        term = st.p64[(size_t)s * P + lane] * (double)st.umax[(size_t)s * R + lane];
+        term = __ldcg(st.p64 + (size_t)s * P + lane) * (double)st.umax[(size_t)s * R + lane];
     for (int c2 = 0; c2 < R - rg; ++c2) {
         double pm = 0.0;
         for (int gi = lane; gi < t.n_groups; gi += 32)
-            pm = fmax(pm, st.p64[(size_t)s * P + rg + (R - rg) * gi + c2]);
+            pm = fmax(pm, __ldcg(st.p64 + (size_t)s * P + rg + (R - rg) * gi + c2));
         pm = warp_max(pm);
         if (lane == rg + c2)
             term = pm * (double)st.umax[(size_t)s * R + lane];
@@ -192,7 +236,7 @@ __device__ void update_scenario(const DevTable &t, const DevState &st, const Sol
         const long long C = t.cap[sp + k];
         if (st.dem_trace)
             st.dem_trace[((size_t)s * T + round) * P + k] = U;
-        lam_out = st.lam[sp + k];
+        lam_out = __ldcg(st.lam + sp + k);
         return price_step(lam_out, U, C, (double)C, eta, a.mode);
     };
 #pragma unroll
@@ -238,7 +282,7 @@ __device__ void update_scenario(const DevTable &t, const DevState &st, const Sol
         } else {
             const long long U = (long long)__ldcg(st.U + sp + k);
             const long long C = t.cap[sp + k];
-            nl = price_step(st.lam[sp + k], U, C, (double)C, eta, a.mode);
+            nl = price_step(__ldcg(st.lam + sp + k), U, C, (double)C, eta, a.mode);
         }
         st.lam[sp + k] = nl;
         if (ZERO_U)
@@ -277,6 +321,9 @@ struct WarpCtx {
     int uniform_k;            // > 0: every job has this many options (a power of two <= 32)
     int log2_k;
     int s;                    // current scenario
+    bool persist;             // persistent pass: the update publishes the scenario's price version
+    const int32_t *scen_tiles;  // persistent pass: tiles of each scenario (arrivals count tiles)
+    int ntiles;               // persistent pass: tiles of the current scenario evaluated since the last flush
     ScenarioPrices sp;
     long long acc[Cols<RT>::N];   // per-lane demand of the globally priced columns
     unsigned long long hacc;
@@ -318,15 +365,32 @@ __device__ void flush(WarpCtx<RT, G> &c, int lane)
             __syncwarp();
             __threadfence();
         }
+        // the persistent pass counts tiles (a warp flushes when its scenario or round changes, whatever
+        // the plan's ranges); the round pass counts the plan's warps
+        const unsigned int add = c.persist ? (unsigned int)c.ntiles : 1u;
+        const unsigned int need = (unsigned int)__ldg((c.persist ? c.scen_tiles : c.scen_warps) + c.s);
+        c.ntiles = 0;
         unsigned int old = 0;
         if (lane == 0)
-            asm volatile("atom.add.release.gpu.u32 %0, [%1], 1;" : "=r"(old) : "l"(c.st.arrive + c.s) : "memory");
+            asm volatile("atom.add.release.gpu.u32 %0, [%1], %2;" : "=r"(old) : "l"(c.st.arrive + c.s), "r"(add)
+                         : "memory");
         old = __shfl_sync(FULL, old, 0);
-        if (old + 1 == (unsigned int)__ldg(c.scen_warps + c.s)) {
+        if (old + add == need) {
             asm volatile("fence.acq_rel.gpu;" ::: "memory");
             update_scenario<G ? 8 : 1>(c.t, c.st, c.a, c.s, c.round, lane);
             if (lane == 0)
                 c.st.arrive[c.s] = 0u;     // every warp of this pass has arrived
+            if (c.persist) {
+                // publish the scenario's next round: every lane's writes (prices, bound, cleared
+                // demand) are fenced before lane 0's release of the version; a stopped scenario
+                // releases every later round at once (its warps then skip it)
+                __threadfence();
+                __syncwarp();
+                if (lane == 0) {
+                    const unsigned int v = c.st.frozen[c.s] ? kVerStopped : (unsigned int)(c.round + 1);
+                    asm volatile("st.release.gpu.u32 [%0], %1;" ::"l"(c.st.ver + c.s), "r"(v) : "memory");
+                }
+            }
         }
     }
 }

@@ -30,7 +30,8 @@ EXPORTED = [
     "esp_debug_tile_options", "esp_debug_plan", "esp_debug_stats", "esp_debug_resident",
     "esp_debug_sort_layout", "esp_debug_plan_runs", "esp_debug_set_sorted_layout", "esp_debug_set_pdl", "esp_debug_set_plan_waves",
     "esp_debug_hold_barrier", "esp_debug_set_wait_limit", "esp_debug_hold_stage", "esp_debug_fail_alloc",
-    "esp_debug_pass_kernel", "esp_debug_set_interleave",
+    "esp_debug_pass_kernel", "esp_debug_set_interleave", "esp_debug_set_stage_f32",
+    "esp_debug_set_persistent", "esp_debug_persistent", "esp_debug_persist_waits",
     "esp_evaluate_noalloc",
     "esp_set_penalties", "esp_adaptive_threshold", "esp_effective_capacity", "esp_load_placement",
     "esp_iac_create", "esp_iac_set_stream", "esp_iac_load_model", "esp_iac_predict", "esp_iac_predict_host",
@@ -105,6 +106,10 @@ def load_library(path: Optional[str] = None):
         "esp_debug_fail_alloc": ([vp, i64], st),
         "esp_debug_pass_kernel": ([vp, ctypes.POINTER(i32)], st),
         "esp_debug_set_interleave": ([vp, i32], st),
+        "esp_debug_set_stage_f32": ([vp, i32], st),
+        "esp_debug_set_persistent": ([vp, i32], st),
+        "esp_debug_persistent": ([vp, ctypes.POINTER(i32)], st),
+        "esp_debug_persist_waits": ([vp, ctypes.POINTER(i64), ctypes.POINTER(i64), i32], st),
         "esp_set_penalties": ([vp, ctypes.c_double, vp, ctypes.c_double, vp, vp], st),
         "esp_load_placement": ([vp, i32, i32, i32, i32, i32, i32, vp, vp, vp, vp, i32, vp, vp, vp], st),
         "esp_adaptive_threshold": ([i64, vp, ctypes.c_double, ctypes.c_double, ctypes.c_double, ctypes.c_double, vp],
@@ -482,9 +487,36 @@ def esp_debug_set_interleave(ctx: int, enable: bool) -> None:
     _check(load_library().esp_debug_set_interleave(ctx, 1 if enable else 0), "esp_debug_set_interleave")
 
 
+def esp_debug_set_stage_f32(ctx: int, enable: bool) -> None:
+    """Later loads store the units of the tile-interleaved table as fp32 where every unit is below 2^23
+    (True, the default) or keep them as integers."""
+    _check(load_library().esp_debug_set_stage_f32(ctx, 1 if enable else 0), "esp_debug_set_stage_f32")
+
+
+def esp_debug_set_persistent(ctx: int, mode: int) -> None:
+    """Persistent pass of later solves: -1 automatic (the default), 0 never (one launch per round), 1
+    wherever the table can take it."""
+    _check(load_library().esp_debug_set_persistent(ctx, int(mode)), "esp_debug_set_persistent")
+
+
+def esp_debug_persistent(ctx: int) -> int:
+    """CTAs of the persistent launch a plain solve of the loaded table uses (0: one launch per round)."""
+    g = ctypes.c_int32()
+    _check(load_library().esp_debug_persistent(ctx, ctypes.byref(g)), "esp_debug_persistent")
+    return g.value
+
+
+def esp_debug_persist_waits(ctx: int, reset: bool = True):
+    """(nanoseconds, number) of the persistent pass's waits for a scenario's prices that had to poll."""
+    ns, n = ctypes.c_int64(), ctypes.c_int64()
+    _check(load_library().esp_debug_persist_waits(ctx, ctypes.byref(ns), ctypes.byref(n), 1 if reset else 0),
+           "esp_debug_persist_waits")
+    return ns.value, n.value
+
+
 def esp_debug_pass_kernel(ctx: int) -> int:
     """How the loaded table is evaluated: 0 per-warp pass, two copies per tile; 1 per-warp pass on the
-    tile-interleaved table, one copy per tile; 2 factored placement."""
+    tile-interleaved table, one copy per tile; 2 factored placement; 3 as 1 with fp32 units."""
     k = ctypes.c_int32()
     _check(load_library().esp_debug_pass_kernel(ctx, ctypes.byref(k)), "esp_debug_pass_kernel")
     return k.value

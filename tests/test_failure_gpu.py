@@ -40,7 +40,7 @@ def test_stage_wait_timeout_reports_and_poisons(interleave, table):
     s = esp.Solver()
     esp.esp_debug_set_interleave(s.ctx, interleave)
     s.load(t)
-    assert esp.esp_debug_pass_kernel(s.ctx) == (1 if interleave else 0)
+    assert esp.esp_debug_pass_kernel(s.ctx) == (3 if interleave else 0)
     ref = s.solve(0.05, 10)
     esp.esp_debug_set_wait_limit(s.ctx, 20)
     esp.esp_debug_hold_stage(s.ctx)

@@ -333,7 +333,8 @@ def test_programmatic_dependent_launch_is_transparent(graph):
     s.close()
 
 
-@pytest.mark.parametrize("case", ["whatif", "heavy", "ragged256", "k1", "k2", "r4k8", "r5k4"])
+@pytest.mark.parametrize("case", ["whatif", "heavy", "ragged256", "k1", "k2", "r4k8", "r5k4", "big_units_k16",
+                                  "big_units_ragged"])
 def test_interleaved_tiles_equal_separate_arrays(case):
     """The per-warp pass reads each tile's units and values with one bulk copy from a tile-interleaved
     copy of the table (the default wherever every tile allows it) or with two copies from the separate
@@ -350,6 +351,10 @@ def test_interleaved_tiles_equal_separate_arrays(case):
         t = W.random_table(rng, S=2, J=2000, R=6, kmin=K, kmax=K, umax=5000)
     elif case == "r4k8":
         t = W.random_table(rng, S=2, J=900, R=4, kmin=8, kmax=8, umax=5000)
+    elif case == "big_units_k16":     # units up to 2^24: fp32 would not hold them exactly
+        t = W.random_table(rng, S=2, J=900, R=6, kmin=16, kmax=16, umax=1 << 24)
+    elif case == "big_units_ragged":
+        t = W.random_table(rng, S=2, J=700, R=6, kmin=1, kmax=200, umax=1 << 24)
     else:
         t = W.random_table(rng, S=2, J=900, R=5, kmin=4, kmax=4, umax=5000)
     a = esp.Solver(t)
@@ -357,11 +362,19 @@ def test_interleaved_tiles_equal_separate_arrays(case):
     esp.esp_debug_set_interleave(b.ctx, False)
     b.load(t)
     assert esp.esp_debug_pass_kernel(b.ctx) == 0
+    c = esp.Solver()
+    esp.esp_debug_set_stage_f32(c.ctx, False)
+    c.load(t)
     T = 30
     sa = a.solve(0.05, T, traces=True)
     sb = b.solve(0.05, T, traces=True)
+    sc = c.solve(0.05, T, traces=True)
     for f in ("lam", "sel", "demand", "lambda_trace", "demand_trace", "selhash_trace"):
         assert np.array_equal(getattr(sa, f), getattr(sb, f), equal_nan=True), f
+        assert np.array_equal(getattr(sc, f), getattr(sb, f), equal_nan=True), f
     check_solution(t, sa, list(range(t.S)), 0.05, T, esp.ESP_PRICE_NORMALIZED, esp.ESP_STEP_FIXED)
-    if case in ("whatif", "heavy", "ragged256", "r4k8", "r5k4"):
-        assert esp.esp_debug_pass_kernel(a.ctx) == 1, "the table should take the interleaved tiles"
+    if case in ("whatif", "heavy", "ragged256", "r4k8", "r5k4", "big_units_k16", "big_units_ragged"):
+        # R = 4, 6, 8 with every unit below 2^23: fp32 units in the interleaved tiles
+        f32 = case not in ("r5k4", "big_units_k16", "big_units_ragged")
+        assert esp.esp_debug_pass_kernel(a.ctx) == (3 if f32 else 1), "the table should take the interleaved tiles"
+        assert esp.esp_debug_pass_kernel(c.ctx) == 1

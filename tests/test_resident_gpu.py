@@ -202,14 +202,15 @@ def test_resident_in_graph_with_pass_events():
 
 def test_resident_falls_back_to_streaming_when_predicted_slower():
     """A batch of many scenarios needs many waves of clusters: the cost model predicts the resident solve
-    slower than streaming, so ESP_FLAG_RESIDENT runs the streaming path (T + 3 launches) with the same
-    results, unless a cluster size is forced. One 2048-job scenario keeps the resident solve."""
+    slower than streaming, so ESP_FLAG_RESIDENT runs the streaming path (its rounds in one persistent
+    launch: 4 launches) with the same results, unless a cluster size is forced. One 2048-job scenario
+    keeps the resident solve."""
     w = W.whatif_batch(scenarios=list(range(256)))
     t = w.table
     s = esp.Solver(t)
     assert esp.esp_debug_resident(s.ctx) is not None          # it could run resident ...
     a = s.solve(w.eta0, 20, flags=RES)
-    assert s.launches() == 20 + 3                             # ... but streams
+    assert s.launches() == 4                                  # ... but streams
     b = s.solve(w.eta0, 20)
     assert np.array_equal(a.lam, b.lam) and np.array_equal(a.sel, b.sel)
     cs, _ = esp.esp_debug_resident(s.ctx)
