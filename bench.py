@@ -407,8 +407,13 @@ def time_streaming(esp, solver, w, T, args, dist, barrier, stream, clk=None):
     ev_avg_ms = pass_ms / max(n_pass, 1)
     ev_achieved = bytes_pass / (ev_avg_ms / 1e3) / 1e9 if n_pass else None
     kind = {0: "k_pass (per-warp pass, two bulk copies per tile)",
-            1: "k_pass (per-warp pass, one bulk copy per tile from the tile-interleaved table)"}.get(
+            1: "k_pass (per-warp pass, one bulk copy per tile from the tile-interleaved table)",
+            3: "k_pass (per-warp pass, one bulk copy per tile, fp32 units)"}.get(
         esp.esp_debug_pass_kernel(ctx), "k_place (factored placement pass)")
+    persist = esp.esp_debug_persistent(ctx) > 0
+    if persist:
+        kind = ("k_pass_persist (rounds 0..T-1 in one cooperative launch, scenarios released by their price "
+                "updates; one bulk copy per tile, fp32 units) + k_pass (final pass)")
     roofline = {"bound": "hbm", "kernel": kind + ": best response + demand aggregation + fused price update",
                 "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
                 "traffic": kernel_traffic(w.name, t.n_opt),
@@ -416,16 +421,38 @@ def time_streaming(esp, solver, w, T, args, dist, barrier, stream, clk=None):
                 "frac_of_nominal_8tbs": achieved / 8000.0,
                 "bytes_per_launch": bytes_pass, "avg_launch_ms": avg_ms,
                 "launches_per_step": T + 1,
+                "persistent": persist,
+                "per_round_note": ("the T rounds run in one launch: bytes_per_launch and avg_launch_ms are per "
+                                   "round (the step's time over its T + 1 evaluation passes)") if persist else
+                                  "one launch per round",
                 "event_timed": {"avg_launch_ms": ev_avg_ms, "achieved": ev_achieved,
                                 "frac": (ev_achieved / peak) if ev_achieved else None, "launches": n_pass,
                                 "ms_per_step_outside_passes": other_ms,
                                 "note": "separate solves with an event pair around every pass (each pass then "
-                                        "launches alone, without overlapping the kernel before it)"},
+                                        "launches alone, without overlapping the kernel before it; per-pass "
+                                        "events always use one launch per round)"},
                 "exact_resolutions_per_pass": n_res / max(1, (args.warmup + args.steps) * (T + 1)),
                 "duplicates_marked": n_marked}
     return {"value": value, "unit": "option-evals/s", "ms_per_step": step_s * 1e3,
             "rounds_per_sec": T / step_s, "evals_per_step": evals_step, "roofline": roofline,
             "launches_per_step": launches_per_step, "device_ms_last_solve": float(res["device_ms"][0])}
+
+
+def gpu_local_cpus(device: int):
+    """The host CPUs on the GPU's own NUMA node (from the PCI device's local_cpulist), or None."""
+    try:
+        import torch
+        p = torch.cuda.get_device_properties(device)
+        bus = f"{p.pci_domain_id:04x}:{p.pci_bus_id:02x}:{p.pci_device_id:02x}.0"
+        with open(f"/sys/bus/pci/devices/{bus}/local_cpulist") as f:
+            spec = f.read().strip()
+        cpus = set()
+        for part in spec.split(","):
+            a, _, b = part.partition("-")
+            cpus.update(range(int(a), int(b or a) + 1))
+        return cpus or None
+    except Exception:
+        return None
 
 
 def time_e2e(esp, solver, w, T, args, dist, barrier, stream, local):
@@ -435,10 +462,31 @@ def time_e2e(esp, solver, w, T, args, dist, barrier, stream, local):
     (esp_solve_async); every step still pays its own copies, inside the timed region."""
     import torch
     t = w.table
+    # the host buffers live on the GPU's own NUMA node: the pinned copies are made (first touched) by
+    # this thread while it runs on that node's CPUs
+    near = gpu_local_cpus(local)
+    numa = "not bound (GPU-local CPUs unknown)"
+    if near:
+        try:
+            os.sched_setaffinity(0, near)
+            numa = f"host buffers first touched on the GPU's NUMA node ({len(near)} CPUs)"
+        except Exception:
+            pass
     pin = lambda a: torch.from_numpy(np.ascontiguousarray(a)).pin_memory()  # noqa: E731
     h_off, h_units, h_vals = pin(t.job_off), pin(t.units), pin(t.values)
     h_grp = None if t.group is None else pin(t.group.view(np.int16))
     h_cap = pin(t.capacity)
+    # the upload alone: the host-to-device copy of the step's inputs (a plain torch copy)
+    d_probe = torch.empty(h_units.numel() * 4 + h_vals.numel() * 8, dtype=torch.uint8, device="cuda")
+    probe = []
+    for _ in range(3):
+        torch.cuda.synchronize()
+        p0 = time.perf_counter()
+        d_probe[:h_units.numel() * 4].copy_(h_units.view(torch.uint8).reshape(-1), non_blocking=True)
+        d_probe[h_units.numel() * 4:].copy_(h_vals.view(torch.uint8).reshape(-1), non_blocking=True)
+        torch.cuda.synchronize()
+        probe.append((time.perf_counter() - p0) * 1e3)
+    del d_probe
     h_sel = [torch.empty((t.S, t.J), dtype=torch.int32).pin_memory() for _ in range(2)]
     h_lam = [torch.empty((t.S, t.P), dtype=torch.float64).pin_memory() for _ in range(2)]
     # a cold load: a new context (fresh buffers, nothing planned yet), on a stream of its own so that
@@ -453,26 +501,42 @@ def time_e2e(esp, solver, w, T, args, dist, barrier, stream, local):
     ctxs = [solver.ctx, other.ctx]
     prm = [s.params(w.eta0, T, mode=w.mode, step=w.step) for s in (solver, other)]
 
+    prof = []
+
     def load(i):
         esp.esp_load_options(ctxs[i], t.S, t.J, t.R, t.P, t.r_global, h_off, h_units, h_vals, h_grp, h_cap)
+        prof.append(esp.esp_debug_load_profile(ctxs[i]))
+
+    split = {"load": 0.0, "wait": 0.0}
 
     def run(steps):
         load(0)
         esp.esp_solve_async(ctxs[0], prm[0])
         for i in range(steps):
             cur, nxt = i % 2, (i + 1) % 2
+            c0 = time.perf_counter()
             if i + 1 < steps:
                 load(nxt)          # overlaps the current solve
+            c1 = time.perf_counter()
             esp.esp_get_selection(ctxs[cur], h_sel[cur])
             esp.esp_get_prices(ctxs[cur], h_lam[cur])
+            c2 = time.perf_counter()
+            split["load"] += c1 - c0
+            split["wait"] += c2 - c1
             if i + 1 < steps:
                 esp.esp_solve_async(ctxs[nxt], prm[nxt])
 
     run(max(2, args.warmup))
     barrier()
+    split["load"] = split["wait"] = 0.0
+    prof.clear()
+    # at least 8 steps: the pipeline's first upload has no solve to hide under
+    steps = max(args.steps, 8)
     t0 = time.perf_counter()
-    run(args.steps)
-    e2e_s = (time.perf_counter() - t0) / args.steps
+    run(steps)
+    e2e_s = (time.perf_counter() - t0) / steps
+    phases = np.mean([p[0] for p in prof], axis=0).tolist() if prof else None
+    allocs = int(sum(p[1] + p[2] for p in prof))
     barrier()
     # a warm load alone (same offsets: the host plan is reused), for the split of a step
     w0 = time.perf_counter()
@@ -486,8 +550,15 @@ def time_e2e(esp, solver, w, T, args, dist, barrier, stream, local):
     other.close()
     return {"value": e2e_value, "unit": "option-evals/s", "h2d_bytes_per_step": int(h2d),
             "d2h_bytes_per_step": int(d2h), "ms_per_step": e2e_s * 1e3,
-            "cold_load_ms": cold_ms, "warm_load_ms": warm_ms,
-            "pipeline": "two contexts: step i+1's upload overlaps step i's solve"}
+            "cold_load_ms": cold_ms, "warm_load_ms": warm_ms, "upload_alone_ms": probe,
+            "steps": steps,
+            "split_ms_per_step": {"load_overlapping_solve": split["load"] * 1e3 / steps,
+                                  "wait_for_solve_and_read_back": split["wait"] * 1e3 / steps},
+            "load_profile_ms": {"uploads_validation_queued": phases[0], "sorted_layout_queued": phases[1],
+                                "occupancy": phases[2], "planned": phases[3], "validated_marked": phases[4],
+                                "state_queued": phases[5], "returned": phases[6],
+                                "cuda_malloc_free_calls": allocs} if phases else None,
+            "pipeline": "two contexts: step i+1's upload overlaps step i's solve", "host_memory": numa}
 
 
 def run_ours(args):

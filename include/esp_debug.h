@@ -115,6 +115,14 @@ esp_status esp_debug_persistent(esp_ctx *ctx, int32_t *grid);
  * Waits for the context's stream; reset != 0 zeroes both. */
 esp_status esp_debug_persist_waits(esp_ctx *ctx, int64_t *ns, int64_t *waits, int32_t reset);
 
+/* Profile of the last esp_load_options / esp_load_options_device of this context: ms[0..6] the host
+ * milliseconds from its start until its uploads and validation were queued, until the sorted layout
+ * was queued, until the occupancy of the pass kernels was known, until the pass was planned, until
+ * the uploads, validation and duplicate marks were done, until the tiles, interleaved table and solve
+ * state were queued, and until it returned; *mallocs and *frees the cudaMalloc and cudaFree calls it
+ * made (a reload of a table of the same shape makes none). */
+esp_status esp_debug_load_profile(esp_ctx *ctx, double *ms, int64_t *mallocs, int64_t *frees);
+
 /* enable = 0 makes later loads keep integer units in the tile-interleaved table; 1 restores the
  * default (fp32 units where every unit is below 2^23 and the table has no group column, R = 4, 6 or 8,
  * uniform or sorted). Results are identical either way. */

@@ -32,6 +32,7 @@ EXPORTED = [
     "esp_debug_hold_barrier", "esp_debug_set_wait_limit", "esp_debug_hold_stage", "esp_debug_fail_alloc",
     "esp_debug_pass_kernel", "esp_debug_set_interleave", "esp_debug_set_stage_f32",
     "esp_debug_set_persistent", "esp_debug_persistent", "esp_debug_persist_waits",
+    "esp_debug_load_profile",
     "esp_evaluate_noalloc",
     "esp_set_penalties", "esp_adaptive_threshold", "esp_effective_capacity", "esp_load_placement",
     "esp_iac_create", "esp_iac_set_stream", "esp_iac_load_model", "esp_iac_predict", "esp_iac_predict_host",
@@ -110,6 +111,8 @@ def load_library(path: Optional[str] = None):
         "esp_debug_set_persistent": ([vp, i32], st),
         "esp_debug_persistent": ([vp, ctypes.POINTER(i32)], st),
         "esp_debug_persist_waits": ([vp, ctypes.POINTER(i64), ctypes.POINTER(i64), i32], st),
+        "esp_debug_load_profile": ([vp, ctypes.POINTER(ctypes.c_double), ctypes.POINTER(i64), ctypes.POINTER(i64)],
+                                   st),
         "esp_set_penalties": ([vp, ctypes.c_double, vp, ctypes.c_double, vp, vp], st),
         "esp_load_placement": ([vp, i32, i32, i32, i32, i32, i32, vp, vp, vp, vp, i32, vp, vp, vp], st),
         "esp_adaptive_threshold": ([i64, vp, ctypes.c_double, ctypes.c_double, ctypes.c_double, ctypes.c_double, vp],
@@ -512,6 +515,15 @@ def esp_debug_persist_waits(ctx: int, reset: bool = True):
     _check(load_library().esp_debug_persist_waits(ctx, ctypes.byref(ns), ctypes.byref(n), 1 if reset else 0),
            "esp_debug_persist_waits")
     return ns.value, n.value
+
+
+def esp_debug_load_profile(ctx: int):
+    """(host ms at the seven phase ends of the last load, cudaMalloc calls, cudaFree calls)."""
+    ms = (ctypes.c_double * 7)()
+    nm, nf = ctypes.c_int64(), ctypes.c_int64()
+    _check(load_library().esp_debug_load_profile(ctx, ms, ctypes.byref(nm), ctypes.byref(nf)),
+           "esp_debug_load_profile")
+    return list(ms), nm.value, nf.value
 
 
 def esp_debug_pass_kernel(ctx: int) -> int:
