@@ -8,6 +8,7 @@
 #include <stdint.h>
 
 #include "esp.h"
+#include "esp_iac.h"
 
 #ifdef __cplusplus
 extern "C" {
@@ -133,6 +134,16 @@ esp_status esp_debug_set_stage_f32(esp_ctx *ctx, int32_t enable);
  * values, one bulk copy per tile) wherever every tile allows it (esp_debug_pass_kernel then reports
  * 1). Results are identical either way. */
 esp_status esp_debug_set_interleave(esp_ctx *ctx, int32_t enable);
+
+/* Failure-detection hooks of the IAC predictor's tensor-core kernel (esp_iac.h). limit_ms bounds each
+ * wait for an MMA group (in polls of at most 1 ms; 0 restores the default, about 4 s).
+ * esp_iac_debug_hold_commit makes the next tensor-path launch leave its first MMA group in CTA 0's
+ * first warpgroup uncommitted, so that warpgroup's wait runs out: no memory is accessed out of place,
+ * the warpgroup then makes its barrier track every MMA still in flight, waits for them and leaves,
+ * and esp_iac_synchronize answers ESP_ERR_TIMEOUT; the handle then answers ESP_ERR_STATE (destroy it;
+ * the device stays usable). One launch only; ESP_ERR_UNSUPPORTED on the CUDA-core path. */
+esp_status esp_iac_debug_set_wait_limit(esp_iac *m, uint32_t limit_ms);
+esp_status esp_iac_debug_hold_commit(esp_iac *m);
 
 #ifdef __cplusplus
 }

@@ -17,6 +17,7 @@
 
 #include <cuda_runtime.h>
 
+#include "esp_debug.h"
 #include "esp_iac.h"
 #include "esp_iac_tc.cuh"
 
@@ -191,9 +192,9 @@ __device__ __forceinline__ bool wg_sync_and(int id, bool v)
     return r != 0;
 }
 
-__device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity)
+__device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity, uint32_t polls)
 {
-    for (uint32_t it = 0; it < kIacWaitPolls; ++it) {
+    for (uint32_t it = 0; it < polls; ++it) {
         uint32_t done;
         asm volatile(
             "{\n\t.reg .pred p;\n\t"
@@ -275,10 +276,42 @@ __device__ __forceinline__ void fetch_pair(PairRows &r, int64_t p, int64_t n_pai
     }
 }
 
+// Issues the MMAs of one operand slice (three split products per k-step, ks_n k-steps): A from the
+// warpgroup's buffer (hi, lo) with row-group stride a_sbo, B from the staged weights at b_hi / b_lo
+// (k-step b_ks0 onwards, row-group stride b_sbo). acc0: the first product accumulates into D.
+__device__ __forceinline__ void issue_split_mmas(uint32_t d, uint32_t a_hi, uint32_t a_lo, uint32_t a_sbo,
+                                                 uint32_t b_hi, uint32_t b_lo, uint32_t b_sbo, int b_ks0, int ks_n,
+                                                 bool acc0)
+{
+    for (int ks = 0; ks < ks_n; ++ks) {
+        const uint64_t ah = smem_desc(a_hi + ks * 256, 128, a_sbo);
+        const uint64_t al = smem_desc(a_lo + ks * 256, 128, a_sbo);
+        const uint64_t bh = smem_desc(b_hi + (b_ks0 + ks) * 256, 128, b_sbo);
+        const uint64_t bl = smem_desc(b_lo + (b_ks0 + ks) * 256, 128, b_sbo);
+        mma_tf32(d, ah, bh, (acc0 || ks > 0) ? 1u : 0u);
+        mma_tf32(d, ah, bl, 1u);
+        mma_tf32(d, al, bh, 1u);
+    }
+}
+
+// Hands the warpgroup's operand buffer and tensor memory to the MMAs: the generic-proxy stores are
+// made visible to the async proxy and the warpgroup meets at its named barrier.
+__device__ __forceinline__ void to_mma(int bar_id)
+{
+    fence_async_smem();
+    tc_fence_before();
+    asm volatile("bar.sync %0, 128;" ::"r"(bar_id) : "memory");
+    tc_fence_after();
+}
+
+// wait_polls: bounded waits poll this many times (a suspend of up to 1 ms each); hold != 0 (a
+// failure-detection hook): the first MMA group of CTA 0's first warpgroup is never committed, so that
+// warpgroup's wait runs out.
 __global__ void __launch_bounds__(iac_tc::kThreads, 1) k_iac_tc(const __grid_constant__ IacEpilogue ep,
                                                                  const uint4 *bimg, const float *jf, int32_t n_rows,
                                                                  const int2 *pairs, int64_t n_pairs, float c_mem,
-                                                                 float *out, unsigned int *err)
+                                                                 float *out, unsigned int *err, uint32_t wait_polls,
+                                                                 int32_t hold)
 {
     using namespace iac_tc;
     extern __shared__ unsigned char smem_raw[];
@@ -309,12 +342,19 @@ __global__ void __launch_bounds__(iac_tc::kThreads, 1) k_iac_tc(const __grid_con
     const uint32_t tmem = *slot;
     const uint32_t d1 = tmem + (uint32_t)(wg * 128), d2 = d1 + kN;
     const uint32_t lane_sel = (uint32_t)(32 * (warp & 3)) << 16;   // this warp's quarter of the lanes
-    unsigned char *a_hi = sm + kOffA + wg * 2 * kABytes, *a_lo = a_hi + kABytes;
+    unsigned char *a_hi = sm + kOffA + wg * kABufBytes, *a_lo = a_hi + kA1Bytes;
     const uint32_t a_hi_s = smem_addr(a_hi), a_lo_s = smem_addr(a_lo), sm_s = smem_addr(sm);
     const uint32_t bar = smem_addr(bars + wg);
     const int bar_id = 1 + wg;
     uint32_t phase = 0;
     bool ok = true;
+    bool held = hold != 0 && blockIdx.x == 0 && wg == 0;
+    // one MMA group: issue, commit (unless held), then the warpgroup-wide bounded wait
+    auto wait_group = [&]() {
+        ok = wg_sync_and(bar_id, mbar_wait_bounded(bar, phase, wait_polls));
+        phase ^= 1u;
+        return ok;
+    };
 
     const int64_t tile_stride = (int64_t)gridDim.x * kWG;
     PairRows cur;
@@ -322,124 +362,129 @@ __global__ void __launch_bounds__(iac_tc::kThreads, 1) k_iac_tc(const __grid_con
     for (int64_t tile = (int64_t)blockIdx.x * kWG + wg; tile * kM < n_pairs; tile += tile_stride) {
         const int64_t p = tile * kM + row;
         // ---- the pair's 36 inputs (Sec. 3.3.1), zero for a pair past the end or out of range
-        float x[kK1];
-#pragma unroll
-        for (int q = 0; q < kFeat / 2; ++q) {
-            x[2 * q] = cur.a[q].x;
-            x[2 * q + 1] = cur.a[q].y;
-            x[kFeat + 2 * q] = cur.b[q].x;
-            x[kFeat + 2 * q + 1] = cur.b[q].y;
-        }
-#pragma unroll
-        for (int i = 2 * kFeat; i < kK1; ++i)
-            x[i] = 0.0f;
         const bool valid = cur.valid;
-        if (valid) {
-            const float *a = x, *b = x + kFeat;
-            x[28] = __fmul_rn(__fadd_rn(a[0], b[0]), 0.5f);
-            x[29] = __fmul_rn(__fadd_rn(a[1], b[1]), 0.5f);
-            x[30] = __fmul_rn(__fadd_rn(a[2], b[2]), 0.5f);
-            x[31] = __fmul_rn(__fadd_rn(a[4], b[4]), 0.5f);
-            x[32] = __fadd_rn(a[5], b[5]);
-            x[33] = __fdiv_rn(__fadd_rn(a[3], b[3]), c_mem);
-            const float lo = fminf(a[0], b[0]), hi = fmaxf(a[0], b[0]);
-            x[34] = hi == 0.0f ? 1.0f : __fdiv_rn(lo, hi);
-            x[35] = fabsf(__fsub_rn(intensity(a[0], a[2]), intensity(b[0], b[2])));
-        }
+        {
+            float x[kK1];
 #pragma unroll
-        for (int c = 0; c < kK1 / 4; ++c)
-            store_split4(a_hi, a_lo, cm_off(row, 4 * c, kK1), x[4 * c], x[4 * c + 1], x[4 * c + 2], x[4 * c + 3]);
-        fence_async_smem();
-        tc_fence_before();
-        asm volatile("bar.sync %0, 128;" ::"r"(bar_id) : "memory");
-        tc_fence_after();
-
-        // ---- layer 1: D1 = X W1'^T, three split products per k-step
-        if (row == 0) {
-#pragma unroll
-            for (int ks = 0; ks < kK1 / 8; ++ks) {
-                const uint64_t ah = smem_desc(a_hi_s + ks * 256, 128, kK1 / 4 * 128);
-                const uint64_t al = smem_desc(a_lo_s + ks * 256, 128, kK1 / 4 * 128);
-                const uint64_t bh = smem_desc(sm_s + kOffB1Hi + ks * 256, 128, kK1 / 4 * 128);
-                const uint64_t bl = smem_desc(sm_s + kOffB1Lo + ks * 256, 128, kK1 / 4 * 128);
-                mma_tf32(d1, ah, bh, ks > 0 ? 1u : 0u);
-                mma_tf32(d1, ah, bl, 1u);
-                mma_tf32(d1, al, bh, 1u);
+            for (int q = 0; q < kFeat / 2; ++q) {
+                x[2 * q] = cur.a[q].x;
+                x[2 * q + 1] = cur.a[q].y;
+                x[kFeat + 2 * q] = cur.b[q].x;
+                x[kFeat + 2 * q + 1] = cur.b[q].y;
             }
-            mma_commit(bar);
+#pragma unroll
+            for (int i = 2 * kFeat; i < kK1; ++i)
+                x[i] = 0.0f;
+            if (valid) {
+                const float *a = x, *b = x + kFeat;
+                x[28] = __fmul_rn(__fadd_rn(a[0], b[0]), 0.5f);
+                x[29] = __fmul_rn(__fadd_rn(a[1], b[1]), 0.5f);
+                x[30] = __fmul_rn(__fadd_rn(a[2], b[2]), 0.5f);
+                x[31] = __fmul_rn(__fadd_rn(a[4], b[4]), 0.5f);
+                x[32] = __fadd_rn(a[5], b[5]);
+                x[33] = __fdiv_rn(__fadd_rn(a[3], b[3]), c_mem);
+                const float lo = fminf(a[0], b[0]), hi = fmaxf(a[0], b[0]);
+                x[34] = hi == 0.0f ? 1.0f : __fdiv_rn(lo, hi);
+                x[35] = fabsf(__fsub_rn(intensity(a[0], a[2]), intensity(b[0], b[2])));
+            }
+#pragma unroll
+            for (int c = 0; c < kK1 / 4; ++c)
+                store_split4(a_hi, a_lo, cm_off(row, 4 * c, kK1), x[4 * c], x[4 * c + 1], x[4 * c + 2],
+                             x[4 * c + 3]);
         }
+        to_mma(bar_id);
+
+        // ---- layer 1: D1 = X W1'^T
+        if (row == 0) {
+            issue_split_mmas(d1, a_hi_s, a_lo_s, kK1 / 4 * 128, sm_s + kOffB1Hi, sm_s + kOffB1Lo, kK1 / 4 * 128, 0,
+                             kK1 / 8, false);
+            if (!held)
+                mma_commit(bar);
+        }
+        held = false;
         __syncwarp();
         // the next tile's pair and rows: their latency overlaps this tile's MMAs and epilogues
         PairRows nxt;
         fetch_pair(nxt, p + tile_stride * kM, n_pairs, pairs, jf, n_rows);
-        ok = wg_sync_and(bar_id, mbar_wait_bounded(bar, phase));
-        phase ^= 1u;
-        if (!ok)
+        if (!wait_group())
             break;
         tc_fence_after();
 
-        // ---- epilogue 1: h1 = ReLU(D1 + b1'), split into operand A of layer 2
+        // ---- epilogue 1, first half: h1[0..31] = ReLU(D1 + b1'), split into the operand buffer
         {
-            float v[64];   // both halves requested before one wait, so their latencies overlap
+            float v[32];
             tmem_ld32(d1 | lane_sel, v);
-            tmem_ld32((d1 + 32) | lane_sel, v + 32);
             tmem_wait_ld();
 #pragma unroll
-            for (int c = 0; c < 16; ++c) {
+            for (int c = 0; c < kKH / 4; ++c) {
                 const int o = 4 * c;
-                store_split4(a_hi, a_lo, cm_off(row, o, kK2), fmaxf(__fadd_rn(v[o], ep.b1[o]), 0.0f),
+                store_split4(a_hi, a_lo, cm_off(row, o, kKH), fmaxf(__fadd_rn(v[o], ep.b1[o]), 0.0f),
                              fmaxf(__fadd_rn(v[o + 1], ep.b1[o + 1]), 0.0f),
                              fmaxf(__fadd_rn(v[o + 2], ep.b1[o + 2]), 0.0f),
                              fmaxf(__fadd_rn(v[o + 3], ep.b1[o + 3]), 0.0f));
             }
         }
-        fence_async_smem();
-        tc_fence_before();
-        asm volatile("bar.sync %0, 128;" ::"r"(bar_id) : "memory");
-        tc_fence_after();
-
-        // ---- layer 2: D2 = H1 W2'^T
+        to_mma(bar_id);
+        // ---- layer 2, first half: D2 = H1[:, 0..31] W2'[:, 0..31]^T
         if (row == 0) {
-#pragma unroll
-            for (int ks = 0; ks < kK2 / 8; ++ks) {
-                const uint64_t ah = smem_desc(a_hi_s + ks * 256, 128, kK2 / 4 * 128);
-                const uint64_t al = smem_desc(a_lo_s + ks * 256, 128, kK2 / 4 * 128);
-                const uint64_t bh = smem_desc(sm_s + kOffB2Hi + ks * 256, 128, kK2 / 4 * 128);
-                const uint64_t bl = smem_desc(sm_s + kOffB2Lo + ks * 256, 128, kK2 / 4 * 128);
-                mma_tf32(d2, ah, bh, ks > 0 ? 1u : 0u);
-                mma_tf32(d2, ah, bl, 1u);
-                mma_tf32(d2, al, bh, 1u);
-            }
+            issue_split_mmas(d2, a_hi_s, a_lo_s, kKH / 4 * 128, sm_s + kOffB2Hi, sm_s + kOffB2Lo, kK2 / 4 * 128, 0,
+                             kKH / 8, false);
             mma_commit(bar);
         }
         __syncwarp();
-        ok = wg_sync_and(bar_id, mbar_wait_bounded(bar, phase));
-        phase ^= 1u;
-        if (!ok)
+        // ---- epilogue 1, second half, while those MMAs run (D1's other columns)
+        float h[32];
+        {
+            float v[32];
+            tmem_ld32((d1 + kKH) | lane_sel, v);
+            tmem_wait_ld();
+#pragma unroll
+            for (int i = 0; i < 32; ++i)
+                h[i] = fmaxf(__fadd_rn(v[i], ep.b1[kKH + i]), 0.0f);
+        }
+        if (!wait_group())   // the first half's MMAs have read the buffer
+            break;
+        tc_fence_after();
+#pragma unroll
+        for (int c = 0; c < kKH / 4; ++c)
+            store_split4(a_hi, a_lo, cm_off(row, 4 * c, kKH), h[4 * c], h[4 * c + 1], h[4 * c + 2], h[4 * c + 3]);
+        to_mma(bar_id);
+        // ---- layer 2, second half: D2 += H1[:, 32..63] W2'[:, 32..63]^T
+        if (row == 0) {
+            issue_split_mmas(d2, a_hi_s, a_lo_s, kKH / 4 * 128, sm_s + kOffB2Hi, sm_s + kOffB2Lo, kK2 / 4 * 128,
+                             kKH / 8, kKH / 8, true);
+            mma_commit(bar);
+        }
+        __syncwarp();
+        if (!wait_group())
             break;
         tc_fence_after();
 
         // ---- epilogue 2: S_hat = 1 + ReLU(b3 + sum_o w3_o ReLU(D2_o + b2'_o)), o in order
         float y = ep.b3;
-        {
-            float v[64];
-            tmem_ld32(d2 | lane_sel, v);
-            tmem_ld32((d2 + 32) | lane_sel, v + 32);
+#pragma unroll
+        for (int half = 0; half < 2; ++half) {
+            float v[32];
+            tmem_ld32((d2 + 32 * half) | lane_sel, v);
             tmem_wait_ld();
 #pragma unroll
-            for (int o = 0; o < kN; ++o)
-                y = __fmaf_rn(ep.w3[o], fmaxf(__fadd_rn(v[o], ep.b2[o]), 0.0f), y);
+            for (int o = 0; o < 32; ++o)
+                y = __fmaf_rn(ep.w3[32 * half + o], fmaxf(__fadd_rn(v[o], ep.b2[32 * half + o]), 0.0f), y);
         }
         if (p < n_pairs)
             out[p] = valid ? __fadd_rn(1.0f, fmaxf(y, 0.0f)) : __int_as_float(0x7fffffff);
-        // the next tile rewrites operand A (its MMAs have completed) and D1/D2 (read above: the
-        // tcgen05.fence before the next warpgroup barrier orders those reads before the next MMAs)
+        // the next tile rewrites the operand buffer (every MMA reading it has completed) and D1/D2 (read
+        // above: the tcgen05 fence before the next named barrier orders those reads before the next MMAs)
         cur = nxt;
     }
     if (!ok) {
-        // an MMA group did not complete in time: give it one more bounded wait before the tensor
-        // memory is released, and report the timeout
-        mbar_wait_bounded(bar, phase ^ 1u);
+        // an MMA group did not complete in time: the mbarrier is made to track every MMA of this
+        // warpgroup still in flight, whose completion is awaited (bounded) before the tensor memory
+        // is released; the timeout is reported
+        if (row == 0)
+            mma_commit(bar);
+        phase ^= 1u;   // the phase the failed wait was for
+        mbar_wait_bounded(bar, phase, wait_polls);
         if (row == 0)
             atomicOr(err, kIacErrTimeout);
     }
@@ -495,6 +540,10 @@ struct esp_iac {
     std::vector<uint32_t> h_bimg;         // tensor path: split W1', W2' (host copy of the upload)
     uint4 *d_bimg = nullptr;
     unsigned int *d_err = nullptr;        // device error word (timeouts of the tensor path)
+    // failure-detection hooks (esp_debug.h): polls of a bounded wait (about 1 ms each), and the next
+    // tensor-path launch leaving one MMA group uncommitted
+    uint32_t wait_polls = kIacWaitPolls;
+    bool hold_commit = false;
     // buffers of esp_iac_predict_host
     float *d_rows = nullptr, *d_out = nullptr;
     int2 *d_pairs = nullptr;
@@ -532,8 +581,11 @@ cudaError_t launch_iac_tc(esp_iac *m, int32_t n_rows, const float *rows, int64_t
 {
     const int64_t tiles = (n_pairs + iac_tc::kM - 1) / iac_tc::kM;
     const int grid = (int)std::min<int64_t>((tiles + iac_tc::kWG - 1) / iac_tc::kWG, m->sm_count);
+    const int32_t hold = m->hold_commit ? 1 : 0;
+    m->hold_commit = false;   // the hook holds one launch only
     k_iac_tc<<<grid, iac_tc::kThreads, iac_tc::kSmemBytes, m->stream>>>(m->ep, m->d_bimg, rows, n_rows, pairs,
-                                                                       n_pairs, c_mem, out, m->d_err);
+                                                                       n_pairs, c_mem, out, m->d_err, m->wait_polls,
+                                                                       hold);
     return cudaGetLastError();
 }
 
@@ -700,6 +752,26 @@ esp_status esp_iac_synchronize(esp_iac *m)
         m->poisoned = true;
         return ESP_ERR_TIMEOUT;
     }
+    return ESP_OK;
+}
+
+esp_status esp_iac_debug_set_wait_limit(esp_iac *m, uint32_t limit_ms)
+{
+    const esp_status st = check_handle(m);
+    if (st != ESP_OK)
+        return st;
+    m->wait_polls = limit_ms == 0 ? kIacWaitPolls : limit_ms;
+    return ESP_OK;
+}
+
+esp_status esp_iac_debug_hold_commit(esp_iac *m)
+{
+    const esp_status st = check_handle(m);
+    if (st != ESP_OK)
+        return st;
+    if (m->path != ESP_IAC_PATH_TENSOR)
+        return ESP_ERR_UNSUPPORTED;
+    m->hold_commit = true;
     return ESP_OK;
 }
 

@@ -4,20 +4,24 @@
 //
 // Tile: 128 pairs (one per TMEM lane and per thread of a warpgroup) x 64 hidden units. Layer 1 is
 // D1[128 x 64] = X[128 x 40] * W1'^T (36 inputs padded to 40 = 5 MMA k-steps of 8), layer 2 is
-// D2 = H1[128 x 64] * W2'^T (8 k-steps); the output layer (64 terms) and the biases run in the
-// epilogue on the CUDA cores. Split: every operand a = a_hi + a_lo with a_hi = a truncated to tf32
-// (exact) and a_lo = tf32(a - a_hi) (round to nearest, ties away), and each k-step issues
-// a_hi*b_hi + a_hi*b_lo + a_lo*b_hi into the same fp32 accumulator; per product the dropped term
-// and the roundings of the low parts are below 2^-19 |a b|.
+// D2 = H1[128 x 64] * W2'^T (8 k-steps) issued in two halves of 32 columns of H1; the output layer
+// (64 terms) and the biases run in the epilogue on the CUDA cores. Split: every operand
+// a = a_hi + a_lo with a_hi = a truncated to tf32 (exact) and a_lo = tf32(a - a_hi) (round to
+// nearest, ties away), and each k-step issues a_hi*b_hi + a_hi*b_lo + a_lo*b_hi into the same fp32
+// accumulator; per product the dropped term and the roundings of the low parts are below 2^-19 |a b|.
 //
-// CTA: two warpgroups, each running its own sequence of tiles (one warpgroup's epilogue overlaps the
-// other's MMAs), the split weights W1', W2' staged once per CTA (53,248 bytes), 64 KB of operand A
-// per warpgroup, 256 TMEM columns (D1, D2 of each warpgroup). Operands use the canonical
+// CTA: four warpgroups, each running its own sequence of tiles, so that four tiles' dependency
+// chains (features, MMA 1, epilogue 1 in two halves each followed by its MMAs, epilogue 2) overlap
+// on one SM; the split weights W1', W2' are staged once per CTA (53,248 bytes). A warpgroup's operand
+// A buffer (40 KB) holds X (hi and lo, 2 x 20 KB), then each half of H1 in turn (2 x 16 KB): the
+// second half is written once the first half's MMAs have completed, while the first half's epilogue
+// already overlaps them; 128 TMEM columns per warpgroup (D1, D2). Operands use the canonical
 // no-swizzle K-major layout: 8-row x 16-byte core matrices of 128 contiguous bytes, consecutive
 // along K (leading offset 128 B), row groups of 8 at a stride of K/4 * 128 B. One elected thread
 // per warpgroup issues the MMAs and commits them to the warpgroup's mbarrier; every wait is bounded
 // and a timeout ends the warpgroup's loop (the decision is made warpgroup-wide by a reducing
-// barrier), flags the error word, and the CTA still frees its tensor memory.
+// barrier), flags the error word, makes the mbarrier track every MMA still in flight and waits for
+// them (bounded) before the CTA frees its tensor memory.
 #pragma once
 
 #include <cstdint>
@@ -28,19 +32,24 @@ constexpr int kM = 128;          // pairs per tile
 constexpr int kN = 64;           // hidden units (narrower models are zero-padded)
 constexpr int kK1 = 40;          // 36 inputs padded to a multiple of the tf32 MMA K (8)
 constexpr int kK2 = 64;
-constexpr int kWG = 2;           // warpgroups per CTA
+constexpr int kKH = 32;          // layer 2 in two halves of 32 columns of H1
+constexpr int kWG = 4;           // warpgroups per CTA
 constexpr int kThreads = 128 * kWG;
-constexpr int kTmemCols = 256;   // D1 and D2 (64 fp32 columns each) per warpgroup
+constexpr int kTmemCols = 512;   // D1 and D2 (64 fp32 columns each) per warpgroup
 
 constexpr int kB1Bytes = kN * kK1 * 4;                      // 10,240
 constexpr int kB2Bytes = kN * kK2 * 4;                      // 16,384
 constexpr int kBImgBytes = 2 * kB1Bytes + 2 * kB2Bytes;     // hi, lo of W1' then of W2'
-constexpr int kABytes = kM * kK2 * 4;                       // 32,768 per part (hi or lo)
+constexpr int kA1Bytes = kM * kK1 * 4;                      // 20,480: one part (hi or lo) of X
+constexpr int kAHBytes = kM * kKH * 4;                      // 16,384: one part of a half of H1
+constexpr int kABufBytes = 2 * kA1Bytes;                    // a warpgroup's buffer: hi at 0, lo at kA1Bytes
 constexpr int kOffB1Hi = 0, kOffB1Lo = kB1Bytes, kOffB2Hi = 2 * kB1Bytes, kOffB2Lo = 2 * kB1Bytes + kB2Bytes;
-constexpr int kOffA = kBImgBytes;                           // warpgroup g: hi at kOffA + 2g kABytes, lo after it
-constexpr int kOffBar = kOffA + kWG * 2 * kABytes;
+constexpr int kOffA = kBImgBytes;                           // warpgroup g's buffer at kOffA + g kABufBytes
+constexpr int kOffBar = kOffA + kWG * kABufBytes;
 constexpr int kOffSlot = kOffBar + 8 * kWG;
 constexpr int kSmemBytes = kOffSlot + 16 + 1024;            // + alignment slack of the dynamic base
+static_assert(kAHBytes <= kA1Bytes, "a half of H1 fits where X was");
+static_assert(kSmemBytes <= 232448, "shared memory of one CTA");
 
 // Byte offset of element (row, col) in the canonical no-swizzle K-major layout of a K-wide operand.
 __host__ __device__ constexpr int cm_off(int row, int col, int K)

@@ -37,6 +37,7 @@ EXPORTED = [
     "esp_set_penalties", "esp_adaptive_threshold", "esp_effective_capacity", "esp_load_placement",
     "esp_iac_create", "esp_iac_set_stream", "esp_iac_load_model", "esp_iac_predict", "esp_iac_predict_host",
     "esp_iac_last_launch_count", "esp_iac_destroy", "esp_iac_set_path", "esp_iac_synchronize",
+    "esp_iac_debug_set_wait_limit", "esp_iac_debug_hold_commit",
 ]
 
 
@@ -129,6 +130,8 @@ def load_library(path: Optional[str] = None):
         "esp_iac_destroy": ([vp], None),
         "esp_iac_set_path": ([vp, i32], st),
         "esp_iac_synchronize": ([vp], st),
+        "esp_iac_debug_set_wait_limit": ([vp, u32], st),
+        "esp_iac_debug_hold_commit": ([vp], st),
     }
     for name, (args, res) in sig.items():
         fn = getattr(lib, name)
@@ -583,6 +586,16 @@ def esp_iac_set_path(h: int, path: int) -> None:
 
 def esp_iac_synchronize(h: int) -> None:
     _check(load_library().esp_iac_synchronize(h), "esp_iac_synchronize")
+
+
+def esp_iac_debug_set_wait_limit(h: int, limit_ms: int) -> None:
+    """Test hook: bound of each wait of the tensor-core kernel for an MMA group (0: the default)."""
+    _check(load_library().esp_iac_debug_set_wait_limit(h, int(limit_ms)), "esp_iac_debug_set_wait_limit")
+
+
+def esp_iac_debug_hold_commit(h: int) -> None:
+    """Test hook: the next tensor-path launch leaves one MMA group uncommitted (its wait runs out)."""
+    _check(load_library().esp_iac_debug_hold_commit(h), "esp_iac_debug_hold_commit")
 
 
 def esp_iac_last_launch_count(h: int) -> int:

@@ -85,3 +85,35 @@ def test_allocation_failure_is_reported_and_recoverable():
     sol = s.solve(0.05, 15)
     assert np.array_equal(sol.lam, ref.lam) and np.array_equal(sol.sel, ref.sel)
     s.close()
+
+
+def test_iac_mma_wait_timeout_reports_and_poisons():
+    """The tensor-core IAC kernel's bounded MMA wait: one MMA group left uncommitted (no access out of
+    place) makes its warpgroup's wait run out after the host-set limit; the call answers
+    ESP_ERR_TIMEOUT, the handle ESP_ERR_STATE from then on, and a new handle predicts exactly as
+    before."""
+    w = W.iac_batch(S=4)
+    rows, pairs = w.rows, w.pairs
+    pred = esp.Predictor(w.model)
+    ref = pred.predict(rows, pairs, w.c_mem)
+    esp.esp_iac_debug_set_wait_limit(pred.h, 20)
+    esp.esp_iac_debug_hold_commit(pred.h)
+    t0 = time.perf_counter()
+    with pytest.raises(esp.EspError) as e:
+        pred.predict(rows, pairs, w.c_mem)
+    dt = time.perf_counter() - t0
+    assert e.value.status == esp.ESP_ERR_TIMEOUT
+    assert dt < 10.0, f"the timeout took {dt:.1f} s"
+    with pytest.raises(esp.EspError) as e2:
+        pred.predict(rows, pairs, w.c_mem)
+    assert e2.value.status == esp.ESP_ERR_STATE
+    pred.close()
+    fresh = esp.Predictor(w.model)
+    again = fresh.predict(rows, pairs, w.c_mem)
+    fresh.close()
+    assert np.array_equal(again, ref)
+    fma = esp.Predictor(w.model, path=esp.ESP_IAC_PATH_FMA)
+    with pytest.raises(esp.EspError) as e3:
+        esp.esp_iac_debug_hold_commit(fma.h)
+    assert e3.value.status == esp.ESP_ERR_UNSUPPORTED
+    fma.close()
