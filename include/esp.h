@@ -93,6 +93,9 @@ typedef struct {
     int64_t *demand_trace;  /* S*T*P: U^t, the demand of round t's selection */
     uint64_t *selhash_trace;/* S*T: sum over jobs j of splitmix64_mix((j << 32) | c_j) of round t */
     double *dual_trace;     /* S*(T+1): g(lambda^t) of Eq. lagrangian; entry rounds_run is the final one */
+    uint64_t *round_time_trace; /* S*T: the GPU's global timer (ns) when round t's price update of the
+                               scenario was applied (on every solve path); differences of consecutive
+                               entries are the scenario's round times */
 } esp_params;
 
 typedef struct {

@@ -23,7 +23,7 @@ struct GraphKey {
     double eta0 = 0, tol = 0;
     int32_t step = -1, mode = -1, T = -1;
     uint32_t flags = 0;
-    const void *lt = nullptr, *dt = nullptr, *ht = nullptr, *gt = nullptr;
+    const void *lt = nullptr, *dt = nullptr, *ht = nullptr, *gt = nullptr, *tt = nullptr;
     bool has_l0 = false;
     int res = -1;   // resident option in use, -1: streaming
     bool hold = false;
@@ -34,7 +34,8 @@ struct GraphKey {
     {
         return eta0 == o.eta0 && tol == o.tol && step == o.step && mode == o.mode && T == o.T && flags == o.flags &&
                persist == o.persist && args == o.args &&
-               lt == o.lt && dt == o.dt && ht == o.ht && gt == o.gt && has_l0 == o.has_l0 && res == o.res &&
+               lt == o.lt && dt == o.dt && ht == o.ht && gt == o.gt && tt == o.tt && has_l0 == o.has_l0 &&
+               res == o.res &&
                hold == o.hold && hold_tx == o.hold_tx && wait_ms == o.wait_ms;
     }
 };
@@ -165,6 +166,7 @@ struct esp_ctx {
     DevArr<long long> dt;
     DevArr<unsigned long long> ht;
     DevArr<double> gt;
+    DevArr<unsigned long long> tt;
 
     cudaGraphExec_t gexec = nullptr;
     GraphKey gkey;
@@ -404,6 +406,7 @@ DevState dev_state(const esp_ctx *c)
     s.dem_trace = nullptr;
     s.hash_trace = nullptr;
     s.dual_trace = nullptr;
+    s.time_trace = nullptr;
     return s;
 }
 
@@ -1184,6 +1187,7 @@ esp_status enqueue_solve(esp_ctx *ctx, const esp_params *p, const DevState &st, 
     key.T = T;
     key.flags = p->flags;
     key.lt = st.lam_trace;
+    key.tt = st.time_trace;
     key.dt = st.dem_trace;
     key.ht = st.hash_trace;
     key.gt = st.dual_trace;
@@ -1423,7 +1427,8 @@ esp_status esp_solve_async(esp_ctx *ctx, const esp_params *params)
         return ESP_ERR_NOT_LOADED;
     if ((st = check_params(ctx, params)) != ESP_OK)
         return st;
-    if (params->lambda_trace || params->demand_trace || params->selhash_trace || params->dual_trace)
+    if (params->lambda_trace || params->demand_trace || params->selhash_trace || params->dual_trace ||
+        params->round_time_trace)
         return ESP_ERR_INVALID_ARG;
     ESP_CUDA(cudaSetDevice(ctx->device));
     const size_t SP = (size_t)ctx->S * ctx->P;
@@ -1479,6 +1484,13 @@ esp_status esp_solve(esp_ctx *ctx, const esp_params *params, esp_result *out)
         ESP_CUDA(cudaMemcpyAsync(ctx->gt.p, params->dual_trace, S * (T + 1) * 8, cudaMemcpyHostToDevice, ctx->stream));
         ds.dual_trace = ctx->gt.p;
     }
+    if (params->round_time_trace && T > 0) {
+        if ((st = grow(ctx, ctx->tt, S * T)) != ESP_OK)
+            return st;
+        ESP_CUDA(cudaMemcpyAsync(ctx->tt.p, params->round_time_trace, S * T * 8, cudaMemcpyHostToDevice,
+                                 ctx->stream));
+        ds.time_trace = ctx->tt.p;
+    }
     if ((st = enqueue_solve(ctx, params, ds, params->lambda0 != nullptr)) != ESP_OK)
         return st;
     ctx->solved = true;
@@ -1493,6 +1505,9 @@ esp_status esp_solve(esp_ctx *ctx, const esp_params *params, esp_result *out)
         ESP_CUDA(cudaMemcpyAsync(params->selhash_trace, ctx->ht.p, S * T * 8, cudaMemcpyDeviceToHost, ctx->stream));
     if (params->dual_trace)
         ESP_CUDA(cudaMemcpyAsync(params->dual_trace, ctx->gt.p, S * (T + 1) * 8, cudaMemcpyDeviceToHost, ctx->stream));
+    if (ds.time_trace)
+        ESP_CUDA(cudaMemcpyAsync(params->round_time_trace, ctx->tt.p, S * T * 8, cudaMemcpyDeviceToHost,
+                                 ctx->stream));
     if (out)
         return read_results(ctx, out);
     ESP_CUDA(cudaStreamSynchronize(ctx->stream));
@@ -1937,6 +1952,7 @@ void esp_destroy(esp_ctx *ctx)
     if (ctx->dt.p) cudaFree(ctx->dt.p);
     if (ctx->ht.p) cudaFree(ctx->ht.p);
     if (ctx->gt.p) cudaFree(ctx->gt.p);
+    if (ctx->tt.p) cudaFree(ctx->tt.p);
     for (cudaEvent_t e : ctx->ev_pool)
         cudaEventDestroy(e);
     for (cudaEvent_t e : ctx->graph_pool)

@@ -56,6 +56,7 @@ struct DevState {
     long long *dem_trace;     // S*T*P or nullptr
     unsigned long long *hash_trace; // S*T or nullptr
     double *dual_trace;       // S*(T+1) or nullptr
+    unsigned long long *time_trace; // S*T or nullptr: global timer when each round's update was applied
 };
 
 struct DevPlan {

@@ -642,6 +642,8 @@ __global__ void __launch_bounds__(kPlaceResWarps * 32, 1) k_place_res(DevTable t
             }
             const double M = st.vmax[sc] + warp_sum_fixed(term);
             if (lane == 0) {
+                if (lead && st.time_trace)
+                    st.time_trace[(size_t)sc * T + round] = global_ns();
                 rounds_s[sc] = round + 1;
                 if (conv) {
                     conv_s[sc] = 1;

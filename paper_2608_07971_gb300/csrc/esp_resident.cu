@@ -28,6 +28,7 @@
 
 #include "esp_device.cuh"
 #include "esp_kernels.h"
+#include "esp_ptx.cuh"
 
 namespace esp {
 
@@ -568,6 +569,8 @@ __global__ void __launch_bounds__(kResThreads, ESP_RES_MIN_CTAS) k_resident(DevT
                 stop = true;
             } else {
                 rounds = round + 1;
+                if (st.time_trace && lead && lane == 0)
+                    st.time_trace[(size_t)s * T + round] = global_ns();
                 if (st.lam_trace && lead && c < R)
                     st.lam_trace[((size_t)s * (T + 1) + round + 1) * P + c] = nl;
                 stop = false;

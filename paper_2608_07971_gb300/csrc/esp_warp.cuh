@@ -11,6 +11,7 @@
 
 #include "esp_device.cuh"
 #include "esp_kernels.h"
+#include "esp_ptx.cuh"
 
 namespace esp {
 
@@ -292,6 +293,8 @@ __device__ void update_scenario(const DevTable &t, const DevState &st, const Sol
     }
     const bool conv = (a.tol > 0.0) && (dmax <= a.tol * fmax(1.0, amax));
     if (lane == 0) {
+        if (st.time_trace)
+            st.time_trace[(size_t)s * T + round] = global_ns();
         st.rounds_run[s] = round + 1;
         if (conv) {
             st.converged[s] = 1;

@@ -52,7 +52,7 @@ class esp_params(ctypes.Structure):
                 ("max_rounds", ctypes.c_int32), ("flags", ctypes.c_uint32), ("tol", ctypes.c_double),
                 ("lambda0", ctypes.c_void_p), ("lambda_trace", ctypes.c_void_p),
                 ("demand_trace", ctypes.c_void_p), ("selhash_trace", ctypes.c_void_p),
-                ("dual_trace", ctypes.c_void_p)]
+                ("dual_trace", ctypes.c_void_p), ("round_time_trace", ctypes.c_void_p)]
 
 
 class esp_result(ctypes.Structure):
@@ -320,6 +320,7 @@ class Solution:
     demand_trace: Optional[np.ndarray] = None   # S x T x P
     selhash_trace: Optional[np.ndarray] = None  # S x T
     dual_trace: Optional[np.ndarray] = None     # S x (T+1)
+    round_time_trace: Optional[np.ndarray] = None  # S x T, GPU global timer (ns) of each round's update
 
 
 class Solver:
@@ -375,11 +376,12 @@ class Solver:
         T = rounds
         l0 = None if lambda0 is None else np.ascontiguousarray(lambda0, np.float64).reshape(S, P)
         prm = self.params(eta0, rounds, mode, step, tol, flags, l0)
-        lt = dt = ht = gt = None
-        if traces:          # True: every trace; "prices": the price and demand trajectories only
+        lt = dt = ht = gt = tt = None
+        if traces:          # True: every trace; "prices": the price, demand and round-time trajectories
             lt = np.full((S, T + 1, P), np.nan)
             dt = np.zeros((S, T, P), np.int64)
-            prm.lambda_trace, prm.demand_trace = _p(lt), _p(dt)
+            tt = np.zeros((S, T), np.uint64)
+            prm.lambda_trace, prm.demand_trace, prm.round_time_trace = _p(lt), _p(dt), _p(tt)
             if traces is True:
                 ht = np.zeros((S, T), np.uint64)
                 gt = np.full((S, T + 1), np.nan)
@@ -392,7 +394,7 @@ class Solver:
         esp_get_prices(self.ctx, lam)
         esp_get_selection(self.ctx, sel)
         esp_get_demand(self.ctx, dem)
-        return Solution(lam, sel, dem, res, status, lt, dt, ht, gt)
+        return Solution(lam, sel, dem, res, status, lt, dt, ht, gt, tt)
 
     def evaluate(self, lam, mode=ESP_PRICE_NORMALIZED, flags=0):
         S, J, R, P = self.shape
