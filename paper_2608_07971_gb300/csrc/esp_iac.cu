@@ -122,9 +122,10 @@ void fill_params(IacParams<H> &dst, int hp, const std::vector<float> &w1, const 
 
 // ---- tensor-core path (esp_iac_tc.cuh)
 
+static_assert(kIn < iac_tc::kK1, "X has a padding column for layer 1's bias");
+
 struct IacEpilogue {
-    float b1[iac_tc::kN];   // folded layer-1 bias (zero beyond H)
-    float b2[iac_tc::kN];
+    float b2[iac_tc::kN];   // folded layer-2 bias (zero beyond H); layer 1's enters the MMAs
     float w3[iac_tc::kN];
     float b3;
 };
@@ -153,6 +154,17 @@ __device__ __forceinline__ void mma_tf32(uint32_t d_tmem, uint64_t a, uint64_t b
         "setp.ne.b32 p, %4, 0;\n\t"
         "tcgen05.mma.cta_group::1.kind::tf32 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
         "l"(a), "l"(b), "r"(iac_tc::kIdesc), "r"(accumulate)
+        : "memory");
+}
+
+// The same MMA with A in tensor memory (lane = row, one tf32 column per k), B from shared memory.
+__device__ __forceinline__ void mma_tf32_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b, uint32_t accumulate)
+{
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::tf32 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "r"(a_tmem), "l"(b), "r"(iac_tc::kIdesc), "r"(accumulate)
         : "memory");
 }
 
@@ -232,6 +244,35 @@ __device__ __forceinline__ void tmem_wait_ld()
     asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
+// 32 consecutive 32-bit columns of this thread's TMEM lane.
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t *r)
+{
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, "
+        "%15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32};" ::"r"(taddr),
+        "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]),
+        "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15]), "r"(r[16]),
+        "r"(r[17]), "r"(r[18]), "r"(r[19]), "r"(r[20]), "r"(r[21]), "r"(r[22]), "r"(r[23]), "r"(r[24]),
+        "r"(r[25]), "r"(r[26]), "r"(r[27]), "r"(r[28]), "r"(r[29]), "r"(r[30]), "r"(r[31])
+        : "memory");
+}
+
+__device__ __forceinline__ void tmem_wait_st()
+{
+    asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
+// 32 values split into tf32 high and low parts.
+__device__ __forceinline__ void split32(const float *h, uint32_t *hi, uint32_t *lo)
+{
+    using namespace iac_tc;
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+        hi[i] = tf32_trunc_bits(__float_as_uint(h[i]));
+        lo[i] = tf32_round_bits(__float_as_uint(__fsub_rn(h[i], __uint_as_float(hi[i]))));
+    }
+}
+
 // Four consecutive values of a row, split into tf32 high and low parts, stored as one 16-byte chunk
 // of each part.
 __device__ __forceinline__ void store_split4(unsigned char *hi, unsigned char *lo, int off, float a, float b, float c,
@@ -294,14 +335,19 @@ __device__ __forceinline__ void issue_split_mmas(uint32_t d, uint32_t a_hi, uint
     }
 }
 
-// Hands the warpgroup's operand buffer and tensor memory to the MMAs: the generic-proxy stores are
-// made visible to the async proxy and the warpgroup meets at its named barrier.
-__device__ __forceinline__ void to_mma(int bar_id)
+// Layer 2's MMAs for one half of H1 (ks_n k-steps): A from Q in tensor memory (hi at a_t, lo at
+// a_t + 32), B from the staged weights at b_hi / b_lo (k-step b_ks0 onwards, row-group stride b_sbo).
+__device__ __forceinline__ void issue_split_mmas_ts(uint32_t d, uint32_t a_t, uint32_t b_hi, uint32_t b_lo,
+                                                    uint32_t b_sbo, int b_ks0, int ks_n, bool acc0)
 {
-    fence_async_smem();
-    tc_fence_before();
-    asm volatile("bar.sync %0, 128;" ::"r"(bar_id) : "memory");
-    tc_fence_after();
+    for (int ks = 0; ks < ks_n; ++ks) {
+        const uint32_t ah = a_t + 8 * ks, al = a_t + iac_tc::kKH + 8 * ks;
+        const uint64_t bh = smem_desc(b_hi + (b_ks0 + ks) * 256, 128, b_sbo);
+        const uint64_t bl = smem_desc(b_lo + (b_ks0 + ks) * 256, 128, b_sbo);
+        mma_tf32_ts(d, ah, bh, (acc0 || ks > 0) ? 1u : 0u);
+        mma_tf32_ts(d, ah, bl, 1u);
+        mma_tf32_ts(d, al, bh, 1u);
+    }
 }
 
 // wait_polls: bounded waits poll this many times (a suspend of up to 1 ms each); hold != 0 (a
@@ -340,148 +386,178 @@ __global__ void __launch_bounds__(iac_tc::kThreads, 1) k_iac_tc(const __grid_con
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *slot;
-    const uint32_t d1 = tmem + (uint32_t)(wg * 128), d2 = d1 + kN;
     const uint32_t lane_sel = (uint32_t)(32 * (warp & 3)) << 16;   // this warp's quarter of the lanes
+    // the warpgroup's two regions of 64 columns: a tile's accumulators (D1, then D2) in one, its half
+    // of H1 in the other, the roles swapped from one tile to the next
+    const uint32_t t_base = tmem + (uint32_t)(wg * 2 * kN);
     unsigned char *a_hi = sm + kOffA + wg * kABufBytes, *a_lo = a_hi + kA1Bytes;
     const uint32_t a_hi_s = smem_addr(a_hi), a_lo_s = smem_addr(a_lo), sm_s = smem_addr(sm);
     const uint32_t bar = smem_addr(bars + wg);
     const int bar_id = 1 + wg;
+    // the thread that issues the warpgroup's MMAs: lane 0 of its warp wg, so that the four issuers
+    // sit in four different SM sub-partitions (warp w runs on sub-partition w mod 4)
+    const bool issuer = row == 32 * wg;
     uint32_t phase = 0;
     bool ok = true;
-    bool held = hold != 0 && blockIdx.x == 0 && wg == 0;
-    // one MMA group: issue, commit (unless held), then the warpgroup-wide bounded wait
+    // The MMA groups are committed to the warpgroup's mbarrier one at a time. Every thread waits for
+    // a group itself (bounded), agreed warp-wide so that the warp-collective tcgen05 loads and stores
+    // after it run in every lane or in none; the warpgroup-wide agreement is taken at the next
+    // hand-off barrier, which a timeout in any warp turns into a common exit.
     auto wait_group = [&]() {
-        ok = wg_sync_and(bar_id, mbar_wait_bounded(bar, phase, wait_polls));
+        const bool mine = mbar_wait_bounded(bar, phase, wait_polls);
         phase ^= 1u;
+        return __all_sync(0xffffffffu, mine);
+    };
+    // Hands the warpgroup's operand writes (X in shared memory, H1 in tensor memory) to the MMA issuer
+    // and ANDs the waits of every warp; false: some warp's wait ran out.
+    auto hand_off = [&](bool mine) {
+        fence_async_smem();
+        tc_fence_before();
+        ok = wg_sync_and(bar_id, mine);
+        tc_fence_after();
         return ok;
+    };
+    // a pair's 36 inputs (Sec. 3.3.1), zero for a pair past the end or out of range, split into X
+    auto store_inputs = [&](const PairRows &r) {
+        float x[kK1];
+#pragma unroll
+        for (int q = 0; q < kFeat / 2; ++q) {
+            x[2 * q] = r.a[q].x;
+            x[2 * q + 1] = r.a[q].y;
+            x[kFeat + 2 * q] = r.b[q].x;
+            x[kFeat + 2 * q + 1] = r.b[q].y;
+        }
+        x[kIn] = 1.0f;   // the column that carries layer 1's bias
+#pragma unroll
+        for (int i = kIn + 1; i < kK1; ++i)
+            x[i] = 0.0f;
+        if (r.valid) {
+            const float *a = x, *b = x + kFeat;
+            x[28] = __fmul_rn(__fadd_rn(a[0], b[0]), 0.5f);
+            x[29] = __fmul_rn(__fadd_rn(a[1], b[1]), 0.5f);
+            x[30] = __fmul_rn(__fadd_rn(a[2], b[2]), 0.5f);
+            x[31] = __fmul_rn(__fadd_rn(a[4], b[4]), 0.5f);
+            x[32] = __fadd_rn(a[5], b[5]);
+            x[33] = __fdiv_rn(__fadd_rn(a[3], b[3]), c_mem);
+            const float lo = fminf(a[0], b[0]), hi = fmaxf(a[0], b[0]);
+            x[34] = hi == 0.0f ? 1.0f : __fdiv_rn(lo, hi);
+            x[35] = fabsf(__fsub_rn(intensity(a[0], a[2]), intensity(b[0], b[2])));
+        }
+#pragma unroll
+        for (int c = 0; c < kK1 / 4; ++c)
+            store_split4(a_hi, a_lo, cm_off(row, 4 * c, kK1), x[4 * c], x[4 * c + 1], x[4 * c + 2], x[4 * c + 3]);
+    };
+    // layer 1 of a tile: D1 = X W1'^T into region d (hold: this group is not committed), after a
+    // hand-off of the tile's X
+    auto issue_layer1 = [&](uint32_t d, bool hold_group) {
+        if (issuer) {
+            issue_split_mmas(d, a_hi_s, a_lo_s, kK1 / 4 * 128, sm_s + kOffB1Hi, sm_s + kOffB1Lo, kK1 / 4 * 128, 0,
+                             kK1 / 8, false);
+            if (!hold_group)
+                mma_commit(bar);
+        }
+        __syncwarp();
     };
 
     const int64_t tile_stride = (int64_t)gridDim.x * kWG;
-    PairRows cur;
-    fetch_pair(cur, ((int64_t)blockIdx.x * kWG + wg) * kM + row, n_pairs, pairs, jf, n_rows);
-    for (int64_t tile = (int64_t)blockIdx.x * kWG + wg; tile * kM < n_pairs; tile += tile_stride) {
+    int64_t tile = (int64_t)blockIdx.x * kWG + wg;
+    uint32_t par = 0;   // region of the current tile's accumulators
+    bool valid = false;
+    if (tile * kM < n_pairs) {
+        PairRows first;
+        fetch_pair(first, tile * kM + row, n_pairs, pairs, jf, n_rows);
+        store_inputs(first);
+        valid = first.valid;
+        hand_off(true);
+        issue_layer1(t_base, hold != 0 && blockIdx.x == 0 && wg == 0);
+    }
+    for (; tile * kM < n_pairs; tile += tile_stride, par ^= 1u) {
         const int64_t p = tile * kM + row;
-        // ---- the pair's 36 inputs (Sec. 3.3.1), zero for a pair past the end or out of range
-        const bool valid = cur.valid;
-        {
-            float x[kK1];
-#pragma unroll
-            for (int q = 0; q < kFeat / 2; ++q) {
-                x[2 * q] = cur.a[q].x;
-                x[2 * q + 1] = cur.a[q].y;
-                x[kFeat + 2 * q] = cur.b[q].x;
-                x[kFeat + 2 * q + 1] = cur.b[q].y;
-            }
-#pragma unroll
-            for (int i = 2 * kFeat; i < kK1; ++i)
-                x[i] = 0.0f;
-            if (valid) {
-                const float *a = x, *b = x + kFeat;
-                x[28] = __fmul_rn(__fadd_rn(a[0], b[0]), 0.5f);
-                x[29] = __fmul_rn(__fadd_rn(a[1], b[1]), 0.5f);
-                x[30] = __fmul_rn(__fadd_rn(a[2], b[2]), 0.5f);
-                x[31] = __fmul_rn(__fadd_rn(a[4], b[4]), 0.5f);
-                x[32] = __fadd_rn(a[5], b[5]);
-                x[33] = __fdiv_rn(__fadd_rn(a[3], b[3]), c_mem);
-                const float lo = fminf(a[0], b[0]), hi = fmaxf(a[0], b[0]);
-                x[34] = hi == 0.0f ? 1.0f : __fdiv_rn(lo, hi);
-                x[35] = fabsf(__fsub_rn(intensity(a[0], a[2]), intensity(b[0], b[2])));
-            }
-#pragma unroll
-            for (int c = 0; c < kK1 / 4; ++c)
-                store_split4(a_hi, a_lo, cm_off(row, 4 * c, kK1), x[4 * c], x[4 * c + 1], x[4 * c + 2],
-                             x[4 * c + 3]);
-        }
-        to_mma(bar_id);
-
-        // ---- layer 1: D1 = X W1'^T
-        if (row == 0) {
-            issue_split_mmas(d1, a_hi_s, a_lo_s, kK1 / 4 * 128, sm_s + kOffB1Hi, sm_s + kOffB1Lo, kK1 / 4 * 128, 0,
-                             kK1 / 8, false);
-            if (!held)
-                mma_commit(bar);
-        }
-        held = false;
-        __syncwarp();
-        // the next tile's pair and rows: their latency overlaps this tile's MMAs and epilogues
-        PairRows nxt;
-        fetch_pair(nxt, p + tile_stride * kM, n_pairs, pairs, jf, n_rows);
-        if (!wait_group())
-            break;
-        tc_fence_after();
-
-        // ---- epilogue 1, first half: h1[0..31] = ReLU(D1 + b1'), split into the operand buffer
-        {
-            float v[32];
-            tmem_ld32(d1 | lane_sel, v);
-            tmem_wait_ld();
-#pragma unroll
-            for (int c = 0; c < kKH / 4; ++c) {
-                const int o = 4 * c;
-                store_split4(a_hi, a_lo, cm_off(row, o, kKH), fmaxf(__fadd_rn(v[o], ep.b1[o]), 0.0f),
-                             fmaxf(__fadd_rn(v[o + 1], ep.b1[o + 1]), 0.0f),
-                             fmaxf(__fadd_rn(v[o + 2], ep.b1[o + 2]), 0.0f),
-                             fmaxf(__fadd_rn(v[o + 3], ep.b1[o + 3]), 0.0f));
-            }
-        }
-        to_mma(bar_id);
-        // ---- layer 2, first half: D2 = H1[:, 0..31] W2'[:, 0..31]^T
-        if (row == 0) {
-            issue_split_mmas(d2, a_hi_s, a_lo_s, kKH / 4 * 128, sm_s + kOffB2Hi, sm_s + kOffB2Lo, kK2 / 4 * 128, 0,
-                             kKH / 8, false);
-            mma_commit(bar);
-        }
-        __syncwarp();
-        // ---- epilogue 1, second half, while those MMAs run (D1's other columns)
+        const uint32_t tD = t_base + par * kN, tH = t_base + (par ^ 1u) * kN;   // MMA view (lane 0)
+        const uint32_t tD_w = tD | lane_sel, tH_w = tH | lane_sel;             // this warp's lanes
+        const bool more = (tile + tile_stride) * kM < n_pairs;
+        // ---- epilogue 1: h1 = ReLU(D1) (D1 holds the bias); the first half split into H, the second kept in
+        // registers
+        bool mine = wait_group();   // layer 1
         float h[32];
-        {
-            float v[32];
-            tmem_ld32((d1 + kKH) | lane_sel, v);
+        if (mine) {
+            tc_fence_after();
+            float v[64];
+            tmem_ld32(tD_w, v);
+            tmem_ld32(tD_w + kKH, v + kKH);
             tmem_wait_ld();
+            uint32_t hi[32], lo[32];
 #pragma unroll
             for (int i = 0; i < 32; ++i)
-                h[i] = fmaxf(__fadd_rn(v[i], ep.b1[kKH + i]), 0.0f);
-        }
-        if (!wait_group())   // the first half's MMAs have read the buffer
-            break;
-        tc_fence_after();
+                h[i] = fmaxf(v[i], 0.0f);
+            split32(h, hi, lo);
+            tmem_st32(tH_w, hi);
+            tmem_st32(tH_w + kKH, lo);
 #pragma unroll
-        for (int c = 0; c < kKH / 4; ++c)
-            store_split4(a_hi, a_lo, cm_off(row, 4 * c, kKH), h[4 * c], h[4 * c + 1], h[4 * c + 2], h[4 * c + 3]);
-        to_mma(bar_id);
-        // ---- layer 2, second half: D2 += H1[:, 32..63] W2'[:, 32..63]^T
-        if (row == 0) {
-            issue_split_mmas(d2, a_hi_s, a_lo_s, kKH / 4 * 128, sm_s + kOffB2Hi, sm_s + kOffB2Lo, kK2 / 4 * 128,
-                             kKH / 8, kKH / 8, true);
+            for (int i = 0; i < 32; ++i)
+                h[i] = fmaxf(v[kKH + i], 0.0f);
+            tmem_wait_st();
+        }
+        if (!hand_off(mine))   // D1 is read (its region takes D2), the first half of H1 is in H
+            break;
+        // ---- layer 2, first half: D2 = H1[:, 0..31] W2'[:, 0..31]^T
+        if (issuer) {
+            issue_split_mmas_ts(tD, tH, sm_s + kOffB2Hi, sm_s + kOffB2Lo, kK2 / 4 * 128, 0, kKH / 8, false);
             mma_commit(bar);
         }
         __syncwarp();
-        if (!wait_group())
+        // while those MMAs run: the second half's split, and the next tile's pair and rows
+        uint32_t hi2[32], lo2[32];
+        split32(h, hi2, lo2);
+        PairRows nxt;
+        fetch_pair(nxt, p + tile_stride * kM, n_pairs, pairs, jf, n_rows);
+        mine = wait_group();   // the first half's MMAs have read H
+        if (mine) {
+            tc_fence_after();
+            tmem_st32(tH_w, hi2);
+            tmem_st32(tH_w + kKH, lo2);
+            tmem_wait_st();
+        }
+        if (!hand_off(mine))
             break;
-        tc_fence_after();
+        // ---- layer 2, second half: D2 += H1[:, 32..63] W2'[:, 32..63]^T
+        if (issuer) {
+            issue_split_mmas_ts(tD, tH, sm_s + kOffB2Hi, sm_s + kOffB2Lo, kK2 / 4 * 128, kKH / 8, kKH / 8, true);
+            mma_commit(bar);
+        }
+        __syncwarp();
+        // the next tile's inputs while those MMAs run (the MMAs that read X have completed)
+        const bool cur_valid = valid;
+        if (more) {
+            store_inputs(nxt);
+            valid = nxt.valid;
+        }
+        if (!hand_off(wait_group()))   // layer 2 is done; the next tile's X is in the buffer
+            break;
+        // the next tile's layer 1 into H (read by the MMAs just completed) runs during epilogue 2
+        if (more)
+            issue_layer1(tH, false);
 
         // ---- epilogue 2: S_hat = 1 + ReLU(b3 + sum_o w3_o ReLU(D2_o + b2'_o)), o in order
         float y = ep.b3;
-#pragma unroll
-        for (int half = 0; half < 2; ++half) {
-            float v[32];
-            tmem_ld32((d2 + 32 * half) | lane_sel, v);
+        {
+            float v[64];
+            tmem_ld32(tD_w, v);
+            tmem_ld32(tD_w + 32, v + 32);
             tmem_wait_ld();
 #pragma unroll
-            for (int o = 0; o < 32; ++o)
-                y = __fmaf_rn(ep.w3[32 * half + o], fmaxf(__fadd_rn(v[o], ep.b2[32 * half + o]), 0.0f), y);
+            for (int o = 0; o < 64; ++o)
+                y = __fmaf_rn(ep.w3[o], fmaxf(__fadd_rn(v[o], ep.b2[o]), 0.0f), y);
         }
         if (p < n_pairs)
-            out[p] = valid ? __fadd_rn(1.0f, fmaxf(y, 0.0f)) : __int_as_float(0x7fffffff);
-        // the next tile rewrites the operand buffer (every MMA reading it has completed) and D1/D2 (read
-        // above: the tcgen05 fence before the next named barrier orders those reads before the next MMAs)
-        cur = nxt;
+            out[p] = cur_valid ? __fadd_rn(1.0f, fmaxf(y, 0.0f)) : __int_as_float(0x7fffffff);
+        // the next tile's epilogue 1 writes this region (its half of H1) after these reads completed
     }
     if (!ok) {
         // an MMA group did not complete in time: the mbarrier is made to track every MMA of this
         // warpgroup still in flight, whose completion is awaited (bounded) before the tensor memory
         // is released; the timeout is reported
-        if (row == 0)
+        if (issuer)
             mma_commit(bar);
         phase ^= 1u;   // the phase the failed wait was for
         mbar_wait_bounded(bar, phase, wait_polls);
@@ -495,8 +571,10 @@ __global__ void __launch_bounds__(iac_tc::kThreads, 1) k_iac_tc(const __grid_con
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols) : "memory");
 }
 
-// Split images of W1' (64 x 40) and W2' (64 x 64) in the canonical layout, hi then lo of each.
-void build_bimg(int H, const std::vector<float> &w1, const std::vector<float> &w2, std::vector<uint32_t> &img)
+// Split images of [W1' | b1'] (64 x 40: the bias in column 36, which meets X's column of ones) and W2'
+// (64 x 64) in the canonical layout, hi then lo of each.
+void build_bimg(int H, const std::vector<float> &w1, const std::vector<float> &b1, const std::vector<float> &w2,
+                std::vector<uint32_t> &img)
 {
     using namespace iac_tc;
     img.assign(kBImgBytes / 4, 0u);
@@ -516,6 +594,7 @@ void build_bimg(int H, const std::vector<float> &w1, const std::vector<float> &w
     for (int o = 0; o < H; ++o) {
         for (int k = 0; k < kIn; ++k)
             put(kOffB1Hi, kK1, o, k, w1[(size_t)o * kIn + k]);
+        put(kOffB1Hi, kK1, o, kIn, b1[o]);
         for (int i = 0; i < H; ++i)
             put(kOffB2Hi, kK2, o, i, w2[(size_t)o * H + i]);
     }
@@ -802,15 +881,15 @@ esp_status esp_iac_load_model(esp_iac *m, int32_t H, const float *W1, const floa
         return ESP_ERR_INVALID_ARG;
     std::vector<float> w3(W3, W3 + H);
     m->loaded = false;
-    // tensor path: biases and output weights for the epilogue, split weight images for the MMAs
+    // tensor path: layer 2's bias and the output weights for the epilogue, split weight images (with
+    // layer 1's bias) for the MMAs
     std::memset(&m->ep, 0, sizeof(m->ep));
     for (int o = 0; o < H; ++o) {
-        m->ep.b1[o] = b1f[o];
         m->ep.b2[o] = b2f[o];
         m->ep.w3[o] = w3[o];
     }
     m->ep.b3 = b3;
-    build_bimg(H, w1f, w2f, m->h_bimg);
+    build_bimg(H, w1f, b1f, w2f, m->h_bimg);
     IAC_CUDA(cudaSetDevice(m->device));
     IAC_CUDA(cudaMemcpyAsync(m->d_bimg, m->h_bimg.data(), iac_tc::kBImgBytes, cudaMemcpyHostToDevice, m->stream));
     IAC_CUDA(cudaStreamSynchronize(m->stream));

@@ -3,25 +3,33 @@
 // fp32-level accuracy.
 //
 // Tile: 128 pairs (one per TMEM lane and per thread of a warpgroup) x 64 hidden units. Layer 1 is
-// D1[128 x 64] = X[128 x 40] * W1'^T (36 inputs padded to 40 = 5 MMA k-steps of 8), layer 2 is
-// D2 = H1[128 x 64] * W2'^T (8 k-steps) issued in two halves of 32 columns of H1; the output layer
-// (64 terms) and the biases run in the epilogue on the CUDA cores. Split: every operand
+// D1[128 x 64] = X[128 x 40] * [W1' | b1']^T: the 36 inputs, a column of ones that carries the bias
+// (b1' in column 36 of the weights) and zero padding to 40 = 5 MMA k-steps of 8. Layer 2 is
+// D2 = H1[128 x 64] * W2'^T (8 k-steps) issued in two halves of 32 columns of H1; its bias, the
+// output layer (64 terms) and the ReLUs run in the epilogues on the CUDA cores. Split: every operand
 // a = a_hi + a_lo with a_hi = a truncated to tf32 (exact) and a_lo = tf32(a - a_hi) (round to
 // nearest, ties away), and each k-step issues a_hi*b_hi + a_hi*b_lo + a_lo*b_hi into the same fp32
 // accumulator; per product the dropped term and the roundings of the low parts are below 2^-19 |a b|.
 //
+// Operands. Shared-memory bandwidth bounds this kernel: an M = 128, N = 64, K = 8 tf32 MMA reads
+// 6 KB of operands from shared memory, more than the tensor core's time for it at 128 B per cycle.
+// So layer 2 takes its A operand (H1) from tensor memory, where the epilogue writes it with
+// tcgen05.st, and reads only B from shared memory; layer 1 keeps X in shared memory (X, D1 and a
+// half of H1 do not fit together in a warpgroup's columns). Each warpgroup owns 128 TMEM columns: P
+// (64) holds D1, then D2 once D1 has been read into registers; Q (64) holds a half of H1, hi at Q
+// and lo at Q + 32 (lane = row, column = k, the layout of an M = 128 operand in tensor memory). The
+// second half is written once the first half's MMAs have completed.
+//
 // CTA: four warpgroups, each running its own sequence of tiles, so that four tiles' dependency
-// chains (features, MMA 1, epilogue 1 in two halves each followed by its MMAs, epilogue 2) overlap
-// on one SM; the split weights W1', W2' are staged once per CTA (53,248 bytes). A warpgroup's operand
-// A buffer (40 KB) holds X (hi and lo, 2 x 20 KB), then each half of H1 in turn (2 x 16 KB): the
-// second half is written once the first half's MMAs have completed, while the first half's epilogue
-// already overlaps them; 128 TMEM columns per warpgroup (D1, D2). Operands use the canonical
-// no-swizzle K-major layout: 8-row x 16-byte core matrices of 128 contiguous bytes, consecutive
-// along K (leading offset 128 B), row groups of 8 at a stride of K/4 * 128 B. One elected thread
-// per warpgroup issues the MMAs and commits them to the warpgroup's mbarrier; every wait is bounded
-// and a timeout ends the warpgroup's loop (the decision is made warpgroup-wide by a reducing
-// barrier), flags the error word, makes the mbarrier track every MMA still in flight and waits for
-// them (bounded) before the CTA frees its tensor memory.
+// chains (features, MMA 1, epilogue 1, the two halves of layer 2, epilogue 2) overlap on one SM; the
+// next tile's inputs are computed and stored while the current tile's last MMAs run. The split weights
+// W1', W2' are staged once per CTA (53,248 bytes); a warpgroup's X buffer holds hi and lo (2 x 20 KB).
+// Shared-memory operands use the canonical no-swizzle K-major layout: 8-row x 16-byte core matrices
+// of 128 contiguous bytes, consecutive along K (leading offset 128 B), row groups of 8 at a stride of
+// K/4 * 128 B. One elected thread per warpgroup issues the MMAs and commits them to the warpgroup's
+// mbarrier; every wait is bounded and a timeout ends the warpgroup's loop (the decision is made
+// warpgroup-wide by a reducing barrier), flags the error word, makes the mbarrier track every MMA
+// still in flight and waits for them (bounded) before the CTA frees its tensor memory.
 #pragma once
 
 #include <cstdint>
@@ -30,25 +38,25 @@ namespace iac_tc {
 
 constexpr int kM = 128;          // pairs per tile
 constexpr int kN = 64;           // hidden units (narrower models are zero-padded)
-constexpr int kK1 = 40;          // 36 inputs padded to a multiple of the tf32 MMA K (8)
+constexpr int kK1 = 40;          // 36 inputs and the bias column, padded to a multiple of the tf32 MMA K (8)
 constexpr int kK2 = 64;
 constexpr int kKH = 32;          // layer 2 in two halves of 32 columns of H1
 constexpr int kWG = 4;           // warpgroups per CTA
 constexpr int kThreads = 128 * kWG;
-constexpr int kTmemCols = 512;   // D1 and D2 (64 fp32 columns each) per warpgroup
+constexpr int kTmemCols = 512;   // P (D1, then D2) and Q (a half of H1, hi and lo): 128 per warpgroup
 
 constexpr int kB1Bytes = kN * kK1 * 4;                      // 10,240
 constexpr int kB2Bytes = kN * kK2 * 4;                      // 16,384
 constexpr int kBImgBytes = 2 * kB1Bytes + 2 * kB2Bytes;     // hi, lo of W1' then of W2'
 constexpr int kA1Bytes = kM * kK1 * 4;                      // 20,480: one part (hi or lo) of X
-constexpr int kAHBytes = kM * kKH * 4;                      // 16,384: one part of a half of H1
-constexpr int kABufBytes = 2 * kA1Bytes;                    // a warpgroup's buffer: hi at 0, lo at kA1Bytes
+constexpr int kABufBytes = 2 * kA1Bytes;                    // a warpgroup's X: hi at 0, lo at kA1Bytes
 constexpr int kOffB1Hi = 0, kOffB1Lo = kB1Bytes, kOffB2Hi = 2 * kB1Bytes, kOffB2Lo = 2 * kB1Bytes + kB2Bytes;
 constexpr int kOffA = kBImgBytes;                           // warpgroup g's buffer at kOffA + g kABufBytes
 constexpr int kOffBar = kOffA + kWG * kABufBytes;
 constexpr int kOffSlot = kOffBar + 8 * kWG;
 constexpr int kSmemBytes = kOffSlot + 16 + 1024;            // + alignment slack of the dynamic base
-static_assert(kAHBytes <= kA1Bytes, "a half of H1 fits where X was");
+static_assert(2 * kN * kWG <= kTmemCols, "P and Q of every warpgroup");
+static_assert(2 * kKH == kN, "a half of H1, hi and lo, fills Q");
 static_assert(kSmemBytes <= 232448, "shared memory of one CTA");
 
 // Byte offset of element (row, col) in the canonical no-swizzle K-major layout of a K-wide operand.

@@ -14,7 +14,8 @@ and the final 1 + ReLU(y) adds u (1 + M3). The tensor-core path (hidden layers a
 a three-term tf32 split, esp_iac.h) differs in the two hidden dot products: each product is within
 2^-19 = 32u relative (the dropped low-times-low term and the roundings of the low parts), the
 tensor core accumulates 64 products (zero padding included) in fp32 whose additions may truncate
-(2u each), and the bias is added in the epilogue: 40 u and (H + 3) u become 160 u and 200 u. The
+(2u each), layer 1's bias enters as one more product (a column of ones times b1', inside M1) and
+layer 2's is added in the epilogue: 40 u and (H + 3) u become 160 u and 200 u. The
 test allows twice the bound per pair, and checks that the typical error stays near fp32 rounding.
 """
 
@@ -127,6 +128,17 @@ def test_parity_ragged(lib, H, path):
     pairs = W.iac_pairs(11, 3, 64, 8)[: 1000 + 37]     # a ragged tail after several tiles
     got, ref = check(esp, random_model(H, H), rows, pairs, W.IAC_C_MEM, path)
     assert (ref > 1.0).any()
+
+
+def test_parity_several_tiles_per_warpgroup(lib):
+    """1,024 tiles of 128 pairs, a ragged last one: on a full grid (152 CTAs x 4 warpgroups) most
+    warpgroups of the tensor path run two tiles in turn, the second with the roles of their two
+    tensor-memory regions swapped; every pair is checked."""
+    from paper_2608_07971_gb300 import esp
+    w = W.iac_batch(S=4, J=2048, K=16, H=64, seed=9)
+    pairs = w.pairs[: len(w.pairs) - 51]
+    got, ref = check(esp, w.model, w.rows, pairs, w.c_mem, "tensor")
+    assert (ref > 1.0).mean() > 0.2
 
 
 @pytest.mark.parametrize("path", ["tensor", "fma"])
