@@ -335,7 +335,7 @@ __device__ __forceinline__ void issue_split_mmas(uint32_t d, uint32_t a_hi, uint
     }
 }
 
-// Layer 2's MMAs for one half of H1 (ks_n k-steps): A from Q in tensor memory (hi at a_t, lo at
+// Layer 2's MMAs for one half of H1 (ks_n k-steps): A from tensor memory (hi at a_t, lo at
 // a_t + 32), B from the staged weights at b_hi / b_lo (k-step b_ks0 onwards, row-group stride b_sbo).
 __device__ __forceinline__ void issue_split_mmas_ts(uint32_t d, uint32_t a_t, uint32_t b_hi, uint32_t b_lo,
                                                     uint32_t b_sbo, int b_ks0, int ks_n, bool acc0)

@@ -11,14 +11,17 @@
 // nearest, ties away), and each k-step issues a_hi*b_hi + a_hi*b_lo + a_lo*b_hi into the same fp32
 // accumulator; per product the dropped term and the roundings of the low parts are below 2^-19 |a b|.
 //
-// Operands. Shared-memory bandwidth bounds this kernel: an M = 128, N = 64, K = 8 tf32 MMA reads
-// 6 KB of operands from shared memory, more than the tensor core's time for it at 128 B per cycle.
-// So layer 2 takes its A operand (H1) from tensor memory, where the epilogue writes it with
-// tcgen05.st, and reads only B from shared memory; layer 1 keeps X in shared memory (X, D1 and a
-// half of H1 do not fit together in a warpgroup's columns). Each warpgroup owns 128 TMEM columns: P
-// (64) holds D1, then D2 once D1 has been read into registers; Q (64) holds a half of H1, hi at Q
-// and lo at Q + 32 (lane = row, column = k, the layout of an M = 128 operand in tensor memory). The
-// second half is written once the first half's MMAs have completed.
+// Operands. An M = 128, N = 64, K = 8 tf32 MMA with both operands in shared memory reads 6 KB, more
+// than the tensor core's time for it at 128 B per cycle, so with both layers reading A from shared
+// memory the kernel was bound by shared-memory bandwidth. Layer 2 therefore takes its A operand (H1)
+// from tensor memory, where the epilogue writes it with tcgen05.st, and reads only B from shared
+// memory; layer 1 keeps X in shared memory (X, D1 and a half of H1 do not fit together in a
+// warpgroup's columns). Each warpgroup owns two regions of 64 TMEM columns: one holds a tile's
+// accumulators (D1, then D2 once D1 has been read into registers), the other a half of H1, hi at its
+// column 0 and lo at 32 (lane = row, column = k, the layout of an M = 128 operand in tensor memory);
+// the second half is written once the first half's MMAs have completed. The roles swap from one tile
+// to the next, so the next tile's layer 1 is issued as soon as layer 2 completes and runs during the
+// output epilogue.
 //
 // CTA: four warpgroups, each running its own sequence of tiles, so that four tiles' dependency
 // chains (features, MMA 1, epilogue 1, the two halves of layer 2, epilogue 2) overlap on one SM; the
@@ -26,10 +29,12 @@
 // W1', W2' are staged once per CTA (53,248 bytes); a warpgroup's X buffer holds hi and lo (2 x 20 KB).
 // Shared-memory operands use the canonical no-swizzle K-major layout: 8-row x 16-byte core matrices
 // of 128 contiguous bytes, consecutive along K (leading offset 128 B), row groups of 8 at a stride of
-// K/4 * 128 B. One elected thread per warpgroup issues the MMAs and commits them to the warpgroup's
-// mbarrier; every wait is bounded and a timeout ends the warpgroup's loop (the decision is made
-// warpgroup-wide by a reducing barrier), flags the error word, makes the mbarrier track every MMA
-// still in flight and waits for them (bounded) before the CTA frees its tensor memory.
+// K/4 * 128 B. One elected thread per warpgroup, each in a different SM sub-partition, issues the
+// MMAs and commits them to the warpgroup's mbarrier; every wait is bounded, agreed warp-wide (the
+// tcgen05 loads and stores after it are warp-collective) and warpgroup-wide at the next hand-off
+// barrier (a reducing barrier). A timeout ends the warpgroup's loop, flags the error word, makes the
+// mbarrier track every MMA still in flight and waits for them (bounded) before the CTA frees its
+// tensor memory.
 #pragma once
 
 #include <cstdint>
@@ -43,7 +48,7 @@ constexpr int kK2 = 64;
 constexpr int kKH = 32;          // layer 2 in two halves of 32 columns of H1
 constexpr int kWG = 4;           // warpgroups per CTA
 constexpr int kThreads = 128 * kWG;
-constexpr int kTmemCols = 512;   // P (D1, then D2) and Q (a half of H1, hi and lo): 128 per warpgroup
+constexpr int kTmemCols = 512;   // two regions of 64 columns per warpgroup (accumulators; a half of H1)
 
 constexpr int kB1Bytes = kN * kK1 * 4;                      // 10,240
 constexpr int kB2Bytes = kN * kK2 * 4;                      // 16,384
@@ -55,8 +60,8 @@ constexpr int kOffA = kBImgBytes;                           // warpgroup g's buf
 constexpr int kOffBar = kOffA + kWG * kABufBytes;
 constexpr int kOffSlot = kOffBar + 8 * kWG;
 constexpr int kSmemBytes = kOffSlot + 16 + 1024;            // + alignment slack of the dynamic base
-static_assert(2 * kN * kWG <= kTmemCols, "P and Q of every warpgroup");
-static_assert(2 * kKH == kN, "a half of H1, hi and lo, fills Q");
+static_assert(2 * kN * kWG <= kTmemCols, "the two regions of every warpgroup");
+static_assert(2 * kKH == kN, "a half of H1, hi and lo, fills a region");
 static_assert(kSmemBytes <= 232448, "shared memory of one CTA");
 
 // Byte offset of element (row, col) in the canonical no-swizzle K-major layout of a K-wide operand.
