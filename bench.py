@@ -276,17 +276,23 @@ class ClockSampler:
 
 def cpu_baseline(w: W.Workload, T: int, budget_s: float) -> dict:
     """The oracle as it stands, single-threaded, on whole scenarios of the same workload until the
-    time budget is spent (at least one scenario; the first `rounds` of it if one scenario alone would
-    far exceed the budget)."""
+    time budget is spent (at least one scenario; a prefix of its rounds if one scenario alone would
+    take more than 2.5 budgets at the rate a short probe measures on this host)."""
     import oracle
     t = w.table
     ot = oracle.OracleTable(t)
     lib = oracle.load()
     per_round = t.n_opt / t.S
-    # rough rate to bound a single scenario: 3 ns per option-evaluation
+    # the oracle's rate on this host, from a few rounds of the first scenario (not counted): a
+    # scenario that would take well over the budget runs a prefix of its rounds
+    probe = min(T, 4)
+    n0 = int(t.job_off[t.J] - t.job_off[0])
+    p0 = time.perf_counter()
+    oracle.solve_scenario(ot, 0, w.eta0, probe, mode=w.mode, step=w.step, lib=lib)
+    s_per_eval = (time.perf_counter() - p0) / max(1, n0 * (probe + 1))
     rounds = T
-    if per_round * (T + 1) * 3e-9 > 4 * budget_s:
-        rounds = max(1, int(budget_s / (per_round * 3e-9)) - 1)
+    if per_round * (T + 1) * s_per_eval > 2.5 * budget_s:
+        rounds = max(1, int(budget_s / (per_round * s_per_eval)) - 1)
     evals, n, t0 = 0, 0, time.perf_counter()
     while n < t.S:
         oracle.solve_scenario(ot, n, w.eta0, rounds, mode=w.mode, step=w.step, lib=lib)
